@@ -1,0 +1,197 @@
+"""fp64 CPU oracle for the NAMOH routed-attention path.
+
+TEST INFRASTRUCTURE ONLY: the tests, ``__graft_entry__.smoke()`` and the
+benchmark's CPU-baseline leg are the only callers.  The CUDA library never
+imports, links or executes anything here, and this package imports nothing from
+the CUDA library: the two share only the seeded input generators in
+``namoh_inputs``.
+
+The arithmetic lives in ``namoh_oracle.c`` (plain C, fp64, built with gcc); this
+module only marshals numpy arrays.  Each wrapper names the passage of the paper
+it follows:
+
+* ``route``        Sec. 3.1 Eq. (namoh-gates) and the ordered index sets I_i;
+                   Sec. 3.2 Eq. (namoh-head-rope) for the rank rho.
+* ``rope``         Sec. 3.2 Eq. (namoh-head-rope), half-split RoPE.
+* ``prefill``      Sec. 3.1 Eq. (namoh-attention) over packed (batch, head)
+                   subsequences (Sec. 3.2 "Efficient execution"); App. C
+                   "Adopted KV-group routing" for g > 1.
+* ``prefill_rows`` the same for a chosen subset of query rows.
+* ``decode_step``  Sec. 3.1 (last paragraph): append to and attend within only
+                   the selected heads' histories.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "namoh_oracle.c")
+_LIB_PATH = os.path.join(_HERE, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+OK = 0
+ERR_ARG = -1
+ERR_NONFINITE = -2
+ERR_NOMEM = -3
+ERR_CAPACITY = -4
+
+
+class OracleError(RuntimeError):
+    pass
+
+
+def build(force: bool = False) -> str:
+    """Compile the C oracle with gcc (fp64, no fast-math, no FMA contraction)."""
+    if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
+        tmp = _LIB_PATH + f".tmp{os.getpid()}"
+        cmd = ["gcc", "-O2", "-std=c11", "-D_POSIX_C_SOURCE=200809L", "-ffp-contract=off",
+               "-fPIC", "-shared", "-pthread", "-o", tmp, _SRC, "-lm"]
+        subprocess.run(cmd, check=True)
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        build()
+        lib = ctypes.CDLL(_LIB_PATH)
+        P = ctypes.c_void_p
+        i32, i64, f64 = ctypes.c_int, ctypes.c_long, ctypes.c_double
+        lib.oracle_route_topk.argtypes = [P, i64, i32, i32, P, P]
+        lib.oracle_dispatch.argtypes = [P, i32, i32, i32, i32, P, P, P, P, P]
+        lib.oracle_rope.argtypes = [P, i64, i32, i64, P, f64, P]
+        lib.oracle_prefill.argtypes = [P, P, P, i32, i32, i32, f64, P, P, P, P, P, i32]
+        lib.oracle_prefill_rows.argtypes = [P, P, P, i32, i32, i32, f64, P, P, P, P, P, i64, P]
+        lib.oracle_decode_step.argtypes = [P, P, P, P, P, i32, i32, i32, i32, i32, f64,
+                                           P, P, P, P, P, P]
+        lib.oracle_default_threads.argtypes = []
+        for fn in ("oracle_route_topk", "oracle_dispatch", "oracle_rope", "oracle_prefill",
+                   "oracle_prefill_rows", "oracle_decode_step", "oracle_default_threads"):
+            getattr(lib, fn).restype = ctypes.c_int
+        _lib = lib
+        return lib
+
+
+def _ptr(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _check(rc: int, what: str):
+    if rc != OK:
+        raise OracleError(f"{what} failed with oracle status {rc}")
+
+
+def default_threads() -> int:
+    return int(_load().oracle_default_threads())
+
+
+def route(scores: np.ndarray, K: int) -> dict:
+    """Routing and dispatch for scores [B, T, H] (fp32 router logits).
+
+    Returns topk_head [B,T,K] int32, gate [B,T,K] fp64, n [B,H], seg_offsets [B*H+1],
+    rank [B,T,K], row [B,T,K] and row_src [B*T*K] (all int32).
+    """
+    lib = _load()
+    scores = np.ascontiguousarray(scores, dtype=np.float32)
+    B, T, H = scores.shape
+    topk = np.empty((B, T, K), np.int32)
+    gate = np.empty((B, T, K), np.float64)
+    _check(lib.oracle_route_topk(_ptr(scores), B * T, H, K, _ptr(topk), _ptr(gate)), "route_topk")
+    n = np.empty((B, H), np.int32)
+    seg = np.empty(B * H + 1, np.int32)
+    rank = np.empty((B, T, K), np.int32)
+    row = np.empty((B, T, K), np.int32)
+    row_src = np.empty(B * T * K, np.int32)
+    _check(lib.oracle_dispatch(_ptr(topk), B, T, H, K, _ptr(n), _ptr(seg), _ptr(rank), _ptr(row),
+                               _ptr(row_src)), "dispatch")
+    return dict(topk_head=topk, gate=gate, n=n, seg_offsets=seg, rank=rank, row=row, row_src=row_src)
+
+
+def rope(x_bits: np.ndarray, pos: np.ndarray, base: float) -> np.ndarray:
+    """Rotate bf16 rows x [rows, d] (raw uint16 bits) to positions pos [rows]; fp64 out."""
+    lib = _load()
+    x_bits = np.ascontiguousarray(x_bits, dtype=np.uint16)
+    rows, d = x_bits.shape
+    pos = np.ascontiguousarray(pos, dtype=np.int64)
+    out = np.empty((rows, d), np.float64)
+    _check(lib.oracle_rope(_ptr(x_bits), rows, d, d, _ptr(pos), float(base), _ptr(out)), "rope")
+    return out
+
+
+def prefill(q: np.ndarray, k: np.ndarray, v: np.ndarray, seg_offsets: np.ndarray, row_src: np.ndarray,
+            gate: np.ndarray, d: int, g: int, base: float, nthreads: int | None = None,
+            return_krot: bool = False):
+    """Prefill over packed rows.  q [R*g, d], k/v [R, d] as bf16 bits; gate indexed by row_src.
+
+    Returns y [R*g, d] fp64 laid out by (row_src * g + j), i.e. [B, T, K, g, d] flattened.
+    """
+    lib = _load()
+    q = np.ascontiguousarray(q, dtype=np.uint16)
+    k = np.ascontiguousarray(k, dtype=np.uint16)
+    v = np.ascontiguousarray(v, dtype=np.uint16)
+    seg = np.ascontiguousarray(seg_offsets, dtype=np.int32)
+    rs = np.ascontiguousarray(row_src, dtype=np.int32)
+    gt = np.ascontiguousarray(gate, dtype=np.float64).reshape(-1)
+    R = int(seg[-1])
+    y = np.zeros((R * g, d), np.float64)
+    krot = np.empty((R, d), np.float64) if return_krot else None
+    nthreads = default_threads() if nthreads is None else int(nthreads)
+    rc = lib.oracle_prefill(_ptr(q), _ptr(k), _ptr(v), len(seg) - 1, d, g, float(base), _ptr(seg), _ptr(rs),
+                            _ptr(gt), _ptr(y), _ptr(krot) if krot is not None else None, nthreads)
+    _check(rc, "prefill")
+    return (y, krot) if return_krot else y
+
+
+def prefill_rows(q, k, v, seg_offsets, row_src, gate, d: int, g: int, base: float,
+                 rows: np.ndarray, heads: np.ndarray) -> np.ndarray:
+    """Outputs g*h for the listed (packed row, group head) queries only: [len(rows), d] fp64."""
+    lib = _load()
+    q = np.ascontiguousarray(q, dtype=np.uint16)
+    k = np.ascontiguousarray(k, dtype=np.uint16)
+    v = np.ascontiguousarray(v, dtype=np.uint16)
+    seg = np.ascontiguousarray(seg_offsets, dtype=np.int32)
+    rs = np.ascontiguousarray(row_src, dtype=np.int32)
+    gt = np.ascontiguousarray(gate, dtype=np.float64).reshape(-1)
+    rows = np.ascontiguousarray(rows, dtype=np.int64)
+    heads = np.ascontiguousarray(heads, dtype=np.int32)
+    out = np.empty((len(rows), d), np.float64)
+    rc = lib.oracle_prefill_rows(_ptr(q), _ptr(k), _ptr(v), len(seg) - 1, d, g, float(base), _ptr(seg),
+                                 _ptr(rs), _ptr(gt), _ptr(rows), _ptr(heads), len(rows), _ptr(out))
+    _check(rc, "prefill_rows")
+    return out
+
+
+def decode_step(topk_head, gate, q, k, v, Hr: int, d: int, g: int, base: float,
+                k_cache: np.ndarray, v_cache: np.ndarray, seg_base: np.ndarray, seg_len: np.ndarray,
+                seg_cap: np.ndarray) -> np.ndarray:
+    """One decode step.  k_cache/v_cache [cap_total, d] fp64 and seg_len are updated in place.
+
+    topk_head/gate [B, Kr]; q [B, Kr*g, d], k/v [B, Kr, d] as bf16 bits.  Returns y [B, Kr*g, d].
+    """
+    lib = _load()
+    topk_head = np.ascontiguousarray(topk_head, dtype=np.int32)
+    B, Kr = topk_head.shape
+    gate = np.ascontiguousarray(gate, dtype=np.float64)
+    q = np.ascontiguousarray(q, dtype=np.uint16)
+    k = np.ascontiguousarray(k, dtype=np.uint16)
+    v = np.ascontiguousarray(v, dtype=np.uint16)
+    for name, arr, dt in (("k_cache", k_cache, np.float64), ("v_cache", v_cache, np.float64),
+                          ("seg_base", seg_base, np.int64), ("seg_len", seg_len, np.int32),
+                          ("seg_cap", seg_cap, np.int32)):
+        if arr.dtype != dt or not arr.flags.c_contiguous:
+            raise OracleError(f"{name} must be a contiguous {np.dtype(dt).name} array")
+    y = np.zeros((B, Kr * g, d), np.float64)
+    rc = lib.oracle_decode_step(_ptr(topk_head), _ptr(gate), _ptr(q), _ptr(k), _ptr(v), B, Hr, Kr, d, g,
+                                float(base), _ptr(k_cache), _ptr(v_cache), _ptr(seg_base), _ptr(seg_len),
+                                _ptr(seg_cap), _ptr(y))
+    _check(rc, "decode_step")
+    return y

@@ -1,0 +1,497 @@
+/*
+ * namoh_oracle.c -- plain fp64 CPU oracle for the NAMOH routed-attention path.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the correctness authority that the
+ * CUDA path is compared against.  Only the test suite, the smoke check and the
+ * benchmark's CPU-baseline leg may load it; the product path never does.  It
+ * shares no code, header, table or helper with the CUDA library.
+ *
+ * Everything here follows the paper's definitions literally, in fp64:
+ *   - routing:   Sec. 3.1, Eq. (namoh-gates)  a_t = softmax(x_t W_r), S_K(t) = TopK(a_t),
+ *                m_{t,i} = 1{i in S_K(t)}, g_{t,i} = m_{t,i} a_{t,i}  (no renormalisation,
+ *                App. A, Eq. (namoh-biased-routing) and the sentence after it).
+ *   - dispatch:  Sec. 3.1, ordered index sets I_i = {t : m_{t,i} = 1}, n_i = |I_i|;
+ *                Sec. 3.2 "Efficient execution": each (batch, head) subsequence is packed
+ *                as an independent sequence.
+ *   - rank:      Sec. 3.2, Eq. (namoh-head-rope)  rho_i(t) = sum_{s<=t} m_{s,i} - 1.
+ *   - RoPE:      Sec. 3.2, Eq. (namoh-head-rope)  q~ = q R(rho), k~ = k R(rho).
+ *   - attention: Sec. 3.1, Eq. (namoh-attention)  h_{t,i} = Attn(q~_{t,i}, [k~_{s,i}], [v_{s,i}]),
+ *                s in I_i, s <= t, standard scaled dot-product attention.
+ *   - combine:   Sec. 3.1, Eq. (namoh-attention)  the per-slot term g_{t,i} h_{t,i}
+ *                (the W_O projection is outside this path).
+ *   - decode:    Sec. 3.1 (last paragraph) and Sec. 3.2: a new token appends to and attends
+ *                within only its selected heads' histories; its rank is the current length.
+ *   - GQA:       App. C, "Adopted KV-group routing": K/g of H/g groups are selected, the g
+ *                query heads of a group share its gate, key/value history and rank.
+ *
+ * Readings where the paper is silent (each listed in the design notes):
+ *   - TopK compares the raw fp32 router logits (softmax is monotone, so the selected
+ *     set equals TopK of a_t); ties go to the lower head index; slots are ordered by
+ *     descending score.
+ *   - RoPE is the half-split form: pairs (j, j + d/2), theta_j = base^(-2j/d),
+ *     x'_j = x_j cos - x_{j+d/2} sin,  x'_{j+d/2} = x_{j+d/2} cos + x_j sin.
+ *   - Attention scale 1/sqrt(d_head).
+ *   - Packed rows: segments in (batch, head) order, rows ascending in t inside a segment.
+ *
+ * Inputs in bf16 are passed as raw uint16 bit patterns and widened exactly.
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#include <unistd.h>
+
+#define ORACLE_OK 0
+#define ORACLE_ERR_ARG (-1)
+#define ORACLE_ERR_NONFINITE (-2)
+#define ORACLE_ERR_NOMEM (-3)
+#define ORACLE_ERR_CAPACITY (-4)
+
+/* ------------------------------------------------------------------------- */
+/* small helpers                                                             */
+/* ------------------------------------------------------------------------- */
+
+static double bf16_to_double(uint16_t bits)
+{
+    uint32_t u = ((uint32_t)bits) << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+/* A tiny parallel-for over [0, n) with a shared atomic counter. */
+typedef void (*item_fn)(long item, void *ctx);
+struct pool_job {
+    long n;
+    long next;
+    item_fn fn;
+    void *ctx;
+};
+
+static void *pool_worker(void *arg)
+{
+    struct pool_job *job = (struct pool_job *)arg;
+    for (;;) {
+        long i = __atomic_fetch_add(&job->next, 1, __ATOMIC_RELAXED);
+        if (i >= job->n) break;
+        job->fn(i, job->ctx);
+    }
+    return NULL;
+}
+
+static void parallel_for(long n, int nthreads, item_fn fn, void *ctx)
+{
+    struct pool_job job = {n, 0, fn, ctx};
+    if (nthreads <= 1 || n <= 1) {
+        pool_worker(&job);
+        return;
+    }
+    if (nthreads > 256) nthreads = 256;
+    pthread_t tid[256];
+    int started = 0;
+    for (int i = 0; i < nthreads - 1; ++i) {
+        if (pthread_create(&tid[i], NULL, pool_worker, &job) == 0) ++started;
+    }
+    pool_worker(&job);
+    for (int i = 0; i < started; ++i) pthread_join(tid[i], NULL);
+}
+
+/* ------------------------------------------------------------------------- */
+/* Routing and dispatch (Sec. 3.1 Eq. namoh-gates; Sec. 3.2 Eq. namoh-head-rope) */
+/* ------------------------------------------------------------------------- */
+
+/* Head a precedes head b in the TopK order: larger score first, ties to the
+ * lower index.  Scores are compared exactly as fp32 values (+0 == -0). */
+static int head_precedes(const float *s, int a, int b)
+{
+    if (s[a] > s[b]) return 1;
+    if (s[a] < s[b]) return 0;
+    return a < b;
+}
+
+/*
+ * oracle_route_topk: per token, S_K(t) and g_{t,i}.
+ *   scores    [N, H] fp32 router logits x_t W_r (N = B*T tokens)
+ *   topk_head [N, K] selected heads in descending score order (ties -> lower index)
+ *   gate      [N, K] fp64 softmax over all H heads, taken at the selected heads
+ * Returns ORACLE_ERR_NONFINITE if any score is NaN or infinite (outside the contract).
+ */
+int oracle_route_topk(const float *scores, long N, int H, int K, int32_t *topk_head, double *gate)
+{
+    if (!scores || !topk_head || !gate || N < 0 || H < 1 || K < 1 || K > H || H > 1024) return ORACLE_ERR_ARG;
+    int order[1024];
+    for (long t = 0; t < N; ++t) {
+        const float *s = scores + t * (long)H;
+        for (int i = 0; i < H; ++i)
+            if (!isfinite(s[i])) return ORACLE_ERR_NONFINITE;
+        /* insertion sort of head indices by (score desc, index asc) */
+        for (int i = 0; i < H; ++i) {
+            int j = i;
+            while (j > 0 && head_precedes(s, i, order[j - 1])) {
+                order[j] = order[j - 1];
+                --j;
+            }
+            order[j] = i;
+        }
+        /* affinities a_t = softmax over all H heads, in fp64 */
+        double mx = (double)s[order[0]];
+        double z = 0.0;
+        for (int i = 0; i < H; ++i) z += exp((double)s[i] - mx);
+        for (int k = 0; k < K; ++k) {
+            topk_head[t * K + k] = order[k];
+            gate[t * K + k] = exp((double)s[order[k]] - mx) / z;
+        }
+    }
+    return ORACLE_OK;
+}
+
+/*
+ * oracle_dispatch: ordered index sets I_i per (batch, head), walking t = 0..T-1
+ * and appending each token to the heads it selected.
+ *   topk_head   [B, T, K]
+ *   n           [B*H]      n_{b,h} = |I_h| within sequence b
+ *   seg_offsets [B*H + 1]  exclusive prefix sum of n in (b, h) order
+ *   rank        [B, T, K]  rho_h(t), zero-based rank within the head's subsequence
+ *   row         [B, T, K]  packed row = seg_offsets[b*H + h] + rho
+ *   row_src     [B*T*K]    inverse map: row_src[row] = (b*T + t)*K + k
+ */
+int oracle_dispatch(const int32_t *topk_head, int B, int T, int H, int K,
+                    int32_t *n, int32_t *seg_offsets, int32_t *rank, int32_t *row, int32_t *row_src)
+{
+    if (!topk_head || !n || !seg_offsets || !rank || !row || !row_src) return ORACLE_ERR_ARG;
+    if (B < 0 || T < 0 || H < 1 || K < 1 || K > H) return ORACLE_ERR_ARG;
+    for (long i = 0; i < (long)B * H; ++i) n[i] = 0;
+    /* ranks: append in token order */
+    for (int b = 0; b < B; ++b) {
+        for (int t = 0; t < T; ++t) {
+            for (int k = 0; k < K; ++k) {
+                long idx = ((long)b * T + t) * K + k;
+                int h = topk_head[idx];
+                if (h < 0 || h >= H) return ORACLE_ERR_ARG;
+                rank[idx] = n[(long)b * H + h];
+                n[(long)b * H + h] += 1;
+            }
+        }
+    }
+    seg_offsets[0] = 0;
+    for (long i = 0; i < (long)B * H; ++i) seg_offsets[i + 1] = seg_offsets[i] + n[i];
+    for (int b = 0; b < B; ++b) {
+        for (int t = 0; t < T; ++t) {
+            for (int k = 0; k < K; ++k) {
+                long idx = ((long)b * T + t) * K + k;
+                int h = topk_head[idx];
+                int r = seg_offsets[(long)b * H + h] + rank[idx];
+                row[idx] = r;
+                row_src[r] = (int32_t)idx;
+            }
+        }
+    }
+    return ORACLE_OK;
+}
+
+/* ------------------------------------------------------------------------- */
+/* RoPE (Sec. 3.2, Eq. namoh-head-rope), half-split pairs                     */
+/* ------------------------------------------------------------------------- */
+
+/* x [d] (widened bf16) rotated to position p: out [d] */
+static void rope_rotate(const double *x, int d, double p, double base, double *out)
+{
+    int half = d / 2;
+    for (int j = 0; j < half; ++j) {
+        double theta = pow(base, -2.0 * (double)j / (double)d);
+        double ang = p * theta;
+        double c = cos(ang), s = sin(ang);
+        double x0 = x[j], x1 = x[j + half];
+        out[j] = x0 * c - x1 * s;
+        out[j + half] = x1 * c + x0 * s;
+    }
+}
+
+/*
+ * oracle_rope: rotate each bf16 row x[i, :] (row stride ld elements) to
+ * position pos[i] and write fp64 rows out[i, :].
+ */
+int oracle_rope(const uint16_t *x, long rows, int d, long ld, const int64_t *pos, double base, double *out)
+{
+    if (!x || !pos || !out || rows < 0 || d < 2 || (d & 1) || ld < d) return ORACLE_ERR_ARG;
+    double *tmp = (double *)malloc(sizeof(double) * (size_t)d);
+    if (!tmp) return ORACLE_ERR_NOMEM;
+    for (long i = 0; i < rows; ++i) {
+        for (int c = 0; c < d; ++c) tmp[c] = bf16_to_double(x[i * ld + c]);
+        rope_rotate(tmp, d, (double)pos[i], base, out + i * (long)d);
+    }
+    free(tmp);
+    return ORACLE_OK;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Scaled dot-product attention of one query over a history (Eq. namoh-attention) */
+/* ------------------------------------------------------------------------- */
+
+/* q [d], keys [len, d], values [len, d] -> h [d]; weights scratch [len] */
+static void attend(const double *q, const double *keys, const double *values, long len, int d,
+                   double *weights, double *h)
+{
+    double scale = 1.0 / sqrt((double)d);
+    double mx = -INFINITY;
+    for (long s = 0; s < len; ++s) {
+        double acc = 0.0;
+        for (int c = 0; c < d; ++c) acc += q[c] * keys[s * d + c];
+        weights[s] = acc * scale;
+        if (weights[s] > mx) mx = weights[s];
+    }
+    double z = 0.0;
+    for (long s = 0; s < len; ++s) {
+        weights[s] = exp(weights[s] - mx);
+        z += weights[s];
+    }
+    for (int c = 0; c < d; ++c) h[c] = 0.0;
+    for (long s = 0; s < len; ++s) {
+        double w = weights[s] / z;
+        for (int c = 0; c < d; ++c) h[c] += w * values[s * d + c];
+    }
+}
+
+/* ------------------------------------------------------------------------- */
+/* Prefill: RoPE at rank, routed causal attention, gate-weighted combine      */
+/* ------------------------------------------------------------------------- */
+
+struct prefill_ctx {
+    const uint16_t *q, *v;
+    const double *krot;        /* [R, d] rotated keys */
+    const int32_t *seg_offsets;
+    const int32_t *row_src;
+    const double *gate;
+    double *y;
+    int nseg, d, g;
+    double base;
+    long *item_seg, *item_r0; /* work items: (segment, first local query) */
+    int chunk;
+    int status;
+};
+
+static void prefill_item(long it, void *vctx)
+{
+    struct prefill_ctx *c = (struct prefill_ctx *)vctx;
+    int d = c->d, g = c->g;
+    long s = c->item_seg[it];
+    long r0 = c->item_r0[it];
+    long off = c->seg_offsets[s];
+    long n = c->seg_offsets[s + 1] - off;
+    long r1 = r0 + c->chunk < n ? r0 + c->chunk : n;
+    double *vals = (double *)malloc(sizeof(double) * (size_t)(r1 > 0 ? r1 : 1) * d);
+    double *w = (double *)malloc(sizeof(double) * (size_t)(r1 > 0 ? r1 : 1));
+    double *qin = (double *)malloc(sizeof(double) * (size_t)d);
+    double *qr = (double *)malloc(sizeof(double) * (size_t)d);
+    double *h = (double *)malloc(sizeof(double) * (size_t)d);
+    if (!vals || !w || !qin || !qr || !h) {
+        c->status = ORACLE_ERR_NOMEM;
+        free(vals); free(w); free(qin); free(qr); free(h);
+        return;
+    }
+    for (long sidx = 0; sidx < r1; ++sidx)
+        for (int cc = 0; cc < d; ++cc) vals[sidx * d + cc] = bf16_to_double(c->v[(off + sidx) * d + cc]);
+    for (long r = r0; r < r1; ++r) {
+        long row = off + r;
+        long dst = c->row_src[row];
+        for (int j = 0; j < g; ++j) {
+            for (int cc = 0; cc < d; ++cc) qin[cc] = bf16_to_double(c->q[(row * g + j) * d + cc]);
+            rope_rotate(qin, d, (double)r, c->base, qr);
+            /* causal history: local ranks 0..r of this head (s in I_i, s <= t) */
+            attend(qr, c->krot + off * d, vals, r + 1, d, w, h);
+            double gt = c->gate[dst];
+            for (int cc = 0; cc < d; ++cc) c->y[(dst * g + j) * d + cc] = gt * h[cc];
+        }
+    }
+    free(vals); free(w); free(qin); free(qr); free(h);
+}
+
+struct rotk_ctx {
+    const uint16_t *k;
+    const int32_t *seg_offsets;
+    double *krot;
+    int d;
+    double base;
+};
+
+static void rotate_k_segment(long s, void *vctx)
+{
+    struct rotk_ctx *c = (struct rotk_ctx *)vctx;
+    int d = c->d;
+    long off = c->seg_offsets[s], end = c->seg_offsets[s + 1];
+    double *tmp = (double *)malloc(sizeof(double) * (size_t)d);
+    if (!tmp) return;
+    for (long row = off; row < end; ++row) {
+        for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(c->k[row * d + cc]);
+        rope_rotate(tmp, d, (double)(row - off), c->base, c->krot + row * d);
+    }
+    free(tmp);
+}
+
+/*
+ * oracle_prefill: full prefill over packed rows.
+ *   q        [R*g, d] bf16, query row of packed row r and group head j at r*g + j
+ *   k, v     [R, d]   bf16 packed rows (segments in (b, h) order)
+ *   nseg     number of segments (B * H, or B * H/g under KV-group routing)
+ *   seg_offsets [nseg+1], row_src [R], gate [R] (indexed by row_src value)
+ *   y        [R*g, d] fp64 output indexed by (row_src*g + j): the per-slot combine g*h
+ *   k_rot    [R, d]   fp64 rotated keys, or NULL
+ */
+int oracle_prefill(const uint16_t *q, const uint16_t *k, const uint16_t *v, int nseg, int d, int g,
+                   double base, const int32_t *seg_offsets, const int32_t *row_src, const double *gate,
+                   double *y, double *k_rot, int nthreads)
+{
+    if (!q || !k || !v || !seg_offsets || !row_src || !gate || !y) return ORACLE_ERR_ARG;
+    if (nseg < 0 || d < 2 || (d & 1) || g < 1) return ORACLE_ERR_ARG;
+    long R = seg_offsets[nseg];
+    double *krot = k_rot;
+    if (!krot) {
+        krot = (double *)malloc(sizeof(double) * (size_t)(R > 0 ? R : 1) * d);
+        if (!krot) return ORACLE_ERR_NOMEM;
+    }
+    struct rotk_ctx rk = {k, seg_offsets, krot, d, base};
+    parallel_for(nseg, nthreads, rotate_k_segment, &rk);
+
+    const int chunk = 64;
+    long nitems = 0;
+    for (int s = 0; s < nseg; ++s) {
+        long n = seg_offsets[s + 1] - seg_offsets[s];
+        nitems += (n + chunk - 1) / chunk;
+    }
+    long *item_seg = (long *)malloc(sizeof(long) * (size_t)(nitems > 0 ? nitems : 1));
+    long *item_r0 = (long *)malloc(sizeof(long) * (size_t)(nitems > 0 ? nitems : 1));
+    if (!item_seg || !item_r0) {
+        free(item_seg); free(item_r0);
+        if (!k_rot) free(krot);
+        return ORACLE_ERR_NOMEM;
+    }
+    long it = 0;
+    for (int s = 0; s < nseg; ++s) {
+        long n = seg_offsets[s + 1] - seg_offsets[s];
+        for (long r0 = 0; r0 < n; r0 += chunk) {
+            item_seg[it] = s;
+            item_r0[it] = r0;
+            ++it;
+        }
+    }
+    struct prefill_ctx ctx = {q, v, krot, seg_offsets, row_src, gate, y, nseg, d, g, base,
+                              item_seg, item_r0, chunk, ORACLE_OK};
+    parallel_for(nitems, nthreads, prefill_item, &ctx);
+    free(item_seg); free(item_r0);
+    if (!k_rot) free(krot);
+    return ctx.status;
+}
+
+/*
+ * oracle_prefill_rows: the same computation for a chosen list of query rows only
+ * (used for sampled checks at sizes where the full oracle would be slow).
+ *   rows [nrows] packed row indices, heads [nrows] group head j of each query
+ *   out  [nrows, d] fp64 g*h for those queries
+ */
+int oracle_prefill_rows(const uint16_t *q, const uint16_t *k, const uint16_t *v, int nseg, int d, int g,
+                        double base, const int32_t *seg_offsets, const int32_t *row_src, const double *gate,
+                        const int64_t *rows, const int32_t *heads, long nrows, double *out)
+{
+    if (!q || !k || !v || !seg_offsets || !row_src || !gate || !rows || !heads || !out) return ORACLE_ERR_ARG;
+    long R = seg_offsets[nseg];
+    double *tmp = (double *)malloc(sizeof(double) * (size_t)d);
+    double *qr = (double *)malloc(sizeof(double) * (size_t)d);
+    double *h = (double *)malloc(sizeof(double) * (size_t)d);
+    int st = ORACLE_OK;
+    for (long i = 0; i < nrows && st == ORACLE_OK; ++i) {
+        long row = rows[i];
+        int j = heads[i];
+        if (row < 0 || row >= R || j < 0 || j >= g) { st = ORACLE_ERR_ARG; break; }
+        /* the segment containing this row */
+        int lo = 0, hi = nseg;
+        while (hi - lo > 1) {
+            int mid = (lo + hi) / 2;
+            if (seg_offsets[mid] <= row) lo = mid; else hi = mid;
+        }
+        long off = seg_offsets[lo];
+        long r = row - off;
+        double *keys = (double *)malloc(sizeof(double) * (size_t)(r + 1) * d);
+        double *vals = (double *)malloc(sizeof(double) * (size_t)(r + 1) * d);
+        double *w = (double *)malloc(sizeof(double) * (size_t)(r + 1));
+        if (!keys || !vals || !w) { free(keys); free(vals); free(w); st = ORACLE_ERR_NOMEM; break; }
+        for (long s = 0; s <= r; ++s) {
+            for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(k[(off + s) * d + cc]);
+            rope_rotate(tmp, d, (double)s, base, keys + s * d);
+            for (int cc = 0; cc < d; ++cc) vals[s * d + cc] = bf16_to_double(v[(off + s) * d + cc]);
+        }
+        for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(q[(row * g + j) * d + cc]);
+        rope_rotate(tmp, d, (double)r, base, qr);
+        attend(qr, keys, vals, r + 1, d, w, h);
+        double gt = gate[row_src[row]];
+        for (int cc = 0; cc < d; ++cc) out[i * d + cc] = gt * h[cc];
+        free(keys); free(vals); free(w);
+    }
+    free(tmp); free(qr); free(h);
+    return st;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Decode step (Sec. 3.1 last paragraph; Sec. 3.2 "Efficient execution")     */
+/* ------------------------------------------------------------------------- */
+
+/*
+ * oracle_decode_step: one new token per sequence.
+ *   topk_head [B, Kr] selected heads (groups), gate [B, Kr] their gates
+ *   q [B, Kr*g, d] bf16; k, v [B, Kr, d] bf16
+ *   k_cache, v_cache [cap_total, d] fp64 histories (k_cache holds rotated keys);
+ *   seg_base [B*Hr], seg_len [B*Hr] (updated in place), seg_cap [B*Hr]
+ *   y [B, Kr*g, d] fp64: g * h for each selected (group) head
+ * For each (b, slot): rho = seg_len; k~ = k R(rho) and v are appended at rho;
+ * q~ = q R(rho) attends over the rho + 1 entries; seg_len += 1.
+ */
+int oracle_decode_step(const int32_t *topk_head, const double *gate, const uint16_t *q, const uint16_t *k,
+                       const uint16_t *v, int B, int Hr, int Kr, int d, int g, double base,
+                       double *k_cache, double *v_cache, const int64_t *seg_base, int32_t *seg_len,
+                       const int32_t *seg_cap, double *y)
+{
+    if (!topk_head || !gate || !q || !k || !v || !k_cache || !v_cache || !seg_base || !seg_len || !seg_cap || !y)
+        return ORACLE_ERR_ARG;
+    double *tmp = (double *)malloc(sizeof(double) * (size_t)d);
+    double *qr = (double *)malloc(sizeof(double) * (size_t)d);
+    double *h = (double *)malloc(sizeof(double) * (size_t)d);
+    if (!tmp || !qr || !h) { free(tmp); free(qr); free(h); return ORACLE_ERR_NOMEM; }
+    int st = ORACLE_OK;
+    for (int b = 0; b < B && st == ORACLE_OK; ++b) {
+        for (int kk = 0; kk < Kr; ++kk) {
+            int head = topk_head[b * Kr + kk];
+            if (head < 0 || head >= Hr) { st = ORACLE_ERR_ARG; break; }
+            long s = (long)b * Hr + head;
+            long rho = seg_len[s];
+            if (rho >= seg_cap[s]) { st = ORACLE_ERR_CAPACITY; break; }
+            long base_row = seg_base[s];
+            for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(k[((long)b * Kr + kk) * d + cc]);
+            rope_rotate(tmp, d, (double)rho, base, k_cache + (base_row + rho) * d);
+            for (int cc = 0; cc < d; ++cc)
+                v_cache[(base_row + rho) * d + cc] = bf16_to_double(v[((long)b * Kr + kk) * d + cc]);
+            double *w = (double *)malloc(sizeof(double) * (size_t)(rho + 1));
+            if (!w) { st = ORACLE_ERR_NOMEM; break; }
+            for (int j = 0; j < g; ++j) {
+                long qi = ((long)b * Kr + kk) * g + j;
+                for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(q[qi * d + cc]);
+                rope_rotate(tmp, d, (double)rho, base, qr);
+                attend(qr, k_cache + base_row * d, v_cache + base_row * d, rho + 1, d, w, h);
+                for (int cc = 0; cc < d; ++cc) y[qi * d + cc] = gate[b * Kr + kk] * h[cc];
+            }
+            free(w);
+            seg_len[s] = (int32_t)(rho + 1);
+        }
+    }
+    free(tmp); free(qr); free(h);
+    return st;
+}
+
+/* Number of worker threads the oracle would use by default. */
+int oracle_default_threads(void)
+{
+    long n = 1;
+#ifdef _SC_NPROCESSORS_ONLN
+    n = sysconf(_SC_NPROCESSORS_ONLN);
+#endif
+    return n > 0 ? (int)n : 1;
+}

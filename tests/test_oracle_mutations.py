@@ -1,0 +1,52 @@
+"""The oracle's pins must fail when a plausible mistake is planted in the oracle.
+
+Each case copies the oracle's C source to a temporary directory, applies one textual
+mutation (a dropped term, a wrong sign, an off-by-one index, a wrong tie rule ...),
+and runs the pin tests against that copy in a subprocess.  The mutated copy never
+touches the real oracle build.
+"""
+import os
+import shutil
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "namoh_oracle.c")
+
+MUTATIONS = {
+    "rope_sign": ("out[j + half] = x1 * c + x0 * s;", "out[j + half] = x1 * c - x0 * s;"),
+    "no_scale": ("double scale = 1.0 / sqrt((double)d);", "double scale = 1.0;"),
+    "causal_drops_self": ("attend(qr, c->krot + off * d, vals, r + 1, d, w, h);",
+                          "attend(qr, c->krot + off * d, vals, r > 0 ? r : 1, d, w, h);"),
+    "ties_to_upper_index": ("return a < b;", "return a > b;"),
+    "theta_exponent": ("double theta = pow(base, -2.0 * (double)j / (double)d);",
+                       "double theta = pow(base, -1.0 * (double)j / (double)d);"),
+    "gates_renormalised": ("for (int i = 0; i < H; ++i) z += exp((double)s[i] - mx);",
+                           "for (int i = 0; i < K; ++i) z += exp((double)s[order[i]] - mx);"),
+    "query_rank_shift": ("rope_rotate(qin, d, (double)r, c->base, qr);",
+                         "rope_rotate(qin, d, (double)(r + 1), c->base, qr);"),
+    "decode_rank_shift": ("rope_rotate(tmp, d, (double)rho, base, qr);",
+                          "rope_rotate(tmp, d, (double)(rho + 1), base, qr);"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_pins_catch_mutation(tmp_path, name):
+    before, after = MUTATIONS[name]
+    src = open(SRC).read()
+    assert src.count(before) == 1, f"mutation anchor for {name} not found exactly once"
+    shutil.copytree(os.path.join(ROOT, "oracle"), tmp_path / "oracle",
+                    ignore=shutil.ignore_patterns("*.so", "*.tmp*", "__pycache__"))
+    (tmp_path / "oracle" / "namoh_oracle.c").write_text(src.replace(before, after))
+    shutil.copy(os.path.join(ROOT, "namoh_inputs.py"), tmp_path)
+    shutil.copytree(os.path.join(ROOT, "paper_2609_38832_gb300"), tmp_path / "paper_2609_38832_gb300",
+                    ignore=shutil.ignore_patterns("*.so", "__pycache__", "csrc", "_build"))
+    os.makedirs(tmp_path / "tests")
+    for f in ("conftest.py", "test_oracle_route.py", "test_oracle_attention.py", "test_accounting.py"):
+        shutil.copy(os.path.join(ROOT, "tests", f), tmp_path / "tests")
+    shutil.copytree(os.path.join(ROOT, "tests", "golden"), tmp_path / "tests" / "golden")
+    r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider", "-m", "not gpu",
+                        "tests"], cwd=tmp_path, capture_output=True, text=True, timeout=600)
+    assert r.returncode != 0, f"mutation {name} survived the pins:\n{r.stdout[-2000:]}"
