@@ -1,0 +1,201 @@
+/*
+ * namoh.h -- C ABI of the NAMOH routed-attention path on GB300 (sm_103a).
+ *
+ * NAMOH (mixture-of-head native sparse attention): each token activates K of H
+ * heads; each head runs causal attention only over the subsequence of tokens
+ * routed to it, with RoPE applied at the token's rank inside that subsequence.
+ *
+ * Conventions shared by every entry point
+ *   - All array arguments are DEVICE pointers to caller-owned memory, unless a
+ *     comment says otherwise.  The library never allocates, frees or keeps
+ *     device memory in these calls; scratch space is the caller's `workspace`
+ *     (size from the matching *_workspace_size query, 256-byte aligned).
+ *   - bf16 tensors are passed as `uint16_t*` (raw bf16 bit patterns), row-major,
+ *     rows 16-byte aligned.
+ *   - `stream` is a cudaStream_t passed as `void*` (NULL = legacy default
+ *     stream).  Calls only enqueue work on it and return; they never
+ *     synchronise the host.
+ *   - Argument errors are detected on the host before any launch and return a
+ *     negative namoh_status with nothing enqueued.  A launch failure returns
+ *     NAMOH_ERR_CUDA.
+ *   - Data-dependent conditions found on the device (non-finite router logits,
+ *     a full KV segment, a wait that timed out) are OR-ed as NAMOH_DEV_* bits
+ *     into the caller's device word `*dev_status`; read it after synchronising.
+ *     Kernels never trap: the affected outputs are left unspecified.
+ *   - Global state: only a lazily filled per-device cache of properties and the
+ *     driver's tensor-map encoder; calls are thread-safe.
+ *
+ * Notation (the paper's): B sequences of T tokens; H routed query heads, K
+ * active per token; d_head the head width; g query heads per KV group
+ * (App. C "Adopted KV-group routing"; g = 1 without grouping).  With grouping
+ * the router selects Kr = K/g of Hr = H/g groups, and everything keyed by
+ * "head" below is keyed by group.  R = B*T*Kr packed key/value rows.
+ */
+#ifndef NAMOH_H
+#define NAMOH_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define NAMOH_API __attribute__((visibility("default")))
+#else
+#define NAMOH_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Host return codes. */
+typedef enum namoh_status {
+    NAMOH_OK = 0,
+    NAMOH_ERR_INVALID_ARG = -1, /* a pointer, size or alignment violates the contract */
+    NAMOH_ERR_UNSUPPORTED = -2, /* valid but not built: d_head, group, or the device */
+    NAMOH_ERR_WORKSPACE = -3,   /* workspace NULL, misaligned or smaller than required */
+    NAMOH_ERR_CUDA = -4         /* a CUDA runtime/driver call or a launch failed */
+} namoh_status;
+
+/* Bits OR-ed into *dev_status by the kernels. */
+#define NAMOH_DEV_NONFINITE_SCORE 0x1u /* a router logit was NaN or infinite */
+#define NAMOH_DEV_CAPACITY 0x2u        /* a KV segment had no room for its rows */
+#define NAMOH_DEV_TIMEOUT 0x4u         /* a pipeline wait exceeded its limit */
+
+/* Limits of this build. */
+#define NAMOH_MAX_HEADS 64 /* H (or Hr) routed units */
+
+/* Human-readable text for a namoh_status value.  Host function. */
+NAMOH_API const char *namoh_status_string(int status);
+
+/* ABI version: (major << 16) | minor. */
+NAMOH_API int namoh_version(void);
+
+/* ------------------------------------------------------------------------- *
+ * Routing and dispatch.
+ * Sec. 3.1, Eq. (namoh-gates): a_t = softmax(x_t W_r), S_K(t) = TopK(a_t),
+ *   g_{t,i} = m_{t,i} a_{t,i} (not renormalised over the selected heads).
+ * Sec. 3.1: ordered index sets I_i = {t : m_{t,i} = 1}, lengths n_i.
+ * Sec. 3.2, Eq. (namoh-head-rope): rho_i(t) = sum_{s<=t} m_{s,i} - 1.
+ * Sec. 3.2 "Efficient execution": each (batch, head) subsequence is packed as
+ *   one independent sequence.
+ *
+ * scores      [B, T, H] fp32 router logits x_t W_r.  Selection compares these
+ *             exactly (softmax is monotone); ties go to the lower head index.
+ * topk_head   [B, T, K] int32 out: selected heads in descending score order
+ *             ("slots"); every per-slot array below follows this order.
+ * gate        [B, T, K] fp32 out: softmax over all H logits at the selected heads.
+ * The remaining outputs form the packed layout; pass all four, or all four
+ * NULL to skip it (e.g. when routing one decode token):
+ * rank        [B, T, K] int32 out: rho of (t, slot) inside its (b, head) segment.
+ * row         [B, T, K] int32 out: packed row = seg_offsets[b*H + head] + rank.
+ * seg_offsets [B*H + 1] int32 out: exclusive prefix sum of n over (b, head)
+ *             order; seg_offsets[B*H] = B*T*K.  Rows ascend in t in a segment.
+ * row_src     [B*T*K]   int32 out: inverse of row: row_src[row] = (b*T + t)*K + slot.
+ * Requires 1 <= K <= H <= NAMOH_MAX_HEADS, B >= 1, T >= 1, B*T*K < 2^31.
+ * Non-finite logits set NAMOH_DEV_NONFINITE_SCORE (that token's outputs are
+ * unspecified but in range).  Integer outputs are deterministic.
+ * ------------------------------------------------------------------------- */
+NAMOH_API size_t namoh_route_workspace_size(int B, int T, int H, int K);
+NAMOH_API int namoh_route(const float *scores, int B, int T, int H, int K, int32_t *topk_head, float *gate,
+                int32_t *rank, int32_t *row, int32_t *seg_offsets, int32_t *row_src, void *workspace,
+                size_t workspace_bytes, uint32_t *dev_status, void *stream);
+
+/* ------------------------------------------------------------------------- *
+ * Prefill: head-relative RoPE, routed causal attention, gate-weighted combine.
+ * Sec. 3.2, Eq. (namoh-head-rope): q~ = q R(rho), k~ = k R(rho), half-split
+ *   pairs (j, j + d/2), theta_j = rope_base^(-2j/d).
+ * Sec. 3.1, Eq. (namoh-attention): h_{t,i} = softmax(q~ k~^T / sqrt(d)) v over
+ *   s in I_i, s <= t; the combine writes the per-slot term g_{t,i} h_{t,i}
+ *   (the W_O projection is outside this path).
+ * App. C "Adopted KV-group routing": the g query heads of a group share its
+ *   keys, values, gate and rank.
+ * Sec. 3.2 "Efficient execution": length-aware scheduling of query tiles.
+ *
+ * q           [R*g, d] bf16: query of packed row r and group head j at row r*g + j.
+ * k, v        [R, d]   bf16: packed rows in segment order (as produced by the
+ *             routing above with H = Hr, K = Kr).
+ * seg_offsets [B*Hr + 1], row_src [R], gate [R] (indexed by row_src value):
+ *             namoh_route outputs for the Hr-way routing.
+ * y           [B, T, K, d] bf16 out (= [B, T, Kr, g, d]): g_{t,i} h_{t,i} per slot.
+ * k_cache     out: rotated keys k~ (bf16, d per row); v_cache out: values.
+ * seg_base    NULL: the caches are packed like k/v ([R, d]); v_cache may then
+ *             equal v (no copy).  Otherwise [B*Hr] int64 first cache row of
+ *             each segment, with seg_cap [B*Hr] int32 its capacity in rows and
+ *             cache_rows the rows allocated in each cache (for bounds); a
+ *             segment longer than its capacity sets NAMOH_DEV_CAPACITY and its
+ *             rows and outputs are skipped.
+ * seg_len     NULL or [B*Hr] int32 out: n of each segment (decode state).
+ * Supports d_head in {64, 128}, g in {1, 2, 4, 8}, rope_base > 1, T <= 2^20.
+ * k_cache must not alias k.  Runs the three stages below in order.
+ * ------------------------------------------------------------------------- */
+NAMOH_API size_t namoh_prefill_workspace_size(int B, int T, int H, int K, int d_head, int group);
+NAMOH_API int namoh_prefill(const uint16_t *q, const uint16_t *k, const uint16_t *v, int B, int T, int H, int K,
+                  int d_head, int group, float rope_base, const int32_t *seg_offsets, const int32_t *row_src,
+                  const float *gate, uint16_t *y, uint16_t *k_cache, uint16_t *v_cache, const int64_t *seg_base,
+                  const int32_t *seg_cap, int64_t cache_rows, int32_t *seg_len, void *workspace,
+                  size_t workspace_bytes, uint32_t *dev_status, void *stream);
+
+/* ------------------------------------------------------------------------- *
+ * The three stages of namoh_prefill, callable one by one (same arguments and
+ * rules as namoh_prefill unless stated).
+ *
+ * namoh_rope_pack (Sec. 3.2, Eq. namoh-head-rope): rotates every query row to
+ *   its rank into q_rot [R*g, d] bf16 (caller-owned), writes k~ to k_cache and
+ *   copies v to v_cache (unless v_cache == v, allowed only without seg_base).
+ *
+ * namoh_attention_plan (Sec. 3.2 "Efficient execution", length-aware
+ *   scheduling): writes into `plan` (namoh_attention_plan_size bytes, 16-byte
+ *   aligned, caller-owned) the list of 128-row query tiles of every segment and
+ *   group head, longest causal workload first.  Segments longer than seg_cap
+ *   (when seg_cap is not NULL) are left out.  A plan depends only on
+ *   seg_offsets and may be reused by any number of namoh_attention calls on the
+ *   same stream; two calls must not use one plan concurrently.
+ *
+ * namoh_attention (Sec. 3.1, Eq. namoh-attention and the combine): one
+ *   persistent kernel (one CTA per SM) that takes tiles from the plan longest
+ *   first and writes y = g_{t,i} h_{t,i}.  k_cache / v_cache hold k~ and v at
+ *   seg_base (or packed rows when seg_base is NULL).
+ * ------------------------------------------------------------------------- */
+NAMOH_API int namoh_rope_pack(const uint16_t *q, const uint16_t *k, const uint16_t *v, int B, int T, int H, int K,
+                              int d_head, int group, float rope_base, const int32_t *seg_offsets, uint16_t *q_rot,
+                              uint16_t *k_cache, uint16_t *v_cache, const int64_t *seg_base, const int32_t *seg_cap,
+                              int64_t cache_rows, uint32_t *dev_status, void *stream);
+NAMOH_API size_t namoh_attention_plan_size(int B, int T, int H, int K, int group);
+NAMOH_API int namoh_attention_plan(const int32_t *seg_offsets, int B, int T, int H, int K, int group,
+                                   const int32_t *seg_cap, void *plan, size_t plan_bytes, void *stream);
+NAMOH_API int namoh_attention(const uint16_t *q_rot, const uint16_t *k_cache, const uint16_t *v_cache, int B, int T,
+                              int H, int K, int d_head, int group, const int32_t *seg_offsets, const int32_t *row_src,
+                              const float *gate, const int64_t *seg_base, int64_t cache_rows, void *plan,
+                              size_t plan_bytes, uint16_t *y, uint32_t *dev_status, void *stream);
+
+/* ------------------------------------------------------------------------- *
+ * Decode: one new token per sequence.
+ * Sec. 3.1 (last paragraph): the token appends to and attends within only its
+ *   selected heads' caches; prefill and incremental decoding are the same
+ *   causal computation.  Sec. 3.2: the new token's rank is the current length.
+ * Sec. 3.2 "Efficient execution": only active head queries run and only their
+ *   caches are read or updated.
+ *
+ * topk_head, gate [B, Kr]: routing of the new tokens (namoh_route with T = 1).
+ * q [B, K, d], k [B, Kr, d], v [B, Kr, d] bf16: projections of the new tokens
+ *   for the selected (group) heads, in slot order.
+ * For each (b, slot) with head h, segment s = b*Hr + h, rho = seg_len[s]:
+ *   k~ = k R(rho) and v are written at cache row seg_base[s] + rho, every q of
+ *   the group is rotated to rho and attends over the rho + 1 rows, and
+ *   y[b, slot*g + j] = gate * h; finally seg_len[s] = rho + 1.
+ * A full segment (rho >= seg_cap[s]) sets NAMOH_DEV_CAPACITY; its y is zero
+ *   and its length is unchanged.
+ * Supports d_head in {64, 128}, g in {1, 2, 4, 8}.
+ * ------------------------------------------------------------------------- */
+NAMOH_API size_t namoh_decode_workspace_size(int B, int H, int K, int d_head, int group);
+NAMOH_API int namoh_decode(const int32_t *topk_head, const float *gate, const uint16_t *q, const uint16_t *k,
+                 const uint16_t *v, int B, int H, int K, int d_head, int group, float rope_base,
+                 uint16_t *k_cache, uint16_t *v_cache, const int64_t *seg_base, int32_t *seg_len,
+                 const int32_t *seg_cap, int64_t cache_rows, uint16_t *y, void *workspace,
+                 size_t workspace_bytes, uint32_t *dev_status, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* NAMOH_H */

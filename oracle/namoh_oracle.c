@@ -398,7 +398,11 @@ int oracle_prefill_rows(const uint16_t *q, const uint16_t *k, const uint16_t *v,
     double *tmp = (double *)malloc(sizeof(double) * (size_t)d);
     double *qr = (double *)malloc(sizeof(double) * (size_t)d);
     double *h = (double *)malloc(sizeof(double) * (size_t)d);
-    int st = ORACLE_OK;
+    /* rotated keys / widened values of the current segment, extended as needed
+     * (rows listed in segment order reuse them) */
+    double *keys = NULL, *vals = NULL, *w = NULL;
+    long cached_seg = -1, cached_len = 0, cap_rows = 0;
+    int st = (tmp && qr && h) ? ORACLE_OK : ORACLE_ERR_NOMEM;
     for (long i = 0; i < nrows && st == ORACLE_OK; ++i) {
         long row = rows[i];
         int j = heads[i];
@@ -410,23 +414,34 @@ int oracle_prefill_rows(const uint16_t *q, const uint16_t *k, const uint16_t *v,
             if (seg_offsets[mid] <= row) lo = mid; else hi = mid;
         }
         long off = seg_offsets[lo];
+        long n = seg_offsets[lo + 1] - off;
         long r = row - off;
-        double *keys = (double *)malloc(sizeof(double) * (size_t)(r + 1) * d);
-        double *vals = (double *)malloc(sizeof(double) * (size_t)(r + 1) * d);
-        double *w = (double *)malloc(sizeof(double) * (size_t)(r + 1));
-        if (!keys || !vals || !w) { free(keys); free(vals); free(w); st = ORACLE_ERR_NOMEM; break; }
-        for (long s = 0; s <= r; ++s) {
+        if (lo != cached_seg) {
+            cached_seg = lo;
+            cached_len = 0;
+        }
+        if (cap_rows < n) {
+            free(keys); free(vals); free(w);
+            keys = (double *)malloc(sizeof(double) * (size_t)n * d);
+            vals = (double *)malloc(sizeof(double) * (size_t)n * d);
+            w = (double *)malloc(sizeof(double) * (size_t)n);
+            cap_rows = n;
+            cached_len = 0;
+            if (!keys || !vals || !w) { st = ORACLE_ERR_NOMEM; break; }
+        }
+        for (long s = cached_len; s <= r; ++s) {
             for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(k[(off + s) * d + cc]);
             rope_rotate(tmp, d, (double)s, base, keys + s * d);
             for (int cc = 0; cc < d; ++cc) vals[s * d + cc] = bf16_to_double(v[(off + s) * d + cc]);
         }
+        if (r + 1 > cached_len) cached_len = r + 1;
         for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(q[(row * g + j) * d + cc]);
         rope_rotate(tmp, d, (double)r, base, qr);
         attend(qr, keys, vals, r + 1, d, w, h);
         double gt = gate[row_src[row]];
         for (int cc = 0; cc < d; ++cc) out[i * d + cc] = gt * h[cc];
-        free(keys); free(vals); free(w);
     }
+    free(keys); free(vals); free(w);
     free(tmp); free(qr); free(h);
     return st;
 }

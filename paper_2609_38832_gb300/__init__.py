@@ -1,1 +1,218 @@
+"""NAMOH routed attention on GB300 (sm_103a): Python binding of the C ABI.
 
+The three calls keep the C names (``namoh_route``, ``namoh_prefill``,
+``namoh_decode``).  They only marshal torch tensors into device pointers and the
+current CUDA stream; every step of the path runs in the CUDA kernels of
+``libnamoh.so``.  PyTorch supplies device memory and streams.  There is no CPU
+or PyTorch fallback: a missing library or a non-CUDA tensor is an error.
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import Optional
+
+import torch
+
+from . import _abi
+from ._abi import (NAMOH_DEV_CAPACITY, NAMOH_DEV_NONFINITE_SCORE, NAMOH_DEV_TIMEOUT, NamohError)
+
+__all__ = ["namoh_route", "namoh_prefill", "namoh_decode", "namoh_rope_pack", "namoh_attention_plan",
+           "namoh_attention", "RouteOutputs", "Workspace", "NamohError",
+           "NAMOH_DEV_CAPACITY", "NAMOH_DEV_NONFINITE_SCORE", "NAMOH_DEV_TIMEOUT", "library_path"]
+
+
+def library_path() -> str:
+    return _abi.LIB_PATH
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("namoh: every tensor argument must live on a CUDA device")
+    if not t.is_contiguous():
+        raise ValueError("namoh: tensor arguments must be contiguous")
+    return t.data_ptr()
+
+
+def _stream(stream: Optional[torch.cuda.Stream]):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+class Workspace:
+    """A reusable device scratch buffer (grown on demand, 256-byte aligned by the allocator)."""
+
+    def __init__(self, device=None):
+        self.device = device
+        self.buf: Optional[torch.Tensor] = None
+
+    def get(self, nbytes: int, device) -> torch.Tensor:
+        nbytes = max(int(nbytes), 256)
+        if self.buf is None or self.buf.numel() < nbytes or self.buf.device != torch.device(device):
+            self.buf = torch.empty(nbytes, dtype=torch.uint8, device=device)
+        return self.buf
+
+
+def _ws(ws: Optional[Workspace], nbytes: int, device) -> torch.Tensor:
+    return (ws or Workspace()).get(nbytes, device)
+
+
+def _status(status: Optional[torch.Tensor], device) -> torch.Tensor:
+    if status is None:
+        status = torch.zeros(1, dtype=torch.int32, device=device)
+    return status
+
+
+@dataclasses.dataclass
+class RouteOutputs:
+    topk_head: torch.Tensor
+    gate: torch.Tensor
+    rank: Optional[torch.Tensor]
+    row: Optional[torch.Tensor]
+    seg_offsets: Optional[torch.Tensor]
+    row_src: Optional[torch.Tensor]
+    status: torch.Tensor
+
+
+def namoh_route(scores: torch.Tensor, K: int, compact: bool = True, workspace: Optional[Workspace] = None,
+                status: Optional[torch.Tensor] = None, out: Optional[RouteOutputs] = None,
+                stream=None) -> RouteOutputs:
+    """Routing and dispatch of scores [B, T, H] fp32 (see namoh_route in include/namoh.h)."""
+    lib = _abi.load()
+    if scores.dtype != torch.float32 or scores.dim() != 3:
+        raise ValueError("scores must be a [B, T, H] float32 tensor")
+    B, T, H = scores.shape
+    dev = scores.device
+    if out is None:
+        i32 = dict(dtype=torch.int32, device=dev)
+        out = RouteOutputs(
+            topk_head=torch.empty((B, T, K), **i32), gate=torch.empty((B, T, K), dtype=torch.float32, device=dev),
+            rank=torch.empty((B, T, K), **i32) if compact else None,
+            row=torch.empty((B, T, K), **i32) if compact else None,
+            seg_offsets=torch.empty(B * H + 1, **i32) if compact else None,
+            row_src=torch.empty(B * T * K, **i32) if compact else None,
+            status=_status(status, dev))
+    nbytes = lib.namoh_route_workspace_size(B, T, H, K)
+    ws = _ws(workspace, nbytes, dev)
+    rc = lib.namoh_route(_ptr(scores), B, T, H, K, _ptr(out.topk_head), _ptr(out.gate), _ptr(out.rank), _ptr(out.row),
+                         _ptr(out.seg_offsets), _ptr(out.row_src), _ptr(ws), ws.numel(), _ptr(out.status),
+                         _stream(stream))
+    _abi.check("namoh_route", rc)
+    return out
+
+
+def namoh_prefill(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, seg_offsets: torch.Tensor,
+                  row_src: torch.Tensor, gate: torch.Tensor, *, B: int, T: int, H: int, K: int, group: int = 1,
+                  rope_base: float = 10000.0, y: Optional[torch.Tensor] = None,
+                  k_cache: Optional[torch.Tensor] = None, v_cache: Optional[torch.Tensor] = None,
+                  seg_base: Optional[torch.Tensor] = None, seg_cap: Optional[torch.Tensor] = None,
+                  seg_len: Optional[torch.Tensor] = None, workspace: Optional[Workspace] = None,
+                  status: Optional[torch.Tensor] = None, stream=None):
+    """Prefill over packed rows (see namoh_prefill in include/namoh.h).
+
+    q [R*g, d], k / v [R, d] bf16; returns (y [B, T, K, d], k_cache, v_cache).
+    With v_cache omitted and no seg_base, v itself serves as the value cache.
+    """
+    lib = _abi.load()
+    d = q.shape[-1]
+    dev = q.device
+    for name, t in (("q", q), ("k", k), ("v", v)):
+        if t.dtype != torch.bfloat16:
+            raise ValueError(f"{name} must be bfloat16")
+    if y is None:
+        y = torch.empty((B, T, K, d), dtype=torch.bfloat16, device=dev)
+    if k_cache is None:
+        k_cache = torch.empty_like(k)
+    if v_cache is None:
+        v_cache = v if seg_base is None else torch.empty_like(v)
+    cache_rows = k_cache.shape[0]
+    nbytes = lib.namoh_prefill_workspace_size(B, T, H, K, d, group)
+    if nbytes == 0:
+        raise NamohError("namoh_prefill_workspace_size", _abi.NAMOH_ERR_UNSUPPORTED)
+    ws = _ws(workspace, nbytes, dev)
+    st = _status(status, dev)
+    rc = lib.namoh_prefill(_ptr(q), _ptr(k), _ptr(v), B, T, H, K, d, group, float(rope_base), _ptr(seg_offsets),
+                           _ptr(row_src), _ptr(gate), _ptr(y), _ptr(k_cache), _ptr(v_cache), _ptr(seg_base),
+                           _ptr(seg_cap), cache_rows, _ptr(seg_len), _ptr(ws), ws.numel(), _ptr(st), _stream(stream))
+    _abi.check("namoh_prefill", rc)
+    return y, k_cache, v_cache
+
+
+def namoh_rope_pack(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, seg_offsets: torch.Tensor, *, B: int, T: int,
+                    H: int, K: int, group: int = 1, rope_base: float = 10000.0, q_rot: Optional[torch.Tensor] = None,
+                    k_cache: Optional[torch.Tensor] = None, v_cache: Optional[torch.Tensor] = None,
+                    seg_base: Optional[torch.Tensor] = None, seg_cap: Optional[torch.Tensor] = None,
+                    status: Optional[torch.Tensor] = None, stream=None):
+    """Prefill stage 1: RoPE at rank and cache pack.  Returns (q_rot, k_cache, v_cache)."""
+    lib = _abi.load()
+    d = q.shape[-1]
+    dev = q.device
+    q_rot = torch.empty_like(q) if q_rot is None else q_rot
+    k_cache = torch.empty_like(k) if k_cache is None else k_cache
+    if v_cache is None:
+        v_cache = v if seg_base is None else torch.empty_like(v)
+    st = _status(status, dev)
+    rc = lib.namoh_rope_pack(_ptr(q), _ptr(k), _ptr(v), B, T, H, K, d, group, float(rope_base), _ptr(seg_offsets),
+                             _ptr(q_rot), _ptr(k_cache), _ptr(v_cache), _ptr(seg_base), _ptr(seg_cap),
+                             k_cache.shape[0], _ptr(st), _stream(stream))
+    _abi.check("namoh_rope_pack", rc)
+    return q_rot, k_cache, v_cache
+
+
+def namoh_attention_plan(seg_offsets: torch.Tensor, *, B: int, T: int, H: int, K: int, group: int = 1,
+                         seg_cap: Optional[torch.Tensor] = None, plan: Optional[torch.Tensor] = None,
+                         stream=None) -> torch.Tensor:
+    """Prefill stage 2: the longest-first tile list.  Returns the plan buffer (uint8 tensor)."""
+    lib = _abi.load()
+    nbytes = lib.namoh_attention_plan_size(B, T, H, K, group)
+    if nbytes == 0:
+        raise NamohError("namoh_attention_plan_size", _abi.NAMOH_ERR_INVALID_ARG)
+    if plan is None or plan.numel() < nbytes:
+        plan = torch.empty(nbytes, dtype=torch.uint8, device=seg_offsets.device)
+    rc = lib.namoh_attention_plan(_ptr(seg_offsets), B, T, H, K, group, _ptr(seg_cap), _ptr(plan), plan.numel(),
+                                  _stream(stream))
+    _abi.check("namoh_attention_plan", rc)
+    return plan
+
+
+def namoh_attention(q_rot: torch.Tensor, k_cache: torch.Tensor, v_cache: torch.Tensor, seg_offsets: torch.Tensor,
+                    row_src: torch.Tensor, gate: torch.Tensor, plan: torch.Tensor, *, B: int, T: int, H: int, K: int,
+                    group: int = 1, seg_base: Optional[torch.Tensor] = None, y: Optional[torch.Tensor] = None,
+                    status: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Prefill stage 3: routed causal attention + gate-weighted combine.  Returns y [B, T, K, d]."""
+    lib = _abi.load()
+    d = q_rot.shape[-1]
+    dev = q_rot.device
+    if y is None:
+        y = torch.empty((B, T, K, d), dtype=torch.bfloat16, device=dev)
+    st = _status(status, dev)
+    rc = lib.namoh_attention(_ptr(q_rot), _ptr(k_cache), _ptr(v_cache), B, T, H, K, d, group, _ptr(seg_offsets),
+                             _ptr(row_src), _ptr(gate), _ptr(seg_base), k_cache.shape[0], _ptr(plan), plan.numel(),
+                             _ptr(y), _ptr(st), _stream(stream))
+    _abi.check("namoh_attention", rc)
+    return y
+
+
+def namoh_decode(topk_head: torch.Tensor, gate: torch.Tensor, q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, *,
+                 H: int, K: int, group: int = 1, rope_base: float = 10000.0, k_cache: torch.Tensor,
+                 v_cache: torch.Tensor, seg_base: torch.Tensor, seg_len: torch.Tensor, seg_cap: torch.Tensor,
+                 y: Optional[torch.Tensor] = None, workspace: Optional[Workspace] = None,
+                 status: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """One decode step (see namoh_decode in include/namoh.h).  Returns y [B, K, d] bf16."""
+    lib = _abi.load()
+    B = topk_head.shape[0]
+    d = q.shape[-1]
+    dev = q.device
+    if y is None:
+        y = torch.empty((B, K, d), dtype=torch.bfloat16, device=dev)
+    nbytes = lib.namoh_decode_workspace_size(B, H, K, d, group)
+    if nbytes == 0:
+        raise NamohError("namoh_decode_workspace_size", _abi.NAMOH_ERR_UNSUPPORTED)
+    ws = _ws(workspace, nbytes, dev)
+    st = _status(status, dev)
+    rc = lib.namoh_decode(_ptr(topk_head), _ptr(gate), _ptr(q), _ptr(k), _ptr(v), B, H, K, d, group,
+                          float(rope_base), _ptr(k_cache), _ptr(v_cache), _ptr(seg_base), _ptr(seg_len),
+                          _ptr(seg_cap), k_cache.shape[0], _ptr(y), _ptr(ws), ws.numel(), _ptr(st), _stream(stream))
+    _abi.check("namoh_decode", rc)
+    return y

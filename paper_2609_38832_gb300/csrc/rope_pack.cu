@@ -1,0 +1,105 @@
+// rope_pack.cu -- head-relative RoPE at the packed rank (Sec. 3.2, Eq. namoh-head-rope).
+//
+// One group of D/16 threads per packed row r: the row's segment s is found by binary
+// search over seg_offsets, rho = r - seg_offsets[s].  Each thread owns 8 rotation pairs
+// (j, j + D/2) and moves them with 16-byte loads/stores.  The angle is computed once per
+// row and applied to K and to all g query heads of the row (KV-group routing shares the
+// rank, App. C).  Outputs: Q~ (bf16 scratch for the attention kernel), K~ into the key
+// cache, and V copied into the value cache unless the caller passed v_cache == v.
+#include "common.cuh"
+
+namespace namoh {
+
+template <int D>
+__global__ void __launch_bounds__(256) rope_pack_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ k,
+                                                        const uint16_t* __restrict__ v, int R, int g,
+                                                        const int32_t* __restrict__ seg_offsets, int nseg,
+                                                        const int64_t* __restrict__ seg_base,
+                                                        const int32_t* __restrict__ seg_cap, long long cache_rows,
+                                                        uint16_t* __restrict__ q_rot, uint16_t* __restrict__ k_cache,
+                                                        uint16_t* __restrict__ v_cache, int copy_v, RopeTable tab,
+                                                        uint32_t* __restrict__ status) {
+  constexpr int LPR = D / 16;  // threads per row
+  constexpr int HALF = D / 2;
+  const int lane_in_row = threadIdx.x % LPR;
+  const int j0 = lane_in_row * 8;
+  const long long groups = (long long)gridDim.x * (blockDim.x / LPR);
+  float th_hi[8], th_lo[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    th_hi[i] = tab.theta_hi[j0 + i];
+    th_lo[i] = tab.theta_lo[j0 + i];
+  }
+  for (long long r = (long long)blockIdx.x * (blockDim.x / LPR) + threadIdx.x / LPR; r < R; r += groups) {
+    // segment of row r: last s with seg_offsets[s] <= r
+    int lo = 0, hi = nseg;
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (__ldg(seg_offsets + mid) <= r) lo = mid; else hi = mid;
+    }
+    const int rho = (int)(r - __ldg(seg_offsets + lo));
+    long long dst = r;
+    bool write_cache = true;
+    if (seg_base) {
+      dst = __ldg(seg_base + lo) + rho;
+      if (rho >= __ldg(seg_cap + lo) || dst < 0 || dst >= cache_rows) {
+        write_cache = false;
+        if (lane_in_row == 0) report(status, NAMOH_DEV_CAPACITY);
+      }
+    }
+    float sn[8], cs[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) rope_sincos((float)rho, th_hi[i], th_lo[i], tab, &sn[i], &cs[i]);
+
+    auto rotate = [&](const uint16_t* src, uint16_t* dst_row) {
+      const uint4 a = __ldg(reinterpret_cast<const uint4*>(src + j0));
+      const uint4 b = __ldg(reinterpret_cast<const uint4*>(src + HALF + j0));
+      const uint32_t av[4] = {a.x, a.y, a.z, a.w};
+      const uint32_t bv[4] = {b.x, b.y, b.z, b.w};
+      uint32_t oa[4], ob[4];
+#pragma unroll
+      for (int p = 0; p < 4; ++p) {
+        const float x0 = bf16_lo(av[p]), x1 = bf16_hi(av[p]);
+        const float y0 = bf16_lo(bv[p]), y1 = bf16_hi(bv[p]);
+        const int i0 = 2 * p, i1 = 2 * p + 1;
+        // x'_j = x_j cos - x_{j+D/2} sin ;  x'_{j+D/2} = x_{j+D/2} cos + x_j sin
+        oa[p] = pack_bf16x2(fmaf(x0, cs[i0], -y0 * sn[i0]), fmaf(x1, cs[i1], -y1 * sn[i1]));
+        ob[p] = pack_bf16x2(fmaf(y0, cs[i0], x0 * sn[i0]), fmaf(y1, cs[i1], x1 * sn[i1]));
+      }
+      *reinterpret_cast<uint4*>(dst_row + j0) = make_uint4(oa[0], oa[1], oa[2], oa[3]);
+      *reinterpret_cast<uint4*>(dst_row + HALF + j0) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
+    };
+
+    for (int j = 0; j < g; ++j) rotate(q + ((size_t)r * g + j) * D, q_rot + ((size_t)r * g + j) * D);
+    if (write_cache) {
+      rotate(k + (size_t)r * D, k_cache + (size_t)dst * D);
+      if (copy_v) {
+        const uint4* vs = reinterpret_cast<const uint4*>(v + (size_t)r * D);
+        uint4* vd = reinterpret_cast<uint4*>(v_cache + (size_t)dst * D);
+        vd[lane_in_row] = __ldg(vs + lane_in_row);
+        vd[lane_in_row + LPR] = __ldg(vs + lane_in_row + LPR);
+      }
+    }
+  }
+}
+
+cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const uint16_t* v, int R, int g,
+                             const int32_t* seg_offsets, int nseg, const int64_t* seg_base, const int32_t* seg_cap,
+                             long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache, bool copy_v,
+                             const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream) {
+  if (R == 0) return cudaSuccess;
+  const int threads = 256;
+  const int rows_per_block = threads / (D / 16);
+  long long blocks = ((long long)R + rows_per_block - 1) / rows_per_block;
+  const long long cap = (long long)sm_count * 8;
+  if (blocks > cap) blocks = cap;
+  if (D == 128)
+    rope_pack_kernel<128><<<(int)blocks, threads, 0, stream>>>(q, k, v, R, g, seg_offsets, nseg, seg_base, seg_cap,
+                                                               cache_rows, q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status);
+  else
+    rope_pack_kernel<64><<<(int)blocks, threads, 0, stream>>>(q, k, v, R, g, seg_offsets, nseg, seg_base, seg_cap,
+                                                              cache_rows, q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status);
+  return cudaGetLastError();
+}
+
+}  // namespace namoh

@@ -1,0 +1,279 @@
+// route.cu -- routing and dispatch (Sec. 3.1 Eq. namoh-gates; Sec. 3.2 Eq. namoh-head-rope).
+//
+// Four launches, all stream-ordered, no host synchronisation:
+//   1. route_topk_kernel   one thread per token: TopK of the fp32 logits (descending,
+//                          ties to the lower head index), fp32 softmax gates over all H,
+//                          and per-chunk head counts (one block = one 256-token chunk).
+//   2. route_scan_chunks   per sequence: exclusive scan of the chunk counts over chunks
+//                          for every head -> chunk base ranks; totals n[b, h].
+//   3. route_scan_segments exclusive scan of n over (b, h) -> seg_offsets.
+//   4. route_rank_kernel   per chunk: warp ballots give each (token, slot) its rank among
+//                          the chunk's earlier tokens for that head; adds the chunk base
+//                          -> rank, row and row_src.
+// All integer work is exact, so the packed layout is deterministic and bit-identical to
+// a sequential append in token order.
+#include <float.h>
+
+#include "common.cuh"
+
+namespace namoh {
+namespace {
+
+constexpr int kChunk = 256;  // tokens per block in the top-K and rank kernels
+
+template <int HMAX>
+__global__ void __launch_bounds__(kChunk) route_topk_kernel(const float* __restrict__ scores, int T, int H, int K,
+                                                            int nchunks, int32_t* __restrict__ topk_head,
+                                                            float* __restrict__ gate,
+                                                            int32_t* __restrict__ chunk_count,
+                                                            uint32_t* __restrict__ status) {
+  extern __shared__ float s_scores[];  // [kChunk][H + 1]
+  __shared__ int s_cnt[NAMOH_MAX_HEADS];
+  __shared__ int s_bad;
+  const int c = blockIdx.x;
+  const int b = blockIdx.y;
+  const int t0 = c * kChunk;
+  const int ntok = min(kChunk, T - t0);
+  const int tid = threadIdx.x;
+  const int lane = tid & 31, warp = tid >> 5;
+  const int ld = H + 1;
+  if (tid < NAMOH_MAX_HEADS) s_cnt[tid] = 0;
+  if (tid == 0) s_bad = 0;
+
+  // coalesced staging: one warp per token row
+  const float* src = scores + ((size_t)b * T + t0) * H;
+  for (int r = warp; r < ntok; r += kChunk / 32)
+    for (int h = lane; h < H; h += 32) s_scores[r * ld + h] = __ldg(src + (size_t)r * H + h);
+  __syncthreads();
+
+  if (tid < ntok) {
+    float sc[HMAX];
+    bool bad = false;
+#pragma unroll
+    for (int h = 0; h < HMAX; ++h) {
+      float x = (h < H) ? s_scores[tid * ld + h] : -FLT_MAX;
+      if (h < H && !isfinite(x)) {
+        bad = true;
+        x = -FLT_MAX;
+      }
+      sc[h] = x;
+    }
+    // softmax denominator over all H logits (fp32)
+    float mx = -FLT_MAX;
+#pragma unroll
+    for (int h = 0; h < HMAX; ++h)
+      if (h < H) mx = fmaxf(mx, sc[h]);
+    float z = 0.f;
+#pragma unroll
+    for (int h = 0; h < HMAX; ++h)
+      if (h < H) z += expf(sc[h] - mx);
+    const float inv_z = 1.0f / z;
+
+    // K passes; pass k picks the best head strictly after the previous pick in the
+    // total order (score desc, index asc).
+    float pv = 0.f;
+    int pi = -1;
+    const size_t base = ((size_t)b * T + t0 + tid) * K;
+    for (int k = 0; k < K; ++k) {
+      float bv = 0.f;
+      int bi = -1;
+#pragma unroll
+      for (int h = 0; h < HMAX; ++h) {
+        const float x = sc[h];
+        const bool elig = (h < H) && (pi < 0 || x < pv || (x == pv && h > pi));
+        const bool better = elig && (bi < 0 || x > bv);
+        bv = better ? x : bv;
+        bi = better ? h : bi;
+      }
+      topk_head[base + k] = bi;
+      gate[base + k] = expf(bv - mx) * inv_z;
+      if (chunk_count) atomicAdd(&s_cnt[bi], 1);
+      pv = bv;
+      pi = bi;
+    }
+    if (bad) s_bad = 1;
+  }
+  __syncthreads();
+  if (chunk_count && tid < H) chunk_count[((size_t)b * nchunks + c) * H + tid] = s_cnt[tid];
+  if (tid == 0 && s_bad) report(status, NAMOH_DEV_NONFINITE_SCORE);
+}
+
+// Per sequence b (one block): for every head, exclusive scan of chunk counts over chunks.
+// Thread (h, p) owns the chunk range [p*per, (p+1)*per).
+__global__ void __launch_bounds__(1024) route_scan_chunks(const int32_t* __restrict__ chunk_count, int H,
+                                                          int nchunks, int32_t* __restrict__ chunk_base,
+                                                          int32_t* __restrict__ n_out) {
+  __shared__ int s_part[1024];
+  const int b = blockIdx.x;
+  const int tid = threadIdx.x;
+  const int P = blockDim.x / H;  // parts per head
+  const int h = tid % H, p = tid / H;
+  const int per = (nchunks + P - 1) / P;
+  const int c0 = p * per, c1 = min(nchunks, c0 + per);
+  const int32_t* cc = chunk_count + (size_t)b * nchunks * H;
+  int sum = 0;
+  if (p < P)
+    for (int c = c0; c < c1; ++c) sum += cc[(size_t)c * H + h];
+  s_part[tid] = (p < P) ? sum : 0;
+  __syncthreads();
+  if (p < P) {
+    int before = 0;
+    for (int q = 0; q < p; ++q) before += s_part[q * H + h];
+    int run = before;
+    int32_t* out = chunk_base + (size_t)b * nchunks * H;
+    for (int c = c0; c < c1; ++c) {
+      out[(size_t)c * H + h] = run;
+      run += cc[(size_t)c * H + h];
+    }
+    if (p == P - 1) n_out[(size_t)b * H + h] = run;
+  }
+}
+
+// One block: seg_offsets = exclusive scan of n over (b, h) order.
+__global__ void __launch_bounds__(1024) route_scan_segments(const int32_t* __restrict__ n, int nseg,
+                                                            int32_t* __restrict__ seg_offsets) {
+  __shared__ int s_sum[1024];
+  const int tid = threadIdx.x;
+  const int per = (nseg + blockDim.x - 1) / blockDim.x;
+  const int i0 = tid * per, i1 = min(nseg, i0 + per);
+  int sum = 0;
+  for (int i = i0; i < i1; ++i) sum += n[i];
+  s_sum[tid] = sum;
+  __syncthreads();
+  // Hillis-Steele inclusive scan over the per-thread sums
+  for (int off = 1; off < (int)blockDim.x; off <<= 1) {
+    int v = (tid >= off) ? s_sum[tid - off] : 0;
+    __syncthreads();
+    s_sum[tid] += v;
+    __syncthreads();
+  }
+  int run = s_sum[tid] - sum;
+  for (int i = i0; i < i1; ++i) {
+    seg_offsets[i] = run;
+    run += n[i];
+  }
+  if (tid == blockDim.x - 1) seg_offsets[nseg] = s_sum[tid];
+}
+
+// Per chunk: rank = chunk base + rank among this chunk's earlier tokens for the head.
+__global__ void __launch_bounds__(kChunk) route_rank_kernel(const int32_t* __restrict__ topk_head, int T, int H,
+                                                            int K, int nchunks,
+                                                            const int32_t* __restrict__ chunk_base,
+                                                            const int32_t* __restrict__ seg_offsets,
+                                                            int32_t* __restrict__ rank, int32_t* __restrict__ row,
+                                                            int32_t* __restrict__ row_src) {
+  __shared__ uint32_t s_bal[kChunk / 32][NAMOH_MAX_HEADS];
+  __shared__ int s_wbase[kChunk / 32][NAMOH_MAX_HEADS];
+  __shared__ int s_cbase[NAMOH_MAX_HEADS];  // rank of the chunk's first token for each head
+  __shared__ int s_soff[NAMOH_MAX_HEADS];   // segment offset of each head in this sequence
+  const int c = blockIdx.x, b = blockIdx.y;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int t = c * kChunk + tid;
+  const bool valid = t < T;
+  const size_t tok = (size_t)b * T + t;
+  if (tid < H) {
+    s_cbase[tid] = chunk_base[((size_t)b * nchunks + c) * H + tid];
+    s_soff[tid] = seg_offsets[(size_t)b * H + tid];
+  }
+  uint64_t mask = 0;
+  if (valid)
+    for (int k = 0; k < K; ++k) mask |= 1ull << topk_head[tok * K + k];
+  for (int h = 0; h < H; ++h) {
+    const uint32_t bal = __ballot_sync(0xffffffffu, (mask >> h) & 1ull);
+    if (lane == 0) s_bal[warp][h] = bal;
+  }
+  __syncthreads();
+  for (int i = tid; i < (kChunk / 32) * H; i += kChunk) {
+    const int w = i / H, h = i % H;
+    int before = 0;
+    for (int q = 0; q < w; ++q) before += __popc(s_bal[q][h]);
+    s_wbase[w][h] = before;
+  }
+  __syncthreads();
+  if (!valid) return;
+  const uint32_t lt = (1u << lane) - 1u;
+  for (int k = 0; k < K; ++k) {
+    const int h = topk_head[tok * K + k];
+    const int rho = s_cbase[h] + s_wbase[warp][h] + __popc(s_bal[warp][h] & lt);
+    const int r = s_soff[h] + rho;
+    rank[tok * K + k] = rho;
+    row[tok * K + k] = r;
+    row_src[r] = (int32_t)(tok * K + k);
+  }
+}
+
+template <int HMAX>
+cudaError_t launch_topk(const float* scores, int B, int T, int H, int K, int nchunks, int32_t* topk, float* gate,
+                        int32_t* chunk_count, uint32_t* status, cudaStream_t stream) {
+  const size_t smem = (size_t)kChunk * (H + 1) * sizeof(float);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(route_topk_kernel<HMAX>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  dim3 grid(nchunks, B);
+  route_topk_kernel<HMAX><<<grid, kChunk, smem, stream>>>(scores, T, H, K, nchunks, topk, gate, chunk_count, status);
+  return cudaGetLastError();
+}
+
+}  // namespace
+}  // namespace namoh
+
+using namespace namoh;
+
+extern "C" size_t namoh_route_workspace_size(int B, int T, int H, int K) {
+  if (B < 1 || T < 1 || H < 1 || K < 1) return 0;
+  const size_t nchunks = ((size_t)T + kChunk - 1) / kChunk;
+  WorkspaceCarver ws{nullptr, 0, 0};
+  ws.take<int32_t>((size_t)B * nchunks * H);  // chunk counts
+  ws.take<int32_t>((size_t)B * nchunks * H);  // chunk bases
+  ws.take<int32_t>((size_t)B * H);            // n
+  return align_up(ws.used, 256);
+}
+
+extern "C" int namoh_route(const float* scores, int B, int T, int H, int K, int32_t* topk_head, float* gate,
+                           int32_t* rank, int32_t* row, int32_t* seg_offsets, int32_t* row_src, void* workspace,
+                           size_t workspace_bytes, uint32_t* dev_status, void* stream_v) {
+  if (!scores || !topk_head || !gate || !dev_status) return NAMOH_ERR_INVALID_ARG;
+  if (B < 1 || T < 1 || H < 1 || K < 1 || K > H || H > NAMOH_MAX_HEADS) return NAMOH_ERR_INVALID_ARG;
+  if ((long long)B * T * K >= (1ll << 31) || (long long)B * H >= (1ll << 20)) return NAMOH_ERR_INVALID_ARG;
+  const bool compact = seg_offsets != nullptr;
+  if (compact != (rank != nullptr) || compact != (row != nullptr) || compact != (row_src != nullptr))
+    return NAMOH_ERR_INVALID_ARG;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
+  const int nchunks = (T + kChunk - 1) / kChunk;
+
+  int32_t* chunk_count = nullptr;
+  int32_t* chunk_base = nullptr;
+  int32_t* n = nullptr;
+  if (compact) {
+    if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return NAMOH_ERR_WORKSPACE;
+    WorkspaceCarver ws{static_cast<char*>(workspace), workspace_bytes, 0};
+    chunk_count = ws.take<int32_t>((size_t)B * nchunks * H);
+    chunk_base = ws.take<int32_t>((size_t)B * nchunks * H);
+    n = ws.take<int32_t>((size_t)B * H);
+    if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
+  }
+
+  cudaError_t e;
+  if (H <= 8)
+    e = launch_topk<8>(scores, B, T, H, K, nchunks, topk_head, gate, chunk_count, dev_status, stream);
+  else if (H <= 16)
+    e = launch_topk<16>(scores, B, T, H, K, nchunks, topk_head, gate, chunk_count, dev_status, stream);
+  else if (H <= 32)
+    e = launch_topk<32>(scores, B, T, H, K, nchunks, topk_head, gate, chunk_count, dev_status, stream);
+  else
+    e = launch_topk<64>(scores, B, T, H, K, nchunks, topk_head, gate, chunk_count, dev_status, stream);
+  if (e != cudaSuccess) return NAMOH_ERR_CUDA;
+  if (!compact) return NAMOH_OK;
+
+  const int scan_threads = 1024 - (1024 % H);
+  route_scan_chunks<<<B, scan_threads, 0, stream>>>(chunk_count, H, nchunks, chunk_base, n);
+  if (cudaGetLastError() != cudaSuccess) return NAMOH_ERR_CUDA;
+  route_scan_segments<<<1, 1024, 0, stream>>>(n, B * H, seg_offsets);
+  if (cudaGetLastError() != cudaSuccess) return NAMOH_ERR_CUDA;
+  route_rank_kernel<<<dim3(nchunks, B), kChunk, 0, stream>>>(topk_head, T, H, K, nchunks, chunk_base, seg_offsets,
+                                                             rank, row, row_src);
+  if (cudaGetLastError() != cudaSuccess) return NAMOH_ERR_CUDA;
+  return NAMOH_OK;
+}

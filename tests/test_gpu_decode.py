@@ -1,0 +1,198 @@
+"""GPU parity of the decode step (Sec. 3.1 last paragraph; Sec. 3.2 "Efficient execution").
+
+Each new token routes (T = 1), appends k~ and v to its selected heads' caches at rank
+seg_len, attends over seg_len + 1 rows, writes g * h and bumps seg_len.
+"""
+import numpy as np
+import pytest
+import torch
+
+import namoh_inputs as ni
+from _gpu_helpers import assert_close_attention, bf16_to_f64, dev_bf16, host_bf16_bits
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def namoh():
+    import paper_2609_38832_gb300 as pkg
+    return pkg
+
+
+def _prefix_state(namoh, B, T, Hr, Kr, d, g, base, headroom, seed):
+    """GPU prefill of a T-token prefix into caches with `headroom` free rows per segment."""
+    scores = ni.router_scores(seed, B, T, Hr)
+    R = B * T * Kr
+    q, k, v = ni.qkv_rows(seed, R, d, g)
+    ro = namoh.namoh_route(torch.from_numpy(scores).cuda(), Kr)
+    seg = ro.seg_offsets.cpu().numpy().astype(np.int64)
+    nseg = B * Hr
+    seg_base = seg[:-1] + np.arange(nseg) * headroom
+    n = seg[1:] - seg[:-1]
+    cap = (n + headroom).astype(np.int32)
+    rows = int(seg[-1] + nseg * headroom)
+    kc = torch.zeros((rows, d), dtype=torch.bfloat16, device="cuda")
+    vc = torch.zeros((rows, d), dtype=torch.bfloat16, device="cuda")
+    seg_len = torch.zeros(nseg, dtype=torch.int32, device="cuda")
+    namoh.namoh_prefill(dev_bf16(q), dev_bf16(k), dev_bf16(v), ro.seg_offsets, ro.row_src, ro.gate, B=B, T=T,
+                        H=Hr * g, K=Kr * g, group=g, rope_base=base, k_cache=kc, v_cache=vc,
+                        seg_base=torch.from_numpy(seg_base).cuda(), seg_cap=torch.from_numpy(cap).cuda(),
+                        seg_len=seg_len, status=ro.status)
+    torch.cuda.synchronize()
+    assert int(ro.status.item()) == 0
+    return dict(kc=kc, vc=vc, seg_len=seg_len, seg_base=seg_base, cap=cap, n=n,
+                seg_base_d=torch.from_numpy(seg_base).cuda(), cap_d=torch.from_numpy(cap).cuda())
+
+
+def _oracle_caches(st, d):
+    """fp64 copies of the GPU caches (the oracle continues from the same stored prefix)."""
+    kc = bf16_to_f64(st["kc"]).copy()
+    vc = bf16_to_f64(st["vc"]).copy()
+    return kc, vc, st["seg_base"].astype(np.int64).copy(), st["seg_len"].cpu().numpy().astype(np.int32).copy(), \
+        st["cap"].astype(np.int32).copy()
+
+
+@pytest.mark.parametrize("B,T,Hr,Kr,d,g,steps", [
+    (3, 300, 8, 2, 128, 1, 5),
+    (2, 257, 4, 4, 64, 1, 3),
+    (2, 200, 4, 2, 128, 2, 4),
+    (1, 130, 8, 1, 128, 8, 3),
+    (64, 40, 32, 4, 128, 1, 2),
+])
+def test_decode_matches_oracle(namoh, oracle_mod, B, T, Hr, Kr, d, g, steps):
+    base = 10000.0
+    st = _prefix_state(namoh, B, T, Hr, Kr, d, g, base, steps, seed=21)
+    okc, ovc, obase, olen, ocap = _oracle_caches(st, d)
+    sc, q, k, v = ni.decode_step_inputs(22, steps, B, Hr, Kr, d, g)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for t in range(steps):
+        ro = namoh.namoh_route(torch.from_numpy(sc[t][:, None, :]).cuda(), Kr, compact=False)
+        y = namoh.namoh_decode(ro.topk_head.view(B, Kr), ro.gate.view(B, Kr), dev_bf16(q[t]), dev_bf16(k[t]),
+                               dev_bf16(v[t]), H=Hr * g, K=Kr * g, group=g, rope_base=base, k_cache=st["kc"],
+                               v_cache=st["vc"], seg_base=st["seg_base_d"], seg_len=st["seg_len"],
+                               seg_cap=st["cap_d"], status=status)
+        torch.cuda.synchronize()
+        ref = oracle_mod.route(sc[t][:, None, :], Kr)
+        np.testing.assert_array_equal(ro.topk_head.cpu().numpy(), ref["topk_head"])
+        y_ref = oracle_mod.decode_step(ref["topk_head"][:, 0], ref["gate"][:, 0], q[t], k[t], v[t], Hr, d, g, base,
+                                       okc, ovc, obase, olen, ocap)
+        gate = np.repeat(ref["gate"][:, 0], g, axis=1)
+        assert_close_attention(bf16_to_f64(y), y_ref, gate, what=f"step {t}")
+        np.testing.assert_array_equal(st["seg_len"].cpu().numpy(), olen)
+    assert int(status.item()) == 0
+    # M_KV = T K after the prefix and + K per step (App. C Eq. app-routed-kv)
+    assert int(st["seg_len"].sum().item()) == B * (T + steps) * Kr
+
+
+def test_prefill_then_decode_equals_longer_prefill(namoh, oracle_mod):
+    """Prefill over T tokens plus decode steps reproduces prefill over T + steps tokens."""
+    B, T, Hr, Kr, d, steps, base = 2, 200, 8, 2, 128, 3, 10000.0
+    Tt = T + steps
+    s = ni.router_scores(31, B, Tt, Hr)
+    R = B * Tt * Kr
+    q, k, v = ni.qkv_rows(31, R, d)
+    ref = oracle_mod.route(s, Kr)
+    ro = namoh.namoh_route(torch.from_numpy(s).cuda(), Kr)
+    y_full, _, _ = namoh.namoh_prefill(dev_bf16(q), dev_bf16(k), dev_bf16(v), ro.seg_offsets, ro.row_src, ro.gate,
+                                       B=B, T=Tt, H=Hr, K=Kr, rope_base=base)
+    # prefix rows: the packed rows of tokens < T keep their order
+    tok = ref["row_src"] // Kr % Tt
+    keep = np.nonzero(tok < T)[0]
+    ro_p = namoh.namoh_route(torch.from_numpy(np.ascontiguousarray(s[:, :T])).cuda(), Kr)
+    seg = ro_p.seg_offsets.cpu().numpy().astype(np.int64)
+    nseg = B * Hr
+    seg_base = seg[:-1] + np.arange(nseg) * steps
+    cap = (seg[1:] - seg[:-1] + steps).astype(np.int32)
+    rows = int(seg[-1] + nseg * steps)
+    kc = torch.zeros((rows, d), dtype=torch.bfloat16, device="cuda")
+    vc = torch.zeros_like(kc)
+    seg_len = torch.zeros(nseg, dtype=torch.int32, device="cuda")
+    sb, cp = torch.from_numpy(seg_base).cuda(), torch.from_numpy(cap).cuda()
+    namoh.namoh_prefill(dev_bf16(q[keep]), dev_bf16(k[keep]), dev_bf16(v[keep]), ro_p.seg_offsets, ro_p.row_src,
+                        ro_p.gate, B=B, T=T, H=Hr, K=Kr, rope_base=base, k_cache=kc, v_cache=vc, seg_base=sb,
+                        seg_cap=cp, seg_len=seg_len)
+    yf = bf16_to_f64(y_full).reshape(B, Tt, Kr, d)
+    for t in range(T, Tt):
+        rows_t = ref["row"][:, t]
+        yd = namoh.namoh_decode(ro.topk_head[:, t].contiguous(), ro.gate[:, t].contiguous(), dev_bf16(q[rows_t]),
+                                dev_bf16(k[rows_t]), dev_bf16(v[rows_t]), H=Hr, K=Kr, rope_base=base, k_cache=kc,
+                                v_cache=vc, seg_base=sb, seg_len=seg_len, seg_cap=cp)
+        torch.cuda.synchronize()
+        assert_close_attention(bf16_to_f64(yd), yf[:, t], ref["gate"][:, t], what=f"token {t}")
+
+
+def test_decode_full_segment_sets_capacity(namoh):
+    B, T, Hr, Kr, d = 2, 100, 4, 2, 128
+    st = _prefix_state(namoh, B, T, Hr, Kr, d, 1, 1e4, 0, seed=41)  # no headroom: every segment is full
+    sc, q, k, v = ni.decode_step_inputs(42, 1, B, Hr, Kr, d)
+    ro = namoh.namoh_route(torch.from_numpy(sc[0][:, None, :]).cuda(), Kr, compact=False)
+    before = st["seg_len"].clone()
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    y = namoh.namoh_decode(ro.topk_head.view(B, Kr), ro.gate.view(B, Kr), dev_bf16(q[0]), dev_bf16(k[0]),
+                           dev_bf16(v[0]), H=Hr, K=Kr, k_cache=st["kc"], v_cache=st["vc"], seg_base=st["seg_base_d"],
+                           seg_len=st["seg_len"], seg_cap=st["cap_d"], status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) & namoh.NAMOH_DEV_CAPACITY
+    assert torch.equal(st["seg_len"], before)
+    assert float(y.float().abs().max().item()) == 0.0
+
+
+def test_decode_full_size_sampled(namoh, oracle_mod):
+    """64 sequences with 131072-token routed prefixes (H = 32, K = 4, d = 128): the 17 GB cache
+    is seeded N(0, 1) bf16 on the device; two decode steps; 8 sequences checked against the oracle."""
+    wl = ni.DECODE
+    B, Hr, Kr, d = wl.B, wl.Hr, wl.Kr, wl.d
+    s = ni.router_scores(wl.seed, B, wl.prefix, Hr)
+    ro = namoh.namoh_route(torch.from_numpy(s).cuda(), Kr)
+    del s
+    seg = ro.seg_offsets.cpu().numpy().astype(np.int64)
+    del ro
+    steps = 2
+    nseg = B * Hr
+    n = seg[1:] - seg[:-1]
+    seg_base = seg[:-1] + np.arange(nseg) * steps
+    cap = (n + steps).astype(np.int32)
+    rows = int(seg[-1] + nseg * steps)
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(wl.seed)
+    kc = torch.randn((rows, d), generator=gen, device="cuda", dtype=torch.bfloat16)
+    vc = torch.randn((rows, d), generator=gen, device="cuda", dtype=torch.bfloat16)
+    seg_len = torch.from_numpy(n.astype(np.int32)).cuda()
+    sb, cp = torch.from_numpy(seg_base).cuda(), torch.from_numpy(cap).cuda()
+    sc, q, k, v = ni.decode_step_inputs(wl.seed, steps, B, Hr, Kr, d)
+    check = list(range(0, B, 8))
+    # oracle copies of the checked sequences' segments
+    o_kc = {}
+    for b in check:
+        for h in range(Hr):
+            sidx = b * Hr + h
+            lo, hi = int(seg_base[sidx]), int(seg_base[sidx] + cap[sidx])
+            o_kc[sidx] = (bf16_to_f64(kc[lo:hi]), bf16_to_f64(vc[lo:hi]))
+    o_len = n.astype(np.int32).copy()
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for t in range(steps):
+        rt = namoh.namoh_route(torch.from_numpy(sc[t][:, None, :]).cuda(), Kr, compact=False)
+        y = namoh.namoh_decode(rt.topk_head.view(B, Kr), rt.gate.view(B, Kr), dev_bf16(q[t]), dev_bf16(k[t]),
+                               dev_bf16(v[t]), H=Hr, K=Kr, rope_base=wl.base, k_cache=kc, v_cache=vc, seg_base=sb,
+                               seg_len=seg_len, seg_cap=cp, status=status)
+        torch.cuda.synchronize()
+        yh = bf16_to_f64(y)
+        top = rt.topk_head.view(B, Kr).cpu().numpy()
+        gate = rt.gate.view(B, Kr).cpu().numpy().astype(np.float64)
+        for b in check:
+            for slot in range(Kr):
+                sidx = b * Hr + int(top[b, slot])
+                okc, ovc = o_kc[sidx]
+                one_base = np.zeros(1, np.int64)
+                one_len = o_len[sidx:sidx + 1].copy()
+                one_cap = cap[sidx:sidx + 1].copy()
+                y_ref = oracle_mod.decode_step(np.zeros((1, 1), np.int32), gate[b:b + 1, slot:slot + 1],
+                                               q[t][b:b + 1, slot:slot + 1], k[t][b:b + 1, slot:slot + 1],
+                                               v[t][b:b + 1, slot:slot + 1], 1, d, 1, wl.base, okc, ovc, one_base,
+                                               one_len, one_cap)
+                o_len[sidx] = one_len[0]
+                assert_close_attention(yh[b:b + 1, slot:slot + 1], y_ref, gate[b:b + 1, slot:slot + 1],
+                                       what=f"step {t} seq {b} slot {slot}")
+        np.testing.assert_array_equal(seg_len.cpu().numpy()[[b * Hr + h for b in check for h in range(Hr)]],
+                                      o_len[[b * Hr + h for b in check for h in range(Hr)]])
+    assert int(status.item()) == 0
