@@ -3,8 +3,10 @@
 Step (the whole hot path over one batch): route + dispatch, RoPE at rank / cache pack,
 length-aware plan, routed causal attention with the gate-weighted combine, on the
 balanced prefill workload (4 sequences x 4096 tokens, H = 16, K = 4, d = 128, bf16,
-RoPE base 1e4), inputs resident in HBM.  L2 (129 MB) is flushed by writing a 512 MB
-buffer before every timed step, because that workload's inputs (51 MB) fit in L2.
+RoPE base 1e4), inputs resident in HBM.  L2 (129 MB) is flushed by writing a 2 GB
+buffer before every timed step, because that workload's inputs (51 MB) fit in L2.  The
+flush also keeps the GPU busy while the host enqueues the step, so the CUDA events
+between stages measure device time without host launch gaps (checked and reported).
 
 The decode workload (64 sequences with 131072-token routed prefixes, H = 32, K = 4,
 d = 128, 17.4 GB KV cache) is measured in the same run and reported under "decode".
@@ -131,7 +133,7 @@ def cpu_model():
 
 
 # --------------------------------------------------------------------------- oracle (CPU baseline)
-def oracle_prefill_sample(wl: ni.PrefillWorkload, min_seconds: float = 10.0, max_reps: int = 8):
+def oracle_prefill_sample(wl: ni.PrefillWorkload, min_seconds: float = 10.0, max_reps: int = 64):
     """The oracle, as it stands, on the full workload (route + prefill), repeated until min_seconds."""
     import oracle
     oracle.build()
@@ -181,7 +183,7 @@ def run_gpu(args, rank: int, world: int):
     k_cache = torch.empty_like(k)
     plan = namoh.namoh_attention_plan(ro.seg_offsets, B=B, T=T, H=H, K=K, group=g)
     y = torch.empty((B, T, K, d), dtype=torch.bfloat16, device=dev)
-    flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
+    flush = torch.empty(2 << 30, dtype=torch.uint8, device=dev)
 
     def step(ev=None):
         if ev is not None:
@@ -201,6 +203,7 @@ def run_gpu(args, rank: int, world: int):
         if ev is not None:
             ev[4].record()
 
+    clocks = ClockSampler(dev.index).__enter__()
     for _ in range(args.warmup):
         flush.fill_(1)
         step()
@@ -208,16 +211,24 @@ def run_gpu(args, rank: int, world: int):
     n_seg = acc.segment_lengths(ro.seg_offsets.cpu().numpy())
     flops = acc.attention_flops(n_seg, d, g)
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
+    fl_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+    enqueue_s = []
     barrier(world)
     torch.cuda.synchronize()
-    with ClockSampler(dev.index) as clocks:
-        t0 = time.perf_counter()
-        for i in range(args.steps):
-            flush.fill_(i & 0xFF)
-            step(evs[i])
-        torch.cuda.synchronize()
-        wall = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        fl_ev[i][0].record()
+        flush.fill_(i & 0xFF)
+        fl_ev[i][1].record()
+        te = time.perf_counter()
+        step(evs[i])
+        enqueue_s.append(time.perf_counter() - te)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t0
     barrier(world)
+    flush_ms = [a.elapsed_time(b) for a, b in fl_ev]
+    # the host finished enqueueing each step before the flush ahead of it ended
+    gapless = all(e * 1e3 < f for e, f in zip(enqueue_s, flush_ms))
     stage = np.array([[evs[i][j].elapsed_time(evs[i][j + 1]) for j in range(4)] for i in range(args.steps)])
     step_ms = float(stage.sum(1).mean())
     step_ms = max_over_ranks(step_ms, world)
@@ -292,14 +303,16 @@ def run_gpu(args, rank: int, world: int):
                 "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                 "api": "namoh_route + namoh_prefill from pinned host buffers, y copied back"},
         "gpu_launches": 7 * args.steps,
-        "clocks": clocks.summary(),
         "wall_s_timed_region": wall,
+        "host_enqueue_ms_max": 1e3 * max(enqueue_s), "flush_ms_min": min(flush_ms), "stage_timing_gapless": gapless,
         "device_status": st,
     }
 
     if not args.no_decode:
         line["decode"] = run_decode(args, dev, pk, pk_kind)
         line["gpu_launches"] += line["decode"].pop("launches")
+    clocks.__exit__(None, None, None)
+    line["clocks"] = clocks.summary()
     return line
 
 
