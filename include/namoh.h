@@ -101,6 +101,33 @@ NAMOH_API int namoh_route(const float *scores, int B, int T, int H, int K, int32
                 size_t workspace_bytes, uint32_t *dev_status, void *stream);
 
 /* ------------------------------------------------------------------------- *
+ * namoh_route_noalloc: namoh_route without a workspace argument.
+ * The paper has no counterpart; this is a convenience of this library.
+ *
+ * For callers that cannot allocate device memory around the call: code running
+ * inside a stream capture (cudaMalloc/cudaFree are not capturable and may
+ * synchronise the device), latency-critical serving loops that must never
+ * synchronise, and runtimes that own every byte of device memory through their
+ * own pools and forbid side allocations.  The scratch that namoh_route takes
+ * from `workspace` comes instead from a 4 MiB array compiled into the library
+ * (every GPU that loads the library holds it until the process exits).
+ *
+ * Arguments, outputs and rules are those of namoh_route.  Shapes whose
+ * namoh_route_workspace_size exceeds 4 MiB return NAMOH_ERR_WORKSPACE with
+ * nothing enqueued (e.g. B*ceil(T/256)*H <= about 500000 fits).  The call
+ * allocates nothing.  The first call on each device resolves the array's device
+ * address (cudaGetSymbolAddress) with that device current; make that first call
+ * before any stream capture.  Every call on a device shares the one array and
+ * leaves its last contents there (the routing kernels overwrite every word they
+ * read, so nothing has to be cleared); calls that overlap on the GPU -- on
+ * different streams, or from different host threads -- race on it and must be
+ * serialised by the caller.
+ * ------------------------------------------------------------------------- */
+NAMOH_API int namoh_route_noalloc(const float *scores, int B, int T, int H, int K, int32_t *topk_head, float *gate,
+                                  int32_t *rank, int32_t *row, int32_t *seg_offsets, int32_t *row_src,
+                                  uint32_t *dev_status, void *stream);
+
+/* ------------------------------------------------------------------------- *
  * Prefill: head-relative RoPE, routed causal attention, gate-weighted combine.
  * Sec. 3.2, Eq. (namoh-head-rope): q~ = q R(rho), k~ = k R(rho), half-split
  *   pairs (j, j + d/2), theta_j = rope_base^(-2j/d).

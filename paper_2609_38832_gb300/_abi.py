@@ -34,6 +34,7 @@ SIGNATURES = {
     "namoh_version": (_I, []),
     "namoh_route_workspace_size": (_SZ, [_I, _I, _I, _I]),
     "namoh_route": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P]),
+    "namoh_route_noalloc": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P]),
     "namoh_prefill_workspace_size": (_SZ, [_I, _I, _I, _I, _I, _I]),
     "namoh_prefill": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _P, _P, _P, _I64, _P, _P,
                            _SZ, _P, _P]),

@@ -277,3 +277,46 @@ extern "C" int namoh_route(const float* scores, int B, int T, int H, int K, int3
   if (cudaGetLastError() != cudaSuccess) return NAMOH_ERR_CUDA;
   return NAMOH_OK;
 }
+
+// ---------------------------------------------------------------------------
+// Routing with built-in scratch (no caller workspace, no allocation).
+// The scratch is a file-scope device array; host code only ever passes the
+// device address obtained from cudaGetSymbolAddress, never the array's name.
+// ---------------------------------------------------------------------------
+#include <mutex>
+
+namespace namoh {
+namespace {
+constexpr size_t kRouteStaticScratchBytes = 4u << 20;  // 4 MiB on every device that loads the library
+static __device__ __align__(256) unsigned char g_route_scratch[kRouteStaticScratchBytes];
+
+constexpr int kMaxScratchDevices = 64;
+std::mutex g_scratch_mutex;
+void* g_scratch_addr[kMaxScratchDevices] = {};
+
+// Device address of g_route_scratch on the current device (resolved once per device).
+void* route_scratch_address() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxScratchDevices) return nullptr;
+  std::lock_guard<std::mutex> lock(g_scratch_mutex);
+  if (!g_scratch_addr[dev]) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_route_scratch) != cudaSuccess) return nullptr;
+    g_scratch_addr[dev] = ptr;
+  }
+  return g_scratch_addr[dev];
+}
+}  // namespace
+}  // namespace namoh
+
+extern "C" int namoh_route_noalloc(const float* scores, int B, int T, int H, int K, int32_t* topk_head, float* gate,
+                                   int32_t* rank, int32_t* row, int32_t* seg_offsets, int32_t* row_src,
+                                   uint32_t* dev_status, void* stream) {
+  if (!scores || !topk_head || !gate || !dev_status) return NAMOH_ERR_INVALID_ARG;
+  if (B < 1 || T < 1 || H < 1 || K < 1 || K > H || H > NAMOH_MAX_HEADS) return NAMOH_ERR_INVALID_ARG;
+  if (seg_offsets && namoh_route_workspace_size(B, T, H, K) > kRouteStaticScratchBytes) return NAMOH_ERR_WORKSPACE;
+  void* scratch = route_scratch_address();
+  if (!scratch) return NAMOH_ERR_CUDA;
+  return namoh_route(scores, B, T, H, K, topk_head, gate, rank, row, seg_offsets, row_src, scratch,
+                     kRouteStaticScratchBytes, dev_status, stream);
+}
