@@ -290,7 +290,7 @@ def run_gpu(args, rank: int, world: int):
         "data": "synthetic",
         "config": {"workload": wl.name, "B": B, "T": T, "H": H, "K": K, "d_head": d, "group": g,
                    "rope_base": wl.base, "parallelism": f"replicas{world}",
-                   "l2": "flushed before every timed step (512 MB write)", "seed": wl.seed,
+                   "l2": "flushed before every timed step (2 GB write)", "seed": wl.seed,
                    "c_attn": acc.interaction_count(n_seg, g), "flops_per_step": flops,
                    "cv2_mean": float(np.mean([acc.cv2(n_seg[b * wl.Hr:(b + 1) * wl.Hr]) for b in range(B)]))},
         "stages_ms": {"route": float(stage[:, 0].mean()), "rope_pack": float(stage[:, 1].mean()),
