@@ -59,7 +59,9 @@ typedef enum namoh_status {
 /* Bits OR-ed into *dev_status by the kernels. */
 #define NAMOH_DEV_NONFINITE_SCORE 0x1u /* a router logit was NaN or infinite */
 #define NAMOH_DEV_CAPACITY 0x2u        /* a KV segment had no room for its rows */
-#define NAMOH_DEV_TIMEOUT 0x4u         /* a pipeline wait exceeded its limit */
+#define NAMOH_DEV_TIMEOUT 0x4u         /* a pipeline wait exceeded its limit; bits 16-23 then
+                                          hold the barrier's index in its kernel's barrier block
+                                          and bits 24-31 the warp that gave up */
 
 /* Limits of this build. */
 #define NAMOH_MAX_HEADS 64 /* H (or Hr) routed units */
@@ -69,6 +71,11 @@ NAMOH_API const char *namoh_status_string(int status);
 
 /* ABI version: (major << 16) | minor. */
 NAMOH_API int namoh_version(void);
+
+/* Detail of the last NAMOH_ERR_CUDA returned on the calling thread: which launch
+ * or CUDA call failed and the CUDA error name and text.  Thread-local, valid
+ * until the thread's next failing call.  Host function. */
+NAMOH_API const char *namoh_last_error_string(void);
 
 /* ------------------------------------------------------------------------- *
  * Routing and dispatch.
@@ -118,8 +125,9 @@ NAMOH_API int namoh_route(const float *scores, int B, int T, int H, int K, int32
  * allocates nothing.  The first call on each device resolves the array's device
  * address (cudaGetSymbolAddress) with that device current; make that first call
  * before any stream capture.  Every call on a device shares the one array and
- * leaves its last contents there (the routing kernels overwrite every word they
- * read, so nothing has to be cleared); calls that overlap on the GPU -- on
+ * leaves its last contents there; the only word that must start at zero (a
+ * ticket counter) is cleared by the first routing kernel of each call, and every
+ * other word is written before it is read.  Calls that overlap on the GPU -- on
  * different streams, or from different host threads -- race on it and must be
  * serialised by the caller.
  * ------------------------------------------------------------------------- */

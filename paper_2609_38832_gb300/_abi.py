@@ -32,6 +32,7 @@ _F = ctypes.c_float
 SIGNATURES = {
     "namoh_status_string": (ctypes.c_char_p, [_I]),
     "namoh_version": (_I, []),
+    "namoh_last_error_string": (ctypes.c_char_p, []),
     "namoh_route_workspace_size": (_SZ, [_I, _I, _I, _I]),
     "namoh_route": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P]),
     "namoh_route_noalloc": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P]),
@@ -52,6 +53,8 @@ class NamohError(RuntimeError):
     def __init__(self, fn: str, status: int):
         self.status = status
         text = load().namoh_status_string(status).decode() if _lib is not None else str(status)
+        if status == NAMOH_ERR_CUDA and _lib is not None:
+            text += ": " + _lib.namoh_last_error_string().decode()
         super().__init__(f"{fn} returned {status} ({text})")
 
 

@@ -1,6 +1,7 @@
 // api.cu -- shared host-side pieces of the C ABI: status strings, the per-device
 // property cache, the driver tensor-map encoder and the RoPE frequency table.
 #include <math.h>
+#include <stdio.h>
 #include <mutex>
 
 #include "common.cuh"
@@ -43,6 +44,22 @@ bool current_device_info(DeviceInfo* out) {
   *out = info;
   return true;
 }
+
+namespace {
+thread_local char g_last_error[160] = "no error";
+}
+
+int cuda_fail(cudaError_t e, const char* where) {
+  snprintf(g_last_error, sizeof g_last_error, "%s: %s (%s)", where, cudaGetErrorName(e), cudaGetErrorString(e));
+  return NAMOH_ERR_CUDA;
+}
+
+int cuda_check_launch(const char* where) {
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? NAMOH_OK : cuda_fail(e, where);
+}
+
+const char* last_error_text() { return g_last_error; }
 
 EncodeTiledFn tensor_map_encoder() {
   std::call_once(g_encoder_once, [] {
@@ -94,3 +111,5 @@ extern "C" const char* namoh_status_string(int status) {
 }
 
 extern "C" int namoh_version(void) { return (1 << 16) | 0; }
+
+extern "C" const char* namoh_last_error_string(void) { return namoh::last_error_text(); }

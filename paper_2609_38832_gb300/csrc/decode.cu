@@ -347,7 +347,7 @@ extern "C" int namoh_decode(const int32_t* topk_head, const float* gate, const u
   carve_decode(ws, &dw, pairs, g, D);
   if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
   DeviceInfo info;
-  if (!current_device_info(&info)) return NAMOH_ERR_CUDA;
+  if (!current_device_info(&info)) return cuda_fail(cudaGetLastError(), "device query");
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
 
   RopeTable tab;
@@ -360,7 +360,7 @@ extern "C" int namoh_decode(const int32_t* topk_head, const float* gate, const u
     decode_append_kernel<64><<<pairs, 32, 0, stream>>>(topk_head, q, k, v, Hr, Kr, g, k_cache, v_cache, seg_base,
                                                        seg_len, seg_cap, cache_rows, tab, dw.q_rot, dw.info,
                                                        dev_status);
-  if (cudaGetLastError() != cudaSuccess) return NAMOH_ERR_CUDA;
+  if (const int st = cuda_check_launch("decode_append_kernel launch")) return st;
 
   const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)D));
   int splits = 1;
@@ -368,12 +368,12 @@ extern "C" int namoh_decode(const int32_t* topk_head, const float* gate, const u
                                                    scale_log2, dw.part, stream, &splits)
                              : launch_split_g<64>(g, k_cache, v_cache, dw.q_rot, dw.info, pairs, info.sm_count,
                                                   scale_log2, dw.part, stream, &splits);
-  if (e != cudaSuccess) return NAMOH_ERR_CUDA;
+  if (e != cudaSuccess) return cuda_fail(e, "decode_split_kernel launch");
   const int mthreads = g * D < 1024 ? g * D : 1024;
   if (D == 128)
     decode_merge_kernel<128><<<pairs, mthreads, 0, stream>>>(dw.info, gate, dw.part, splits, g, y, seg_len);
   else
     decode_merge_kernel<64><<<pairs, mthreads, 0, stream>>>(dw.info, gate, dw.part, splits, g, y, seg_len);
-  if (cudaGetLastError() != cudaSuccess) return NAMOH_ERR_CUDA;
+  if (const int st = cuda_check_launch("decode_merge_kernel launch")) return st;
   return NAMOH_OK;
 }

@@ -3,27 +3,32 @@
 // "Efficient execution": packed variable-length subsequences and length-aware scheduling;
 // App. C "Adopted KV-group routing" for g > 1).
 //
-// Work unit ("item"): one 128-row query tile of one segment for one group head j.  Within
-// a segment, queries and keys share local ranks, so query tile qt needs key tiles 0..qt
-// and only tile qt is masked (key rank <= query rank).
+// Work unit ("item"): one 128-row query tile t of one segment for one group head j.  Within
+// a segment, queries and keys share local ranks, so tile t needs key tiles 0..t and only
+// tile t is masked (key rank <= query rank).
 //
 // Schedule (length-aware, longest first): a one-block "plan" kernel lists the items in
-// order of decreasing cost (qt + 1 key tiles).  The persistent attention kernel launches
+// order of decreasing cost (t + 1 key tiles).  The persistent attention kernel launches
 // one CTA per SM; each CTA's producer warp takes the next item from an atomic counter
 // (greedy list scheduling in longest-first order) and hands it to the other warps through
 // a two-slot ring in shared memory.  The last CTA to finish resets the counter, so a plan
 // can be reused by later launches on the same stream.
 //
 // Attention CTA (192 threads, one CTA per SM):
-//   warp 0      TMA producer: Q tile, then K and V tiles into 2-stage rings (128B swizzle)
-//   warp 1      MMA issuer (one lane) and TMEM owner: S = Q K^T into one of two TMEM
-//               S buffers, then O += P V into the TMEM O accumulator (tcgen05, M = 128)
-//   warps 2-5   softmax / epilogue: thread i owns query row i (TMEM lane i).  Online
-//               softmax in fp32 with exp2; the running max is only moved when it grows by
-//               more than 2^8 (then O in TMEM is rescaled); P is written to shared memory
-//               as bf16 in the MMA operand layout.  The epilogue divides by the row sum,
-//               multiplies by the routing gate and scatters bf16 rows to y[row_src].
-// TMEM: S0 = cols [0,128), S1 = [128,256), O = [256, 256 + D).
+//   warps 0-3   softmax / epilogue: thread i owns query row i (TMEM lane i).  Online
+//               softmax in fp32 with exp2; the running max only moves when it grows by
+//               more than 2^8 (O in TMEM is then rescaled).  P is written back to TMEM as
+//               bf16 over the S columns it came from.  The epilogue divides by the row
+//               sum, multiplies by the routing gate and scatters bf16 rows to y[row_src].
+//   warp 4      TMA producer: the Q tile, then K(0), K(1), V(0), K(2), V(1), ... through a
+//               6-slot ring (128B swizzle) two key tiles ahead of the MMAs.
+//   warp 5      MMA issuer (one lane) and TMEM owner.  tcgen05.mma instructions into one
+//               accumulator run back to back while instructions into different
+//               accumulators overlap, so with three S/P buffers the issuer interleaves
+//               PV(kv) (A = P in TMEM, B = V as the MN-major operand) with S(kv+2) = Q K^T
+//               instruction by instruction while the softmax works on S(kv+1).
+// TMEM: S/P buffers at cols [0,128), [128,256), [256,384); O at [384, 384 + D).
+// Shared memory (d = 128): Q 32 KB + 6 x 32 KB ring = 224 KB.
 // Every mbarrier wait is bounded (NAMOH_DEV_TIMEOUT, then all roles drain and exit).
 #include "common.cuh"
 
@@ -36,35 +41,44 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
 
 namespace attn {
 
-constexpr int BM = 128;             // query rows per tile
-constexpr int BN = 128;             // keys per tile
-constexpr int kThreads = 192;       // 6 warps
+constexpr int BM = 128;              // query rows per tile (one tile per work item)
+constexpr int BN = 128;              // keys per tile
+constexpr int kItemRows = BM;
+constexpr int kSoftmaxWarps = 4;     // warps 0-3: thread i owns query row i (TMEM lane i)
+constexpr int kWarpLoad = 4;
+constexpr int kWarpMma = 5;
+constexpr int kThreads = 192;
 constexpr int kTmemCols = 512;
-constexpr int kTmemS0 = 0, kTmemS1 = 128, kTmemO = 256;
+constexpr int kSBufs = 3;            // S/P buffers in TMEM
+// TMEM columns: S/P buffers at 0, 128, 256; O at 384.  P (bf16, two per 32-bit column)
+// overwrites the first BN/2 columns of the S buffer it was computed from.
+__host__ __device__ constexpr uint32_t tmem_s_col(int b) { return 128u * (uint32_t)b; }
+constexpr uint32_t kTmemO = 384;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
+constexpr int kRing = 6;                   // K/V ring: K(0), K(1), V(0), K(2), V(1), K(3), ...
 
 template <int D>
 struct Smem {
-  static constexpr int kAtoms = D / 64;                  // 64-column (128-byte) swizzle atoms per row
-  static constexpr int kTileBytes = BM * D * 2;          // one Q / K / V tile
-  static constexpr int kAtomBytes = BM * 128;            // 16 KB: 128 rows x 128 bytes
+  static constexpr int kAtoms = D / 64;          // 64-column (128-byte) swizzle atoms per row
+  static constexpr int kTileBytes = BM * D * 2;  // one Q / K / V tile
+  static constexpr int kAtomBytes = BM * 128;    // 16 KB: 128 rows x 128 bytes
   static constexpr int kQ = 0;
-  static constexpr int kK0 = kQ + kTileBytes;
-  static constexpr int kV0 = kK0 + 2 * kTileBytes;
-  static constexpr int kP = kV0 + 2 * kTileBytes;
-  static constexpr int kPBytes = BM * BN * 2;
-  static constexpr int kBar = kP + kPBytes;
-  static constexpr int kBytes = kBar + 256;
-  static constexpr int kAlloc = kBytes + 1024;           // slack for 1024-byte alignment
+  static constexpr int kRing0 = kTileBytes;
+  static constexpr int kBar = kRing0 + kRing * kTileBytes;
+  static constexpr int kBytes = kBar + 512;
+  static constexpr int kAlloc = kBytes + 1024;   // slack for 1024-byte alignment
 };
 
 struct Bars {
   uint64_t item_full[2], item_empty[2];
   uint64_t q_full, q_empty;
-  uint64_t k_full[2], k_empty[2];
-  uint64_t v_full[2], v_empty[2];
-  uint64_t s_full[2], s_free[2];
-  uint64_t p_full, o_ready, o_free;
+  uint64_t ring_full[kRing], ring_empty[kRing];
+  uint64_t s_full[kSBufs];  // S written into buffer b (one barrier per buffer: at an item
+                            // boundary two S are issued back to back, and a parity wait
+                            // must never fall two phases behind)
+  uint64_t p_full;   // P of the current key tile in TMEM (and O rescaled if needed)
+  uint64_t o_ready;  // a PV completed (in issue order)
+  uint64_t o_free;   // epilogue finished reading O
   uint64_t drain;
   int2 item_slot[2];
   uint32_t tmem_base;
@@ -76,7 +90,7 @@ struct Params {
   const int64_t* seg_base;     // [nseg] or null (cache rows = packed rows)
   const int32_t* row_src;      // [R]
   const float* gate;           // [R] indexed by row_src value
-  const int2* items;           // {segment * g + j, qt}, longest first
+  const int2* items;           // {segment * g + j, query tile}, longest first
   const int* nitems;
   int* sched;                  // [0] next item, [1] CTAs finished
   uint16_t* y;                 // [R * g, D] indexed by row_src * g + j
@@ -123,30 +137,27 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     for (int i = 0; i < 2; ++i) {
       mbar_init(&bars->item_full[i], 1);
-      mbar_init(&bars->item_empty[i], 5);  // MMA warp + 4 softmax warps
+      mbar_init(&bars->item_empty[i], 1 + kSoftmaxWarps);
+    }
+    for (int i = 0; i < kRing; ++i) {
+      mbar_init(&bars->ring_full[i], 1);
+      mbar_init(&bars->ring_empty[i], 1);
     }
     mbar_init(&bars->q_full, 1);
     mbar_init(&bars->q_empty, 1);
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&bars->k_full[i], 1);
-      mbar_init(&bars->k_empty[i], 1);
-      mbar_init(&bars->v_full[i], 1);
-      mbar_init(&bars->v_empty[i], 1);
-      mbar_init(&bars->s_full[i], 1);
-      mbar_init(&bars->s_free[i], 4);
-    }
-    mbar_init(&bars->p_full, 4);
+    for (int i = 0; i < kSBufs; ++i) mbar_init(&bars->s_full[i], 1);
+    mbar_init(&bars->p_full, kSoftmaxWarps);
     mbar_init(&bars->o_ready, 1);
-    mbar_init(&bars->o_free, 4);
+    mbar_init(&bars->o_free, kSoftmaxWarps);
     mbar_init(&bars->drain, 1);
     bars->abort_flag = 0;
     mbar_fence_init();
   }
-  if (warp == 1) {
+  if (warp == kWarpMma) {
     tmem_alloc(&bars->tmem_base, kTmemCols);
     tmem_relinquish();
   }
-  if (warp == 0 && lane == 0) {
+  if (warp == kWarpLoad && lane == 0) {
     tma_prefetch_desc(&tm_q);
     tma_prefetch_desc(&tm_k);
     tma_prefetch_desc(&tm_v);
@@ -156,11 +167,22 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = bars->tmem_base;
 
-  if (warp == 0) {
-    // ------------------------------------------------------------------ producer
+  if (warp == kWarpLoad) {
+    // ------------------------------------------------------------------ TMA producer
     if (lane == 0) {
-      uint32_t kv_iter = 0, item_iter = 0;
+      uint32_t ring_iter = 0, item_iter = 0;
       bool ok = true;
+      auto load_tile = [&](const CUtensorMap* tm, int32_t row) {
+        const int slot = ring_iter % kRing;
+        const uint32_t use = ring_iter / kRing;
+        if (use > 0 && !mbar_wait(&bars->ring_empty[slot], (use - 1) & 1, abort_flag, p.status)) return false;
+        mbar_arrive_expect_tx(&bars->ring_full[slot], L::kTileBytes);
+        for (int a = 0; a < L::kAtoms; ++a)
+          tma_load_2d(smem + L::kRing0 + slot * L::kTileBytes + a * L::kAtomBytes, tm, a * 64, row,
+                      &bars->ring_full[slot]);
+        ++ring_iter;
+        return true;
+      };
       while (ok) {
         const int it = atomicAdd(p.sched, 1);
         const int2 item = it < nitems ? p.items[it] : make_int2(-1, -1);
@@ -172,27 +194,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (item.x < 0) break;
         const int seg = item.x / p.g, j = item.x % p.g, qt = item.y;
         const int off = p.seg_offsets[seg];
-        const long long kvb = p.seg_base ? p.seg_base[seg] : (long long)off;
+        const int kvb = (int)(p.seg_base ? p.seg_base[seg] : (long long)off);
+        const int nkv = qt + 1;
         if (item_iter > 0) ok = mbar_wait(&bars->q_empty, (item_iter - 1) & 1, abort_flag, p.status);
         if (!ok) break;
         mbar_arrive_expect_tx(&bars->q_full, L::kTileBytes);
         for (int a = 0; a < L::kAtoms; ++a)
           tma_load_2d(smem + L::kQ + a * L::kAtomBytes, &tm_q, j * D + a * 64, off + qt * BM, &bars->q_full);
-        for (int kv = 0; kv <= qt && ok; ++kv, ++kv_iter) {
-          const int st = kv_iter & 1;
-          const uint32_t use = kv_iter >> 1;
-          if (use > 0) ok = mbar_wait(&bars->k_empty[st], (use - 1) & 1, abort_flag, p.status);
-          if (!ok) break;
-          mbar_arrive_expect_tx(&bars->k_full[st], L::kTileBytes);
-          for (int a = 0; a < L::kAtoms; ++a)
-            tma_load_2d(smem + L::kK0 + st * L::kTileBytes + a * L::kAtomBytes, &tm_k, a * 64,
-                        (int)(kvb + (long long)kv * BN), &bars->k_full[st]);
-          if (use > 0) ok = mbar_wait(&bars->v_empty[st], (use - 1) & 1, abort_flag, p.status);
-          if (!ok) break;
-          mbar_arrive_expect_tx(&bars->v_full[st], L::kTileBytes);
-          for (int a = 0; a < L::kAtoms; ++a)
-            tma_load_2d(smem + L::kV0 + st * L::kTileBytes + a * L::kAtomBytes, &tm_v, a * 64,
-                        (int)(kvb + (long long)kv * BN), &bars->v_full[st]);
+        // K(0), K(1), then V(kv), K(kv + 2) for kv = 0, 1, ...
+        ok = load_tile(&tm_k, kvb);
+        if (ok && nkv > 1) ok = load_tile(&tm_k, kvb + BN);
+        for (int kv = 0; kv < nkv && ok; ++kv) {
+          ok = load_tile(&tm_v, kvb + kv * BN);
+          if (ok && kv + 2 < nkv) ok = load_tile(&tm_k, kvb + (kv + 2) * BN);
         }
         ++item_iter;
       }
@@ -203,14 +217,39 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-  } else if (warp == 1) {
+  } else if (warp == kWarpMma) {
     // ------------------------------------------------------------------ MMA issuer
+    // tcgen05.mma instructions into one accumulator run back to back; instructions into
+    // different accumulators overlap.  With three S/P buffers, PV(kv) (A = P from TMEM)
+    // and S(kv+2) (into the buffer PV(kv-1) finished with) are independent, and are
+    // issued interleaved instruction by instruction while the softmax works on S(kv+1).
     constexpr uint32_t idesc_qk = make_idesc_bf16(BM, BN, false, false);
     constexpr uint32_t idesc_pv = make_idesc_bf16(BM, D, false, true);
     const uint32_t q_addr = smem_u32(smem + L::kQ);
-    const uint32_t p_addr = smem_u32(smem + L::kP);
-    uint32_t kv_iter = 0, s_iter = 0, pv_iter = 0, item_iter = 0;
+    uint32_t ring_iter = 0, item_iter = 0, s_iter = 0, p_iter = 0;
     bool ok = true;
+    auto slot_addr = [&](uint32_t r) { return smem_u32(smem + L::kRing0 + (r % kRing) * L::kTileBytes); };
+    auto wait_ring = [&](uint32_t r) {
+      return warp_wait(&bars->ring_full[r % kRing], (r / kRing) & 1, abort_flag, p.status);
+    };
+    // S into buffer s_iter % 3 from ring entry r_k (alone, not interleaved)
+    auto issue_s_alone = [&](uint32_t r_k) {
+      const uint32_t k_addr = slot_addr(r_k);
+      const uint32_t d = tmem + tmem_s_col(s_iter % kSBufs);
+      if (lane == 0) {
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * L::kAtomBytes + (kk & 3) * 32;
+          mma_bf16_ss(d, make_smem_desc_sw128(q_addr + off, 16, 1024), make_smem_desc_sw128(k_addr + off, 16, 1024),
+                      idesc_qk, kk > 0 ? 1u : 0u);
+        }
+        mma_commit(&bars->s_full[s_iter % kSBufs]);
+        mma_commit(&bars->ring_empty[r_k % kRing]);
+      }
+      __syncwarp();
+      ++s_iter;
+    };
+
     while (ok) {
       int2 item;
       ok = take_item(bars, item_iter, &item, abort_flag, p.status);
@@ -218,72 +257,82 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int seg = item.x / p.g, qt = item.y;
       const int n = p.seg_offsets[seg + 1] - p.seg_offsets[seg];
       const int nkv = qt + 1;
+      // ring entries of this item, in load order: K(0), K(1) if nkv > 1, then for each kv:
+      // V(kv) followed by K(kv+2) while kv + 2 < nkv
+      const uint32_t rk0 = ring_iter, rk1 = ring_iter + 1;
+      const int m = nkv > 2 ? nkv - 2 : 0;  // key tiles followed by a K load
+      const uint32_t base = ring_iter + (nkv > 1 ? 2u : 1u);
+      auto rv = [&](int kv) -> uint32_t { return kv < m ? base + 2u * kv : base + 2u * m + (kv - m); };
+      auto rk = [&](int kv) -> uint32_t { return base + 2u * (kv - 2) + 1u; };  // K(kv), kv >= 2
+
       ok = warp_wait(&bars->q_full, item_iter & 1, abort_flag, p.status);
-      for (int jj = 0; jj <= nkv && ok; ++jj) {
-        if (jj < nkv) {
-          // S_jj = Q K_jj^T
-          const uint32_t kvi = kv_iter + jj;
-          const int st = kvi & 1;
-          ok = warp_wait(&bars->k_full[st], (kvi >> 1) & 1, abort_flag, p.status);
-          const int sb = s_iter & 1;
-          if (ok && s_iter >= 2) ok = warp_wait(&bars->s_free[sb], ((s_iter >> 1) - 1) & 1, abort_flag, p.status);
-          if (!ok) break;
-          tc_fence_after();
-          if (lane == 0) {
-            const uint32_t k_addr = smem_u32(smem + L::kK0 + st * L::kTileBytes);
-            const uint32_t d_tmem = tmem + (sb ? kTmemS1 : kTmemS0);
+      if (ok) ok = wait_ring(rk0);
+      if (!ok) break;
+      tc_fence_after();
+      issue_s_alone(rk0);
+      if (nkv > 1) {
+        ok = wait_ring(rk1);
+        if (!ok) break;
+        tc_fence_after();
+        issue_s_alone(rk1);
+      }
+      if (lane == 0 && nkv <= 2) mma_commit(&bars->q_empty);  // every S of this item issued
+      __syncwarp();
+
+      for (int kv = 0; kv < nkv && ok; ++kv) {
+        // PV(kv) needs P(kv); S(kv+2) needs K(kv+2) and the buffer PV(kv-1) read from
+        ok = warp_wait(&bars->p_full, p_iter & 1, abort_flag, p.status);
+        ++p_iter;
+        const uint32_t r_v = rv(kv);
+        if (ok) ok = wait_ring(r_v);
+        if (ok && kv == 0 && item_iter > 0) ok = warp_wait(&bars->o_free, (item_iter - 1) & 1, abort_flag, p.status);
+        const bool with_s = kv + 2 < nkv;
+        const uint32_t r_k2 = with_s ? rk(kv + 2) : 0;
+        if (ok && with_s) ok = wait_ring(r_k2);
+        if (!ok) break;
+        const int valid_keys = n - kv * BN;  // keys of this tile inside the segment
+        if (valid_keys < BN) {
+          // rows past the segment end may hold anything (other segments, unwritten cache
+          // rows): zero them so that 0-weight columns of P cannot meet NaN in V
+          uint8_t* vtile = smem + L::kRing0 + (r_v % kRing) * L::kTileBytes;
+          for (int a = 0; a < L::kAtoms; ++a) {
+            uint4* base = reinterpret_cast<uint4*>(vtile + a * L::kAtomBytes);
+            for (int i = valid_keys * 8 + lane; i < BN * 8; i += 32) base[i] = make_uint4(0, 0, 0, 0);
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+        }
+        tc_fence_after();
+        if (lane == 0) {
+          // P(kv) sits in the buffer of S(kv): S and P are counted alike across items
+          const uint32_t pbuf = tmem + tmem_s_col((int)((p_iter - 1) % kSBufs));
+          const uint32_t sbuf = tmem + tmem_s_col((int)(s_iter % kSBufs));
+          const uint32_t v_addr = slot_addr(r_v);
+          const uint32_t k_addr = with_s ? slot_addr(r_k2) : 0;
 #pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
+          for (int kk = 0; kk < 8; ++kk) {
+            // PV: K extent = BN keys, 16 per instruction (8 instructions)
+            mma_bf16_ts(tmem + kTmemO, pbuf + kk * 8, make_smem_desc_sw128(v_addr + kk * 2048, L::kAtomBytes, 1024),
+                        idesc_pv, (kv > 0 || kk > 0) ? 1u : 0u);
+            // S: K extent = D, 16 per instruction (D / 16 instructions)
+            if (with_s && kk < D / 16) {
               const uint32_t off = (kk >> 2) * L::kAtomBytes + (kk & 3) * 32;
-              mma_bf16_ss(d_tmem, make_smem_desc_sw128(q_addr + off, 16, 1024),
+              mma_bf16_ss(sbuf, make_smem_desc_sw128(q_addr + off, 16, 1024),
                           make_smem_desc_sw128(k_addr + off, 16, 1024), idesc_qk, kk > 0 ? 1u : 0u);
             }
-            mma_commit(&bars->s_full[sb]);
-            mma_commit(&bars->k_empty[st]);
-            if (jj == nkv - 1) mma_commit(&bars->q_empty);
           }
-          __syncwarp();
-          ++s_iter;
+          mma_commit(&bars->o_ready);
+          mma_commit(&bars->ring_empty[r_v % kRing]);
+          if (with_s) {
+            mma_commit(&bars->s_full[s_iter % kSBufs]);
+            mma_commit(&bars->ring_empty[r_k2 % kRing]);
+            if (kv + 2 == nkv - 1) mma_commit(&bars->q_empty);
+          }
         }
-        if (jj >= 1) {
-          // O += P_{jj-1} V_{jj-1}
-          const int pj = jj - 1;
-          const uint32_t kvi = kv_iter + pj;
-          const int st = kvi & 1;
-          ok = warp_wait(&bars->p_full, pv_iter & 1, abort_flag, p.status);
-          if (ok) ok = warp_wait(&bars->v_full[st], (kvi >> 1) & 1, abort_flag, p.status);
-          if (ok && pj == 0 && item_iter > 0) ok = warp_wait(&bars->o_free, (item_iter - 1) & 1, abort_flag, p.status);
-          if (!ok) break;
-          uint8_t* vtile = smem + L::kV0 + st * L::kTileBytes;
-          const int valid_keys = n - pj * BN;  // keys of this tile inside the segment
-          if (valid_keys < BN) {
-            // rows past the segment end may hold anything (other segments, unwritten cache
-            // rows): zero them so that 0-weight columns of P cannot meet NaN in V
-            for (int a = 0; a < L::kAtoms; ++a) {
-              uint4* base = reinterpret_cast<uint4*>(vtile + a * L::kAtomBytes);
-              for (int i = valid_keys * 8 + lane; i < BN * 8; i += 32) base[i] = make_uint4(0, 0, 0, 0);
-            }
-            fence_proxy_async_smem();
-          }
-          __syncwarp();
-          tc_fence_after();
-          if (lane == 0) {
-            const uint32_t v_addr = smem_u32(vtile);
-#pragma unroll
-            for (int kk = 0; kk < BN / 16; ++kk) {
-              const uint32_t a_off = (kk >> 2) * L::kAtomBytes + (kk & 3) * 32;
-              mma_bf16_ss(tmem + kTmemO, make_smem_desc_sw128(p_addr + a_off, 16, 1024),
-                          make_smem_desc_sw128(v_addr + kk * 2048, L::kAtomBytes, 1024), idesc_pv,
-                          (pj > 0 || kk > 0) ? 1u : 0u);
-            }
-            mma_commit(&bars->o_ready);
-            mma_commit(&bars->v_empty[st]);
-          }
-          __syncwarp();
-          ++pv_iter;
-        }
+        __syncwarp();
+        if (with_s) ++s_iter;
       }
-      kv_iter += nkv;
+      ring_iter += 2 * nkv;
       ++item_iter;
     }
     if (!ok && lane == 0) {
@@ -296,55 +345,62 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else {
     // ------------------------------------------------------------------ softmax / epilogue
-    const int quad = warp & 3;              // TMEM lane quadrant of this warp
-    const int row = quad * 32 + lane;       // query row within the tile
-    const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
-    uint8_t* p_tile = smem + L::kP;
+    const int row = warp * 32 + lane;  // query row within the tile (warp w reads TMEM lanes 32w..32w+31)
+    const uint32_t lane_addr = (uint32_t)(warp * 32) << 16;
+    const uint32_t o_addr = tmem + lane_addr + kTmemO;
     uint32_t s_iter = 0, o_iter = 0, item_iter = 0;
     bool ok = true;
     while (ok) {
       int2 item;
       ok = take_item(bars, item_iter, &item, abort_flag, p.status);
-      if (!ok || item.x < 0) break;
       ++item_iter;
+      if (!ok || item.x < 0) break;
       const int seg = item.x / p.g, j = item.x % p.g, qt = item.y;
       const int off = p.seg_offsets[seg];
       const int n = p.seg_offsets[seg + 1] - off;
-      const int nkv = qt + 1;
+      // epilogue operands now, so that their latency hides behind the item
       const int qrank = qt * BM + row;
+      const bool valid = qrank < n;
+      long long dst_row = 0;
+      float gt = 0.f;
+      if (valid) {
+        const int src = p.row_src[off + qrank];
+        dst_row = (long long)src * p.g + j;
+        gt = p.gate[src];
+      }
       float m_use = 0.f, l_sum = 0.f;
-      for (int jj = 0; jj < nkv && ok; ++jj) {
-        const int sb = s_iter & 1;
-        ok = warp_wait(&bars->s_full[sb], (s_iter >> 1) & 1, abort_flag, p.status);
+      for (int kv = 0; kv <= qt && ok; ++kv) {
+        const uint32_t s_addr = tmem + lane_addr + tmem_s_col((int)(s_iter % kSBufs));
+        ok = warp_wait(&bars->s_full[s_iter % kSBufs], (s_iter / kSBufs) & 1, abort_flag, p.status);
+        ++s_iter;
         if (!ok) break;
         tc_fence_after();
-        float s[BN];
+        float sv[BN];
 #pragma unroll
         for (int c = 0; c < BN / 32; ++c) {
           uint32_t r[32];
-          tmem_ld32(tmem + lane_addr + (sb ? kTmemS1 : kTmemS0) + c * 32, r);
+          tmem_ld32(s_addr + c * 32, r);
 #pragma unroll
-          for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(r[i]);
+          for (int i = 0; i < 32; ++i) sv[c * 32 + i] = __uint_as_float(r[i]);
         }
         tmem_wait_ld();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&bars->s_free[sb]);
-        ++s_iter;
-
-        // causal mask inside the diagonal tile: key rank jj*BN + c <= query rank
-        if (jj == qt) {
+        // causal mask on the diagonal tile: key rank kv*BN + c <= query rank
+        if (kv == qt) {
 #pragma unroll
           for (int c = 0; c < BN; ++c)
-            if (c > row) s[c] = -INFINITY;
+            if (c > row) sv[c] = -INFINITY;
         }
-        float mx = s[0];
+        float m8[8];
 #pragma unroll
-        for (int c = 1; c < BN; ++c) mx = fmaxf(mx, s[c]);
+        for (int i = 0; i < 8; ++i) m8[i] = sv[i];
+#pragma unroll
+        for (int c = 8; c < BN; ++c) m8[c & 7] = fmaxf(m8[c & 7], sv[c]);
+        const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
+                               fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
         const float m_tile = mx * p.scale_log2;
         float alpha = 1.f;
         bool rescale = false;
-        if (jj == 0) {
+        if (kv == 0) {
           m_use = m_tile;
         } else if (m_tile > m_use + kRescaleThreshold) {
           alpha = fast_exp2(m_use - m_tile);
@@ -352,18 +408,27 @@ __global__ void __launch_bounds__(kThreads, 1)
           rescale = true;
         }
         uint32_t pk[BN / 2];
-        float rowsum = 0.f;
+        float sum4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int c = 0; c < BN; c += 2) {
-          const float e0 = fast_exp2(fmaf(s[c], p.scale_log2, -m_use));
-          const float e1 = fast_exp2(fmaf(s[c + 1], p.scale_log2, -m_use));
-          rowsum += e0 + e1;
+          const float e0 = fast_exp2(fmaf(sv[c], p.scale_log2, -m_use));
+          const float e1 = fast_exp2(fmaf(sv[c + 1], p.scale_log2, -m_use));
+          sum4[(c >> 1) & 3] += e0 + e1;
           pk[c / 2] = pack_bf16x2(e0, e1);
         }
-        l_sum = l_sum * alpha + rowsum;
-
-        // P buffer and O are free once PV of the previous tile completed
-        if (jj > 0) {
+        l_sum = l_sum * alpha + ((sum4[0] + sum4[1]) + (sum4[2] + sum4[3]));
+        // P over the S columns just read (every S value is in registers)
+        {
+          uint32_t r[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) r[i] = pk[i];
+          tmem_st32(s_addr, r);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) r[i] = pk[32 + i];
+          tmem_st32(s_addr + 32, r);
+        }
+        // O may only be rescaled once the previous PV completed
+        if (kv > 0) {
           ok = warp_wait(&bars->o_ready, o_iter & 1, abort_flag, p.status);
           ++o_iter;
           if (!ok) break;
@@ -372,23 +437,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
               uint32_t r[32];
-              tmem_ld32(tmem + lane_addr + kTmemO + c * 32, r);
+              tmem_ld32(o_addr + c * 32, r);
               tmem_wait_ld();
 #pragma unroll
               for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-              tmem_st32(tmem + lane_addr + kTmemO + c * 32, r);
+              tmem_st32(o_addr + c * 32, r);
             }
-            tmem_wait_st();
           }
         }
-        // P row -> shared memory, K-major 128B-swizzled (16-byte chunk index ^= row % 8)
-#pragma unroll
-        for (int ch = 0; ch < BN / 8; ++ch) {
-          const int atom = ch >> 3, cc = ch & 7;
-          uint4* dst = reinterpret_cast<uint4*>(p_tile + atom * L::kAtomBytes + row * 128 + ((cc ^ (row & 7)) << 4));
-          *dst = make_uint4(pk[ch * 4 + 0], pk[ch * 4 + 1], pk[ch * 4 + 2], pk[ch * 4 + 3]);
-        }
-        fence_proxy_async_smem();
+        tmem_wait_st();
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars->p_full);
@@ -399,19 +456,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       ++o_iter;
       if (!ok) break;
       tc_fence_after();
-      const bool valid = qrank < n;
-      const long long prow = (long long)off + qrank;
-      long long dst_row = 0;
-      float scale = 0.f;
-      if (valid) {
-        const int src = p.row_src[prow];
-        dst_row = (long long)src * p.g + j;
-        scale = p.gate[src] / l_sum;
-      }
+      const float scale = valid ? gt / l_sum : 0.f;
 #pragma unroll
       for (int c = 0; c < D / 32; ++c) {
         uint32_t r[32];
-        tmem_ld32(tmem + lane_addr + kTmemO + c * 32, r);
+        tmem_ld32(o_addr + c * 32, r);
         tmem_wait_ld();
         if (valid) {
           uint4* dst = reinterpret_cast<uint4*>(p.y + dst_row * D + c * 32);
@@ -435,7 +484,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+  if (warp == kWarpMma) tmem_dealloc(tmem, kTmemCols);
   if (threadIdx.x == 0) {
     // every fetch of this CTA happened before the barrier above; the last CTA resets
     __threadfence();
@@ -447,24 +496,28 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// One block.  Items ordered by decreasing cost (qt descending), then (segment, j).
+// One block.  Items are the 128-row query tiles q of every segment and group head j,
+// ordered by decreasing cost (q descending: tile q needs q + 1 key tiles), then (segment, j).
 // Segments longer than their cache capacity are skipped (the RoPE stage reports them).
-// Also zeroes the dynamic scheduler's counters.
+// Also zeroes the dynamic scheduler's counters.  seg_offsets (and seg_cap) are staged in
+// shared memory first so that no loop below waits on global memory.
 __global__ void __launch_bounds__(1024) plan_kernel(const int32_t* __restrict__ seg_offsets, int nseg,
                                                     const int32_t* __restrict__ seg_cap, int g, int max_qtiles,
                                                     int* __restrict__ header, int2* __restrict__ items) {
   extern __shared__ int s_dyn[];
-  int* s_count = s_dyn;               // [max_qtiles]: segments with more than q tiles
-  int* s_start = s_dyn + max_qtiles;  // [max_qtiles]: first item of cost q + 1
+  int* s_count = s_dyn;                   // [max_qtiles]: segments with more than q query tiles
+  int* s_start = s_dyn + max_qtiles;      // [max_qtiles]: first item of cost q + 1
+  int* s_ntile = s_dyn + 2 * max_qtiles;  // [nseg]: query tiles of each segment (0 if skipped)
   const int tid = threadIdx.x;
   for (int q = tid; q < max_qtiles; q += blockDim.x) s_count[q] = 0;
-  __syncthreads();
   for (int s = tid; s < nseg; s += blockDim.x) {
-    const int n = seg_offsets[s + 1] - seg_offsets[s];
-    if (seg_cap && n > seg_cap[s]) continue;
-    const int nt = min((n + BM - 1) / BM, max_qtiles);
-    if (nt > 0) atomicAdd(&s_count[nt - 1], 1);  // histogram of tile counts
+    const int n = __ldg(seg_offsets + s + 1) - __ldg(seg_offsets + s);
+    const bool skip = seg_cap && n > __ldg(seg_cap + s);
+    s_ntile[s] = skip ? 0 : min((n + kItemRows - 1) / kItemRows, max_qtiles);
   }
+  __syncthreads();
+  for (int s = tid; s < nseg; s += blockDim.x)
+    if (s_ntile[s] > 0) atomicAdd(&s_count[s_ntile[s] - 1], 1);  // histogram of tile counts
   __syncthreads();
   if (tid == 0) {
     int above = 0, run = 0;  // above: segments with more than q tiles
@@ -482,12 +535,9 @@ __global__ void __launch_bounds__(1024) plan_kernel(const int32_t* __restrict__ 
   for (int q = tid; q < max_qtiles; q += blockDim.x) {
     if (s_count[q] == 0) continue;
     int pos = s_start[q];
-    for (int s = 0; s < nseg; ++s) {
-      const int n = seg_offsets[s + 1] - seg_offsets[s];
-      if (seg_cap && n > seg_cap[s]) continue;
-      if (n > q * BM)
+    for (int s = 0; s < nseg; ++s)
+      if (s_ntile[s] > q)
         for (int j = 0; j < g; ++j) items[pos++] = make_int2(s * g + j, q);
-    }
   }
 }
 
@@ -523,6 +573,7 @@ __global__ void seg_len_kernel(const int32_t* __restrict__ seg_offsets, int nseg
 }
 
 constexpr int kMaxPrefillT = 1 << 20;  // the plan keeps 2 ints per query tile in shared memory
+constexpr int kMaxPrefillSegments = 1 << 15;  // and one int per segment
 
 bool supported_dims(int d_head, int g) {
   return (d_head == 64 || d_head == 128) && (g == 1 || g == 2 || g == 4 || g == 8);
@@ -537,27 +588,30 @@ int check_shape(int B, int T, int H, int K, int d_head, int group, int* Hr, int*
   *Hr = H / group;
   *Kr = K / group;
   *R = (long long)B * T * *Kr;
-  if (*R * group >= (1ll << 31) || (long long)B * *Hr >= (1ll << 24)) return NAMOH_ERR_INVALID_ARG;
+  if (*R * group >= (1ll << 31)) return NAMOH_ERR_INVALID_ARG;
+  if ((long long)B * *Hr > kMaxPrefillSegments) return NAMOH_ERR_UNSUPPORTED;
   return NAMOH_OK;
 }
 
 size_t plan_bytes_for(int B, int T, int Hr, int Kr, int g) {
   const long long R = (long long)B * T * Kr;
-  const long long max_items = ((R + attn::BM - 1) / attn::BM + (long long)B * Hr) * g;
+  const long long max_items = ((R + attn::kItemRows - 1) / attn::kItemRows + (long long)B * Hr) * g;
   return 16 + (size_t)max_items * sizeof(int2);
 }
 
 int launch_plan(const int32_t* seg_offsets, int nseg, int T, int g, const int32_t* seg_cap, void* plan,
                 cudaStream_t stream) {
-  const int max_qtiles = (T + attn::BM - 1) / attn::BM;
-  const int smem = 2 * max_qtiles * (int)sizeof(int);
-  if (smem > 48 * 1024 &&
-      cudaFuncSetAttribute(attn::plan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
-    return NAMOH_ERR_CUDA;
+  const int max_qtiles = (T + attn::kItemRows - 1) / attn::kItemRows;  // query tiles per segment, at most
+  const int smem = (2 * max_qtiles + nseg) * (int)sizeof(int);
+  if (smem > 200 * 1024) return NAMOH_ERR_UNSUPPORTED;
+  if (smem > 48 * 1024) {
+    const cudaError_t e = cudaFuncSetAttribute(attn::plan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return cuda_fail(e, "plan_kernel shared memory attribute");
+  }
   int* header = static_cast<int*>(plan);
   int2* items = reinterpret_cast<int2*>(static_cast<char*>(plan) + 16);
   attn::plan_kernel<<<1, 1024, smem, stream>>>(seg_offsets, nseg, seg_cap, g, max_qtiles, header, items);
-  return cudaGetLastError() == cudaSuccess ? NAMOH_OK : NAMOH_ERR_CUDA;
+  return cuda_check_launch("plan_kernel launch");
 }
 
 int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint16_t* v_cache, int B, int T, int Hr,
@@ -568,7 +622,7 @@ int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint1
   CUtensorMap tq, tk, tv;
   if (!attn::encode_rows_map(&tq, q_rot, R, g * D) || !attn::encode_rows_map(&tk, k_cache, cache_rows, D) ||
       !attn::encode_rows_map(&tv, v_cache, cache_rows, D))
-    return NAMOH_ERR_CUDA;
+    return cuda_fail(cudaErrorInvalidValue, "cuTensorMapEncodeTiled");
   attn::Params p;
   p.seg_offsets = seg_offsets;
   p.seg_base = seg_base;
@@ -583,10 +637,10 @@ int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint1
   p.status = dev_status;
   const cudaError_t e = (D == 128) ? attn::launch_attn<128>(tq, tk, tv, p, info.sm_count, stream)
                                    : attn::launch_attn<64>(tq, tk, tv, p, info.sm_count, stream);
-  return e == cudaSuccess ? NAMOH_OK : NAMOH_ERR_CUDA;
+  return e == cudaSuccess ? NAMOH_OK : cuda_fail(e, "attn_fwd_kernel launch");
 }
 
-bool device_ok(DeviceInfo* info) {
+bool device_ok(DeviceInfo* info) {  // a Blackwell datacenter part with the shared memory the kernel needs
   return current_device_info(info) && info->major == 10 &&
          (size_t)attn::Smem<128>::kAlloc <= info->max_smem_optin;
 }
@@ -616,13 +670,13 @@ extern "C" int namoh_rope_pack(const uint16_t* q, const uint16_t* k, const uint1
     cache_rows = R;
   }
   DeviceInfo info;
-  if (!current_device_info(&info)) return NAMOH_ERR_CUDA;
+  if (!current_device_info(&info)) return cuda_fail(cudaGetLastError(), "device query");
   RopeTable tab;
   fill_rope_table(&tab, d_head, (double)rope_base);
   const cudaError_t e = launch_rope_pack(d_head, q, k, v, (int)R, group, seg_offsets, B * Hr, seg_base, seg_cap,
                                          cache_rows, q_rot, k_cache, v_cache, v_cache != v, tab, dev_status,
                                          info.sm_count, reinterpret_cast<cudaStream_t>(stream_v));
-  return e == cudaSuccess ? NAMOH_OK : NAMOH_ERR_CUDA;
+  return e == cudaSuccess ? NAMOH_OK : cuda_fail(e, "rope_pack_kernel launch");
 }
 
 extern "C" size_t namoh_attention_plan_size(int B, int T, int H, int K, int group) {
@@ -711,14 +765,15 @@ extern "C" int namoh_prefill(const uint16_t* q, const uint16_t* k, const uint16_
 
   RopeTable tab;
   fill_rope_table(&tab, d_head, (double)rope_base);
-  if (launch_rope_pack(d_head, q, k, v, (int)R, group, seg_offsets, B * Hr, seg_base, seg_cap, cache_rows, q_rot,
-                       k_cache, v_cache, v_cache != v, tab, dev_status, info.sm_count, stream) != cudaSuccess)
-    return NAMOH_ERR_CUDA;
+  const cudaError_t er = launch_rope_pack(d_head, q, k, v, (int)R, group, seg_offsets, B * Hr, seg_base, seg_cap,
+                                          cache_rows, q_rot, k_cache, v_cache, v_cache != v, tab, dev_status,
+                                          info.sm_count, stream);
+  if (er != cudaSuccess) return cuda_fail(er, "rope_pack_kernel launch");
   st = launch_plan(seg_offsets, B * Hr, T, group, seg_base ? seg_cap : nullptr, plan, stream);
   if (st != NAMOH_OK) return st;
   if (seg_len) {
     seg_len_kernel<<<(B * Hr + 255) / 256, 256, 0, stream>>>(seg_offsets, B * Hr, seg_len);
-    if (cudaGetLastError() != cudaSuccess) return NAMOH_ERR_CUDA;
+    if (const int st2 = cuda_check_launch("seg_len_kernel launch")) return st2;
   }
   return launch_attention(q_rot, k_cache, v_cache, B, T, Hr, Kr, d_head, group, seg_offsets, row_src, gate, seg_base,
                           cache_rows, plan, y, dev_status, info, stream);

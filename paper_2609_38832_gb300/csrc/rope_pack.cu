@@ -10,6 +10,8 @@
 
 namespace namoh {
 
+constexpr int kRopeStageMax = 8192;  // seg_offsets entries staged in shared memory (32 KB)
+
 template <int D>
 __global__ void __launch_bounds__(256) rope_pack_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ k,
                                                         const uint16_t* __restrict__ v, int R, int g,
@@ -21,6 +23,14 @@ __global__ void __launch_bounds__(256) rope_pack_kernel(const uint16_t* __restri
                                                         uint32_t* __restrict__ status) {
   constexpr int LPR = D / 16;  // threads per row
   constexpr int HALF = D / 2;
+  constexpr int GMAX = 8;      // largest group size
+  extern __shared__ int32_t s_off[];  // seg_offsets staged when they fit (nseg + 1 <= kStageMax)
+  const bool staged = (nseg + 1) <= kRopeStageMax;
+  if (staged) {
+    for (int i = threadIdx.x; i <= nseg; i += blockDim.x) s_off[i] = __ldg(seg_offsets + i);
+    __syncthreads();
+  }
+  const int32_t* offs = staged ? s_off : seg_offsets;
   const int lane_in_row = threadIdx.x % LPR;
   const int j0 = lane_in_row * 8;
   const long long groups = (long long)gridDim.x * (blockDim.x / LPR);
@@ -31,13 +41,29 @@ __global__ void __launch_bounds__(256) rope_pack_kernel(const uint16_t* __restri
     th_lo[i] = tab.theta_lo[j0 + i];
   }
   for (long long r = (long long)blockIdx.x * (blockDim.x / LPR) + threadIdx.x / LPR; r < R; r += groups) {
+    // every load of this row first, so their latencies overlap
+    uint4 ka = __ldg(reinterpret_cast<const uint4*>(k + (size_t)r * D + j0));
+    uint4 kb = __ldg(reinterpret_cast<const uint4*>(k + (size_t)r * D + HALF + j0));
+    uint4 qa[GMAX], qb[GMAX];
+#pragma unroll
+    for (int j = 0; j < GMAX; ++j) {
+      if (j < g) {
+        qa[j] = __ldg(reinterpret_cast<const uint4*>(q + ((size_t)r * g + j) * D + j0));
+        qb[j] = __ldg(reinterpret_cast<const uint4*>(q + ((size_t)r * g + j) * D + HALF + j0));
+      }
+    }
+    uint4 va = make_uint4(0, 0, 0, 0), vb = va;
+    if (copy_v) {
+      va = __ldg(reinterpret_cast<const uint4*>(v + (size_t)r * D) + lane_in_row);
+      vb = __ldg(reinterpret_cast<const uint4*>(v + (size_t)r * D) + lane_in_row + LPR);
+    }
     // segment of row r: last s with seg_offsets[s] <= r
     int lo = 0, hi = nseg;
     while (hi - lo > 1) {
       const int mid = (lo + hi) >> 1;
-      if (__ldg(seg_offsets + mid) <= r) lo = mid; else hi = mid;
+      if (offs[mid] <= r) lo = mid; else hi = mid;
     }
-    const int rho = (int)(r - __ldg(seg_offsets + lo));
+    const int rho = (int)(r - offs[lo]);
     long long dst = r;
     bool write_cache = true;
     if (seg_base) {
@@ -51,9 +77,8 @@ __global__ void __launch_bounds__(256) rope_pack_kernel(const uint16_t* __restri
 #pragma unroll
     for (int i = 0; i < 8; ++i) rope_sincos((float)rho, th_hi[i], th_lo[i], tab, &sn[i], &cs[i]);
 
-    auto rotate = [&](const uint16_t* src, uint16_t* dst_row) {
-      const uint4 a = __ldg(reinterpret_cast<const uint4*>(src + j0));
-      const uint4 b = __ldg(reinterpret_cast<const uint4*>(src + HALF + j0));
+    // x'_j = x_j cos - x_{j+D/2} sin ;  x'_{j+D/2} = x_{j+D/2} cos + x_j sin
+    auto rotate = [&](const uint4& a, const uint4& b, uint16_t* dst_row) {
       const uint32_t av[4] = {a.x, a.y, a.z, a.w};
       const uint32_t bv[4] = {b.x, b.y, b.z, b.w};
       uint32_t oa[4], ob[4];
@@ -62,22 +87,21 @@ __global__ void __launch_bounds__(256) rope_pack_kernel(const uint16_t* __restri
         const float x0 = bf16_lo(av[p]), x1 = bf16_hi(av[p]);
         const float y0 = bf16_lo(bv[p]), y1 = bf16_hi(bv[p]);
         const int i0 = 2 * p, i1 = 2 * p + 1;
-        // x'_j = x_j cos - x_{j+D/2} sin ;  x'_{j+D/2} = x_{j+D/2} cos + x_j sin
         oa[p] = pack_bf16x2(fmaf(x0, cs[i0], -y0 * sn[i0]), fmaf(x1, cs[i1], -y1 * sn[i1]));
         ob[p] = pack_bf16x2(fmaf(y0, cs[i0], x0 * sn[i0]), fmaf(y1, cs[i1], x1 * sn[i1]));
       }
       *reinterpret_cast<uint4*>(dst_row + j0) = make_uint4(oa[0], oa[1], oa[2], oa[3]);
       *reinterpret_cast<uint4*>(dst_row + HALF + j0) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
     };
-
-    for (int j = 0; j < g; ++j) rotate(q + ((size_t)r * g + j) * D, q_rot + ((size_t)r * g + j) * D);
+#pragma unroll
+    for (int j = 0; j < GMAX; ++j)
+      if (j < g) rotate(qa[j], qb[j], q_rot + ((size_t)r * g + j) * D);
     if (write_cache) {
-      rotate(k + (size_t)r * D, k_cache + (size_t)dst * D);
+      rotate(ka, kb, k_cache + (size_t)dst * D);
       if (copy_v) {
-        const uint4* vs = reinterpret_cast<const uint4*>(v + (size_t)r * D);
         uint4* vd = reinterpret_cast<uint4*>(v_cache + (size_t)dst * D);
-        vd[lane_in_row] = __ldg(vs + lane_in_row);
-        vd[lane_in_row + LPR] = __ldg(vs + lane_in_row + LPR);
+        vd[lane_in_row] = va;
+        vd[lane_in_row + LPR] = vb;
       }
     }
   }
@@ -93,11 +117,12 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
   long long blocks = ((long long)R + rows_per_block - 1) / rows_per_block;
   const long long cap = (long long)sm_count * 8;
   if (blocks > cap) blocks = cap;
+  const size_t smem = (nseg + 1 <= kRopeStageMax) ? (size_t)(nseg + 1) * sizeof(int32_t) : 0;
   if (D == 128)
-    rope_pack_kernel<128><<<(int)blocks, threads, 0, stream>>>(q, k, v, R, g, seg_offsets, nseg, seg_base, seg_cap,
+    rope_pack_kernel<128><<<(int)blocks, threads, smem, stream>>>(q, k, v, R, g, seg_offsets, nseg, seg_base, seg_cap,
                                                                cache_rows, q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status);
   else
-    rope_pack_kernel<64><<<(int)blocks, threads, 0, stream>>>(q, k, v, R, g, seg_offsets, nseg, seg_base, seg_cap,
+    rope_pack_kernel<64><<<(int)blocks, threads, smem, stream>>>(q, k, v, R, g, seg_offsets, nseg, seg_base, seg_cap,
                                                               cache_rows, q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status);
   return cudaGetLastError();
 }

@@ -1,13 +1,13 @@
 // route.cu -- routing and dispatch (Sec. 3.1 Eq. namoh-gates; Sec. 3.2 Eq. namoh-head-rope).
 //
-// Four launches, all stream-ordered, no host synchronisation:
+// Three launches, all stream-ordered, no host synchronisation:
 //   1. route_topk_kernel   one thread per token: TopK of the fp32 logits (descending,
 //                          ties to the lower head index), fp32 softmax gates over all H,
 //                          and per-chunk head counts (one block = one 256-token chunk).
-//   2. route_scan_chunks   per sequence: exclusive scan of the chunk counts over chunks
-//                          for every head -> chunk base ranks; totals n[b, h].
-//   3. route_scan_segments exclusive scan of n over (b, h) -> seg_offsets.
-//   4. route_rank_kernel   per chunk: warp ballots give each (token, slot) its rank among
+//   2. route_scan_kernel   one block per sequence: exclusive scan of the chunk counts over
+//                          chunks for every head -> chunk base ranks and totals n[b, h];
+//                          the last block to finish scans n over (b, h) -> seg_offsets.
+//   3. route_rank_kernel   per chunk: warp ballots give each (token, slot) its rank among
 //                          the chunk's earlier tokens for that head; adds the chunk base
 //                          -> rank, row and row_src.
 // All integer work is exact, so the packed layout is deterministic and bit-identical to
@@ -26,54 +26,64 @@ __global__ void __launch_bounds__(kChunk) route_topk_kernel(const float* __restr
                                                             int nchunks, int32_t* __restrict__ topk_head,
                                                             float* __restrict__ gate,
                                                             int32_t* __restrict__ chunk_count,
+                                                            int* __restrict__ scan_ticket,
                                                             uint32_t* __restrict__ status) {
-  extern __shared__ float s_scores[];  // [kChunk][H + 1]
   __shared__ int s_cnt[NAMOH_MAX_HEADS];
   __shared__ int s_bad;
   const int c = blockIdx.x;
   const int b = blockIdx.y;
-  const int t0 = c * kChunk;
-  const int ntok = min(kChunk, T - t0);
   const int tid = threadIdx.x;
-  const int lane = tid & 31, warp = tid >> 5;
-  const int ld = H + 1;
+  const int t = c * kChunk + tid;
   if (tid < NAMOH_MAX_HEADS) s_cnt[tid] = 0;
   if (tid == 0) s_bad = 0;
-
-  // coalesced staging: one warp per token row
-  const float* src = scores + ((size_t)b * T + t0) * H;
-  for (int r = warp; r < ntok; r += kChunk / 32)
-    for (int h = lane; h < H; h += 32) s_scores[r * ld + h] = __ldg(src + (size_t)r * H + h);
+  if (scan_ticket && b == 0 && c == 0 && tid == 0) *scan_ticket = 0;  // consumed by route_scan_kernel
   __syncthreads();
 
-  if (tid < ntok) {
+  if (t < T) {
+    // this token's H logits: independent loads, all in flight together
+    const size_t tok = (size_t)b * T + t;
+    const float* src = scores + tok * H;
     float sc[HMAX];
+    if ((H & 3) == 0 && (reinterpret_cast<uintptr_t>(src) & 15u) == 0) {
+#pragma unroll
+      for (int h4 = 0; h4 < HMAX / 4; ++h4) {
+        float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (h4 * 4 < H) x = __ldg(reinterpret_cast<const float4*>(src) + h4);
+        sc[4 * h4 + 0] = x.x;
+        sc[4 * h4 + 1] = x.y;
+        sc[4 * h4 + 2] = x.z;
+        sc[4 * h4 + 3] = x.w;
+      }
+    } else {
+#pragma unroll
+      for (int h = 0; h < HMAX; ++h) sc[h] = (h < H) ? __ldg(src + h) : 0.f;
+    }
     bool bad = false;
 #pragma unroll
     for (int h = 0; h < HMAX; ++h) {
-      float x = (h < H) ? s_scores[tid * ld + h] : -FLT_MAX;
-      if (h < H && !isfinite(x)) {
+      if (h < H && !isfinite(sc[h])) {
         bad = true;
-        x = -FLT_MAX;
+        sc[h] = -FLT_MAX;
       }
-      sc[h] = x;
     }
-    // softmax denominator over all H logits (fp32)
+    // softmax denominator over all H logits (fp32); pairwise partial maxima / sums
     float mx = -FLT_MAX;
 #pragma unroll
     for (int h = 0; h < HMAX; ++h)
       if (h < H) mx = fmaxf(mx, sc[h]);
-    float z = 0.f;
+    float z0 = 0.f, z1 = 0.f;
 #pragma unroll
-    for (int h = 0; h < HMAX; ++h)
-      if (h < H) z += expf(sc[h] - mx);
-    const float inv_z = 1.0f / z;
+    for (int h = 0; h < HMAX; h += 2) {
+      if (h < H) z0 += expf(sc[h] - mx);
+      if (h + 1 < H) z1 += expf(sc[h + 1] - mx);
+    }
+    const float inv_z = 1.0f / (z0 + z1);
 
     // K passes; pass k picks the best head strictly after the previous pick in the
     // total order (score desc, index asc).
     float pv = 0.f;
     int pi = -1;
-    const size_t base = ((size_t)b * T + t0 + tid) * K;
+    const size_t base = tok * K;
     for (int k = 0; k < K; ++k) {
       float bv = 0.f;
       int bi = -1;
@@ -98,61 +108,64 @@ __global__ void __launch_bounds__(kChunk) route_topk_kernel(const float* __restr
   if (tid == 0 && s_bad) report(status, NAMOH_DEV_NONFINITE_SCORE);
 }
 
-// Per sequence b (one block): for every head, exclusive scan of chunk counts over chunks.
-// Thread (h, p) owns the chunk range [p*per, (p+1)*per).
-__global__ void __launch_bounds__(1024) route_scan_chunks(const int32_t* __restrict__ chunk_count, int H,
+// One block per sequence b: for every head, exclusive scan of the chunk counts over chunks
+// (thread (h, p) owns the chunk range [p*per, (p+1)*per)) -> chunk bases and n[b, h].
+// The last block to finish (ticket) scans n over (b, h) order into seg_offsets.
+__global__ void __launch_bounds__(1024) route_scan_kernel(const int32_t* __restrict__ chunk_count, int B, int H,
                                                           int nchunks, int32_t* __restrict__ chunk_base,
-                                                          int32_t* __restrict__ n_out) {
+                                                          int32_t* __restrict__ n_out, int* __restrict__ ticket,
+                                                          int32_t* __restrict__ seg_offsets) {
   __shared__ int s_part[1024];
+  __shared__ int s_last;
   const int b = blockIdx.x;
   const int tid = threadIdx.x;
-  const int P = blockDim.x / H;  // parts per head
+  const int P = blockDim.x / H;  // parts per head (blockDim is a multiple of H)
   const int h = tid % H, p = tid / H;
   const int per = (nchunks + P - 1) / P;
-  const int c0 = p * per, c1 = min(nchunks, c0 + per);
+  const int c0 = min(nchunks, p * per), c1 = min(nchunks, c0 + per);
   const int32_t* cc = chunk_count + (size_t)b * nchunks * H;
   int sum = 0;
-  if (p < P)
-    for (int c = c0; c < c1; ++c) sum += cc[(size_t)c * H + h];
-  s_part[tid] = (p < P) ? sum : 0;
+  for (int c = c0; c < c1; ++c) sum += __ldg(cc + (size_t)c * H + h);
+  s_part[tid] = sum;
   __syncthreads();
-  if (p < P) {
-    int before = 0;
-    for (int q = 0; q < p; ++q) before += s_part[q * H + h];
-    int run = before;
-    int32_t* out = chunk_base + (size_t)b * nchunks * H;
-    for (int c = c0; c < c1; ++c) {
-      out[(size_t)c * H + h] = run;
-      run += cc[(size_t)c * H + h];
-    }
-    if (p == P - 1) n_out[(size_t)b * H + h] = run;
+  int before = 0;
+  for (int q = 0; q < p; ++q) before += s_part[q * H + h];
+  int run = before;
+  int32_t* out = chunk_base + (size_t)b * nchunks * H;
+  for (int c = c0; c < c1; ++c) {
+    out[(size_t)c * H + h] = run;
+    run += __ldg(cc + (size_t)c * H + h);
   }
-}
+  if (p == P - 1) n_out[(size_t)b * H + h] = run;
 
-// One block: seg_offsets = exclusive scan of n over (b, h) order.
-__global__ void __launch_bounds__(1024) route_scan_segments(const int32_t* __restrict__ n, int nseg,
-                                                            int32_t* __restrict__ seg_offsets) {
-  __shared__ int s_sum[1024];
-  const int tid = threadIdx.x;
-  const int per = (nseg + blockDim.x - 1) / blockDim.x;
-  const int i0 = tid * per, i1 = min(nseg, i0 + per);
-  int sum = 0;
-  for (int i = i0; i < i1; ++i) sum += n[i];
-  s_sum[tid] = sum;
+  // the last sequence block to finish builds seg_offsets
+  __threadfence();
   __syncthreads();
-  // Hillis-Steele inclusive scan over the per-thread sums
-  for (int off = 1; off < (int)blockDim.x; off <<= 1) {
-    int v = (tid >= off) ? s_sum[tid - off] : 0;
+  if (tid == 0) s_last = (atomicAdd(ticket, 1) == B - 1);
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const int nseg = B * H;
+  const volatile int32_t* nv = n_out;
+  const int per2 = (nseg + blockDim.x - 1) / blockDim.x;
+  const int i0 = min(nseg, tid * per2), i1 = min(nseg, i0 + per2);
+  int s2 = 0;
+  for (int i = i0; i < i1; ++i) s2 += nv[i];
+  __syncthreads();
+  s_part[tid] = s2;
+  __syncthreads();
+  for (int off = 1; off < (int)blockDim.x; off <<= 1) {  // Hillis-Steele inclusive scan
+    const int v = (tid >= off) ? s_part[tid - off] : 0;
     __syncthreads();
-    s_sum[tid] += v;
+    s_part[tid] += v;
     __syncthreads();
   }
-  int run = s_sum[tid] - sum;
+  int r2 = s_part[tid] - s2;
   for (int i = i0; i < i1; ++i) {
-    seg_offsets[i] = run;
-    run += n[i];
+    seg_offsets[i] = r2;
+    r2 += nv[i];
   }
-  if (tid == blockDim.x - 1) seg_offsets[nseg] = s_sum[tid];
+  if (tid == blockDim.x - 1) seg_offsets[nseg] = s_part[tid];
 }
 
 // Per chunk: rank = chunk base + rank among this chunk's earlier tokens for the head.
@@ -204,15 +217,10 @@ __global__ void __launch_bounds__(kChunk) route_rank_kernel(const int32_t* __res
 
 template <int HMAX>
 cudaError_t launch_topk(const float* scores, int B, int T, int H, int K, int nchunks, int32_t* topk, float* gate,
-                        int32_t* chunk_count, uint32_t* status, cudaStream_t stream) {
-  const size_t smem = (size_t)kChunk * (H + 1) * sizeof(float);
-  if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(route_topk_kernel<HMAX>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
-    if (e != cudaSuccess) return e;
-  }
+                        int32_t* chunk_count, int* ticket, uint32_t* status, cudaStream_t stream) {
   dim3 grid(nchunks, B);
-  route_topk_kernel<HMAX><<<grid, kChunk, smem, stream>>>(scores, T, H, K, nchunks, topk, gate, chunk_count, status);
+  route_topk_kernel<HMAX><<<grid, kChunk, 0, stream>>>(scores, T, H, K, nchunks, topk, gate, chunk_count, ticket,
+                                                       status);
   return cudaGetLastError();
 }
 
@@ -228,6 +236,7 @@ extern "C" size_t namoh_route_workspace_size(int B, int T, int H, int K) {
   ws.take<int32_t>((size_t)B * nchunks * H);  // chunk counts
   ws.take<int32_t>((size_t)B * nchunks * H);  // chunk bases
   ws.take<int32_t>((size_t)B * H);            // n
+  ws.take<int>(1);                            // scan ticket
   return align_up(ws.used, 256);
 }
 
@@ -246,35 +255,35 @@ extern "C" int namoh_route(const float* scores, int B, int T, int H, int K, int3
   int32_t* chunk_count = nullptr;
   int32_t* chunk_base = nullptr;
   int32_t* n = nullptr;
+  int* ticket = nullptr;
   if (compact) {
     if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return NAMOH_ERR_WORKSPACE;
     WorkspaceCarver ws{static_cast<char*>(workspace), workspace_bytes, 0};
     chunk_count = ws.take<int32_t>((size_t)B * nchunks * H);
     chunk_base = ws.take<int32_t>((size_t)B * nchunks * H);
     n = ws.take<int32_t>((size_t)B * H);
+    ticket = ws.take<int>(1);
     if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
   }
 
   cudaError_t e;
   if (H <= 8)
-    e = launch_topk<8>(scores, B, T, H, K, nchunks, topk_head, gate, chunk_count, dev_status, stream);
+    e = launch_topk<8>(scores, B, T, H, K, nchunks, topk_head, gate, chunk_count, ticket, dev_status, stream);
   else if (H <= 16)
-    e = launch_topk<16>(scores, B, T, H, K, nchunks, topk_head, gate, chunk_count, dev_status, stream);
+    e = launch_topk<16>(scores, B, T, H, K, nchunks, topk_head, gate, chunk_count, ticket, dev_status, stream);
   else if (H <= 32)
-    e = launch_topk<32>(scores, B, T, H, K, nchunks, topk_head, gate, chunk_count, dev_status, stream);
+    e = launch_topk<32>(scores, B, T, H, K, nchunks, topk_head, gate, chunk_count, ticket, dev_status, stream);
   else
-    e = launch_topk<64>(scores, B, T, H, K, nchunks, topk_head, gate, chunk_count, dev_status, stream);
-  if (e != cudaSuccess) return NAMOH_ERR_CUDA;
+    e = launch_topk<64>(scores, B, T, H, K, nchunks, topk_head, gate, chunk_count, ticket, dev_status, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "route_topk_kernel launch");
   if (!compact) return NAMOH_OK;
 
   const int scan_threads = 1024 - (1024 % H);
-  route_scan_chunks<<<B, scan_threads, 0, stream>>>(chunk_count, H, nchunks, chunk_base, n);
-  if (cudaGetLastError() != cudaSuccess) return NAMOH_ERR_CUDA;
-  route_scan_segments<<<1, 1024, 0, stream>>>(n, B * H, seg_offsets);
-  if (cudaGetLastError() != cudaSuccess) return NAMOH_ERR_CUDA;
+  route_scan_kernel<<<B, scan_threads, 0, stream>>>(chunk_count, B, H, nchunks, chunk_base, n, ticket, seg_offsets);
+  if (const int st = cuda_check_launch("route_scan_kernel launch")) return st;
   route_rank_kernel<<<dim3(nchunks, B), kChunk, 0, stream>>>(topk_head, T, H, K, nchunks, chunk_base, seg_offsets,
                                                              rank, row, row_src);
-  if (cudaGetLastError() != cudaSuccess) return NAMOH_ERR_CUDA;
+  if (const int st = cuda_check_launch("route_rank_kernel launch")) return st;
   return NAMOH_OK;
 }
 
@@ -316,7 +325,7 @@ extern "C" int namoh_route_noalloc(const float* scores, int B, int T, int H, int
   if (B < 1 || T < 1 || H < 1 || K < 1 || K > H || H > NAMOH_MAX_HEADS) return NAMOH_ERR_INVALID_ARG;
   if (seg_offsets && namoh_route_workspace_size(B, T, H, K) > kRouteStaticScratchBytes) return NAMOH_ERR_WORKSPACE;
   void* scratch = route_scratch_address();
-  if (!scratch) return NAMOH_ERR_CUDA;
+  if (!scratch) return cuda_fail(cudaErrorInvalidSymbol, "cudaGetSymbolAddress of the routing scratch");
   return namoh_route(scores, B, T, H, K, topk_head, gate, rank, row, seg_offsets, row_src, scratch,
                      kRouteStaticScratchBytes, dev_status, stream);
 }
