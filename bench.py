@@ -192,16 +192,13 @@ def run_gpu(args, rank: int, world: int):
         if ev is not None:
             ev[1].record()
         namoh.namoh_rope_pack(q, k, v, ro.seg_offsets, B=B, T=T, H=H, K=K, group=g, rope_base=wl.base, q_rot=q_rot,
-                              k_cache=k_cache, v_cache=v, status=status)
+                              k_cache=k_cache, v_cache=v, status=status, plan=plan)
         if ev is not None:
             ev[2].record()
-        namoh.namoh_attention_plan(ro.seg_offsets, B=B, T=T, H=H, K=K, group=g, plan=plan)
-        if ev is not None:
-            ev[3].record()
         namoh.namoh_attention(q_rot, k_cache, v, ro.seg_offsets, ro.row_src, ro.gate, plan, B=B, T=T, H=H, K=K,
                               group=g, y=y, status=status)
         if ev is not None:
-            ev[4].record()
+            ev[3].record()
 
     clocks = ClockSampler(dev.index).__enter__()
     for _ in range(args.warmup):
@@ -210,7 +207,7 @@ def run_gpu(args, rank: int, world: int):
     torch.cuda.synchronize()
     n_seg = acc.segment_lengths(ro.seg_offsets.cpu().numpy())
     flops = acc.attention_flops(n_seg, d, g)
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
     fl_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
     enqueue_s = []
     barrier(world)
@@ -229,10 +226,10 @@ def run_gpu(args, rank: int, world: int):
     flush_ms = [a.elapsed_time(b) for a, b in fl_ev]
     # the host finished enqueueing each step before the flush ahead of it ended
     gapless = all(e * 1e3 < f for e, f in zip(enqueue_s, flush_ms))
-    stage = np.array([[evs[i][j].elapsed_time(evs[i][j + 1]) for j in range(4)] for i in range(args.steps)])
+    stage = np.array([[evs[i][j].elapsed_time(evs[i][j + 1]) for j in range(3)] for i in range(args.steps)])
     step_ms = float(stage.sum(1).mean())
     step_ms = max_over_ranks(step_ms, world)
-    attn_ms = float(stage[:, 3].mean())
+    attn_ms = float(stage[:, 2].mean())
     st = int(status.item())
 
     # ---- end to end through the public API with host buffers (pinned), copies timed
@@ -293,8 +290,8 @@ def run_gpu(args, rank: int, world: int):
                    "l2": "flushed before every timed step (2 GB write)", "seed": wl.seed,
                    "c_attn": acc.interaction_count(n_seg, g), "flops_per_step": flops,
                    "cv2_mean": float(np.mean([acc.cv2(n_seg[b * wl.Hr:(b + 1) * wl.Hr]) for b in range(B)]))},
-        "stages_ms": {"route": float(stage[:, 0].mean()), "rope_pack": float(stage[:, 1].mean()),
-                      "plan": float(stage[:, 2].mean()), "attention": attn_ms},
+        "stages_ms": {"route": float(stage[:, 0].mean()), "rope_pack_plan": float(stage[:, 1].mean()),
+                      "attention": attn_ms},
         "roofline": {"kernel": "attn_fwd_kernel<128>", "bound": "tensor", "achieved": achieved, "peak": peak_tf,
                      "unit": "TFLOP/s", "frac": achieved / peak_tf, "traffic": traffic,
                      "peak_source": f"{pk_kind} bf16 dense (burst)",
@@ -302,7 +299,8 @@ def run_gpu(args, rank: int, world: int):
         "e2e": {"value": world * flops / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s", "ms_per_step": e2e_ms,
                 "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                 "api": "namoh_route + namoh_prefill from pinned host buffers, y copied back"},
-        "gpu_launches": 7 * args.steps,
+        # per timed step: route (3 kernels) + rope/plan (1) + attention (1); the e2e loop the same again
+        "gpu_launches": 2 * 5 * args.steps,
         "wall_s_timed_region": wall,
         "host_enqueue_ms_max": 1e3 * max(enqueue_s), "flush_ms_min": min(flush_ms), "stage_timing_gapless": gapless,
         "device_status": st,

@@ -101,6 +101,9 @@ NAMOH_API const char *namoh_last_error_string(void);
  * Requires 1 <= K <= H <= NAMOH_MAX_HEADS, B >= 1, T >= 1, B*T*K < 2^31.
  * Non-finite logits set NAMOH_DEV_NONFINITE_SCORE (that token's outputs are
  * unspecified but in range).  Integer outputs are deterministic.
+ * When every 256-token chunk fits on the GPU at once (B*ceil(T/256) blocks), the
+ * packed layout is built in one cooperative launch (after a 4-byte memset of
+ * the workspace); otherwise in three launches.  Both give identical results.
  * ------------------------------------------------------------------------- */
 NAMOH_API size_t namoh_route_workspace_size(int B, int T, int H, int K);
 NAMOH_API int namoh_route(const float *scores, int B, int T, int H, int K, int32_t *topk_head, float *gate,
@@ -126,8 +129,8 @@ NAMOH_API int namoh_route(const float *scores, int B, int T, int H, int K, int32
  * address (cudaGetSymbolAddress) with that device current; make that first call
  * before any stream capture.  Every call on a device shares the one array and
  * leaves its last contents there; the only word that must start at zero (a
- * ticket counter) is cleared by the first routing kernel of each call, and every
- * other word is written before it is read.  Calls that overlap on the GPU -- on
+ * grid-barrier counter) is cleared by a memset that each call enqueues first,
+ * and every other word is written before it is read.  Calls that overlap on the GPU -- on
  * different streams, or from different host threads -- race on it and must be
  * serialised by the caller.
  * ------------------------------------------------------------------------- */
@@ -177,6 +180,9 @@ NAMOH_API int namoh_prefill(const uint16_t *q, const uint16_t *k, const uint16_t
  * namoh_rope_pack (Sec. 3.2, Eq. namoh-head-rope): rotates every query row to
  *   its rank into q_rot [R*g, d] bf16 (caller-owned), writes k~ to k_cache and
  *   copies v to v_cache (unless v_cache == v, allowed only without seg_base).
+ *   plan: NULL, or a buffer as namoh_attention_plan takes (plan_bytes long); the
+ *   same launch then also writes the plan that namoh_attention_plan would write
+ *   with seg_cap (or NULL when seg_base is NULL), saving one kernel launch.
  *
  * namoh_attention_plan (Sec. 3.2 "Efficient execution", length-aware
  *   scheduling): writes into `plan` (namoh_attention_plan_size bytes, 16-byte
@@ -194,7 +200,8 @@ NAMOH_API int namoh_prefill(const uint16_t *q, const uint16_t *k, const uint16_t
 NAMOH_API int namoh_rope_pack(const uint16_t *q, const uint16_t *k, const uint16_t *v, int B, int T, int H, int K,
                               int d_head, int group, float rope_base, const int32_t *seg_offsets, uint16_t *q_rot,
                               uint16_t *k_cache, uint16_t *v_cache, const int64_t *seg_base, const int32_t *seg_cap,
-                              int64_t cache_rows, uint32_t *dev_status, void *stream);
+                              int64_t cache_rows, uint32_t *dev_status, void *plan, size_t plan_bytes,
+                              void *stream);
 NAMOH_API size_t namoh_attention_plan_size(int B, int T, int H, int K, int group);
 NAMOH_API int namoh_attention_plan(const int32_t *seg_offsets, int B, int T, int H, int K, int group,
                                    const int32_t *seg_cap, void *plan, size_t plan_bytes, void *stream);

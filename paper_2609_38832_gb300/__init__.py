@@ -143,8 +143,11 @@ def namoh_rope_pack(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, seg_offse
                     H: int, K: int, group: int = 1, rope_base: float = 10000.0, q_rot: Optional[torch.Tensor] = None,
                     k_cache: Optional[torch.Tensor] = None, v_cache: Optional[torch.Tensor] = None,
                     seg_base: Optional[torch.Tensor] = None, seg_cap: Optional[torch.Tensor] = None,
-                    status: Optional[torch.Tensor] = None, stream=None):
-    """Prefill stage 1: RoPE at rank and cache pack.  Returns (q_rot, k_cache, v_cache)."""
+                    status: Optional[torch.Tensor] = None, plan: Optional[torch.Tensor] = None, stream=None):
+    """Prefill stage 1: RoPE at rank and cache pack.  Returns (q_rot, k_cache, v_cache).
+
+    With ``plan`` (a buffer from namoh_attention_plan) the same launch also rebuilds the
+    attention plan for these seg_offsets."""
     lib = _abi.load()
     d = q.shape[-1]
     dev = q.device
@@ -155,7 +158,8 @@ def namoh_rope_pack(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, seg_offse
     st = _status(status, dev)
     rc = lib.namoh_rope_pack(_ptr(q), _ptr(k), _ptr(v), B, T, H, K, d, group, float(rope_base), _ptr(seg_offsets),
                              _ptr(q_rot), _ptr(k_cache), _ptr(v_cache), _ptr(seg_base), _ptr(seg_cap),
-                             k_cache.shape[0], _ptr(st), _stream(stream))
+                             k_cache.shape[0], _ptr(st), _ptr(plan), 0 if plan is None else plan.numel(),
+                             _stream(stream))
     _abi.check("namoh_rope_pack", rc)
     return q_rot, k_cache, v_cache
 

@@ -39,7 +39,8 @@ SIGNATURES = {
     "namoh_prefill_workspace_size": (_SZ, [_I, _I, _I, _I, _I, _I]),
     "namoh_prefill": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _P, _P, _P, _I64, _P, _P,
                            _SZ, _P, _P]),
-    "namoh_rope_pack": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _P, _I64, _P, _P]),
+    "namoh_rope_pack": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _P, _I64, _P, _P, _SZ,
+                             _P]),
     "namoh_attention_plan_size": (_SZ, [_I, _I, _I, _I, _I]),
     "namoh_attention_plan": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _SZ, _P]),
     "namoh_attention": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _P, _I64, _P, _SZ, _P, _P, _P]),

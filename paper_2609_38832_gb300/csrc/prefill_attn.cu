@@ -31,19 +31,22 @@
 // Shared memory (d = 128): Q 32 KB + 6 x 32 KB ring = 224 KB.
 // Every mbarrier wait is bounded (NAMOH_DEV_TIMEOUT, then all roles drain and exit).
 #include "common.cuh"
+#include "plan.cuh"
 
 namespace namoh {
 
 cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const uint16_t* v, int R, int g,
                              const int32_t* seg_offsets, int nseg, const int64_t* seg_base, const int32_t* seg_cap,
                              long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache, bool copy_v,
-                             const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream);
+                             const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream,
+                             void* plan, int plan_qtiles, const int32_t* plan_cap);
 
 namespace attn {
 
 constexpr int BM = 128;              // query rows per tile (one tile per work item)
 constexpr int BN = 128;              // keys per tile
 constexpr int kItemRows = BM;
+static_assert(kItemRows == kPlanTileRows, "the plan and the kernel must agree on the query tile");
 constexpr int kSoftmaxWarps = 4;     // warps 0-3: thread i owns query row i (TMEM lane i)
 constexpr int kWarpLoad = 4;
 constexpr int kWarpMma = 5;
@@ -496,49 +499,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// One block.  Items are the 128-row query tiles q of every segment and group head j,
-// ordered by decreasing cost (q descending: tile q needs q + 1 key tiles), then (segment, j).
-// Segments longer than their cache capacity are skipped (the RoPE stage reports them).
-// Also zeroes the dynamic scheduler's counters.  seg_offsets (and seg_cap) are staged in
-// shared memory first so that no loop below waits on global memory.
+// One block builds the work list (see build_plan) and zeroes the scheduler's counters.
 __global__ void __launch_bounds__(1024) plan_kernel(const int32_t* __restrict__ seg_offsets, int nseg,
                                                     const int32_t* __restrict__ seg_cap, int g, int max_qtiles,
                                                     int* __restrict__ header, int2* __restrict__ items) {
   extern __shared__ int s_dyn[];
-  int* s_count = s_dyn;                   // [max_qtiles]: segments with more than q query tiles
-  int* s_start = s_dyn + max_qtiles;      // [max_qtiles]: first item of cost q + 1
-  int* s_ntile = s_dyn + 2 * max_qtiles;  // [nseg]: query tiles of each segment (0 if skipped)
-  const int tid = threadIdx.x;
-  for (int q = tid; q < max_qtiles; q += blockDim.x) s_count[q] = 0;
-  for (int s = tid; s < nseg; s += blockDim.x) {
-    const int n = __ldg(seg_offsets + s + 1) - __ldg(seg_offsets + s);
-    const bool skip = seg_cap && n > __ldg(seg_cap + s);
-    s_ntile[s] = skip ? 0 : min((n + kItemRows - 1) / kItemRows, max_qtiles);
-  }
-  __syncthreads();
-  for (int s = tid; s < nseg; s += blockDim.x)
-    if (s_ntile[s] > 0) atomicAdd(&s_count[s_ntile[s] - 1], 1);  // histogram of tile counts
-  __syncthreads();
-  if (tid == 0) {
-    int above = 0, run = 0;  // above: segments with more than q tiles
-    for (int q = max_qtiles - 1; q >= 0; --q) {
-      above += s_count[q];
-      s_count[q] = above;
-      s_start[q] = run;
-      run += above * g;
-    }
-    header[0] = 0;  // next item
-    header[1] = 0;  // CTAs finished
-    header[2] = run;
-  }
-  __syncthreads();
-  for (int q = tid; q < max_qtiles; q += blockDim.x) {
-    if (s_count[q] == 0) continue;
-    int pos = s_start[q];
-    for (int s = 0; s < nseg; ++s)
-      if (s_ntile[s] > q)
-        for (int j = 0; j < g; ++j) items[pos++] = make_int2(s * g + j, q);
-  }
+  build_plan(seg_offsets, nseg, seg_cap, g, max_qtiles, header, items, s_dyn);
 }
 
 bool encode_rows_map(CUtensorMap* map, const void* base, long long rows, int row_elems) {
@@ -599,10 +565,16 @@ size_t plan_bytes_for(int B, int T, int Hr, int Kr, int g) {
   return 16 + (size_t)max_items * sizeof(int2);
 }
 
+int plan_qtiles_for(int T) { return (T + kPlanTileRows - 1) / kPlanTileRows; }  // query tiles per segment, at most
+
+// The RoPE launch builds the plan in one extra block when the plan's shared memory is small
+// enough not to cut the RoPE blocks' occupancy.
+constexpr int kFusedPlanSmemMax = 32 * 1024;
+
 int launch_plan(const int32_t* seg_offsets, int nseg, int T, int g, const int32_t* seg_cap, void* plan,
                 cudaStream_t stream) {
-  const int max_qtiles = (T + attn::kItemRows - 1) / attn::kItemRows;  // query tiles per segment, at most
-  const int smem = (2 * max_qtiles + nseg) * (int)sizeof(int);
+  const int max_qtiles = plan_qtiles_for(T);
+  const int smem = plan_smem_ints(max_qtiles, nseg) * (int)sizeof(int);
   if (smem > 200 * 1024) return NAMOH_ERR_UNSUPPORTED;
   if (smem > 48 * 1024) {
     const cudaError_t e = cudaFuncSetAttribute(attn::plan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
@@ -612,6 +584,27 @@ int launch_plan(const int32_t* seg_offsets, int nseg, int T, int g, const int32_
   int2* items = reinterpret_cast<int2*>(static_cast<char*>(plan) + 16);
   attn::plan_kernel<<<1, 1024, smem, stream>>>(seg_offsets, nseg, seg_cap, g, max_qtiles, header, items);
   return cuda_check_launch("plan_kernel launch");
+}
+
+// RoPE + cache pack; with a plan buffer also the attention plan (in the same launch when
+// the plan's shared memory is small, else as a second kernel).
+int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int Hr, int R,
+                         int d_head, int group, float rope_base, const int32_t* seg_offsets, uint16_t* q_rot,
+                         uint16_t* k_cache, uint16_t* v_cache, const int64_t* seg_base, const int32_t* seg_cap,
+                         long long cache_rows, uint32_t* dev_status, void* plan, const DeviceInfo& info,
+                         cudaStream_t stream) {
+  RopeTable tab;
+  fill_rope_table(&tab, d_head, (double)rope_base);
+  const int nseg = B * Hr;
+  const int qtiles = plan_qtiles_for(T);
+  const int32_t* plan_cap = seg_base ? seg_cap : nullptr;
+  const bool fuse_plan = plan && plan_smem_ints(qtiles, nseg) * (int)sizeof(int) <= kFusedPlanSmemMax;
+  const cudaError_t e = launch_rope_pack(d_head, q, k, v, R, group, seg_offsets, nseg, seg_base, seg_cap, cache_rows,
+                                         q_rot, k_cache, v_cache, v_cache != v, tab, dev_status, info.sm_count, stream,
+                                         fuse_plan ? plan : nullptr, qtiles, plan_cap);
+  if (e != cudaSuccess) return cuda_fail(e, "rope_pack_kernel launch");
+  if (plan && !fuse_plan) return launch_plan(seg_offsets, nseg, T, group, plan_cap, plan, stream);
+  return NAMOH_OK;
 }
 
 int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint16_t* v_cache, int B, int T, int Hr,
@@ -653,7 +646,8 @@ using namespace namoh;
 extern "C" int namoh_rope_pack(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int H, int K,
                                int d_head, int group, float rope_base, const int32_t* seg_offsets, uint16_t* q_rot,
                                uint16_t* k_cache, uint16_t* v_cache, const int64_t* seg_base, const int32_t* seg_cap,
-                               int64_t cache_rows, uint32_t* dev_status, void* stream_v) {
+                               int64_t cache_rows, uint32_t* dev_status, void* plan, size_t plan_bytes,
+                               void* stream_v) {
   if (!q || !k || !v || !seg_offsets || !q_rot || !k_cache || !v_cache || !dev_status) return NAMOH_ERR_INVALID_ARG;
   int Hr, Kr;
   long long R;
@@ -669,14 +663,13 @@ extern "C" int namoh_rope_pack(const uint16_t* q, const uint16_t* k, const uint1
   } else {
     cache_rows = R;
   }
+  if (plan && ((reinterpret_cast<uintptr_t>(plan) & 15u) || plan_bytes < plan_bytes_for(B, T, Hr, Kr, group)))
+    return NAMOH_ERR_WORKSPACE;
   DeviceInfo info;
   if (!current_device_info(&info)) return cuda_fail(cudaGetLastError(), "device query");
-  RopeTable tab;
-  fill_rope_table(&tab, d_head, (double)rope_base);
-  const cudaError_t e = launch_rope_pack(d_head, q, k, v, (int)R, group, seg_offsets, B * Hr, seg_base, seg_cap,
-                                         cache_rows, q_rot, k_cache, v_cache, v_cache != v, tab, dev_status,
-                                         info.sm_count, reinterpret_cast<cudaStream_t>(stream_v));
-  return e == cudaSuccess ? NAMOH_OK : cuda_fail(e, "rope_pack_kernel launch");
+  return launch_rope_and_plan(q, k, v, B, T, Hr, (int)R, d_head, group, rope_base, seg_offsets, q_rot, k_cache,
+                              v_cache, seg_base, seg_cap, cache_rows, dev_status, plan, info,
+                              reinterpret_cast<cudaStream_t>(stream_v));
 }
 
 extern "C" size_t namoh_attention_plan_size(int B, int T, int H, int K, int group) {
@@ -763,13 +756,8 @@ extern "C" int namoh_prefill(const uint16_t* q, const uint16_t* k, const uint16_
   if (!device_ok(&info)) return NAMOH_ERR_UNSUPPORTED;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
 
-  RopeTable tab;
-  fill_rope_table(&tab, d_head, (double)rope_base);
-  const cudaError_t er = launch_rope_pack(d_head, q, k, v, (int)R, group, seg_offsets, B * Hr, seg_base, seg_cap,
-                                          cache_rows, q_rot, k_cache, v_cache, v_cache != v, tab, dev_status,
-                                          info.sm_count, stream);
-  if (er != cudaSuccess) return cuda_fail(er, "rope_pack_kernel launch");
-  st = launch_plan(seg_offsets, B * Hr, T, group, seg_base ? seg_cap : nullptr, plan, stream);
+  st = launch_rope_and_plan(q, k, v, B, T, Hr, (int)R, d_head, group, rope_base, seg_offsets, q_rot, k_cache, v_cache,
+                            seg_base, seg_cap, cache_rows, dev_status, plan, info, stream);
   if (st != NAMOH_OK) return st;
   if (seg_len) {
     seg_len_kernel<<<(B * Hr + 255) / 256, 256, 0, stream>>>(seg_offsets, B * Hr, seg_len);

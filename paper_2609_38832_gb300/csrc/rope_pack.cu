@@ -5,52 +5,63 @@
 // (j, j + D/2) and moves them with 16-byte loads/stores.  The angle is computed once per
 // row and applied to K and to all g query heads of the row (KV-group routing shares the
 // rank, App. C).  Outputs: Q~ (bf16 scratch for the attention kernel), K~ into the key
-// cache, and V copied into the value cache unless the caller passed v_cache == v.
+// cache, and V copied into the value cache unless the caller passed v_cache == v.  When
+// given a plan buffer, one extra block builds the attention work list in the same launch.
 #include "common.cuh"
+#include "plan.cuh"
 
 namespace namoh {
 
 constexpr int kRopeStageMax = 8192;  // seg_offsets entries staged in shared memory (32 KB)
 
-template <int D>
+// With a plan header given, block 0 builds the attention work list (it depends only on
+// seg_offsets) while the other blocks rotate rows; it goes first so that it is resident in
+// the first wave.
+template <int D, int G>
 __global__ void __launch_bounds__(256) rope_pack_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ k,
-                                                        const uint16_t* __restrict__ v, int R, int g,
+                                                        const uint16_t* __restrict__ v, int R,
                                                         const int32_t* __restrict__ seg_offsets, int nseg,
                                                         const int64_t* __restrict__ seg_base,
                                                         const int32_t* __restrict__ seg_cap, long long cache_rows,
                                                         uint16_t* __restrict__ q_rot, uint16_t* __restrict__ k_cache,
                                                         uint16_t* __restrict__ v_cache, int copy_v, RopeTable tab,
-                                                        uint32_t* __restrict__ status) {
+                                                        uint32_t* __restrict__ status, int* __restrict__ plan_header,
+                                                        int2* __restrict__ plan_items, const int32_t* __restrict__ plan_cap,
+                                                        int plan_qtiles) {
   constexpr int LPR = D / 16;  // threads per row
   constexpr int HALF = D / 2;
-  constexpr int GMAX = 8;      // largest group size
-  extern __shared__ int32_t s_off[];  // seg_offsets staged when they fit (nseg + 1 <= kStageMax)
+  extern __shared__ int32_t s_dyn[];
+  const int first = plan_header ? 1 : 0;
+  if ((int)blockIdx.x < first) {
+    build_plan(seg_offsets, nseg, plan_cap, G, plan_qtiles, plan_header, plan_items, s_dyn);
+    return;
+  }
+  const int rope_blocks = gridDim.x - first;
+  const int block = blockIdx.x - first;
   const bool staged = (nseg + 1) <= kRopeStageMax;
   if (staged) {
-    for (int i = threadIdx.x; i <= nseg; i += blockDim.x) s_off[i] = __ldg(seg_offsets + i);
+    for (int i = threadIdx.x; i <= nseg; i += blockDim.x) s_dyn[i] = __ldg(seg_offsets + i);
     __syncthreads();
   }
-  const int32_t* offs = staged ? s_off : seg_offsets;
+  const int32_t* offs = staged ? s_dyn : seg_offsets;
   const int lane_in_row = threadIdx.x % LPR;
   const int j0 = lane_in_row * 8;
-  const long long groups = (long long)gridDim.x * (blockDim.x / LPR);
+  const long long groups = (long long)rope_blocks * (blockDim.x / LPR);
   float th_hi[8], th_lo[8];
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     th_hi[i] = tab.theta_hi[j0 + i];
     th_lo[i] = tab.theta_lo[j0 + i];
   }
-  for (long long r = (long long)blockIdx.x * (blockDim.x / LPR) + threadIdx.x / LPR; r < R; r += groups) {
+  for (long long r = (long long)block * (blockDim.x / LPR) + threadIdx.x / LPR; r < R; r += groups) {
     // every load of this row first, so their latencies overlap
-    uint4 ka = __ldg(reinterpret_cast<const uint4*>(k + (size_t)r * D + j0));
-    uint4 kb = __ldg(reinterpret_cast<const uint4*>(k + (size_t)r * D + HALF + j0));
-    uint4 qa[GMAX], qb[GMAX];
+    const uint4 ka = __ldg(reinterpret_cast<const uint4*>(k + (size_t)r * D + j0));
+    const uint4 kb = __ldg(reinterpret_cast<const uint4*>(k + (size_t)r * D + HALF + j0));
+    uint4 qa[G], qb[G];
 #pragma unroll
-    for (int j = 0; j < GMAX; ++j) {
-      if (j < g) {
-        qa[j] = __ldg(reinterpret_cast<const uint4*>(q + ((size_t)r * g + j) * D + j0));
-        qb[j] = __ldg(reinterpret_cast<const uint4*>(q + ((size_t)r * g + j) * D + HALF + j0));
-      }
+    for (int j = 0; j < G; ++j) {
+      qa[j] = __ldg(reinterpret_cast<const uint4*>(q + ((size_t)r * G + j) * D + j0));
+      qb[j] = __ldg(reinterpret_cast<const uint4*>(q + ((size_t)r * G + j) * D + HALF + j0));
     }
     uint4 va = make_uint4(0, 0, 0, 0), vb = va;
     if (copy_v) {
@@ -94,8 +105,7 @@ __global__ void __launch_bounds__(256) rope_pack_kernel(const uint16_t* __restri
       *reinterpret_cast<uint4*>(dst_row + HALF + j0) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
     };
 #pragma unroll
-    for (int j = 0; j < GMAX; ++j)
-      if (j < g) rotate(qa[j], qb[j], q_rot + ((size_t)r * g + j) * D);
+    for (int j = 0; j < G; ++j) rotate(qa[j], qb[j], q_rot + ((size_t)r * G + j) * D);
     if (write_cache) {
       rotate(ka, kb, k_cache + (size_t)dst * D);
       if (copy_v) {
@@ -107,24 +117,62 @@ __global__ void __launch_bounds__(256) rope_pack_kernel(const uint16_t* __restri
   }
 }
 
+template <int D>
+cudaError_t launch_rope_pack_d(int g, dim3 grid, size_t smem, cudaStream_t stream, const uint16_t* q,
+                               const uint16_t* k, const uint16_t* v, int R, const int32_t* seg_offsets, int nseg,
+                               const int64_t* seg_base, const int32_t* seg_cap, long long cache_rows, uint16_t* q_rot,
+                               uint16_t* k_cache, uint16_t* v_cache, int copy_v, const RopeTable& tab,
+                               uint32_t* status, int* plan_header, int2* plan_items, const int32_t* plan_cap,
+                               int plan_qtiles) {
+  switch (g) {
+#define NAMOH_ROPE_CASE(GG)                                                                                     \
+  case GG:                                                                                                      \
+    if (smem > 48 * 1024) {                                                                                     \
+      cudaError_t e = cudaFuncSetAttribute(rope_pack_kernel<D, GG>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
+                                           (int)smem);                                                          \
+      if (e != cudaSuccess) return e;                                                                           \
+    }                                                                                                           \
+    rope_pack_kernel<D, GG><<<grid, 256, smem, stream>>>(q, k, v, R, seg_offsets, nseg, seg_base, seg_cap,       \
+                                                         cache_rows, q_rot, k_cache, v_cache, copy_v, tab, status, \
+                                                         plan_header, plan_items, plan_cap, plan_qtiles);        \
+    break;
+    NAMOH_ROPE_CASE(1)
+    NAMOH_ROPE_CASE(2)
+    NAMOH_ROPE_CASE(4)
+    NAMOH_ROPE_CASE(8)
+#undef NAMOH_ROPE_CASE
+    default:
+      return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
 cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const uint16_t* v, int R, int g,
                              const int32_t* seg_offsets, int nseg, const int64_t* seg_base, const int32_t* seg_cap,
                              long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache, bool copy_v,
-                             const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream) {
-  if (R == 0) return cudaSuccess;
+                             const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream,
+                             void* plan, int plan_qtiles, const int32_t* plan_cap) {
   const int threads = 256;
   const int rows_per_block = threads / (D / 16);
   long long blocks = ((long long)R + rows_per_block - 1) / rows_per_block;
   const long long cap = (long long)sm_count * 8;
   if (blocks > cap) blocks = cap;
-  const size_t smem = (nseg + 1 <= kRopeStageMax) ? (size_t)(nseg + 1) * sizeof(int32_t) : 0;
+  int* plan_header = static_cast<int*>(plan);
+  int2* plan_items = plan ? reinterpret_cast<int2*>(static_cast<char*>(plan) + 16) : nullptr;
+  const long long grid = blocks + (plan ? 1 : 0);
+  if (grid == 0) return cudaSuccess;
+  size_t smem = (nseg + 1 <= kRopeStageMax) ? (size_t)(nseg + 1) * sizeof(int32_t) : 0;
+  if (plan) {
+    const size_t ps = (size_t)plan_smem_ints(plan_qtiles, nseg) * sizeof(int);
+    if (ps > smem) smem = ps;
+  }
   if (D == 128)
-    rope_pack_kernel<128><<<(int)blocks, threads, smem, stream>>>(q, k, v, R, g, seg_offsets, nseg, seg_base, seg_cap,
-                                                               cache_rows, q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status);
-  else
-    rope_pack_kernel<64><<<(int)blocks, threads, smem, stream>>>(q, k, v, R, g, seg_offsets, nseg, seg_base, seg_cap,
-                                                              cache_rows, q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status);
-  return cudaGetLastError();
+    return launch_rope_pack_d<128>(g, dim3((unsigned)grid), smem, stream, q, k, v, R, seg_offsets, nseg, seg_base,
+                                   seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status,
+                                   plan_header, plan_items, plan_cap, plan_qtiles);
+  return launch_rope_pack_d<64>(g, dim3((unsigned)grid), smem, stream, q, k, v, R, seg_offsets, nseg, seg_base,
+                                seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status,
+                                plan_header, plan_items, plan_cap, plan_qtiles);
 }
 
 }  // namespace namoh

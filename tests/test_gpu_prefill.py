@@ -135,3 +135,35 @@ def _sampled_check(namoh, oracle_mod, wl: ni.PrefillWorkload, nsamples: int = 16
 @pytest.mark.parametrize("wl", [ni.BALANCED, ni.SKEWED, *ni.H_SWEEP, ni.GQA], ids=lambda w: w.name)
 def test_prefill_full_size_sampled(namoh, oracle_mod, wl):
     _sampled_check(namoh, oracle_mod, wl)
+
+
+def test_prefill_many_segments_unstaged(namoh, oracle_mod):
+    """B*H = 8320 segments: more offsets than the RoPE kernel stages in shared memory and a
+    plan too large to build inside the RoPE launch (separate plan kernel)."""
+    _full_check(namoh, oracle_mod, ni.PrefillWorkload("many_segments", B=130, T=64, H=64, K=2, d=64, seed=11))
+
+
+@pytest.mark.parametrize("wl", [ni.PR1, ni.PrefillWorkload("gqa_g4_staged", B=2, T=900, H=16, K=8, d=128, g=4, seed=12)],
+                         ids=lambda w: w.name)
+def test_staged_calls_match_prefill(namoh, wl):
+    """namoh_rope_pack (building the plan in the same launch, or not) + namoh_attention give
+    the bytes namoh_prefill gives."""
+    scores = wl.scores()
+    q, k, v = (dev_bf16(a) for a in wl.qkv())
+    ro = namoh.namoh_route(torch.from_numpy(scores).cuda(), wl.Kr)
+    y_ref, _, _ = namoh.namoh_prefill(q, k, v, ro.seg_offsets, ro.row_src, ro.gate, B=wl.B, T=wl.T, H=wl.H, K=wl.K,
+                                      group=wl.g, rope_base=wl.base, status=ro.status)
+    kw = dict(B=wl.B, T=wl.T, H=wl.H, K=wl.K, group=wl.g)
+    for fused in (True, False):
+        plan = namoh.namoh_attention_plan(ro.seg_offsets, **kw)
+        plan.fill_(0xAB)  # stale bytes: the fused launch must rebuild every word it uses
+        if fused:
+            q_rot, kc, vc = namoh.namoh_rope_pack(q, k, v, ro.seg_offsets, rope_base=wl.base, status=ro.status,
+                                                  plan=plan, **kw)
+        else:
+            q_rot, kc, vc = namoh.namoh_rope_pack(q, k, v, ro.seg_offsets, rope_base=wl.base, status=ro.status, **kw)
+            namoh.namoh_attention_plan(ro.seg_offsets, plan=plan, **kw)
+        y = namoh.namoh_attention(q_rot, kc, vc, ro.seg_offsets, ro.row_src, ro.gate, plan, status=ro.status, **kw)
+        torch.cuda.synchronize()
+        assert torch.equal(y.view(torch.int16), y_ref.view(torch.int16)), f"fused plan = {fused}"
+    assert int(ro.status.item()) == 0

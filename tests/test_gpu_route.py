@@ -41,6 +41,8 @@ def _check_route(namoh, oracle_mod, s: np.ndarray, K: int):
     (2, 300, 64, 1),     # K = 1 with the widest router
     (1, 1, 8, 2),        # one token
     (4, 4096, 16, 4),    # balanced routing at full size
+    (2, 19200, 64, 8),   # 150 chunks of the widest router: close to one resident block per SM
+    (3, 70000, 16, 4),   # more chunks than fit on the GPU at once: the three-launch path
 ])
 def test_route_matches_oracle(namoh, oracle_mod, B, T, H, K):
     _check_route(namoh, oracle_mod, ni.router_scores(0, B, T, H), K)
@@ -105,3 +107,16 @@ def test_route_nonfinite_sets_status(namoh):
     top = out.topk_head.cpu().numpy()
     assert top.min() >= 0 and top.max() < 8  # still in range
     assert int(out.seg_offsets[-1].item()) == 300 * 2
+
+
+def test_route_repeated_calls_reuse_workspace(namoh, oracle_mod):
+    """Back-to-back calls on one workspace (the grid-barrier counter is reset by every call)."""
+    ws = namoh.Workspace()
+    for seed in (3, 4, 3):
+        s = ni.router_scores(seed, 2, 3000, 16)
+        out = namoh.namoh_route(torch.from_numpy(s).cuda(), 4, workspace=ws)
+        torch.cuda.synchronize()
+        r = oracle_mod.route(s, 4)
+        np.testing.assert_array_equal(out.row_src.cpu().numpy(), r["row_src"])
+        np.testing.assert_array_equal(out.seg_offsets.cpu().numpy(), r["seg_offsets"])
+        assert int(out.status.item()) == 0
