@@ -79,14 +79,20 @@ struct Bars {
   uint64_t s_full[kSBufs];  // S written into buffer b (one barrier per buffer: at an item
                             // boundary two S are issued back to back, and a parity wait
                             // must never fall two phases behind)
-  uint64_t p_full;   // P of the current key tile in TMEM (and O rescaled if needed)
-  uint64_t o_ready;  // a PV completed (in issue order)
-  uint64_t o_free;   // epilogue finished reading O
+  uint64_t p_full[2];   // P of key tile i in TMEM (and O rescaled if needed): p_full[i & 1],
+                        // phase i >> 1.  The softmax may run two tiles ahead of the MMA warp
+                        // (S(i) is issued only after P(i-2) was taken), never more.
+  uint64_t o_ready[2];  // PV number i (counted over the CTA's life) completed: o_ready[i & 1],
+                        // phase i >> 1.  Two barriers, so that consumers may skip PVs they
+                        // do not need and still wait on an exact phase.
+  uint64_t o_free;      // epilogue finished reading O
   uint64_t drain;
-  int2 item_slot[2];
+  int4 item_slot[2];    // {segment * g + j, query tile, seg_offsets[segment], n}
   uint32_t tmem_base;
   int abort_flag;
 };
+
+static_assert(sizeof(Bars) <= 512, "barrier block");
 
 struct Params {
   const int32_t* seg_offsets;  // [nseg + 1]
@@ -110,13 +116,15 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
 }
 
 // Consumer side of the item ring: every lane waits, reads the item, one lane releases the slot.
-__device__ __forceinline__ bool take_item(Bars* bars, uint32_t idx, int2* item, volatile int* abort_flag,
+__device__ __forceinline__ bool take_item(Bars* bars, uint32_t idx, int4* item, volatile int* abort_flag,
                                           uint32_t* status) {
   const int slot = idx & 1;
   if (!warp_wait(&bars->item_full[slot], (idx >> 1) & 1, abort_flag, status)) return false;
   const volatile int* src = reinterpret_cast<const volatile int*>(&bars->item_slot[slot]);
   item->x = src[0];
   item->y = src[1];
+  item->z = src[2];
+  item->w = src[3];
   __syncwarp();
   if ((threadIdx.x & 31) == 0) mbar_arrive(&bars->item_empty[slot]);
   return true;
@@ -149,8 +157,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&bars->q_full, 1);
     mbar_init(&bars->q_empty, 1);
     for (int i = 0; i < kSBufs; ++i) mbar_init(&bars->s_full[i], 1);
-    mbar_init(&bars->p_full, kSoftmaxWarps);
-    mbar_init(&bars->o_ready, 1);
+    mbar_init(&bars->p_full[0], kSoftmaxWarps);
+    mbar_init(&bars->p_full[1], kSoftmaxWarps);
+    mbar_init(&bars->o_ready[0], 1);
+    mbar_init(&bars->o_ready[1], 1);
     mbar_init(&bars->o_free, kSoftmaxWarps);
     mbar_init(&bars->drain, 1);
     bars->abort_flag = 0;
@@ -188,16 +198,24 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       while (ok) {
         const int it = atomicAdd(p.sched, 1);
-        const int2 item = it < nitems ? p.items[it] : make_int2(-1, -1);
+        // the segment's offsets travel with the item, so no consumer loads them
+        int4 item = make_int4(-1, -1, 0, 0);
+        int kvb = 0;
+        if (it < nitems) {
+          const int2 w = p.items[it];
+          const int sg = w.x / p.g;
+          const int o = p.seg_offsets[sg];
+          item = make_int4(w.x, w.y, o, p.seg_offsets[sg + 1] - o);
+          kvb = (int)(p.seg_base ? p.seg_base[sg] : (long long)o);
+        }
         const int slot = item_iter & 1;
         if (item_iter >= 2) ok = mbar_wait(&bars->item_empty[slot], ((item_iter >> 1) - 1) & 1, abort_flag, p.status);
         if (!ok) break;
         bars->item_slot[slot] = item;
         mbar_arrive(&bars->item_full[slot]);
         if (item.x < 0) break;
-        const int seg = item.x / p.g, j = item.x % p.g, qt = item.y;
-        const int off = p.seg_offsets[seg];
-        const int kvb = (int)(p.seg_base ? p.seg_base[seg] : (long long)off);
+        const int j = item.x % p.g, qt = item.y;
+        const int off = item.z;
         const int nkv = qt + 1;
         if (item_iter > 0) ok = mbar_wait(&bars->q_empty, (item_iter - 1) & 1, abort_flag, p.status);
         if (!ok) break;
@@ -226,39 +244,34 @@ __global__ void __launch_bounds__(kThreads, 1)
     // different accumulators overlap.  With three S/P buffers, PV(kv) (A = P from TMEM)
     // and S(kv+2) (into the buffer PV(kv-1) finished with) are independent, and are
     // issued interleaved instruction by instruction while the softmax works on S(kv+1).
+    // The MMA queue is shallow: issuing a burst blocks until most of it has executed, so
+    // whatever runs between two bursts leaves the tensor pipe idle.  The warp therefore
+    // runs converged (one elected lane issues; descriptors are warp-uniform bases plus
+    // constant offsets), the next step's K/V waits sit in the middle of the current
+    // burst, and only P(kv+1) is waited between bursts (a softmax that rescales O waits
+    // for PV(kv), so P(kv+1) cannot be required earlier).
     constexpr uint32_t idesc_qk = make_idesc_bf16(BM, BN, false, false);
     constexpr uint32_t idesc_pv = make_idesc_bf16(BM, D, false, true);
-    const uint32_t q_addr = smem_u32(smem + L::kQ);
+    const uint64_t q_desc = make_smem_desc_sw128(smem_u32(smem + L::kQ), 16, 1024);
+    // descriptor offsets (16-byte units) of the K-extent steps: S walks the 128-byte swizzle
+    // atom 32 bytes at a time, then the next 64-column atom; PV walks 16 keys = 2048 bytes
+    auto qk_off = [](int kk) -> uint64_t { return (uint64_t)(((kk >> 2) * L::kAtomBytes + (kk & 3) * 32) >> 4); };
+    auto pv_off = [](int kk) -> uint64_t { return (uint64_t)((kk * 2048) >> 4); };
     uint32_t ring_iter = 0, item_iter = 0, s_iter = 0, p_iter = 0;
     bool ok = true;
     auto slot_addr = [&](uint32_t r) { return smem_u32(smem + L::kRing0 + (r % kRing) * L::kTileBytes); };
-    auto wait_ring = [&](uint32_t r) {
+    auto ring_ready = [&](uint32_t r) {
       return warp_wait(&bars->ring_full[r % kRing], (r / kRing) & 1, abort_flag, p.status);
     };
-    // S into buffer s_iter % 3 from ring entry r_k (alone, not interleaved)
-    auto issue_s_alone = [&](uint32_t r_k) {
-      const uint32_t k_addr = slot_addr(r_k);
-      const uint32_t d = tmem + tmem_s_col(s_iter % kSBufs);
-      if (lane == 0) {
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * L::kAtomBytes + (kk & 3) * 32;
-          mma_bf16_ss(d, make_smem_desc_sw128(q_addr + off, 16, 1024), make_smem_desc_sw128(k_addr + off, 16, 1024),
-                      idesc_qk, kk > 0 ? 1u : 0u);
-        }
-        mma_commit(&bars->s_full[s_iter % kSBufs]);
-        mma_commit(&bars->ring_empty[r_k % kRing]);
-      }
-      __syncwarp();
-      ++s_iter;
+    auto p_ready = [&](uint32_t i) {  // P of tile number i
+      return warp_wait(&bars->p_full[i & 1], (i >> 1) & 1, abort_flag, p.status);
     };
 
     while (ok) {
-      int2 item;
+      int4 item;
       ok = take_item(bars, item_iter, &item, abort_flag, p.status);
       if (!ok || item.x < 0) break;
-      const int seg = item.x / p.g, qt = item.y;
-      const int n = p.seg_offsets[seg + 1] - p.seg_offsets[seg];
+      const int qt = item.y, n = item.w;
       const int nkv = qt + 1;
       // ring entries of this item, in load order: K(0), K(1) if nkv > 1, then for each kv:
       // V(kv) followed by K(kv+2) while kv + 2 < nkv
@@ -268,77 +281,83 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto rv = [&](int kv) -> uint32_t { return kv < m ? base + 2u * kv : base + 2u * m + (kv - m); };
       auto rk = [&](int kv) -> uint32_t { return base + 2u * (kv - 2) + 1u; };  // K(kv), kv >= 2
 
-      ok = warp_wait(&bars->q_full, item_iter & 1, abort_flag, p.status);
-      if (ok) ok = wait_ring(rk0);
+      // prologue: S(0) and S(1) interleaved (independent buffers), then PV(0)'s operands
+      ok = warp_wait(&bars->q_full, item_iter & 1, abort_flag, p.status) && ring_ready(rk0) &&
+           (nkv == 1 || ring_ready(rk1));
       if (!ok) break;
       tc_fence_after();
-      issue_s_alone(rk0);
-      if (nkv > 1) {
-        ok = wait_ring(rk1);
-        if (!ok) break;
-        tc_fence_after();
-        issue_s_alone(rk1);
+      {
+        const uint32_t s0 = tmem + tmem_s_col((int)(s_iter % kSBufs));
+        const uint32_t s1 = tmem + tmem_s_col((int)((s_iter + 1) % kSBufs));
+        const uint64_t k0 = make_smem_desc_sw128(slot_addr(rk0), 16, 1024);
+        const uint64_t k1 = make_smem_desc_sw128(slot_addr(rk1), 16, 1024);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          mma_bf16_ss(s0, q_desc + qk_off(kk), k0 + qk_off(kk), idesc_qk, kk > 0 ? 1u : 0u);
+          if (nkv > 1) mma_bf16_ss(s1, q_desc + qk_off(kk), k1 + qk_off(kk), idesc_qk, kk > 0 ? 1u : 0u);
+        }
+        mma_commit(&bars->s_full[s_iter % kSBufs]);
+        mma_commit(&bars->ring_empty[rk0 % kRing]);
+        if (nkv > 1) {
+          mma_commit(&bars->s_full[(s_iter + 1) % kSBufs]);
+          mma_commit(&bars->ring_empty[rk1 % kRing]);
+        }
+        if (nkv <= 2) mma_commit(&bars->q_empty);  // every S of this item issued
       }
-      if (lane == 0 && nkv <= 2) mma_commit(&bars->q_empty);  // every S of this item issued
-      __syncwarp();
+      s_iter += nkv > 1 ? 2u : 1u;
+      ok = ring_ready(rv(0)) && (nkv <= 2 || ring_ready(rk(2))) &&
+           (item_iter == 0 || warp_wait(&bars->o_free, (item_iter - 1) & 1, abort_flag, p.status)) && p_ready(p_iter);
+      if (!ok) break;
 
-      for (int kv = 0; kv < nkv && ok; ++kv) {
-        // PV(kv) needs P(kv); S(kv+2) needs K(kv+2) and the buffer PV(kv-1) read from
-        ok = warp_wait(&bars->p_full, p_iter & 1, abort_flag, p.status);
-        ++p_iter;
+      for (int kv = 0; kv < nkv; ++kv) {
+        // here V(kv), K(kv+2), a free O and P(kv) are all in place
         const uint32_t r_v = rv(kv);
-        if (ok) ok = wait_ring(r_v);
-        if (ok && kv == 0 && item_iter > 0) ok = warp_wait(&bars->o_free, (item_iter - 1) & 1, abort_flag, p.status);
         const bool with_s = kv + 2 < nkv;
-        const uint32_t r_k2 = with_s ? rk(kv + 2) : 0;
-        if (ok && with_s) ok = wait_ring(r_k2);
-        if (!ok) break;
+        const bool has_next = kv + 1 < nkv;
+        const uint32_t r_k2 = with_s ? rk(kv + 2) : r_v;
+        const uint32_t pv_index = p_iter++;
         const int valid_keys = n - kv * BN;  // keys of this tile inside the segment
         if (valid_keys < BN) {
           // rows past the segment end may hold anything (other segments, unwritten cache
           // rows): zero them so that 0-weight columns of P cannot meet NaN in V
           uint8_t* vtile = smem + L::kRing0 + (r_v % kRing) * L::kTileBytes;
           for (int a = 0; a < L::kAtoms; ++a) {
-            uint4* base = reinterpret_cast<uint4*>(vtile + a * L::kAtomBytes);
-            for (int i = valid_keys * 8 + lane; i < BN * 8; i += 32) base[i] = make_uint4(0, 0, 0, 0);
+            uint4* vb = reinterpret_cast<uint4*>(vtile + a * L::kAtomBytes);
+            for (int i = valid_keys * 8 + lane; i < BN * 8; i += 32) vb[i] = make_uint4(0, 0, 0, 0);
           }
           fence_proxy_async_smem();
           __syncwarp();
         }
         tc_fence_after();
-        if (lane == 0) {
-          // P(kv) sits in the buffer of S(kv): S and P are counted alike across items
-          const uint32_t pbuf = tmem + tmem_s_col((int)((p_iter - 1) % kSBufs));
-          const uint32_t sbuf = tmem + tmem_s_col((int)(s_iter % kSBufs));
-          const uint32_t v_addr = slot_addr(r_v);
-          const uint32_t k_addr = with_s ? slot_addr(r_k2) : 0;
+        // P(kv) sits in the buffer of S(kv): S and P are counted alike across items
+        const uint32_t pbuf = tmem + tmem_s_col((int)(pv_index % kSBufs));
+        const uint32_t sbuf = tmem + tmem_s_col((int)(s_iter % kSBufs));
+        const uint64_t v_desc = make_smem_desc_sw128(slot_addr(r_v), L::kAtomBytes, 1024);
+        const uint64_t k_desc = make_smem_desc_sw128(slot_addr(r_k2), 16, 1024);
 #pragma unroll
-          for (int kk = 0; kk < 8; ++kk) {
-            // PV: K extent = BN keys, 16 per instruction (8 instructions)
-            mma_bf16_ts(tmem + kTmemO, pbuf + kk * 8, make_smem_desc_sw128(v_addr + kk * 2048, L::kAtomBytes, 1024),
-                        idesc_pv, (kv > 0 || kk > 0) ? 1u : 0u);
-            // S: K extent = D, 16 per instruction (D / 16 instructions)
-            if (with_s && kk < D / 16) {
-              const uint32_t off = (kk >> 2) * L::kAtomBytes + (kk & 3) * 32;
-              mma_bf16_ss(sbuf, make_smem_desc_sw128(q_addr + off, 16, 1024),
-                          make_smem_desc_sw128(k_addr + off, 16, 1024), idesc_qk, kk > 0 ? 1u : 0u);
-            }
-          }
-          mma_commit(&bars->o_ready);
-          mma_commit(&bars->ring_empty[r_v % kRing]);
-          if (with_s) {
-            mma_commit(&bars->s_full[s_iter % kSBufs]);
-            mma_commit(&bars->ring_empty[r_k2 % kRing]);
-            if (kv + 2 == nkv - 1) mma_commit(&bars->q_empty);
-          }
+        for (int kk = 0; kk < 8; ++kk) {
+          // PV: K extent = BN keys, 16 per instruction (8 instructions)
+          mma_bf16_ts(tmem + kTmemO, pbuf + kk * 8, v_desc + pv_off(kk), idesc_pv, (kv > 0 || kk > 0) ? 1u : 0u);
+          // S: K extent = D, 16 per instruction (D / 16 instructions)
+          if (with_s && kk < D / 16) mma_bf16_ss(sbuf, q_desc + qk_off(kk), k_desc + qk_off(kk), idesc_qk, kk > 0 ? 1u : 0u);
+          // the next step's K/V, while the queue holds this burst's instructions
+          if (kk == 3 && has_next) ok = ring_ready(rv(kv + 1)) && (kv + 3 >= nkv || ring_ready(rk(kv + 3)));
         }
-        __syncwarp();
-        if (with_s) ++s_iter;
+        mma_commit(&bars->o_ready[pv_index & 1]);
+        mma_commit(&bars->ring_empty[r_v % kRing]);
+        if (with_s) {
+          mma_commit(&bars->s_full[s_iter % kSBufs]);
+          mma_commit(&bars->ring_empty[r_k2 % kRing]);
+          if (kv + 2 == nkv - 1) mma_commit(&bars->q_empty);
+          ++s_iter;
+        }
+        if (ok && has_next) ok = p_ready(p_iter);
+        if (!ok) break;
       }
       ring_iter += 2 * nkv;
       ++item_iter;
     }
-    if (!ok && lane == 0) {
+    if (!ok) {
       // wait (bounded) for MMAs already issued before TMEM is released
       mma_commit(&bars->drain);
       const uint64_t t0 = global_timer_ns();
@@ -351,31 +370,30 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int row = warp * 32 + lane;  // query row within the tile (warp w reads TMEM lanes 32w..32w+31)
     const uint32_t lane_addr = (uint32_t)(warp * 32) << 16;
     const uint32_t o_addr = tmem + lane_addr + kTmemO;
-    uint32_t s_iter = 0, o_iter = 0, item_iter = 0;
+    // s_iter counts key tiles over the CTA's life; tile i's S, P and PV all carry number i.
+    uint32_t s_iter = 0, item_iter = 0;
     bool ok = true;
+    // Waits for PV number i.  Exact whenever PV i-2 is known complete and PV i+2 is not yet
+    // issued: true inside the softmax of tile i+1 (its S was committed after PV i-1) and in
+    // the epilogue of an item whose last tile is i.
+    auto wait_pv = [&](uint32_t i) { return warp_wait(&bars->o_ready[i & 1], (i >> 1) & 1, abort_flag, p.status); };
     while (ok) {
-      int2 item;
+      int4 item;
       ok = take_item(bars, item_iter, &item, abort_flag, p.status);
       ++item_iter;
       if (!ok || item.x < 0) break;
-      const int seg = item.x / p.g, j = item.x % p.g, qt = item.y;
-      const int off = p.seg_offsets[seg];
-      const int n = p.seg_offsets[seg + 1] - off;
-      // epilogue operands now, so that their latency hides behind the item
+      const int j = item.x % p.g, qt = item.y, off = item.z, n = item.w;
+      // the output row now (its latency hides behind the first tile); the gate after it
       const int qrank = qt * BM + row;
       const bool valid = qrank < n;
-      long long dst_row = 0;
+      int src = 0;
+      if (valid) src = p.row_src[off + qrank];
       float gt = 0.f;
-      if (valid) {
-        const int src = p.row_src[off + qrank];
-        dst_row = (long long)src * p.g + j;
-        gt = p.gate[src];
-      }
       float m_use = 0.f, l_sum = 0.f;
       for (int kv = 0; kv <= qt && ok; ++kv) {
         const uint32_t s_addr = tmem + lane_addr + tmem_s_col((int)(s_iter % kSBufs));
         ok = warp_wait(&bars->s_full[s_iter % kSBufs], (s_iter / kSBufs) & 1, abort_flag, p.status);
-        ++s_iter;
+        const uint32_t tile = s_iter++;
         if (!ok) break;
         tc_fence_after();
         float sv[BN];
@@ -430,13 +448,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int i = 0; i < 32; ++i) r[i] = pk[32 + i];
           tmem_st32(s_addr + 32, r);
         }
-        // O may only be rescaled once the previous PV completed
-        if (kv > 0) {
-          ok = warp_wait(&bars->o_ready, o_iter & 1, abort_flag, p.status);
-          ++o_iter;
+        // O may only be rescaled once the previous PV completed; without a rescale this
+        // tile's softmax does not touch O and overlaps that PV
+        if (kv > 0 && __any_sync(0xffffffffu, rescale)) {
+          ok = wait_pv(tile - 1);
           if (!ok) break;
           tc_fence_after();
-          if (__any_sync(0xffffffffu, rescale)) {
+          {
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
               uint32_t r[32];
@@ -451,31 +469,29 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_wait_st();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&bars->p_full);
+        if (lane == 0) mbar_arrive(&bars->p_full[tile & 1]);
+        if (kv == 0 && valid) gt = p.gate[src];  // used in the epilogue only
       }
       if (!ok) break;
-      // epilogue: O / l * gate -> y[row_src]
-      ok = warp_wait(&bars->o_ready, o_iter & 1, abort_flag, p.status);
-      ++o_iter;
+      // epilogue: O / l * gate -> y[row_src * g + j]
+      ok = wait_pv(s_iter - 1);
       if (!ok) break;
       tc_fence_after();
       const float scale = valid ? gt / l_sum : 0.f;
+      uint32_t o[D / 32][32];
 #pragma unroll
-      for (int c = 0; c < D / 32; ++c) {
-        uint32_t r[32];
-        tmem_ld32(o_addr + c * 32, r);
-        tmem_wait_ld();
-        if (valid) {
-          uint4* dst = reinterpret_cast<uint4*>(p.y + dst_row * D + c * 32);
+      for (int c = 0; c < D / 32; ++c) tmem_ld32(o_addr + c * 32, o[c]);
+      tmem_wait_ld();
+      if (valid) {
+        uint4* dst = reinterpret_cast<uint4*>(p.y + ((long long)src * p.g + j) * D);
 #pragma unroll
-          for (int q4 = 0; q4 < 4; ++q4) {
-            uint32_t w[4];
+        for (int q4 = 0; q4 < D / 8; ++q4) {
+          uint32_t w[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e)
-              w[e] = pack_bf16x2(__uint_as_float(r[q4 * 8 + 2 * e]) * scale,
-                                 __uint_as_float(r[q4 * 8 + 2 * e + 1]) * scale);
-            dst[q4] = make_uint4(w[0], w[1], w[2], w[3]);
-          }
+          for (int e = 0; e < 4; ++e)
+            w[e] = pack_bf16x2(__uint_as_float(o[q4 / 4][(q4 % 4) * 8 + 2 * e]) * scale,
+                               __uint_as_float(o[q4 / 4][(q4 % 4) * 8 + 2 * e + 1]) * scale);
+          dst[q4] = make_uint4(w[0], w[1], w[2], w[3]);
         }
       }
       tc_fence_before();
