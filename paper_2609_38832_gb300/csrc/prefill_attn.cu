@@ -18,8 +18,10 @@
 //   warps 0-3   softmax / epilogue: thread i owns query row i (TMEM lane i).  Online
 //               softmax in fp32 with exp2; the running max only moves when it grows by
 //               more than 2^8 (O in TMEM is then rescaled).  P is written back to TMEM as
-//               bf16 over the S columns it came from.  The epilogue divides by the row
-//               sum, multiplies by the routing gate and scatters bf16 rows to y[row_src].
+//               bf16 over the S columns it came from.  The epilogue reads O out of TMEM
+//               (freeing it for the next item at once), divides by the row sum, multiplies
+//               by the routing gate and writes bf16 rows to y[row_src], a 32-byte sector per
+//               store.
 //   warp 4      TMA producer: the Q tile, then K(0), K(1), V(0), K(2), V(1), ... through a
 //               6-slot ring (128B swizzle) two key tiles ahead of the MMAs.
 //   warp 5      MMA issuer (one lane) and TMEM owner.  tcgen05.mma instructions into one
@@ -104,6 +106,7 @@ struct Params {
   int* sched;                  // [0] next item, [1] CTAs finished
   uint16_t* y;                 // [R * g, D] indexed by row_src * g + j
   int g;
+  int y_sector_aligned;        // y is 32-byte aligned: rows go out as whole 32-byte sectors
   float scale_log2;            // log2(e) / sqrt(D)
   uint32_t* status;
 };
@@ -473,30 +476,35 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (kv == 0 && valid) gt = p.gate[src];  // used in the epilogue only
       }
       if (!ok) break;
-      // epilogue: O / l * gate -> y[row_src * g + j]
+      // epilogue: O out of TMEM (O is then free for the next item), O / l * gate as bf16
+      // to y[row_src * g + j], 32 bytes (one whole sector) per store where y allows it
       ok = wait_pv(s_iter - 1);
       if (!ok) break;
       tc_fence_after();
-      const float scale = valid ? gt / l_sum : 0.f;
       uint32_t o[D / 32][32];
 #pragma unroll
       for (int c = 0; c < D / 32; ++c) tmem_ld32(o_addr + c * 32, o[c]);
       tmem_wait_ld();
-      if (valid) {
-        uint4* dst = reinterpret_cast<uint4*>(p.y + ((long long)src * p.g + j) * D);
-#pragma unroll
-        for (int q4 = 0; q4 < D / 8; ++q4) {
-          uint32_t w[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e)
-            w[e] = pack_bf16x2(__uint_as_float(o[q4 / 4][(q4 % 4) * 8 + 2 * e]) * scale,
-                               __uint_as_float(o[q4 / 4][(q4 % 4) * 8 + 2 * e + 1]) * scale);
-          dst[q4] = make_uint4(w[0], w[1], w[2], w[3]);
-        }
-      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars->o_free);
+      if (valid) {
+        const float scale = gt / l_sum;
+        uint32_t w[D / 2];
+#pragma unroll
+        for (int e = 0; e < D / 2; ++e)
+          w[e] = pack_bf16x2(__uint_as_float(o[e / 16][(e % 16) * 2]) * scale,
+                             __uint_as_float(o[e / 16][(e % 16) * 2 + 1]) * scale);
+        uint16_t* dst = p.y + ((long long)src * p.g + j) * D;
+        if (p.y_sector_aligned) {
+#pragma unroll
+          for (int c = 0; c < D / 16; ++c) st_global_v8(dst + c * 16, w + c * 8);
+        } else {
+#pragma unroll
+          for (int c = 0; c < D / 8; ++c)
+            *reinterpret_cast<uint4*>(dst + c * 8) = make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
+        }
+      }
     }
   }
 
@@ -642,6 +650,7 @@ int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint1
   p.items = reinterpret_cast<const int2*>(static_cast<char*>(plan) + 16);
   p.y = y;
   p.g = g;
+  p.y_sector_aligned = (reinterpret_cast<uintptr_t>(y) & 31u) == 0;
   p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)D));
   p.status = dev_status;
   const cudaError_t e = (D == 128) ? attn::launch_attn<128>(tq, tk, tv, p, info.sm_count, stream)

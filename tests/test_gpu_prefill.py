@@ -167,3 +167,23 @@ def test_staged_calls_match_prefill(namoh, wl):
         torch.cuda.synchronize()
         assert torch.equal(y.view(torch.int16), y_ref.view(torch.int16)), f"fused plan = {fused}"
     assert int(ro.status.item()) == 0
+
+
+def test_attention_output_not_sector_aligned(namoh):
+    """y only 16-byte aligned (not 32): rows take the 16-byte store path, same bytes."""
+    wl = ni.PrefillWorkload("y_offset", B=2, T=600, H=8, K=2, d=128, seed=13)
+    scores = wl.scores()
+    q, k, v = (dev_bf16(a) for a in wl.qkv())
+    ro = namoh.namoh_route(torch.from_numpy(scores).cuda(), wl.Kr)
+    kw = dict(B=wl.B, T=wl.T, H=wl.H, K=wl.K, group=wl.g)
+    y_ref, _, _ = namoh.namoh_prefill(q, k, v, ro.seg_offsets, ro.row_src, ro.gate, rope_base=wl.base,
+                                      status=ro.status, **kw)
+    numel = wl.B * wl.T * wl.K * wl.d
+    big = torch.empty(numel + 8, dtype=torch.bfloat16, device="cuda")
+    y_off = big[8:].view(wl.B, wl.T, wl.K, wl.d)
+    assert y_off.data_ptr() % 32 == 16
+    y, _, _ = namoh.namoh_prefill(q, k, v, ro.seg_offsets, ro.row_src, ro.gate, rope_base=wl.base, y=y_off,
+                                  status=ro.status, **kw)
+    torch.cuda.synchronize()
+    assert torch.equal(y.view(torch.int16), y_ref.view(torch.int16))
+    assert int(ro.status.item()) == 0
