@@ -102,9 +102,17 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // Bounded wait.  `abort_flag` (shared memory) lets one role that gave up stop the
 // others: once it is set every wait returns false immediately.  Returns true when
 // the phase with the given parity completed.
+static __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                            uint32_t* status);
+// The first try is inline; the polling loop and the timeout report stay out of line, so that
+// the many waits of a pipeline loop keep its code small.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
                                           uint32_t* status) {
   if (mbar_try_wait(bar, parity)) return true;
+  return mbar_wait_slow(bar, parity, abort_flag, status);
+}
+static __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                            uint32_t* status) {
   const uint64_t t0 = global_timer_ns();
   while (true) {
     if (*abort_flag) return false;
