@@ -337,14 +337,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t sbuf = tmem + tmem_s_col((int)(s_iter % kSBufs));
         const uint64_t v_desc = make_smem_desc_sw128(slot_addr(r_v), L::kAtomBytes, 1024);
         const uint64_t k_desc = make_smem_desc_sw128(slot_addr(r_k2), 16, 1024);
+        // the next step's ring entries, computed before the burst so that the burst itself is
+        // straight-line code (one variant with S(kv+2), one without)
+        const uint32_t r_vn = has_next ? rv(kv + 1) : r_v;
+        const bool next_k = kv + 3 < nkv;
+        const uint32_t r_kn = next_k ? rk(kv + 3) : r_v;
+        const uint32_t acc0 = kv > 0 ? 1u : 0u;
+        if (with_s) {
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          // PV: K extent = BN keys, 16 per instruction (8 instructions)
-          mma_bf16_ts(tmem + kTmemO, pbuf + kk * 8, v_desc + pv_off(kk), idesc_pv, (kv > 0 || kk > 0) ? 1u : 0u);
-          // S: K extent = D, 16 per instruction (D / 16 instructions)
-          if (with_s && kk < D / 16) mma_bf16_ss(sbuf, q_desc + qk_off(kk), k_desc + qk_off(kk), idesc_qk, kk > 0 ? 1u : 0u);
-          // the next step's K/V, while the queue holds this burst's instructions
-          if (kk == 3 && has_next) ok = ring_ready(rv(kv + 1)) && (kv + 3 >= nkv || ring_ready(rk(kv + 3)));
+          for (int kk = 0; kk < 8; ++kk) {
+            // PV: K extent = BN keys, 16 per instruction; S: K extent = D, 16 per instruction
+            mma_bf16_ts(tmem + kTmemO, pbuf + kk * 8, v_desc + pv_off(kk), idesc_pv, kk > 0 ? 1u : acc0);
+            if (kk < D / 16) mma_bf16_ss(sbuf, q_desc + qk_off(kk), k_desc + qk_off(kk), idesc_qk, kk > 0 ? 1u : 0u);
+            // the next step's K/V, while the queue holds this burst's instructions
+            if (kk == 3 && has_next) ok = ring_ready(r_vn) && (!next_k || ring_ready(r_kn));
+          }
+        } else {
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) {
+            mma_bf16_ts(tmem + kTmemO, pbuf + kk * 8, v_desc + pv_off(kk), idesc_pv, kk > 0 ? 1u : acc0);
+            if (kk == 3 && has_next) ok = ring_ready(r_vn);
+          }
         }
         mma_commit(&bars->o_ready[pv_index & 1]);
         mma_commit(&bars->ring_empty[r_v % kRing]);

@@ -1,141 +1,213 @@
 // rope_pack.cu -- head-relative RoPE at the packed rank (Sec. 3.2, Eq. namoh-head-rope).
 //
-// One group of D/16 threads per packed row r: the row's segment s is found by binary
-// search over seg_offsets, rho = r - seg_offsets[s].  Each thread owns 8 rotation pairs
-// (j, j + D/2) and moves them with 16-byte loads/stores.  The angle is computed once per
-// row and applied to K and to all g query heads of the row (KV-group routing shares the
-// rank, App. C).  Outputs: Q~ (bf16 scratch for the attention kernel), K~ into the key
-// cache, and V copied into the value cache unless the caller passed v_cache == v.  When
-// given a plan buffer, one extra block builds the attention work list in the same launch.
+// Packed rows are contiguous in q, k and v, so each block streams chunks of packed rows
+// (their g query rows, the key row and, when it is copied, the value row) into shared
+// memory with 1D bulk copies through a kRopeStages-deep mbarrier pipeline, and rotates them
+// from there: the loads of several chunks are in flight at any time, with no per-thread
+// load latency on the way.  A group of D/16 threads owns one packed row of a chunk (for
+// g >= 4, half of its query heads or less): the row's segment s comes from a binary search
+// over seg_offsets (staged in shared memory), rho = r - seg_offsets[s], and each thread
+// rotates 8 pairs (j, j + D/2) with angles it computes once for the row; KV-group routing
+// shares the rank between the key and the row's g query heads (App. C).
+// Outputs: Q~ (bf16 scratch for the attention kernel), K~ into the key cache, and V copied
+// into the value cache unless the caller passed v_cache == v.  Given a plan buffer, block 0
+// builds the attention work list in the same launch.
 #include "common.cuh"
 #include "plan.cuh"
 
 namespace namoh {
 
+constexpr int kRopeThreads = 256;
+constexpr int kRopeStages = 3;
 constexpr int kRopeStageMax = 8192;  // seg_offsets entries staged in shared memory (32 KB)
 
-// With a plan header given, block 0 builds the attention work list (it depends only on
-// seg_offsets) while the other blocks rotate rows; it goes first so that it is resident in
-// the first wave.
 template <int D, int G>
-__global__ void __launch_bounds__(256) rope_pack_kernel(const uint16_t* __restrict__ q, const uint16_t* __restrict__ k,
-                                                        const uint16_t* __restrict__ v, int R,
-                                                        const int32_t* __restrict__ seg_offsets, int nseg,
-                                                        const int64_t* __restrict__ seg_base,
-                                                        const int32_t* __restrict__ seg_cap, long long cache_rows,
-                                                        uint16_t* __restrict__ q_rot, uint16_t* __restrict__ k_cache,
-                                                        uint16_t* __restrict__ v_cache, int copy_v, RopeTable tab,
-                                                        uint32_t* __restrict__ status, int* __restrict__ plan_header,
-                                                        int2* __restrict__ plan_items, const int32_t* __restrict__ plan_cap,
-                                                        int plan_qtiles) {
-  constexpr int LPR = D / 16;  // threads per row
+struct RopeChunk {
+  static constexpr int kLpr = D / 16;                    // threads per group (8 pairs each)
+  static constexpr int kGroups = kRopeThreads / kLpr;    // 32 (D = 128) or 64 (D = 64)
+  static constexpr int kGpr = G >= 4 ? G / 2 : 1;        // groups per packed row
+  static constexpr int kHeads = G / kGpr;                // query heads per group
+  static constexpr int kRows = kGroups / kGpr;           // packed rows per chunk
+  static constexpr int kQBytes = kRows * G * D * 2;
+  static constexpr int kKBytes = kRows * D * 2;
+  static constexpr int kStageBytes = kQBytes + 2 * kKBytes;  // Q, K, V
+  static_assert(kStageBytes % 128 == 0, "stage alignment");
+};
+
+__host__ __device__ constexpr size_t rope_offs_bytes(int nseg) {
+  return nseg + 1 <= kRopeStageMax ? ((size_t)(nseg + 1) * 4 + 15) / 16 * 16 : 0;
+}
+
+template <int D, int G>
+__host__ __device__ constexpr size_t rope_smem_bytes(int nseg) {
+  return (size_t)kRopeStages * RopeChunk<D, G>::kStageBytes + rope_offs_bytes(nseg) + kRopeStages * sizeof(uint64_t);
+}
+
+template <int D, int G>
+__global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
+    const uint16_t* __restrict__ q, const uint16_t* __restrict__ k, const uint16_t* __restrict__ v, int R,
+    const int32_t* __restrict__ seg_offsets, int nseg, const int64_t* __restrict__ seg_base,
+    const int32_t* __restrict__ seg_cap, long long cache_rows, uint16_t* __restrict__ q_rot,
+    uint16_t* __restrict__ k_cache, uint16_t* __restrict__ v_cache, int copy_v, RopeTable tab,
+    uint32_t* __restrict__ status, int* __restrict__ plan_header, int2* __restrict__ plan_items,
+    const int32_t* __restrict__ plan_cap, int plan_qtiles) {
+  using C = RopeChunk<D, G>;
   constexpr int HALF = D / 2;
-  extern __shared__ int32_t s_dyn[];
+  extern __shared__ __align__(128) uint8_t smem_raw[];
+  __shared__ int s_abort;
   const int first = plan_header ? 1 : 0;
   if ((int)blockIdx.x < first) {
-    build_plan(seg_offsets, nseg, plan_cap, G, plan_qtiles, plan_header, plan_items, s_dyn);
+    build_plan(seg_offsets, nseg, plan_cap, G, plan_qtiles, plan_header, plan_items, reinterpret_cast<int*>(smem_raw));
     return;
   }
-  const int rope_blocks = gridDim.x - first;
-  const int block = blockIdx.x - first;
-  const bool staged = (nseg + 1) <= kRopeStageMax;
-  if (staged) {
-    for (int i = threadIdx.x; i <= nseg; i += blockDim.x) s_dyn[i] = __ldg(seg_offsets + i);
-    __syncthreads();
+  const int nblk = gridDim.x - first, blk = blockIdx.x - first;
+  const int nchunks = (R + C::kRows - 1) / C::kRows;
+  uint8_t* stages = smem_raw;
+  int32_t* s_offs = reinterpret_cast<int32_t*>(smem_raw + kRopeStages * C::kStageBytes);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + kRopeStages * C::kStageBytes + rope_offs_bytes(nseg));
+  const bool staged = nseg + 1 <= kRopeStageMax;
+
+  // chunk c into stage st: its rows' Q (g rows each), K and V, one bulk copy per array
+  auto issue = [&](int c, int st) {
+    const int r0 = c * C::kRows;
+    const int rows = min(C::kRows, R - r0);
+    uint8_t* base = stages + st * C::kStageBytes;
+    const uint32_t qb = (uint32_t)rows * G * D * 2, kb = (uint32_t)rows * D * 2;
+    mbar_arrive_expect_tx(&full[st], qb + kb + (copy_v ? kb : 0u));
+    bulk_load(base, q + (size_t)r0 * G * D, qb, &full[st]);
+    bulk_load(base + C::kQBytes, k + (size_t)r0 * D, kb, &full[st]);
+    if (copy_v) bulk_load(base + C::kQBytes + C::kKBytes, v + (size_t)r0 * D, kb, &full[st]);
+  };
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kRopeStages; ++i) mbar_init(&full[i], 1);
+    s_abort = 0;
+    mbar_fence_init();
+    for (int i = 0; i < kRopeStages; ++i)
+      if (blk + i * nblk < nchunks) issue(blk + i * nblk, i);
   }
-  const int32_t* offs = staged ? s_dyn : seg_offsets;
-  const int lane_in_row = threadIdx.x % LPR;
-  const int j0 = lane_in_row * 8;
-  const long long groups = (long long)rope_blocks * (blockDim.x / LPR);
+  if (staged)
+    for (int i = threadIdx.x; i <= nseg; i += blockDim.x) s_offs[i] = __ldg(seg_offsets + i);
+  __syncthreads();
+  const int32_t* offs = staged ? s_offs : seg_offsets;
+
+  const int grp = threadIdx.x / C::kLpr, lig = threadIdx.x % C::kLpr;
+  const int prow = grp / C::kGpr;  // packed row within the chunk
+  const int hsub = grp % C::kGpr;  // which share of the row's query heads
+  const int j0 = lig * 8;
   float th_hi[8], th_lo[8];
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     th_hi[i] = tab.theta_hi[j0 + i];
     th_lo[i] = tab.theta_lo[j0 + i];
   }
-  for (long long r = (long long)block * (blockDim.x / LPR) + threadIdx.x / LPR; r < R; r += groups) {
-    // every load of this row first, so their latencies overlap
-    const uint4 ka = __ldg(reinterpret_cast<const uint4*>(k + (size_t)r * D + j0));
-    const uint4 kb = __ldg(reinterpret_cast<const uint4*>(k + (size_t)r * D + HALF + j0));
-    uint4 qa[G], qb[G];
-#pragma unroll
-    for (int j = 0; j < G; ++j) {
-      qa[j] = __ldg(reinterpret_cast<const uint4*>(q + ((size_t)r * G + j) * D + j0));
-      qb[j] = __ldg(reinterpret_cast<const uint4*>(q + ((size_t)r * G + j) * D + HALF + j0));
+  bool ok = true;
+  int it = 0;
+  for (int c = blk; c < nchunks; c += nblk, ++it) {
+    const int st = it % kRopeStages;
+    ok = mbar_wait(&full[st], (it / kRopeStages) & 1, &s_abort, status);
+    if (!__syncthreads_and(ok)) {
+      ok = false;
+      break;
     }
-    uint4 va = make_uint4(0, 0, 0, 0), vb = va;
-    if (copy_v) {
-      va = __ldg(reinterpret_cast<const uint4*>(v + (size_t)r * D) + lane_in_row);
-      vb = __ldg(reinterpret_cast<const uint4*>(v + (size_t)r * D) + lane_in_row + LPR);
-    }
-    // segment of row r: last s with seg_offsets[s] <= r
-    int lo = 0, hi = nseg;
-    while (hi - lo > 1) {
-      const int mid = (lo + hi) >> 1;
-      if (offs[mid] <= r) lo = mid; else hi = mid;
-    }
-    const int rho = (int)(r - offs[lo]);
-    long long dst = r;
-    bool write_cache = true;
-    if (seg_base) {
-      dst = __ldg(seg_base + lo) + rho;
-      if (rho >= __ldg(seg_cap + lo) || dst < 0 || dst >= cache_rows) {
-        write_cache = false;
-        if (lane_in_row == 0) report(status, NAMOH_DEV_CAPACITY);
+    const uint8_t* base = stages + st * C::kStageBytes;
+    const long long r = (long long)c * C::kRows + prow;
+    if (r < R) {
+      // segment of row r: last s with seg_offsets[s] <= r
+      int lo = 0, hi = nseg;
+      while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (offs[mid] <= r) lo = mid; else hi = mid;
       }
-    }
-    float sn[8], cs[8];
+      const int rho = (int)(r - offs[lo]);
+      float sn[8], cs[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) rope_sincos((float)rho, th_hi[i], th_lo[i], tab, &sn[i], &cs[i]);
+      for (int i = 0; i < 8; ++i) rope_sincos((float)rho, th_hi[i], th_lo[i], tab, &sn[i], &cs[i]);
 
-    // x'_j = x_j cos - x_{j+D/2} sin ;  x'_{j+D/2} = x_{j+D/2} cos + x_j sin
-    auto rotate = [&](const uint4& a, const uint4& b, uint16_t* dst_row) {
-      const uint32_t av[4] = {a.x, a.y, a.z, a.w};
-      const uint32_t bv[4] = {b.x, b.y, b.z, b.w};
-      uint32_t oa[4], ob[4];
+      // x'_j = x_j cos - x_{j+D/2} sin ;  x'_{j+D/2} = x_{j+D/2} cos + x_j sin
+      auto rotate = [&](const uint8_t* src_row, uint16_t* dst_row) {
+        const uint4 a = *reinterpret_cast<const uint4*>(src_row + j0 * 2);
+        const uint4 b = *reinterpret_cast<const uint4*>(src_row + (HALF + j0) * 2);
+        const uint32_t av[4] = {a.x, a.y, a.z, a.w};
+        const uint32_t bv[4] = {b.x, b.y, b.z, b.w};
+        uint32_t oa[4], ob[4];
 #pragma unroll
-      for (int p = 0; p < 4; ++p) {
-        const float x0 = bf16_lo(av[p]), x1 = bf16_hi(av[p]);
-        const float y0 = bf16_lo(bv[p]), y1 = bf16_hi(bv[p]);
-        const int i0 = 2 * p, i1 = 2 * p + 1;
-        oa[p] = pack_bf16x2(fmaf(x0, cs[i0], -y0 * sn[i0]), fmaf(x1, cs[i1], -y1 * sn[i1]));
-        ob[p] = pack_bf16x2(fmaf(y0, cs[i0], x0 * sn[i0]), fmaf(y1, cs[i1], x1 * sn[i1]));
-      }
-      *reinterpret_cast<uint4*>(dst_row + j0) = make_uint4(oa[0], oa[1], oa[2], oa[3]);
-      *reinterpret_cast<uint4*>(dst_row + HALF + j0) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
-    };
+        for (int p = 0; p < 4; ++p) {
+          const float x0 = bf16_lo(av[p]), x1 = bf16_hi(av[p]);
+          const float y0 = bf16_lo(bv[p]), y1 = bf16_hi(bv[p]);
+          const int i0 = 2 * p, i1 = 2 * p + 1;
+          oa[p] = pack_bf16x2(fmaf(x0, cs[i0], -y0 * sn[i0]), fmaf(x1, cs[i1], -y1 * sn[i1]));
+          ob[p] = pack_bf16x2(fmaf(y0, cs[i0], x0 * sn[i0]), fmaf(y1, cs[i1], x1 * sn[i1]));
+        }
+        *reinterpret_cast<uint4*>(dst_row + j0) = make_uint4(oa[0], oa[1], oa[2], oa[3]);
+        *reinterpret_cast<uint4*>(dst_row + HALF + j0) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
+      };
 #pragma unroll
-    for (int j = 0; j < G; ++j) rotate(qa[j], qb[j], q_rot + ((size_t)r * G + j) * D);
-    if (write_cache) {
-      rotate(ka, kb, k_cache + (size_t)dst * D);
-      if (copy_v) {
-        uint4* vd = reinterpret_cast<uint4*>(v_cache + (size_t)dst * D);
-        vd[lane_in_row] = va;
-        vd[lane_in_row + LPR] = vb;
+      for (int h = 0; h < C::kHeads; ++h) {
+        const int head = hsub * C::kHeads + h;
+        rotate(base + ((size_t)prow * G + head) * D * 2, q_rot + ((size_t)r * G + head) * D);
       }
+      if (hsub == 0) {
+        long long dst = r;
+        bool write_cache = true;
+        if (seg_base) {
+          dst = __ldg(seg_base + lo) + rho;
+          if (rho >= __ldg(seg_cap + lo) || dst < 0 || dst >= cache_rows) {
+            write_cache = false;
+            if (lig == 0) report(status, NAMOH_DEV_CAPACITY);
+          }
+        }
+        if (write_cache) {
+          rotate(base + C::kQBytes + (size_t)prow * D * 2, k_cache + (size_t)dst * D);
+          if (copy_v) {
+            const uint4* vs = reinterpret_cast<const uint4*>(base + C::kQBytes + C::kKBytes + (size_t)prow * D * 2);
+            uint4* vd = reinterpret_cast<uint4*>(v_cache + (size_t)dst * D);
+            vd[lig] = vs[lig];
+            vd[lig + C::kLpr] = vs[lig + C::kLpr];
+          }
+        }
+      }
+    }
+    __syncthreads();  // stage st fully read: refill it
+    if (threadIdx.x == 0 && c + kRopeStages * nblk < nchunks) issue(c + kRopeStages * nblk, st);
+  }
+  if (!ok && threadIdx.x == 0) {
+    // a wait gave up: let bulk copies still in flight land before the block exits
+    const uint64_t t0 = global_timer_ns();
+    while (global_timer_ns() - t0 < 1000000ull) {
     }
   }
 }
 
 template <int D>
-cudaError_t launch_rope_pack_d(int g, dim3 grid, size_t smem, cudaStream_t stream, const uint16_t* q,
-                               const uint16_t* k, const uint16_t* v, int R, const int32_t* seg_offsets, int nseg,
-                               const int64_t* seg_base, const int32_t* seg_cap, long long cache_rows, uint16_t* q_rot,
-                               uint16_t* k_cache, uint16_t* v_cache, int copy_v, const RopeTable& tab,
-                               uint32_t* status, int* plan_header, int2* plan_items, const int32_t* plan_cap,
-                               int plan_qtiles) {
+cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, bool with_plan, cudaStream_t stream,
+                               const uint16_t* q, const uint16_t* k, const uint16_t* v, int R,
+                               const int32_t* seg_offsets, const int64_t* seg_base, const int32_t* seg_cap,
+                               long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache,
+                               int copy_v, const RopeTable& tab, uint32_t* status, int* plan_header,
+                               int2* plan_items, const int32_t* plan_cap, int plan_qtiles) {
   switch (g) {
-#define NAMOH_ROPE_CASE(GG)                                                                                     \
-  case GG:                                                                                                      \
-    if (smem > 48 * 1024) {                                                                                     \
+#define NAMOH_ROPE_CASE(GG)                                                                                       \
+  case GG: {                                                                                                      \
+    using C = RopeChunk<D, GG>;                                                                                  \
+    const size_t rope_smem = rope_smem_bytes<D, GG>(nseg);                                                       \
+    const size_t smem = rope_smem > plan_smem ? rope_smem : plan_smem;                                           \
+    /* two blocks per SM when their shared memory fits (228 KB per SM, 1 KB reserved per block) */              \
+    const int per_sm = (smem + 1024) * 2 <= 233472 ? 2 : 1;                                                      \
+    const long long nchunks = ((long long)R + C::kRows - 1) / C::kRows;                                        \
+    long long blocks = (long long)per_sm * sm_count;                                                             \
+    if (blocks > nchunks) blocks = nchunks;                                                                      \
+    const long long grid = blocks + (with_plan ? 1 : 0);                                                         \
+    if (grid == 0) return cudaSuccess;                                                                           \
+    if (smem > 48 * 1024) {                                                                                      \
       cudaError_t e = cudaFuncSetAttribute(rope_pack_kernel<D, GG>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
-                                           (int)smem);                                                          \
-      if (e != cudaSuccess) return e;                                                                           \
-    }                                                                                                           \
-    rope_pack_kernel<D, GG><<<grid, 256, smem, stream>>>(q, k, v, R, seg_offsets, nseg, seg_base, seg_cap,       \
-                                                         cache_rows, q_rot, k_cache, v_cache, copy_v, tab, status, \
-                                                         plan_header, plan_items, plan_cap, plan_qtiles);        \
-    break;
+                                           (int)smem);                                                           \
+      if (e != cudaSuccess) return e;                                                                            \
+    }                                                                                                            \
+    rope_pack_kernel<D, GG><<<(unsigned)grid, kRopeThreads, smem, stream>>>(                                     \
+        q, k, v, R, seg_offsets, nseg, seg_base, seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v, tab,      \
+        status, plan_header, plan_items, plan_cap, plan_qtiles);                                                 \
+    break;                                                                                                       \
+  }
     NAMOH_ROPE_CASE(1)
     NAMOH_ROPE_CASE(2)
     NAMOH_ROPE_CASE(4)
@@ -152,26 +224,16 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache, bool copy_v,
                              const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream,
                              void* plan, int plan_qtiles, const int32_t* plan_cap) {
-  const int threads = 256;
-  const int rows_per_block = threads / (D / 16);
-  long long blocks = ((long long)R + rows_per_block - 1) / rows_per_block;
-  const long long cap = (long long)sm_count * 8;
-  if (blocks > cap) blocks = cap;
   int* plan_header = static_cast<int*>(plan);
   int2* plan_items = plan ? reinterpret_cast<int2*>(static_cast<char*>(plan) + 16) : nullptr;
-  const long long grid = blocks + (plan ? 1 : 0);
-  if (grid == 0) return cudaSuccess;
-  size_t smem = (nseg + 1 <= kRopeStageMax) ? (size_t)(nseg + 1) * sizeof(int32_t) : 0;
-  if (plan) {
-    const size_t ps = (size_t)plan_smem_ints(plan_qtiles, nseg) * sizeof(int);
-    if (ps > smem) smem = ps;
-  }
+  const size_t plan_smem = plan ? (size_t)plan_smem_ints(plan_qtiles, nseg) * sizeof(int) : 0;
+  if (R == 0 && !plan) return cudaSuccess;
   if (D == 128)
-    return launch_rope_pack_d<128>(g, dim3((unsigned)grid), smem, stream, q, k, v, R, seg_offsets, nseg, seg_base,
-                                   seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status,
+    return launch_rope_pack_d<128>(g, sm_count, nseg, plan_smem, plan != nullptr, stream, q, k, v, R, seg_offsets,
+                                   seg_base, seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status,
                                    plan_header, plan_items, plan_cap, plan_qtiles);
-  return launch_rope_pack_d<64>(g, dim3((unsigned)grid), smem, stream, q, k, v, R, seg_offsets, nseg, seg_base,
-                                seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status,
+  return launch_rope_pack_d<64>(g, sm_count, nseg, plan_smem, plan != nullptr, stream, q, k, v, R, seg_offsets,
+                                seg_base, seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status,
                                 plan_header, plan_items, plan_cap, plan_qtiles);
 }
 
