@@ -269,6 +269,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto p_ready = [&](uint32_t i) {  // P of tile number i
       return warp_wait(&bars->p_full[i & 1], (i >> 1) & 1, abort_flag, p.status);
     };
+    // Ring entries a and b (b may equal a): both tries in flight together, one warp vote; the
+    // bounded slow path only when one of them is not there yet.
+    auto ring_ready2 = [&](uint32_t a, uint32_t b) {
+      const bool fa = mbar_try_wait(&bars->ring_full[a % kRing], (a / kRing) & 1);
+      const bool fb = mbar_try_wait(&bars->ring_full[b % kRing], (b / kRing) & 1);
+      if (__all_sync(0xffffffffu, fa && fb)) return true;
+      return ring_ready(a) && ring_ready(b);
+    };
 
     while (ok) {
       int4 item;
@@ -350,7 +358,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mma_bf16_ts(tmem + kTmemO, pbuf + kk * 8, v_desc + pv_off(kk), idesc_pv, kk > 0 ? 1u : acc0);
             if (kk < D / 16) mma_bf16_ss(sbuf, q_desc + qk_off(kk), k_desc + qk_off(kk), idesc_qk, kk > 0 ? 1u : 0u);
             // the next step's K/V, while the queue holds this burst's instructions
-            if (kk == 3 && has_next) ok = ring_ready(r_vn) && (!next_k || ring_ready(r_kn));
+            if (kk == 3 && has_next) ok = ring_ready2(r_vn, next_k ? r_kn : r_vn);
           }
         } else {
 #pragma unroll
