@@ -218,6 +218,19 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
       : "memory");
 }
 
+// Read-only global loads issued exactly here: the asm statement keeps its place among the
+// other asm statements, so a load meant to run early is not sunk to its first use.
+__device__ __forceinline__ int ld_issue_s32(const int32_t* p) {
+  int v;
+  asm volatile("ld.global.nc.b32 %0, [%1];" : "=r"(v) : "l"(p));
+  return v;
+}
+__device__ __forceinline__ float ld_issue_f32(const float* p) {
+  float v;
+  asm volatile("ld.global.nc.f32 %0, [%1];" : "=f"(v) : "l"(p));
+  return v;
+}
+
 // 32-byte global store (one whole L2 sector); dst must be 32-byte aligned.
 __device__ __forceinline__ void st_global_v8(void* dst, const uint32_t* w) {
   asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(dst), "r"(w[0]), "r"(w[1]), "r"(w[2]),

@@ -316,55 +316,62 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (nkv <= 2) mma_commit(&bars->q_empty);  // every S of this item issued
       }
       s_iter += nkv > 1 ? 2u : 1u;
-      ok = ring_ready(rv(0)) && (nkv <= 2 || ring_ready(rk(2))) &&
+      // rows past the segment end may hold anything (other segments, unwritten cache rows):
+      // zero them in the last V tile so that 0-weight columns of P cannot meet NaN in V
+      auto zero_v_tail = [&](uint32_t r, int valid_keys) {
+        uint8_t* vtile = smem + L::kRing0 + (r % kRing) * L::kTileBytes;
+        for (int a = 0; a < L::kAtoms; ++a) {
+          uint4* vb = reinterpret_cast<uint4*>(vtile + a * L::kAtomBytes);
+          for (int i = valid_keys * 8 + lane; i < BN * 8; i += 32) vb[i] = make_uint4(0, 0, 0, 0);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+      };
+      // step kv's ring entries: V(kv) and, while kv + 2 < nkv, K(kv+2)
+      uint32_t r_v = rv(0);
+      uint32_t r_k2 = nkv > 2 ? rk(2) : r_v;
+      ok = ring_ready2(r_v, r_k2) &&
            (item_iter == 0 || warp_wait(&bars->o_free, (item_iter - 1) & 1, abort_flag, p.status)) && p_ready(p_iter);
       if (!ok) break;
+      if (n < BN) zero_v_tail(r_v, n);  // a one-tile item whose only tile is partial
 
+      // Everything a step needs besides its commits and P(kv+1) -- the next step's ring
+      // entries, their waits, a partial last V tile -- is done in the middle of the burst,
+      // where the issuing thread would otherwise wait for the MMA queue.
       for (int kv = 0; kv < nkv; ++kv) {
         // here V(kv), K(kv+2), a free O and P(kv) are all in place
-        const uint32_t r_v = rv(kv);
         const bool with_s = kv + 2 < nkv;
         const bool has_next = kv + 1 < nkv;
-        const uint32_t r_k2 = with_s ? rk(kv + 2) : r_v;
         const uint32_t pv_index = p_iter++;
-        const int valid_keys = n - kv * BN;  // keys of this tile inside the segment
-        if (valid_keys < BN) {
-          // rows past the segment end may hold anything (other segments, unwritten cache
-          // rows): zero them so that 0-weight columns of P cannot meet NaN in V
-          uint8_t* vtile = smem + L::kRing0 + (r_v % kRing) * L::kTileBytes;
-          for (int a = 0; a < L::kAtoms; ++a) {
-            uint4* vb = reinterpret_cast<uint4*>(vtile + a * L::kAtomBytes);
-            for (int i = valid_keys * 8 + lane; i < BN * 8; i += 32) vb[i] = make_uint4(0, 0, 0, 0);
-          }
-          fence_proxy_async_smem();
-          __syncwarp();
-        }
         tc_fence_after();
         // P(kv) sits in the buffer of S(kv): S and P are counted alike across items
         const uint32_t pbuf = tmem + tmem_s_col((int)(pv_index % kSBufs));
         const uint32_t sbuf = tmem + tmem_s_col((int)(s_iter % kSBufs));
         const uint64_t v_desc = make_smem_desc_sw128(slot_addr(r_v), L::kAtomBytes, 1024);
         const uint64_t k_desc = make_smem_desc_sw128(slot_addr(r_k2), 16, 1024);
-        // the next step's ring entries, computed before the burst so that the burst itself is
-        // straight-line code (one variant with S(kv+2), one without)
-        const uint32_t r_vn = has_next ? rv(kv + 1) : r_v;
-        const bool next_k = kv + 3 < nkv;
-        const uint32_t r_kn = next_k ? rk(kv + 3) : r_v;
         const uint32_t acc0 = kv > 0 ? 1u : 0u;
+        const uint32_t r_vn = has_next ? rv(kv + 1) : r_v;
+        const uint32_t r_kn = kv + 3 < nkv ? rk(kv + 3) : r_vn;
+        auto mid_burst = [&]() {
+          if (has_next) {
+            ok = ring_ready2(r_vn, r_kn);
+            const int next_valid = n - (kv + 1) * BN;
+            if (ok && next_valid < BN) zero_v_tail(r_vn, next_valid);
+          }
+        };
         if (with_s) {
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
             // PV: K extent = BN keys, 16 per instruction; S: K extent = D, 16 per instruction
             mma_bf16_ts(tmem + kTmemO, pbuf + kk * 8, v_desc + pv_off(kk), idesc_pv, kk > 0 ? 1u : acc0);
             if (kk < D / 16) mma_bf16_ss(sbuf, q_desc + qk_off(kk), k_desc + qk_off(kk), idesc_qk, kk > 0 ? 1u : 0u);
-            // the next step's K/V, while the queue holds this burst's instructions
-            if (kk == 3 && has_next) ok = ring_ready2(r_vn, next_k ? r_kn : r_vn);
+            if (kk == 3) mid_burst();
           }
         } else {
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
             mma_bf16_ts(tmem + kTmemO, pbuf + kk * 8, v_desc + pv_off(kk), idesc_pv, kk > 0 ? 1u : acc0);
-            if (kk == 3 && has_next) ok = ring_ready(r_vn);
+            if (kk == 3) mid_burst();
           }
         }
         mma_commit(&bars->o_ready[pv_index & 1]);
@@ -377,6 +384,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (ok && has_next) ok = p_ready(p_iter);
         if (!ok) break;
+        r_v = r_vn;
+        r_k2 = r_kn;
       }
       ring_iter += 2 * nkv;
       ++item_iter;
@@ -411,7 +420,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int qrank = qt * BM + row;
       const bool valid = qrank < n;
       int src = 0;
-      if (valid) src = p.row_src[off + qrank];
+      if (valid) src = ld_issue_s32(p.row_src + off + qrank);
       float gt = 0.f;
       float m_use = 0.f, l_sum = 0.f;
       for (int kv = 0; kv <= qt && ok; ++kv) {
@@ -494,7 +503,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars->p_full[tile & 1]);
-        if (kv == 0 && valid) gt = p.gate[src];  // used in the epilogue only
+        if (kv == 0 && valid) gt = ld_issue_f32(p.gate + src);  // used in the epilogue only
       }
       if (!ok) break;
       // epilogue: O out of TMEM (O is then free for the next item), O / l * gate as bf16
