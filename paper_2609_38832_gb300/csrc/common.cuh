@@ -53,6 +53,23 @@ struct WorkspaceCarver {
   bool fits() const { return used <= cap; }
 };
 
+// Launch with programmatic stream serialization (see pdl_wait()).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // ---------------------------------------------------------------------------
 // device helpers
 // ---------------------------------------------------------------------------
@@ -217,6 +234,14 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
       "@e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n\t}" ::"r"(smem_u32(bar))
       : "memory");
 }
+
+// Programmatic dependent launch.  A kernel launched with programmatic stream serialization
+// may start while the kernel before it in the stream still runs; pdl_wait() blocks until
+// that kernel has completed and its writes are visible, so everything before it may only
+// touch this kernel's own state.  pdl_launch_dependents() lets the next such kernel start
+// launching (it still waits in its own pdl_wait()).  Both are no-ops in a normal launch.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" :::); }
 
 // Read-only global loads issued exactly here: the asm statement keeps its place among the
 // other asm statements, so a load meant to run early is not sunk to its first use.

@@ -146,7 +146,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int G = gridDim.x;
-  const int nitems = *p.nitems;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < 2; ++i) {
@@ -182,6 +181,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars->tmem_base;
+  // set-up above touched only this CTA's own state; the plan and Q~/K~ come from the kernel
+  // before it (programmatic dependent launch)
+  pdl_launch_dependents();
+  pdl_wait();
+  const int nitems = *p.nitems;
 
   if (warp == kWarpLoad) {
     // ------------------------------------------------------------------ TMA producer
@@ -580,8 +584,8 @@ cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUte
   const int smem = Smem<D>::kAlloc;
   cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  attn_fwd_kernel<D><<<grid, kThreads, smem, stream>>>(tq, tk, tv, p);
-  return cudaGetLastError();
+  e = launch_pdl(attn_fwd_kernel<D>, dim3(grid), dim3(kThreads), (size_t)smem, stream, tq, tk, tv, p);
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace attn

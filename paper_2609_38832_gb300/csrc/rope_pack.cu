@@ -11,7 +11,9 @@
 // shares the rank between the key and the row's g query heads (App. C).
 // Outputs: Q~ (bf16 scratch for the attention kernel), K~ into the key cache, and V copied
 // into the value cache unless the caller passed v_cache == v.  Given a plan buffer, block 0
-// builds the attention work list in the same launch.
+// builds the attention work list in the same launch.  Launched with programmatic dependent
+// launch: set-up overlaps the routing kernel's tail, and every read of routing outputs or
+// inputs comes after pdl_wait().
 #include "common.cuh"
 #include "plan.cuh"
 
@@ -55,8 +57,10 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
   constexpr int HALF = D / 2;
   extern __shared__ __align__(128) uint8_t smem_raw[];
   __shared__ int s_abort;
+  pdl_launch_dependents();  // the attention kernel may start launching; it waits for this grid
   const int first = plan_header ? 1 : 0;
   if ((int)blockIdx.x < first) {
+    pdl_wait();
     build_plan(seg_offsets, nseg, plan_cap, G, plan_qtiles, plan_header, plan_items, reinterpret_cast<int*>(smem_raw));
     return;
   }
@@ -82,9 +86,11 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     for (int i = 0; i < kRopeStages; ++i) mbar_init(&full[i], 1);
     s_abort = 0;
     mbar_fence_init();
+  }
+  pdl_wait();  // routing outputs (and q, k, v) are visible from here
+  if (threadIdx.x == 0)
     for (int i = 0; i < kRopeStages; ++i)
       if (blk + i * nblk < nchunks) issue(blk + i * nblk, i);
-  }
   if (staged)
     for (int i = threadIdx.x; i <= nseg; i += blockDim.x) s_offs[i] = __ldg(seg_offsets + i);
   __syncthreads();
@@ -203,10 +209,9 @@ cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, 
                                            (int)smem);                                                           \
       if (e != cudaSuccess) return e;                                                                            \
     }                                                                                                            \
-    rope_pack_kernel<D, GG><<<(unsigned)grid, kRopeThreads, smem, stream>>>(                                     \
-        q, k, v, R, seg_offsets, nseg, seg_base, seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v, tab,      \
-        status, plan_header, plan_items, plan_cap, plan_qtiles);                                                 \
-    break;                                                                                                       \
+    return launch_pdl(rope_pack_kernel<D, GG>, dim3((unsigned)grid), dim3(kRopeThreads), smem, stream, q, k, v, R,  \
+                      seg_offsets, nseg, seg_base, seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v, tab,    \
+                      status, plan_header, plan_items, plan_cap, plan_qtiles);                                   \
   }
     NAMOH_ROPE_CASE(1)
     NAMOH_ROPE_CASE(2)
