@@ -356,9 +356,9 @@ def run_gpu(args, rank: int, world: int):
                 "pipeline": f"host->device copies, compute and device->host copies on three streams, consecutive "
                             f"steps overlapped; {NSET} rotating device input/output sets ({NSET} x 51 MB > L2), "
                             f"no flush", "y_readback_matches_device": e2e_y_ok},
-        # per step: route (one cooperative kernel after a 4-byte memset) + RoPE/plan (1) + attention
-        # (1), in each of the three timed passes (headline, stage breakdown, end to end)
-        "gpu_launches": 3 * 3 * args.steps,
+        # per step: route (2 kernels) + RoPE/plan (1) + attention (1), in each of the three timed
+        # passes (headline, stage breakdown, end to end)
+        "gpu_launches": 4 * 3 * args.steps,
         "wall_s_timed_region": wall,
         "host_enqueue_ms_max": 1e3 * max(enqueue_s), "flush_ms_min": min(flush_ms), "stage_timing_gapless": gapless,
         "device_status": st,

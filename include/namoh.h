@@ -101,9 +101,10 @@ NAMOH_API const char *namoh_last_error_string(void);
  * Requires 1 <= K <= H <= NAMOH_MAX_HEADS, B >= 1, T >= 1, B*T*K < 2^31.
  * Non-finite logits set NAMOH_DEV_NONFINITE_SCORE (that token's outputs are
  * unspecified but in range).  Integer outputs are deterministic.
- * When every 256-token chunk fits on the GPU at once (B*ceil(T/256) blocks), the
- * packed layout is built in one cooperative launch (after a 4-byte memset of
- * the workspace); otherwise in three launches.  Both give identical results.
+ * The packed layout takes two kernel launches (three when ceil(T/256)*H exceeds
+ * 4096), chained by programmatic dependent launch: the first touches no global
+ * memory before the work ahead of it in the stream has completed.  Every path
+ * gives identical results.
  * ------------------------------------------------------------------------- */
 NAMOH_API size_t namoh_route_workspace_size(int B, int T, int H, int K);
 NAMOH_API int namoh_route(const float *scores, int B, int T, int H, int K, int32_t *topk_head, float *gate,
@@ -128,9 +129,8 @@ NAMOH_API int namoh_route(const float *scores, int B, int T, int H, int K, int32
  * allocates nothing.  The first call on each device resolves the array's device
  * address (cudaGetSymbolAddress) with that device current; make that first call
  * before any stream capture.  Every call on a device shares the one array and
- * leaves its last contents there; the only word that must start at zero (a
- * grid-barrier counter) is cleared by a memset that each call enqueues first,
- * and every other word is written before it is read.  Calls that overlap on the GPU -- on
+ * leaves its last contents there; every word of it is written before it is
+ * read.  Calls that overlap on the GPU -- on
  * different streams, or from different host threads -- race on it and must be
  * serialised by the caller.
  * ------------------------------------------------------------------------- */

@@ -448,13 +448,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int c = 0; c < BN; ++c)
             if (c > row) sv[c] = -INFINITY;
         }
+        // row max: three-input max instructions over eight independent accumulators
         float m8[8];
+        static_assert(BN == 128, "the max tree below covers 128 columns");
 #pragma unroll
-        for (int i = 0; i < 8; ++i) m8[i] = sv[i];
+        for (int i = 0; i < 8; ++i) m8[i] = fmax3(sv[i], sv[8 + i], sv[16 + i]);
 #pragma unroll
-        for (int c = 8; c < BN; ++c) m8[c & 7] = fmaxf(m8[c & 7], sv[c]);
-        const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
-                               fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
+        for (int c = 24; c < 120; c += 16) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) m8[i] = fmax3(m8[i], sv[c + i], sv[c + 8 + i]);
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) m8[i] = fmaxf(m8[i], sv[120 + i]);
+        const float mx = fmax3(fmax3(m8[0], m8[1], m8[2]), fmax3(m8[3], m8[4], m8[5]), fmaxf(m8[6], m8[7]));
         const float m_tile = mx * p.scale_log2;
         float alpha = 1.f;
         bool rescale = false;
@@ -465,16 +471,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           m_use = m_tile;
           rescale = true;
         }
+        // P = exp2(S * scale - m_use): scale-and-subtract and the row sum on fp32 pairs
         uint32_t pk[BN / 2];
-        float sum4[4] = {0.f, 0.f, 0.f, 0.f};
+        uint64_t sum2[4] = {0ull, 0ull, 0ull, 0ull};
+        const uint64_t sc2 = f2_pack(p.scale_log2, p.scale_log2), nm2 = f2_pack(-m_use, -m_use);
 #pragma unroll
         for (int c = 0; c < BN; c += 2) {
-          const float e0 = fast_exp2(fmaf(sv[c], p.scale_log2, -m_use));
-          const float e1 = fast_exp2(fmaf(sv[c + 1], p.scale_log2, -m_use));
-          sum4[(c >> 1) & 3] += e0 + e1;
+          float x0, x1;
+          f2_unpack(f2_fma(f2_pack(sv[c], sv[c + 1]), sc2, nm2), x0, x1);
+          const float e0 = fast_exp2(x0), e1 = fast_exp2(x1);
+          sum2[(c >> 1) & 3] = f2_add(sum2[(c >> 1) & 3], f2_pack(e0, e1));
           pk[c / 2] = pack_bf16x2(e0, e1);
         }
-        l_sum = l_sum * alpha + ((sum4[0] + sum4[1]) + (sum4[2] + sum4[3]));
+        float sa, sb;
+        f2_unpack(f2_add(f2_add(sum2[0], sum2[1]), f2_add(sum2[2], sum2[3])), sa, sb);
+        l_sum = l_sum * alpha + (sa + sb);
         // P over the S columns just read (every S value is in registers)
         {
           uint32_t r[32];

@@ -3,21 +3,19 @@
 // Every token selects exactly K heads, so sequence b's rows start at b*T*K and each
 // sequence's segment offsets depend only on that sequence's own head counts.
 //
-// One cooperative launch when the chunks of all sequences fit on the GPU at once:
-//   route_fused_kernel     per 256-token chunk: TopK + gates and chunk head counts; one
-//                          bounded grid barrier; then every chunk sums its sequence's count
-//                          table itself (chunk bases, n, segment offsets) and ranks its
-//                          tokens with warp ballots.
-// Otherwise three stream-ordered launches:
-//   1. route_topk_kernel   one thread per token: TopK of the fp32 logits (descending,
-//                          ties to the lower head index), fp32 softmax gates over all H,
-//                          and per-chunk head counts (one block = one 256-token chunk).
-//   2. route_scan_kernel   one block per sequence: exclusive scan of the chunk counts over
-//                          chunks for every head -> chunk base ranks, n[b, h] and the
-//                          sequence's segment offsets.
-//   3. route_rank_kernel   per chunk: warp ballots give each (token, slot) its rank among
-//                          the chunk's earlier tokens for that head; adds the chunk base
-//                          -> rank, row and row_src.
+// The packed layout takes two launches, chained by programmatic dependent launch (the
+// second is resident and waiting before the first ends):
+//   1. route_local_kernel  one block per 256-token chunk, one thread per token: TopK of the
+//                          fp32 logits (descending, ties to the lower head index), fp32
+//                          softmax gates over all H, the chunk's head counts, and each
+//                          (token, slot)'s rank among the chunk's earlier tokens for its head
+//                          (warp ballots; written to `rank` for the second pass).
+//   2. route_final_kernel  one block per chunk: sums its sequence's chunk-count table (chunk
+//                          base per head, n[b, h], segment offsets), then the final rank, row
+//                          and row_src of its tokens.
+// When the count tables are large (many chunks x heads) a third launch between the two,
+// route_scan_kernel (one block per sequence), scans them once and the final pass reads the
+// chunk bases.  Without the packed layout (e.g. one decode token) only route_topk_kernel runs.
 // All integer work is exact, so the packed layout is deterministic and bit-identical to
 // a sequential append in token order, on either path.
 #include <float.h>
@@ -31,12 +29,11 @@ namespace {
 
 constexpr int kChunk = 256;  // tokens per block in the top-K and rank kernels
 
-// TopK and gates of token `tok` (Sec. 3.1 Eq. namoh-gates).  Writes topk_head and gate,
-// adds the picks to s_cnt (when given) and returns the picked heads as a bit mask.
+// TopK and gates of token `tok` (Sec. 3.1 Eq. namoh-gates).  Writes topk_head and gate and
+// returns the picked heads as a bit mask.
 template <int HMAX>
 __device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores, size_t tok, int H, int K,
-                                               int32_t* __restrict__ topk_head, float* __restrict__ gate, int* s_cnt,
-                                               int* s_bad) {
+                                               int32_t* __restrict__ topk_head, float* __restrict__ gate, int* s_bad) {
   // this token's H logits: independent loads, all in flight together
   const float* src = scores + tok * H;
   float sc[HMAX];
@@ -94,7 +91,6 @@ __device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores,
     }
     topk_head[base + k] = bi;
     gate[base + k] = expf(bv - mx) * inv_z;
-    if (s_cnt) atomicAdd(&s_cnt[bi], 1);
     mask |= 1ull << bi;
     pv = bv;
     pi = bi;
@@ -103,25 +99,18 @@ __device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores,
   return mask;
 }
 
+// TopK and gates only (no packed layout), one thread per token.
 template <int HMAX>
 __global__ void __launch_bounds__(kChunk) route_topk_kernel(const float* __restrict__ scores, int T, int H, int K,
-                                                            int nchunks, int32_t* __restrict__ topk_head,
-                                                            float* __restrict__ gate,
-                                                            int32_t* __restrict__ chunk_count,
+                                                            int32_t* __restrict__ topk_head, float* __restrict__ gate,
                                                             uint32_t* __restrict__ status) {
-  __shared__ int s_cnt[NAMOH_MAX_HEADS];
   __shared__ int s_bad;
-  const int c = blockIdx.x;
-  const int b = blockIdx.y;
-  const int tid = threadIdx.x;
-  const int t = c * kChunk + tid;
-  if (tid < NAMOH_MAX_HEADS) s_cnt[tid] = 0;
-  if (tid == 0) s_bad = 0;
+  const int t = blockIdx.x * kChunk + threadIdx.x;
+  if (threadIdx.x == 0) s_bad = 0;
   __syncthreads();
-  if (t < T) topk_token<HMAX>(scores, (size_t)b * T + t, H, K, topk_head, gate, chunk_count ? s_cnt : nullptr, &s_bad);
+  if (t < T) topk_token<HMAX>(scores, (size_t)blockIdx.y * T + t, H, K, topk_head, gate, &s_bad);
   __syncthreads();
-  if (chunk_count && tid < H) chunk_count[((size_t)b * nchunks + c) * H + tid] = s_cnt[tid];
-  if (tid == 0 && s_bad) report(status, NAMOH_DEV_NONFINITE_SCORE);
+  if (threadIdx.x == 0 && s_bad) report(status, NAMOH_DEV_NONFINITE_SCORE);
 }
 
 // One block per sequence b: for every head, exclusive scan of the chunk counts over chunks
@@ -134,6 +123,8 @@ __global__ void __launch_bounds__(1024) route_scan_kernel(const int32_t* __restr
   __shared__ int s_n[NAMOH_MAX_HEADS];
   const int b = blockIdx.x;
   const int tid = threadIdx.x;
+  pdl_launch_dependents();
+  pdl_wait();  // pass 1 complete and visible
   const int P = blockDim.x / H;  // parts per head (blockDim is a multiple of H)
   const int h = tid % H, p = tid / H;
   const int per = (nchunks + P - 1) / P;
@@ -163,186 +154,125 @@ __global__ void __launch_bounds__(1024) route_scan_kernel(const int32_t* __restr
   }
 }
 
-// Ranks of one chunk's (token, slot) pairs (Sec. 3.2 Eq. namoh-head-rope): rho = chunk base
-// + rank among this chunk's earlier tokens for the head (warp ballots).  s_cbase and s_soff
-// (chunk base and segment offset per head) must be ready in shared memory; `mask` holds the
-// thread's picked heads (0 past the end).  Ends with no block barrier pending.
-struct RankSmem {
-  uint32_t bal[kChunk / 32][NAMOH_MAX_HEADS];
-  int wbase[kChunk / 32][NAMOH_MAX_HEADS];
-  int cbase[NAMOH_MAX_HEADS];  // rank of the chunk's first token for each head
-  int soff[NAMOH_MAX_HEADS];   // segment offset of each head in this sequence
-};
-
-__device__ __forceinline__ void rank_chunk(RankSmem& sm, uint64_t mask, bool valid, size_t tok, int H, int K,
-                                           const int32_t* topk_head, int32_t* __restrict__ rank,
-                                           int32_t* __restrict__ row, int32_t* __restrict__ row_src) {
+// Pass 1 of the packed layout (one block per chunk, one thread per token): TopK and gates,
+// the chunk's head counts, and rank_local = the (token, slot)'s rank among this chunk's
+// earlier tokens for its head (Sec. 3.2 Eq. namoh-head-rope restricted to the chunk).
+// rank_local goes to `rank`, which the final pass turns into the full rank.
+template <int HMAX>
+__global__ void __launch_bounds__(kChunk) route_local_kernel(const float* __restrict__ scores, int T, int H, int K,
+                                                             int nchunks, int32_t* __restrict__ topk_head,
+                                                             float* __restrict__ gate, int32_t* __restrict__ rank,
+                                                             int32_t* __restrict__ chunk_count,
+                                                             uint32_t* __restrict__ status) {
+  __shared__ uint32_t s_bal[kChunk / 32][NAMOH_MAX_HEADS];
+  __shared__ int s_bad;
+  pdl_launch_dependents();
+  const int c = blockIdx.x, b = blockIdx.y;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int t = c * kChunk + tid;
+  const bool valid = t < T;
+  const size_t tok = (size_t)b * T + t;
+  if (tid == 0) s_bad = 0;
+  __syncthreads();
+  // the logits may come from the kernel just before this one, and that kernel may still
+  // read this call's outputs: nothing global is touched before the wait
+  pdl_wait();
+  uint64_t mask = 0;
+  if (valid) mask = topk_token<HMAX>(scores, tok, H, K, topk_head, gate, &s_bad);
   for (int h = 0; h < H; ++h) {
     const uint32_t bal = __ballot_sync(0xffffffffu, (mask >> h) & 1ull);
-    if (lane == 0) sm.bal[warp][h] = bal;
+    if (lane == 0) s_bal[warp][h] = bal;
   }
   __syncthreads();
-  for (int i = tid; i < (kChunk / 32) * H; i += kChunk) {
-    const int w = i / H, h = i % H;
-    int before = 0;
-    for (int q = 0; q < w; ++q) before += __popc(sm.bal[q][h]);
-    sm.wbase[w][h] = before;
+  if (tid < H) {
+    int n = 0;
+#pragma unroll
+    for (int w = 0; w < kChunk / 32; ++w) n += __popc(s_bal[w][tid]);
+    chunk_count[((size_t)b * nchunks + c) * H + tid] = n;
   }
-  __syncthreads();
+  if (tid == 0 && s_bad) report(status, NAMOH_DEV_NONFINITE_SCORE);
   if (!valid) return;
   const uint32_t lt = (1u << lane) - 1u;
   for (int k = 0; k < K; ++k) {
-    const int h = topk_head[tok * K + k];
-    const int rho = sm.cbase[h] + sm.wbase[warp][h] + __popc(sm.bal[warp][h] & lt);
-    const int r = sm.soff[h] + rho;
-    rank[tok * K + k] = rho;
-    row[tok * K + k] = r;
-    row_src[r] = (int32_t)(tok * K + k);
+    const int h = topk_head[tok * K + k];  // written above by this thread
+    int before = 0;
+    for (int w = 0; w < warp; ++w) before += __popc(s_bal[w][h]);
+    rank[tok * K + k] = before + __popc(s_bal[warp][h] & lt);
   }
 }
 
-__global__ void __launch_bounds__(kChunk) route_rank_kernel(const int32_t* __restrict__ topk_head, int T, int H,
-                                                            int K, int nchunks,
-                                                            const int32_t* __restrict__ chunk_base,
-                                                            const int32_t* __restrict__ seg_offsets,
-                                                            int32_t* __restrict__ rank, int32_t* __restrict__ row,
-                                                            int32_t* __restrict__ row_src) {
-  __shared__ RankSmem sm;
+// Pass 2 (one block per chunk): this chunk's base rank per head and the sequence's
+// segment offsets -- from the chunk-count table (chunk_base == nullptr: thread (h, p)
+// sums chunks p, p + P, ...), or as written by route_scan_kernel -- then
+// rank = base + rank_local, row = seg_offsets[b*H + head] + rank, row_src[row].
+__global__ void __launch_bounds__(kChunk) route_final_kernel(const int32_t* __restrict__ topk_head, int T, int H,
+                                                             int K, int nchunks, const int32_t* chunk_count,
+                                                             const int32_t* chunk_base, int32_t* __restrict__ rank,
+                                                             int32_t* __restrict__ row, int32_t* seg_offsets,
+                                                             int32_t* __restrict__ row_src, int B) {
+  __shared__ int s_tot[kChunk];
+  __shared__ int s_bef[kChunk];
+  __shared__ int s_cbase[NAMOH_MAX_HEADS];
+  __shared__ int s_soff[NAMOH_MAX_HEADS];
+  pdl_launch_dependents();
   const int c = blockIdx.x, b = blockIdx.y;
   const int tid = threadIdx.x;
   const int t = c * kChunk + tid;
   const bool valid = t < T;
   const size_t tok = (size_t)b * T + t;
-  if (tid < H) {
-    sm.cbase[tid] = chunk_base[((size_t)b * nchunks + c) * H + tid];
-    sm.soff[tid] = seg_offsets[(size_t)b * H + tid];
-  }
-  uint64_t mask = 0;
-  if (valid)
-    for (int k = 0; k < K; ++k) mask |= 1ull << __ldg(topk_head + tok * K + k);
-  rank_chunk(sm, mask, valid, tok, H, K, topk_head, rank, row, row_src);
-}
-
-// Grid barrier for a cooperative launch.  *count must be 0 at launch (the host clears it);
-// every block adds 1 and waits, bounded, until all have.  Returns false after a timeout
-// (NAMOH_DEV_TIMEOUT is reported).
-__device__ __forceinline__ bool grid_barrier(unsigned* count, unsigned nblocks, uint32_t* status) {
-  __shared__ int s_ok;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    __threadfence();
-    atomicAdd(count, 1u);
-    int ok = 1;
-    const uint64_t t0 = global_timer_ns();
-    for (;;) {
-      unsigned v;
-      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(count) : "memory");
-      if (v >= nblocks) break;
-      if (global_timer_ns() - t0 > kWaitLimitNs) {
-        report(status, NAMOH_DEV_TIMEOUT);
-        ok = 0;
-        break;
+  pdl_wait();  // pass 1 (and the scan, when there is one) complete and visible
+  if (chunk_base) {
+    if (tid < H) {
+      s_cbase[tid] = chunk_base[((size_t)b * nchunks + c) * H + tid];
+      s_soff[tid] = seg_offsets[(size_t)b * H + tid];
+    }
+  } else {
+    const int P = kChunk / H;
+    const int h = tid % H, p = tid / H;
+    int tot = 0, bef = 0;
+    if (p < P) {
+      const int32_t* cc = chunk_count + (size_t)b * nchunks * H + h;
+      for (int cj = p; cj < nchunks; cj += P) {
+        const int v = __ldcg(cc + (size_t)cj * H);
+        tot += v;
+        bef += (cj < c) ? v : 0;
       }
-      __nanosleep(64);
     }
-    s_ok = ok;
+    s_tot[tid] = tot;
+    s_bef[tid] = bef;
+    __syncthreads();
+    if (tid < H) {
+      int n = 0, cb = 0;
+      for (int q = 0; q < P; ++q) {
+        n += s_tot[q * H + tid];
+        cb += s_bef[q * H + tid];
+      }
+      s_cbase[tid] = cb;
+      s_tot[tid] = n;  // rows q >= 1 of s_tot are no longer read
+    }
+    __syncthreads();
+    if (tid == 0) {
+      int off = b * T * K;  // < 2^31: checked on the host
+      for (int hh = 0; hh < H; ++hh) {
+        s_soff[hh] = off;
+        off += s_tot[hh];
+      }
+    }
+    __syncthreads();
+    if (c == 0 && tid < H) seg_offsets[(size_t)b * H + tid] = s_soff[tid];
+    if (c == 0 && b == B - 1 && tid == 0) seg_offsets[(size_t)B * H] = B * T * K;
   }
   __syncthreads();
-  return s_ok != 0;
-}
-
-// The whole of routing in one cooperative launch: grid = B * nchunks blocks, all resident.
-template <int HMAX>
-__global__ void __launch_bounds__(kChunk) route_fused_kernel(const float* __restrict__ scores, int T, int H, int K,
-                                                             int nchunks, int32_t* __restrict__ topk_head,
-                                                             float* __restrict__ gate, int32_t* chunk_count,
-                                                             unsigned* barrier, int32_t* __restrict__ rank,
-                                                             int32_t* __restrict__ row,
-                                                             int32_t* __restrict__ seg_offsets,
-                                                             int32_t* __restrict__ row_src, int B,
-                                                             uint32_t* __restrict__ status) {
-  __shared__ RankSmem sm;
-  __shared__ int s_cnt[NAMOH_MAX_HEADS];
-  __shared__ int s_tot[kChunk];
-  __shared__ int s_bef[kChunk];
-  __shared__ int s_bad;
-  const int c = blockIdx.x % nchunks;
-  const int b = blockIdx.x / nchunks;
-  const int tid = threadIdx.x;
-  const int t = c * kChunk + tid;
-  const bool valid = t < T;
-  const size_t tok = (size_t)b * T + t;
-  if (tid < NAMOH_MAX_HEADS) s_cnt[tid] = 0;
-  if (tid == 0) s_bad = 0;
-  __syncthreads();
-  uint64_t mask = 0;
-  if (valid) mask = topk_token<HMAX>(scores, tok, H, K, topk_head, gate, s_cnt, &s_bad);
-  __syncthreads();
-  if (tid < H) chunk_count[((size_t)b * nchunks + c) * H + tid] = s_cnt[tid];
-  if (tid == 0 && s_bad) report(status, NAMOH_DEV_NONFINITE_SCORE);
-  if (!grid_barrier(barrier, gridDim.x, status)) return;
-
-  // this sequence's count table: thread (h, p) sums chunks p, p + P, ... (L2 reads)
-  const int P = kChunk / H;
-  const int h = tid % H, p = tid / H;
-  int tot = 0, bef = 0;
-  if (p < P) {
-    const int32_t* cc = chunk_count + (size_t)b * nchunks * H + h;
-    for (int cj = p; cj < nchunks; cj += P) {
-      const int v = __ldcg(cc + (size_t)cj * H);
-      tot += v;
-      bef += (cj < c) ? v : 0;
-    }
+  if (!valid) return;
+  for (int k = 0; k < K; ++k) {
+    const size_t i = tok * K + k;
+    const int h = topk_head[i];
+    const int rho = s_cbase[h] + rank[i];
+    const int r = s_soff[h] + rho;
+    rank[i] = rho;
+    row[i] = r;
+    row_src[r] = (int32_t)i;
   }
-  s_tot[tid] = tot;
-  s_bef[tid] = bef;
-  __syncthreads();
-  if (tid < H) {
-    int n = 0, cb = 0;
-    for (int q = 0; q < P; ++q) {
-      n += s_tot[q * H + tid];
-      cb += s_bef[q * H + tid];
-    }
-    sm.cbase[tid] = cb;
-    s_tot[tid] = n;  // rows q >= 1 of s_tot are no longer read
-  }
-  __syncthreads();
-  if (tid == 0) {
-    int off = b * T * K;  // < 2^31: checked on the host
-    for (int hh = 0; hh < H; ++hh) {
-      sm.soff[hh] = off;
-      off += s_tot[hh];
-    }
-  }
-  __syncthreads();
-  if (c == 0 && tid < H) seg_offsets[(size_t)b * H + tid] = sm.soff[tid];
-  if (c == 0 && b == B - 1 && tid == 0) seg_offsets[(size_t)B * H] = B * T * K;
-  rank_chunk(sm, mask, valid, tok, H, K, topk_head, rank, row, row_src);
-}
-
-constexpr int kFusedMaxTable = 1 << 15;  // chunk-count entries one sequence may have on the fused path
-
-// Blocks of route_fused_kernel<HMAX> that fit on the current device at once (0 if the
-// device cannot launch cooperatively).  Cached per device.
-template <int HMAX>
-int fused_capacity() {
-  static std::mutex mu;
-  static int cached[64] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
-  std::lock_guard<std::mutex> lock(mu);
-  if (cached[dev] == 0) {
-    int coop = 0, sms = 0, per_sm = 0;
-    if (cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, route_fused_kernel<HMAX>, kChunk, 0) != cudaSuccess) {
-      cudaGetLastError();
-      return 0;
-    }
-    cached[dev] = coop ? sms * per_sm : -1;
-  }
-  return cached[dev] > 0 ? cached[dev] : 0;
 }
 
 struct RouteArgs {
@@ -351,50 +281,35 @@ struct RouteArgs {
   int32_t *topk_head, *rank, *row, *seg_offsets, *row_src;
   float* gate;
   int32_t *chunk_count, *chunk_base;
-  unsigned* barrier;
   uint32_t* status;
 };
 
-// Returns 1 when launched on the fused path, 0 when the shape needs the three-launch path,
-// or a negative status.
-template <int HMAX>
-int try_fused(const RouteArgs& a, cudaStream_t stream) {
-  const long long nblocks = (long long)a.B * a.nchunks;
-  if ((long long)a.nchunks * a.H > kFusedMaxTable || nblocks > fused_capacity<HMAX>()) return 0;
-  cudaError_t e = cudaMemsetAsync(a.barrier, 0, sizeof(unsigned), stream);
-  if (e != cudaSuccess) return cuda_fail(e, "route barrier memset");
-  const float* scores = a.scores;
-  int T = a.T, H = a.H, K = a.K, nchunks = a.nchunks, B = a.B;
-  int32_t *topk = a.topk_head, *cc = a.chunk_count, *rank = a.rank, *row = a.row, *so = a.seg_offsets,
-          *rs = a.row_src;
-  float* gate = a.gate;
-  unsigned* bar = a.barrier;
-  uint32_t* st = a.status;
-  void* args[] = {&scores, &T, &H, &K, &nchunks, &topk, &gate, &cc, &bar, &rank, &row, &so, &rs, &B, &st};
-  e = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(route_fused_kernel<HMAX>), dim3((unsigned)nblocks),
-                                  dim3(kChunk), args, 0, stream);
-  if (e != cudaSuccess) return cuda_fail(e, "route_fused_kernel cooperative launch");
-  return 1;
-}
+// Count tables up to this many entries per sequence are summed by every block of the final
+// pass; larger ones are scanned once by route_scan_kernel.
+constexpr int kFinalMaxTable = 1 << 12;
 
 template <int HMAX>
 int launch_route(const RouteArgs& a, cudaStream_t stream) {
-  const bool compact = a.seg_offsets != nullptr;
-  if (compact) {
-    const int f = try_fused<HMAX>(a, stream);
-    if (f != 0) return f < 0 ? f : NAMOH_OK;
+  const dim3 chunks((unsigned)a.nchunks, (unsigned)a.B);
+  if (a.seg_offsets == nullptr) {
+    route_topk_kernel<HMAX><<<chunks, kChunk, 0, stream>>>(a.scores, a.T, a.H, a.K, a.topk_head, a.gate, a.status);
+    return cuda_check_launch("route_topk_kernel launch");
   }
-  route_topk_kernel<HMAX><<<dim3(a.nchunks, a.B), kChunk, 0, stream>>>(a.scores, a.T, a.H, a.K, a.nchunks, a.topk_head,
-                                                                       a.gate, a.chunk_count, a.status);
-  if (const int st = cuda_check_launch("route_topk_kernel launch")) return st;
-  if (!compact) return NAMOH_OK;
-  const int scan_threads = 1024 - (1024 % a.H);
-  route_scan_kernel<<<a.B, scan_threads, 0, stream>>>(a.chunk_count, a.B, a.T, a.H, a.K, a.nchunks, a.chunk_base,
-                                                      a.seg_offsets);
-  if (const int st = cuda_check_launch("route_scan_kernel launch")) return st;
-  route_rank_kernel<<<dim3(a.nchunks, a.B), kChunk, 0, stream>>>(a.topk_head, a.T, a.H, a.K, a.nchunks, a.chunk_base,
-                                                                 a.seg_offsets, a.rank, a.row, a.row_src);
-  return cuda_check_launch("route_rank_kernel launch");
+  cudaError_t e = launch_pdl(route_local_kernel<HMAX>, chunks, dim3(kChunk), 0, stream, a.scores, a.T, a.H, a.K,
+                             a.nchunks, a.topk_head, a.gate, a.rank, a.chunk_count, a.status);
+  if (e != cudaSuccess) return cuda_fail(e, "route_local_kernel launch");
+  const bool scan = (long long)a.nchunks * a.H > kFinalMaxTable;
+  if (scan) {
+    const int scan_threads = 1024 - (1024 % a.H);
+    e = launch_pdl(route_scan_kernel, dim3((unsigned)a.B), dim3((unsigned)scan_threads), 0, stream,
+                   (const int32_t*)a.chunk_count, a.B, a.T, a.H, a.K, a.nchunks, a.chunk_base, a.seg_offsets);
+    if (e != cudaSuccess) return cuda_fail(e, "route_scan_kernel launch");
+  }
+  e = launch_pdl(route_final_kernel, chunks, dim3(kChunk), 0, stream, (const int32_t*)a.topk_head, a.T, a.H, a.K,
+                 a.nchunks, (const int32_t*)a.chunk_count, (const int32_t*)(scan ? a.chunk_base : nullptr), a.rank,
+                 a.row, a.seg_offsets, a.row_src, a.B);
+  if (e != cudaSuccess) return cuda_fail(e, "route_final_kernel launch");
+  return NAMOH_OK;
 }
 
 }  // namespace
@@ -408,7 +323,6 @@ extern "C" size_t namoh_route_workspace_size(int B, int T, int H, int K) {
   WorkspaceCarver ws{nullptr, 0, 0};
   ws.take<int32_t>((size_t)B * nchunks * H);  // chunk counts
   ws.take<int32_t>((size_t)B * nchunks * H);  // chunk bases
-  ws.take<unsigned>(1);                       // grid barrier counter
   return align_up(ws.used, 256);
 }
 
@@ -441,7 +355,6 @@ extern "C" int namoh_route(const float* scores, int B, int T, int H, int K, int3
     WorkspaceCarver ws{static_cast<char*>(workspace), workspace_bytes, 0};
     a.chunk_count = ws.take<int32_t>((size_t)B * a.nchunks * H);
     a.chunk_base = ws.take<int32_t>((size_t)B * a.nchunks * H);
-    a.barrier = ws.take<unsigned>(1);
     if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
   }
   if (H <= 8) return launch_route<8>(a, stream);

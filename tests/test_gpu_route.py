@@ -41,8 +41,10 @@ def _check_route(namoh, oracle_mod, s: np.ndarray, K: int):
     (2, 300, 64, 1),     # K = 1 with the widest router
     (1, 1, 8, 2),        # one token
     (4, 4096, 16, 4),    # balanced routing at full size
-    (2, 19200, 64, 8),   # 150 chunks of the widest router: close to one resident block per SM
-    (3, 70000, 16, 4),   # more chunks than fit on the GPU at once: the three-launch path
+    (1, 65536, 16, 4),   # 256 chunks x 16 heads = 4096 table entries: the largest summed per block
+    (1, 65537, 16, 4),   # one token more: 4112 entries, the count table is scanned once instead
+    (2, 19200, 64, 8),   # 75 chunks of the widest router (4800 entries): scanned
+    (3, 70000, 16, 4),   # 274 chunks per sequence: scanned
 ])
 def test_route_matches_oracle(namoh, oracle_mod, B, T, H, K):
     _check_route(namoh, oracle_mod, ni.router_scores(0, B, T, H), K)
@@ -110,7 +112,7 @@ def test_route_nonfinite_sets_status(namoh):
 
 
 def test_route_repeated_calls_reuse_workspace(namoh, oracle_mod):
-    """Back-to-back calls on one workspace (the grid-barrier counter is reset by every call)."""
+    """Back-to-back calls on one workspace: nothing carries over from one call to the next."""
     ws = namoh.Workspace()
     for seed in (3, 4, 3):
         s = ni.router_scores(seed, 2, 3000, 16)
