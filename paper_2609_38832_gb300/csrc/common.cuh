@@ -116,6 +116,22 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// As mbar_try_wait, but the thread may sleep in the hardware for up to `ns` nanoseconds
+// waiting for the phase (it wakes when the phase completes): no issue slots are spent on a
+// wait that lasts.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, uint32_t parity, uint32_t ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(ns)
+      : "memory");
+  return ok != 0;
+}
+constexpr uint32_t kWaitSleepNs = 20000;  // longest sleep per try (the abort flag is read in between)
+
 // Bounded wait.  `abort_flag` (shared memory) lets one role that gave up stop the
 // others: once it is set every wait returns false immediately.  Returns true when
 // the phase with the given parity completed.
@@ -133,7 +149,7 @@ static __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parit
   const uint64_t t0 = global_timer_ns();
   while (true) {
     if (*abort_flag) return false;
-    if (mbar_try_wait(bar, parity)) return true;
+    if (mbar_try_wait_sleep(bar, parity, kWaitSleepNs)) return true;
     if (global_timer_ns() - t0 > kWaitLimitNs) {
       *abort_flag = 1;
       // where: barrier word index within its 256-word block, and the warp that gave up

@@ -133,6 +133,101 @@ __device__ __forceinline__ bool take_item(Bars* bars, uint32_t idx, int4* item, 
   return true;
 }
 
+// Online softmax of one S tile for this thread's query row (Sec. 3.1, causal scaled
+// dot-product attention): S from TMEM, the causal mask on the diagonal tile, the running max
+// (moved only when it grows by more than kRescaleThreshold) and row sum, P = exp2(S * scale - m)
+// as bf16 over the first half of the S columns, and O rescaled when the max moved (after
+// PV(tile - 1) completed, through wait_pv).  Returns false when a wait gave up.  Ends with the
+// TMEM stores complete and fenced for the arrive on p_full.
+template <int D, typename WaitPv>
+__device__ __forceinline__ bool softmax_tile(uint32_t s_addr, uint32_t o_addr, int kv, int qt, int row,
+                                             float scale_log2, float& m_use, float& l_sum, uint32_t tile,
+                                             WaitPv&& wait_pv) {
+  float sv[BN];
+#pragma unroll
+  for (int c = 0; c < BN / 32; ++c) {
+    uint32_t r[32];
+    tmem_ld32(s_addr + c * 32, r);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) sv[c * 32 + i] = __uint_as_float(r[i]);
+  }
+  tmem_wait_ld();
+  // causal mask on the diagonal tile: key rank kv*BN + c <= query rank
+  if (kv == qt) {
+#pragma unroll
+    for (int c = 0; c < BN; ++c)
+      if (c > row) sv[c] = -INFINITY;
+  }
+  // row max: three-input max instructions over eight independent accumulators
+  float m8[8];
+  static_assert(BN == 128, "the max tree below covers 128 columns");
+#pragma unroll
+  for (int i = 0; i < 8; ++i) m8[i] = fmax3(sv[i], sv[8 + i], sv[16 + i]);
+#pragma unroll
+  for (int c = 24; c < 120; c += 16) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) m8[i] = fmax3(m8[i], sv[c + i], sv[c + 8 + i]);
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) m8[i] = fmaxf(m8[i], sv[120 + i]);
+  const float mx = fmax3(fmax3(m8[0], m8[1], m8[2]), fmax3(m8[3], m8[4], m8[5]), fmaxf(m8[6], m8[7]));
+  const float m_tile = mx * scale_log2;
+  float alpha = 1.f;
+  bool rescale = false;
+  if (kv == 0) {
+    m_use = m_tile;
+  } else if (m_tile > m_use + kRescaleThreshold) {
+    alpha = fast_exp2(m_use - m_tile);
+    m_use = m_tile;
+    rescale = true;
+  }
+  // P = exp2(S * scale - m_use): scale-and-subtract and the row sum on fp32 pairs
+  uint32_t pk[BN / 2];
+  uint64_t sum2[4] = {0ull, 0ull, 0ull, 0ull};
+  const uint64_t sc2 = f2_pack(scale_log2, scale_log2), nm2 = f2_pack(-m_use, -m_use);
+#pragma unroll
+  for (int c = 0; c < BN; c += 2) {
+    float x0, x1;
+    f2_unpack(f2_fma(f2_pack(sv[c], sv[c + 1]), sc2, nm2), x0, x1);
+    const float e0 = fast_exp2(x0), e1 = fast_exp2(x1);
+    sum2[(c >> 1) & 3] = f2_add(sum2[(c >> 1) & 3], f2_pack(e0, e1));
+    pk[c / 2] = pack_bf16x2(e0, e1);
+  }
+  float sa, sb;
+  f2_unpack(f2_add(f2_add(sum2[0], sum2[1]), f2_add(sum2[2], sum2[3])), sa, sb);
+  l_sum = l_sum * alpha + (sa + sb);
+  // P over the S columns just read (every S value is in registers)
+  {
+    uint32_t r[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) r[i] = pk[i];
+    tmem_st32(s_addr, r);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) r[i] = pk[32 + i];
+    tmem_st32(s_addr + 32, r);
+  }
+  // O may only be rescaled once the previous PV completed; without a rescale this
+  // tile's softmax does not touch O and overlaps that PV
+  if (kv > 0 && __any_sync(0xffffffffu, rescale)) {
+    if (!wait_pv(tile - 1)) return false;
+    tc_fence_after();
+    {
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t r[32];
+        tmem_ld32(o_addr + c * 32, r);
+        tmem_wait_ld();
+#pragma unroll
+        for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+        tmem_st32(o_addr + c * 32, r);
+      }
+    }
+  }
+  tmem_wait_st();
+  tc_fence_before();
+  return true;
+}
+
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
@@ -433,89 +528,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t tile = s_iter++;
         if (!ok) break;
         tc_fence_after();
-        float sv[BN];
-#pragma unroll
-        for (int c = 0; c < BN / 32; ++c) {
-          uint32_t r[32];
-          tmem_ld32(s_addr + c * 32, r);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) sv[c * 32 + i] = __uint_as_float(r[i]);
-        }
-        tmem_wait_ld();
-        // causal mask on the diagonal tile: key rank kv*BN + c <= query rank
-        if (kv == qt) {
-#pragma unroll
-          for (int c = 0; c < BN; ++c)
-            if (c > row) sv[c] = -INFINITY;
-        }
-        // row max: three-input max instructions over eight independent accumulators
-        float m8[8];
-        static_assert(BN == 128, "the max tree below covers 128 columns");
-#pragma unroll
-        for (int i = 0; i < 8; ++i) m8[i] = fmax3(sv[i], sv[8 + i], sv[16 + i]);
-#pragma unroll
-        for (int c = 24; c < 120; c += 16) {
-#pragma unroll
-          for (int i = 0; i < 8; ++i) m8[i] = fmax3(m8[i], sv[c + i], sv[c + 8 + i]);
-        }
-#pragma unroll
-        for (int i = 0; i < 8; ++i) m8[i] = fmaxf(m8[i], sv[120 + i]);
-        const float mx = fmax3(fmax3(m8[0], m8[1], m8[2]), fmax3(m8[3], m8[4], m8[5]), fmaxf(m8[6], m8[7]));
-        const float m_tile = mx * p.scale_log2;
-        float alpha = 1.f;
-        bool rescale = false;
-        if (kv == 0) {
-          m_use = m_tile;
-        } else if (m_tile > m_use + kRescaleThreshold) {
-          alpha = fast_exp2(m_use - m_tile);
-          m_use = m_tile;
-          rescale = true;
-        }
-        // P = exp2(S * scale - m_use): scale-and-subtract and the row sum on fp32 pairs
-        uint32_t pk[BN / 2];
-        uint64_t sum2[4] = {0ull, 0ull, 0ull, 0ull};
-        const uint64_t sc2 = f2_pack(p.scale_log2, p.scale_log2), nm2 = f2_pack(-m_use, -m_use);
-#pragma unroll
-        for (int c = 0; c < BN; c += 2) {
-          float x0, x1;
-          f2_unpack(f2_fma(f2_pack(sv[c], sv[c + 1]), sc2, nm2), x0, x1);
-          const float e0 = fast_exp2(x0), e1 = fast_exp2(x1);
-          sum2[(c >> 1) & 3] = f2_add(sum2[(c >> 1) & 3], f2_pack(e0, e1));
-          pk[c / 2] = pack_bf16x2(e0, e1);
-        }
-        float sa, sb;
-        f2_unpack(f2_add(f2_add(sum2[0], sum2[1]), f2_add(sum2[2], sum2[3])), sa, sb);
-        l_sum = l_sum * alpha + (sa + sb);
-        // P over the S columns just read (every S value is in registers)
-        {
-          uint32_t r[32];
-#pragma unroll
-          for (int i = 0; i < 32; ++i) r[i] = pk[i];
-          tmem_st32(s_addr, r);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) r[i] = pk[32 + i];
-          tmem_st32(s_addr + 32, r);
-        }
-        // O may only be rescaled once the previous PV completed; without a rescale this
-        // tile's softmax does not touch O and overlaps that PV
-        if (kv > 0 && __any_sync(0xffffffffu, rescale)) {
-          ok = wait_pv(tile - 1);
-          if (!ok) break;
-          tc_fence_after();
-          {
-#pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
-              uint32_t r[32];
-              tmem_ld32(o_addr + c * 32, r);
-              tmem_wait_ld();
-#pragma unroll
-              for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-              tmem_st32(o_addr + c * 32, r);
-            }
-          }
-        }
-        tmem_wait_st();
-        tc_fence_before();
+        ok = softmax_tile<D>(s_addr, o_addr, kv, qt, row, p.scale_log2, m_use, l_sum, tile, wait_pv);
+        if (!ok) break;
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars->p_full[tile & 1]);
         if (kv == 0 && valid) gt = ld_issue_f32(p.gate + src);  // used in the epilogue only

@@ -29,14 +29,14 @@ namespace {
 
 constexpr int kChunk = 256;  // tokens per block in the top-K and rank kernels
 
-// TopK and gates of token `tok` (Sec. 3.1 Eq. namoh-gates).  Writes topk_head and gate and
-// returns the picked heads as a bit mask.
+constexpr float kLog2e = 1.4426950408889634f;
+
+// The H logits of token `tok` in registers (independent loads, all in flight together).
+// Non-finite logits become -FLT_MAX and set `bad`.
 template <int HMAX>
-__device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores, size_t tok, int H, int K,
-                                               int32_t* __restrict__ topk_head, float* __restrict__ gate, int* s_bad) {
-  // this token's H logits: independent loads, all in flight together
+__device__ __forceinline__ void load_logits(const float* __restrict__ scores, size_t tok, int H, float (&sc)[HMAX],
+                                            bool& bad) {
   const float* src = scores + tok * H;
-  float sc[HMAX];
   if ((H & 3) == 0 && (reinterpret_cast<uintptr_t>(src) & 15u) == 0) {
 #pragma unroll
     for (int h4 = 0; h4 < HMAX / 4; ++h4) {
@@ -51,7 +51,7 @@ __device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores,
 #pragma unroll
     for (int h = 0; h < HMAX; ++h) sc[h] = (h < H) ? __ldg(src + h) : 0.f;
   }
-  bool bad = false;
+  bad = false;
 #pragma unroll
   for (int h = 0; h < HMAX; ++h) {
     if (h < H && !isfinite(sc[h])) {
@@ -59,21 +59,62 @@ __device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores,
       sc[h] = -FLT_MAX;
     }
   }
-  // softmax denominator over all H logits (fp32); pairwise partial maxima / sums
-  float mx = -FLT_MAX;
+}
+
+// Softmax normaliser over all H logits (Sec. 3.1 Eq. namoh-gates), fp32: the max and
+// 1 / sum_h exp(sc_h - max), each exponential as exp2((sc_h - max) * log2 e).
+template <int HMAX>
+__device__ __forceinline__ void softmax_norm(const float (&sc)[HMAX], int H, float& mx, float& inv_z) {
+  mx = -FLT_MAX;
 #pragma unroll
   for (int h = 0; h < HMAX; ++h)
     if (h < H) mx = fmaxf(mx, sc[h]);
   float z0 = 0.f, z1 = 0.f;
 #pragma unroll
   for (int h = 0; h < HMAX; h += 2) {
-    if (h < H) z0 += expf(sc[h] - mx);
-    if (h + 1 < H) z1 += expf(sc[h + 1] - mx);
+    if (h < H) z0 += fast_exp2((sc[h] - mx) * kLog2e);
+    if (h + 1 < H) z1 += fast_exp2((sc[h + 1] - mx) * kLog2e);
   }
-  const float inv_z = 1.0f / (z0 + z1);
+  inv_z = 1.0f / (z0 + z1);
+}
 
-  // K passes; pass k picks the best head strictly after the previous pick in the
-  // total order (score desc, index asc).
+// Top-K in registers: insertion into a list kept in (score desc, index asc) order.  Heads
+// arrive in increasing index, so a head displaces only strictly smaller scores.  Entries
+// past K are scratch.
+template <int HMAX, int KMAX>
+__device__ __forceinline__ void topk_sorted(const float (&sc)[HMAX], int H, int (&hk)[KMAX], float (&vk)[KMAX]) {
+#pragma unroll
+  for (int k = 0; k < KMAX; ++k) {
+    hk[k] = -1;
+    vk[k] = 0.f;
+  }
+#pragma unroll
+  for (int h = 0; h < HMAX; ++h) {
+    if (h < H) {
+      const float x = sc[h];
+#pragma unroll
+      for (int k = KMAX - 1; k >= 0; --k) {
+        const bool beats_prev = k > 0 && (hk[k > 0 ? k - 1 : 0] < 0 || x > vk[k > 0 ? k - 1 : 0]);
+        const bool beats = hk[k] < 0 || x > vk[k];
+        if (beats_prev) {
+          vk[k] = vk[k > 0 ? k - 1 : 0];
+          hk[k] = hk[k > 0 ? k - 1 : 0];
+        } else if (beats) {
+          vk[k] = x;
+          hk[k] = h;
+        }
+      }
+    }
+  }
+}
+
+// Top-K for any K <= H: pass k picks the best head strictly after the previous pick in the
+// total order (score desc, index asc) and writes it out with its gate.  Returns the picked
+// heads as a bit mask.
+template <int HMAX>
+__device__ __forceinline__ uint64_t topk_passes(const float (&sc)[HMAX], int H, int K, float mx, float inv_z,
+                                                size_t tok, int32_t* __restrict__ topk_head,
+                                                float* __restrict__ gate) {
   float pv = 0.f;
   int pi = -1;
   uint64_t mask = 0;
@@ -90,17 +131,62 @@ __device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores,
       bi = better ? h : bi;
     }
     topk_head[base + k] = bi;
-    gate[base + k] = expf(bv - mx) * inv_z;
+    gate[base + k] = fast_exp2((bv - mx) * kLog2e) * inv_z;
     mask |= 1ull << bi;
     pv = bv;
     pi = bi;
   }
-  if (bad) *s_bad = 1;
   return mask;
 }
 
+// TopK and gates of token `tok` (Sec. 3.1 Eq. namoh-gates), written to topk_head and gate
+// ([tok, K] rows).  With KMAX > 0 (K <= KMAX) the picks also stay in hk for the caller;
+// with KMAX == 0 any K is taken, the picks only go to memory.  Returns the picked heads as a
+// bit mask.
+template <int HMAX, int KMAX>
+__device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores, size_t tok, int H, int K,
+                                               int32_t* __restrict__ topk_head, float* __restrict__ gate, int* s_bad,
+                                               int (&hk)[KMAX > 0 ? KMAX : 1]) {
+  float sc[HMAX];
+  bool bad;
+  load_logits<HMAX>(scores, tok, H, sc, bad);
+  if (bad) *s_bad = 1;
+  float mx, inv_z;
+  softmax_norm<HMAX>(sc, H, mx, inv_z);
+  if constexpr (KMAX == 0) {
+    return topk_passes<HMAX>(sc, H, K, mx, inv_z, tok, topk_head, gate);
+  } else {
+    float vk[KMAX];
+    topk_sorted<HMAX, KMAX>(sc, H, hk, vk);
+    float g[KMAX];
+    uint64_t mask = 0;
+#pragma unroll
+    for (int k = 0; k < KMAX; ++k) {
+      g[k] = fast_exp2((vk[k] - mx) * kLog2e) * inv_z;
+      if (k < K) mask |= 1ull << hk[k];
+    }
+    const size_t base = tok * K;
+    if (KMAX == 4 && K == 4 && (reinterpret_cast<uintptr_t>(topk_head + base) & 15u) == 0 &&
+        (reinterpret_cast<uintptr_t>(gate + base) & 15u) == 0) {
+      *reinterpret_cast<int4*>(topk_head + base) = make_int4(hk[0], hk[KMAX > 1 ? 1 : 0], hk[KMAX > 2 ? 2 : 0],
+                                                             hk[KMAX > 3 ? 3 : 0]);
+      *reinterpret_cast<float4*>(gate + base) = make_float4(g[0], g[KMAX > 1 ? 1 : 0], g[KMAX > 2 ? 2 : 0],
+                                                            g[KMAX > 3 ? 3 : 0]);
+    } else {
+#pragma unroll
+      for (int k = 0; k < KMAX; ++k) {
+        if (k < K) {
+          topk_head[base + k] = hk[k];
+          gate[base + k] = g[k];
+        }
+      }
+    }
+    return mask;
+  }
+}
+
 // TopK and gates only (no packed layout), one thread per token.
-template <int HMAX>
+template <int HMAX, int KMAX>
 __global__ void __launch_bounds__(kChunk) route_topk_kernel(const float* __restrict__ scores, int T, int H, int K,
                                                             int32_t* __restrict__ topk_head, float* __restrict__ gate,
                                                             uint32_t* __restrict__ status) {
@@ -108,7 +194,8 @@ __global__ void __launch_bounds__(kChunk) route_topk_kernel(const float* __restr
   const int t = blockIdx.x * kChunk + threadIdx.x;
   if (threadIdx.x == 0) s_bad = 0;
   __syncthreads();
-  if (t < T) topk_token<HMAX>(scores, (size_t)blockIdx.y * T + t, H, K, topk_head, gate, &s_bad);
+  int hk[KMAX > 0 ? KMAX : 1];
+  if (t < T) topk_token<HMAX, KMAX>(scores, (size_t)blockIdx.y * T + t, H, K, topk_head, gate, &s_bad, hk);
   __syncthreads();
   if (threadIdx.x == 0 && s_bad) report(status, NAMOH_DEV_NONFINITE_SCORE);
 }
@@ -158,7 +245,7 @@ __global__ void __launch_bounds__(1024) route_scan_kernel(const int32_t* __restr
 // the chunk's head counts, and rank_local = the (token, slot)'s rank among this chunk's
 // earlier tokens for its head (Sec. 3.2 Eq. namoh-head-rope restricted to the chunk).
 // rank_local goes to `rank`, which the final pass turns into the full rank.
-template <int HMAX>
+template <int HMAX, int KMAX>
 __global__ void __launch_bounds__(kChunk) route_local_kernel(const float* __restrict__ scores, int T, int H, int K,
                                                              int nchunks, int32_t* __restrict__ topk_head,
                                                              float* __restrict__ gate, int32_t* __restrict__ rank,
@@ -178,7 +265,8 @@ __global__ void __launch_bounds__(kChunk) route_local_kernel(const float* __rest
   // read this call's outputs: nothing global is touched before the wait
   pdl_wait();
   uint64_t mask = 0;
-  if (valid) mask = topk_token<HMAX>(scores, tok, H, K, topk_head, gate, &s_bad);
+  int hk[KMAX > 0 ? KMAX : 1];
+  if (valid) mask = topk_token<HMAX, KMAX>(scores, tok, H, K, topk_head, gate, &s_bad, hk);
   for (int h = 0; h < H; ++h) {
     const uint32_t bal = __ballot_sync(0xffffffffu, (mask >> h) & 1ull);
     if (lane == 0) s_bal[warp][h] = bal;
@@ -193,11 +281,26 @@ __global__ void __launch_bounds__(kChunk) route_local_kernel(const float* __rest
   if (tid == 0 && s_bad) report(status, NAMOH_DEV_NONFINITE_SCORE);
   if (!valid) return;
   const uint32_t lt = (1u << lane) - 1u;
-  for (int k = 0; k < K; ++k) {
-    const int h = topk_head[tok * K + k];  // written above by this thread
+  auto local_rank = [&](int h) {
     int before = 0;
     for (int w = 0; w < warp; ++w) before += __popc(s_bal[w][h]);
-    rank[tok * K + k] = before + __popc(s_bal[warp][h] & lt);
+    return before + __popc(s_bal[warp][h] & lt);
+  };
+  const size_t base = tok * K;
+  if constexpr (KMAX > 0) {
+    int rk[KMAX];
+#pragma unroll
+    for (int k = 0; k < KMAX; ++k) rk[k] = k < K ? local_rank(hk[k]) : 0;
+    if (KMAX == 4 && K == 4 && (reinterpret_cast<uintptr_t>(rank + base) & 15u) == 0) {
+      *reinterpret_cast<int4*>(rank + base) = make_int4(rk[0], rk[KMAX > 1 ? 1 : 0], rk[KMAX > 2 ? 2 : 0],
+                                                        rk[KMAX > 3 ? 3 : 0]);
+    } else {
+#pragma unroll
+      for (int k = 0; k < KMAX; ++k)
+        if (k < K) rank[base + k] = rk[k];
+    }
+  } else {
+    for (int k = 0; k < K; ++k) rank[base + k] = local_rank(topk_head[base + k]);  // written above by this thread
   }
 }
 
@@ -220,7 +323,17 @@ __global__ void __launch_bounds__(kChunk) route_final_kernel(const int32_t* __re
   const int t = c * kChunk + tid;
   const bool valid = t < T;
   const size_t tok = (size_t)b * T + t;
+  const size_t base = tok * K;
   pdl_wait();  // pass 1 (and the scan, when there is one) complete and visible
+  // this token's heads and local ranks first: their loads overlap the count-table work
+  const bool vec4 = K == 4 && (reinterpret_cast<uintptr_t>(topk_head + base) & 15u) == 0 &&
+                    (reinterpret_cast<uintptr_t>(rank + base) & 15u) == 0 &&
+                    (reinterpret_cast<uintptr_t>(row + base) & 15u) == 0;
+  int4 h4 = make_int4(0, 0, 0, 0), r4 = make_int4(0, 0, 0, 0);
+  if (valid && vec4) {
+    h4 = __ldcg(reinterpret_cast<const int4*>(topk_head + base));
+    r4 = __ldcg(reinterpret_cast<const int4*>(rank + base));
+  }
   if (chunk_base) {
     if (tid < H) {
       s_cbase[tid] = chunk_base[((size_t)b * nchunks + c) * H + tid];
@@ -264,8 +377,22 @@ __global__ void __launch_bounds__(kChunk) route_final_kernel(const int32_t* __re
   }
   __syncthreads();
   if (!valid) return;
+  if (vec4) {
+    const int hs[4] = {h4.x, h4.y, h4.z, h4.w}, ls[4] = {r4.x, r4.y, r4.z, r4.w};
+    int rho[4], rw[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      rho[k] = s_cbase[hs[k]] + ls[k];
+      rw[k] = s_soff[hs[k]] + rho[k];
+    }
+    *reinterpret_cast<int4*>(rank + base) = make_int4(rho[0], rho[1], rho[2], rho[3]);
+    *reinterpret_cast<int4*>(row + base) = make_int4(rw[0], rw[1], rw[2], rw[3]);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) row_src[rw[k]] = (int32_t)(base + k);
+    return;
+  }
   for (int k = 0; k < K; ++k) {
-    const size_t i = tok * K + k;
+    const size_t i = base + k;
     const int h = topk_head[i];
     const int rho = s_cbase[h] + rank[i];
     const int r = s_soff[h] + rho;
@@ -288,14 +415,14 @@ struct RouteArgs {
 // pass; larger ones are scanned once by route_scan_kernel.
 constexpr int kFinalMaxTable = 1 << 12;
 
-template <int HMAX>
+template <int HMAX, int KMAX>
 int launch_route(const RouteArgs& a, cudaStream_t stream) {
   const dim3 chunks((unsigned)a.nchunks, (unsigned)a.B);
   if (a.seg_offsets == nullptr) {
-    route_topk_kernel<HMAX><<<chunks, kChunk, 0, stream>>>(a.scores, a.T, a.H, a.K, a.topk_head, a.gate, a.status);
+    route_topk_kernel<HMAX, KMAX><<<chunks, kChunk, 0, stream>>>(a.scores, a.T, a.H, a.K, a.topk_head, a.gate, a.status);
     return cuda_check_launch("route_topk_kernel launch");
   }
-  cudaError_t e = launch_pdl(route_local_kernel<HMAX>, chunks, dim3(kChunk), 0, stream, a.scores, a.T, a.H, a.K,
+  cudaError_t e = launch_pdl(route_local_kernel<HMAX, KMAX>, chunks, dim3(kChunk), 0, stream, a.scores, a.T, a.H, a.K,
                              a.nchunks, a.topk_head, a.gate, a.rank, a.chunk_count, a.status);
   if (e != cudaSuccess) return cuda_fail(e, "route_local_kernel launch");
   const bool scan = (long long)a.nchunks * a.H > kFinalMaxTable;
@@ -357,10 +484,14 @@ extern "C" int namoh_route(const float* scores, int B, int T, int H, int K, int3
     a.chunk_base = ws.take<int32_t>((size_t)B * a.nchunks * H);
     if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
   }
-  if (H <= 8) return launch_route<8>(a, stream);
-  if (H <= 16) return launch_route<16>(a, stream);
-  if (H <= 32) return launch_route<32>(a, stream);
-  return launch_route<64>(a, stream);
+  // picks held in registers for K <= 8; larger K takes K passes over the logits
+  if (H <= 8) return K <= 4 ? launch_route<8, 4>(a, stream) : launch_route<8, 8>(a, stream);
+  if (H <= 16) return K <= 4 ? launch_route<16, 4>(a, stream) : K <= 8 ? launch_route<16, 8>(a, stream)
+                                                                        : launch_route<16, 0>(a, stream);
+  if (H <= 32) return K <= 4 ? launch_route<32, 4>(a, stream) : K <= 8 ? launch_route<32, 8>(a, stream)
+                                                                        : launch_route<32, 0>(a, stream);
+  return K <= 4 ? launch_route<64, 4>(a, stream) : K <= 8 ? launch_route<64, 8>(a, stream)
+                                                          : launch_route<64, 0>(a, stream);
 }
 
 // ---------------------------------------------------------------------------
