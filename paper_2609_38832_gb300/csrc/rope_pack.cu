@@ -22,6 +22,9 @@ namespace namoh {
 constexpr int kRopeThreads = 256;
 constexpr int kRopeStages = 3;
 constexpr int kRopeStageMax = 8192;  // seg_offsets entries staged in shared memory (32 KB)
+constexpr size_t kSmemPerSm = 233472;  // shared memory per SM (228 KB); each resident block also takes 1 KB
+// the least dynamic shared memory with which three blocks no longer fit on one SM
+constexpr size_t kSmemThirdPlus = kSmemPerSm / 3 - 1024 + 16;
 
 template <int D, int G>
 struct RopeChunk {
@@ -196,9 +199,12 @@ cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, 
   case GG: {                                                                                                      \
     using C = RopeChunk<D, GG>;                                                                                  \
     const size_t rope_smem = rope_smem_bytes<D, GG>(nseg);                                                       \
-    const size_t smem = rope_smem > plan_smem ? rope_smem : plan_smem;                                           \
-    /* two blocks per SM when their shared memory fits (228 KB per SM, 1 KB reserved per block) */              \
-    const int per_sm = (smem + 1024) * 2 <= 233472 ? 2 : 1;                                                      \
+    const size_t smem0 = rope_smem > plan_smem ? rope_smem : plan_smem;                                          \
+    /* two blocks per SM when their shared memory fits (228 KB per SM, 1 KB reserved per block); the */          \
+    /* block scheduler packs blocks as deep as resources allow, so each block also asks for more than */          \
+    /* a third of the SM, which keeps it to two per SM and spreads the grid over every SM */                     \
+    const int per_sm = (smem0 + 1024) * 2 <= kSmemPerSm ? 2 : 1;                                                  \
+    const size_t smem = per_sm == 2 && smem0 < kSmemThirdPlus ? kSmemThirdPlus : smem0;                          \
     const long long nchunks = ((long long)R + C::kRows - 1) / C::kRows;                                        \
     long long blocks = (long long)per_sm * sm_count;                                                             \
     if (blocks > nchunks) blocks = nchunks;                                                                      \
