@@ -51,12 +51,20 @@ __device__ __forceinline__ void load_logits(const float* __restrict__ scores, si
 #pragma unroll
     for (int h = 0; h < HMAX; ++h) sc[h] = (h < H) ? __ldg(src + h) : 0.f;
   }
-  bad = false;
+  // one sum decides whether any logit needs looking at (it is non-finite when one is, or on
+  // overflow, where the per-logit check then finds nothing to replace)
+  float total = 0.f;
 #pragma unroll
-  for (int h = 0; h < HMAX; ++h) {
-    if (h < H && !isfinite(sc[h])) {
-      bad = true;
-      sc[h] = -FLT_MAX;
+  for (int h = 0; h < HMAX; ++h)
+    if (h < H) total += sc[h];
+  bad = false;
+  if (!isfinite(total)) {
+#pragma unroll
+    for (int h = 0; h < HMAX; ++h) {
+      if (h < H && !isfinite(sc[h])) {
+        bad = true;
+        sc[h] = -FLT_MAX;
+      }
     }
   }
 }
@@ -79,31 +87,30 @@ __device__ __forceinline__ void softmax_norm(const float (&sc)[HMAX], int H, flo
 }
 
 // Top-K in registers: insertion into a list kept in (score desc, index asc) order.  Heads
-// arrive in increasing index, so a head displaces only strictly smaller scores.  Entries
-// past K are scratch.
+// arrive in increasing index, so a head displaces only strictly smaller scores.  Empty
+// entries hold -inf, which every (finite) logit beats; entries past K are scratch.
 template <int HMAX, int KMAX>
 __device__ __forceinline__ void topk_sorted(const float (&sc)[HMAX], int H, int (&hk)[KMAX], float (&vk)[KMAX]) {
 #pragma unroll
   for (int k = 0; k < KMAX; ++k) {
-    hk[k] = -1;
-    vk[k] = 0.f;
+    hk[k] = 0;
+    vk[k] = -INFINITY;
   }
 #pragma unroll
   for (int h = 0; h < HMAX; ++h) {
     if (h < H) {
       const float x = sc[h];
+      bool beats[KMAX];
 #pragma unroll
-      for (int k = KMAX - 1; k >= 0; --k) {
-        const bool beats_prev = k > 0 && (hk[k > 0 ? k - 1 : 0] < 0 || x > vk[k > 0 ? k - 1 : 0]);
-        const bool beats = hk[k] < 0 || x > vk[k];
-        if (beats_prev) {
-          vk[k] = vk[k > 0 ? k - 1 : 0];
-          hk[k] = hk[k > 0 ? k - 1 : 0];
-        } else if (beats) {
-          vk[k] = x;
-          hk[k] = h;
-        }
+      for (int k = 0; k < KMAX; ++k) beats[k] = x > vk[k];
+      // entry k takes entry k-1 when x beats that too, else x when x beats entry k
+#pragma unroll
+      for (int k = KMAX - 1; k >= 1; --k) {
+        vk[k] = beats[k - 1] ? vk[k - 1] : (beats[k] ? x : vk[k]);
+        hk[k] = beats[k - 1] ? hk[k - 1] : (beats[k] ? h : hk[k]);
       }
+      vk[0] = beats[0] ? x : vk[0];
+      hk[0] = beats[0] ? h : hk[0];
     }
   }
 }
