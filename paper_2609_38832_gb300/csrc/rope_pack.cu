@@ -206,7 +206,8 @@ cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, 
     const int per_sm = (smem0 + 1024) * 2 <= kSmemPerSm ? 2 : 1;                                                  \
     const size_t smem = per_sm == 2 && smem0 < kSmemThirdPlus ? kSmemThirdPlus : smem0;                          \
     const long long nchunks = ((long long)R + C::kRows - 1) / C::kRows;                                        \
-    long long blocks = (long long)per_sm * sm_count;                                                             \
+    /* the plan block takes one of the per_sm * sm_count slots: the whole grid is resident at once */          \
+    long long blocks = (long long)per_sm * sm_count - (with_plan ? 1 : 0);                                       \
     if (blocks > nchunks) blocks = nchunks;                                                                      \
     const long long grid = blocks + (with_plan ? 1 : 0);                                                         \
     if (grid == 0) return cudaSuccess;                                                                           \
