@@ -2,10 +2,12 @@
 // execution": length-aware scheduling of query tiles).
 //
 // Items are the 128-row query tiles q of every segment and group head j, ordered by
-// decreasing cost (tile q needs q + 1 key tiles), then (segment, j).  Segments longer
-// than their cache capacity (seg_cap, when given) are left out.  The header holds
-// {next item, CTAs finished, item count}; the attention kernel takes items in order
-// from an atomic counter and its last CTA resets the first two words.
+// decreasing cost (tile q needs q + 1 key tiles), then (segment, j).  Each item carries
+// {segment * g + j, q, seg_offsets[segment], n}, so a CTA starts on it after one load.
+// Segments longer than their cache capacity (seg_cap, when given) are left out.  The
+// header holds {next item, CTAs finished, item count}; the attention kernel's CTAs take
+// item blockIdx first and then items in order from an atomic counter, and its last CTA
+// resets the first two words.
 #pragma once
 
 #include "common.cuh"
@@ -19,7 +21,7 @@ __host__ __device__ inline int plan_smem_ints(int max_qtiles, int nseg) { return
 
 // Executed by one whole block (any size) with plan_smem_ints(...) ints of shared memory.
 __device__ inline void build_plan(const int32_t* __restrict__ seg_offsets, int nseg, const int32_t* __restrict__ seg_cap,
-                                  int g, int max_qtiles, int* __restrict__ header, int2* __restrict__ items,
+                                  int g, int max_qtiles, int* __restrict__ header, int4* __restrict__ items,
                                   int* s_mem) {
   int* s_count = s_mem;                   // [max_qtiles]: segments with more than q query tiles
   int* s_start = s_mem + max_qtiles;      // [max_qtiles]: first item of cost q + 1
@@ -52,8 +54,10 @@ __device__ inline void build_plan(const int32_t* __restrict__ seg_offsets, int n
     if (s_count[q] == 0) continue;
     int pos = s_start[q];
     for (int s = 0; s < nseg; ++s)
-      if (s_ntile[s] > q)
-        for (int j = 0; j < g; ++j) items[pos++] = make_int2(s * g + j, q);
+      if (s_ntile[s] > q) {
+        const int off = __ldg(seg_offsets + s), n = __ldg(seg_offsets + s + 1) - off;
+        for (int j = 0; j < g; ++j) items[pos++] = make_int4(s * g + j, q, off, n);
+      }
   }
 }
 

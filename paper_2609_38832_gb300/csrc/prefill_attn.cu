@@ -101,7 +101,7 @@ struct Params {
   const int64_t* seg_base;     // [nseg] or null (cache rows = packed rows)
   const int32_t* row_src;      // [R]
   const float* gate;           // [R] indexed by row_src value
-  const int2* items;           // {segment * g + j, query tile}, longest first
+  const int4* items;           // {segment * g + j, query tile, seg_offsets[segment], n}, longest first
   const int* nitems;
   int* sched;                  // [0] next item, [1] CTAs finished
   uint16_t* y;                 // [R * g, D] indexed by row_src * g + j
@@ -299,16 +299,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         return true;
       };
       while (ok) {
-        const int it = atomicAdd(p.sched, 1);
-        // the segment's offsets travel with the item, so no consumer loads them
+        // the first item is this CTA's own (the plan's G longest tiles go one per CTA), later
+        // ones come from the counter; the segment's offset and length travel with the item
+        const int it = item_iter == 0 ? (int)blockIdx.x : G + atomicAdd(p.sched, 1);
         int4 item = make_int4(-1, -1, 0, 0);
         int kvb = 0;
         if (it < nitems) {
-          const int2 w = p.items[it];
-          const int sg = w.x / p.g;
-          const int o = p.seg_offsets[sg];
-          item = make_int4(w.x, w.y, o, p.seg_offsets[sg + 1] - o);
-          kvb = (int)(p.seg_base ? p.seg_base[sg] : (long long)o);
+          item = p.items[it];
+          kvb = (int)(p.seg_base ? p.seg_base[item.x / p.g] : (long long)item.z);
         }
         const int slot = item_iter & 1;
         if (item_iter >= 2) ok = mbar_wait(&bars->item_empty[slot], ((item_iter >> 1) - 1) & 1, abort_flag, p.status);
@@ -585,7 +583,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // One block builds the work list (see build_plan) and zeroes the scheduler's counters.
 __global__ void __launch_bounds__(1024) plan_kernel(const int32_t* __restrict__ seg_offsets, int nseg,
                                                     const int32_t* __restrict__ seg_cap, int g, int max_qtiles,
-                                                    int* __restrict__ header, int2* __restrict__ items) {
+                                                    int* __restrict__ header, int4* __restrict__ items) {
   extern __shared__ int s_dyn[];
   build_plan(seg_offsets, nseg, seg_cap, g, max_qtiles, header, items, s_dyn);
 }
@@ -645,7 +643,7 @@ int check_shape(int B, int T, int H, int K, int d_head, int group, int* Hr, int*
 size_t plan_bytes_for(int B, int T, int Hr, int Kr, int g) {
   const long long R = (long long)B * T * Kr;
   const long long max_items = ((R + attn::kItemRows - 1) / attn::kItemRows + (long long)B * Hr) * g;
-  return 16 + (size_t)max_items * sizeof(int2);
+  return 16 + (size_t)max_items * sizeof(int4);
 }
 
 int plan_qtiles_for(int T) { return (T + kPlanTileRows - 1) / kPlanTileRows; }  // query tiles per segment, at most
@@ -664,7 +662,7 @@ int launch_plan(const int32_t* seg_offsets, int nseg, int T, int g, const int32_
     if (e != cudaSuccess) return cuda_fail(e, "plan_kernel shared memory attribute");
   }
   int* header = static_cast<int*>(plan);
-  int2* items = reinterpret_cast<int2*>(static_cast<char*>(plan) + 16);
+  int4* items = reinterpret_cast<int4*>(static_cast<char*>(plan) + 16);
   attn::plan_kernel<<<1, 1024, smem, stream>>>(seg_offsets, nseg, seg_cap, g, max_qtiles, header, items);
   return cuda_check_launch("plan_kernel launch");
 }
@@ -706,7 +704,7 @@ int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint1
   p.gate = gate;
   p.sched = static_cast<int*>(plan);
   p.nitems = static_cast<int*>(plan) + 2;
-  p.items = reinterpret_cast<const int2*>(static_cast<char*>(plan) + 16);
+  p.items = reinterpret_cast<const int4*>(static_cast<char*>(plan) + 16);
   p.y = y;
   p.g = g;
   p.y_sector_aligned = (reinterpret_cast<uintptr_t>(y) & 31u) == 0;

@@ -54,7 +54,7 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     const int32_t* __restrict__ seg_offsets, int nseg, const int64_t* __restrict__ seg_base,
     const int32_t* __restrict__ seg_cap, long long cache_rows, uint16_t* __restrict__ q_rot,
     uint16_t* __restrict__ k_cache, uint16_t* __restrict__ v_cache, int copy_v, RopeTable tab,
-    uint32_t* __restrict__ status, int* __restrict__ plan_header, int2* __restrict__ plan_items,
+    uint32_t* __restrict__ status, int* __restrict__ plan_header, int4* __restrict__ plan_items,
     const int32_t* __restrict__ plan_cap, int plan_qtiles) {
   using C = RopeChunk<D, G>;
   constexpr int HALF = D / 2;
@@ -193,7 +193,7 @@ cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, 
                                const int32_t* seg_offsets, const int64_t* seg_base, const int32_t* seg_cap,
                                long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache,
                                int copy_v, const RopeTable& tab, uint32_t* status, int* plan_header,
-                               int2* plan_items, const int32_t* plan_cap, int plan_qtiles) {
+                               int4* plan_items, const int32_t* plan_cap, int plan_qtiles) {
   switch (g) {
 #define NAMOH_ROPE_CASE(GG)                                                                                       \
   case GG: {                                                                                                      \
@@ -237,7 +237,7 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream,
                              void* plan, int plan_qtiles, const int32_t* plan_cap) {
   int* plan_header = static_cast<int*>(plan);
-  int2* plan_items = plan ? reinterpret_cast<int2*>(static_cast<char*>(plan) + 16) : nullptr;
+  int4* plan_items = plan ? reinterpret_cast<int4*>(static_cast<char*>(plan) + 16) : nullptr;
   const size_t plan_smem = plan ? (size_t)plan_smem_ints(plan_qtiles, nseg) * sizeof(int) : 0;
   if (R == 0 && !plan) return cudaSuccess;
   if (D == 128)
