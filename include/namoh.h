@@ -112,6 +112,23 @@ NAMOH_API int namoh_route(const float *scores, int B, int T, int H, int K, int32
                 size_t workspace_bytes, uint32_t *dev_status, void *stream);
 
 /* ------------------------------------------------------------------------- *
+ * namoh_route_biased: routing with loss-free balancing biases (App. A,
+ *   Eq. namoh-biased-routing): S_K(t) = TopK_i(a_{t,i} + b_i) on the softmax
+ *   affinities plus a per-head bias, ties to the lower head index; the gates stay
+ *   g_{t,i} = a_{t,i} (the bias does not enter them, no renormalisation).
+ * bias  [H] fp32 device array, finite, caller-owned, read-only; NULL gives
+ *       exactly namoh_route.
+ * Everything else (arguments, outputs, layout, errors) is as namoh_route.  The
+ * affinities are fp32 (exp2 of pre-scaled logit differences), so where two
+ * biased affinities lie within a few fp32 ulps of each other the order between
+ * them is the fp32 one.
+ * ------------------------------------------------------------------------- */
+NAMOH_API int namoh_route_biased(const float *scores, const float *bias, int B, int T, int H, int K,
+                                 int32_t *topk_head, float *gate, int32_t *rank, int32_t *row, int32_t *seg_offsets,
+                                 int32_t *row_src, void *workspace, size_t workspace_bytes, uint32_t *dev_status,
+                                 void *stream);
+
+/* ------------------------------------------------------------------------- *
  * namoh_route_noalloc: namoh_route without a workspace argument.
  * The paper has no counterpart; this is a convenience of this library.
  *

@@ -67,6 +67,7 @@ def _load():
         P = ctypes.c_void_p
         i32, i64, f64 = ctypes.c_int, ctypes.c_long, ctypes.c_double
         lib.oracle_route_topk.argtypes = [P, i64, i32, i32, P, P]
+        lib.oracle_route_biased.argtypes = [P, P, i64, i32, i32, P, P, P]
         lib.oracle_dispatch.argtypes = [P, i32, i32, i32, i32, P, P, P, P, P]
         lib.oracle_rope.argtypes = [P, i64, i32, i64, P, f64, P]
         lib.oracle_prefill.argtypes = [P, P, P, i32, i32, i32, f64, P, P, P, P, P, i32]
@@ -74,7 +75,7 @@ def _load():
         lib.oracle_decode_step.argtypes = [P, P, P, P, P, i32, i32, i32, i32, i32, f64,
                                            P, P, P, P, P, P]
         lib.oracle_default_threads.argtypes = []
-        for fn in ("oracle_route_topk", "oracle_dispatch", "oracle_rope", "oracle_prefill",
+        for fn in ("oracle_route_topk", "oracle_route_biased", "oracle_dispatch", "oracle_rope", "oracle_prefill",
                    "oracle_prefill_rows", "oracle_decode_step", "oracle_default_threads"):
             getattr(lib, fn).restype = ctypes.c_int
         _lib = lib
@@ -114,6 +115,42 @@ def route(scores: np.ndarray, K: int) -> dict:
     _check(lib.oracle_dispatch(_ptr(topk), B, T, H, K, _ptr(n), _ptr(seg), _ptr(rank), _ptr(row),
                                _ptr(row_src)), "dispatch")
     return dict(topk_head=topk, gate=gate, n=n, seg_offsets=seg, rank=rank, row=row, row_src=row_src)
+
+
+def dispatch(topk_head: np.ndarray, H: int) -> dict:
+    """Dispatch (Sec. 3.1 index sets, Sec. 3.2 ranks and packing) of given picks topk_head [B, T, K]."""
+    lib = _load()
+    topk = np.ascontiguousarray(topk_head, dtype=np.int32)
+    B, T, K = topk.shape
+    n = np.empty((B, H), np.int32)
+    seg = np.empty(B * H + 1, np.int32)
+    rank = np.empty((B, T, K), np.int32)
+    row = np.empty((B, T, K), np.int32)
+    row_src = np.empty(B * T * K, np.int32)
+    _check(lib.oracle_dispatch(_ptr(topk), B, T, H, K, _ptr(n), _ptr(seg), _ptr(rank), _ptr(row),
+                               _ptr(row_src)), "dispatch")
+    return dict(n=n, seg_offsets=seg, rank=rank, row=row, row_src=row_src)
+
+
+def route_biased(scores: np.ndarray, K: int, bias: np.ndarray) -> dict:
+    """Biased routing (App. A, Eq. namoh-biased-routing) and dispatch for scores [B, T, H].
+
+    As route(), plus key [B, T, H] = a + b in fp64, the quantity the selection ranks.
+    """
+    lib = _load()
+    scores = np.ascontiguousarray(scores, dtype=np.float32)
+    bias = np.ascontiguousarray(bias, dtype=np.float32)
+    B, T, H = scores.shape
+    if bias.shape != (H,):
+        raise ValueError("bias must have shape [H]")
+    topk = np.empty((B, T, K), np.int32)
+    gate = np.empty((B, T, K), np.float64)
+    key = np.empty((B, T, H), np.float64)
+    _check(lib.oracle_route_biased(_ptr(scores), _ptr(bias), B * T, H, K, _ptr(topk), _ptr(gate), _ptr(key)),
+           "route_biased")
+    out = dispatch(topk, H)
+    out.update(topk_head=topk, gate=gate, key=key)
+    return out
 
 
 def rope(x_bits: np.ndarray, pos: np.ndarray, base: float) -> np.ndarray:

@@ -147,6 +147,58 @@ int oracle_route_topk(const float *scores, long N, int H, int K, int32_t *topk_h
 }
 
 /*
+ * oracle_route_biased: App. A, Eq. (namoh-biased-routing).  In fp64, per token:
+ *   a_t = softmax(x_t W_r) over all H heads,
+ *   S_K(t) = TopK_i(a_{t,i} + b_i)  (larger first, ties to the lower index),
+ *   g_{t,i} = a_{t,i} at the selected heads (the bias stays out of the gates).
+ *   bias      [H] fp32 per-head biases
+ *   topk_head [N, K], gate [N, K] as oracle_route_topk
+ *   key       [N, H] out: a_{t,i} + b_i, the quantity the selection ranks
+ */
+int oracle_route_biased(const float *scores, const float *bias, long N, int H, int K, int32_t *topk_head,
+                        double *gate, double *key)
+{
+    if (!scores || !bias || !topk_head || !gate || !key || N < 0 || H < 1 || K < 1 || K > H || H > 1024)
+        return ORACLE_ERR_ARG;
+    int order[1024];
+    double a[1024];
+    for (int i = 0; i < H; ++i)
+        if (!isfinite(bias[i])) return ORACLE_ERR_NONFINITE;
+    for (long t = 0; t < N; ++t) {
+        const float *s = scores + t * (long)H;
+        double *kt = key + t * (long)H;
+        double mx = -INFINITY;
+        for (int i = 0; i < H; ++i) {
+            if (!isfinite(s[i])) return ORACLE_ERR_NONFINITE;
+            if ((double)s[i] > mx) mx = (double)s[i];
+        }
+        double z = 0.0;
+        for (int i = 0; i < H; ++i) {
+            a[i] = exp((double)s[i] - mx);
+            z += a[i];
+        }
+        for (int i = 0; i < H; ++i) {
+            a[i] /= z;
+            kt[i] = a[i] + (double)bias[i];
+        }
+        /* insertion sort of head indices by (key desc, index asc) */
+        for (int i = 0; i < H; ++i) {
+            int j = i;
+            while (j > 0 && kt[i] > kt[order[j - 1]]) {
+                order[j] = order[j - 1];
+                --j;
+            }
+            order[j] = i;
+        }
+        for (int k = 0; k < K; ++k) {
+            topk_head[t * K + k] = order[k];
+            gate[t * K + k] = a[order[k]];
+        }
+    }
+    return ORACLE_OK;
+}
+
+/*
  * oracle_dispatch: ordered index sets I_i per (batch, head), walking t = 0..T-1
  * and appending each token to the heads it selected.
  *   topk_head   [B, T, K]

@@ -77,13 +77,19 @@ class RouteOutputs:
 
 def namoh_route(scores: torch.Tensor, K: int, compact: bool = True, workspace: Optional[Workspace] = None,
                 status: Optional[torch.Tensor] = None, out: Optional[RouteOutputs] = None,
-                stream=None) -> RouteOutputs:
-    """Routing and dispatch of scores [B, T, H] fp32 (see namoh_route in include/namoh.h)."""
+                stream=None, bias: Optional[torch.Tensor] = None) -> RouteOutputs:
+    """Routing and dispatch of scores [B, T, H] fp32 (see namoh_route in include/namoh.h).
+
+    With ``bias`` ([H] fp32 on the device) the selection is TopK(a + b) on the softmax
+    affinities while the gates stay a (namoh_route_biased)."""
     lib = _abi.load()
     if scores.dtype != torch.float32 or scores.dim() != 3:
         raise ValueError("scores must be a [B, T, H] float32 tensor")
     B, T, H = scores.shape
     dev = scores.device
+    if bias is not None and (bias.dtype != torch.float32 or bias.shape != (H,) or bias.device != dev
+                             or not bias.is_contiguous()):
+        raise ValueError("bias must be a contiguous [H] float32 tensor on the scores' device")
     if out is None:
         i32 = dict(dtype=torch.int32, device=dev)
         out = RouteOutputs(
@@ -95,10 +101,12 @@ def namoh_route(scores: torch.Tensor, K: int, compact: bool = True, workspace: O
             status=_status(status, dev))
     nbytes = lib.namoh_route_workspace_size(B, T, H, K)
     ws = _ws(workspace, nbytes, dev)
-    rc = lib.namoh_route(_ptr(scores), B, T, H, K, _ptr(out.topk_head), _ptr(out.gate), _ptr(out.rank), _ptr(out.row),
-                         _ptr(out.seg_offsets), _ptr(out.row_src), _ptr(ws), ws.numel(), _ptr(out.status),
-                         _stream(stream))
-    _abi.check("namoh_route", rc)
+    outs = (_ptr(out.topk_head), _ptr(out.gate), _ptr(out.rank), _ptr(out.row), _ptr(out.seg_offsets),
+            _ptr(out.row_src), _ptr(ws), ws.numel(), _ptr(out.status), _stream(stream))
+    if bias is None:
+        _abi.check("namoh_route", lib.namoh_route(_ptr(scores), B, T, H, K, *outs))
+    else:
+        _abi.check("namoh_route_biased", lib.namoh_route_biased(_ptr(scores), _ptr(bias), B, T, H, K, *outs))
     return out
 
 

@@ -35,6 +35,7 @@ SIGNATURES = {
     "namoh_last_error_string": (ctypes.c_char_p, []),
     "namoh_route_workspace_size": (_SZ, [_I, _I, _I, _I]),
     "namoh_route": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P]),
+    "namoh_route_biased": (_I, [_P, _P, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P]),
     "namoh_route_noalloc": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P]),
     "namoh_prefill_workspace_size": (_SZ, [_I, _I, _I, _I, _I, _I]),
     "namoh_prefill": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _P, _P, _P, _I64, _P, _P,

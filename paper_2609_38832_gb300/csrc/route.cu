@@ -118,9 +118,9 @@ __device__ __forceinline__ void topk_sorted(const float (&sc)[HMAX], int H, int 
 // Top-K for any K <= H: pass k picks the best head strictly after the previous pick in the
 // total order (score desc, index asc) and writes it out with its gate.  Returns the picked
 // heads as a bit mask.
-template <int HMAX>
-__device__ __forceinline__ uint64_t topk_passes(const float (&sc)[HMAX], int H, int K, float mx, float inv_z,
-                                                size_t tok, int32_t* __restrict__ topk_head,
+template <int HMAX, bool kBiased>
+__device__ __forceinline__ uint64_t topk_passes(const float (&sc)[HMAX], const float (&a)[HMAX], int H, int K,
+                                                float mx, float inv_z, size_t tok, int32_t* __restrict__ topk_head,
                                                 float* __restrict__ gate) {
   float pv = 0.f;
   int pi = -1;
@@ -138,7 +138,7 @@ __device__ __forceinline__ uint64_t topk_passes(const float (&sc)[HMAX], int H, 
       bi = better ? h : bi;
     }
     topk_head[base + k] = bi;
-    gate[base + k] = fast_exp2((bv - mx) * kLog2e) * inv_z;
+    gate[base + k] = kBiased ? a[bi] : fast_exp2((bv - mx) * kLog2e) * inv_z;
     mask |= 1ull << bi;
     pv = bv;
     pi = bi;
@@ -148,11 +148,13 @@ __device__ __forceinline__ uint64_t topk_passes(const float (&sc)[HMAX], int H, 
 
 // TopK and gates of token `tok` (Sec. 3.1 Eq. namoh-gates), written to topk_head and gate
 // ([tok, K] rows).  With KMAX > 0 (K <= KMAX) the picks also stay in hk for the caller;
-// with KMAX == 0 any K is taken, the picks only go to memory.  Returns the picked heads as a
-// bit mask.
-template <int HMAX, int KMAX>
-__device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores, size_t tok, int H, int K,
-                                               int32_t* __restrict__ topk_head, float* __restrict__ gate, int* s_bad,
+// with KMAX == 0 any K is taken, the picks only go to memory.  kBiased: selection on the
+// biased affinities a + b, gates still a (App. A, Eq. namoh-biased-routing).  Returns the
+// picked heads as a bit mask.
+template <int HMAX, int KMAX, bool kBiased>
+__device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores, const float* __restrict__ bias,
+                                               size_t tok, int H, int K, int32_t* __restrict__ topk_head,
+                                               float* __restrict__ gate, int* s_bad,
                                                int (&hk)[KMAX > 0 ? KMAX : 1]) {
   float sc[HMAX];
   bool bad;
@@ -160,8 +162,18 @@ __device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores,
   if (bad) *s_bad = 1;
   float mx, inv_z;
   softmax_norm<HMAX>(sc, H, mx, inv_z);
+  // biased selection ranks the affinities a_h plus the head biases b_h; without a bias the
+  // logits themselves are ranked (softmax is monotone)
+  float a[HMAX];
+  if constexpr (kBiased) {
+#pragma unroll
+    for (int h = 0; h < HMAX; ++h) {
+      a[h] = h < H ? fast_exp2((sc[h] - mx) * kLog2e) * inv_z : 0.f;
+      sc[h] = h < H ? a[h] + __ldg(bias + h) : 0.f;
+    }
+  }
   if constexpr (KMAX == 0) {
-    return topk_passes<HMAX>(sc, H, K, mx, inv_z, tok, topk_head, gate);
+    return topk_passes<HMAX, kBiased>(sc, a, H, K, mx, inv_z, tok, topk_head, gate);
   } else {
     float vk[KMAX];
     topk_sorted<HMAX, KMAX>(sc, H, hk, vk);
@@ -169,7 +181,14 @@ __device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores,
     uint64_t mask = 0;
 #pragma unroll
     for (int k = 0; k < KMAX; ++k) {
-      g[k] = fast_exp2((vk[k] - mx) * kLog2e) * inv_z;
+      if constexpr (kBiased) {
+        float ge = 0.f;
+#pragma unroll
+        for (int h = 0; h < HMAX; ++h) ge = (h == hk[k]) ? a[h] : ge;
+        g[k] = ge;
+      } else {
+        g[k] = fast_exp2((vk[k] - mx) * kLog2e) * inv_z;
+      }
       if (k < K) mask |= 1ull << hk[k];
     }
     const size_t base = tok * K;
@@ -193,8 +212,9 @@ __device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores,
 }
 
 // TopK and gates only (no packed layout), one thread per token.
-template <int HMAX, int KMAX>
-__global__ void __launch_bounds__(kChunk) route_topk_kernel(const float* __restrict__ scores, int T, int H, int K,
+template <int HMAX, int KMAX, bool kBiased>
+__global__ void __launch_bounds__(kChunk) route_topk_kernel(const float* __restrict__ scores,
+                                                            const float* __restrict__ bias, int T, int H, int K,
                                                             int32_t* __restrict__ topk_head, float* __restrict__ gate,
                                                             uint32_t* __restrict__ status) {
   __shared__ int s_bad;
@@ -202,7 +222,7 @@ __global__ void __launch_bounds__(kChunk) route_topk_kernel(const float* __restr
   if (threadIdx.x == 0) s_bad = 0;
   __syncthreads();
   int hk[KMAX > 0 ? KMAX : 1];
-  if (t < T) topk_token<HMAX, KMAX>(scores, (size_t)blockIdx.y * T + t, H, K, topk_head, gate, &s_bad, hk);
+  if (t < T) topk_token<HMAX, KMAX, kBiased>(scores, bias, (size_t)blockIdx.y * T + t, H, K, topk_head, gate, &s_bad, hk);
   __syncthreads();
   if (threadIdx.x == 0 && s_bad) report(status, NAMOH_DEV_NONFINITE_SCORE);
 }
@@ -252,8 +272,9 @@ __global__ void __launch_bounds__(1024) route_scan_kernel(const int32_t* __restr
 // the chunk's head counts, and rank_local = the (token, slot)'s rank among this chunk's
 // earlier tokens for its head (Sec. 3.2 Eq. namoh-head-rope restricted to the chunk).
 // rank_local goes to `rank`, which the final pass turns into the full rank.
-template <int HMAX, int KMAX>
-__global__ void __launch_bounds__(kChunk) route_local_kernel(const float* __restrict__ scores, int T, int H, int K,
+template <int HMAX, int KMAX, bool kBiased>
+__global__ void __launch_bounds__(kChunk) route_local_kernel(const float* __restrict__ scores,
+                                                             const float* __restrict__ bias, int T, int H, int K,
                                                              int nchunks, int32_t* __restrict__ topk_head,
                                                              float* __restrict__ gate, int32_t* __restrict__ rank,
                                                              int32_t* __restrict__ chunk_count,
@@ -273,7 +294,7 @@ __global__ void __launch_bounds__(kChunk) route_local_kernel(const float* __rest
   pdl_wait();
   uint64_t mask = 0;
   int hk[KMAX > 0 ? KMAX : 1];
-  if (valid) mask = topk_token<HMAX, KMAX>(scores, tok, H, K, topk_head, gate, &s_bad, hk);
+  if (valid) mask = topk_token<HMAX, KMAX, kBiased>(scores, bias, tok, H, K, topk_head, gate, &s_bad, hk);
   for (int h = 0; h < H; ++h) {
     const uint32_t bal = __ballot_sync(0xffffffffu, (mask >> h) & 1ull);
     if (lane == 0) s_bal[warp][h] = bal;
@@ -411,6 +432,7 @@ __global__ void __launch_bounds__(kChunk) route_final_kernel(const int32_t* __re
 
 struct RouteArgs {
   const float* scores;
+  const float* bias;  // [H] or nullptr
   int B, T, H, K, nchunks;
   int32_t *topk_head, *rank, *row, *seg_offsets, *row_src;
   float* gate;
@@ -422,15 +444,16 @@ struct RouteArgs {
 // pass; larger ones are scanned once by route_scan_kernel.
 constexpr int kFinalMaxTable = 1 << 12;
 
-template <int HMAX, int KMAX>
+template <int HMAX, int KMAX, bool kBiased>
 int launch_route(const RouteArgs& a, cudaStream_t stream) {
   const dim3 chunks((unsigned)a.nchunks, (unsigned)a.B);
   if (a.seg_offsets == nullptr) {
-    route_topk_kernel<HMAX, KMAX><<<chunks, kChunk, 0, stream>>>(a.scores, a.T, a.H, a.K, a.topk_head, a.gate, a.status);
+    route_topk_kernel<HMAX, KMAX, kBiased><<<chunks, kChunk, 0, stream>>>(a.scores, a.bias, a.T, a.H, a.K, a.topk_head,
+                                                                          a.gate, a.status);
     return cuda_check_launch("route_topk_kernel launch");
   }
-  cudaError_t e = launch_pdl(route_local_kernel<HMAX, KMAX>, chunks, dim3(kChunk), 0, stream, a.scores, a.T, a.H, a.K,
-                             a.nchunks, a.topk_head, a.gate, a.rank, a.chunk_count, a.status);
+  cudaError_t e = launch_pdl(route_local_kernel<HMAX, KMAX, kBiased>, chunks, dim3(kChunk), 0, stream, a.scores, a.bias,
+                             a.T, a.H, a.K, a.nchunks, a.topk_head, a.gate, a.rank, a.chunk_count, a.status);
   if (e != cudaSuccess) return cuda_fail(e, "route_local_kernel launch");
   const bool scan = (long long)a.nchunks * a.H > kFinalMaxTable;
   if (scan) {
@@ -444,6 +467,21 @@ int launch_route(const RouteArgs& a, cudaStream_t stream) {
                  a.row, a.seg_offsets, a.row_src, a.B);
   if (e != cudaSuccess) return cuda_fail(e, "route_final_kernel launch");
   return NAMOH_OK;
+}
+
+// picks held in registers for K <= 8; larger K takes K passes over the logits
+template <bool kBiased>
+int launch_route_h(const RouteArgs& a, cudaStream_t stream) {
+  const int H = a.H, K = a.K;
+  if (H <= 8) return K <= 4 ? launch_route<8, 4, kBiased>(a, stream) : launch_route<8, 8, kBiased>(a, stream);
+  if (H <= 16)
+    return K <= 4 ? launch_route<16, 4, kBiased>(a, stream)
+                  : K <= 8 ? launch_route<16, 8, kBiased>(a, stream) : launch_route<16, 0, kBiased>(a, stream);
+  if (H <= 32)
+    return K <= 4 ? launch_route<32, 4, kBiased>(a, stream)
+                  : K <= 8 ? launch_route<32, 8, kBiased>(a, stream) : launch_route<32, 0, kBiased>(a, stream);
+  return K <= 4 ? launch_route<64, 4, kBiased>(a, stream)
+                : K <= 8 ? launch_route<64, 8, kBiased>(a, stream) : launch_route<64, 0, kBiased>(a, stream);
 }
 
 }  // namespace
@@ -460,9 +498,10 @@ extern "C" size_t namoh_route_workspace_size(int B, int T, int H, int K) {
   return align_up(ws.used, 256);
 }
 
-extern "C" int namoh_route(const float* scores, int B, int T, int H, int K, int32_t* topk_head, float* gate,
-                           int32_t* rank, int32_t* row, int32_t* seg_offsets, int32_t* row_src, void* workspace,
-                           size_t workspace_bytes, uint32_t* dev_status, void* stream_v) {
+extern "C" int namoh_route_biased(const float* scores, const float* bias, int B, int T, int H, int K,
+                                  int32_t* topk_head, float* gate, int32_t* rank, int32_t* row, int32_t* seg_offsets,
+                                  int32_t* row_src, void* workspace, size_t workspace_bytes, uint32_t* dev_status,
+                                  void* stream_v) {
   if (!scores || !topk_head || !gate || !dev_status) return NAMOH_ERR_INVALID_ARG;
   if (B < 1 || T < 1 || H < 1 || K < 1 || K > H || H > NAMOH_MAX_HEADS) return NAMOH_ERR_INVALID_ARG;
   if ((long long)B * T * K >= (1ll << 31) || (long long)B * H >= (1ll << 20)) return NAMOH_ERR_INVALID_ARG;
@@ -472,6 +511,7 @@ extern "C" int namoh_route(const float* scores, int B, int T, int H, int K, int3
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
   RouteArgs a{};
   a.scores = scores;
+  a.bias = bias;
   a.B = B;
   a.T = T;
   a.H = H;
@@ -491,14 +531,14 @@ extern "C" int namoh_route(const float* scores, int B, int T, int H, int K, int3
     a.chunk_base = ws.take<int32_t>((size_t)B * a.nchunks * H);
     if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
   }
-  // picks held in registers for K <= 8; larger K takes K passes over the logits
-  if (H <= 8) return K <= 4 ? launch_route<8, 4>(a, stream) : launch_route<8, 8>(a, stream);
-  if (H <= 16) return K <= 4 ? launch_route<16, 4>(a, stream) : K <= 8 ? launch_route<16, 8>(a, stream)
-                                                                        : launch_route<16, 0>(a, stream);
-  if (H <= 32) return K <= 4 ? launch_route<32, 4>(a, stream) : K <= 8 ? launch_route<32, 8>(a, stream)
-                                                                        : launch_route<32, 0>(a, stream);
-  return K <= 4 ? launch_route<64, 4>(a, stream) : K <= 8 ? launch_route<64, 8>(a, stream)
-                                                          : launch_route<64, 0>(a, stream);
+  return a.bias ? launch_route_h<true>(a, stream) : launch_route_h<false>(a, stream);
+}
+
+extern "C" int namoh_route(const float* scores, int B, int T, int H, int K, int32_t* topk_head, float* gate,
+                           int32_t* rank, int32_t* row, int32_t* seg_offsets, int32_t* row_src, void* workspace,
+                           size_t workspace_bytes, uint32_t* dev_status, void* stream) {
+  return namoh_route_biased(scores, nullptr, B, T, H, K, topk_head, gate, rank, row, seg_offsets, row_src, workspace,
+                            workspace_bytes, dev_status, stream);
 }
 
 // ---------------------------------------------------------------------------

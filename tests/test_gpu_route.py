@@ -122,3 +122,69 @@ def test_route_repeated_calls_reuse_workspace(namoh, oracle_mod):
         np.testing.assert_array_equal(out.row_src.cpu().numpy(), r["row_src"])
         np.testing.assert_array_equal(out.seg_offsets.cpu().numpy(), r["seg_offsets"])
         assert int(out.status.item()) == 0
+
+
+# --------------------------------------------------------------------------- biased selection
+# App. A, Eq. (namoh-biased-routing).  The GPU ranks fp32 affinities (exp2 of pre-scaled logit
+# differences) plus the bias; the oracle ranks the same sums in fp64.  Where two sums lie
+# within the fp32 error bound of each other either order is correct, so the selection is
+# checked for validity within that bound, and for equality with the oracle wherever the
+# margins are larger; the dispatch of the GPU's own picks must then be bit-exact.
+BIAS_EPS = 4e-6
+
+
+def _check_biased(namoh, oracle_mod, scores, K, bias, compact=True):
+    import scipy.special
+    H = scores.shape[-1]
+    dev = torch.device("cuda")
+    out = namoh.namoh_route(torch.from_numpy(scores).to(dev), K, compact=compact,
+                            bias=torch.from_numpy(bias).to(dev))
+    torch.cuda.synchronize()
+    ref = oracle_mod.route_biased(scores, K, bias)
+    top = out.topk_head.cpu().numpy().astype(np.int64)
+    key = ref["key"]
+    sel = np.take_along_axis(key, top, -1)
+    mask = np.zeros(key.shape, bool)
+    np.put_along_axis(mask, top, True, -1)
+    assert (mask.sum(-1) == K).all(), "picks are not K distinct heads"
+    if K < H:
+        assert (sel.min(-1) >= np.where(mask, -np.inf, key).max(-1) - BIAS_EPS).all()
+    assert (np.diff(sel, axis=-1) <= BIAS_EPS).all()
+    ordered = -np.sort(-key, axis=-1)[..., :min(K + 1, H)]
+    clear = (-np.diff(ordered, axis=-1) > BIAS_EPS).all(-1)
+    np.testing.assert_array_equal(top[clear], ref["topk_head"][clear])
+    assert clear.mean() > 0.9  # most tokens are compared exactly
+    a = scipy.special.softmax(scores.astype(np.float64), axis=-1)
+    np.testing.assert_allclose(out.gate.cpu().numpy(), np.take_along_axis(a, top, -1), rtol=GATE_RTOL, atol=0)
+    if compact:
+        d = oracle_mod.dispatch(top, H)
+        np.testing.assert_array_equal(out.rank.cpu().numpy(), d["rank"])
+        np.testing.assert_array_equal(out.row.cpu().numpy(), d["row"])
+        np.testing.assert_array_equal(out.seg_offsets.cpu().numpy(), d["seg_offsets"])
+        np.testing.assert_array_equal(out.row_src.cpu().numpy(), d["row_src"])
+    assert int(out.status.item()) == 0
+
+
+@pytest.mark.parametrize("B,T,H,K", [
+    (4, 4096, 16, 4),    # balanced routing
+    (1, 8192, 32, 4),    # the decode prefix's router
+    (2, 777, 64, 8),     # K = 8 (picks in registers)
+    (1, 300, 64, 16),    # K > 8 (K passes over the logits)
+    (3, 257, 5, 3),      # H not a power of two
+])
+@pytest.mark.parametrize("spread", [0.02, 0.5])
+def test_route_biased_matches_oracle(namoh, oracle_mod, B, T, H, K, spread):
+    bias = (np.random.default_rng(H * 31 + K).standard_normal(H) * spread / H).astype(np.float32)
+    _check_biased(namoh, oracle_mod, ni.router_scores(7, B, T, H), K, bias)
+
+
+def test_route_biased_single_token_without_packing(namoh, oracle_mod):
+    bias = (np.random.default_rng(4).standard_normal(32) * 0.01).astype(np.float32)
+    _check_biased(namoh, oracle_mod, ni.router_scores(9, 64, 1, 32), 4, bias, compact=False)
+
+
+def test_route_biased_dominant_head(namoh, oracle_mod):
+    bias = np.zeros(16, np.float32)
+    bias[11] = 3.0
+    s = ni.router_scores(12, 2, 1000, 16)
+    _check_biased(namoh, oracle_mod, s, 4, bias)

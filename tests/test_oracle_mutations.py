@@ -29,6 +29,10 @@ MUTATIONS = {
                          "rope_rotate(qin, d, (double)(r + 1), c->base, qr);"),
     "decode_rank_shift": ("rope_rotate(tmp, d, (double)rho, base, qr);",
                           "rope_rotate(tmp, d, (double)(rho + 1), base, qr);"),
+    "biased_gate_includes_bias": ("gate[t * K + k] = a[order[k]];", "gate[t * K + k] = kt[order[k]];"),
+    "biased_key_drops_bias": ("kt[i] = a[i] + (double)bias[i];", "kt[i] = a[i];"),
+    "biased_ties_to_upper_index": ("while (j > 0 && kt[i] > kt[order[j - 1]]) {",
+                                   "while (j > 0 && kt[i] >= kt[order[j - 1]]) {"),
 }
 
 

@@ -162,3 +162,74 @@ def test_nonfinite_scores_rejected(oracle_mod):
     s[0, 3, 2] = np.inf
     with pytest.raises(oracle_mod.OracleError):
         oracle_mod.route(s, 2)
+
+
+# --------------------------------------------------------------------------- biased selection
+# App. A, Eq. (namoh-biased-routing): S_K(t) = TopK_i(a_{t,i} + b_i), g_{t,i} = m_{t,i} a_{t,i}.
+
+def _affinity(scores: np.ndarray) -> np.ndarray:
+    return scipy.special.softmax(scores.astype(np.float64), axis=-1)
+
+
+def test_biased_zero_bias_is_plain_routing(oracle_mod):
+    s = ni.router_scores(3, 2, 257, 16)
+    r0 = oracle_mod.route(s, 4)
+    rb = oracle_mod.route_biased(s, 4, np.zeros(16, np.float32))
+    for key in ("topk_head", "rank", "row", "seg_offsets", "row_src"):
+        np.testing.assert_array_equal(rb[key], r0[key])
+    np.testing.assert_allclose(rb["gate"], r0["gate"], rtol=1e-15, atol=0)
+
+
+def test_biased_dominant_bias_takes_slot_zero(oracle_mod):
+    """A bias larger than any affinity difference puts its head first for every token; the
+    other slots are the unbiased TopK of the remaining heads; the gates stay the softmax."""
+    B, T, H, K, hb = 2, 200, 12, 3, 7
+    s = ni.router_scores(5, B, T, H)
+    bias = np.zeros(H, np.float32)
+    bias[hb] = 2.0
+    rb = oracle_mod.route_biased(s, K, bias)
+    assert (rb["topk_head"][..., 0] == hb).all()
+    others = [h for h in range(H) if h != hb]
+    rest = _topk_by_counting(s[..., others], K - 1)
+    np.testing.assert_array_equal(rb["topk_head"][..., 1:], np.array(others)[rest])
+    a = _affinity(s)
+    np.testing.assert_allclose(rb["gate"], np.take_along_axis(a, rb["topk_head"].astype(np.int64), -1),
+                               rtol=1e-12, atol=0)
+
+
+def test_biased_brute_force_subsets(oracle_mod):
+    """On tiny routers the selected set is the K-subset with the largest sum of a + b
+    (enumerated), and the slots come in decreasing a + b."""
+    import itertools
+    rng = np.random.default_rng(11)
+    for H, K in ((5, 2), (6, 3), (7, 4)):
+        s = ni.router_scores(int(rng.integers(1 << 20)), 1, 40, H)
+        bias = (rng.standard_normal(H) * 0.2).astype(np.float32)
+        rb = oracle_mod.route_biased(s, K, bias)
+        key = _affinity(s) + bias.astype(np.float64)
+        for t in range(40):
+            best = max(itertools.combinations(range(H), K), key=lambda c: sum(key[0, t, list(c)]))
+            assert set(rb["topk_head"][0, t].tolist()) == set(best)
+            sel = key[0, t, rb["topk_head"][0, t]]
+            assert (np.diff(sel) <= 0).all()
+
+
+def test_biased_gates_exclude_bias(oracle_mod):
+    s = ni.router_scores(8, 1, 300, 32)
+    bias = (np.random.default_rng(2).standard_normal(32) * 0.05).astype(np.float32)
+    rb = oracle_mod.route_biased(s, 4, bias)
+    a = _affinity(s)
+    np.testing.assert_allclose(rb["gate"], np.take_along_axis(a, rb["topk_head"].astype(np.int64), -1),
+                               rtol=1e-12, atol=0)
+    assert (rb["gate"].sum(-1) < 1.0).all()
+
+
+def test_biased_ties_go_to_lower_index(oracle_mod):
+    """Equal logits and equal biases give equal a + b: the lower head index comes first."""
+    s = np.zeros((1, 3, 8), np.float32)
+    s[0, 1, [2, 5]] = 1.0
+    bias = np.zeros(8, np.float32)
+    bias[[1, 6]] = 0.5
+    rb = oracle_mod.route_biased(s, 3, bias)
+    np.testing.assert_array_equal(rb["topk_head"][0, 0], [1, 6, 0])
+    np.testing.assert_array_equal(rb["topk_head"][0, 1], [1, 6, 2])
