@@ -392,6 +392,15 @@ def run_decode(args, dev, pk, pk_kind):
     ev[5].record()
     torch.cuda.synchronize()
     route_ms = ev[0].elapsed_time(ev[5]) / 5
+    # the same routing with loss-free balancing biases (selection on a + b, gates a)
+    bias = torch.from_numpy((np.random.default_rng(wl.seed).standard_normal(Hr) * 0.02 / Hr).astype(np.float32)).to(dev)
+    namoh.namoh_route(s, Kr, workspace=ws, out=ro, bias=bias)
+    ev[0].record()
+    for i in range(5):
+        namoh.namoh_route(s, Kr, workspace=ws, out=ro, bias=bias)
+    ev[5].record()
+    torch.cuda.synchronize()
+    route_biased_ms = ev[0].elapsed_time(ev[5]) / 5
     route_bytes = acc.route_bytes(B, wl.prefix, Hr, Kr)
     seg = ro.seg_offsets.cpu().numpy().astype(np.int64)
     del s, ro
@@ -462,8 +471,11 @@ def run_decode(args, dev, pk, pk_kind):
         "hbm_peak_source": f"{pk_kind} copy bandwidth {pk['hbm_gbs']} GB/s",
         "prefix_route": {"ms": route_ms, "bytes": route_bytes, "hbm_gbs": route_bytes / (route_ms * 1e-3) / 1e9,
                          "frac_measured_hbm": route_bytes / (route_ms * 1e-3) / 1e9 / pk["hbm_gbs"]},
+        "prefix_route_biased": {"ms": route_biased_ms, "hbm_gbs": route_bytes / (route_biased_ms * 1e-3) / 1e9,
+                                "frac_measured_hbm": route_bytes / (route_biased_ms * 1e-3) / 1e9 / pk["hbm_gbs"],
+                                "note": "selection on softmax affinities plus per-head biases (namoh_route_biased)"},
         "cache_gb": 2 * rows * d * 2 / 1e9, "device_status": int(status.item()),
-        "launches": 4 * steps,
+        "launches": 4 * steps + 2 * 5 * 3,  # decode steps; 5 timed prefix routings of 3 kernels, plain and biased
     }
     del kc, vc
     torch.cuda.empty_cache()
