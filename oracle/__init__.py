@@ -69,11 +69,11 @@ def _load():
         lib.oracle_route_topk.argtypes = [P, i64, i32, i32, P, P]
         lib.oracle_route_biased.argtypes = [P, P, i64, i32, i32, P, P, P]
         lib.oracle_dispatch.argtypes = [P, i32, i32, i32, i32, P, P, P, P, P]
-        lib.oracle_rope.argtypes = [P, i64, i32, i64, P, f64, P]
-        lib.oracle_prefill.argtypes = [P, P, P, i32, i32, i32, f64, P, P, P, P, P, i32]
-        lib.oracle_prefill_rows.argtypes = [P, P, P, i32, i32, i32, f64, P, P, P, P, P, i64, P]
+        lib.oracle_rope.argtypes = [P, i64, i32, i64, P, f64, i32, P]
+        lib.oracle_prefill.argtypes = [P, P, P, i32, i32, i32, f64, P, P, P, P, P, i32, i32, P]
+        lib.oracle_prefill_rows.argtypes = [P, P, P, i32, i32, i32, f64, P, P, P, P, P, i64, P, i32, P]
         lib.oracle_decode_step.argtypes = [P, P, P, P, P, i32, i32, i32, i32, i32, f64,
-                                           P, P, P, P, P, P]
+                                           P, P, P, P, P, P, i32, P]
         lib.oracle_default_threads.argtypes = []
         for fn in ("oracle_route_topk", "oracle_route_biased", "oracle_dispatch", "oracle_rope", "oracle_prefill",
                    "oracle_prefill_rows", "oracle_decode_step", "oracle_default_threads"):
@@ -153,23 +153,34 @@ def route_biased(scores: np.ndarray, K: int, bias: np.ndarray) -> dict:
     return out
 
 
-def rope(x_bits: np.ndarray, pos: np.ndarray, base: float) -> np.ndarray:
-    """Rotate bf16 rows x [rows, d] (raw uint16 bits) to positions pos [rows]; fp64 out."""
+def rope(x_bits: np.ndarray, pos: np.ndarray, base: float, interleaved: bool = False) -> np.ndarray:
+    """Rotate bf16 rows x [rows, d] (raw uint16 bits) to positions pos [rows]; fp64 out.
+
+    Pairs (j, j + d/2) by default, (2j, 2j+1) with interleaved."""
     lib = _load()
     x_bits = np.ascontiguousarray(x_bits, dtype=np.uint16)
     rows, d = x_bits.shape
     pos = np.ascontiguousarray(pos, dtype=np.int64)
     out = np.empty((rows, d), np.float64)
-    _check(lib.oracle_rope(_ptr(x_bits), rows, d, d, _ptr(pos), float(base), _ptr(out)), "rope")
+    _check(lib.oracle_rope(_ptr(x_bits), rows, d, d, _ptr(pos), float(base), int(bool(interleaved)), _ptr(out)),
+           "rope")
     return out
+
+
+def global_positions(row_src: np.ndarray, T: int, K: int) -> np.ndarray:
+    """Position of each packed row under global RoPE: the token's index t in its sequence
+    (row_src[r] = (b*T + t)*K + slot)."""
+    rs = np.asarray(row_src, dtype=np.int64)
+    return np.ascontiguousarray((rs // K) % T, dtype=np.int64)
 
 
 def prefill(q: np.ndarray, k: np.ndarray, v: np.ndarray, seg_offsets: np.ndarray, row_src: np.ndarray,
             gate: np.ndarray, d: int, g: int, base: float, nthreads: int | None = None,
-            return_krot: bool = False):
+            return_krot: bool = False, interleaved: bool = False, pos: np.ndarray | None = None):
     """Prefill over packed rows.  q [R*g, d], k/v [R, d] as bf16 bits; gate indexed by row_src.
 
     Returns y [R*g, d] fp64 laid out by (row_src * g + j), i.e. [B, T, K, g, d] flattened.
+    RoPE positions are the ranks, or pos [R] (e.g. global_positions) when given.
     """
     lib = _load()
     q = np.ascontiguousarray(q, dtype=np.uint16)
@@ -182,14 +193,19 @@ def prefill(q: np.ndarray, k: np.ndarray, v: np.ndarray, seg_offsets: np.ndarray
     y = np.zeros((R * g, d), np.float64)
     krot = np.empty((R, d), np.float64) if return_krot else None
     nthreads = default_threads() if nthreads is None else int(nthreads)
+    pos = None if pos is None else np.ascontiguousarray(pos, dtype=np.int64)
+    if pos is not None and pos.shape != (R,):
+        raise OracleError("pos must hold one position per packed row")
     rc = lib.oracle_prefill(_ptr(q), _ptr(k), _ptr(v), len(seg) - 1, d, g, float(base), _ptr(seg), _ptr(rs),
-                            _ptr(gt), _ptr(y), _ptr(krot) if krot is not None else None, nthreads)
+                            _ptr(gt), _ptr(y), _ptr(krot) if krot is not None else None, nthreads,
+                            int(bool(interleaved)), _ptr(pos) if pos is not None else None)
     _check(rc, "prefill")
     return (y, krot) if return_krot else y
 
 
 def prefill_rows(q, k, v, seg_offsets, row_src, gate, d: int, g: int, base: float,
-                 rows: np.ndarray, heads: np.ndarray) -> np.ndarray:
+                 rows: np.ndarray, heads: np.ndarray, interleaved: bool = False,
+                 pos: np.ndarray | None = None) -> np.ndarray:
     """Outputs g*h for the listed (packed row, group head) queries only: [len(rows), d] fp64."""
     lib = _load()
     q = np.ascontiguousarray(q, dtype=np.uint16)
@@ -201,18 +217,23 @@ def prefill_rows(q, k, v, seg_offsets, row_src, gate, d: int, g: int, base: floa
     rows = np.ascontiguousarray(rows, dtype=np.int64)
     heads = np.ascontiguousarray(heads, dtype=np.int32)
     out = np.empty((len(rows), d), np.float64)
+    pos = None if pos is None else np.ascontiguousarray(pos, dtype=np.int64)
+    if pos is not None and pos.shape != (int(seg[-1]),):
+        raise OracleError("pos must hold one position per packed row")
     rc = lib.oracle_prefill_rows(_ptr(q), _ptr(k), _ptr(v), len(seg) - 1, d, g, float(base), _ptr(seg),
-                                 _ptr(rs), _ptr(gt), _ptr(rows), _ptr(heads), len(rows), _ptr(out))
+                                 _ptr(rs), _ptr(gt), _ptr(rows), _ptr(heads), len(rows), _ptr(out),
+                                 int(bool(interleaved)), _ptr(pos) if pos is not None else None)
     _check(rc, "prefill_rows")
     return out
 
 
 def decode_step(topk_head, gate, q, k, v, Hr: int, d: int, g: int, base: float,
                 k_cache: np.ndarray, v_cache: np.ndarray, seg_base: np.ndarray, seg_len: np.ndarray,
-                seg_cap: np.ndarray) -> np.ndarray:
+                seg_cap: np.ndarray, interleaved: bool = False, token_pos: np.ndarray | None = None) -> np.ndarray:
     """One decode step.  k_cache/v_cache [cap_total, d] fp64 and seg_len are updated in place.
 
     topk_head/gate [B, Kr]; q [B, Kr*g, d], k/v [B, Kr, d] as bf16 bits.  Returns y [B, Kr*g, d].
+    RoPE positions are the ranks, or token_pos [B] (the new tokens' indices) when given.
     """
     lib = _load()
     topk_head = np.ascontiguousarray(topk_head, dtype=np.int32)
@@ -227,8 +248,10 @@ def decode_step(topk_head, gate, q, k, v, Hr: int, d: int, g: int, base: float,
         if arr.dtype != dt or not arr.flags.c_contiguous:
             raise OracleError(f"{name} must be a contiguous {np.dtype(dt).name} array")
     y = np.zeros((B, Kr * g, d), np.float64)
+    token_pos = None if token_pos is None else np.ascontiguousarray(token_pos, dtype=np.int64)
     rc = lib.oracle_decode_step(_ptr(topk_head), _ptr(gate), _ptr(q), _ptr(k), _ptr(v), B, Hr, Kr, d, g,
                                 float(base), _ptr(k_cache), _ptr(v_cache), _ptr(seg_base), _ptr(seg_len),
-                                _ptr(seg_cap), _ptr(y))
+                                _ptr(seg_cap), _ptr(y), int(bool(interleaved)),
+                                _ptr(token_pos) if token_pos is not None else None)
     _check(rc, "decode_step")
     return y

@@ -30,6 +30,8 @@
  *     descending score.
  *   - RoPE is the half-split form: pairs (j, j + d/2), theta_j = base^(-2j/d),
  *     x'_j = x_j cos - x_{j+d/2} sin,  x'_{j+d/2} = x_{j+d/2} cos + x_j sin.
+ *     Variants: interleaved pairs (2j, 2j+1), and the token's global index t as the
+ *     position instead of its rank (the global-RoPE reading of Sec. 3.2).
  *   - Attention scale 1/sqrt(d_head).
  *   - Packed rows: segments in (batch, head) order, rows ascending in t inside a segment.
  *
@@ -243,20 +245,22 @@ int oracle_dispatch(const int32_t *topk_head, int B, int T, int H, int K,
 }
 
 /* ------------------------------------------------------------------------- */
-/* RoPE (Sec. 3.2, Eq. namoh-head-rope), half-split pairs                     */
+/* RoPE (Sec. 3.2, Eq. namoh-head-rope)                                       */
 /* ------------------------------------------------------------------------- */
 
-/* x [d] (widened bf16) rotated to position p: out [d] */
-static void rope_rotate(const double *x, int d, double p, double base, double *out)
+/* x [d] (widened bf16) rotated to position p: out [d].  Pair j (frequency theta_j) is
+ * (x_j, x_{j+d/2}) in the half-split form, (x_{2j}, x_{2j+1}) in the interleaved one. */
+static void rope_rotate(const double *x, int d, double p, double base, int interleaved, double *out)
 {
     int half = d / 2;
     for (int j = 0; j < half; ++j) {
         double theta = pow(base, -2.0 * (double)j / (double)d);
         double ang = p * theta;
         double c = cos(ang), s = sin(ang);
-        double x0 = x[j], x1 = x[j + half];
-        out[j] = x0 * c - x1 * s;
-        out[j + half] = x1 * c + x0 * s;
+        int i0 = interleaved ? 2 * j : j, i1 = interleaved ? 2 * j + 1 : j + half;
+        double x0 = x[i0], x1 = x[i1];
+        out[i0] = x0 * c - x1 * s;
+        out[i1] = x1 * c + x0 * s;
     }
 }
 
@@ -264,14 +268,15 @@ static void rope_rotate(const double *x, int d, double p, double base, double *o
  * oracle_rope: rotate each bf16 row x[i, :] (row stride ld elements) to
  * position pos[i] and write fp64 rows out[i, :].
  */
-int oracle_rope(const uint16_t *x, long rows, int d, long ld, const int64_t *pos, double base, double *out)
+int oracle_rope(const uint16_t *x, long rows, int d, long ld, const int64_t *pos, double base, int interleaved,
+                double *out)
 {
     if (!x || !pos || !out || rows < 0 || d < 2 || (d & 1) || ld < d) return ORACLE_ERR_ARG;
     double *tmp = (double *)malloc(sizeof(double) * (size_t)d);
     if (!tmp) return ORACLE_ERR_NOMEM;
     for (long i = 0; i < rows; ++i) {
         for (int c = 0; c < d; ++c) tmp[c] = bf16_to_double(x[i * ld + c]);
-        rope_rotate(tmp, d, (double)pos[i], base, out + i * (long)d);
+        rope_rotate(tmp, d, (double)pos[i], base, interleaved, out + i * (long)d);
     }
     free(tmp);
     return ORACLE_OK;
@@ -318,6 +323,8 @@ struct prefill_ctx {
     double *y;
     int nseg, d, g;
     double base;
+    int interleaved;
+    const int64_t *pos;       /* [R] position of each packed row, or NULL for its rank */
     long *item_seg, *item_r0; /* work items: (segment, first local query) */
     int chunk;
     int status;
@@ -349,7 +356,7 @@ static void prefill_item(long it, void *vctx)
         long dst = c->row_src[row];
         for (int j = 0; j < g; ++j) {
             for (int cc = 0; cc < d; ++cc) qin[cc] = bf16_to_double(c->q[(row * g + j) * d + cc]);
-            rope_rotate(qin, d, (double)r, c->base, qr);
+            rope_rotate(qin, d, c->pos ? (double)c->pos[row] : (double)r, c->base, c->interleaved, qr);
             /* causal history: local ranks 0..r of this head (s in I_i, s <= t) */
             attend(qr, c->krot + off * d, vals, r + 1, d, w, h);
             double gt = c->gate[dst];
@@ -365,6 +372,8 @@ struct rotk_ctx {
     double *krot;
     int d;
     double base;
+    int interleaved;
+    const int64_t *pos;
 };
 
 static void rotate_k_segment(long s, void *vctx)
@@ -376,7 +385,8 @@ static void rotate_k_segment(long s, void *vctx)
     if (!tmp) return;
     for (long row = off; row < end; ++row) {
         for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(c->k[row * d + cc]);
-        rope_rotate(tmp, d, (double)(row - off), c->base, c->krot + row * d);
+        rope_rotate(tmp, d, c->pos ? (double)c->pos[row] : (double)(row - off), c->base, c->interleaved,
+                    c->krot + row * d);
     }
     free(tmp);
 }
@@ -392,7 +402,7 @@ static void rotate_k_segment(long s, void *vctx)
  */
 int oracle_prefill(const uint16_t *q, const uint16_t *k, const uint16_t *v, int nseg, int d, int g,
                    double base, const int32_t *seg_offsets, const int32_t *row_src, const double *gate,
-                   double *y, double *k_rot, int nthreads)
+                   double *y, double *k_rot, int nthreads, int interleaved, const int64_t *pos)
 {
     if (!q || !k || !v || !seg_offsets || !row_src || !gate || !y) return ORACLE_ERR_ARG;
     if (nseg < 0 || d < 2 || (d & 1) || g < 1) return ORACLE_ERR_ARG;
@@ -402,7 +412,7 @@ int oracle_prefill(const uint16_t *q, const uint16_t *k, const uint16_t *v, int 
         krot = (double *)malloc(sizeof(double) * (size_t)(R > 0 ? R : 1) * d);
         if (!krot) return ORACLE_ERR_NOMEM;
     }
-    struct rotk_ctx rk = {k, seg_offsets, krot, d, base};
+    struct rotk_ctx rk = {k, seg_offsets, krot, d, base, interleaved, pos};
     parallel_for(nseg, nthreads, rotate_k_segment, &rk);
 
     const int chunk = 64;
@@ -427,7 +437,7 @@ int oracle_prefill(const uint16_t *q, const uint16_t *k, const uint16_t *v, int 
             ++it;
         }
     }
-    struct prefill_ctx ctx = {q, v, krot, seg_offsets, row_src, gate, y, nseg, d, g, base,
+    struct prefill_ctx ctx = {q, v, krot, seg_offsets, row_src, gate, y, nseg, d, g, base, interleaved, pos,
                               item_seg, item_r0, chunk, ORACLE_OK};
     parallel_for(nitems, nthreads, prefill_item, &ctx);
     free(item_seg); free(item_r0);
@@ -443,7 +453,8 @@ int oracle_prefill(const uint16_t *q, const uint16_t *k, const uint16_t *v, int 
  */
 int oracle_prefill_rows(const uint16_t *q, const uint16_t *k, const uint16_t *v, int nseg, int d, int g,
                         double base, const int32_t *seg_offsets, const int32_t *row_src, const double *gate,
-                        const int64_t *rows, const int32_t *heads, long nrows, double *out)
+                        const int64_t *rows, const int32_t *heads, long nrows, double *out, int interleaved,
+                        const int64_t *pos)
 {
     if (!q || !k || !v || !seg_offsets || !row_src || !gate || !rows || !heads || !out) return ORACLE_ERR_ARG;
     long R = seg_offsets[nseg];
@@ -483,12 +494,12 @@ int oracle_prefill_rows(const uint16_t *q, const uint16_t *k, const uint16_t *v,
         }
         for (long s = cached_len; s <= r; ++s) {
             for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(k[(off + s) * d + cc]);
-            rope_rotate(tmp, d, (double)s, base, keys + s * d);
+            rope_rotate(tmp, d, pos ? (double)pos[off + s] : (double)s, base, interleaved, keys + s * d);
             for (int cc = 0; cc < d; ++cc) vals[s * d + cc] = bf16_to_double(v[(off + s) * d + cc]);
         }
         if (r + 1 > cached_len) cached_len = r + 1;
         for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(q[(row * g + j) * d + cc]);
-        rope_rotate(tmp, d, (double)r, base, qr);
+        rope_rotate(tmp, d, pos ? (double)pos[row] : (double)r, base, interleaved, qr);
         attend(qr, keys, vals, r + 1, d, w, h);
         double gt = gate[row_src[row]];
         for (int cc = 0; cc < d; ++cc) out[i * d + cc] = gt * h[cc];
@@ -509,13 +520,15 @@ int oracle_prefill_rows(const uint16_t *q, const uint16_t *k, const uint16_t *v,
  *   k_cache, v_cache [cap_total, d] fp64 histories (k_cache holds rotated keys);
  *   seg_base [B*Hr], seg_len [B*Hr] (updated in place), seg_cap [B*Hr]
  *   y [B, Kr*g, d] fp64: g * h for each selected (group) head
- * For each (b, slot): rho = seg_len; k~ = k R(rho) and v are appended at rho;
- * q~ = q R(rho) attends over the rho + 1 entries; seg_len += 1.
+ * For each (b, slot): rho = seg_len; k~ = k R(p) and v are appended at rho;
+ * q~ = q R(p) attends over the rho + 1 entries; seg_len += 1.  The rotation position
+ * p is rho, or token_pos[b] (the new token's index in its sequence) when token_pos is
+ * given; interleaved selects the pairing of rope_rotate.
  */
 int oracle_decode_step(const int32_t *topk_head, const double *gate, const uint16_t *q, const uint16_t *k,
                        const uint16_t *v, int B, int Hr, int Kr, int d, int g, double base,
                        double *k_cache, double *v_cache, const int64_t *seg_base, int32_t *seg_len,
-                       const int32_t *seg_cap, double *y)
+                       const int32_t *seg_cap, double *y, int interleaved, const int64_t *token_pos)
 {
     if (!topk_head || !gate || !q || !k || !v || !k_cache || !v_cache || !seg_base || !seg_len || !seg_cap || !y)
         return ORACLE_ERR_ARG;
@@ -533,7 +546,8 @@ int oracle_decode_step(const int32_t *topk_head, const double *gate, const uint1
             if (rho >= seg_cap[s]) { st = ORACLE_ERR_CAPACITY; break; }
             long base_row = seg_base[s];
             for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(k[((long)b * Kr + kk) * d + cc]);
-            rope_rotate(tmp, d, (double)rho, base, k_cache + (base_row + rho) * d);
+            const double p = token_pos ? (double)token_pos[b] : (double)rho;
+            rope_rotate(tmp, d, p, base, interleaved, k_cache + (base_row + rho) * d);
             for (int cc = 0; cc < d; ++cc)
                 v_cache[(base_row + rho) * d + cc] = bf16_to_double(v[((long)b * Kr + kk) * d + cc]);
             double *w = (double *)malloc(sizeof(double) * (size_t)(rho + 1));
@@ -541,7 +555,7 @@ int oracle_decode_step(const int32_t *topk_head, const double *gate, const uint1
             for (int j = 0; j < g; ++j) {
                 long qi = ((long)b * Kr + kk) * g + j;
                 for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(q[qi * d + cc]);
-                rope_rotate(tmp, d, (double)rho, base, qr);
+                rope_rotate(tmp, d, p, base, interleaved, qr);
                 attend(qr, k_cache + base_row * d, v_cache + base_row * d, rho + 1, d, w, h);
                 for (int cc = 0; cc < d; ++cc) y[qi * d + cc] = gate[b * Kr + kk] * h[cc];
             }

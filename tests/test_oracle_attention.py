@@ -12,6 +12,10 @@ What the paper fixes, each checked by a formulation unlike the oracle's:
   * App. C Eq. (app-routed-kv): M_KV = T K after the prefix, + K per decode step.
   * App. C "Adopted KV-group routing": g query heads share a group's keys, values,
     gate and rank.
+  * Sec. 3.2 (end of "Head-relative positional encoding"): global RoPE replaces rho_i(t) by t
+    -> the brute-force masks with t as the position, and prefill == decode at token index t.
+  * Interleaved pairing (2j, 2j+1) is RoPE as complex multiplication on adjacent pairs, i.e.
+    half-split RoPE conjugated by the pair permutation.
 """
 import numpy as np
 import pytest
@@ -24,13 +28,19 @@ def _widen(bits):
     return ni.bf16_to_f32(bits).astype(np.float64)
 
 
-def _rope_complex(x, pos, base):
-    """RoPE as complex multiplication: (x_j + i x_{j+d/2}) * exp(i * pos * base^(-2j/d))."""
+def _rope_complex(x, pos, base, interleaved=False):
+    """RoPE as complex multiplication: (x_j + i x_{j+d/2}) * exp(i * pos * base^(-2j/d)),
+    or (x_{2j} + i x_{2j+1}) for the interleaved pairing."""
     d = x.shape[-1]
     half = d // 2
-    z = x[..., :half] + 1j * x[..., half:]
+    z = x[..., 0::2] + 1j * x[..., 1::2] if interleaved else x[..., :half] + 1j * x[..., half:]
     freq = np.exp(-np.log(base) * (2.0 * np.arange(half) / d))
     rot = z * np.exp(1j * np.asarray(pos, np.float64)[..., None] * freq)
+    if interleaved:
+        out = np.empty(rot.shape[:-1] + (d,))
+        out[..., 0::2] = rot.real
+        out[..., 1::2] = rot.imag
+        return out
     return np.concatenate([rot.real, rot.imag], axis=-1)
 
 
@@ -68,15 +78,20 @@ def _pack(top, B, T, Hr):
 
 # --------------------------------------------------------------------------- RoPE
 @pytest.mark.parametrize("d,base", [(64, 1e4), (128, 5e5), (8, 10.0)])
-def test_rope_is_complex_rotation(oracle_mod, d, base):
+@pytest.mark.parametrize("interleaved", [False, True])
+def test_rope_is_complex_rotation(oracle_mod, d, base, interleaved):
     rng = np.random.default_rng(0)
     x = ni.bf16_bits(rng.standard_normal((50, d)).astype(np.float32))
     pos = rng.integers(0, 40000, 50)
     pos[0] = 0
-    out = oracle_mod.rope(x, pos, base)
-    np.testing.assert_allclose(out, _rope_complex(_widen(x), pos, base), rtol=0, atol=1e-9)
+    out = oracle_mod.rope(x, pos, base, interleaved)
+    np.testing.assert_allclose(out, _rope_complex(_widen(x), pos, base, interleaved), rtol=0, atol=1e-9)
     np.testing.assert_array_equal(out[0], _widen(x[0]))  # R(0) = I
     np.testing.assert_allclose(np.linalg.norm(out, axis=-1), np.linalg.norm(_widen(x), axis=-1), rtol=1e-12)
+    if interleaved:  # half-split RoPE conjugated by the pair permutation (2j, 2j+1) <-> (j, j + d/2)
+        perm = np.concatenate([np.arange(0, d, 2), np.arange(1, d, 2)])
+        half_split = oracle_mod.rope(x[:, perm], pos, base)
+        np.testing.assert_array_equal(out[:, perm], half_split)
 
 
 def test_rope_relative_property(oracle_mod):
@@ -123,6 +138,10 @@ def test_k_equals_h_is_dense_causal_mha(oracle_mod, B, T, H, d):
     h = _dense_causal_mha(_widen(qb), _widen(kb), _widen(vb), 1e4)
     expect = gate[..., None] * np.take_along_axis(h, top[..., None], axis=2)
     np.testing.assert_allclose(y, expect, rtol=0, atol=1e-11)
+    # with K = H every rank is t, so global RoPE changes nothing
+    yg = oracle_mod.prefill(qp, kp, vp, seg, row_src, gate.reshape(-1), d, 1, 1e4,
+                            pos=oracle_mod.global_positions(row_src, T, H))
+    np.testing.assert_array_equal(yg.reshape(B, T, H, d), y)
 
 
 def test_single_head_k1_is_single_head_attention(oracle_mod):
@@ -141,10 +160,11 @@ def test_single_head_k1_is_single_head_attention(oracle_mod):
 
 
 # --------------------------------------------------------------------------- brute force
-def _brute_force(qf, kf, vf, s, Kr, g, base):
+def _brute_force(qf, kf, vf, s, Kr, g, base, interleaved=False, global_pos=False):
     """Full T x T per-query-head attention with routing masks (App. B definitions).
 
     qf [B, T, Hr*g, d], kf/vf [B, T, Hr, d] fp64; s [B, T, Hr] logits.  Returns y [B, T, Kr, g, d].
+    global_pos encodes token t at position t instead of its rank.
     """
     B, T, Hr = s.shape
     d = qf.shape[-1]
@@ -152,14 +172,16 @@ def _brute_force(qf, kf, vf, s, Kr, g, base):
     mask = np.zeros((B, T, Hr), np.int64)
     np.put_along_axis(mask, top, 1, axis=-1)
     rho = np.cumsum(mask, axis=1) - 1
+    if global_pos:
+        rho = np.broadcast_to(np.arange(T)[None, :, None], (B, T, Hr))
     a = _softmax64(s)
     y = np.zeros((B, T, Kr, g, d))
     causal = np.tril(np.ones((T, T), bool))
     for b in range(B):
         for i in range(Hr):
-            kr = _rope_complex(kf[b, :, i], rho[b, :, i], base)
+            kr = _rope_complex(kf[b, :, i], rho[b, :, i], base, interleaved)
             for j in range(g):
-                qr = _rope_complex(qf[b, :, i * g + j], rho[b, :, i], base)
+                qr = _rope_complex(qf[b, :, i * g + j], rho[b, :, i], base, interleaved)
                 logits = qr @ kr.T / np.sqrt(d)
                 allowed = causal & (mask[b, :, i][:, None] == 1) & (mask[b, :, i][None, :] == 1)
                 for t in range(T):
@@ -172,14 +194,16 @@ def _brute_force(qf, kf, vf, s, Kr, g, base):
     return y, top
 
 
+@pytest.mark.parametrize("variant", ["rank", "interleaved", "global", "global_interleaved"])
 @pytest.mark.parametrize("B,T,Hr,Kr,g,d", [(2, 24, 4, 2, 1, 8), (1, 40, 6, 3, 1, 16), (2, 20, 4, 2, 3, 8)])
-def test_prefill_matches_brute_force_masks(oracle_mod, B, T, Hr, Kr, g, d):
+def test_prefill_matches_brute_force_masks(oracle_mod, B, T, Hr, Kr, g, d, variant):
     rng = np.random.default_rng(4)
     s = ni.router_scores(6, B, T, Hr)
     qb = ni.bf16_bits(rng.standard_normal((B, T, Hr * g, d)).astype(np.float32))
     kb = ni.bf16_bits(rng.standard_normal((B, T, Hr, d)).astype(np.float32))
     vb = ni.bf16_bits(rng.standard_normal((B, T, Hr, d)).astype(np.float32))
-    expect, top = _brute_force(_widen(qb), _widen(kb), _widen(vb), s, Kr, g, 1e4)
+    il, gp = "interleaved" in variant, variant.startswith("global")
+    expect, top = _brute_force(_widen(qb), _widen(kb), _widen(vb), s, Kr, g, 1e4, il, gp)
     seg, row, row_src, _, _ = _pack(top, B, T, Hr)
     R = B * T * Kr
     qp = np.empty((R, g, d), np.uint16); kp = np.empty((R, d), np.uint16); vp = np.empty_like(kp)
@@ -192,12 +216,18 @@ def test_prefill_matches_brute_force_masks(oracle_mod, B, T, Hr, Kr, g, d):
                 kp[r] = kb[b, t, h]
                 vp[r] = vb[b, t, h]
     gate = np.take_along_axis(_softmax64(s), top, -1).reshape(-1)
-    y = oracle_mod.prefill(qp.reshape(R * g, d), kp, vp, seg, row_src, gate, d, g, 1e4)
+    pos = oracle_mod.global_positions(row_src, T, Kr) if gp else None
+    if gp:  # the packed row of (b, t, k) sits at position t
+        expect_pos = np.empty(R, np.int64)
+        expect_pos[row.reshape(-1)] = np.broadcast_to(np.arange(T)[None, :, None], (B, T, Kr)).reshape(-1)
+        np.testing.assert_array_equal(pos, expect_pos)
+    y = oracle_mod.prefill(qp.reshape(R * g, d), kp, vp, seg, row_src, gate, d, g, 1e4, interleaved=il, pos=pos)
     np.testing.assert_allclose(y.reshape(B, T, Kr, g, d), expect, rtol=0, atol=1e-11)
     # the row-subset entry point agrees with the full prefill
     pick = np.arange(0, R, 7)
     heads = (pick % g).astype(np.int32)
-    out = oracle_mod.prefill_rows(qp.reshape(R * g, d), kp, vp, seg, row_src, gate, d, g, 1e4, pick, heads)
+    out = oracle_mod.prefill_rows(qp.reshape(R * g, d), kp, vp, seg, row_src, gate, d, g, 1e4, pick, heads,
+                                  interleaved=il, pos=pos)
     np.testing.assert_allclose(out, y[row_src[pick] * g + heads], rtol=0, atol=1e-13)
 
 
@@ -224,10 +254,13 @@ def test_causal_support_and_weights_sum_to_one(oracle_mod):
 
 
 # --------------------------------------------------------------------------- decode
-def _prefix_cache(oracle_mod, q, k, v, out, T, K, d, g, base, headroom, Hr, B):
+def _prefix_cache(oracle_mod, q, k, v, out, T, K, d, g, base, headroom, Hr, B, interleaved=False,
+                  global_pos=False):
     """Prefill over the first T tokens; returns y and the fp64 caches with headroom."""
     seg = out["seg_offsets"]
-    y, krot = oracle_mod.prefill(q, k, v, seg, out["row_src"], out["gate"], d, g, base, return_krot=True)
+    pos = oracle_mod.global_positions(out["row_src"], T, K) if global_pos else None
+    y, krot = oracle_mod.prefill(q, k, v, seg, out["row_src"], out["gate"], d, g, base, return_krot=True,
+                                 interleaved=interleaved, pos=pos)
     nseg = B * Hr
     n = (seg[1:] - seg[:-1]).astype(np.int32)
     seg_base = (seg[:-1] + np.arange(nseg) * headroom).astype(np.int64)
@@ -240,15 +273,19 @@ def _prefix_cache(oracle_mod, q, k, v, out, T, K, d, g, base, headroom, Hr, B):
     return y, kc, vc, seg_base, n.copy(), cap
 
 
+@pytest.mark.parametrize("variant", ["rank", "interleaved", "global", "global_interleaved"])
 @pytest.mark.parametrize("g", [1, 2])
-def test_prefill_equals_incremental_decode(oracle_mod, g):
+def test_prefill_equals_incremental_decode(oracle_mod, g, variant):
     B, T, Hr, Kr, d, steps, base = 2, 40, 4, 2, 16, 3, 1e4
+    il, gp = "interleaved" in variant, variant.startswith("global")
     Ttot = T + steps
     s = ni.router_scores(8, B, Ttot, Hr)
     full = oracle_mod.route(s, Kr)
     R = B * Ttot * Kr
     q, k, v = ni.qkv_rows(8, R, d, g)
-    y_full = oracle_mod.prefill(q, k, v, full["seg_offsets"], full["row_src"], full["gate"], d, g, base)
+    pos_full = oracle_mod.global_positions(full["row_src"], Ttot, Kr) if gp else None
+    y_full = oracle_mod.prefill(q, k, v, full["seg_offsets"], full["row_src"], full["gate"], d, g, base,
+                                interleaved=il, pos=pos_full)
     # the prefix: drop the rows of the last `steps` tokens (the last rows of their segments)
     tok = full["row_src"] // Kr % Ttot
     keep = np.nonzero(tok < T)[0]
@@ -256,7 +293,7 @@ def test_prefill_equals_incremental_decode(oracle_mod, g):
     np.testing.assert_array_equal(pre["row_src"], full["row_src"][keep] - (full["row_src"][keep] // (Ttot * Kr)) * (steps * Kr))
     qg = q.reshape(R, g, d)
     _, kc, vc, seg_base, n, cap = _prefix_cache(oracle_mod, qg[keep].reshape(-1, d), k[keep], v[keep], pre,
-                                                T, Kr, d, g, base, steps, Hr, B)
+                                                T, Kr, d, g, base, steps, Hr, B, il, gp)
     # M_KV = T K after the prefix
     assert int(n.sum()) == B * T * Kr
     for st in range(steps):
@@ -264,7 +301,8 @@ def test_prefill_equals_incremental_decode(oracle_mod, g):
         top = full["topk_head"][:, t]
         rows = full["row"][:, t]
         yq = oracle_mod.decode_step(top, full["gate"][:, t], qg[rows].reshape(B, Kr * g, d), k[rows], v[rows],
-                                    Hr, d, g, base, kc, vc, seg_base, n, cap)
+                                    Hr, d, g, base, kc, vc, seg_base, n, cap, interleaved=il,
+                                    token_pos=np.full(B, t, np.int64) if gp else None)
         idx = (np.arange(B)[:, None] * Ttot + t) * Kr + np.arange(Kr)[None, :]
         expect = y_full.reshape(B * Ttot * Kr, g, d)[idx.reshape(-1)].reshape(B, Kr * g, d)
         np.testing.assert_allclose(yq, expect, rtol=0, atol=1e-12)

@@ -16,7 +16,13 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 SRC = os.path.join(ROOT, "oracle", "namoh_oracle.c")
 
 MUTATIONS = {
-    "rope_sign": ("out[j + half] = x1 * c + x0 * s;", "out[j + half] = x1 * c - x0 * s;"),
+    "rope_sign": ("out[i1] = x1 * c + x0 * s;", "out[i1] = x1 * c - x0 * s;"),
+    "interleave_pairs_swapped": ("int i0 = interleaved ? 2 * j : j, i1 = interleaved ? 2 * j + 1 : j + half;",
+                                 "int i0 = interleaved ? 2 * j + 1 : j, i1 = interleaved ? 2 * j : j + half;"),
+    "global_key_uses_rank": ("c->pos ? (double)c->pos[row] : (double)(row - off)",
+                             "c->pos ? (double)(row - off) : (double)(row - off)"),
+    "decode_ignores_token_pos": ("const double p = token_pos ? (double)token_pos[b] : (double)rho;",
+                                 "const double p = token_pos ? (double)rho : (double)rho;"),
     "no_scale": ("double scale = 1.0 / sqrt((double)d);", "double scale = 1.0;"),
     "causal_drops_self": ("attend(qr, c->krot + off * d, vals, r + 1, d, w, h);",
                           "attend(qr, c->krot + off * d, vals, r > 0 ? r : 1, d, w, h);"),
@@ -25,10 +31,10 @@ MUTATIONS = {
                        "double theta = pow(base, -1.0 * (double)j / (double)d);"),
     "gates_renormalised": ("for (int i = 0; i < H; ++i) z += exp((double)s[i] - mx);",
                            "for (int i = 0; i < K; ++i) z += exp((double)s[order[i]] - mx);"),
-    "query_rank_shift": ("rope_rotate(qin, d, (double)r, c->base, qr);",
-                         "rope_rotate(qin, d, (double)(r + 1), c->base, qr);"),
-    "decode_rank_shift": ("rope_rotate(tmp, d, (double)rho, base, qr);",
-                          "rope_rotate(tmp, d, (double)(rho + 1), base, qr);"),
+    "query_rank_shift": ("rope_rotate(qin, d, c->pos ? (double)c->pos[row] : (double)r, c->base",
+                         "rope_rotate(qin, d, c->pos ? (double)c->pos[row] : (double)(r + 1), c->base"),
+    "decode_rank_shift": ("const double p = token_pos ? (double)token_pos[b] : (double)rho;",
+                          "const double p = token_pos ? (double)token_pos[b] : (double)(rho + 1);"),
     "biased_gate_includes_bias": ("gate[t * K + k] = a[order[k]];", "gate[t * K + k] = kt[order[k]];"),
     "biased_key_drops_bias": ("kt[i] = a[i] + (double)bias[i];", "kt[i] = a[i];"),
     "biased_ties_to_upper_index": ("while (j > 0 && kt[i] > kt[order[j - 1]]) {",
