@@ -251,6 +251,32 @@ def run_gpu(args, rank: int, world: int):
     attn_ms = float(stage[:, 2].mean())
     st = int(status.item())
 
+    # ---- the RoPE/plan launch alone in each RoPE variant (Sec. 3.2: rank or global position;
+    # half-split or interleaved pairs), L2 flushed before every launch.  Algorithmic bytes:
+    # Q and K read, Q~ and K~ written (V serves as its own cache here), plus row_src for global.
+    R = B * T * wl.Kr
+    rope_bytes = 2 * (R * g * d * 2 + R * d * 2)
+    rope_variants = {}
+    for name, il, gp in (("half_split_rank", False, False), ("interleaved_rank", True, False),
+                         ("half_split_global", False, True), ("interleaved_global", True, True)):
+        evr = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+        for i in range(args.warmup + args.steps):
+            flush.fill_(i & 0xFF)
+            if i >= args.warmup:
+                evr[i - args.warmup][0].record()
+            namoh.namoh_rope_pack(q, k, v, ro.seg_offsets, B=B, T=T, H=H, K=K, group=g, rope_base=wl.base,
+                                  interleaved=il, row_src=ro.row_src if gp else None, q_rot=q_rot, k_cache=k_cache,
+                                  v_cache=v, status=status, plan=plan)
+            if i >= args.warmup:
+                evr[i - args.warmup][1].record()
+        torch.cuda.synchronize()
+        ms = float(np.mean([a.elapsed_time(b) for a, b in evr]))
+        nbytes = rope_bytes + (R * 4 if gp else 0)
+        rope_variants[name] = {"ms": ms, "hbm_gbs": nbytes / (ms * 1e-3) / 1e9,
+                               "hbm_frac": nbytes / (ms * 1e-3) / 1e9 / pk["hbm_gbs"]}
+    rope_variants["bytes"] = "2 (R g d + R d) bf16 (+ 4 R for row_src under global positions), R = B T Kr"
+    st |= int(status.item())
+
     # ---- end to end through the public API with host buffers (pinned), copies timed.
     # Every step copies its own inputs host -> device, runs namoh_route + namoh_prefill and
     # reads its own y back.  Consecutive steps overlap as in serving: the input copies of step
@@ -346,6 +372,7 @@ def run_gpu(args, rank: int, world: int):
                    "cv2_mean": float(np.mean([acc.cv2(n_seg[b * wl.Hr:(b + 1) * wl.Hr]) for b in range(B)]))},
         "stages_ms": {"route": float(stage[:, 0].mean()), "rope_pack_plan": float(stage[:, 1].mean()),
                       "attention": attn_ms, "note": "separate pass, an event between stages (no overlap)"},
+        "rope_variants": rope_variants,
         "roofline": {"kernel": "attn_fwd_kernel<128>", "bound": "tensor", "achieved": achieved, "peak": peak_tf,
                      "unit": "TFLOP/s", "frac": achieved / peak_tf, "traffic": traffic,
                      "peak_source": f"{pk_kind} bf16 dense (burst)",
@@ -357,8 +384,9 @@ def run_gpu(args, rank: int, world: int):
                             f"steps overlapped; {NSET} rotating device input/output sets ({NSET} x 51 MB > L2), "
                             f"no flush", "y_readback_matches_device": e2e_y_ok},
         # per step: route (2 kernels) + RoPE/plan (1) + attention (1), in each of the three timed
-        # passes (headline, stage breakdown, end to end)
-        "gpu_launches": 4 * 3 * args.steps,
+        # passes (headline, stage breakdown, end to end), and one RoPE/plan launch per timed
+        # step in each of the four RoPE variants
+        "gpu_launches": 4 * 3 * args.steps + 4 * args.steps,
         "wall_s_timed_region": wall,
         "host_enqueue_ms_max": 1e3 * max(enqueue_s), "flush_ms_min": min(flush_ms), "stage_timing_gapless": gapless,
         "device_status": st,

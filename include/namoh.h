@@ -63,6 +63,16 @@ typedef enum namoh_status {
                                           hold the barrier's index in its kernel's barrier block
                                           and bits 24-31 the warp that gave up */
 
+/* RoPE variants (the rope_flags argument of the *_ex entry points; 0 = the defaults).
+ * NAMOH_ROPE_INTERLEAVED  rotate pairs (2j, 2j+1) instead of the half-split (j, j + d/2);
+ *                         theta_j = rope_base^(-2j/d) in both.
+ * NAMOH_ROPE_GLOBAL       encode each token at its index t in its sequence instead of
+ *                         its rank rho_i(t) (Sec. 3.2: global-position RoPE replaces
+ *                         rho_i(t) by t).  Cache rows still follow the rank.
+ * Prefill and decode over one cache must use the same flags. */
+#define NAMOH_ROPE_INTERLEAVED 0x1u
+#define NAMOH_ROPE_GLOBAL 0x2u
+
 /* Limits of this build. */
 #define NAMOH_MAX_HEADS 64 /* H (or Hr) routed units */
 
@@ -189,6 +199,15 @@ NAMOH_API int namoh_prefill(const uint16_t *q, const uint16_t *k, const uint16_t
                   const float *gate, uint16_t *y, uint16_t *k_cache, uint16_t *v_cache, const int64_t *seg_base,
                   const int32_t *seg_cap, int64_t cache_rows, int32_t *seg_len, void *workspace,
                   size_t workspace_bytes, uint32_t *dev_status, void *stream);
+/* namoh_prefill_ex: namoh_prefill with rope_flags (NAMOH_ROPE_*; unknown bits are
+ * NAMOH_ERR_INVALID_ARG).  Under NAMOH_ROPE_GLOBAL the position of packed row r is
+ * t = (row_src[r] / Kr) % T.  namoh_prefill is namoh_prefill_ex with rope_flags = 0. */
+NAMOH_API int namoh_prefill_ex(const uint16_t *q, const uint16_t *k, const uint16_t *v, int B, int T, int H, int K,
+                               int d_head, int group, float rope_base, unsigned rope_flags,
+                               const int32_t *seg_offsets, const int32_t *row_src, const float *gate, uint16_t *y,
+                               uint16_t *k_cache, uint16_t *v_cache, const int64_t *seg_base,
+                               const int32_t *seg_cap, int64_t cache_rows, int32_t *seg_len, void *workspace,
+                               size_t workspace_bytes, uint32_t *dev_status, void *stream);
 
 /* ------------------------------------------------------------------------- *
  * The three stages of namoh_prefill, callable one by one (same arguments and
@@ -219,6 +238,15 @@ NAMOH_API int namoh_rope_pack(const uint16_t *q, const uint16_t *k, const uint16
                               uint16_t *k_cache, uint16_t *v_cache, const int64_t *seg_base, const int32_t *seg_cap,
                               int64_t cache_rows, uint32_t *dev_status, void *plan, size_t plan_bytes,
                               void *stream);
+/* namoh_rope_pack_ex: namoh_rope_pack with rope_flags (NAMOH_ROPE_*) and row_src
+ * ([R] int32, the routing's inverse map; read only under NAMOH_ROPE_GLOBAL, where it
+ * must not be NULL). */
+NAMOH_API int namoh_rope_pack_ex(const uint16_t *q, const uint16_t *k, const uint16_t *v, int B, int T, int H,
+                                 int K, int d_head, int group, float rope_base, unsigned rope_flags,
+                                 const int32_t *seg_offsets, const int32_t *row_src, uint16_t *q_rot,
+                                 uint16_t *k_cache, uint16_t *v_cache, const int64_t *seg_base,
+                                 const int32_t *seg_cap, int64_t cache_rows, uint32_t *dev_status, void *plan,
+                                 size_t plan_bytes, void *stream);
 NAMOH_API size_t namoh_attention_plan_size(int B, int T, int H, int K, int group);
 NAMOH_API int namoh_attention_plan(const int32_t *seg_offsets, int B, int T, int H, int K, int group,
                                    const int32_t *seg_cap, void *plan, size_t plan_bytes, void *stream);
@@ -252,6 +280,16 @@ NAMOH_API int namoh_decode(const int32_t *topk_head, const float *gate, const ui
                  uint16_t *k_cache, uint16_t *v_cache, const int64_t *seg_base, int32_t *seg_len,
                  const int32_t *seg_cap, int64_t cache_rows, uint16_t *y, void *workspace,
                  size_t workspace_bytes, uint32_t *dev_status, void *stream);
+/* namoh_decode_ex: namoh_decode with rope_flags (NAMOH_ROPE_*) and token_pos ([B]
+ * int64, the new tokens' indices in their sequences, each in [0, 2^24)): NULL unless
+ * NAMOH_ROPE_GLOBAL is set, and required when it is.  The new token is then rotated
+ * to token_pos[b]; its cache row is still seg_base[s] + rho. */
+NAMOH_API int namoh_decode_ex(const int32_t *topk_head, const float *gate, const uint16_t *q, const uint16_t *k,
+                              const uint16_t *v, int B, int H, int K, int d_head, int group, float rope_base,
+                              unsigned rope_flags, const int64_t *token_pos, uint16_t *k_cache, uint16_t *v_cache,
+                              const int64_t *seg_base, int32_t *seg_len, const int32_t *seg_cap, int64_t cache_rows,
+                              uint16_t *y, void *workspace, size_t workspace_bytes, uint32_t *dev_status,
+                              void *stream);
 
 #ifdef __cplusplus
 }

@@ -110,9 +110,14 @@ def namoh_route(scores: torch.Tensor, K: int, compact: bool = True, workspace: O
     return out
 
 
+def _rope_flags(interleaved: bool, global_positions: bool) -> int:
+    return (_abi.NAMOH_ROPE_INTERLEAVED if interleaved else 0) | (_abi.NAMOH_ROPE_GLOBAL if global_positions else 0)
+
+
 def namoh_prefill(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, seg_offsets: torch.Tensor,
                   row_src: torch.Tensor, gate: torch.Tensor, *, B: int, T: int, H: int, K: int, group: int = 1,
-                  rope_base: float = 10000.0, y: Optional[torch.Tensor] = None,
+                  rope_base: float = 10000.0, interleaved: bool = False, global_positions: bool = False,
+                  y: Optional[torch.Tensor] = None,
                   k_cache: Optional[torch.Tensor] = None, v_cache: Optional[torch.Tensor] = None,
                   seg_base: Optional[torch.Tensor] = None, seg_cap: Optional[torch.Tensor] = None,
                   seg_len: Optional[torch.Tensor] = None, workspace: Optional[Workspace] = None,
@@ -121,6 +126,7 @@ def namoh_prefill(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, seg_offsets
 
     q [R*g, d], k / v [R, d] bf16; returns (y [B, T, K, d], k_cache, v_cache).
     With v_cache omitted and no seg_base, v itself serves as the value cache.
+    interleaved / global_positions select the RoPE variants (NAMOH_ROPE_* in the header).
     """
     lib = _abi.load()
     d = q.shape[-1]
@@ -140,22 +146,25 @@ def namoh_prefill(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, seg_offsets
         raise NamohError("namoh_prefill_workspace_size", _abi.NAMOH_ERR_UNSUPPORTED)
     ws = _ws(workspace, nbytes, dev)
     st = _status(status, dev)
-    rc = lib.namoh_prefill(_ptr(q), _ptr(k), _ptr(v), B, T, H, K, d, group, float(rope_base), _ptr(seg_offsets),
-                           _ptr(row_src), _ptr(gate), _ptr(y), _ptr(k_cache), _ptr(v_cache), _ptr(seg_base),
-                           _ptr(seg_cap), cache_rows, _ptr(seg_len), _ptr(ws), ws.numel(), _ptr(st), _stream(stream))
-    _abi.check("namoh_prefill", rc)
+    rc = lib.namoh_prefill_ex(_ptr(q), _ptr(k), _ptr(v), B, T, H, K, d, group, float(rope_base),
+                              _rope_flags(interleaved, global_positions), _ptr(seg_offsets), _ptr(row_src),
+                              _ptr(gate), _ptr(y), _ptr(k_cache), _ptr(v_cache), _ptr(seg_base), _ptr(seg_cap),
+                              cache_rows, _ptr(seg_len), _ptr(ws), ws.numel(), _ptr(st), _stream(stream))
+    _abi.check("namoh_prefill_ex", rc)
     return y, k_cache, v_cache
 
 
 def namoh_rope_pack(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, seg_offsets: torch.Tensor, *, B: int, T: int,
-                    H: int, K: int, group: int = 1, rope_base: float = 10000.0, q_rot: Optional[torch.Tensor] = None,
+                    H: int, K: int, group: int = 1, rope_base: float = 10000.0, interleaved: bool = False,
+                    row_src: Optional[torch.Tensor] = None, q_rot: Optional[torch.Tensor] = None,
                     k_cache: Optional[torch.Tensor] = None, v_cache: Optional[torch.Tensor] = None,
                     seg_base: Optional[torch.Tensor] = None, seg_cap: Optional[torch.Tensor] = None,
                     status: Optional[torch.Tensor] = None, plan: Optional[torch.Tensor] = None, stream=None):
     """Prefill stage 1: RoPE at rank and cache pack.  Returns (q_rot, k_cache, v_cache).
 
     With ``plan`` (a buffer from namoh_attention_plan) the same launch also rebuilds the
-    attention plan for these seg_offsets."""
+    attention plan for these seg_offsets.  Passing ``row_src`` selects global positions
+    (NAMOH_ROPE_GLOBAL); ``interleaved`` the (2j, 2j+1) pairing."""
     lib = _abi.load()
     d = q.shape[-1]
     dev = q.device
@@ -164,11 +173,12 @@ def namoh_rope_pack(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, seg_offse
     if v_cache is None:
         v_cache = v if seg_base is None else torch.empty_like(v)
     st = _status(status, dev)
-    rc = lib.namoh_rope_pack(_ptr(q), _ptr(k), _ptr(v), B, T, H, K, d, group, float(rope_base), _ptr(seg_offsets),
-                             _ptr(q_rot), _ptr(k_cache), _ptr(v_cache), _ptr(seg_base), _ptr(seg_cap),
-                             k_cache.shape[0], _ptr(st), _ptr(plan), 0 if plan is None else plan.numel(),
-                             _stream(stream))
-    _abi.check("namoh_rope_pack", rc)
+    rc = lib.namoh_rope_pack_ex(_ptr(q), _ptr(k), _ptr(v), B, T, H, K, d, group, float(rope_base),
+                                _rope_flags(interleaved, row_src is not None), _ptr(seg_offsets), _ptr(row_src),
+                                _ptr(q_rot), _ptr(k_cache), _ptr(v_cache), _ptr(seg_base), _ptr(seg_cap),
+                                k_cache.shape[0], _ptr(st), _ptr(plan), 0 if plan is None else plan.numel(),
+                                _stream(stream))
+    _abi.check("namoh_rope_pack_ex", rc)
     return q_rot, k_cache, v_cache
 
 
@@ -207,11 +217,15 @@ def namoh_attention(q_rot: torch.Tensor, k_cache: torch.Tensor, v_cache: torch.T
 
 
 def namoh_decode(topk_head: torch.Tensor, gate: torch.Tensor, q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, *,
-                 H: int, K: int, group: int = 1, rope_base: float = 10000.0, k_cache: torch.Tensor,
+                 H: int, K: int, group: int = 1, rope_base: float = 10000.0, interleaved: bool = False,
+                 token_pos: Optional[torch.Tensor] = None, k_cache: torch.Tensor,
                  v_cache: torch.Tensor, seg_base: torch.Tensor, seg_len: torch.Tensor, seg_cap: torch.Tensor,
                  y: Optional[torch.Tensor] = None, workspace: Optional[Workspace] = None,
                  status: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
-    """One decode step (see namoh_decode in include/namoh.h).  Returns y [B, K, d] bf16."""
+    """One decode step (see namoh_decode in include/namoh.h).  Returns y [B, K, d] bf16.
+
+    token_pos (int64 [B], the new tokens' indices) selects global positions (NAMOH_ROPE_GLOBAL);
+    interleaved the (2j, 2j+1) pairing."""
     lib = _abi.load()
     B = topk_head.shape[0]
     d = q.shape[-1]
@@ -223,8 +237,11 @@ def namoh_decode(topk_head: torch.Tensor, gate: torch.Tensor, q: torch.Tensor, k
         raise NamohError("namoh_decode_workspace_size", _abi.NAMOH_ERR_UNSUPPORTED)
     ws = _ws(workspace, nbytes, dev)
     st = _status(status, dev)
-    rc = lib.namoh_decode(_ptr(topk_head), _ptr(gate), _ptr(q), _ptr(k), _ptr(v), B, H, K, d, group,
-                          float(rope_base), _ptr(k_cache), _ptr(v_cache), _ptr(seg_base), _ptr(seg_len),
-                          _ptr(seg_cap), k_cache.shape[0], _ptr(y), _ptr(ws), ws.numel(), _ptr(st), _stream(stream))
-    _abi.check("namoh_decode", rc)
+    if token_pos is not None and (token_pos.dtype != torch.int64 or token_pos.numel() != B):
+        raise ValueError("token_pos must be int64 with one entry per sequence")
+    rc = lib.namoh_decode_ex(_ptr(topk_head), _ptr(gate), _ptr(q), _ptr(k), _ptr(v), B, H, K, d, group,
+                             float(rope_base), _rope_flags(interleaved, token_pos is not None), _ptr(token_pos),
+                             _ptr(k_cache), _ptr(v_cache), _ptr(seg_base), _ptr(seg_len), _ptr(seg_cap),
+                             k_cache.shape[0], _ptr(y), _ptr(ws), ws.numel(), _ptr(st), _stream(stream))
+    _abi.check("namoh_decode_ex", rc)
     return y

@@ -20,6 +20,9 @@ NAMOH_DEV_NONFINITE_SCORE = 0x1
 NAMOH_DEV_CAPACITY = 0x2
 NAMOH_DEV_TIMEOUT = 0x4
 
+NAMOH_ROPE_INTERLEAVED = 0x1
+NAMOH_ROPE_GLOBAL = 0x2
+
 _lock = threading.Lock()
 _lib = None
 
@@ -28,6 +31,7 @@ _I = ctypes.c_int
 _I64 = ctypes.c_int64
 _SZ = ctypes.c_size_t
 _F = ctypes.c_float
+_U = ctypes.c_uint
 
 SIGNATURES = {
     "namoh_status_string": (ctypes.c_char_p, [_I]),
@@ -42,12 +46,18 @@ SIGNATURES = {
                            _SZ, _P, _P]),
     "namoh_rope_pack": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _P, _I64, _P, _P, _SZ,
                              _P]),
+    "namoh_prefill_ex": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _U, _P, _P, _P, _P, _P, _P, _P, _P, _I64,
+                              _P, _P, _SZ, _P, _P]),
+    "namoh_rope_pack_ex": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _U, _P, _P, _P, _P, _P, _P, _P, _I64, _P,
+                                _P, _SZ, _P]),
     "namoh_attention_plan_size": (_SZ, [_I, _I, _I, _I, _I]),
     "namoh_attention_plan": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _SZ, _P]),
     "namoh_attention": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _P, _I64, _P, _SZ, _P, _P, _P]),
     "namoh_decode_workspace_size": (_SZ, [_I, _I, _I, _I, _I]),
     "namoh_decode": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _I64, _P, _P, _SZ, _P,
                           _P]),
+    "namoh_decode_ex": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _F, _U, _P, _P, _P, _P, _P, _P, _I64, _P, _P,
+                             _SZ, _P, _P]),
 }
 
 

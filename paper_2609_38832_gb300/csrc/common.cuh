@@ -38,6 +38,7 @@ const char* last_error_text();
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+inline bool rope_flags_ok(unsigned f) { return (f & ~(unsigned)(NAMOH_ROPE_INTERLEAVED | NAMOH_ROPE_GLOBAL)) == 0; }
 
 // A simple bump allocator over the caller's workspace.
 struct WorkspaceCarver {
@@ -382,6 +383,38 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 }
 __device__ __forceinline__ float bf16_lo(uint32_t u) { return __uint_as_float(u << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t u) { return __uint_as_float(u & 0xFFFF0000u); }
+
+// Unsigned 32-bit division by a divisor fixed at launch, as a multiply-high and shifts
+// (Granlund and Montgomery, "Division by Invariant Integers using Multiplication", 1994,
+// Fig. 4.1): with l = ceil(log2 d) and m = floor(2^32 (2^l - d) / d) + 1,
+// n / d = (t + ((n - t) >> min(l, 1))) >> max(l - 1, 0), t = mulhi(m, n), for every n < 2^32.
+struct FastDiv {
+  uint32_t m;
+  int sh1, sh2;
+  uint32_t d;
+};
+inline FastDiv make_fastdiv(uint32_t d) {  // host; d >= 1
+  int l = 0;
+  while ((1ull << l) < d) ++l;
+  FastDiv f;
+  f.m = (uint32_t)(((1ull << 32) * ((1ull << l) - d)) / d + 1);
+  f.sh1 = l < 1 ? l : 1;
+  f.sh2 = l > 1 ? l - 1 : 0;
+  f.d = d;
+  return f;
+}
+__device__ __forceinline__ uint32_t fastdiv(uint32_t n, const FastDiv& f) {
+  const uint32_t t = __umulhi(f.m, n);
+  return (t + ((n - t) >> f.sh1)) >> f.sh2;
+}
+
+// A register copy the compiler cannot rematerialise from its source (e.g. re-read from the
+// kernel parameter bank inside a loop).
+__device__ __forceinline__ float opaque_f32(float x) {
+  float y;
+  asm volatile("mov.b32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 
 // RoPE frequency table passed by value to the kernels: theta_j = base^(-2j/d) split as
 // hi + lo (hi = fp32 rounding of the fp64 value, lo = fp32 rounding of the remainder),

@@ -3,9 +3,11 @@
 // or updated; App. C "Adopted KV-group routing" for g > 1).
 //
 // Three launches:
-//   1. decode_append_kernel  one warp per (sequence, slot): rho = seg_len[s]; k~ = k R(rho)
+//   1. decode_append_kernel  one warp per (sequence, slot): rho = seg_len[s]; k~ = k R(p)
 //                            and v are written at cache row seg_base[s] + rho; the g queries
-//                            are rotated to rho (kept in fp32 in the workspace).
+//                            are rotated to p (kept in fp32 in the workspace).  p is rho, or
+//                            the token's index in its sequence under global RoPE (Sec. 3.2);
+//                            pairs (j, j + D/2), or (2j, 2j + 1) when interleaved.
 //   2. decode_split_kernel   grid (splits, pairs): each CTA streams a contiguous range of the
 //                            pair's rho + 1 cache rows.  A half-warp owns one row at a time
 //                            (16 lanes x 16-byte loads = 256 bytes = one bf16 row of d = 128)
@@ -40,7 +42,8 @@ __global__ void decode_append_kernel(const int32_t* __restrict__ topk_head, cons
                                      const int64_t* __restrict__ seg_base, const int32_t* __restrict__ seg_len,
                                      const int32_t* __restrict__ seg_cap, long long cache_rows, RopeTable tab,
                                      float* __restrict__ q_rot, PairInfo* __restrict__ info,
-                                     uint32_t* __restrict__ status) {
+                                     uint32_t* __restrict__ status, const int64_t* __restrict__ token_pos,
+                                     int interleaved) {
   constexpr int HALF = D / 2;
   const int pair = blockIdx.x;  // b * Kr + slot
   const int b = pair / Kr;
@@ -60,27 +63,29 @@ __global__ void decode_append_kernel(const int32_t* __restrict__ topk_head, cons
   }
   if (!room) return;
   const long long dst = base + rho;
+  const float p = token_pos ? (float)token_pos[b] : (float)rho;
   for (int jj = lane; jj < HALF; jj += 32) {
     float sn, cs;
-    rope_sincos((float)rho, tab.theta_hi[jj], tab.theta_lo[jj], tab, &sn, &cs);
+    rope_sincos(p, tab.theta_hi[jj], tab.theta_lo[jj], tab, &sn, &cs);
+    const int i0 = interleaved ? 2 * jj : jj, i1 = interleaved ? 2 * jj + 1 : jj + HALF;
     {
       const uint16_t* kr = k + (size_t)pair * D;
-      const float x0 = __uint_as_float((uint32_t)kr[jj] << 16);
-      const float x1 = __uint_as_float((uint32_t)kr[jj + HALF] << 16);
+      const float x0 = __uint_as_float((uint32_t)kr[i0] << 16);
+      const float x1 = __uint_as_float((uint32_t)kr[i1] << 16);
       const __nv_bfloat16 o0 = __float2bfloat16_rn(fmaf(x0, cs, -x1 * sn));
       const __nv_bfloat16 o1 = __float2bfloat16_rn(fmaf(x1, cs, x0 * sn));
-      k_cache[dst * D + jj] = *reinterpret_cast<const uint16_t*>(&o0);
-      k_cache[dst * D + jj + HALF] = *reinterpret_cast<const uint16_t*>(&o1);
-      v_cache[dst * D + jj] = v[(size_t)pair * D + jj];
-      v_cache[dst * D + jj + HALF] = v[(size_t)pair * D + jj + HALF];
+      k_cache[dst * D + i0] = *reinterpret_cast<const uint16_t*>(&o0);
+      k_cache[dst * D + i1] = *reinterpret_cast<const uint16_t*>(&o1);
+      v_cache[dst * D + i0] = v[(size_t)pair * D + i0];
+      v_cache[dst * D + i1] = v[(size_t)pair * D + i1];
     }
     for (int j = 0; j < g; ++j) {
       const uint16_t* qr = q + ((size_t)pair * g + j) * D;
-      const float x0 = __uint_as_float((uint32_t)qr[jj] << 16);
-      const float x1 = __uint_as_float((uint32_t)qr[jj + HALF] << 16);
+      const float x0 = __uint_as_float((uint32_t)qr[i0] << 16);
+      const float x1 = __uint_as_float((uint32_t)qr[i1] << 16);
       float* out = q_rot + ((size_t)pair * g + j) * D;
-      out[jj] = fmaf(x0, cs, -x1 * sn);
-      out[jj + HALF] = fmaf(x1, cs, x0 * sn);
+      out[i0] = fmaf(x0, cs, -x1 * sn);
+      out[i1] = fmaf(x1, cs, x0 * sn);
     }
   }
 }
@@ -325,17 +330,20 @@ extern "C" size_t namoh_decode_workspace_size(int B, int H, int K, int d_head, i
   return align_up(ws.used, 256);
 }
 
-extern "C" int namoh_decode(const int32_t* topk_head, const float* gate, const uint16_t* q, const uint16_t* k,
-                            const uint16_t* v, int B, int H, int K, int d_head, int group, float rope_base,
-                            uint16_t* k_cache, uint16_t* v_cache, const int64_t* seg_base, int32_t* seg_len,
-                            const int32_t* seg_cap, int64_t cache_rows, uint16_t* y, void* workspace,
-                            size_t workspace_bytes, uint32_t* dev_status, void* stream_v) {
+extern "C" int namoh_decode_ex(const int32_t* topk_head, const float* gate, const uint16_t* q, const uint16_t* k,
+                               const uint16_t* v, int B, int H, int K, int d_head, int group, float rope_base,
+                               unsigned rope_flags, const int64_t* token_pos, uint16_t* k_cache, uint16_t* v_cache,
+                               const int64_t* seg_base, int32_t* seg_len, const int32_t* seg_cap, int64_t cache_rows,
+                               uint16_t* y, void* workspace, size_t workspace_bytes, uint32_t* dev_status,
+                               void* stream_v) {
   if (!topk_head || !gate || !q || !k || !v || !k_cache || !v_cache || !seg_base || !seg_len || !seg_cap || !y ||
       !dev_status)
     return NAMOH_ERR_INVALID_ARG;
   if (B < 1 || group < 1 || H < 1 || K < 1 || K > H || H % group || K % group) return NAMOH_ERR_INVALID_ARG;
   if (H / group > NAMOH_MAX_HEADS || cache_rows < 1 || cache_rows >= (1ll << 40)) return NAMOH_ERR_INVALID_ARG;
   if (!(rope_base > 1.0f) || !isfinite(rope_base)) return NAMOH_ERR_INVALID_ARG;
+  if (!rope_flags_ok(rope_flags) || ((rope_flags & NAMOH_ROPE_GLOBAL) != 0) != (token_pos != nullptr))
+    return NAMOH_ERR_INVALID_ARG;
   if (!decode_dims_ok(d_head, group)) return NAMOH_ERR_UNSUPPORTED;
   if (!aligned16(k_cache) || !aligned16(v_cache) || !aligned16(q) || !aligned16(y)) return NAMOH_ERR_INVALID_ARG;
   const int D = d_head, g = group, Hr = H / g, Kr = K / g;
@@ -352,14 +360,15 @@ extern "C" int namoh_decode(const int32_t* topk_head, const float* gate, const u
 
   RopeTable tab;
   fill_rope_table(&tab, D, (double)rope_base);
+  const int interleaved = (rope_flags & NAMOH_ROPE_INTERLEAVED) ? 1 : 0;
   if (D == 128)
     decode_append_kernel<128><<<pairs, 32, 0, stream>>>(topk_head, q, k, v, Hr, Kr, g, k_cache, v_cache, seg_base,
                                                         seg_len, seg_cap, cache_rows, tab, dw.q_rot, dw.info,
-                                                        dev_status);
+                                                        dev_status, token_pos, interleaved);
   else
     decode_append_kernel<64><<<pairs, 32, 0, stream>>>(topk_head, q, k, v, Hr, Kr, g, k_cache, v_cache, seg_base,
                                                        seg_len, seg_cap, cache_rows, tab, dw.q_rot, dw.info,
-                                                       dev_status);
+                                                       dev_status, token_pos, interleaved);
   if (const int st = cuda_check_launch("decode_append_kernel launch")) return st;
 
   const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)D));
@@ -376,4 +385,13 @@ extern "C" int namoh_decode(const int32_t* topk_head, const float* gate, const u
     decode_merge_kernel<64><<<pairs, mthreads, 0, stream>>>(dw.info, gate, dw.part, splits, g, y, seg_len);
   if (const int st = cuda_check_launch("decode_merge_kernel launch")) return st;
   return NAMOH_OK;
+}
+
+extern "C" int namoh_decode(const int32_t* topk_head, const float* gate, const uint16_t* q, const uint16_t* k,
+                            const uint16_t* v, int B, int H, int K, int d_head, int group, float rope_base,
+                            uint16_t* k_cache, uint16_t* v_cache, const int64_t* seg_base, int32_t* seg_len,
+                            const int32_t* seg_cap, int64_t cache_rows, uint16_t* y, void* workspace,
+                            size_t workspace_bytes, uint32_t* dev_status, void* stream_v) {
+  return namoh_decode_ex(topk_head, gate, q, k, v, B, H, K, d_head, group, rope_base, 0u, nullptr, k_cache, v_cache,
+                         seg_base, seg_len, seg_cap, cache_rows, y, workspace, workspace_bytes, dev_status, stream_v);
 }

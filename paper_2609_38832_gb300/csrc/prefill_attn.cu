@@ -41,7 +41,8 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              const int32_t* seg_offsets, int nseg, const int64_t* seg_base, const int32_t* seg_cap,
                              long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache, bool copy_v,
                              const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream,
-                             void* plan, int plan_qtiles, const int32_t* plan_cap);
+                             void* plan, int plan_qtiles, const int32_t* plan_cap, const int32_t* pos_row_src,
+                             int pos_k, int pos_t, bool interleaved);
 
 namespace attn {
 
@@ -669,11 +670,12 @@ int launch_plan(const int32_t* seg_offsets, int nseg, int T, int g, const int32_
 
 // RoPE + cache pack; with a plan buffer also the attention plan (in the same launch when
 // the plan's shared memory is small, else as a second kernel).
-int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int Hr, int R,
-                         int d_head, int group, float rope_base, const int32_t* seg_offsets, uint16_t* q_rot,
-                         uint16_t* k_cache, uint16_t* v_cache, const int64_t* seg_base, const int32_t* seg_cap,
-                         long long cache_rows, uint32_t* dev_status, void* plan, const DeviceInfo& info,
-                         cudaStream_t stream) {
+// rope_flags: NAMOH_ROPE_GLOBAL takes the positions from row_src (t = (row_src[r] / Kr) % T).
+int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int Hr, int Kr, int R,
+                         int d_head, int group, float rope_base, unsigned rope_flags, const int32_t* seg_offsets,
+                         const int32_t* row_src, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache,
+                         const int64_t* seg_base, const int32_t* seg_cap, long long cache_rows, uint32_t* dev_status,
+                         void* plan, const DeviceInfo& info, cudaStream_t stream) {
   RopeTable tab;
   fill_rope_table(&tab, d_head, (double)rope_base);
   const int nseg = B * Hr;
@@ -682,7 +684,9 @@ int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v
   const bool fuse_plan = plan && plan_smem_ints(qtiles, nseg) * (int)sizeof(int) <= kFusedPlanSmemMax;
   const cudaError_t e = launch_rope_pack(d_head, q, k, v, R, group, seg_offsets, nseg, seg_base, seg_cap, cache_rows,
                                          q_rot, k_cache, v_cache, v_cache != v, tab, dev_status, info.sm_count, stream,
-                                         fuse_plan ? plan : nullptr, qtiles, plan_cap);
+                                         fuse_plan ? plan : nullptr, qtiles, plan_cap,
+                                         (rope_flags & NAMOH_ROPE_GLOBAL) ? row_src : nullptr, Kr, T,
+                                         (rope_flags & NAMOH_ROPE_INTERLEAVED) != 0);
   if (e != cudaSuccess) return cuda_fail(e, "rope_pack_kernel launch");
   if (plan && !fuse_plan) return launch_plan(seg_offsets, nseg, T, group, plan_cap, plan, stream);
   return NAMOH_OK;
@@ -725,17 +729,19 @@ bool device_ok(DeviceInfo* info) {  // a Blackwell datacenter part with the shar
 
 using namespace namoh;
 
-extern "C" int namoh_rope_pack(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int H, int K,
-                               int d_head, int group, float rope_base, const int32_t* seg_offsets, uint16_t* q_rot,
-                               uint16_t* k_cache, uint16_t* v_cache, const int64_t* seg_base, const int32_t* seg_cap,
-                               int64_t cache_rows, uint32_t* dev_status, void* plan, size_t plan_bytes,
-                               void* stream_v) {
+extern "C" int namoh_rope_pack_ex(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int H,
+                                  int K, int d_head, int group, float rope_base, unsigned rope_flags,
+                                  const int32_t* seg_offsets, const int32_t* row_src, uint16_t* q_rot,
+                                  uint16_t* k_cache, uint16_t* v_cache, const int64_t* seg_base,
+                                  const int32_t* seg_cap, int64_t cache_rows, uint32_t* dev_status, void* plan,
+                                  size_t plan_bytes, void* stream_v) {
   if (!q || !k || !v || !seg_offsets || !q_rot || !k_cache || !v_cache || !dev_status) return NAMOH_ERR_INVALID_ARG;
   int Hr, Kr;
   long long R;
   const int st = check_shape(B, T, H, K, d_head, group, &Hr, &Kr, &R);
   if (st != NAMOH_OK) return st;
   if (!(rope_base > 1.0f) || !isfinite(rope_base)) return NAMOH_ERR_INVALID_ARG;
+  if (!rope_flags_ok(rope_flags) || ((rope_flags & NAMOH_ROPE_GLOBAL) && !row_src)) return NAMOH_ERR_INVALID_ARG;
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(q_rot) || !aligned16(k_cache) ||
       !aligned16(v_cache))
     return NAMOH_ERR_INVALID_ARG;
@@ -749,9 +755,18 @@ extern "C" int namoh_rope_pack(const uint16_t* q, const uint16_t* k, const uint1
     return NAMOH_ERR_WORKSPACE;
   DeviceInfo info;
   if (!current_device_info(&info)) return cuda_fail(cudaGetLastError(), "device query");
-  return launch_rope_and_plan(q, k, v, B, T, Hr, (int)R, d_head, group, rope_base, seg_offsets, q_rot, k_cache,
-                              v_cache, seg_base, seg_cap, cache_rows, dev_status, plan, info,
+  return launch_rope_and_plan(q, k, v, B, T, Hr, Kr, (int)R, d_head, group, rope_base, rope_flags, seg_offsets,
+                              row_src, q_rot, k_cache, v_cache, seg_base, seg_cap, cache_rows, dev_status, plan, info,
                               reinterpret_cast<cudaStream_t>(stream_v));
+}
+
+extern "C" int namoh_rope_pack(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int H, int K,
+                               int d_head, int group, float rope_base, const int32_t* seg_offsets, uint16_t* q_rot,
+                               uint16_t* k_cache, uint16_t* v_cache, const int64_t* seg_base, const int32_t* seg_cap,
+                               int64_t cache_rows, uint32_t* dev_status, void* plan, size_t plan_bytes,
+                               void* stream_v) {
+  return namoh_rope_pack_ex(q, k, v, B, T, H, K, d_head, group, rope_base, 0u, seg_offsets, nullptr, q_rot, k_cache,
+                            v_cache, seg_base, seg_cap, cache_rows, dev_status, plan, plan_bytes, stream_v);
 }
 
 extern "C" size_t namoh_attention_plan_size(int B, int T, int H, int K, int group) {
@@ -807,12 +822,12 @@ extern "C" size_t namoh_prefill_workspace_size(int B, int T, int H, int K, int d
   return align_up(ws.used, 256);
 }
 
-extern "C" int namoh_prefill(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int H, int K,
-                             int d_head, int group, float rope_base, const int32_t* seg_offsets,
-                             const int32_t* row_src, const float* gate, uint16_t* y, uint16_t* k_cache,
-                             uint16_t* v_cache, const int64_t* seg_base, const int32_t* seg_cap, int64_t cache_rows,
-                             int32_t* seg_len, void* workspace, size_t workspace_bytes, uint32_t* dev_status,
-                             void* stream_v) {
+extern "C" int namoh_prefill_ex(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int H, int K,
+                                int d_head, int group, float rope_base, unsigned rope_flags,
+                                const int32_t* seg_offsets, const int32_t* row_src, const float* gate, uint16_t* y,
+                                uint16_t* k_cache, uint16_t* v_cache, const int64_t* seg_base,
+                                const int32_t* seg_cap, int64_t cache_rows, int32_t* seg_len, void* workspace,
+                                size_t workspace_bytes, uint32_t* dev_status, void* stream_v) {
   if (!q || !k || !v || !seg_offsets || !row_src || !gate || !y || !k_cache || !v_cache || !dev_status)
     return NAMOH_ERR_INVALID_ARG;
   int Hr, Kr;
@@ -820,6 +835,7 @@ extern "C" int namoh_prefill(const uint16_t* q, const uint16_t* k, const uint16_
   int st = check_shape(B, T, H, K, d_head, group, &Hr, &Kr, &R);
   if (st != NAMOH_OK) return st;
   if (!(rope_base > 1.0f) || !isfinite(rope_base)) return NAMOH_ERR_INVALID_ARG;
+  if (!rope_flags_ok(rope_flags)) return NAMOH_ERR_INVALID_ARG;
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(y) || !aligned16(k_cache) || !aligned16(v_cache))
     return NAMOH_ERR_INVALID_ARG;
   if (k_cache == k) return NAMOH_ERR_INVALID_ARG;
@@ -838,8 +854,8 @@ extern "C" int namoh_prefill(const uint16_t* q, const uint16_t* k, const uint16_
   if (!device_ok(&info)) return NAMOH_ERR_UNSUPPORTED;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
 
-  st = launch_rope_and_plan(q, k, v, B, T, Hr, (int)R, d_head, group, rope_base, seg_offsets, q_rot, k_cache, v_cache,
-                            seg_base, seg_cap, cache_rows, dev_status, plan, info, stream);
+  st = launch_rope_and_plan(q, k, v, B, T, Hr, Kr, (int)R, d_head, group, rope_base, rope_flags, seg_offsets, row_src,
+                            q_rot, k_cache, v_cache, seg_base, seg_cap, cache_rows, dev_status, plan, info, stream);
   if (st != NAMOH_OK) return st;
   if (seg_len) {
     seg_len_kernel<<<(B * Hr + 255) / 256, 256, 0, stream>>>(seg_offsets, B * Hr, seg_len);
@@ -847,4 +863,15 @@ extern "C" int namoh_prefill(const uint16_t* q, const uint16_t* k, const uint16_
   }
   return launch_attention(q_rot, k_cache, v_cache, B, T, Hr, Kr, d_head, group, seg_offsets, row_src, gate, seg_base,
                           cache_rows, plan, y, dev_status, info, stream);
+}
+
+extern "C" int namoh_prefill(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int H, int K,
+                             int d_head, int group, float rope_base, const int32_t* seg_offsets,
+                             const int32_t* row_src, const float* gate, uint16_t* y, uint16_t* k_cache,
+                             uint16_t* v_cache, const int64_t* seg_base, const int32_t* seg_cap, int64_t cache_rows,
+                             int32_t* seg_len, void* workspace, size_t workspace_bytes, uint32_t* dev_status,
+                             void* stream_v) {
+  return namoh_prefill_ex(q, k, v, B, T, H, K, d_head, group, rope_base, 0u, seg_offsets, row_src, gate, y, k_cache,
+                          v_cache, seg_base, seg_cap, cache_rows, seg_len, workspace, workspace_bytes, dev_status,
+                          stream_v);
 }

@@ -9,11 +9,18 @@
 // over seg_offsets (staged in shared memory), rho = r - seg_offsets[s], and each thread
 // rotates 8 pairs (j, j + D/2) with angles it computes once for the row; KV-group routing
 // shares the rank between the key and the row's g query heads (App. C).
+// Variants: the interleaved pairing (2j, 2j+1) keeps the same 16-byte accesses (elements
+// [8l, 8l+8) and [D/2 + 8l, D/2 + 8l + 8) for lane l of a group) and pairs adjacent elements
+// inside them, so the lane's angles are j = 4l..4l+3 and D/4 + 4l..D/4 + 4l+3; global
+// positions (Sec. 3.2: rho_i(t) replaced by t) take t = (row_src[r] / Kr) % T from the
+// routing's inverse map, loaded one chunk ahead; the cache row is still the rank.
 // Outputs: Q~ (bf16 scratch for the attention kernel), K~ into the key cache, and V copied
 // into the value cache unless the caller passed v_cache == v.  Given a plan buffer, block 0
 // builds the attention work list in the same launch.  Launched with programmatic dependent
 // launch: set-up overlaps the routing kernel's tail, and every read of routing outputs or
 // inputs comes after pdl_wait().
+#include <type_traits>
+
 #include "common.cuh"
 #include "plan.cuh"
 
@@ -48,16 +55,21 @@ __host__ __device__ constexpr size_t rope_smem_bytes(int nseg) {
   return (size_t)kRopeStages * RopeChunk<D, G>::kStageBytes + rope_offs_bytes(nseg) + kRopeStages * sizeof(uint64_t);
 }
 
-template <int D, int G>
+// kFlags: NAMOH_ROPE_INTERLEAVED and NAMOH_ROPE_GLOBAL (compile-time, so the default path
+// carries no branch of the variants)
+template <int D, int G, unsigned kFlags>
 __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     const uint16_t* __restrict__ q, const uint16_t* __restrict__ k, const uint16_t* __restrict__ v, int R,
     const int32_t* __restrict__ seg_offsets, int nseg, const int64_t* __restrict__ seg_base,
     const int32_t* __restrict__ seg_cap, long long cache_rows, uint16_t* __restrict__ q_rot,
     uint16_t* __restrict__ k_cache, uint16_t* __restrict__ v_cache, int copy_v, RopeTable tab,
     uint32_t* __restrict__ status, int* __restrict__ plan_header, int4* __restrict__ plan_items,
-    const int32_t* __restrict__ plan_cap, int plan_qtiles) {
+    const int32_t* __restrict__ plan_cap, int plan_qtiles, const int32_t* __restrict__ pos_row_src,
+    FastDiv pos_k, FastDiv pos_t) {
   using C = RopeChunk<D, G>;
   constexpr int HALF = D / 2;
+  constexpr bool kInterleaved = (kFlags & NAMOH_ROPE_INTERLEAVED) != 0;
+  constexpr bool kGlobal = (kFlags & NAMOH_ROPE_GLOBAL) != 0;
   extern __shared__ __align__(128) uint8_t smem_raw[];
   __shared__ int s_abort;
   pdl_launch_dependents();  // the attention kernel may start launching; it waits for this grid
@@ -106,13 +118,26 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
   float th_hi[8], th_lo[8];
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
-    th_hi[i] = tab.theta_hi[j0 + i];
-    th_lo[i] = tab.theta_lo[j0 + i];
+    const int j = kInterleaved ? (i < 4 ? 4 * lig + i : D / 4 + 4 * lig + i - 4) : j0 + i;
+    th_hi[i] = opaque_f32(tab.theta_hi[j]);  // kept in registers across the chunk loop
+    th_lo[i] = opaque_f32(tab.theta_lo[j]);
   }
   bool ok = true;
   int it = 0;
+  // global positions: row_src of this thread's row in the next chunk, loaded a chunk ahead
+  int token_next = 0;
+  if (kGlobal) {
+    const long long r_first = (long long)blk * C::kRows + prow;
+    if (blk < nchunks && r_first < R) token_next = __ldg(pos_row_src + r_first);
+  }
   for (int c = blk; c < nchunks; c += nblk, ++it) {
     const int st = it % kRopeStages;
+    int token_src = 0;  // row_src of this thread's row: (b*T + t)*Kr + slot
+    if (kGlobal) {
+      token_src = token_next;
+      const long long r_next = (long long)(c + nblk) * C::kRows + prow;
+      if (c + nblk < nchunks && r_next < R) token_next = __ldg(pos_row_src + r_next);
+    }
     ok = mbar_wait(&full[st], (it / kRopeStages) & 1, &s_abort, status);
     if (!__syncthreads_and(ok)) {
       ok = false;
@@ -128,27 +153,48 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
         if (offs[mid] <= r) lo = mid; else hi = mid;
       }
       const int rho = (int)(r - offs[lo]);
+      // position: the rank, or the token's index t in its sequence
+      float pos = (float)rho;
+      if (kGlobal) {
+        const uint32_t bt = fastdiv((uint32_t)token_src, pos_k);  // b*T + t
+        pos = (float)(bt - fastdiv(bt, pos_t) * pos_t.d);
+      }
       float sn[8], cs[8];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) rope_sincos((float)rho, th_hi[i], th_lo[i], tab, &sn[i], &cs[i]);
+      for (int i = 0; i < 8; ++i) rope_sincos(pos, th_hi[i], th_lo[i], tab, &sn[i], &cs[i]);
 
       // x'_j = x_j cos - x_{j+D/2} sin ;  x'_{j+D/2} = x_{j+D/2} cos + x_j sin
+      // (interleaved: the same with x_{2j} and x_{2j+1}, one bf16x2 word per pair)
       auto rotate = [&](const uint8_t* src_row, uint16_t* dst_row) {
-        const uint4 a = *reinterpret_cast<const uint4*>(src_row + j0 * 2);
-        const uint4 b = *reinterpret_cast<const uint4*>(src_row + (HALF + j0) * 2);
-        const uint32_t av[4] = {a.x, a.y, a.z, a.w};
-        const uint32_t bv[4] = {b.x, b.y, b.z, b.w};
-        uint32_t oa[4], ob[4];
+        if constexpr (kInterleaved) {
+          const uint4 a = *reinterpret_cast<const uint4*>(src_row + j0 * 2);
+          const uint4 b = *reinterpret_cast<const uint4*>(src_row + (HALF + j0) * 2);
+          const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+          uint32_t o[8];
 #pragma unroll
-        for (int p = 0; p < 4; ++p) {
-          const float x0 = bf16_lo(av[p]), x1 = bf16_hi(av[p]);
-          const float y0 = bf16_lo(bv[p]), y1 = bf16_hi(bv[p]);
-          const int i0 = 2 * p, i1 = 2 * p + 1;
-          oa[p] = pack_bf16x2(fmaf(x0, cs[i0], -y0 * sn[i0]), fmaf(x1, cs[i1], -y1 * sn[i1]));
-          ob[p] = pack_bf16x2(fmaf(y0, cs[i0], x0 * sn[i0]), fmaf(y1, cs[i1], x1 * sn[i1]));
+          for (int p = 0; p < 8; ++p) {
+            const float x0 = bf16_lo(w[p]), x1 = bf16_hi(w[p]);
+            o[p] = pack_bf16x2(fmaf(x0, cs[p], -x1 * sn[p]), fmaf(x1, cs[p], x0 * sn[p]));
+          }
+          *reinterpret_cast<uint4*>(dst_row + j0) = make_uint4(o[0], o[1], o[2], o[3]);
+          *reinterpret_cast<uint4*>(dst_row + HALF + j0) = make_uint4(o[4], o[5], o[6], o[7]);
+        } else {
+          const uint4 a = *reinterpret_cast<const uint4*>(src_row + j0 * 2);
+          const uint4 b = *reinterpret_cast<const uint4*>(src_row + (HALF + j0) * 2);
+          const uint32_t av[4] = {a.x, a.y, a.z, a.w};
+          const uint32_t bv[4] = {b.x, b.y, b.z, b.w};
+          uint32_t oa[4], ob[4];
+#pragma unroll
+          for (int p = 0; p < 4; ++p) {
+            const float x0 = bf16_lo(av[p]), x1 = bf16_hi(av[p]);
+            const float y0 = bf16_lo(bv[p]), y1 = bf16_hi(bv[p]);
+            const int i0 = 2 * p, i1 = 2 * p + 1;
+            oa[p] = pack_bf16x2(fmaf(x0, cs[i0], -y0 * sn[i0]), fmaf(x1, cs[i1], -y1 * sn[i1]));
+            ob[p] = pack_bf16x2(fmaf(y0, cs[i0], x0 * sn[i0]), fmaf(y1, cs[i1], x1 * sn[i1]));
+          }
+          *reinterpret_cast<uint4*>(dst_row + j0) = make_uint4(oa[0], oa[1], oa[2], oa[3]);
+          *reinterpret_cast<uint4*>(dst_row + HALF + j0) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
         }
-        *reinterpret_cast<uint4*>(dst_row + j0) = make_uint4(oa[0], oa[1], oa[2], oa[3]);
-        *reinterpret_cast<uint4*>(dst_row + HALF + j0) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
       };
 #pragma unroll
       for (int h = 0; h < C::kHeads; ++h) {
@@ -187,17 +233,19 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
   }
 }
 
-template <int D>
+template <int D, unsigned F>
 cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, bool with_plan, cudaStream_t stream,
                                const uint16_t* q, const uint16_t* k, const uint16_t* v, int R,
                                const int32_t* seg_offsets, const int64_t* seg_base, const int32_t* seg_cap,
                                long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache,
                                int copy_v, const RopeTable& tab, uint32_t* status, int* plan_header,
-                               int4* plan_items, const int32_t* plan_cap, int plan_qtiles) {
+                               int4* plan_items, const int32_t* plan_cap, int plan_qtiles,
+                               const int32_t* pos_row_src, FastDiv pos_k, FastDiv pos_t) {
   switch (g) {
 #define NAMOH_ROPE_CASE(GG)                                                                                       \
   case GG: {                                                                                                      \
     using C = RopeChunk<D, GG>;                                                                                  \
+    const auto kernel = rope_pack_kernel<D, GG, F>;                                                              \
     const size_t rope_smem = rope_smem_bytes<D, GG>(nseg);                                                       \
     const size_t smem0 = rope_smem > plan_smem ? rope_smem : plan_smem;                                          \
     /* two blocks per SM when their shared memory fits (228 KB per SM, 1 KB reserved per block); the */          \
@@ -212,13 +260,13 @@ cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, 
     const long long grid = blocks + (with_plan ? 1 : 0);                                                         \
     if (grid == 0) return cudaSuccess;                                                                           \
     if (smem > 48 * 1024) {                                                                                      \
-      cudaError_t e = cudaFuncSetAttribute(rope_pack_kernel<D, GG>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
+      cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,                 \
                                            (int)smem);                                                           \
       if (e != cudaSuccess) return e;                                                                            \
     }                                                                                                            \
-    return launch_pdl(rope_pack_kernel<D, GG>, dim3((unsigned)grid), dim3(kRopeThreads), smem, stream, q, k, v, R,  \
-                      seg_offsets, nseg, seg_base, seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v, tab,    \
-                      status, plan_header, plan_items, plan_cap, plan_qtiles);                                   \
+    return launch_pdl(kernel, dim3((unsigned)grid), dim3(kRopeThreads), smem, stream, q, k, v, R, seg_offsets,     \
+                      nseg, seg_base, seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v, tab, status,         \
+                      plan_header, plan_items, plan_cap, plan_qtiles, pos_row_src, pos_k, pos_t);                \
   }
     NAMOH_ROPE_CASE(1)
     NAMOH_ROPE_CASE(2)
@@ -235,18 +283,31 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              const int32_t* seg_offsets, int nseg, const int64_t* seg_base, const int32_t* seg_cap,
                              long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache, bool copy_v,
                              const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream,
-                             void* plan, int plan_qtiles, const int32_t* plan_cap) {
+                             void* plan, int plan_qtiles, const int32_t* plan_cap, const int32_t* pos_row_src,
+                             int pos_k, int pos_t, bool interleaved) {
   int* plan_header = static_cast<int*>(plan);
   int4* plan_items = plan ? reinterpret_cast<int4*>(static_cast<char*>(plan) + 16) : nullptr;
   const size_t plan_smem = plan ? (size_t)plan_smem_ints(plan_qtiles, nseg) * sizeof(int) : 0;
   if (R == 0 && !plan) return cudaSuccess;
-  if (D == 128)
-    return launch_rope_pack_d<128>(g, sm_count, nseg, plan_smem, plan != nullptr, stream, q, k, v, R, seg_offsets,
-                                   seg_base, seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status,
-                                   plan_header, plan_items, plan_cap, plan_qtiles);
-  return launch_rope_pack_d<64>(g, sm_count, nseg, plan_smem, plan != nullptr, stream, q, k, v, R, seg_offsets,
-                                seg_base, seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status,
-                                plan_header, plan_items, plan_cap, plan_qtiles);
+  const unsigned flags = (interleaved ? NAMOH_ROPE_INTERLEAVED : 0u) | (pos_row_src ? NAMOH_ROPE_GLOBAL : 0u);
+  auto go = [&](auto d_tag, auto f_tag) {
+    return launch_rope_pack_d<decltype(d_tag)::value, decltype(f_tag)::value>(
+        g, sm_count, nseg, plan_smem, plan != nullptr, stream, q, k, v, R, seg_offsets, seg_base, seg_cap, cache_rows,
+        q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status, plan_header, plan_items, plan_cap, plan_qtiles,
+        pos_row_src, make_fastdiv((uint32_t)pos_k), make_fastdiv((uint32_t)pos_t));
+  };
+  using D64 = std::integral_constant<int, 64>;
+  using D128 = std::integral_constant<int, 128>;
+  using F0 = std::integral_constant<unsigned, 0u>;
+  using F1 = std::integral_constant<unsigned, 1u>;
+  using F2 = std::integral_constant<unsigned, 2u>;
+  using F3 = std::integral_constant<unsigned, 3u>;
+  switch (flags) {
+    case 0u: return D == 128 ? go(D128{}, F0{}) : go(D64{}, F0{});
+    case 1u: return D == 128 ? go(D128{}, F1{}) : go(D64{}, F1{});
+    case 2u: return D == 128 ? go(D128{}, F2{}) : go(D64{}, F2{});
+    default: return D == 128 ? go(D128{}, F3{}) : go(D64{}, F3{});
+  }
 }
 
 }  // namespace namoh

@@ -77,3 +77,26 @@ def test_argument_errors_return_before_any_launch(lib):
     dargs = [fake, fake, fake, fake, fake, 2, 8, 2, 128, 1, 10000.0, fake, fake, None, fake, fake, 100, fake, fake,
              1 << 20, st, None]
     assert lib.namoh_decode(*dargs) == -1
+
+
+def test_rope_flag_errors_return_before_any_launch(lib):
+    P = ctypes.c_void_p
+    fake = P(256)
+    st = P(512)
+    G, IL = _abi.NAMOH_ROPE_GLOBAL, _abi.NAMOH_ROPE_INTERLEAVED
+    # prefill_ex: an unknown flag bit
+    pargs = [fake, fake, fake, 1, 16, 8, 2, 128, 1, 10000.0, 0x4, fake, fake, fake, fake, fake, fake, None, None, 0,
+             None, fake, 1 << 20, st, None]
+    assert lib.namoh_prefill_ex(*pargs) == -1
+    # rope_pack_ex: global positions need row_src
+    rargs = [fake, fake, fake, 1, 16, 8, 2, 128, 1, 10000.0, G | IL, fake, None, fake, fake, fake, None, None, 0, st,
+             None, 0, None]
+    assert lib.namoh_rope_pack_ex(*rargs) == -1
+    # decode_ex: token_pos exactly when global; unknown bits
+    dargs = [fake, fake, fake, fake, fake, 2, 8, 2, 128, 1, 10000.0, G, None, fake, fake, fake, fake, fake, 100, fake,
+             fake, 1 << 20, st, None]
+    assert lib.namoh_decode_ex(*dargs) == -1
+    a = list(dargs); a[11] = IL; a[12] = fake
+    assert lib.namoh_decode_ex(*a) == -1
+    a = list(dargs); a[11] = 0x8; a[12] = None
+    assert lib.namoh_decode_ex(*a) == -1

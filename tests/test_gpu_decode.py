@@ -19,7 +19,11 @@ def namoh():
     return pkg
 
 
-def _prefix_state(namoh, B, T, Hr, Kr, d, g, base, headroom, seed):
+def _variant(name: str) -> dict:
+    return dict(interleaved="interleaved" in name, global_positions=name.startswith("global"))
+
+
+def _prefix_state(namoh, B, T, Hr, Kr, d, g, base, headroom, seed, variant="rank"):
     """GPU prefill of a T-token prefix into caches with `headroom` free rows per segment."""
     scores = ni.router_scores(seed, B, T, Hr)
     R = B * T * Kr
@@ -37,7 +41,7 @@ def _prefix_state(namoh, B, T, Hr, Kr, d, g, base, headroom, seed):
     namoh.namoh_prefill(dev_bf16(q), dev_bf16(k), dev_bf16(v), ro.seg_offsets, ro.row_src, ro.gate, B=B, T=T,
                         H=Hr * g, K=Kr * g, group=g, rope_base=base, k_cache=kc, v_cache=vc,
                         seg_base=torch.from_numpy(seg_base).cuda(), seg_cap=torch.from_numpy(cap).cuda(),
-                        seg_len=seg_len, status=ro.status)
+                        seg_len=seg_len, status=ro.status, **_variant(variant))
     torch.cuda.synchronize()
     assert int(ro.status.item()) == 0
     return dict(kc=kc, vc=vc, seg_len=seg_len, seg_base=seg_base, cap=cap, n=n,
@@ -60,33 +64,64 @@ def _oracle_caches(st, d):
     (64, 40, 32, 4, 128, 1, 2),
 ])
 def test_decode_matches_oracle(namoh, oracle_mod, B, T, Hr, Kr, d, g, steps):
+    _decode_check(namoh, oracle_mod, B, T, Hr, Kr, d, g, steps, "rank")
+
+
+def _token_positions(B, T, t, steps):
+    """Distinct per-sequence token indices, up to the largest the ABI accepts (2^24 - 1)."""
+    tp = [T + t] + [131072 * b + 11 * b + t for b in range(1, B - 1)] + ([(1 << 24) - steps + t] if B > 1 else [])
+    return np.array(tp, np.int64)
+
+
+def _decode_check(namoh, oracle_mod, B, T, Hr, Kr, d, g, steps, variant):
     base = 10000.0
-    st = _prefix_state(namoh, B, T, Hr, Kr, d, g, base, steps, seed=21)
+    vkw = _variant(variant)
+    st = _prefix_state(namoh, B, T, Hr, Kr, d, g, base, steps, seed=21, variant=variant)
     okc, ovc, obase, olen, ocap = _oracle_caches(st, d)
     sc, q, k, v = ni.decode_step_inputs(22, steps, B, Hr, Kr, d, g)
     status = torch.zeros(1, dtype=torch.int32, device="cuda")
     for t in range(steps):
+        tp = _token_positions(B, T, t, steps) if vkw["global_positions"] else None
         ro = namoh.namoh_route(torch.from_numpy(sc[t][:, None, :]).cuda(), Kr, compact=False)
         y = namoh.namoh_decode(ro.topk_head.view(B, Kr), ro.gate.view(B, Kr), dev_bf16(q[t]), dev_bf16(k[t]),
                                dev_bf16(v[t]), H=Hr * g, K=Kr * g, group=g, rope_base=base, k_cache=st["kc"],
                                v_cache=st["vc"], seg_base=st["seg_base_d"], seg_len=st["seg_len"],
-                               seg_cap=st["cap_d"], status=status)
+                               seg_cap=st["cap_d"], status=status, interleaved=vkw["interleaved"],
+                               token_pos=None if tp is None else torch.from_numpy(tp).cuda())
         torch.cuda.synchronize()
         ref = oracle_mod.route(sc[t][:, None, :], Kr)
         np.testing.assert_array_equal(ro.topk_head.cpu().numpy(), ref["topk_head"])
         y_ref = oracle_mod.decode_step(ref["topk_head"][:, 0], ref["gate"][:, 0], q[t], k[t], v[t], Hr, d, g, base,
-                                       okc, ovc, obase, olen, ocap)
+                                       okc, ovc, obase, olen, ocap, interleaved=vkw["interleaved"], token_pos=tp)
         gate = np.repeat(ref["gate"][:, 0], g, axis=1)
         assert_close_attention(bf16_to_f64(y), y_ref, gate, what=f"step {t}")
         np.testing.assert_array_equal(st["seg_len"].cpu().numpy(), olen)
     assert int(status.item()) == 0
     # M_KV = T K after the prefix and + K per step (App. C Eq. app-routed-kv)
     assert int(st["seg_len"].sum().item()) == B * (T + steps) * Kr
+    # the appended keys: the oracle's k~ rounded to bf16
+    kc_got = bf16_to_f64(st["kc"])
+    for s_ in range(len(olen)):
+        lo, hi = int(obase[s_]), int(obase[s_] + olen[s_])
+        assert np.all(np.abs(kc_got[lo:hi] - okc[lo:hi]) <= np.abs(okc[lo:hi]) * 2.0 ** -7 + 1e-6)
 
 
-def test_prefill_then_decode_equals_longer_prefill(namoh, oracle_mod):
+@pytest.mark.parametrize("variant", ["interleaved", "global", "global_interleaved"])
+@pytest.mark.parametrize("B,T,Hr,Kr,d,g,steps", [
+    (3, 300, 8, 2, 128, 1, 3),
+    (2, 257, 4, 4, 64, 1, 2),
+    (2, 200, 4, 2, 128, 2, 3),
+])
+def test_decode_rope_variants_match_oracle(namoh, oracle_mod, B, T, Hr, Kr, d, g, steps, variant):
+    """Interleaved pairing, and global positions from token_pos (Sec. 3.2: t instead of rho)."""
+    _decode_check(namoh, oracle_mod, B, T, Hr, Kr, d, g, steps, variant)
+
+
+@pytest.mark.parametrize("variant", ["rank", "global_interleaved"])
+def test_prefill_then_decode_equals_longer_prefill(namoh, oracle_mod, variant):
     """Prefill over T tokens plus decode steps reproduces prefill over T + steps tokens."""
     B, T, Hr, Kr, d, steps, base = 2, 200, 8, 2, 128, 3, 10000.0
+    vkw = _variant(variant)
     Tt = T + steps
     s = ni.router_scores(31, B, Tt, Hr)
     R = B * Tt * Kr
@@ -94,7 +129,7 @@ def test_prefill_then_decode_equals_longer_prefill(namoh, oracle_mod):
     ref = oracle_mod.route(s, Kr)
     ro = namoh.namoh_route(torch.from_numpy(s).cuda(), Kr)
     y_full, _, _ = namoh.namoh_prefill(dev_bf16(q), dev_bf16(k), dev_bf16(v), ro.seg_offsets, ro.row_src, ro.gate,
-                                       B=B, T=Tt, H=Hr, K=Kr, rope_base=base)
+                                       B=B, T=Tt, H=Hr, K=Kr, rope_base=base, **vkw)
     # prefix rows: the packed rows of tokens < T keep their order
     tok = ref["row_src"] // Kr % Tt
     keep = np.nonzero(tok < T)[0]
@@ -110,13 +145,16 @@ def test_prefill_then_decode_equals_longer_prefill(namoh, oracle_mod):
     sb, cp = torch.from_numpy(seg_base).cuda(), torch.from_numpy(cap).cuda()
     namoh.namoh_prefill(dev_bf16(q[keep]), dev_bf16(k[keep]), dev_bf16(v[keep]), ro_p.seg_offsets, ro_p.row_src,
                         ro_p.gate, B=B, T=T, H=Hr, K=Kr, rope_base=base, k_cache=kc, v_cache=vc, seg_base=sb,
-                        seg_cap=cp, seg_len=seg_len)
+                        seg_cap=cp, seg_len=seg_len, **vkw)
     yf = bf16_to_f64(y_full).reshape(B, Tt, Kr, d)
     for t in range(T, Tt):
         rows_t = ref["row"][:, t]
         yd = namoh.namoh_decode(ro.topk_head[:, t].contiguous(), ro.gate[:, t].contiguous(), dev_bf16(q[rows_t]),
                                 dev_bf16(k[rows_t]), dev_bf16(v[rows_t]), H=Hr, K=Kr, rope_base=base, k_cache=kc,
-                                v_cache=vc, seg_base=sb, seg_len=seg_len, seg_cap=cp)
+                                v_cache=vc, seg_base=sb, seg_len=seg_len, seg_cap=cp,
+                                interleaved=vkw["interleaved"],
+                                token_pos=torch.full((B,), t, dtype=torch.int64, device="cuda")
+                                if vkw["global_positions"] else None)
         torch.cuda.synchronize()
         assert_close_attention(bf16_to_f64(yd), yf[:, t], ref["gate"][:, t], what=f"token {t}")
 

@@ -30,15 +30,22 @@ def _run_gpu(namoh, wl: ni.PrefillWorkload, scores, q, k, v, **kw):
     return ro, y, kc, vc
 
 
-def _full_check(namoh, oracle_mod, wl: ni.PrefillWorkload, scores=None):
+def _variant(name: str) -> dict:
+    """RoPE variant keywords of namoh_prefill (Sec. 3.2: global positions replace the rank)."""
+    return dict(interleaved="interleaved" in name, global_positions=name.startswith("global"))
+
+
+def _full_check(namoh, oracle_mod, wl: ni.PrefillWorkload, scores=None, variant: str = "rank"):
     scores = wl.scores() if scores is None else scores
     q, k, v = wl.qkv()
-    ro, y, kc, _ = _run_gpu(namoh, wl, scores, q, k, v)
+    kw = _variant(variant)
+    ro, y, kc, _ = _run_gpu(namoh, wl, scores, q, k, v, **kw)
     assert int(ro.status.item()) == 0
     ref = oracle_mod.route(scores, wl.Kr)
     np.testing.assert_array_equal(ro.seg_offsets.cpu().numpy(), ref["seg_offsets"])
+    pos = oracle_mod.global_positions(ref["row_src"], wl.T, wl.Kr) if kw["global_positions"] else None
     y_ref, krot = oracle_mod.prefill(q, k, v, ref["seg_offsets"], ref["row_src"], ref["gate"], wl.d, wl.g, wl.base,
-                                     return_krot=True)
+                                     return_krot=True, interleaved=kw["interleaved"], pos=pos)
     got = bf16_to_f64(y).reshape(-1, wl.d)
     gate = np.repeat(ref["gate"].reshape(-1), wl.g)
     assert_close_attention(got, y_ref, gate)
@@ -114,18 +121,20 @@ def test_prefill_cache_layout_with_headroom_and_capacity(namoh, oracle_mod):
     assert_close_attention(got, y_ref[keep], ref["gate"].reshape(-1)[keep])
 
 
-def _sampled_check(namoh, oracle_mod, wl: ni.PrefillWorkload, nsamples: int = 160):
+def _sampled_check(namoh, oracle_mod, wl: ni.PrefillWorkload, nsamples: int = 160, variant: str = "rank"):
     scores = wl.scores()
     q, k, v = wl.qkv()
-    ro, y, _, _ = _run_gpu(namoh, wl, scores, q, k, v)
+    kw = _variant(variant)
+    ro, y, _, _ = _run_gpu(namoh, wl, scores, q, k, v, **kw)
     assert int(ro.status.item()) == 0
     ref = oracle_mod.route(scores, wl.Kr)
     seg = ro.seg_offsets.cpu().numpy()
     np.testing.assert_array_equal(seg, ref["seg_offsets"])
     rows = sample_rows(seg, nsamples)
     heads = (np.arange(len(rows)) % wl.g).astype(np.int32)
+    pos = oracle_mod.global_positions(ref["row_src"], wl.T, wl.Kr) if kw["global_positions"] else None
     expect = oracle_mod.prefill_rows(q, k, v, ref["seg_offsets"], ref["row_src"], ref["gate"], wl.d, wl.g, wl.base,
-                                     rows, heads)
+                                     rows, heads, interleaved=kw["interleaved"], pos=pos)
     yflat = bf16_to_f64(y).reshape(-1, wl.d)
     dst = ref["row_src"][rows].astype(np.int64) * wl.g + heads
     assert_close_attention(yflat[dst], expect, ref["gate"].reshape(-1)[ref["row_src"][rows]])
@@ -137,6 +146,39 @@ def test_prefill_full_size_sampled(namoh, oracle_mod, wl):
     _sampled_check(namoh, oracle_mod, wl)
 
 
+VARIANTS = ["interleaved", "global", "global_interleaved"]
+
+
+@pytest.mark.parametrize("variant", VARIANTS)
+@pytest.mark.parametrize("wl", [
+    ni.PrefillWorkload("small_d128", B=2, T=700, H=4, K=2, d=128),
+    ni.PrefillWorkload("small_d64_ragged", B=3, T=333, H=6, K=3, d=64, seed=3),
+    ni.PrefillWorkload("gqa_g4_d64", B=2, T=260, H=16, K=8, d=64, g=4, seed=8),
+    ni.PrefillWorkload("base5e5_long_segment", B=1, T=2500, H=4, K=1, d=128, base=500000.0, seed=9),
+], ids=lambda w: w.name)
+def test_prefill_rope_variants_match_oracle(namoh, oracle_mod, wl, variant):
+    """Interleaved pairing and global positions (t instead of rho), against the oracle in the
+    same variant: outputs and the rotated keys in the cache."""
+    _full_check(namoh, oracle_mod, wl, variant=variant)
+
+
+def test_prefill_k_equals_h_global_is_rank(namoh):
+    """K = H: every rank is t, so global positions give the same bytes."""
+    wl = ni.PrefillWorkload("dense_k_eq_h", B=1, T=300, H=4, K=4, d=128, seed=4)
+    scores = wl.scores()
+    q, k, v = wl.qkv()
+    _, y0, kc0, _ = _run_gpu(namoh, wl, scores, q, k, v)
+    _, y1, kc1, _ = _run_gpu(namoh, wl, scores, q, k, v, global_positions=True)
+    assert torch.equal(y0.view(torch.int16), y1.view(torch.int16))
+    assert torch.equal(kc0.view(torch.int16), kc1.view(torch.int16))
+
+
+@pytest.mark.parametrize("variant", ["global", "global_interleaved"])
+def test_prefill_full_size_sampled_global(namoh, oracle_mod, variant):
+    """Global positions reach T - 1 (32767 here, base 5e5) instead of about T K / H."""
+    _sampled_check(namoh, oracle_mod, ni.SKEWED, variant=variant)
+
+
 def test_prefill_many_segments_unstaged(namoh, oracle_mod):
     """B*H = 8320 segments: more offsets than the RoPE kernel stages in shared memory and a
     plan too large to build inside the RoPE launch (separate plan kernel)."""
@@ -145,23 +187,27 @@ def test_prefill_many_segments_unstaged(namoh, oracle_mod):
 
 @pytest.mark.parametrize("wl", [ni.PR1, ni.PrefillWorkload("gqa_g4_staged", B=2, T=900, H=16, K=8, d=128, g=4, seed=12)],
                          ids=lambda w: w.name)
-def test_staged_calls_match_prefill(namoh, wl):
+@pytest.mark.parametrize("variant", ["rank", "global_interleaved"])
+def test_staged_calls_match_prefill(namoh, wl, variant):
     """namoh_rope_pack (building the plan in the same launch, or not) + namoh_attention give
     the bytes namoh_prefill gives."""
     scores = wl.scores()
     q, k, v = (dev_bf16(a) for a in wl.qkv())
     ro = namoh.namoh_route(torch.from_numpy(scores).cuda(), wl.Kr)
+    vkw = _variant(variant)
     y_ref, _, _ = namoh.namoh_prefill(q, k, v, ro.seg_offsets, ro.row_src, ro.gate, B=wl.B, T=wl.T, H=wl.H, K=wl.K,
-                                      group=wl.g, rope_base=wl.base, status=ro.status)
+                                      group=wl.g, rope_base=wl.base, status=ro.status, **vkw)
     kw = dict(B=wl.B, T=wl.T, H=wl.H, K=wl.K, group=wl.g)
+    rkw = dict(interleaved=vkw["interleaved"], row_src=ro.row_src if vkw["global_positions"] else None)
     for fused in (True, False):
         plan = namoh.namoh_attention_plan(ro.seg_offsets, **kw)
         plan.fill_(0xAB)  # stale bytes: the fused launch must rebuild every word it uses
         if fused:
             q_rot, kc, vc = namoh.namoh_rope_pack(q, k, v, ro.seg_offsets, rope_base=wl.base, status=ro.status,
-                                                  plan=plan, **kw)
+                                                  plan=plan, **kw, **rkw)
         else:
-            q_rot, kc, vc = namoh.namoh_rope_pack(q, k, v, ro.seg_offsets, rope_base=wl.base, status=ro.status, **kw)
+            q_rot, kc, vc = namoh.namoh_rope_pack(q, k, v, ro.seg_offsets, rope_base=wl.base, status=ro.status,
+                                                  **kw, **rkw)
             namoh.namoh_attention_plan(ro.seg_offsets, plan=plan, **kw)
         y = namoh.namoh_attention(q_rot, kc, vc, ro.seg_offsets, ro.row_src, ro.gate, plan, status=ro.status, **kw)
         torch.cuda.synchronize()
