@@ -69,13 +69,15 @@ def _load():
         lib.oracle_route_topk.argtypes = [P, i64, i32, i32, P, P]
         lib.oracle_route_biased.argtypes = [P, P, i64, i32, i32, P, P, P]
         lib.oracle_dispatch.argtypes = [P, i32, i32, i32, i32, P, P, P, P, P]
+        lib.oracle_dispatch_varlen.argtypes = [P, P, i32, i32, i32, P, P, P, P, P]
         lib.oracle_rope.argtypes = [P, i64, i32, i64, P, f64, i32, P]
         lib.oracle_prefill.argtypes = [P, P, P, i32, i32, i32, f64, P, P, P, P, P, i32, i32, P]
         lib.oracle_prefill_rows.argtypes = [P, P, P, i32, i32, i32, f64, P, P, P, P, P, i64, P, i32, P]
         lib.oracle_decode_step.argtypes = [P, P, P, P, P, i32, i32, i32, i32, i32, f64,
                                            P, P, P, P, P, P, i32, P]
         lib.oracle_default_threads.argtypes = []
-        for fn in ("oracle_route_topk", "oracle_route_biased", "oracle_dispatch", "oracle_rope", "oracle_prefill",
+        for fn in ("oracle_route_topk", "oracle_route_biased", "oracle_dispatch", "oracle_dispatch_varlen",
+                   "oracle_rope", "oracle_prefill",
                    "oracle_prefill_rows", "oracle_decode_step", "oracle_default_threads"):
             getattr(lib, fn).restype = ctypes.c_int
         _lib = lib
@@ -132,6 +134,39 @@ def dispatch(topk_head: np.ndarray, H: int) -> dict:
     return dict(n=n, seg_offsets=seg, rank=rank, row=row, row_src=row_src)
 
 
+def route_varlen(scores: np.ndarray, cu_seqlens: np.ndarray, K: int, bias: np.ndarray | None = None) -> dict:
+    """Routing and dispatch of a ragged batch: scores [N, H] over the flat token axis, sequence
+    b = tokens cu_seqlens[b] .. cu_seqlens[b+1]-1.  Biased selection when bias [H] is given.
+
+    Returns topk_head [N,K], gate [N,K] fp64, n [B,H], seg_offsets [B*H+1], rank [N,K],
+    row [N,K] and row_src [N*K] (row_src[row] = tok*K + slot).
+    """
+    lib = _load()
+    scores = np.ascontiguousarray(scores, dtype=np.float32)
+    cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
+    N, H = scores.shape
+    B = len(cu) - 1
+    if B < 0 or cu[0] != 0 or cu[-1] != N or np.any(np.diff(cu) < 0):
+        raise OracleError("cu_seqlens must start at 0, not decrease and end at N")
+    topk = np.empty((N, K), np.int32)
+    gate = np.empty((N, K), np.float64)
+    if bias is None:
+        _check(lib.oracle_route_topk(_ptr(scores), N, H, K, _ptr(topk), _ptr(gate)), "route_topk")
+    else:
+        bias = np.ascontiguousarray(bias, dtype=np.float32)
+        key = np.empty((N, H), np.float64)
+        _check(lib.oracle_route_biased(_ptr(scores), _ptr(bias), N, H, K, _ptr(topk), _ptr(gate), _ptr(key)),
+               "route_biased")
+    n = np.empty((B, H), np.int32)
+    seg = np.empty(B * H + 1, np.int32)
+    rank = np.empty((N, K), np.int32)
+    row = np.empty((N, K), np.int32)
+    row_src = np.empty(N * K, np.int32)
+    _check(lib.oracle_dispatch_varlen(_ptr(topk), _ptr(cu), B, H, K, _ptr(n), _ptr(seg), _ptr(rank), _ptr(row),
+                                      _ptr(row_src)), "dispatch_varlen")
+    return dict(topk_head=topk, gate=gate, n=n, seg_offsets=seg, rank=rank, row=row, row_src=row_src)
+
+
 def route_biased(scores: np.ndarray, K: int, bias: np.ndarray) -> dict:
     """Biased routing (App. A, Eq. namoh-biased-routing) and dispatch for scores [B, T, H].
 
@@ -172,6 +207,14 @@ def global_positions(row_src: np.ndarray, T: int, K: int) -> np.ndarray:
     (row_src[r] = (b*T + t)*K + slot)."""
     rs = np.asarray(row_src, dtype=np.int64)
     return np.ascontiguousarray((rs // K) % T, dtype=np.int64)
+
+
+def global_positions_varlen(row_src: np.ndarray, cu_seqlens: np.ndarray, K: int) -> np.ndarray:
+    """Global RoPE positions in a ragged batch: the token's index inside its own sequence."""
+    tok = np.asarray(row_src, dtype=np.int64) // K
+    cu = np.asarray(cu_seqlens, dtype=np.int64)
+    b = np.searchsorted(cu, tok, side="right") - 1
+    return np.ascontiguousarray(tok - cu[b], dtype=np.int64)
 
 
 def prefill(q: np.ndarray, k: np.ndarray, v: np.ndarray, seg_offsets: np.ndarray, row_src: np.ndarray,

@@ -244,6 +244,50 @@ int oracle_dispatch(const int32_t *topk_head, int B, int T, int H, int K,
     return ORACLE_OK;
 }
 
+/*
+ * oracle_dispatch_varlen: the same append over a ragged batch.  Sequence b holds
+ * the tokens cu_seqlens[b] .. cu_seqlens[b+1]-1 of the flat token axis (N tokens in
+ * all); each sequence has its own index sets and ranks (Sec. 3.1, Sec. 3.2).
+ *   topk_head   [N, K]
+ *   n           [B*H], seg_offsets [B*H + 1] as oracle_dispatch
+ *   rank, row   [N, K]
+ *   row_src     [N*K]      inverse map: row_src[row] = tok*K + k (tok on the flat axis)
+ * cu_seqlens must start at 0, not decrease, and end at N.
+ */
+int oracle_dispatch_varlen(const int32_t *topk_head, const int32_t *cu_seqlens, int B, int H, int K,
+                           int32_t *n, int32_t *seg_offsets, int32_t *rank, int32_t *row, int32_t *row_src)
+{
+    if (!topk_head || !cu_seqlens || !n || !seg_offsets || !rank || !row || !row_src) return ORACLE_ERR_ARG;
+    if (B < 0 || H < 1 || K < 1 || K > H || cu_seqlens[0] != 0) return ORACLE_ERR_ARG;
+    for (int b = 0; b < B; ++b)
+        if (cu_seqlens[b + 1] < cu_seqlens[b]) return ORACLE_ERR_ARG;
+    for (long i = 0; i < (long)B * H; ++i) n[i] = 0;
+    for (int b = 0; b < B; ++b) {
+        for (long tok = cu_seqlens[b]; tok < cu_seqlens[b + 1]; ++tok) {
+            for (int k = 0; k < K; ++k) {
+                long idx = tok * K + k;
+                int h = topk_head[idx];
+                if (h < 0 || h >= H) return ORACLE_ERR_ARG;
+                rank[idx] = n[(long)b * H + h];
+                n[(long)b * H + h] += 1;
+            }
+        }
+    }
+    seg_offsets[0] = 0;
+    for (long i = 0; i < (long)B * H; ++i) seg_offsets[i + 1] = seg_offsets[i] + n[i];
+    for (int b = 0; b < B; ++b) {
+        for (long tok = cu_seqlens[b]; tok < cu_seqlens[b + 1]; ++tok) {
+            for (int k = 0; k < K; ++k) {
+                long idx = tok * K + k;
+                int r = seg_offsets[(long)b * H + topk_head[idx]] + rank[idx];
+                row[idx] = r;
+                row_src[r] = (int32_t)idx;
+            }
+        }
+    }
+    return ORACLE_OK;
+}
+
 /* ------------------------------------------------------------------------- */
 /* RoPE (Sec. 3.2, Eq. namoh-head-rope)                                       */
 /* ------------------------------------------------------------------------- */

@@ -319,3 +319,37 @@ def test_decode_capacity_overflow_is_an_error(oracle_mod):
     with pytest.raises(oracle_mod.OracleError):
         oracle_mod.decode_step(np.array([[0]]), np.array([[1.0]]), q, k, v, Hr, d, 1, 1e4, kc, vc, seg_base,
                                seg_len, cap)
+
+
+# --------------------------------------------------------------------------- ragged batches
+@pytest.mark.parametrize("global_pos", [False, True])
+def test_varlen_prefill_equals_each_sequence_alone(oracle_mod, global_pos):
+    """A ragged batch is independent sequences: prefill over the packed batch equals prefill
+    of every sequence on its own (no attention across sequences, positions per sequence)."""
+    lens, H, K, d, g, base = [37, 0, 130, 1, 64], 4, 2, 16, 2, 1e4
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    N = int(cu[-1])
+    s = ni.router_scores(13, 1, N, H)[0]
+    out = oracle_mod.route_varlen(s, cu, K)
+    q, k, v = ni.qkv_rows(13, N * K, d, g)
+    pos = oracle_mod.global_positions_varlen(out["row_src"], cu, K) if global_pos else None
+    y = oracle_mod.prefill(q, k, v, out["seg_offsets"], out["row_src"], out["gate"], d, g, base, pos=pos)
+    y = y.reshape(N, K, g, d)
+    qg = q.reshape(N * K, g, d)
+    for b, L in enumerate(lens):
+        if L == 0:
+            continue
+        one = oracle_mod.route(s[None, cu[b]:cu[b + 1]], K)
+        rows = out["row"][cu[b]:cu[b + 1]]  # this sequence's packed rows, in (t, slot) order
+        # the same rows, re-packed in the single-sequence layout
+        src = np.empty(L * K, np.int64)
+        src[one["row"].reshape(-1)] = rows.reshape(-1)
+        pos1 = oracle_mod.global_positions(one["row_src"], L, K) if global_pos else None
+        y1 = oracle_mod.prefill(qg[src].reshape(-1, d), k[src], v[src], one["seg_offsets"], one["row_src"],
+                                one["gate"], d, g, base, pos=pos1)
+        np.testing.assert_array_equal(y[cu[b]:cu[b + 1]], y1.reshape(L, K, g, d))
+    if global_pos:  # the position is the token's index in its own sequence
+        tok = out["row_src"] // K
+        for r in range(N * K):
+            b = int(np.nonzero(cu[1:] > tok[r])[0][0])
+            assert pos[r] == tok[r] - cu[b]

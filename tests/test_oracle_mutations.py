@@ -21,6 +21,8 @@ MUTATIONS = {
                                  "int i0 = interleaved ? 2 * j + 1 : j, i1 = interleaved ? 2 * j : j + half;"),
     "global_key_uses_rank": ("c->pos ? (double)c->pos[row] : (double)(row - off)",
                              "c->pos ? (double)(row - off) : (double)(row - off)"),
+    "varlen_segments_of_sequence_0": ("int r = seg_offsets[(long)b * H + topk_head[idx]] + rank[idx];",
+                                      "int r = seg_offsets[topk_head[idx]] + rank[idx];"),
     "decode_ignores_token_pos": ("const double p = token_pos ? (double)token_pos[b] : (double)rho;",
                                  "const double p = token_pos ? (double)rho : (double)rho;"),
     "no_scale": ("double scale = 1.0 / sqrt((double)d);", "double scale = 1.0;"),

@@ -233,3 +233,57 @@ def test_biased_ties_go_to_lower_index(oracle_mod):
     rb = oracle_mod.route_biased(s, 3, bias)
     np.testing.assert_array_equal(rb["topk_head"][0, 0], [1, 6, 0])
     np.testing.assert_array_equal(rb["topk_head"][0, 1], [1, 6, 2])
+
+
+# --------------------------------------------------------------------------- ragged batches
+def _ragged_scores(seed, lens, H):
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    s = ni.router_scores(seed, 1, int(cu[-1]), H)[0] if cu[-1] > 0 else np.zeros((0, H), np.float32)
+    return s, cu
+
+
+@pytest.mark.parametrize("lens,H,K", [([5, 0, 300, 1, 256, 257], 8, 2), ([40, 41], 16, 4), ([0], 4, 1), ([9], 3, 3)])
+def test_varlen_dispatch_matches_mask_cumsum(oracle_mod, lens, H, K):
+    """Sec. 3.1 / Eq. (namoh-head-rope) per sequence of a ragged batch: ranks restart at each
+    sequence's first token; n_{b,i} sums to len_b K (Eq. app-assignment-count)."""
+    s, cu = _ragged_scores(11, lens, H)
+    out = oracle_mod.route_varlen(s, cu, K)
+    B, N = len(lens), int(cu[-1])
+    top = out["topk_head"].astype(np.int64)
+    mask = np.zeros((N, H), np.int64)
+    if N:
+        np.put_along_axis(mask, top, 1, axis=-1)
+    seg = [0]
+    for b in range(B):
+        m = mask[cu[b]:cu[b + 1]]
+        rho = np.cumsum(m, axis=0) - 1
+        np.testing.assert_array_equal(out["rank"][cu[b]:cu[b + 1]], np.take_along_axis(rho, top[cu[b]:cu[b + 1]], -1))
+        np.testing.assert_array_equal(out["n"][b], m.sum(0))
+        assert m.sum() == lens[b] * K
+        seg += list(seg[-1] + np.cumsum(m.sum(0)))
+    np.testing.assert_array_equal(out["seg_offsets"], seg)
+    flat = out["row"].reshape(-1)
+    np.testing.assert_array_equal(out["row_src"][flat], np.arange(N * K))
+    tok = out["row_src"] // K
+    for sgi in range(B * H):
+        r = tok[seg[sgi]:seg[sgi + 1]]
+        b = sgi // H
+        assert np.all(np.diff(r) > 0) and np.all((r >= cu[b]) & (r < cu[b + 1]))
+
+
+def test_varlen_uniform_lengths_equal_fixed(oracle_mod):
+    B, T, H, K = 3, 70, 8, 3
+    s = ni.router_scores(12, B, T, H)
+    fixed = oracle_mod.route(s, K)
+    var = oracle_mod.route_varlen(s.reshape(B * T, H), np.arange(B + 1) * T, K)
+    for key in ("topk_head", "gate", "rank", "row"):
+        np.testing.assert_array_equal(var[key], fixed[key].reshape(B * T, K))
+    for key in ("n", "seg_offsets", "row_src"):
+        np.testing.assert_array_equal(var[key], fixed[key])
+
+
+def test_varlen_rejects_bad_cu_seqlens(oracle_mod):
+    s = np.zeros((10, 4), np.float32)
+    for cu in ([1, 10], [0, 6, 4, 10], [0, 9]):
+        with pytest.raises(oracle_mod.OracleError):
+            oracle_mod.route_varlen(s, np.array(cu), 2)
