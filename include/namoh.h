@@ -62,6 +62,7 @@ typedef enum namoh_status {
 #define NAMOH_DEV_TIMEOUT 0x4u         /* a pipeline wait exceeded its limit; bits 16-23 then
                                           hold the barrier's index in its kernel's barrier block
                                           and bits 24-31 the warp that gave up */
+#define NAMOH_DEV_BAD_SEQLENS 0x8u     /* cu_seqlens of a ragged batch was malformed */
 
 /* RoPE variants (the rope_flags argument of the *_ex entry points; 0 = the defaults).
  * NAMOH_ROPE_INTERLEAVED  rotate pairs (2j, 2j+1) instead of the half-split (j, j + d/2);
@@ -139,6 +140,30 @@ NAMOH_API int namoh_route_biased(const float *scores, const float *bias, int B, 
                                  void *stream);
 
 /* ------------------------------------------------------------------------- *
+ * namoh_route_varlen: routing of a ragged batch (sequences of different lengths
+ *   packed back to back, no padding).  Sequence b holds the tokens
+ *   cu_seqlens[b] .. cu_seqlens[b+1]-1 of the flat token axis; ranks, index sets
+ *   and segments are per sequence exactly as in namoh_route (Sec. 3.1, Sec. 3.2).
+ * scores      [total_tokens, H] fp32.
+ * cu_seqlens  [B + 1] int32 device array: 0 = cu_seqlens[0] <= ... <=
+ *             cu_seqlens[B] = total_tokens, every length <= max_seqlen (empty
+ *             sequences are allowed).  A violation found on the device sets
+ *             NAMOH_DEV_BAD_SEQLENS; the outputs are then unspecified but stay a
+ *             layout of rows below total_tokens*K, so later stages stay in bounds.
+ * bias        [H] or NULL: as namoh_route_biased.
+ * topk_head, gate, rank, row [total_tokens, K]; seg_offsets [B*H + 1] with
+ *             seg_offsets[B*H] = total_tokens*K; row_src [total_tokens*K] with
+ *             row_src[row] = tok*K + slot, tok on the flat axis.  The packed layout
+ *             is optional as in namoh_route (without it cu_seqlens is not read).
+ * Workspace: namoh_route_workspace_size(B, max_seqlen, H, K).
+ * Requires 1 <= max_seqlen <= total_tokens, total_tokens*K < 2^31.
+ * ------------------------------------------------------------------------- */
+NAMOH_API int namoh_route_varlen(const float *scores, const float *bias, const int32_t *cu_seqlens, int B,
+                                 int total_tokens, int max_seqlen, int H, int K, int32_t *topk_head, float *gate,
+                                 int32_t *rank, int32_t *row, int32_t *seg_offsets, int32_t *row_src,
+                                 void *workspace, size_t workspace_bytes, uint32_t *dev_status, void *stream);
+
+/* ------------------------------------------------------------------------- *
  * namoh_route_noalloc: namoh_route without a workspace argument.
  * The paper has no counterpart; this is a convenience of this library.
  *
@@ -208,6 +233,24 @@ NAMOH_API int namoh_prefill_ex(const uint16_t *q, const uint16_t *k, const uint1
                                uint16_t *k_cache, uint16_t *v_cache, const int64_t *seg_base,
                                const int32_t *seg_cap, int64_t cache_rows, int32_t *seg_len, void *workspace,
                                size_t workspace_bytes, uint32_t *dev_status, void *stream);
+
+/* namoh_prefill_varlen: namoh_prefill_ex over a ragged batch routed by
+ * namoh_route_varlen.  total_tokens and max_seqlen are the host's copies of
+ * cu_seqlens[B] and the longest length; R = total_tokens * Kr; y is
+ * [total_tokens, K, d].  cu_seqlens ([B + 1], device) is read only for
+ * NAMOH_ROPE_GLOBAL, where the position of a row is its token's index inside its
+ * own sequence.  Workspace: namoh_prefill_varlen_workspace_size.  Requires
+ * 1 <= max_seqlen <= min(total_tokens, 2^20).  The staged calls below are for
+ * fixed-length batches only. */
+NAMOH_API size_t namoh_prefill_varlen_workspace_size(int B, int total_tokens, int max_seqlen, int H, int K,
+                                                     int d_head, int group);
+NAMOH_API int namoh_prefill_varlen(const uint16_t *q, const uint16_t *k, const uint16_t *v, const int32_t *cu_seqlens,
+                                   int B, int total_tokens, int max_seqlen, int H, int K, int d_head, int group,
+                                   float rope_base, unsigned rope_flags, const int32_t *seg_offsets,
+                                   const int32_t *row_src, const float *gate, uint16_t *y, uint16_t *k_cache,
+                                   uint16_t *v_cache, const int64_t *seg_base, const int32_t *seg_cap,
+                                   int64_t cache_rows, int32_t *seg_len, void *workspace, size_t workspace_bytes,
+                                   uint32_t *dev_status, void *stream);
 
 /* ------------------------------------------------------------------------- *
  * The three stages of namoh_prefill, callable one by one (same arguments and

@@ -209,6 +209,25 @@ def global_positions(row_src: np.ndarray, T: int, K: int) -> np.ndarray:
     return np.ascontiguousarray((rs // K) % T, dtype=np.int64)
 
 
+def dispatch_varlen(topk_head: np.ndarray, cu_seqlens: np.ndarray, H: int) -> dict:
+    """Dispatch of given picks topk_head [N, K] over a ragged batch (oracle_dispatch_varlen)."""
+    lib = _load()
+    topk = np.ascontiguousarray(topk_head, dtype=np.int32)
+    cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
+    N, K = topk.shape
+    B = len(cu) - 1
+    if cu[0] != 0 or cu[-1] != N or np.any(np.diff(cu) < 0):
+        raise OracleError("cu_seqlens must start at 0, not decrease and end at N")
+    n = np.empty((B, H), np.int32)
+    seg = np.empty(B * H + 1, np.int32)
+    rank = np.empty((N, K), np.int32)
+    row = np.empty((N, K), np.int32)
+    row_src = np.empty(N * K, np.int32)
+    _check(lib.oracle_dispatch_varlen(_ptr(topk), _ptr(cu), B, H, K, _ptr(n), _ptr(seg), _ptr(rank), _ptr(row),
+                                      _ptr(row_src)), "dispatch_varlen")
+    return dict(n=n, seg_offsets=seg, rank=rank, row=row, row_src=row_src)
+
+
 def global_positions_varlen(row_src: np.ndarray, cu_seqlens: np.ndarray, K: int) -> np.ndarray:
     """Global RoPE positions in a ragged batch: the token's index inside its own sequence."""
     tok = np.asarray(row_src, dtype=np.int64) // K

@@ -14,11 +14,13 @@ from typing import Optional
 import torch
 
 from . import _abi
-from ._abi import (NAMOH_DEV_CAPACITY, NAMOH_DEV_NONFINITE_SCORE, NAMOH_DEV_TIMEOUT, NamohError)
+from ._abi import (NAMOH_DEV_BAD_SEQLENS, NAMOH_DEV_CAPACITY, NAMOH_DEV_NONFINITE_SCORE, NAMOH_DEV_TIMEOUT,
+                   NAMOH_ROPE_GLOBAL, NAMOH_ROPE_INTERLEAVED, NamohError)
 
-__all__ = ["namoh_route", "namoh_prefill", "namoh_decode", "namoh_rope_pack", "namoh_attention_plan",
-           "namoh_attention", "RouteOutputs", "Workspace", "NamohError",
-           "NAMOH_DEV_CAPACITY", "NAMOH_DEV_NONFINITE_SCORE", "NAMOH_DEV_TIMEOUT", "library_path"]
+__all__ = ["namoh_route", "namoh_route_varlen", "namoh_prefill", "namoh_prefill_varlen", "namoh_decode",
+           "namoh_rope_pack", "namoh_attention_plan", "namoh_attention", "RouteOutputs", "Workspace", "NamohError",
+           "NAMOH_DEV_BAD_SEQLENS", "NAMOH_DEV_CAPACITY", "NAMOH_DEV_NONFINITE_SCORE", "NAMOH_DEV_TIMEOUT",
+           "NAMOH_ROPE_GLOBAL", "NAMOH_ROPE_INTERLEAVED", "library_path"]
 
 
 def library_path() -> str:
@@ -110,6 +112,43 @@ def namoh_route(scores: torch.Tensor, K: int, compact: bool = True, workspace: O
     return out
 
 
+def namoh_route_varlen(scores: torch.Tensor, cu_seqlens: torch.Tensor, max_seqlen: int, K: int,
+                       compact: bool = True, workspace: Optional[Workspace] = None,
+                       status: Optional[torch.Tensor] = None, out: Optional[RouteOutputs] = None, stream=None,
+                       bias: Optional[torch.Tensor] = None) -> RouteOutputs:
+    """Routing of a ragged batch (see namoh_route_varlen in include/namoh.h): scores [N, H] fp32
+    over the flat token axis, cu_seqlens [B + 1] int32 on the device, max_seqlen the longest
+    sequence.  Per-token outputs are [N, K]; row_src[row] = tok*K + slot."""
+    lib = _abi.load()
+    if scores.dtype != torch.float32 or scores.dim() != 2:
+        raise ValueError("scores must be a [N, H] float32 tensor")
+    if cu_seqlens.dtype != torch.int32 or cu_seqlens.dim() != 1 or cu_seqlens.device != scores.device:
+        raise ValueError("cu_seqlens must be a 1-D int32 tensor on the scores' device")
+    N, H = scores.shape
+    B = cu_seqlens.numel() - 1
+    dev = scores.device
+    if bias is not None and (bias.dtype != torch.float32 or bias.shape != (H,) or bias.device != dev
+                             or not bias.is_contiguous()):
+        raise ValueError("bias must be a contiguous [H] float32 tensor on the scores' device")
+    if out is None:
+        i32 = dict(dtype=torch.int32, device=dev)
+        out = RouteOutputs(
+            topk_head=torch.empty((N, K), **i32), gate=torch.empty((N, K), dtype=torch.float32, device=dev),
+            rank=torch.empty((N, K), **i32) if compact else None,
+            row=torch.empty((N, K), **i32) if compact else None,
+            seg_offsets=torch.empty(B * H + 1, **i32) if compact else None,
+            row_src=torch.empty(N * K, **i32) if compact else None,
+            status=_status(status, dev))
+    nbytes = lib.namoh_route_workspace_size(B, max_seqlen, H, K)
+    ws = _ws(workspace, nbytes, dev)
+    rc = lib.namoh_route_varlen(_ptr(scores), _ptr(bias), _ptr(cu_seqlens), B, N, int(max_seqlen), H, K,
+                                _ptr(out.topk_head), _ptr(out.gate), _ptr(out.rank), _ptr(out.row),
+                                _ptr(out.seg_offsets), _ptr(out.row_src), _ptr(ws), ws.numel(), _ptr(out.status),
+                                _stream(stream))
+    _abi.check("namoh_route_varlen", rc)
+    return out
+
+
 def _rope_flags(interleaved: bool, global_positions: bool) -> int:
     return (_abi.NAMOH_ROPE_INTERLEAVED if interleaved else 0) | (_abi.NAMOH_ROPE_GLOBAL if global_positions else 0)
 
@@ -151,6 +190,45 @@ def namoh_prefill(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, seg_offsets
                               _ptr(gate), _ptr(y), _ptr(k_cache), _ptr(v_cache), _ptr(seg_base), _ptr(seg_cap),
                               cache_rows, _ptr(seg_len), _ptr(ws), ws.numel(), _ptr(st), _stream(stream))
     _abi.check("namoh_prefill_ex", rc)
+    return y, k_cache, v_cache
+
+
+def namoh_prefill_varlen(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, cu_seqlens: torch.Tensor,
+                         max_seqlen: int, seg_offsets: torch.Tensor, row_src: torch.Tensor, gate: torch.Tensor, *,
+                         H: int, K: int, group: int = 1, rope_base: float = 10000.0, interleaved: bool = False,
+                         global_positions: bool = False, y: Optional[torch.Tensor] = None,
+                         k_cache: Optional[torch.Tensor] = None, v_cache: Optional[torch.Tensor] = None,
+                         seg_base: Optional[torch.Tensor] = None, seg_cap: Optional[torch.Tensor] = None,
+                         seg_len: Optional[torch.Tensor] = None, workspace: Optional[Workspace] = None,
+                         status: Optional[torch.Tensor] = None, stream=None):
+    """Prefill over a ragged batch routed by namoh_route_varlen (see namoh_prefill_varlen in
+    include/namoh.h).  q [N*Kr*g, d], k / v [N*Kr, d] bf16 packed rows; returns
+    (y [N, K, d], k_cache, v_cache) with N = gate.shape[0] tokens."""
+    lib = _abi.load()
+    d = q.shape[-1]
+    dev = q.device
+    for name, t in (("q", q), ("k", k), ("v", v)):
+        if t.dtype != torch.bfloat16:
+            raise ValueError(f"{name} must be bfloat16")
+    B = cu_seqlens.numel() - 1
+    N = gate.shape[0]
+    if y is None:
+        y = torch.empty((N, K, d), dtype=torch.bfloat16, device=dev)
+    if k_cache is None:
+        k_cache = torch.empty_like(k)
+    if v_cache is None:
+        v_cache = v if seg_base is None else torch.empty_like(v)
+    nbytes = lib.namoh_prefill_varlen_workspace_size(B, N, int(max_seqlen), H, K, d, group)
+    if nbytes == 0:
+        raise NamohError("namoh_prefill_varlen_workspace_size", _abi.NAMOH_ERR_UNSUPPORTED)
+    ws = _ws(workspace, nbytes, dev)
+    st = _status(status, dev)
+    rc = lib.namoh_prefill_varlen(_ptr(q), _ptr(k), _ptr(v), _ptr(cu_seqlens), B, N, int(max_seqlen), H, K, d, group,
+                                  float(rope_base), _rope_flags(interleaved, global_positions), _ptr(seg_offsets),
+                                  _ptr(row_src), _ptr(gate), _ptr(y), _ptr(k_cache), _ptr(v_cache), _ptr(seg_base),
+                                  _ptr(seg_cap), k_cache.shape[0], _ptr(seg_len), _ptr(ws), ws.numel(), _ptr(st),
+                                  _stream(stream))
+    _abi.check("namoh_prefill_varlen", rc)
     return y, k_cache, v_cache
 
 

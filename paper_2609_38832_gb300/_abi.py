@@ -19,6 +19,7 @@ NAMOH_ERR_CUDA = -4
 NAMOH_DEV_NONFINITE_SCORE = 0x1
 NAMOH_DEV_CAPACITY = 0x2
 NAMOH_DEV_TIMEOUT = 0x4
+NAMOH_DEV_BAD_SEQLENS = 0x8
 
 NAMOH_ROPE_INTERLEAVED = 0x1
 NAMOH_ROPE_GLOBAL = 0x2
@@ -40,6 +41,7 @@ SIGNATURES = {
     "namoh_route_workspace_size": (_SZ, [_I, _I, _I, _I]),
     "namoh_route": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P]),
     "namoh_route_biased": (_I, [_P, _P, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P]),
+    "namoh_route_varlen": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P]),
     "namoh_route_noalloc": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P]),
     "namoh_prefill_workspace_size": (_SZ, [_I, _I, _I, _I, _I, _I]),
     "namoh_prefill": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _P, _P, _P, _I64, _P, _P,
@@ -48,6 +50,9 @@ SIGNATURES = {
                              _P]),
     "namoh_prefill_ex": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _U, _P, _P, _P, _P, _P, _P, _P, _P, _I64,
                               _P, _P, _SZ, _P, _P]),
+    "namoh_prefill_varlen_workspace_size": (_SZ, [_I, _I, _I, _I, _I, _I, _I]),
+    "namoh_prefill_varlen": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _F, _U, _P, _P, _P, _P, _P, _P, _P,
+                                  _P, _I64, _P, _P, _SZ, _P, _P]),
     "namoh_rope_pack_ex": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _U, _P, _P, _P, _P, _P, _P, _P, _I64, _P,
                                 _P, _SZ, _P]),
     "namoh_attention_plan_size": (_SZ, [_I, _I, _I, _I, _I]),

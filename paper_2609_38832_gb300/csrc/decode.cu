@@ -52,7 +52,7 @@ __global__ void decode_append_kernel(const int32_t* __restrict__ topk_head, cons
   const int s = b * Hr + h;
   const int rho = seg_len[s];
   const long long base = seg_base[s];
-  const bool room = rho < seg_cap[s] && base + rho < cache_rows && base >= 0;
+  const bool room = rho >= 0 && rho < seg_cap[s] && base + rho < cache_rows && base >= 0;
   if (lane == 0) {
     PairInfo pi;
     pi.base = base;

@@ -31,7 +31,7 @@ __device__ inline void build_plan(const int32_t* __restrict__ seg_offsets, int n
   for (int s = tid; s < nseg; s += blockDim.x) {
     const int n = __ldg(seg_offsets + s + 1) - __ldg(seg_offsets + s);
     const bool skip = seg_cap && n > __ldg(seg_cap + s);
-    s_ntile[s] = skip ? 0 : min((n + kPlanTileRows - 1) / kPlanTileRows, max_qtiles);
+    s_ntile[s] = skip || n <= 0 ? 0 : min((n + kPlanTileRows - 1) / kPlanTileRows, max_qtiles);
   }
   __syncthreads();
   for (int s = tid; s < nseg; s += blockDim.x)

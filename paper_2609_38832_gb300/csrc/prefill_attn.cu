@@ -42,7 +42,7 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache, bool copy_v,
                              const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream,
                              void* plan, int plan_qtiles, const int32_t* plan_cap, const int32_t* pos_row_src,
-                             int pos_k, int pos_t, bool interleaved);
+                             int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved);
 
 namespace attn {
 
@@ -106,6 +106,7 @@ struct Params {
   const int* nitems;
   int* sched;                  // [0] next item, [1] CTAs finished
   uint16_t* y;                 // [R * g, D] indexed by row_src * g + j
+  int rows;                    // R: a row_src value at or above it is skipped (inconsistent layout)
   int g;
   int y_sector_aligned;        // y is 32-byte aligned: rows go out as whole 32-byte sectors
   float scale_log2;            // log2(e) / sqrt(D)
@@ -531,7 +532,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!ok) break;
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars->p_full[tile & 1]);
-        if (kv == 0 && valid) gt = ld_issue_f32(p.gate + src);  // used in the epilogue only
+        if (kv == 0 && valid) {  // the gate, used in the epilogue only
+          if ((unsigned)src < (unsigned)p.rows) gt = ld_issue_f32(p.gate + src);
+          else src = -1;
+        }
       }
       if (!ok) break;
       // epilogue: O out of TMEM (O is then free for the next item), O / l * gate as bf16
@@ -546,7 +550,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars->o_free);
-      if (valid) {
+      if (valid && src >= 0) {
         const float scale = gt / l_sum;
         uint32_t w[D / 2];
 #pragma unroll
@@ -617,7 +621,7 @@ cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUte
 namespace {
 __global__ void seg_len_kernel(const int32_t* __restrict__ seg_offsets, int nseg, int32_t* __restrict__ seg_len) {
   const int s = blockIdx.x * blockDim.x + threadIdx.x;
-  if (s < nseg) seg_len[s] = seg_offsets[s + 1] - seg_offsets[s];
+  if (s < nseg) seg_len[s] = max(seg_offsets[s + 1] - seg_offsets[s], 0);
 }
 
 constexpr int kMaxPrefillT = 1 << 20;  // the plan keeps 2 ints per query tile in shared memory
@@ -628,24 +632,32 @@ bool supported_dims(int d_head, int g) {
 }
 
 // Shape checks shared by the prefill stages.  Fills Hr, Kr, R on success.
-int check_shape(int B, int T, int H, int K, int d_head, int group, int* Hr, int* Kr, long long* R) {
+// Shapes of B sequences of at most T tokens holding `tokens` tokens in all (B*T, or the
+// total of a ragged batch): R = tokens * Kr packed rows.
+int check_dims(int B, int T, long long tokens, int H, int K, int d_head, int group, int* Hr, int* Kr, long long* R) {
   if (B < 1 || T < 1 || group < 1 || H < 1 || K < 1 || K > H || H % group || K % group) return NAMOH_ERR_INVALID_ARG;
   if (H / group > NAMOH_MAX_HEADS) return NAMOH_ERR_INVALID_ARG;
   if (d_head >= 0 && !supported_dims(d_head, group)) return NAMOH_ERR_UNSUPPORTED;
   if (T > kMaxPrefillT) return NAMOH_ERR_UNSUPPORTED;
   *Hr = H / group;
   *Kr = K / group;
-  *R = (long long)B * T * *Kr;
+  *R = tokens * *Kr;
   if (*R * group >= (1ll << 31)) return NAMOH_ERR_INVALID_ARG;
   if ((long long)B * *Hr > kMaxPrefillSegments) return NAMOH_ERR_UNSUPPORTED;
   return NAMOH_OK;
 }
 
-size_t plan_bytes_for(int B, int T, int Hr, int Kr, int g) {
-  const long long R = (long long)B * T * Kr;
-  const long long max_items = ((R + attn::kItemRows - 1) / attn::kItemRows + (long long)B * Hr) * g;
+int check_shape(int B, int T, int H, int K, int d_head, int group, int* Hr, int* Kr, long long* R) {
+  return check_dims(B, T, (long long)B * T, H, K, d_head, group, Hr, Kr, R);
+}
+
+// plan bytes for R packed rows in nseg segments: at most ceil(R/128) + nseg query tiles, g items each
+size_t plan_bytes_rows(long long R, int nseg, int g) {
+  const long long max_items = ((R + attn::kItemRows - 1) / attn::kItemRows + nseg) * g;
   return 16 + (size_t)max_items * sizeof(int4);
 }
+
+size_t plan_bytes_for(int B, int T, int Hr, int Kr, int g) { return plan_bytes_rows((long long)B * T * Kr, B * Hr, g); }
 
 int plan_qtiles_for(int T) { return (T + kPlanTileRows - 1) / kPlanTileRows; }  // query tiles per segment, at most
 
@@ -670,12 +682,13 @@ int launch_plan(const int32_t* seg_offsets, int nseg, int T, int g, const int32_
 
 // RoPE + cache pack; with a plan buffer also the attention plan (in the same launch when
 // the plan's shared memory is small, else as a second kernel).
-// rope_flags: NAMOH_ROPE_GLOBAL takes the positions from row_src (t = (row_src[r] / Kr) % T).
+// rope_flags: NAMOH_ROPE_GLOBAL takes the positions from row_src: t = (row_src[r] / Kr) % T,
+// or row_src[r] / Kr - cu_seqlens[b] in a ragged batch (T is then the longest sequence).
 int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int Hr, int Kr, int R,
-                         int d_head, int group, float rope_base, unsigned rope_flags, const int32_t* seg_offsets,
-                         const int32_t* row_src, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache,
-                         const int64_t* seg_base, const int32_t* seg_cap, long long cache_rows, uint32_t* dev_status,
-                         void* plan, const DeviceInfo& info, cudaStream_t stream) {
+                         int d_head, int group, float rope_base, unsigned rope_flags, const int32_t* cu_seqlens,
+                         const int32_t* seg_offsets, const int32_t* row_src, uint16_t* q_rot, uint16_t* k_cache,
+                         uint16_t* v_cache, const int64_t* seg_base, const int32_t* seg_cap, long long cache_rows,
+                         uint32_t* dev_status, void* plan, const DeviceInfo& info, cudaStream_t stream) {
   RopeTable tab;
   fill_rope_table(&tab, d_head, (double)rope_base);
   const int nseg = B * Hr;
@@ -685,18 +698,17 @@ int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v
   const cudaError_t e = launch_rope_pack(d_head, q, k, v, R, group, seg_offsets, nseg, seg_base, seg_cap, cache_rows,
                                          q_rot, k_cache, v_cache, v_cache != v, tab, dev_status, info.sm_count, stream,
                                          fuse_plan ? plan : nullptr, qtiles, plan_cap,
-                                         (rope_flags & NAMOH_ROPE_GLOBAL) ? row_src : nullptr, Kr, T,
-                                         (rope_flags & NAMOH_ROPE_INTERLEAVED) != 0);
+                                         (rope_flags & NAMOH_ROPE_GLOBAL) ? row_src : nullptr, Kr, T, cu_seqlens,
+                                         Hr, (rope_flags & NAMOH_ROPE_INTERLEAVED) != 0);
   if (e != cudaSuccess) return cuda_fail(e, "rope_pack_kernel launch");
   if (plan && !fuse_plan) return launch_plan(seg_offsets, nseg, T, group, plan_cap, plan, stream);
   return NAMOH_OK;
 }
 
-int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint16_t* v_cache, int B, int T, int Hr,
-                     int Kr, int D, int g, const int32_t* seg_offsets, const int32_t* row_src, const float* gate,
+int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint16_t* v_cache, long long R, int D,
+                     int g, const int32_t* seg_offsets, const int32_t* row_src, const float* gate,
                      const int64_t* seg_base, long long cache_rows, void* plan, uint16_t* y, uint32_t* dev_status,
                      const DeviceInfo& info, cudaStream_t stream) {
-  const long long R = (long long)B * T * Kr;
   CUtensorMap tq, tk, tv;
   if (!attn::encode_rows_map(&tq, q_rot, R, g * D) || !attn::encode_rows_map(&tk, k_cache, cache_rows, D) ||
       !attn::encode_rows_map(&tv, v_cache, cache_rows, D))
@@ -710,6 +722,7 @@ int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint1
   p.nitems = static_cast<int*>(plan) + 2;
   p.items = reinterpret_cast<const int4*>(static_cast<char*>(plan) + 16);
   p.y = y;
+  p.rows = (int)R;
   p.g = g;
   p.y_sector_aligned = (reinterpret_cast<uintptr_t>(y) & 31u) == 0;
   p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)D));
@@ -755,9 +768,9 @@ extern "C" int namoh_rope_pack_ex(const uint16_t* q, const uint16_t* k, const ui
     return NAMOH_ERR_WORKSPACE;
   DeviceInfo info;
   if (!current_device_info(&info)) return cuda_fail(cudaGetLastError(), "device query");
-  return launch_rope_and_plan(q, k, v, B, T, Hr, Kr, (int)R, d_head, group, rope_base, rope_flags, seg_offsets,
-                              row_src, q_rot, k_cache, v_cache, seg_base, seg_cap, cache_rows, dev_status, plan, info,
-                              reinterpret_cast<cudaStream_t>(stream_v));
+  return launch_rope_and_plan(q, k, v, B, T, Hr, Kr, (int)R, d_head, group, rope_base, rope_flags, nullptr,
+                              seg_offsets, row_src, q_rot, k_cache, v_cache, seg_base, seg_cap, cache_rows, dev_status,
+                              plan, info, reinterpret_cast<cudaStream_t>(stream_v));
 }
 
 extern "C" int namoh_rope_pack(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int H, int K,
@@ -808,32 +821,21 @@ extern "C" int namoh_attention(const uint16_t* q_rot, const uint16_t* k_cache, c
     return NAMOH_ERR_WORKSPACE;
   DeviceInfo info;
   if (!device_ok(&info)) return NAMOH_ERR_UNSUPPORTED;
-  return launch_attention(q_rot, k_cache, v_cache, B, T, Hr, Kr, d_head, group, seg_offsets, row_src, gate, seg_base,
-                          cache_rows, plan, y, dev_status, info, reinterpret_cast<cudaStream_t>(stream_v));
+  return launch_attention(q_rot, k_cache, v_cache, R, d_head, group, seg_offsets, row_src, gate, seg_base, cache_rows,
+                          plan, y, dev_status, info, reinterpret_cast<cudaStream_t>(stream_v));
 }
 
-extern "C" size_t namoh_prefill_workspace_size(int B, int T, int H, int K, int d_head, int group) {
-  int Hr, Kr;
-  long long R;
-  if (check_shape(B, T, H, K, d_head, group, &Hr, &Kr, &R) != NAMOH_OK) return 0;
-  WorkspaceCarver ws{nullptr, 0, 0};
-  ws.take<uint16_t>((size_t)R * group * d_head);
-  ws.take<char>(plan_bytes_for(B, T, Hr, Kr, group));
-  return align_up(ws.used, 256);
-}
-
-extern "C" int namoh_prefill_ex(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int H, int K,
-                                int d_head, int group, float rope_base, unsigned rope_flags,
-                                const int32_t* seg_offsets, const int32_t* row_src, const float* gate, uint16_t* y,
-                                uint16_t* k_cache, uint16_t* v_cache, const int64_t* seg_base,
-                                const int32_t* seg_cap, int64_t cache_rows, int32_t* seg_len, void* workspace,
-                                size_t workspace_bytes, uint32_t* dev_status, void* stream_v) {
+namespace namoh {
+namespace {
+// Shared body of namoh_prefill_ex and namoh_prefill_varlen: R packed rows in B*Hr segments
+// of at most T rows; cu_seqlens (ragged batch) only enters the global RoPE positions.
+int prefill_impl(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int Hr, int Kr, long long R,
+                 int d_head, int group, float rope_base, unsigned rope_flags, const int32_t* cu_seqlens,
+                 const int32_t* seg_offsets, const int32_t* row_src, const float* gate, uint16_t* y, uint16_t* k_cache,
+                 uint16_t* v_cache, const int64_t* seg_base, const int32_t* seg_cap, int64_t cache_rows,
+                 int32_t* seg_len, void* workspace, size_t workspace_bytes, uint32_t* dev_status, void* stream_v) {
   if (!q || !k || !v || !seg_offsets || !row_src || !gate || !y || !k_cache || !v_cache || !dev_status)
     return NAMOH_ERR_INVALID_ARG;
-  int Hr, Kr;
-  long long R;
-  int st = check_shape(B, T, H, K, d_head, group, &Hr, &Kr, &R);
-  if (st != NAMOH_OK) return st;
   if (!(rope_base > 1.0f) || !isfinite(rope_base)) return NAMOH_ERR_INVALID_ARG;
   if (!rope_flags_ok(rope_flags)) return NAMOH_ERR_INVALID_ARG;
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(y) || !aligned16(k_cache) || !aligned16(v_cache))
@@ -847,22 +849,85 @@ extern "C" int namoh_prefill_ex(const uint16_t* q, const uint16_t* k, const uint
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return NAMOH_ERR_WORKSPACE;
   WorkspaceCarver ws{static_cast<char*>(workspace), workspace_bytes, 0};
   uint16_t* q_rot = ws.take<uint16_t>((size_t)R * group * d_head);
-  const size_t pbytes = plan_bytes_for(B, T, Hr, Kr, group);
-  void* plan = ws.take<char>(pbytes);
+  void* plan = ws.take<char>(plan_bytes_rows(R, B * Hr, group));
   if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
   DeviceInfo info;
   if (!device_ok(&info)) return NAMOH_ERR_UNSUPPORTED;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
 
-  st = launch_rope_and_plan(q, k, v, B, T, Hr, Kr, (int)R, d_head, group, rope_base, rope_flags, seg_offsets, row_src,
-                            q_rot, k_cache, v_cache, seg_base, seg_cap, cache_rows, dev_status, plan, info, stream);
+  int st = launch_rope_and_plan(q, k, v, B, T, Hr, Kr, (int)R, d_head, group, rope_base, rope_flags, cu_seqlens,
+                                seg_offsets, row_src, q_rot, k_cache, v_cache, seg_base, seg_cap, cache_rows,
+                                dev_status, plan, info, stream);
   if (st != NAMOH_OK) return st;
   if (seg_len) {
     seg_len_kernel<<<(B * Hr + 255) / 256, 256, 0, stream>>>(seg_offsets, B * Hr, seg_len);
     if (const int st2 = cuda_check_launch("seg_len_kernel launch")) return st2;
   }
-  return launch_attention(q_rot, k_cache, v_cache, B, T, Hr, Kr, d_head, group, seg_offsets, row_src, gate, seg_base,
-                          cache_rows, plan, y, dev_status, info, stream);
+  return launch_attention(q_rot, k_cache, v_cache, R, d_head, group, seg_offsets, row_src, gate, seg_base, cache_rows,
+                          plan, y, dev_status, info, stream);
+}
+
+size_t prefill_workspace_rows(long long R, int nseg, int d_head, int group) {
+  WorkspaceCarver ws{nullptr, 0, 0};
+  ws.take<uint16_t>((size_t)R * group * d_head);
+  ws.take<char>(plan_bytes_rows(R, nseg, group));
+  return align_up(ws.used, 256);
+}
+
+// shapes of a ragged batch: T = max_seqlen <= total_tokens, R = total_tokens * Kr
+int check_varlen(int B, int total_tokens, int max_seqlen, int H, int K, int d_head, int group, int* Hr, int* Kr,
+                 long long* R) {
+  if (max_seqlen < 1 || total_tokens < max_seqlen) return NAMOH_ERR_INVALID_ARG;
+  return check_dims(B, max_seqlen, total_tokens, H, K, d_head, group, Hr, Kr, R);
+}
+}  // namespace
+}  // namespace namoh
+
+extern "C" size_t namoh_prefill_workspace_size(int B, int T, int H, int K, int d_head, int group) {
+  int Hr, Kr;
+  long long R;
+  if (check_shape(B, T, H, K, d_head, group, &Hr, &Kr, &R) != NAMOH_OK) return 0;
+  return prefill_workspace_rows(R, B * Hr, d_head, group);
+}
+
+extern "C" int namoh_prefill_ex(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int H, int K,
+                                int d_head, int group, float rope_base, unsigned rope_flags,
+                                const int32_t* seg_offsets, const int32_t* row_src, const float* gate, uint16_t* y,
+                                uint16_t* k_cache, uint16_t* v_cache, const int64_t* seg_base,
+                                const int32_t* seg_cap, int64_t cache_rows, int32_t* seg_len, void* workspace,
+                                size_t workspace_bytes, uint32_t* dev_status, void* stream_v) {
+  int Hr, Kr;
+  long long R;
+  const int st = check_shape(B, T, H, K, d_head, group, &Hr, &Kr, &R);
+  if (st != NAMOH_OK) return st;
+  return prefill_impl(q, k, v, B, T, Hr, Kr, R, d_head, group, rope_base, rope_flags, nullptr, seg_offsets, row_src,
+                      gate, y, k_cache, v_cache, seg_base, seg_cap, cache_rows, seg_len, workspace, workspace_bytes,
+                      dev_status, stream_v);
+}
+
+extern "C" size_t namoh_prefill_varlen_workspace_size(int B, int total_tokens, int max_seqlen, int H, int K,
+                                                      int d_head, int group) {
+  int Hr, Kr;
+  long long R;
+  if (check_varlen(B, total_tokens, max_seqlen, H, K, d_head, group, &Hr, &Kr, &R) != NAMOH_OK) return 0;
+  return prefill_workspace_rows(R, B * Hr, d_head, group);
+}
+
+extern "C" int namoh_prefill_varlen(const uint16_t* q, const uint16_t* k, const uint16_t* v,
+                                    const int32_t* cu_seqlens, int B, int total_tokens, int max_seqlen, int H, int K,
+                                    int d_head, int group, float rope_base, unsigned rope_flags,
+                                    const int32_t* seg_offsets, const int32_t* row_src, const float* gate,
+                                    uint16_t* y, uint16_t* k_cache, uint16_t* v_cache, const int64_t* seg_base,
+                                    const int32_t* seg_cap, int64_t cache_rows, int32_t* seg_len, void* workspace,
+                                    size_t workspace_bytes, uint32_t* dev_status, void* stream_v) {
+  if (!cu_seqlens) return NAMOH_ERR_INVALID_ARG;
+  int Hr, Kr;
+  long long R;
+  const int st = check_varlen(B, total_tokens, max_seqlen, H, K, d_head, group, &Hr, &Kr, &R);
+  if (st != NAMOH_OK) return st;
+  return prefill_impl(q, k, v, B, max_seqlen, Hr, Kr, R, d_head, group, rope_base, rope_flags, cu_seqlens,
+                      seg_offsets, row_src, gate, y, k_cache, v_cache, seg_base, seg_cap, cache_rows, seg_len,
+                      workspace, workspace_bytes, dev_status, stream_v);
 }
 
 extern "C" int namoh_prefill(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int H, int K,

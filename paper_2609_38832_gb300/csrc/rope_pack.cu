@@ -13,7 +13,8 @@
 // [8l, 8l+8) and [D/2 + 8l, D/2 + 8l + 8) for lane l of a group) and pairs adjacent elements
 // inside them, so the lane's angles are j = 4l..4l+3 and D/4 + 4l..D/4 + 4l+3; global
 // positions (Sec. 3.2: rho_i(t) replaced by t) take t = (row_src[r] / Kr) % T from the
-// routing's inverse map, loaded one chunk ahead; the cache row is still the rank.
+// routing's inverse map, loaded one chunk ahead -- in a ragged batch t = row_src[r] / Kr -
+// cu_seqlens[b], b = segment / Hr; the cache row is still the rank.
 // Outputs: Q~ (bf16 scratch for the attention kernel), K~ into the key cache, and V copied
 // into the value cache unless the caller passed v_cache == v.  Given a plan buffer, block 0
 // builds the attention work list in the same launch.  Launched with programmatic dependent
@@ -55,8 +56,10 @@ __host__ __device__ constexpr size_t rope_smem_bytes(int nseg) {
   return (size_t)kRopeStages * RopeChunk<D, G>::kStageBytes + rope_offs_bytes(nseg) + kRopeStages * sizeof(uint64_t);
 }
 
-// kFlags: NAMOH_ROPE_INTERLEAVED and NAMOH_ROPE_GLOBAL (compile-time, so the default path
-// carries no branch of the variants)
+// kFlags: NAMOH_ROPE_INTERLEAVED, NAMOH_ROPE_GLOBAL and kRopeRagged (global positions in a
+// ragged batch), compile-time so that no variant carries another's branches
+constexpr unsigned kRopeRagged = 0x4u;
+
 template <int D, int G, unsigned kFlags>
 __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     const uint16_t* __restrict__ q, const uint16_t* __restrict__ k, const uint16_t* __restrict__ v, int R,
@@ -65,11 +68,12 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     uint16_t* __restrict__ k_cache, uint16_t* __restrict__ v_cache, int copy_v, RopeTable tab,
     uint32_t* __restrict__ status, int* __restrict__ plan_header, int4* __restrict__ plan_items,
     const int32_t* __restrict__ plan_cap, int plan_qtiles, const int32_t* __restrict__ pos_row_src,
-    FastDiv pos_k, FastDiv pos_t) {
+    FastDiv pos_k, FastDiv pos_t, const int32_t* __restrict__ pos_cu, FastDiv pos_hr) {
   using C = RopeChunk<D, G>;
   constexpr int HALF = D / 2;
   constexpr bool kInterleaved = (kFlags & NAMOH_ROPE_INTERLEAVED) != 0;
   constexpr bool kGlobal = (kFlags & NAMOH_ROPE_GLOBAL) != 0;
+  constexpr bool kRagged = (kFlags & kRopeRagged) != 0;
   extern __shared__ __align__(128) uint8_t smem_raw[];
   __shared__ int s_abort;
   pdl_launch_dependents();  // the attention kernel may start launching; it waits for this grid
@@ -156,8 +160,11 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
       // position: the rank, or the token's index t in its sequence
       float pos = (float)rho;
       if (kGlobal) {
-        const uint32_t bt = fastdiv((uint32_t)token_src, pos_k);  // b*T + t
-        pos = (float)(bt - fastdiv(bt, pos_t) * pos_t.d);
+        const uint32_t tok = fastdiv((uint32_t)token_src, pos_k);  // b*T + t, or the flat token index
+        if constexpr (kRagged)
+          pos = (float)((int)tok - __ldg(pos_cu + fastdiv((uint32_t)lo, pos_hr)));
+        else
+          pos = (float)(tok - fastdiv(tok, pos_t) * pos_t.d);
       }
       float sn[8], cs[8];
 #pragma unroll
@@ -240,7 +247,8 @@ cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, 
                                long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache,
                                int copy_v, const RopeTable& tab, uint32_t* status, int* plan_header,
                                int4* plan_items, const int32_t* plan_cap, int plan_qtiles,
-                               const int32_t* pos_row_src, FastDiv pos_k, FastDiv pos_t) {
+                               const int32_t* pos_row_src, FastDiv pos_k, FastDiv pos_t, const int32_t* pos_cu,
+                               FastDiv pos_hr) {
   switch (g) {
 #define NAMOH_ROPE_CASE(GG)                                                                                       \
   case GG: {                                                                                                      \
@@ -266,7 +274,7 @@ cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, 
     }                                                                                                            \
     return launch_pdl(kernel, dim3((unsigned)grid), dim3(kRopeThreads), smem, stream, q, k, v, R, seg_offsets,     \
                       nseg, seg_base, seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v, tab, status,         \
-                      plan_header, plan_items, plan_cap, plan_qtiles, pos_row_src, pos_k, pos_t);                \
+                      plan_header, plan_items, plan_cap, plan_qtiles, pos_row_src, pos_k, pos_t, pos_cu, pos_hr); \
   }
     NAMOH_ROPE_CASE(1)
     NAMOH_ROPE_CASE(2)
@@ -284,17 +292,19 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache, bool copy_v,
                              const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream,
                              void* plan, int plan_qtiles, const int32_t* plan_cap, const int32_t* pos_row_src,
-                             int pos_k, int pos_t, bool interleaved) {
+                             int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved) {
   int* plan_header = static_cast<int*>(plan);
   int4* plan_items = plan ? reinterpret_cast<int4*>(static_cast<char*>(plan) + 16) : nullptr;
   const size_t plan_smem = plan ? (size_t)plan_smem_ints(plan_qtiles, nseg) * sizeof(int) : 0;
   if (R == 0 && !plan) return cudaSuccess;
-  const unsigned flags = (interleaved ? NAMOH_ROPE_INTERLEAVED : 0u) | (pos_row_src ? NAMOH_ROPE_GLOBAL : 0u);
+  const unsigned flags = (interleaved ? NAMOH_ROPE_INTERLEAVED : 0u) | (pos_row_src ? NAMOH_ROPE_GLOBAL : 0u) |
+                         (pos_row_src && pos_cu ? kRopeRagged : 0u);
   auto go = [&](auto d_tag, auto f_tag) {
     return launch_rope_pack_d<decltype(d_tag)::value, decltype(f_tag)::value>(
         g, sm_count, nseg, plan_smem, plan != nullptr, stream, q, k, v, R, seg_offsets, seg_base, seg_cap, cache_rows,
         q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status, plan_header, plan_items, plan_cap, plan_qtiles,
-        pos_row_src, make_fastdiv((uint32_t)pos_k), make_fastdiv((uint32_t)pos_t));
+        pos_row_src, make_fastdiv((uint32_t)pos_k), make_fastdiv((uint32_t)pos_t), pos_cu,
+        make_fastdiv((uint32_t)pos_hr));
   };
   using D64 = std::integral_constant<int, 64>;
   using D128 = std::integral_constant<int, 128>;
@@ -302,11 +312,15 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
   using F1 = std::integral_constant<unsigned, 1u>;
   using F2 = std::integral_constant<unsigned, 2u>;
   using F3 = std::integral_constant<unsigned, 3u>;
+  using F6 = std::integral_constant<unsigned, 6u>;
+  using F7 = std::integral_constant<unsigned, 7u>;
   switch (flags) {
     case 0u: return D == 128 ? go(D128{}, F0{}) : go(D64{}, F0{});
     case 1u: return D == 128 ? go(D128{}, F1{}) : go(D64{}, F1{});
     case 2u: return D == 128 ? go(D128{}, F2{}) : go(D64{}, F2{});
-    default: return D == 128 ? go(D128{}, F3{}) : go(D64{}, F3{});
+    case 3u: return D == 128 ? go(D128{}, F3{}) : go(D64{}, F3{});
+    case 6u: return D == 128 ? go(D128{}, F6{}) : go(D64{}, F6{});
+    default: return D == 128 ? go(D128{}, F7{}) : go(D64{}, F7{});
   }
 }
 

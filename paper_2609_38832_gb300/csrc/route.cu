@@ -1,7 +1,8 @@
 // route.cu -- routing and dispatch (Sec. 3.1 Eq. namoh-gates; Sec. 3.2 Eq. namoh-head-rope).
 //
-// Every token selects exactly K heads, so sequence b's rows start at b*T*K and each
-// sequence's segment offsets depend only on that sequence's own head counts.
+// Every token selects exactly K heads, so sequence b's rows start at (its first token)*K --
+// b*T*K, or cu_seqlens[b]*K in a ragged batch -- and each sequence's segment offsets depend
+// only on that sequence's own head counts.
 //
 // The packed layout takes two launches, chained by programmatic dependent launch (the
 // second is resident and waiting before the first ends):
@@ -30,6 +31,25 @@ namespace {
 constexpr int kChunk = 256;  // tokens per block in the top-K and rank kernels
 
 constexpr float kLog2e = 1.4426950408889634f;
+
+// Token range [start, start + len) of sequence b: b*T and T, or from cu_seqlens in a ragged
+// batch (T = the longest sequence then).  A malformed cu_seqlens entry (decreasing, outside
+// [0, total], cu_seqlens[0] != 0, cu_seqlens[B] != total, or longer than T) clears `ok`; the
+// range is clamped into [0, total] and to T tokens, so every access stays inside the arrays.
+struct SeqRange {
+  int start, len;
+  bool ok;
+};
+__device__ __forceinline__ SeqRange seq_range(const int32_t* __restrict__ cu, int b, int B, int T, int total) {
+  if (!cu) return {b * T, T, true};
+  int s0 = __ldg(cu + b), s1 = __ldg(cu + b + 1);
+  const bool ok = s0 >= 0 && s1 >= s0 && s1 <= total && s1 - s0 <= T && (b > 0 || s0 == 0) &&
+                  (b < B - 1 || s1 == total);
+  s0 = min(max(s0, 0), total);
+  s1 = min(max(s1, s0), total);
+  s1 = min(s1, s0 + T);
+  return {s0, s1 - s0, ok};
+}
 
 // The H logits of token `tok` in registers (independent loads, all in flight together).
 // Non-finite logits become -FLT_MAX and set `bad`.
@@ -232,7 +252,8 @@ __global__ void __launch_bounds__(kChunk) route_topk_kernel(const float* __restr
 // seg_offsets[b*H + h] = b*T*K + sum of n[b, h'] over h' < h.
 __global__ void __launch_bounds__(1024) route_scan_kernel(const int32_t* __restrict__ chunk_count, int B, int T,
                                                           int H, int K, int nchunks, int32_t* __restrict__ chunk_base,
-                                                          int32_t* __restrict__ seg_offsets) {
+                                                          int32_t* __restrict__ seg_offsets,
+                                                          const int32_t* __restrict__ cu_seqlens, int total) {
   __shared__ int s_part[1024];
   __shared__ int s_n[NAMOH_MAX_HEADS];
   const int b = blockIdx.x;
@@ -259,7 +280,7 @@ __global__ void __launch_bounds__(1024) route_scan_kernel(const int32_t* __restr
   if (p == P - 1) s_n[h] = run;
   __syncthreads();
   if (tid == 0) {
-    int off = b * T * K;  // < 2^31: checked on the host
+    int off = seq_range(cu_seqlens, b, B, T, total).start * K;  // < 2^31: checked on the host
     for (int hh = 0; hh < H; ++hh) {
       seg_offsets[(size_t)b * H + hh] = off;
       off += s_n[hh];
@@ -278,20 +299,24 @@ __global__ void __launch_bounds__(kChunk) route_local_kernel(const float* __rest
                                                              int nchunks, int32_t* __restrict__ topk_head,
                                                              float* __restrict__ gate, int32_t* __restrict__ rank,
                                                              int32_t* __restrict__ chunk_count,
-                                                             uint32_t* __restrict__ status) {
+                                                             uint32_t* __restrict__ status,
+                                                             const int32_t* __restrict__ cu_seqlens, int B,
+                                                             int total) {
   __shared__ uint32_t s_bal[kChunk / 32][NAMOH_MAX_HEADS];
   __shared__ int s_bad;
   pdl_launch_dependents();
   const int c = blockIdx.x, b = blockIdx.y;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int t = c * kChunk + tid;
-  const bool valid = t < T;
-  const size_t tok = (size_t)b * T + t;
   if (tid == 0) s_bad = 0;
   __syncthreads();
   // the logits may come from the kernel just before this one, and that kernel may still
   // read this call's outputs: nothing global is touched before the wait
   pdl_wait();
+  const SeqRange sr = seq_range(cu_seqlens, b, B, T, total);
+  if (!sr.ok && c == 0 && tid == 0) report(status, NAMOH_DEV_BAD_SEQLENS);
+  const bool valid = t < sr.len;
+  const size_t tok = (size_t)sr.start + t;
   uint64_t mask = 0;
   int hk[KMAX > 0 ? KMAX : 1];
   if (valid) mask = topk_token<HMAX, KMAX, kBiased>(scores, bias, tok, H, K, topk_head, gate, &s_bad, hk);
@@ -340,7 +365,8 @@ __global__ void __launch_bounds__(kChunk) route_final_kernel(const int32_t* __re
                                                              int K, int nchunks, const int32_t* chunk_count,
                                                              const int32_t* chunk_base, int32_t* __restrict__ rank,
                                                              int32_t* __restrict__ row, int32_t* seg_offsets,
-                                                             int32_t* __restrict__ row_src, int B) {
+                                                             int32_t* __restrict__ row_src, int B,
+                                                             const int32_t* __restrict__ cu_seqlens, int total) {
   __shared__ int s_tot[kChunk];
   __shared__ int s_bef[kChunk];
   __shared__ int s_cbase[NAMOH_MAX_HEADS];
@@ -349,10 +375,11 @@ __global__ void __launch_bounds__(kChunk) route_final_kernel(const int32_t* __re
   const int c = blockIdx.x, b = blockIdx.y;
   const int tid = threadIdx.x;
   const int t = c * kChunk + tid;
-  const bool valid = t < T;
-  const size_t tok = (size_t)b * T + t;
-  const size_t base = tok * K;
   pdl_wait();  // pass 1 (and the scan, when there is one) complete and visible
+  const SeqRange sr = seq_range(cu_seqlens, b, B, T, total);
+  const bool valid = t < sr.len;
+  const size_t tok = (size_t)sr.start + t;
+  const size_t base = tok * K;
   // this token's heads and local ranks first: their loads overlap the count-table work
   const bool vec4 = K == 4 && (reinterpret_cast<uintptr_t>(topk_head + base) & 15u) == 0 &&
                     (reinterpret_cast<uintptr_t>(rank + base) & 15u) == 0 &&
@@ -393,7 +420,7 @@ __global__ void __launch_bounds__(kChunk) route_final_kernel(const int32_t* __re
     }
     __syncthreads();
     if (tid == 0) {
-      int off = b * T * K;  // < 2^31: checked on the host
+      int off = sr.start * K;  // < 2^31: checked on the host
       for (int hh = 0; hh < H; ++hh) {
         s_soff[hh] = off;
         off += s_tot[hh];
@@ -401,7 +428,7 @@ __global__ void __launch_bounds__(kChunk) route_final_kernel(const int32_t* __re
     }
     __syncthreads();
     if (c == 0 && tid < H) seg_offsets[(size_t)b * H + tid] = s_soff[tid];
-    if (c == 0 && b == B - 1 && tid == 0) seg_offsets[(size_t)B * H] = B * T * K;
+    if (c == 0 && b == B - 1 && tid == 0) seg_offsets[(size_t)B * H] = (sr.start + sr.len) * K;
   }
   __syncthreads();
   if (!valid) return;
@@ -433,6 +460,8 @@ __global__ void __launch_bounds__(kChunk) route_final_kernel(const int32_t* __re
 struct RouteArgs {
   const float* scores;
   const float* bias;  // [H] or nullptr
+  const int32_t* cu_seqlens;  // [B + 1] for a ragged batch (T = longest sequence), or nullptr
+  int total;                  // tokens in all (ragged batch)
   int B, T, H, K, nchunks;
   int32_t *topk_head, *rank, *row, *seg_offsets, *row_src;
   float* gate;
@@ -453,18 +482,20 @@ int launch_route(const RouteArgs& a, cudaStream_t stream) {
     return cuda_check_launch("route_topk_kernel launch");
   }
   cudaError_t e = launch_pdl(route_local_kernel<HMAX, KMAX, kBiased>, chunks, dim3(kChunk), 0, stream, a.scores, a.bias,
-                             a.T, a.H, a.K, a.nchunks, a.topk_head, a.gate, a.rank, a.chunk_count, a.status);
+                             a.T, a.H, a.K, a.nchunks, a.topk_head, a.gate, a.rank, a.chunk_count, a.status,
+                             a.cu_seqlens, a.B, a.total);
   if (e != cudaSuccess) return cuda_fail(e, "route_local_kernel launch");
   const bool scan = (long long)a.nchunks * a.H > kFinalMaxTable;
   if (scan) {
     const int scan_threads = 1024 - (1024 % a.H);
     e = launch_pdl(route_scan_kernel, dim3((unsigned)a.B), dim3((unsigned)scan_threads), 0, stream,
-                   (const int32_t*)a.chunk_count, a.B, a.T, a.H, a.K, a.nchunks, a.chunk_base, a.seg_offsets);
+                   (const int32_t*)a.chunk_count, a.B, a.T, a.H, a.K, a.nchunks, a.chunk_base, a.seg_offsets,
+                   a.cu_seqlens, a.total);
     if (e != cudaSuccess) return cuda_fail(e, "route_scan_kernel launch");
   }
   e = launch_pdl(route_final_kernel, chunks, dim3(kChunk), 0, stream, (const int32_t*)a.topk_head, a.T, a.H, a.K,
                  a.nchunks, (const int32_t*)a.chunk_count, (const int32_t*)(scan ? a.chunk_base : nullptr), a.rank,
-                 a.row, a.seg_offsets, a.row_src, a.B);
+                 a.row, a.seg_offsets, a.row_src, a.B, a.cu_seqlens, a.total);
   if (e != cudaSuccess) return cuda_fail(e, "route_final_kernel launch");
   return NAMOH_OK;
 }
@@ -498,13 +529,18 @@ extern "C" size_t namoh_route_workspace_size(int B, int T, int H, int K) {
   return align_up(ws.used, 256);
 }
 
-extern "C" int namoh_route_biased(const float* scores, const float* bias, int B, int T, int H, int K,
-                                  int32_t* topk_head, float* gate, int32_t* rank, int32_t* row, int32_t* seg_offsets,
-                                  int32_t* row_src, void* workspace, size_t workspace_bytes, uint32_t* dev_status,
-                                  void* stream_v) {
+namespace namoh {
+namespace {
+// Shared body of the routing entry points.  cu_seqlens == nullptr: B sequences of T tokens;
+// else a ragged batch of `total` tokens whose longest sequence has T tokens.
+int route_impl(const float* scores, const float* bias, const int32_t* cu_seqlens, int B, int T, int total, int H,
+               int K, int32_t* topk_head, float* gate, int32_t* rank, int32_t* row, int32_t* seg_offsets,
+               int32_t* row_src, void* workspace, size_t workspace_bytes, uint32_t* dev_status, void* stream_v) {
   if (!scores || !topk_head || !gate || !dev_status) return NAMOH_ERR_INVALID_ARG;
   if (B < 1 || T < 1 || H < 1 || K < 1 || K > H || H > NAMOH_MAX_HEADS) return NAMOH_ERR_INVALID_ARG;
-  if ((long long)B * T * K >= (1ll << 31) || (long long)B * H >= (1ll << 20)) return NAMOH_ERR_INVALID_ARG;
+  const long long tokens = cu_seqlens ? (long long)total : (long long)B * T;
+  if (tokens * K >= (1ll << 31) || (long long)B * H >= (1ll << 20)) return NAMOH_ERR_INVALID_ARG;
+  if (cu_seqlens && total < T) return NAMOH_ERR_INVALID_ARG;
   const bool compact = seg_offsets != nullptr;
   if (compact != (rank != nullptr) || compact != (row != nullptr) || compact != (row_src != nullptr))
     return NAMOH_ERR_INVALID_ARG;
@@ -512,11 +548,18 @@ extern "C" int namoh_route_biased(const float* scores, const float* bias, int B,
   RouteArgs a{};
   a.scores = scores;
   a.bias = bias;
+  a.cu_seqlens = cu_seqlens;
+  a.total = total;
   a.B = B;
   a.T = T;
+  if (cu_seqlens && !compact) {  // picks only: one flat sequence of every token
+    a.cu_seqlens = nullptr;
+    a.B = 1;
+    a.T = total;
+  }
   a.H = H;
   a.K = K;
-  a.nchunks = (T + kChunk - 1) / kChunk;
+  a.nchunks = (a.T + kChunk - 1) / kChunk;
   a.topk_head = topk_head;
   a.gate = gate;
   a.rank = rank;
@@ -532,6 +575,25 @@ extern "C" int namoh_route_biased(const float* scores, const float* bias, int B,
     if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
   }
   return a.bias ? launch_route_h<true>(a, stream) : launch_route_h<false>(a, stream);
+}
+}  // namespace
+}  // namespace namoh
+
+extern "C" int namoh_route_biased(const float* scores, const float* bias, int B, int T, int H, int K,
+                                  int32_t* topk_head, float* gate, int32_t* rank, int32_t* row, int32_t* seg_offsets,
+                                  int32_t* row_src, void* workspace, size_t workspace_bytes, uint32_t* dev_status,
+                                  void* stream_v) {
+  return route_impl(scores, bias, nullptr, B, T, 0, H, K, topk_head, gate, rank, row, seg_offsets, row_src, workspace,
+                    workspace_bytes, dev_status, stream_v);
+}
+
+extern "C" int namoh_route_varlen(const float* scores, const float* bias, const int32_t* cu_seqlens, int B,
+                                  int total_tokens, int max_seqlen, int H, int K, int32_t* topk_head, float* gate,
+                                  int32_t* rank, int32_t* row, int32_t* seg_offsets, int32_t* row_src,
+                                  void* workspace, size_t workspace_bytes, uint32_t* dev_status, void* stream_v) {
+  if (!cu_seqlens || total_tokens < 1) return NAMOH_ERR_INVALID_ARG;
+  return route_impl(scores, bias, cu_seqlens, B, max_seqlen, total_tokens, H, K, topk_head, gate, rank, row,
+                    seg_offsets, row_src, workspace, workspace_bytes, dev_status, stream_v);
 }
 
 extern "C" int namoh_route(const float* scores, int B, int T, int H, int K, int32_t* topk_head, float* gate,
