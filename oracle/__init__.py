@@ -75,10 +75,13 @@ def _load():
         lib.oracle_prefill_rows.argtypes = [P, P, P, i32, i32, i32, f64, P, P, P, P, P, i64, P, i32, P]
         lib.oracle_decode_step.argtypes = [P, P, P, P, P, i32, i32, i32, i32, i32, f64,
                                            P, P, P, P, P, P, i32, P]
+        lib.oracle_proj_qkv.argtypes = [P, i32, P, i32, i32, i32, i32, P, i32, P, P, P, P, i32]
+        lib.oracle_proj_out.argtypes = [P, P, i64, i32, i32, i32, P, i32, i32, P, i32]
         lib.oracle_default_threads.argtypes = []
         for fn in ("oracle_route_topk", "oracle_route_biased", "oracle_dispatch", "oracle_dispatch_varlen",
                    "oracle_rope", "oracle_prefill",
-                   "oracle_prefill_rows", "oracle_decode_step", "oracle_default_threads"):
+                   "oracle_prefill_rows", "oracle_decode_step", "oracle_proj_qkv", "oracle_proj_out",
+                   "oracle_default_threads"):
             getattr(lib, fn).restype = ctypes.c_int
         _lib = lib
         return lib
@@ -317,3 +320,40 @@ def decode_step(topk_head, gate, q, k, v, Hr: int, d: int, g: int, base: float,
                                 _ptr(token_pos) if token_pos is not None else None)
     _check(rc, "decode_step")
     return y
+
+
+def proj_qkv(x, w_qkv, seg_offsets, row_src, Hr: int, Kr: int, g: int, d: int, nthreads: int | None = None):
+    """Eq. (namoh-qkv) in the packed layout: x [N, d_model] and w_qkv [Hr, (g+2) d, d_model] as
+    bf16 bits.  Returns fp64 q [R g, d], k [R, d], v [R, d]."""
+    lib = _load()
+    x = np.ascontiguousarray(x, dtype=np.uint16)
+    w = np.ascontiguousarray(w_qkv, dtype=np.uint16)
+    seg = np.ascontiguousarray(seg_offsets, dtype=np.int32)
+    rs = np.ascontiguousarray(row_src, dtype=np.int32)
+    d_model = x.shape[1]
+    if w.shape != (Hr, (g + 2) * d, d_model):
+        raise OracleError("w_qkv must be [Hr, (g+2) d, d_model]")
+    R = int(seg[-1])
+    q = np.empty((R * g, d)); k = np.empty((R, d)); v = np.empty((R, d))
+    nthreads = default_threads() if nthreads is None else int(nthreads)
+    _check(lib.oracle_proj_qkv(_ptr(x), d_model, _ptr(w), Hr, Kr, g, d, _ptr(seg), len(seg) - 1, _ptr(rs), _ptr(q),
+                               _ptr(k), _ptr(v), nthreads), "proj_qkv")
+    return q, k, v
+
+
+def proj_out(y, topk_head, w_o, g: int, d: int, nthreads: int | None = None):
+    """Eq. (namoh-attention) output projection: y [N, Kr, g, d] (fp64 per-slot g h), topk_head
+    [N, Kr], w_o [Hr, d_model, g d] bf16 bits.  Returns o [N, d_model] fp64."""
+    lib = _load()
+    topk = np.ascontiguousarray(topk_head, dtype=np.int32)
+    N, Kr = topk.shape
+    y = np.ascontiguousarray(y, dtype=np.float64).reshape(N, Kr, g * d)
+    w = np.ascontiguousarray(w_o, dtype=np.uint16)
+    Hr, d_model, gd = w.shape
+    if gd != g * d:
+        raise OracleError("w_o must be [Hr, d_model, g d]")
+    o = np.empty((N, d_model))
+    nthreads = default_threads() if nthreads is None else int(nthreads)
+    _check(lib.oracle_proj_out(_ptr(y), _ptr(topk), N, Kr, g, d, _ptr(w), Hr, d_model, _ptr(o), nthreads),
+           "proj_out")
+    return o

@@ -17,8 +17,9 @@
  *   - RoPE:      Sec. 3.2, Eq. (namoh-head-rope)  q~ = q R(rho), k~ = k R(rho).
  *   - attention: Sec. 3.1, Eq. (namoh-attention)  h_{t,i} = Attn(q~_{t,i}, [k~_{s,i}], [v_{s,i}]),
  *                s in I_i, s <= t, standard scaled dot-product attention.
- *   - combine:   Sec. 3.1, Eq. (namoh-attention)  the per-slot term g_{t,i} h_{t,i}
- *                (the W_O projection is outside this path).
+ *   - combine:   Sec. 3.1, Eq. (namoh-attention)  the per-slot term g_{t,i} h_{t,i}.
+ *   - layer:     Sec. 3.1, Eq. (namoh-qkv)  q, k, v = x_t W^(i) for active pairs only, in the
+ *                packed layout; Eq. (namoh-attention)  o_t = sum_i g_{t,i} h_{t,i} W_O^(i).
  *   - decode:    Sec. 3.1 (last paragraph) and Sec. 3.2: a new token appends to and attends
  *                within only its selected heads' histories; its rank is the current length.
  *   - GQA:       App. C, "Adopted KV-group routing": K/g of H/g groups are selected, the g
@@ -609,6 +610,109 @@ int oracle_decode_step(const int32_t *topk_head, const double *gate, const uint1
     }
     free(tmp); free(qr); free(h);
     return st;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Projections around the path (Sec. 3.1, Eq. namoh-qkv and Eq. namoh-attention) */
+/* ------------------------------------------------------------------------- */
+
+struct proj_qkv_ctx {
+    const uint16_t *x, *w;
+    const int32_t *seg_offsets, *row_src;
+    int nseg, Hr, Kr, g, d, d_model;
+    double *q, *k, *v;
+};
+
+/* One packed row r: the token is row_src[r] / Kr, the group head that of r's segment. */
+static void proj_qkv_row(long r, void *arg)
+{
+    const struct proj_qkv_ctx *c = (const struct proj_qkv_ctx *)arg;
+    int lo = 0, hi = c->nseg;
+    while (hi - lo > 1) {
+        int mid = (lo + hi) / 2;
+        if (c->seg_offsets[mid] <= r) lo = mid; else hi = mid;
+    }
+    const int hr = lo % c->Hr;
+    const long tok = c->row_src[r] / c->Kr;
+    const int ncols = (c->g + 2) * c->d;
+    const uint16_t *xr = c->x + tok * (long)c->d_model;
+    for (int n = 0; n < ncols; ++n) {
+        const uint16_t *wr = c->w + ((long)hr * ncols + n) * c->d_model;
+        double acc = 0.0;
+        for (int m = 0; m < c->d_model; ++m) acc += bf16_to_double(xr[m]) * bf16_to_double(wr[m]);
+        if (n < c->g * c->d) c->q[(r * c->g + n / c->d) * c->d + n % c->d] = acc;
+        else if (n < (c->g + 1) * c->d) c->k[r * c->d + (n - c->g * c->d)] = acc;
+        else c->v[r * c->d + (n - (c->g + 1) * c->d)] = acc;
+    }
+}
+
+/*
+ * oracle_proj_qkv: Sec. 3.1, Eq. (namoh-qkv): only active token-head pairs project,
+ *   q_{t,i} = x_t W_Q^(i), k_{t,i} = x_t W_K^(i), v_{t,i} = x_t W_V^(i), t in I_i,
+ * in the packed-row layout of the routing (App. C: a KV group projects one key and one
+ * value and g queries, one per query head of the group).
+ *   x           [N, d_model] bf16 token representations (N tokens on the flat axis)
+ *   w           [Hr, (g+2) d, d_model] bf16: for group i, rows j d .. j d + d - 1 hold
+ *               W_Q of query head i g + j transposed (row c = column c of W_Q), then
+ *               d rows of W_K^(i) transposed, then d rows of W_V^(i) transposed
+ *   seg_offsets [nseg + 1], row_src [R]: the routing's packed layout (nseg = B Hr)
+ *   q [R g, d], k [R, d], v [R, d] fp64 out, q of row r and query head j at row r g + j
+ */
+int oracle_proj_qkv(const uint16_t *x, int d_model, const uint16_t *w, int Hr, int Kr, int g, int d,
+                    const int32_t *seg_offsets, int nseg, const int32_t *row_src, double *q, double *k, double *v,
+                    int nthreads)
+{
+    if (!x || !w || !seg_offsets || !row_src || !q || !k || !v) return ORACLE_ERR_ARG;
+    if (d_model < 1 || Hr < 1 || Kr < 1 || g < 1 || d < 1 || nseg < 1) return ORACLE_ERR_ARG;
+    struct proj_qkv_ctx c = {x, w, seg_offsets, row_src, nseg, Hr, Kr, g, d, d_model, q, k, v};
+    parallel_for(seg_offsets[nseg], nthreads, proj_qkv_row, &c);
+    return ORACLE_OK;
+}
+
+struct proj_out_ctx {
+    const double *y;
+    const uint16_t *w;
+    const int32_t *topk_head;
+    int Kr, g, d, d_model;
+    double *o;
+};
+
+/* One token t: o_t = sum over its slots k and the g query heads j of the slot's group. */
+static void proj_out_token(long t, void *arg)
+{
+    const struct proj_out_ctx *c = (const struct proj_out_ctx *)arg;
+    const int gd = c->g * c->d;
+    for (int m = 0; m < c->d_model; ++m) {
+        double acc = 0.0;
+        for (int k = 0; k < c->Kr; ++k) {
+            const int hr = c->topk_head[t * c->Kr + k];
+            const double *yk = c->y + (t * c->Kr + k) * (long)gd;
+            const uint16_t *wr = c->w + ((long)hr * c->d_model + m) * gd;
+            for (int e = 0; e < gd; ++e) acc += yk[e] * bf16_to_double(wr[e]);
+        }
+        c->o[t * c->d_model + m] = acc;
+    }
+}
+
+/*
+ * oracle_proj_out: Sec. 3.1, Eq. (namoh-attention): o_t = sum_{i in S_K(t)} g_{t,i} h_{t,i} W_O^(i),
+ * from the combine's per-slot terms y = g h.
+ *   y          [N, Kr, g, d] fp64 per-slot terms (slot k of token t, query head j of its group)
+ *   topk_head  [N, Kr]: the group of each slot
+ *   w          [Hr, d_model, g d] bf16: for group i, row m holds column m of W_O of query
+ *              heads i g .. i g + g - 1, one after the other (W_O^(i g + j) row c at j d + c)
+ *   o          [N, d_model] fp64 out
+ */
+int oracle_proj_out(const double *y, const int32_t *topk_head, long N, int Kr, int g, int d, const uint16_t *w,
+                    int Hr, int d_model, double *o, int nthreads)
+{
+    if (!y || !topk_head || !w || !o || N < 0 || Kr < 1 || g < 1 || d < 1 || Hr < 1 || d_model < 1)
+        return ORACLE_ERR_ARG;
+    for (long i = 0; i < N * Kr; ++i)
+        if (topk_head[i] < 0 || topk_head[i] >= Hr) return ORACLE_ERR_ARG;
+    struct proj_out_ctx c = {y, w, topk_head, Kr, g, d, d_model, o};
+    parallel_for(N, nthreads, proj_out_token, &c);
+    return ORACLE_OK;
 }
 
 /* Number of worker threads the oracle would use by default. */

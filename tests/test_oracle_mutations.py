@@ -23,6 +23,10 @@ MUTATIONS = {
                              "c->pos ? (double)(row - off) : (double)(row - off)"),
     "varlen_segments_of_sequence_0": ("int r = seg_offsets[(long)b * H + topk_head[idx]] + rank[idx];",
                                       "int r = seg_offsets[topk_head[idx]] + rank[idx];"),
+    "proj_query_heads_swapped": ("c->q[(r * c->g + n / c->d) * c->d + n % c->d] = acc;",
+                                 "c->q[(r * c->g + (c->g - 1 - n / c->d)) * c->d + n % c->d] = acc;"),
+    "proj_wrong_group": ("const int hr = lo % c->Hr;", "const int hr = (lo + 1) % c->Hr;"),
+    "proj_out_drops_first_slot": ("for (int k = 0; k < c->Kr; ++k) {", "for (int k = 1; k < c->Kr; ++k) {"),
     "decode_ignores_token_pos": ("const double p = token_pos ? (double)token_pos[b] : (double)rho;",
                                  "const double p = token_pos ? (double)rho : (double)rho;"),
     "no_scale": ("double scale = 1.0 / sqrt((double)d);", "double scale = 1.0;"),
@@ -56,7 +60,8 @@ def test_pins_catch_mutation(tmp_path, name):
     shutil.copytree(os.path.join(ROOT, "paper_2609_38832_gb300"), tmp_path / "paper_2609_38832_gb300",
                     ignore=shutil.ignore_patterns("*.so", "__pycache__", "csrc", "_build"))
     os.makedirs(tmp_path / "tests")
-    for f in ("conftest.py", "test_oracle_route.py", "test_oracle_attention.py", "test_accounting.py"):
+    for f in ("conftest.py", "test_oracle_route.py", "test_oracle_attention.py", "test_oracle_layer.py",
+              "test_accounting.py"):
         shutil.copy(os.path.join(ROOT, "tests", f), tmp_path / "tests")
     shutil.copytree(os.path.join(ROOT, "tests", "golden"), tmp_path / "tests" / "golden")
     r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider", "-m", "not gpu",
