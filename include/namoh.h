@@ -334,6 +334,44 @@ NAMOH_API int namoh_decode_ex(const int32_t *topk_head, const float *gate, const
                               uint16_t *y, void *workspace, size_t workspace_bytes, uint32_t *dev_status,
                               void *stream);
 
+/* ------------------------------------------------------------------------- *
+ * The projections around the path (the full attention layer).
+ * Sec. 3.1, Eq. (namoh-qkv): only an active token-head pair projects,
+ *   q_{t,i} = x_t W_Q^(i), k_{t,i} = x_t W_K^(i), v_{t,i} = x_t W_V^(i), t in I_i.
+ * Sec. 3.1, Eq. (namoh-attention): o_t = sum_{i in S_K(t)} g_{t,i} h_{t,i} W_O^(i).
+ * App. C: a KV group projects one key, one value and g queries (one per query head).
+ * Both run as one grouped GEMM over the packed rows of the routing (tcgen05 tiles of 128
+ * rows, the rows gathered from the token axis by TMA), so they follow namoh_route or
+ * namoh_route_varlen directly: seg_offsets [B*Hr + 1] and row_src [R] are its outputs,
+ * R = total_tokens * Kr (total_tokens = B*T for a fixed-length batch).
+ *
+ * namoh_proj_qkv
+ *   x      [total_tokens, d_model] bf16 token representations.
+ *   w_qkv  [Hr, (g+2) d, d_model] bf16, one block per KV group i: rows j d .. j d + d - 1
+ *          hold W_Q of query head i g + j transposed (row c = column c of W_Q), then d rows
+ *          of W_K^(i) transposed, then d rows of W_V^(i) transposed.
+ *   q [R*g, d], k [R, d], v [R, d] bf16 out: exactly namoh_prefill's inputs.
+ * namoh_proj_out
+ *   y      [total_tokens, K, d] bf16: namoh_prefill's output (per-slot g h).
+ *   w_o    [Hr, d_model, g d] bf16, one block per group: row m holds column m of W_O of the
+ *          group's query heads one after the other (W_O^(i g + j) row c at column j d + c).
+ *   o      [total_tokens, d_model] fp32 out; accumulate = 0 overwrites it, 1 adds to it
+ *          (e.g. onto a residual).  Each token's slots are added in an unspecified order.
+ * Workspace: namoh_proj_workspace_size (the tile list of the segments).
+ * Supports d_head in {64, 128}, g in {1, 2, 4, 8}, d_model a multiple of 64 up to 65536.
+ * x, w, q, k, v, y, o 16-byte aligned.  Rows of an inconsistent layout (a malformed
+ * cu_seqlens) are computed from clamped indices and write nothing outside the outputs.
+ * ------------------------------------------------------------------------- */
+NAMOH_API size_t namoh_proj_workspace_size(int B, int H, int K, int group);
+NAMOH_API int namoh_proj_qkv(const uint16_t *x, int total_tokens, int d_model, const uint16_t *w_qkv, int B, int H,
+                             int K, int d_head, int group, const int32_t *seg_offsets, const int32_t *row_src,
+                             uint16_t *q, uint16_t *k, uint16_t *v, void *workspace, size_t workspace_bytes,
+                             uint32_t *dev_status, void *stream);
+NAMOH_API int namoh_proj_out(const uint16_t *y, int total_tokens, int d_model, const uint16_t *w_o, int B, int H,
+                             int K, int d_head, int group, const int32_t *seg_offsets, const int32_t *row_src,
+                             float *o, int accumulate, void *workspace, size_t workspace_bytes,
+                             uint32_t *dev_status, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -18,6 +18,7 @@ from ._abi import (NAMOH_DEV_BAD_SEQLENS, NAMOH_DEV_CAPACITY, NAMOH_DEV_NONFINIT
                    NAMOH_ROPE_GLOBAL, NAMOH_ROPE_INTERLEAVED, NamohError)
 
 __all__ = ["namoh_route", "namoh_route_varlen", "namoh_prefill", "namoh_prefill_varlen", "namoh_decode",
+           "namoh_proj_qkv", "namoh_proj_out",
            "namoh_rope_pack", "namoh_attention_plan", "namoh_attention", "RouteOutputs", "Workspace", "NamohError",
            "NAMOH_DEV_BAD_SEQLENS", "NAMOH_DEV_CAPACITY", "NAMOH_DEV_NONFINITE_SCORE", "NAMOH_DEV_TIMEOUT",
            "NAMOH_ROPE_GLOBAL", "NAMOH_ROPE_INTERLEAVED", "library_path"]
@@ -292,6 +293,63 @@ def namoh_attention(q_rot: torch.Tensor, k_cache: torch.Tensor, v_cache: torch.T
                              _ptr(y), _ptr(st), _stream(stream))
     _abi.check("namoh_attention", rc)
     return y
+
+
+def namoh_proj_qkv(x: torch.Tensor, w_qkv: torch.Tensor, seg_offsets: torch.Tensor, row_src: torch.Tensor, *,
+                   B: int, H: int, K: int, group: int = 1, q: Optional[torch.Tensor] = None,
+                   k: Optional[torch.Tensor] = None, v: Optional[torch.Tensor] = None,
+                   workspace: Optional[Workspace] = None, status: Optional[torch.Tensor] = None, stream=None):
+    """Eq. (namoh-qkv) for the active pairs only (see namoh_proj_qkv in include/namoh.h).
+
+    x [N, d_model], w_qkv [Hr, (g+2) d, d_model] bf16; returns packed q [R*g, d], k [R, d],
+    v [R, d] (R = N*K/g), ready for namoh_prefill."""
+    lib = _abi.load()
+    if x.dtype != torch.bfloat16 or w_qkv.dtype != torch.bfloat16 or w_qkv.dim() != 3:
+        raise ValueError("x and w_qkv must be bfloat16; w_qkv [Hr, (g+2) d, d_model]")
+    N, d_model = x.shape
+    Hr, ncols, wd = w_qkv.shape
+    d = ncols // (group + 2)
+    if Hr != H // group or ncols != (group + 2) * d or wd != d_model:
+        raise ValueError("w_qkv must be [H/g, (g+2) d_head, d_model]")
+    R = N * (K // group)
+    dev = x.device
+    q = torch.empty((R * group, d), dtype=torch.bfloat16, device=dev) if q is None else q
+    k = torch.empty((R, d), dtype=torch.bfloat16, device=dev) if k is None else k
+    v = torch.empty((R, d), dtype=torch.bfloat16, device=dev) if v is None else v
+    ws = _ws(workspace, lib.namoh_proj_workspace_size(B, H, K, group), dev)
+    st = _status(status, dev)
+    rc = lib.namoh_proj_qkv(_ptr(x), N, d_model, _ptr(w_qkv), B, H, K, d, group, _ptr(seg_offsets), _ptr(row_src),
+                            _ptr(q), _ptr(k), _ptr(v), _ptr(ws), ws.numel(), _ptr(st), _stream(stream))
+    _abi.check("namoh_proj_qkv", rc)
+    return q, k, v
+
+
+def namoh_proj_out(y: torch.Tensor, w_o: torch.Tensor, seg_offsets: torch.Tensor, row_src: torch.Tensor, *,
+                   B: int, H: int, K: int, group: int = 1, o: Optional[torch.Tensor] = None,
+                   accumulate: bool = False, workspace: Optional[Workspace] = None,
+                   status: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """o_t = sum over the token's slots of y W_O (see namoh_proj_out in include/namoh.h).
+
+    y [N, K, d] bf16 (namoh_prefill's output), w_o [Hr, d_model, g d] bf16; returns o [N, d_model]
+    fp32 (added onto ``o`` when accumulate)."""
+    lib = _abi.load()
+    if y.dtype != torch.bfloat16 or w_o.dtype != torch.bfloat16 or w_o.dim() != 3:
+        raise ValueError("y and w_o must be bfloat16; w_o [Hr, d_model, g d]")
+    d = y.shape[-1]
+    N = y.numel() // (K * d)  # y is [N, K, d] or [B, T, K, d]
+    Hr, d_model, gd = w_o.shape
+    if Hr != H // group or gd != group * d:
+        raise ValueError("w_o must be [H/g, d_model, g d_head]")
+    dev = y.device
+    if o is None:
+        o = torch.empty((N, d_model), dtype=torch.float32, device=dev)
+        accumulate = False
+    ws = _ws(workspace, lib.namoh_proj_workspace_size(B, H, K, group), dev)
+    st = _status(status, dev)
+    rc = lib.namoh_proj_out(_ptr(y), N, d_model, _ptr(w_o), B, H, K, d, group, _ptr(seg_offsets), _ptr(row_src),
+                            _ptr(o), 1 if accumulate else 0, _ptr(ws), ws.numel(), _ptr(st), _stream(stream))
+    _abi.check("namoh_proj_out", rc)
+    return o
 
 
 def namoh_decode(topk_head: torch.Tensor, gate: torch.Tensor, q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, *,

@@ -19,7 +19,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(PKG, "_build")
 LIB_PATH = os.path.join(PKG, "libnamoh.so")
 
-SOURCES = ["api.cu", "route.cu", "rope_pack.cu", "prefill_attn.cu", "decode.cu"]
+SOURCES = ["api.cu", "route.cu", "rope_pack.cu", "prefill_attn.cu", "decode.cu", "proj.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
           "-diag-suppress", "177"]
@@ -42,7 +42,7 @@ def _stale(out: str, deps: list[str]) -> bool:
 def build(force: bool = False, verbose: bool = False) -> str:
     nvcc = _nvcc()
     os.makedirs(BUILD_DIR, exist_ok=True)
-    headers = [os.path.join(CSRC, "common.cuh"), os.path.join(INCLUDE, "namoh.h")]
+    headers = [os.path.join(CSRC, "common.cuh"), os.path.join(CSRC, "plan.cuh"), os.path.join(INCLUDE, "namoh.h")]
     objs = []
     jobs = []
     for src in SOURCES:
