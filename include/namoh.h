@@ -357,12 +357,13 @@ NAMOH_API int namoh_decode_ex(const int32_t *topk_head, const float *gate, const
  *          group's query heads one after the other (W_O^(i g + j) row c at column j d + c).
  *   o      [total_tokens, d_model] fp32 out; accumulate = 0 overwrites it, 1 adds to it
  *          (e.g. onto a residual).  Each token's slots are added in an unspecified order.
- * Workspace: namoh_proj_workspace_size (the tile list of the segments).
- * Supports d_head in {64, 128}, g in {1, 2, 4, 8}, d_model a multiple of 64 up to 65536.
+ * Workspace: namoh_proj_workspace_size (the list of 128-row tiles of the segments).
+ * Supports d_head in {64, 128}, g in {1, 2, 4, 8}, d_model a multiple of 64 up to 65536, and
+ * B*(H/g + 1) <= 51200.
  * x, w, q, k, v, y, o 16-byte aligned.  Rows of an inconsistent layout (a malformed
  * cu_seqlens) are computed from clamped indices and write nothing outside the outputs.
  * ------------------------------------------------------------------------- */
-NAMOH_API size_t namoh_proj_workspace_size(int B, int H, int K, int group);
+NAMOH_API size_t namoh_proj_workspace_size(int B, int total_tokens, int H, int K, int group);
 NAMOH_API int namoh_proj_qkv(const uint16_t *x, int total_tokens, int d_model, const uint16_t *w_qkv, int B, int H,
                              int K, int d_head, int group, const int32_t *seg_offsets, const int32_t *row_src,
                              uint16_t *q, uint16_t *k, uint16_t *v, void *workspace, size_t workspace_bytes,

@@ -10,15 +10,22 @@
 //                         into o[t] (fp32): the token's K slots sum there.
 // Only active token-head pairs are computed (Sec. 3.1: inactive pairs generate nothing).
 //
-// One persistent CTA per SM, 192 threads:
+// One persistent CTA per SM, 288 threads:
 //   warps 0-3  epilogue: TMEM lane = tile row; fp32 accumulators -> bf16 rows (QKV) or fp32
 //              reductions into o (OUT)
-//   warp 4     loads: per 64-wide slice of the contraction, 32 TMA gather4 copies (one per lane,
-//              four token rows each) fill the 128-row A tile in the 128-byte-swizzled layout,
-//              and one TMA tile copy brings the group's BN x 64 weight tile
-//   warp 5     TMEM owner and MMA issue: tcgen05.mma kind::f16, M = 128, N = BN, K = 16
-// Work items are (128-row tile of a segment, BN-column tile), taken in a static round robin;
-// the N tiles of one row tile are adjacent items, so the gathered rows are reused from L2.
+//   warps 4-7  loads: per 64-wide slice of the contraction the 128 gathered A rows arrive by
+//              16-byte cp.async copies (a warp moves four whole 128-byte rows per instruction)
+//              into the 128-byte-swizzled layout, and one TMA tile copy brings the group's
+//              BN x 64 weight tile.  A thread retires stage j once its copies of it have
+//              landed (wait_group, kLag stages later), fences them into the async proxy and
+//              arrives on the stage's barrier.  (TMA gather4 moves only 512 bytes per
+//              instruction and measured 7x slower here.)
+//   warp 8     TMEM owner and MMA issue: tcgen05.mma kind::f16, M = 128, N = BN, K = 16
+// Work items are (128-row tile of a segment, BN-column tile) from a list ordered by sequence,
+// then position in the segment, then head: CTAs running at the same time work on the same
+// stretch of tokens across heads, so x rows (QKV) and o rows (OUT) are reused from L2, and
+// the N tiles of one row tile are adjacent items.  A static round robin hands out the items;
+// the loaders fetch the next item's row indices during the current one.
 // Two TMEM accumulators let the epilogue of one item overlap the main loop of the next.
 // Every wait is bounded (NAMOH_DEV_TIMEOUT).
 #include "common.cuh"
@@ -28,8 +35,9 @@ namespace proj {
 
 constexpr int BM = 128;  // packed rows per tile
 constexpr int BK = 64;   // contraction elements per stage: one 128-byte swizzle row
-constexpr int kThreads = 192;
-constexpr int kSmemBudget = 212 * 1024;
+constexpr int kThreads = 288;
+constexpr int kSmemBudget = 208 * 1024;
+constexpr int kMaxTileListBytes = 200 * 1024;  // shared memory of the tile-list builder
 
 enum Mode { kQKV = 0, kOut = 1 };
 
@@ -40,19 +48,23 @@ struct Layout {
   static constexpr int kB = BN * 128;
   static constexpr int kStage = kA + kB;
   static constexpr int kStages = kSmemBudget / kStage > 6 ? 6 : kSmemBudget / kStage;
+  static constexpr int kLag = kStages - 2;  // stages of copies a loader keeps in flight before retiring one
+  static_assert(kLag >= 1, "pipeline depth");
   static constexpr int kBar = kStages * kStage;
   static constexpr int kAlloc = kBar + 256 + 1024;  // barriers, plus slack for 1024-byte alignment
 };
 
 struct Params {
   const int32_t* seg_offsets;  // [nseg + 1]
-  const int32_t* tile_prefix;  // [nseg + 1]: 128-row tiles of the segments before s; [nseg] = all
+  const int2* tiles;           // {segment, tile index in it}, in work order
+  const int32_t* ntiles;       // [1]: length of the list
   const int32_t* row_src;      // [R]
   int nseg, Hr, Kr;
   int a_rows;                  // rows of the gathered tensor (tokens for QKV, token slots for OUT)
   int kdim;                    // contraction length: d_model (QKV) or g d (OUT)
   int ncols;                   // output columns per group: (g + 2) d (QKV) or d_model (OUT)
   int g, d;
+  const void* a;               // the gathered tensor: x [a_rows, kdim] (QKV) or y (OUT)
   uint16_t *q, *k, *v;         // QKV outputs
   float* o;                    // OUT output [ntok, d_model]
   int ntok;
@@ -71,21 +83,14 @@ struct Tile {
   int seg, row0, rows, hr, nt;
 };
 
-// Item -> (segment, rows, column tile).  The segment is the last s with tile_prefix[s] <= the
-// item's row tile (empty segments have no tiles, so the search passes over them).
-__device__ __forceinline__ Tile decode_item(const Params& p, int item, int nt_count) {
+// Row tile -> its segment, first row and rows.
+__device__ __forceinline__ Tile decode_tile(const Params& p, int2 st) {
   Tile t;
-  const int mtg = item / nt_count;
-  t.nt = item - mtg * nt_count;
-  int lo = 0, hi = p.nseg;
-  while (hi - lo > 1) {
-    const int mid = (lo + hi) >> 1;
-    if (__ldg(p.tile_prefix + mid) <= mtg) lo = mid; else hi = mid;
-  }
-  t.seg = lo;
-  t.row0 = __ldg(p.seg_offsets + lo) + (mtg - __ldg(p.tile_prefix + lo)) * BM;
-  t.rows = min(BM, __ldg(p.seg_offsets + lo + 1) - t.row0);
-  t.hr = lo % p.Hr;
+  t.seg = st.x;
+  t.row0 = __ldg(p.seg_offsets + st.x) + st.y * BM;
+  t.rows = min(BM, __ldg(p.seg_offsets + st.x + 1) - t.row0);
+  t.hr = st.x % p.Hr;
+  t.nt = 0;
   return t;
 }
 
@@ -94,49 +99,52 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
   return __all_sync(0xffffffffu, ok);
 }
 
-// Four rows (y0..y3) x 64 columns from x into shared memory, 128-byte swizzled like a 4-row
-// box of the same tensor map (its box is one row high).
-__device__ __forceinline__ void tma_gather4(void* smem_dst, const CUtensorMap* map, int32_t x, int32_t y0, int32_t y1,
-                                            int32_t y2, int32_t y3, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(smem_u32(smem_dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y0), "r"(y1), "r"(y2), "r"(y3), "r"(smem_u32(bar))
-      : "memory");
+// 16 bytes global -> shared through the L1 path (no registers), completed by wait_group.
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gmem_src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem_dst)), "l"(gmem_src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-// 128-row tiles of each segment, scanned: one block.
-__global__ void __launch_bounds__(1024) tile_prefix_kernel(const int32_t* __restrict__ seg_offsets, int nseg,
-                                                           int32_t* __restrict__ tile_prefix) {
-  __shared__ int s_sum[1024];
-  const int tid = threadIdx.x, nthr = blockDim.x;
-  const int per = (nseg + nthr - 1) / nthr;
-  const int s0 = min(nseg, tid * per), s1 = min(nseg, s0 + per);
-  auto tiles = [&](int s) {
+// The row-tile list in work order (one block).  Sequence b's tiles come before b + 1's; inside
+// a sequence, tile p of every head before tile p + 1 of any, heads in order.  Tile (b, p, h)
+// lands at  (tiles of sequences before b) + sum_h' min(p, n_tiles(b, h')) + #{h' < h : n_tiles(b, h') > p}.
+__global__ void __launch_bounds__(1024) tile_list_kernel(const int32_t* __restrict__ seg_offsets, int nseg, int Hr,
+                                                         int2* __restrict__ tiles, int32_t* __restrict__ ntiles) {
+  extern __shared__ int s_nt[];  // [nseg] tiles per segment, then [nseg / Hr] per-sequence bases
+  int* s_base = s_nt + nseg;
+  const int B = nseg / Hr;
+  const int tid = threadIdx.x;
+  for (int s = tid; s < nseg; s += blockDim.x) {
     const int n = __ldg(seg_offsets + s + 1) - __ldg(seg_offsets + s);
-    return n > 0 ? (n + BM - 1) / BM : 0;
-  };
-  int sum = 0;
-  for (int s = s0; s < s1; ++s) sum += tiles(s);
-  s_sum[tid] = sum;
+    s_nt[s] = n > 0 ? (n + BM - 1) / BM : 0;
+  }
   __syncthreads();
-  for (int off = 1; off < nthr; off <<= 1) {
-    const int add = tid >= off ? s_sum[tid - off] : 0;
-    __syncthreads();
-    s_sum[tid] += add;
-    __syncthreads();
+  if (tid == 0) {
+    int run = 0;
+    for (int b = 0; b < B; ++b) {
+      s_base[b] = run;
+      for (int h = 0; h < Hr; ++h) run += s_nt[b * Hr + h];
+    }
+    *ntiles = run;
   }
-  int run = s_sum[tid] - sum;
-  for (int s = s0; s < s1; ++s) {
-    tile_prefix[s] = run;
-    run += tiles(s);
+  __syncthreads();
+  for (int s = tid; s < nseg; s += blockDim.x) {
+    const int b = s / Hr, h = s - b * Hr;
+    const int* nt = s_nt + b * Hr;
+    for (int q = 0; q < nt[h]; ++q) {
+      int pos = s_base[b];
+      for (int h2 = 0; h2 < Hr; ++h2) pos += min(q, nt[h2]) + (h2 < h && nt[h2] > q ? 1 : 0);
+      tiles[pos] = make_int2(s, q);
+    }
   }
-  if (tid == nthr - 1) tile_prefix[nseg] = s_sum[nthr - 1];
 }
 
 template <int BN, int kMode>
-__global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant__ CUtensorMap tm_a,
-                                                           const __grid_constant__ CUtensorMap tm_b, Params p) {
+__global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant__ CUtensorMap tm_b, Params p) {
   using L = Layout<BN>;
   constexpr int S = L::kStages;
   extern __shared__ uint8_t smem_raw[];
@@ -147,7 +155,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
-      mbar_init(&bars->full[i], 1);
+      mbar_init(&bars->full[i], 129);  // 128 loader threads + the weight tile's expect_tx
       mbar_init(&bars->empty[i], 1);
     }
     for (int i = 0; i < 2; ++i) {
@@ -157,11 +165,8 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     bars->abort_flag = 0;
     mbar_fence_init();
   }
-  if (warp == 4 && lane == 0) {
-    tma_prefetch_desc(&tm_a);
-    tma_prefetch_desc(&tm_b);
-  }
-  if (warp == 5) {
+  if (warp == 4 && lane == 0) tma_prefetch_desc(&tm_b);
+  if (warp == 8) {
     tmem_alloc(&bars->tmem_base, 512);
     tmem_relinquish();
   }
@@ -169,44 +174,98 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars->tmem_base;
-  pdl_wait();  // the routing layout, the tile prefix and the inputs are visible from here
+  pdl_wait();  // the routing layout, the tile list and the inputs are visible from here
 
   const int nt_count = p.ncols / BN;
-  const int nitems = __ldg(p.tile_prefix + p.nseg) * nt_count;
+  const int nitems = __ldg(p.ntiles) * nt_count;
   const int nk = p.kdim / BK;
 
-  if (warp == 4) {
-    // ---- loads
+  if (warp >= 4 && warp < 8) {
+    // ---- loads: thread lt moves 16-byte chunk (lt & 7) of rows (lt >> 3) + 16 w, w = 0..7
+    constexpr int kLag = L::kLag;
+    const int lt = threadIdx.x - 128;
+    const int rq = lt >> 3, ch = lt & 7;
+    const uint16_t* a_base = static_cast<const uint16_t*>(p.a);
+    // row -> the gathered A row (rows past the segment's end load row 0 and are not stored;
+    // indices are clamped into the tensor)
+    auto a_row = [&](const Tile& t, int r) -> int {
+      int row = 0;
+      if (r < t.rows) {
+        const int src = __ldg(p.row_src + t.row0 + r);
+        row = kMode == kQKV ? src / p.Kr : src;
+      }
+      return min(max(row, 0), p.a_rows - 1);
+    };
     uint32_t it = 0;
     bool ok = true;
-    for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x) {
-      const Tile t = decode_item(p, item, nt_count);
-      int c[4];
+    int item = blockIdx.x;
+    Tile t{};
+    int rows_a[8];
+    if (item < nitems) {
+      t = decode_tile(p, __ldg(p.tiles + item / nt_count));
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int r = 4 * lane + e;
-        int row = 0;  // rows past the segment's end load row 0; their outputs are not stored
-        if (r < t.rows) {
-          const int src = __ldg(p.row_src + t.row0 + r);
-          row = kMode == kQKV ? src / p.Kr : src;
-        }
-        c[e] = min(max(row, 0), p.a_rows - 1);
-      }
+      for (int w = 0; w < 8; ++w) rows_a[w] = a_row(t, rq + 16 * w);
+    }
+    const bool prefetch = nk >= 12;
+    for (; item < nitems && ok; item += gridDim.x) {
+      t.nt = item % nt_count;
       const int b_row = t.hr * p.ncols + t.nt * BN;
+      // the next item's tile and rows, fetched over the first k-blocks of this one
+      const int next = item + gridDim.x;
+      int2 nx_st = make_int2(0, 0);
+      Tile nx{};
+      int nx_rows[8];
+      const uint16_t* src[8];
+#pragma unroll
+      for (int w = 0; w < 8; ++w) src[w] = a_base + (size_t)rows_a[w] * p.kdim + ch * 8;
       for (int kb = 0; kb < nk; ++kb, ++it) {
+        if (prefetch && next < nitems) {
+          if (kb == 0) nx_st = __ldg(p.tiles + next / nt_count);
+          if (kb == 4) nx = decode_tile(p, nx_st);
+          if (kb == 8) {
+#pragma unroll
+            for (int w = 0; w < 8; ++w) nx_rows[w] = a_row(nx, rq + 16 * w);
+          }
+        }
         const int slot = it % S;
         if (it >= (uint32_t)S && !warp_wait(&bars->empty[slot], ((it / S) - 1) & 1, abort_flag, p.status)) {
           ok = false;
           break;
         }
         uint8_t* a = smem + slot * L::kStage;
-        if (lane == 0) mbar_arrive_expect_tx(&bars->full[slot], L::kStage);
-        __syncwarp();
-        tma_gather4(a + lane * 512, &tm_a, kb * BK, c[0], c[1], c[2], c[3], &bars->full[slot]);
-        if (lane == 0) tma_load_2d(a + L::kA, &tm_b, kb * BK, b_row, &bars->full[slot]);
+        if (lt == 0) {
+          mbar_arrive_expect_tx(&bars->full[slot], L::kB);
+          tma_load_2d(a + L::kA, &tm_b, kb * BK, b_row, &bars->full[slot]);
+        }
+#pragma unroll
+        for (int w = 0; w < 8; ++w) {
+          const int r = rq + 16 * w;
+          cp_async16(a + r * 128 + ((ch ^ (r & 7)) << 4), src[w] + kb * BK);
+        }
+        cp_async_commit();
+        if (it >= (uint32_t)kLag) {
+          cp_async_wait<kLag>();
+          fence_proxy_async_smem();
+          mbar_arrive(&bars->full[(it - kLag) % S]);
+        }
+      }
+      if (!ok || next >= nitems) break;
+      if (prefetch) {
+        t = nx;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) rows_a[w] = nx_rows[w];
+      } else {
+        t = decode_tile(p, __ldg(p.tiles + next / nt_count));
+#pragma unroll
+        for (int w = 0; w < 8; ++w) rows_a[w] = a_row(t, rq + 16 * w);
       }
     }
-  } else if (warp == 5) {
+    if (ok) {  // retire the last stages
+      cp_async_wait<0>();
+      fence_proxy_async_smem();
+      for (uint32_t j = it > (uint32_t)kLag ? it - kLag : 0; j < it; ++j) mbar_arrive(&bars->full[j % S]);
+    }
+  } else if (warp == 8) {
     // ---- MMA issue
     constexpr uint32_t idesc = make_idesc_bf16(BM, BN, false, false);
     uint32_t it = 0;
@@ -240,7 +299,8 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     const uint32_t lane_addr = (uint32_t)(warp * 32) << 16;
     int li = 0;
     for (int item = blockIdx.x; item < nitems; item += gridDim.x, ++li) {
-      const Tile t = decode_item(p, item, nt_count);
+      Tile t = decode_tile(p, __ldg(p.tiles + item / nt_count));
+      t.nt = item % nt_count;
       const int buf = li & 1;
       const bool valid = row < t.rows;
       const int r = t.row0 + row;
@@ -296,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     }
   }
   __syncthreads();
-  if (warp == 5) {
+  if (warp == 8) {
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
@@ -315,14 +375,13 @@ bool encode_map(CUtensorMap* map, const void* base, long long rows, int cols, in
 }
 
 template <int BN, int kMode>
-cudaError_t launch_bn(const Params& p, const void* a, long long a_rows, const void* b, long long b_rows, int grid,
-                      cudaStream_t stream) {
-  CUtensorMap ta, tb;
-  if (!encode_map(&ta, a, a_rows, p.kdim, 1) || !encode_map(&tb, b, b_rows, p.kdim, BN)) return cudaErrorInvalidValue;
+cudaError_t launch_bn(const Params& p, const void* b, long long b_rows, int grid, cudaStream_t stream) {
+  CUtensorMap tb;
+  if (!encode_map(&tb, b, b_rows, p.kdim, BN)) return cudaErrorInvalidValue;
   const int smem = Layout<BN>::kAlloc;
   cudaError_t e = cudaFuncSetAttribute(proj_kernel<BN, kMode>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  return launch_pdl(proj_kernel<BN, kMode>, dim3(grid), dim3(kThreads), (size_t)smem, stream, ta, tb, p);
+  return launch_pdl(proj_kernel<BN, kMode>, dim3(grid), dim3(kThreads), (size_t)smem, stream, tb, p);
 }
 
 // The widest column tile (multiple of 32, at most 256) that divides the output columns.
@@ -333,15 +392,14 @@ int pick_bn(int ncols) {
 }
 
 template <int kMode>
-cudaError_t launch(int bn, const Params& p, const void* a, long long a_rows, const void* b, long long b_rows,
-                   int grid, cudaStream_t stream) {
+cudaError_t launch(int bn, const Params& p, const void* b, long long b_rows, int grid, cudaStream_t stream) {
   switch (bn) {
-    case 256: return launch_bn<256, kMode>(p, a, a_rows, b, b_rows, grid, stream);
-    case 192: return launch_bn<192, kMode>(p, a, a_rows, b, b_rows, grid, stream);
-    case 160: return launch_bn<160, kMode>(p, a, a_rows, b, b_rows, grid, stream);
-    case 128: return launch_bn<128, kMode>(p, a, a_rows, b, b_rows, grid, stream);
-    case 96: return launch_bn<96, kMode>(p, a, a_rows, b, b_rows, grid, stream);
-    default: return launch_bn<64, kMode>(p, a, a_rows, b, b_rows, grid, stream);
+    case 256: return launch_bn<256, kMode>(p, b, b_rows, grid, stream);
+    case 192: return launch_bn<192, kMode>(p, b, b_rows, grid, stream);
+    case 160: return launch_bn<160, kMode>(p, b, b_rows, grid, stream);
+    case 128: return launch_bn<128, kMode>(p, b, b_rows, grid, stream);
+    case 96: return launch_bn<96, kMode>(p, b, b_rows, grid, stream);
+    default: return launch_bn<64, kMode>(p, b, b_rows, grid, stream);
   }
 }
 
@@ -351,6 +409,8 @@ int check_common(int B, int total_tokens, int d_model, int H, int K, int d_head,
     return NAMOH_ERR_INVALID_ARG;
   if (H / group > NAMOH_MAX_HEADS || (long long)B * (H / group) >= (1ll << 24)) return NAMOH_ERR_INVALID_ARG;
   if ((d_head != 64 && d_head != 128) || (group & (group - 1)) || group > 8) return NAMOH_ERR_UNSUPPORTED;
+  // the list builder keeps B*Hr + B ints in shared memory
+  if (((long long)B * (H / group) + B) * 4 > kMaxTileListBytes) return NAMOH_ERR_UNSUPPORTED;
   if (d_model < BK || d_model % BK || d_model > (1 << 16)) return NAMOH_ERR_UNSUPPORTED;
   *Hr = H / group;
   *Kr = K / group;
@@ -364,21 +424,35 @@ int check_common(int B, int total_tokens, int d_model, int H, int K, int d_head,
 
 using namespace namoh;
 
-extern "C" size_t namoh_proj_workspace_size(int B, int H, int K, int group) {
-  if (B < 1 || group < 1 || H < 1 || K < 1 || H % group) return 0;
-  return align_up((size_t)(B * (H / group) + 1) * sizeof(int32_t), 256);
+namespace {
+// The row-tile list: at most ceil(R / 128) + nseg tiles, plus its length.
+size_t tile_list_bytes(long long R, int nseg) {
+  return 16 + (size_t)((R + proj::BM - 1) / proj::BM + nseg) * sizeof(int2);
 }
 
-namespace {
-int proj_prologue(const int32_t* seg_offsets, int nseg, void* workspace, size_t workspace_bytes, int32_t** prefix,
-                  cudaStream_t stream) {
+int proj_prologue(const int32_t* seg_offsets, int nseg, int Hr, long long R, void* workspace, size_t workspace_bytes,
+                  proj::Params* p, cudaStream_t stream) {
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return NAMOH_ERR_WORKSPACE;
-  if (workspace_bytes < (size_t)(nseg + 1) * sizeof(int32_t)) return NAMOH_ERR_WORKSPACE;
-  *prefix = static_cast<int32_t*>(workspace);
-  proj::tile_prefix_kernel<<<1, 1024, 0, stream>>>(seg_offsets, nseg, *prefix);
-  return cuda_check_launch("tile_prefix_kernel launch");
+  if (workspace_bytes < tile_list_bytes(R, nseg)) return NAMOH_ERR_WORKSPACE;
+  int32_t* ntiles = static_cast<int32_t*>(workspace);
+  int2* tiles = reinterpret_cast<int2*>(static_cast<char*>(workspace) + 16);
+  const int smem = (nseg + nseg / Hr) * (int)sizeof(int);
+  if (smem > 48 * 1024) {
+    const cudaError_t e =
+        cudaFuncSetAttribute(proj::tile_list_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return cuda_fail(e, "tile_list_kernel shared memory attribute");
+  }
+  proj::tile_list_kernel<<<1, 1024, smem, stream>>>(seg_offsets, nseg, Hr, tiles, ntiles);
+  p->tiles = tiles;
+  p->ntiles = ntiles;
+  return cuda_check_launch("tile_list_kernel launch");
 }
 }  // namespace
+
+extern "C" size_t namoh_proj_workspace_size(int B, int total_tokens, int H, int K, int group) {
+  if (B < 1 || total_tokens < 1 || group < 1 || H < 1 || K < 1 || H % group || K % group) return 0;
+  return align_up(tile_list_bytes((long long)total_tokens * (K / group), B * (H / group)), 256);
+}
 
 extern "C" int namoh_proj_qkv(const uint16_t* x, int total_tokens, int d_model, const uint16_t* w_qkv, int B, int H,
                               int K, int d_head, int group, const int32_t* seg_offsets, const int32_t* row_src,
@@ -396,16 +470,15 @@ extern "C" int namoh_proj_qkv(const uint16_t* x, int total_tokens, int d_model, 
   if (!current_device_info(&info) || info.major != 10) return NAMOH_ERR_UNSUPPORTED;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
   const int nseg = B * Hr;
-  int32_t* prefix = nullptr;
-  st = proj_prologue(seg_offsets, nseg, workspace, workspace_bytes, &prefix, stream);
-  if (st != NAMOH_OK) return st;
   proj::Params p{};
+  st = proj_prologue(seg_offsets, nseg, Hr, (long long)total_tokens * Kr, workspace, workspace_bytes, &p, stream);
+  if (st != NAMOH_OK) return st;
   p.seg_offsets = seg_offsets;
-  p.tile_prefix = prefix;
   p.row_src = row_src;
   p.nseg = nseg;
   p.Hr = Hr;
   p.Kr = Kr;
+  p.a = x;
   p.a_rows = total_tokens;
   p.kdim = d_model;
   p.ncols = ncols;
@@ -418,8 +491,7 @@ extern "C" int namoh_proj_qkv(const uint16_t* x, int total_tokens, int d_model, 
   p.out_aligned32 = ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k) |
                       reinterpret_cast<uintptr_t>(v)) & 31u) == 0;
   p.status = dev_status;
-  const cudaError_t e = proj::launch<proj::kQKV>(bn, p, x, total_tokens, w_qkv, (long long)Hr * ncols,
-                                                 info.sm_count, stream);
+  const cudaError_t e = proj::launch<proj::kQKV>(bn, p, w_qkv, (long long)Hr * ncols, info.sm_count, stream);
   return e == cudaSuccess ? NAMOH_OK : cuda_fail(e, "proj_kernel (qkv) launch");
 }
 
@@ -442,16 +514,15 @@ extern "C" int namoh_proj_out(const uint16_t* y, int total_tokens, int d_model, 
     if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync of o");
   }
   const int nseg = B * Hr;
-  int32_t* prefix = nullptr;
-  st = proj_prologue(seg_offsets, nseg, workspace, workspace_bytes, &prefix, stream);
-  if (st != NAMOH_OK) return st;
   proj::Params p{};
+  st = proj_prologue(seg_offsets, nseg, Hr, (long long)total_tokens * Kr, workspace, workspace_bytes, &p, stream);
+  if (st != NAMOH_OK) return st;
   p.seg_offsets = seg_offsets;
-  p.tile_prefix = prefix;
   p.row_src = row_src;
   p.nseg = nseg;
   p.Hr = Hr;
   p.Kr = Kr;
+  p.a = y;
   p.a_rows = total_tokens * Kr;
   p.kdim = group * d_head;
   p.ncols = d_model;
@@ -460,7 +531,6 @@ extern "C" int namoh_proj_out(const uint16_t* y, int total_tokens, int d_model, 
   p.o = o;
   p.ntok = total_tokens;
   p.status = dev_status;
-  const cudaError_t e = proj::launch<proj::kOut>(bn, p, y, (long long)total_tokens * Kr, w_o, (long long)Hr * d_model,
-                                                 info.sm_count, stream);
+  const cudaError_t e = proj::launch<proj::kOut>(bn, p, w_o, (long long)Hr * d_model, info.sm_count, stream);
   return e == cudaSuccess ? NAMOH_OK : cuda_fail(e, "proj_kernel (out) launch");
 }
