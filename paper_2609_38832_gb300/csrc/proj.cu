@@ -1,18 +1,14 @@
-// proj.cu -- the projections around the routed-attention path (Sec. 3.1).
+// proj.cu -- the QKV projection (Sec. 3.1, Eq. namoh-qkv) and the entry points of both
+// projections (the output projection's kernels are in proj_out.cu).
 //
-// Both are grouped GEMMs over the packed rows of the routing (one group per KV-group head i,
-// App. C), with the A rows gathered from the token axis:
-//   QKV (Eq. namoh-qkv):  row r of segment (b, i) computes x_t [W_Q^(ig..ig+g-1) | W_K^(i) | W_V^(i)]
-//                         for t = row_src[r] / Kr, written as g query rows, one key row and one
-//                         value row in packed order -- the inputs of namoh_prefill.
-//   OUT (Eq. namoh-attention, o_t = sum_i g h W_O^(i)): row r computes y_r [W_O^(ig); ...;
-//                         W_O^(ig+g-1)] from the combine's per-slot terms y = g h and adds it
-//                         into o[t] (fp32): the token's K slots sum there.
-// Only active token-head pairs are computed (Sec. 3.1: inactive pairs generate nothing).
+// A grouped GEMM over the packed rows of the routing (one group per KV-group head i, App. C),
+// with the A rows gathered from the token axis: row r of segment (b, i) computes
+// x_t [W_Q^(ig..ig+g-1) | W_K^(i) | W_V^(i)] for t = row_src[r] / Kr, written as g query rows,
+// one key row and one value row in packed order -- the inputs of namoh_prefill.  Only active
+// token-head pairs are computed (Sec. 3.1: inactive pairs generate nothing).
 //
 // One persistent CTA per SM, 288 threads:
-//   warps 0-3  epilogue: TMEM lane = tile row; fp32 accumulators -> bf16 rows (QKV) or fp32
-//              reductions into o (OUT)
+//   warps 0-3  epilogue: TMEM lane = tile row; fp32 accumulators -> bf16 q, k, v rows
 //   warps 4-7  loads: per 64-wide slice of the contraction the 128 gathered A rows arrive by
 //              16-byte cp.async copies (a warp moves four whole 128-byte rows per instruction)
 //              into the 128-byte-swizzled layout, and one TMA tile copy brings the group's
@@ -23,7 +19,7 @@
 //   warp 8     TMEM owner and MMA issue: tcgen05.mma kind::f16, M = 128, N = BN, K = 16
 // Work items are (128-row tile of a segment, BN-column tile) from a list ordered by sequence,
 // then position in the segment, then head: CTAs running at the same time work on the same
-// stretch of tokens across heads, so x rows (QKV) and o rows (OUT) are reused from L2, and
+// stretch of tokens across heads, so x rows are reused from L2, and
 // the N tiles of one row tile are adjacent items.  A static round robin hands out the items;
 // the loaders fetch the next item's row indices during the current one.
 // Two TMEM accumulators let the epilogue of one item overlap the main loop of the next.
@@ -39,7 +35,6 @@ constexpr int kThreads = 288;
 constexpr int kSmemBudget = 208 * 1024;
 constexpr int kMaxTileListBytes = 200 * 1024;  // shared memory of the tile-list builder
 
-enum Mode { kQKV = 0, kOut = 1 };
 
 template <int BN>
 struct Layout {
@@ -60,14 +55,12 @@ struct Params {
   const int32_t* ntiles;       // [1]: length of the list
   const int32_t* row_src;      // [R]
   int nseg, Hr, Kr;
-  int a_rows;                  // rows of the gathered tensor (tokens for QKV, token slots for OUT)
-  int kdim;                    // contraction length: d_model (QKV) or g d (OUT)
-  int ncols;                   // output columns per group: (g + 2) d (QKV) or d_model (OUT)
+  int a_rows;                  // tokens (rows of x)
+  int kdim;                    // contraction length: d_model
+  int ncols;                   // output columns per group: (g + 2) d
   int g, d;
-  const void* a;               // the gathered tensor: x [a_rows, kdim] (QKV) or y (OUT)
-  uint16_t *q, *k, *v;         // QKV outputs
-  float* o;                    // OUT output [ntok, d_model]
-  int ntok;
+  const void* a;               // x [a_rows, kdim]
+  uint16_t *q, *k, *v;         // outputs
   int out_aligned32;           // q, k, v 32-byte aligned: whole-sector stores
   uint32_t* status;
 };
@@ -143,7 +136,7 @@ __global__ void __launch_bounds__(1024) tile_list_kernel(const int32_t* __restri
   }
 }
 
-template <int BN, int kMode>
+template <int BN>
 __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant__ CUtensorMap tm_b, Params p) {
   using L = Layout<BN>;
   constexpr int S = L::kStages;
@@ -190,10 +183,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     // indices are clamped into the tensor)
     auto a_row = [&](const Tile& t, int r) -> int {
       int row = 0;
-      if (r < t.rows) {
-        const int src = __ldg(p.row_src + t.row0 + r);
-        row = kMode == kQKV ? src / p.Kr : src;
-      }
+      if (r < t.rows) row = ld_issue_s32(p.row_src + t.row0 + r) / p.Kr;
       return min(max(row, 0), p.a_rows - 1);
     };
     uint32_t it = 0;
@@ -210,21 +200,34 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     for (; item < nitems && ok; item += gridDim.x) {
       t.nt = item % nt_count;
       const int b_row = t.hr * p.ncols + t.nt * BN;
-      // the next item's tile and rows, fetched over the first k-blocks of this one
+      // the next item's tile and rows, fetched over the first k-blocks of this one, each load
+      // issued four k-blocks before its value is used
       const int next = item + gridDim.x;
-      int2 nx_st = make_int2(0, 0);
+      int nx_seg = 0, nx_q = 0, nx_lo = 0, nx_hi = 0;
       Tile nx{};
-      int nx_rows[8];
+      int nx_src[8];
       const uint16_t* src[8];
 #pragma unroll
       for (int w = 0; w < 8; ++w) src[w] = a_base + (size_t)rows_a[w] * p.kdim + ch * 8;
       for (int kb = 0; kb < nk; ++kb, ++it) {
         if (prefetch && next < nitems) {
-          if (kb == 0) nx_st = __ldg(p.tiles + next / nt_count);
-          if (kb == 4) nx = decode_tile(p, nx_st);
-          if (kb == 8) {
+          if (kb == 0) {
+            const int32_t* e = reinterpret_cast<const int32_t*>(p.tiles + next / nt_count);
+            nx_seg = ld_issue_s32(e);
+            nx_q = ld_issue_s32(e + 1);
+          } else if (kb == 4) {
+            nx_lo = ld_issue_s32(p.seg_offsets + nx_seg);
+            nx_hi = ld_issue_s32(p.seg_offsets + nx_seg + 1);
+          } else if (kb == 8) {
+            nx.seg = nx_seg;
+            nx.row0 = nx_lo + nx_q * BM;
+            nx.rows = min(BM, nx_hi - nx.row0);
+            nx.hr = nx_seg % p.Hr;
 #pragma unroll
-            for (int w = 0; w < 8; ++w) nx_rows[w] = a_row(nx, rq + 16 * w);
+            for (int w = 0; w < 8; ++w) {
+              const int r = rq + 16 * w;
+              nx_src[w] = r < nx.rows ? ld_issue_s32(p.row_src + nx.row0 + r) : 0;
+            }
           }
         }
         const int slot = it % S;
@@ -253,7 +256,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
       if (prefetch) {
         t = nx;
 #pragma unroll
-        for (int w = 0; w < 8; ++w) rows_a[w] = nx_rows[w];
+        for (int w = 0; w < 8; ++w) rows_a[w] = min(max(nx_src[w] / p.Kr, 0), p.a_rows - 1);
       } else {
         t = decode_tile(p, __ldg(p.tiles + next / nt_count));
 #pragma unroll
@@ -304,7 +307,6 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
       const int buf = li & 1;
       const bool valid = row < t.rows;
       const int r = t.row0 + row;
-      int src = valid ? __ldg(p.row_src + r) : 0;
       if (!warp_wait(&bars->acc_full[buf], (li >> 1) & 1, abort_flag, p.status)) break;
       tc_fence_after();
 #pragma unroll 1
@@ -314,31 +316,21 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
         tmem_wait_ld();
         if (!valid) continue;
         const int n = t.nt * BN + c * 32;  // first output column of the chunk
-        if constexpr (kMode == kQKV) {
-          uint16_t* dst;
-          const int gd = p.g * p.d;
-          if (n < gd) dst = p.q + ((long long)r * p.g + n / p.d) * p.d + n % p.d;
-          else if (n < gd + p.d) dst = p.k + (long long)r * p.d + (n - gd);
-          else dst = p.v + (long long)r * p.d + (n - gd - p.d);
-          uint32_t w[16];
+        uint16_t* dst;
+        const int gd = p.g * p.d;
+        if (n < gd) dst = p.q + ((long long)r * p.g + n / p.d) * p.d + n % p.d;
+        else if (n < gd + p.d) dst = p.k + (long long)r * p.d + (n - gd);
+        else dst = p.v + (long long)r * p.d + (n - gd - p.d);
+        uint32_t w[16];
 #pragma unroll
-          for (int e = 0; e < 16; ++e) w[e] = pack_bf16x2(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
-          if (p.out_aligned32) {
-            st_global_v8(dst, w);
-            st_global_v8(dst + 16, w + 8);
-          } else {
-            uint4* d4 = reinterpret_cast<uint4*>(dst);
-#pragma unroll
-            for (int e = 0; e < 4; ++e) d4[e] = make_uint4(w[4 * e], w[4 * e + 1], w[4 * e + 2], w[4 * e + 3]);
-          }
+        for (int e = 0; e < 16; ++e) w[e] = pack_bf16x2(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
+        if (p.out_aligned32) {
+          st_global_v8(dst, w);
+          st_global_v8(dst + 16, w + 8);
         } else {
-          const int tok = src / p.Kr;
-          if (tok < 0 || tok >= p.ntok) continue;  // an inconsistent layout: nothing outside o
-          float4* dst = reinterpret_cast<float4*>(p.o + (long long)tok * p.ncols + n);
+          uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
-          for (int e = 0; e < 8; ++e)
-            atomicAdd(dst + e, make_float4(__uint_as_float(v[4 * e]), __uint_as_float(v[4 * e + 1]),
-                                           __uint_as_float(v[4 * e + 2]), __uint_as_float(v[4 * e + 3])));
+          for (int e = 0; e < 4; ++e) d4[e] = make_uint4(w[4 * e], w[4 * e + 1], w[4 * e + 2], w[4 * e + 3]);
         }
       }
       tc_fence_before();
@@ -374,14 +366,14 @@ bool encode_map(CUtensorMap* map, const void* base, long long rows, int cols, in
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, int kMode>
+template <int BN>
 cudaError_t launch_bn(const Params& p, const void* b, long long b_rows, int grid, cudaStream_t stream) {
   CUtensorMap tb;
   if (!encode_map(&tb, b, b_rows, p.kdim, BN)) return cudaErrorInvalidValue;
   const int smem = Layout<BN>::kAlloc;
-  cudaError_t e = cudaFuncSetAttribute(proj_kernel<BN, kMode>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaError_t e = cudaFuncSetAttribute(proj_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  return launch_pdl(proj_kernel<BN, kMode>, dim3(grid), dim3(kThreads), (size_t)smem, stream, tb, p);
+  return launch_pdl(proj_kernel<BN>, dim3(grid), dim3(kThreads), (size_t)smem, stream, tb, p);
 }
 
 // The widest column tile (multiple of 32, at most 256) that divides the output columns.
@@ -391,15 +383,14 @@ int pick_bn(int ncols) {
   return 0;
 }
 
-template <int kMode>
 cudaError_t launch(int bn, const Params& p, const void* b, long long b_rows, int grid, cudaStream_t stream) {
   switch (bn) {
-    case 256: return launch_bn<256, kMode>(p, b, b_rows, grid, stream);
-    case 192: return launch_bn<192, kMode>(p, b, b_rows, grid, stream);
-    case 160: return launch_bn<160, kMode>(p, b, b_rows, grid, stream);
-    case 128: return launch_bn<128, kMode>(p, b, b_rows, grid, stream);
-    case 96: return launch_bn<96, kMode>(p, b, b_rows, grid, stream);
-    default: return launch_bn<64, kMode>(p, b, b_rows, grid, stream);
+    case 256: return launch_bn<256>(p, b, b_rows, grid, stream);
+    case 192: return launch_bn<192>(p, b, b_rows, grid, stream);
+    case 160: return launch_bn<160>(p, b, b_rows, grid, stream);
+    case 128: return launch_bn<128>(p, b, b_rows, grid, stream);
+    case 96: return launch_bn<96>(p, b, b_rows, grid, stream);
+    default: return launch_bn<64>(p, b, b_rows, grid, stream);
   }
 }
 
@@ -423,6 +414,13 @@ int check_common(int B, int total_tokens, int d_model, int H, int K, int d_head,
 }  // namespace namoh
 
 using namespace namoh;
+
+namespace namoh {  // the output projection, in proj_out.cu
+size_t proj_out_workspace(long long total_tokens, int Kr, int gd, int nseg);
+int launch_proj_out(const uint16_t* y, int total_tokens, int d_model, const uint16_t* w_o, int Hr, int Kr, int gd,
+                    int nseg, const int32_t* seg_offsets, const int32_t* row_src, float* o, int accumulate,
+                    void* workspace, size_t workspace_bytes, uint32_t* dev_status, int sm_count, cudaStream_t stream);
+}  // namespace namoh
 
 namespace {
 // The row-tile list: at most ceil(R / 128) + nseg tiles, plus its length.
@@ -449,9 +447,12 @@ int proj_prologue(const int32_t* seg_offsets, int nseg, int Hr, long long R, voi
 }
 }  // namespace
 
-extern "C" size_t namoh_proj_workspace_size(int B, int total_tokens, int H, int K, int group) {
-  if (B < 1 || total_tokens < 1 || group < 1 || H < 1 || K < 1 || H % group || K % group) return 0;
-  return align_up(tile_list_bytes((long long)total_tokens * (K / group), B * (H / group)), 256);
+extern "C" size_t namoh_proj_workspace_size(int B, int total_tokens, int H, int K, int d_head, int group) {
+  if (B < 1 || total_tokens < 1 || group < 1 || H < 1 || K < 1 || H % group || K % group || d_head < 1) return 0;
+  const int Hr = H / group, Kr = K / group;
+  const size_t qkv = align_up(tile_list_bytes((long long)total_tokens * Kr, B * Hr), 256);
+  const size_t out = proj_out_workspace(total_tokens, Kr, group * d_head, B * Hr);
+  return qkv > out ? qkv : out;
 }
 
 extern "C" int namoh_proj_qkv(const uint16_t* x, int total_tokens, int d_model, const uint16_t* w_qkv, int B, int H,
@@ -487,11 +488,10 @@ extern "C" int namoh_proj_qkv(const uint16_t* x, int total_tokens, int d_model, 
   p.q = q;
   p.k = k;
   p.v = v;
-  p.ntok = total_tokens;
   p.out_aligned32 = ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k) |
                       reinterpret_cast<uintptr_t>(v)) & 31u) == 0;
   p.status = dev_status;
-  const cudaError_t e = proj::launch<proj::kQKV>(bn, p, w_qkv, (long long)Hr * ncols, info.sm_count, stream);
+  const cudaError_t e = proj::launch(bn, p, w_qkv, (long long)Hr * ncols, info.sm_count, stream);
   return e == cudaSuccess ? NAMOH_OK : cuda_fail(e, "proj_kernel (qkv) launch");
 }
 
@@ -501,36 +501,12 @@ extern "C" int namoh_proj_out(const uint16_t* y, int total_tokens, int d_model, 
                               void* stream_v) {
   if (!y || !w_o || !seg_offsets || !row_src || !o || !dev_status) return NAMOH_ERR_INVALID_ARG;
   int Hr, Kr;
-  int st = proj::check_common(B, total_tokens, d_model, H, K, d_head, group, &Hr, &Kr);
+  const int st = proj::check_common(B, total_tokens, d_model, H, K, d_head, group, &Hr, &Kr);
   if (st != NAMOH_OK) return st;
   if (!aligned16(y) || !aligned16(w_o) || !aligned16(o)) return NAMOH_ERR_INVALID_ARG;
-  const int bn = proj::pick_bn(d_model);
-  if (bn == 0) return NAMOH_ERR_UNSUPPORTED;
   DeviceInfo info;
   if (!current_device_info(&info) || info.major != 10) return NAMOH_ERR_UNSUPPORTED;
-  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
-  if (!accumulate) {
-    const cudaError_t e = cudaMemsetAsync(o, 0, (size_t)total_tokens * d_model * sizeof(float), stream);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync of o");
-  }
-  const int nseg = B * Hr;
-  proj::Params p{};
-  st = proj_prologue(seg_offsets, nseg, Hr, (long long)total_tokens * Kr, workspace, workspace_bytes, &p, stream);
-  if (st != NAMOH_OK) return st;
-  p.seg_offsets = seg_offsets;
-  p.row_src = row_src;
-  p.nseg = nseg;
-  p.Hr = Hr;
-  p.Kr = Kr;
-  p.a = y;
-  p.a_rows = total_tokens * Kr;
-  p.kdim = group * d_head;
-  p.ncols = d_model;
-  p.g = group;
-  p.d = d_head;
-  p.o = o;
-  p.ntok = total_tokens;
-  p.status = dev_status;
-  const cudaError_t e = proj::launch<proj::kOut>(bn, p, w_o, (long long)Hr * d_model, info.sm_count, stream);
-  return e == cudaSuccess ? NAMOH_OK : cuda_fail(e, "proj_kernel (out) launch");
+  return launch_proj_out(y, total_tokens, d_model, w_o, Hr, Kr, group * d_head, B * Hr, seg_offsets, row_src, o,
+                         accumulate ? 1 : 0, workspace, workspace_bytes, dev_status, info.sm_count,
+                         reinterpret_cast<cudaStream_t>(stream_v));
 }
