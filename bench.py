@@ -395,9 +395,101 @@ def run_gpu(args, rank: int, world: int):
     if not args.no_decode:
         line["decode"] = run_decode(args, dev, pk, pk_kind)
         line["gpu_launches"] += line["decode"].pop("launches")
+    if not args.no_layer:
+        line["layer"] = run_layer(args, dev, pk, pk_kind)
+        line["gpu_launches"] += line["layer"].pop("launches")
     clocks.__exit__(None, None, None)
     line["clocks"] = clocks.summary()
     return line
+
+
+LAYER_D_MODEL = 2048  # the paper's model width (its experiments fix 2048)
+
+
+def run_layer(args, dev, pk, pk_kind):
+    """The balanced workload as a whole attention layer at d_model = 2048: the sparse QKV
+    projection (Eq. namoh-qkv), routing, RoPE + routed attention + combine, and the output
+    projection (Eq. namoh-attention), random bf16 weights.  Each stage and the whole step are
+    timed with the L2 flushed before every timed launch sequence."""
+    import torch
+
+    import paper_2609_38832_gb300 as namoh
+
+    wl = ni.BALANCED
+    B, T, H, K, d, g = wl.B, wl.T, wl.H, wl.K, wl.d, wl.g
+    Hr, Kr = H // g, K // g
+    d_model = LAYER_D_MODEL
+    N, R = B * T, B * T * Kr
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(wl.seed)
+    x = torch.randn((N, d_model), generator=gen, device=dev).to(torch.bfloat16)
+    w_qkv = (torch.randn((Hr, (g + 2) * d, d_model), generator=gen, device=dev) / d_model ** 0.5).to(torch.bfloat16)
+    w_o = (torch.randn((Hr, d_model, g * d), generator=gen, device=dev) / (g * d) ** 0.5).to(torch.bfloat16)
+    scores = torch.from_numpy(wl.scores()).to(dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    ws_r, ws_p, ws_l = namoh.Workspace(), namoh.Workspace(), namoh.Workspace()
+    ro = namoh.namoh_route(scores, Kr, workspace=ws_r, status=status)
+    q = torch.empty((R * g, d), dtype=torch.bfloat16, device=dev)
+    k = torch.empty((R, d), dtype=torch.bfloat16, device=dev)
+    v = torch.empty((R, d), dtype=torch.bfloat16, device=dev)
+    k_cache = torch.empty_like(k)
+    y = torch.empty((B, T, K, d), dtype=torch.bfloat16, device=dev)
+    o = torch.empty((N, d_model), dtype=torch.float32, device=dev)
+    flush = torch.empty(2 << 30, dtype=torch.uint8, device=dev)
+
+    def qkv():
+        namoh.namoh_proj_qkv(x, w_qkv, ro.seg_offsets, ro.row_src, B=B, H=H, K=K, group=g, q=q, k=k, v=v,
+                             workspace=ws_l, status=status)
+
+    def out():
+        namoh.namoh_proj_out(y, w_o, ro.seg_offsets, ro.row_src, B=B, H=H, K=K, group=g, o=o, workspace=ws_l,
+                             status=status)
+
+    def step():
+        namoh.namoh_route(scores, Kr, workspace=ws_r, status=status, out=ro)
+        qkv()
+        namoh.namoh_prefill(q, k, v, ro.seg_offsets, ro.row_src, ro.gate, B=B, T=T, H=H, K=K, group=g,
+                            rope_base=wl.base, y=y, k_cache=k_cache, workspace=ws_p, status=status)
+        out()
+
+    def timed(fn):
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+        for i in range(args.warmup + args.steps):
+            flush.fill_(i & 0xFF)
+            if i >= args.warmup:
+                evs[i - args.warmup][0].record()
+            fn()
+            if i >= args.warmup:
+                evs[i - args.warmup][1].record()
+        torch.cuda.synchronize()
+        return float(np.mean([a.elapsed_time(b) for a, b in evs]))
+
+    step()
+    torch.cuda.synchronize()
+    n_seg = acc.segment_lengths(ro.seg_offsets.cpu().numpy())
+    f_attn = acc.attention_flops(n_seg, d, g)
+    f_qkv = 2.0 * R * d_model * (g + 2) * d
+    f_out = 2.0 * R * g * d * d_model
+    ms_qkv, ms_out, ms_step = timed(qkv), timed(out), timed(step)
+    peak = pk["bf16_tflops"]
+    tf = lambda f, ms: f / (ms * 1e-3) / 1e12  # noqa: E731
+    return {
+        "workload": f"{wl.name} with d_model={d_model}, random bf16 weights",
+        "qkv_projection": {"ms": ms_qkv, "tflops": tf(f_qkv, ms_qkv), "frac_bf16": tf(f_qkv, ms_qkv) / peak,
+                           "flops": f_qkv, "kernel": "proj_kernel (tcgen05, rows gathered by cp.async)"},
+        "out_projection": {"ms": ms_out, "tflops": tf(f_out, ms_out), "frac_bf16": tf(f_out, ms_out) / peak,
+                           "flops": f_out, "kernel": "proj_out_kernel (token windows, fp32 o written once)"},
+        "layer_step": {"ms": ms_step, "tflops": tf(f_qkv + f_attn + f_out, ms_step),
+                       "frac_bf16": tf(f_qkv + f_attn + f_out, ms_step) / peak,
+                       "flops": f_qkv + f_attn + f_out,
+                       "stages": "route, QKV projection, RoPE + attention + combine, output projection"},
+        "peak_source": f"{pk_kind} bf16 dense (burst)",
+        "l2": "flushed before every timed launch sequence (2 GB write)",
+        "device_status": int(status.item()),
+        # timed launches: QKV (tile list + GEMM), OUT (pack, table, bounds, GEMM), and the step
+        # (route 2 + QKV 2 + prefill 2 + OUT 4)
+        "launches": args.steps * (2 + 4 + 10),
+    }
 
 
 def run_decode(args, dev, pk, pk_kind):
@@ -534,6 +626,7 @@ def main():
     ap.add_argument("--impl", choices=["namoh", "reference"], default="namoh")
     ap.add_argument("--decode-steps", type=int, default=64)
     ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-layer", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
