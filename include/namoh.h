@@ -356,17 +356,18 @@ NAMOH_API int namoh_decode_ex(const int32_t *topk_head, const float *gate, const
  *   w_o    [Hr, d_model, g d] bf16, one block per group: row m holds column m of W_O of the
  *          group's query heads one after the other (W_O^(i g + j) row c at column j d + c).
  *   o      [total_tokens, d_model] fp32 out; accumulate = 0 overwrites it, 1 adds to it
- *          (e.g. onto a residual).  Each o element is written once: the work is cut into
- *          windows of 256 tokens whose K slots meet in one CTA; a token's slots are summed in
- *          segment order, so the result is deterministic.
- * Workspace: namoh_proj_workspace_size (one size for both calls: the list of 128-row tiles
- * of the segments, or the packed copy of y and the window tables).
+ *          (e.g. onto a residual).  Two passes: each packed row's product with its group's
+ *          W_O is rounded to bf16 into the workspace at its token-slot row, then each token's K
+ *          rows are summed in slot order in fp32 (deterministic, no atomics).
+ * Workspace: namoh_proj_workspace_size (one size serves both calls: the list of 128-row
+ * tiles of the segments, plus the per-slot products of the output projection,
+ * total_tokens*K/g*d_model bf16).
  * Supports d_head in {64, 128}, g in {1, 2, 4, 8}, d_model a multiple of 64 up to 65536, and
  * B*(H/g + 1) <= 51200.
  * x, w, q, k, v, y, o 16-byte aligned.  Rows of an inconsistent layout (a malformed
  * cu_seqlens) are computed from clamped indices and write nothing outside the outputs.
  * ------------------------------------------------------------------------- */
-NAMOH_API size_t namoh_proj_workspace_size(int B, int total_tokens, int H, int K, int d_head, int group);
+NAMOH_API size_t namoh_proj_workspace_size(int B, int total_tokens, int d_model, int H, int K, int group);
 NAMOH_API int namoh_proj_qkv(const uint16_t *x, int total_tokens, int d_model, const uint16_t *w_qkv, int B, int H,
                              int K, int d_head, int group, const int32_t *seg_offsets, const int32_t *row_src,
                              uint16_t *q, uint16_t *k, uint16_t *v, void *workspace, size_t workspace_bytes,

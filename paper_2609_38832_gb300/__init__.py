@@ -316,7 +316,7 @@ def namoh_proj_qkv(x: torch.Tensor, w_qkv: torch.Tensor, seg_offsets: torch.Tens
     q = torch.empty((R * group, d), dtype=torch.bfloat16, device=dev) if q is None else q
     k = torch.empty((R, d), dtype=torch.bfloat16, device=dev) if k is None else k
     v = torch.empty((R, d), dtype=torch.bfloat16, device=dev) if v is None else v
-    ws = _ws(workspace, lib.namoh_proj_workspace_size(B, N, H, K, d, group), dev)
+    ws = _ws(workspace, lib.namoh_proj_workspace_size(B, N, d_model, H, K, group), dev)
     st = _status(status, dev)
     rc = lib.namoh_proj_qkv(_ptr(x), N, d_model, _ptr(w_qkv), B, H, K, d, group, _ptr(seg_offsets), _ptr(row_src),
                             _ptr(q), _ptr(k), _ptr(v), _ptr(ws), ws.numel(), _ptr(st), _stream(stream))
@@ -344,7 +344,7 @@ def namoh_proj_out(y: torch.Tensor, w_o: torch.Tensor, seg_offsets: torch.Tensor
     if o is None:
         o = torch.empty((N, d_model), dtype=torch.float32, device=dev)
         accumulate = False
-    ws = _ws(workspace, lib.namoh_proj_workspace_size(B, N, H, K, d, group), dev)
+    ws = _ws(workspace, lib.namoh_proj_workspace_size(B, N, d_model, H, K, group), dev)
     st = _status(status, dev)
     rc = lib.namoh_proj_out(_ptr(y), N, d_model, _ptr(w_o), B, H, K, d, group, _ptr(seg_offsets), _ptr(row_src),
                             _ptr(o), 1 if accumulate else 0, _ptr(ws), ws.numel(), _ptr(st), _stream(stream))

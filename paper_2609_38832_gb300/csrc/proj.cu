@@ -1,11 +1,15 @@
-// proj.cu -- the QKV projection (Sec. 3.1, Eq. namoh-qkv) and the entry points of both
-// projections (the output projection's kernels are in proj_out.cu).
+// proj.cu -- the projections around the routed-attention path (Sec. 3.1).
 //
-// A grouped GEMM over the packed rows of the routing (one group per KV-group head i, App. C),
-// with the A rows gathered from the token axis: row r of segment (b, i) computes
-// x_t [W_Q^(ig..ig+g-1) | W_K^(i) | W_V^(i)] for t = row_src[r] / Kr, written as g query rows,
-// one key row and one value row in packed order -- the inputs of namoh_prefill.  Only active
-// token-head pairs are computed (Sec. 3.1: inactive pairs generate nothing).
+// One grouped GEMM over the packed rows of the routing (one group per KV-group head i, App. C),
+// the A rows gathered from the token axis, in two modes:
+//   QKV   (Eq. namoh-qkv): row r of segment (b, i) computes x_t [W_Q^(ig..ig+g-1) | W_K^(i) |
+//         W_V^(i)] for t = row_src[r] / Kr, written as g query rows, one key row and one value
+//         row in packed order -- the inputs of namoh_prefill.
+//   OUT_P (Eq. namoh-attention): row r computes P_r = y_r [W_O^(ig); ...; W_O^(ig+g-1)] from
+//         the combine's per-slot terms y = g h (A row = y[row_src[r]]), written (bf16) at the
+//         token-slot row row_src[r]; combine_kernel then sums each token's K adjacent P rows
+//         into o in fp32.
+// Only active token-head pairs are computed (Sec. 3.1: inactive pairs generate nothing).
 //
 // One persistent CTA per SM, 288 threads:
 //   warps 0-3  epilogue: TMEM lane = tile row; fp32 accumulators -> bf16 q, k, v rows
@@ -59,8 +63,8 @@ struct Params {
   int kdim;                    // contraction length: d_model
   int ncols;                   // output columns per group: (g + 2) d
   int g, d;
-  const void* a;               // x [a_rows, kdim]
-  uint16_t *q, *k, *v;         // outputs
+  const void* a;               // x [a_rows, kdim] (QKV), y [a_rows = N*Kr, g d] (OUT_P)
+  uint16_t *q, *k, *v;         // outputs (OUT_P: q = P [a_rows, ncols])
   int out_aligned32;           // q, k, v 32-byte aligned: whole-sector stores
   uint32_t* status;
 };
@@ -136,7 +140,9 @@ __global__ void __launch_bounds__(1024) tile_list_kernel(const int32_t* __restri
   }
 }
 
-template <int BN>
+enum Mode { kQKV = 0, kOutP = 1 };
+
+template <int BN, int kMode>
 __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant__ CUtensorMap tm_b, Params p) {
   using L = Layout<BN>;
   constexpr int S = L::kStages;
@@ -169,8 +175,10 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
   const uint32_t tmem = bars->tmem_base;
   pdl_wait();  // the routing layout, the tile list and the inputs are visible from here
 
+  // A CTA takes row tiles mt = blockIdx.x, + gridDim.x, ... and runs every column tile of each
+  // before the next (the tile's rows are decoded once and re-gathered from L2).
   const int nt_count = p.ncols / BN;
-  const int nitems = __ldg(p.ntiles) * nt_count;
+  const int ntiles = __ldg(p.ntiles);
   const int nk = p.kdim / BK;
 
   if (warp >= 4 && warp < 8) {
@@ -179,88 +187,95 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     const int lt = threadIdx.x - 128;
     const int rq = lt >> 3, ch = lt & 7;
     const uint16_t* a_base = static_cast<const uint16_t*>(p.a);
-    // row -> the gathered A row (rows past the segment's end load row 0 and are not stored;
-    // indices are clamped into the tensor)
-    auto a_row = [&](const Tile& t, int r) -> int {
-      int row = 0;
-      if (r < t.rows) row = ld_issue_s32(p.row_src + t.row0 + r) / p.Kr;
+    // routing row_src value -> the gathered A row, clamped into the tensor (rows past the
+    // segment's end load row 0 and are not stored)
+    auto a_row_of = [&](int src) -> int {
+      const int row = kMode == kQKV ? src / p.Kr : src;
       return min(max(row, 0), p.a_rows - 1);
     };
     uint32_t it = 0;
     bool ok = true;
-    int item = blockIdx.x;
+    int mt = blockIdx.x;
     Tile t{};
     int rows_a[8];
-    if (item < nitems) {
-      t = decode_tile(p, __ldg(p.tiles + item / nt_count));
+    if (mt < ntiles) {
+      t = decode_tile(p, __ldg(p.tiles + mt));
 #pragma unroll
-      for (int w = 0; w < 8; ++w) rows_a[w] = a_row(t, rq + 16 * w);
+      for (int w = 0; w < 8; ++w) {
+        const int r = rq + 16 * w;
+        rows_a[w] = a_row_of(r < t.rows ? ld_issue_s32(p.row_src + t.row0 + r) : 0);
+      }
     }
-    const bool prefetch = nk >= 12;
-    for (; item < nitems && ok; item += gridDim.x) {
-      t.nt = item % nt_count;
-      const int b_row = t.hr * p.ncols + t.nt * BN;
-      // the next item's tile and rows, fetched over the first k-blocks of this one, each load
-      // issued four k-blocks before its value is used
-      const int next = item + gridDim.x;
+    // the next row tile's entry, offsets and row indices are fetched during this one's k-blocks
+    // (kq counts them across its column tiles), each load issued four k-blocks before its use
+    const bool prefetch = nt_count * nk >= 12;
+    for (; mt < ntiles && ok; mt += gridDim.x) {
+      const int next = mt + gridDim.x;
       int nx_seg = 0, nx_q = 0, nx_lo = 0, nx_hi = 0;
       Tile nx{};
       int nx_src[8];
       const uint16_t* src[8];
 #pragma unroll
       for (int w = 0; w < 8; ++w) src[w] = a_base + (size_t)rows_a[w] * p.kdim + ch * 8;
-      for (int kb = 0; kb < nk; ++kb, ++it) {
-        if (prefetch && next < nitems) {
-          if (kb == 0) {
-            const int32_t* e = reinterpret_cast<const int32_t*>(p.tiles + next / nt_count);
-            nx_seg = ld_issue_s32(e);
-            nx_q = ld_issue_s32(e + 1);
-          } else if (kb == 4) {
-            nx_lo = ld_issue_s32(p.seg_offsets + nx_seg);
-            nx_hi = ld_issue_s32(p.seg_offsets + nx_seg + 1);
-          } else if (kb == 8) {
-            nx.seg = nx_seg;
-            nx.row0 = nx_lo + nx_q * BM;
-            nx.rows = min(BM, nx_hi - nx.row0);
-            nx.hr = nx_seg % p.Hr;
+      int kq = 0;
+      for (int nt = 0; nt < nt_count && ok; ++nt) {
+        const int b_row = t.hr * p.ncols + nt * BN;
+        for (int kb = 0; kb < nk; ++kb, ++it, ++kq) {
+          if (prefetch && next < ntiles) {
+            if (kq == 0) {
+              const int32_t* e = reinterpret_cast<const int32_t*>(p.tiles + next);
+              nx_seg = ld_issue_s32(e);
+              nx_q = ld_issue_s32(e + 1);
+            } else if (kq == 4) {
+              nx_lo = ld_issue_s32(p.seg_offsets + nx_seg);
+              nx_hi = ld_issue_s32(p.seg_offsets + nx_seg + 1);
+            } else if (kq == 8) {
+              nx.seg = nx_seg;
+              nx.row0 = nx_lo + nx_q * BM;
+              nx.rows = min(BM, nx_hi - nx.row0);
+              nx.hr = nx_seg % p.Hr;
 #pragma unroll
-            for (int w = 0; w < 8; ++w) {
-              const int r = rq + 16 * w;
-              nx_src[w] = r < nx.rows ? ld_issue_s32(p.row_src + nx.row0 + r) : 0;
+              for (int w = 0; w < 8; ++w) {
+                const int r = rq + 16 * w;
+                nx_src[w] = r < nx.rows ? ld_issue_s32(p.row_src + nx.row0 + r) : 0;
+              }
             }
           }
-        }
-        const int slot = it % S;
-        if (it >= (uint32_t)S && !warp_wait(&bars->empty[slot], ((it / S) - 1) & 1, abort_flag, p.status)) {
-          ok = false;
-          break;
-        }
-        uint8_t* a = smem + slot * L::kStage;
-        if (lt == 0) {
-          mbar_arrive_expect_tx(&bars->full[slot], L::kB);
-          tma_load_2d(a + L::kA, &tm_b, kb * BK, b_row, &bars->full[slot]);
-        }
+          const int slot = it % S;
+          if (it >= (uint32_t)S && !warp_wait(&bars->empty[slot], ((it / S) - 1) & 1, abort_flag, p.status)) {
+            ok = false;
+            break;
+          }
+          uint8_t* a = smem + slot * L::kStage;
+          if (lt == 0) {
+            mbar_arrive_expect_tx(&bars->full[slot], L::kB);
+            tma_load_2d(a + L::kA, &tm_b, kb * BK, b_row, &bars->full[slot]);
+          }
 #pragma unroll
-        for (int w = 0; w < 8; ++w) {
-          const int r = rq + 16 * w;
-          cp_async16(a + r * 128 + ((ch ^ (r & 7)) << 4), src[w] + kb * BK);
-        }
-        cp_async_commit();
-        if (it >= (uint32_t)kLag) {
-          cp_async_wait<kLag>();
-          fence_proxy_async_smem();
-          mbar_arrive(&bars->full[(it - kLag) % S]);
+          for (int w = 0; w < 8; ++w) {
+            const int r = rq + 16 * w;
+            cp_async16(a + r * 128 + ((ch ^ (r & 7)) << 4), src[w] + kb * BK);
+          }
+          cp_async_commit();
+          if (it >= (uint32_t)kLag) {
+            cp_async_wait<kLag>();
+            fence_proxy_async_smem();
+            mbar_arrive(&bars->full[(it - kLag) % S]);
+          }
         }
       }
-      if (!ok || next >= nitems) break;
+      if (!ok || next >= ntiles) break;
       if (prefetch) {
         t = nx;
 #pragma unroll
-        for (int w = 0; w < 8; ++w) rows_a[w] = min(max(nx_src[w] / p.Kr, 0), p.a_rows - 1);
+        for (int w = 0; w < 8; ++w) rows_a[w] = a_row_of(nx_src[w]);
       } else {
-        t = decode_tile(p, __ldg(p.tiles + next / nt_count));
+        t = decode_tile(p, __ldg(p.tiles + next));
 #pragma unroll
-        for (int w = 0; w < 8; ++w) rows_a[w] = a_row(t, rq + 16 * w);
+        for (int w = 0; w < 8; ++w) {
+          const int r = rq + 16 * w;
+          rows_a[w] = a_row_of(r < t.rows ? ld_issue_s32(p.row_src + t.row0 + r) : 0);
+        }
       }
     }
     if (ok) {  // retire the last stages
@@ -274,68 +289,85 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     uint32_t it = 0;
     bool ok = true;
     int li = 0;
-    for (int item = blockIdx.x; item < nitems && ok; item += gridDim.x, ++li) {
-      const int buf = li & 1;
-      if (li >= 2 && !warp_wait(&bars->acc_empty[buf], ((li >> 1) - 1) & 1, abort_flag, p.status)) break;
-      tc_fence_after();
-      const uint32_t d_tmem = tmem + buf * 256;
-      for (int kb = 0; kb < nk; ++kb, ++it) {
-        const int slot = it % S;
-        if (!warp_wait(&bars->full[slot], (it / S) & 1, abort_flag, p.status)) {
+    for (int mt = blockIdx.x; mt < ntiles && ok; mt += gridDim.x) {
+      for (int nt = 0; nt < nt_count && ok; ++nt, ++li) {
+        const int buf = li & 1;
+        if (li >= 2 && !warp_wait(&bars->acc_empty[buf], ((li >> 1) - 1) & 1, abort_flag, p.status)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint64_t a_desc = make_smem_desc_sw128(smem_u32(smem + slot * L::kStage), 16, 1024);
-        const uint64_t b_desc = make_smem_desc_sw128(smem_u32(smem + slot * L::kStage + L::kA), 16, 1024);
+        const uint32_t d_tmem = tmem + buf * 256;
+        for (int kb = 0; kb < nk; ++kb, ++it) {
+          const int slot = it % S;
+          if (!warp_wait(&bars->full[slot], (it / S) & 1, abort_flag, p.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t a_desc = make_smem_desc_sw128(smem_u32(smem + slot * L::kStage), 16, 1024);
+          const uint64_t b_desc = make_smem_desc_sw128(smem_u32(smem + slot * L::kStage + L::kA), 16, 1024);
 #pragma unroll
-        for (int kk = 0; kk < BK / 16; ++kk)
-          mma_bf16_ss(d_tmem, a_desc + (uint64_t)(kk * 2), b_desc + (uint64_t)(kk * 2), idesc,
-                      (kb | kk) ? 1u : 0u);
-        mma_commit(&bars->empty[slot]);
+          for (int kk = 0; kk < BK / 16; ++kk)
+            mma_bf16_ss(d_tmem, a_desc + (uint64_t)(kk * 2), b_desc + (uint64_t)(kk * 2), idesc,
+                        (kb | kk) ? 1u : 0u);
+          mma_commit(&bars->empty[slot]);
+        }
+        if (ok) mma_commit(&bars->acc_full[buf]);
       }
-      if (ok) mma_commit(&bars->acc_full[buf]);
     }
   } else {
     // ---- epilogue: thread = tile row = TMEM lane
     const int row = warp * 32 + lane;
     const uint32_t lane_addr = (uint32_t)(warp * 32) << 16;
     int li = 0;
-    for (int item = blockIdx.x; item < nitems; item += gridDim.x, ++li) {
-      Tile t = decode_tile(p, __ldg(p.tiles + item / nt_count));
-      t.nt = item % nt_count;
-      const int buf = li & 1;
+    bool ok = true;
+    for (int mt = blockIdx.x; mt < ntiles && ok; mt += gridDim.x) {
+      const Tile t = decode_tile(p, __ldg(p.tiles + mt));
       const bool valid = row < t.rows;
       const int r = t.row0 + row;
-      if (!warp_wait(&bars->acc_full[buf], (li >> 1) & 1, abort_flag, p.status)) break;
-      tc_fence_after();
-#pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld32(tmem + lane_addr + buf * 256 + c * 32, v);
-        tmem_wait_ld();
-        if (!valid) continue;
-        const int n = t.nt * BN + c * 32;  // first output column of the chunk
-        uint16_t* dst;
-        const int gd = p.g * p.d;
-        if (n < gd) dst = p.q + ((long long)r * p.g + n / p.d) * p.d + n % p.d;
-        else if (n < gd + p.d) dst = p.k + (long long)r * p.d + (n - gd);
-        else dst = p.v + (long long)r * p.d + (n - gd - p.d);
-        uint32_t w[16];
-#pragma unroll
-        for (int e = 0; e < 16; ++e) w[e] = pack_bf16x2(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
-        if (p.out_aligned32) {
-          st_global_v8(dst, w);
-          st_global_v8(dst + 16, w + 8);
-        } else {
-          uint4* d4 = reinterpret_cast<uint4*>(dst);
-#pragma unroll
-          for (int e = 0; e < 4; ++e) d4[e] = make_uint4(w[4 * e], w[4 * e + 1], w[4 * e + 2], w[4 * e + 3]);
+      // OUT_P writes row r's partial product at its token-slot row row_src[r]
+      const int dst_row = kMode == kOutP && valid ? ld_issue_s32(p.row_src + r) : r;
+      for (int nt = 0; nt < nt_count; ++nt, ++li) {
+        const int buf = li & 1;
+        if (!warp_wait(&bars->acc_full[buf], (li >> 1) & 1, abort_flag, p.status)) {
+          ok = false;
+          break;
         }
+        tc_fence_after();
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t v[32];
+          tmem_ld32(tmem + lane_addr + buf * 256 + c * 32, v);
+          tmem_wait_ld();
+          if (!valid) continue;
+          const int n = nt * BN + c * 32;  // first output column of the chunk
+          uint16_t* dst;
+          if constexpr (kMode == kQKV) {
+            const int gd = p.g * p.d;
+            if (n < gd) dst = p.q + ((long long)r * p.g + n / p.d) * p.d + n % p.d;
+            else if (n < gd + p.d) dst = p.k + (long long)r * p.d + (n - gd);
+            else dst = p.v + (long long)r * p.d + (n - gd - p.d);
+          } else {
+            if (dst_row < 0 || dst_row >= p.a_rows) continue;  // an inconsistent layout
+            dst = p.q + (long long)dst_row * p.ncols + n;
+          }
+          uint32_t w[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) w[e] = pack_bf16x2(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
+          if (p.out_aligned32) {
+            st_global_v8(dst, w);
+            st_global_v8(dst + 16, w + 8);
+          } else {
+            uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) d4[e] = make_uint4(w[4 * e], w[4 * e + 1], w[4 * e + 2], w[4 * e + 3]);
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->acc_empty[buf]);
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->acc_empty[buf]);
     }
   }
 
@@ -354,6 +386,38 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
   }
 }
 
+// o[t] (+)= sum_k P[t Kr + k] in fp32: a token's Kr slot rows are adjacent in P.
+__global__ void combine_kernel(const uint16_t* __restrict__ P, long long ntok, int Kr, int d_model,
+                               float* __restrict__ o, int accumulate) {
+  const int v8 = d_model / 8;  // 16-byte vectors of P per row
+  const long long n = ntok * v8;
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+    const long long t = i / v8;
+    const int c = (int)(i - t * v8);
+    float a[8];
+    if (accumulate) {
+      const float4 o0 = reinterpret_cast<const float4*>(o + t * d_model)[2 * c];
+      const float4 o1 = reinterpret_cast<const float4*>(o + t * d_model)[2 * c + 1];
+      a[0] = o0.x; a[1] = o0.y; a[2] = o0.z; a[3] = o0.w;
+      a[4] = o1.x; a[5] = o1.y; a[6] = o1.z; a[7] = o1.w;
+    } else {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) a[e] = 0.f;
+    }
+    for (int k = 0; k < Kr; ++k) {
+      const uint4 w = __ldg(reinterpret_cast<const uint4*>(P + (t * Kr + k) * d_model) + c);
+      const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        a[2 * e] += bf16_lo(ws[e]);
+        a[2 * e + 1] += bf16_hi(ws[e]);
+      }
+    }
+    reinterpret_cast<float4*>(o + t * d_model)[2 * c] = make_float4(a[0], a[1], a[2], a[3]);
+    reinterpret_cast<float4*>(o + t * d_model)[2 * c + 1] = make_float4(a[4], a[5], a[6], a[7]);
+  }
+}
+
 bool encode_map(CUtensorMap* map, const void* base, long long rows, int cols, int box_rows) {
   EncodeTiledFn enc = tensor_map_encoder();
   if (!enc) return false;
@@ -366,14 +430,14 @@ bool encode_map(CUtensorMap* map, const void* base, long long rows, int cols, in
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN>
+template <int BN, int kMode>
 cudaError_t launch_bn(const Params& p, const void* b, long long b_rows, int grid, cudaStream_t stream) {
   CUtensorMap tb;
   if (!encode_map(&tb, b, b_rows, p.kdim, BN)) return cudaErrorInvalidValue;
   const int smem = Layout<BN>::kAlloc;
-  cudaError_t e = cudaFuncSetAttribute(proj_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaError_t e = cudaFuncSetAttribute(proj_kernel<BN, kMode>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  return launch_pdl(proj_kernel<BN>, dim3(grid), dim3(kThreads), (size_t)smem, stream, tb, p);
+  return launch_pdl(proj_kernel<BN, kMode>, dim3(grid), dim3(kThreads), (size_t)smem, stream, tb, p);
 }
 
 // The widest column tile (multiple of 32, at most 256) that divides the output columns.
@@ -383,14 +447,15 @@ int pick_bn(int ncols) {
   return 0;
 }
 
+template <int kMode>
 cudaError_t launch(int bn, const Params& p, const void* b, long long b_rows, int grid, cudaStream_t stream) {
   switch (bn) {
-    case 256: return launch_bn<256>(p, b, b_rows, grid, stream);
-    case 192: return launch_bn<192>(p, b, b_rows, grid, stream);
-    case 160: return launch_bn<160>(p, b, b_rows, grid, stream);
-    case 128: return launch_bn<128>(p, b, b_rows, grid, stream);
-    case 96: return launch_bn<96>(p, b, b_rows, grid, stream);
-    default: return launch_bn<64>(p, b, b_rows, grid, stream);
+    case 256: return launch_bn<256, kMode>(p, b, b_rows, grid, stream);
+    case 192: return launch_bn<192, kMode>(p, b, b_rows, grid, stream);
+    case 160: return launch_bn<160, kMode>(p, b, b_rows, grid, stream);
+    case 128: return launch_bn<128, kMode>(p, b, b_rows, grid, stream);
+    case 96: return launch_bn<96, kMode>(p, b, b_rows, grid, stream);
+    default: return launch_bn<64, kMode>(p, b, b_rows, grid, stream);
   }
 }
 
@@ -415,12 +480,6 @@ int check_common(int B, int total_tokens, int d_model, int H, int K, int d_head,
 
 using namespace namoh;
 
-namespace namoh {  // the output projection, in proj_out.cu
-size_t proj_out_workspace(long long total_tokens, int Kr, int gd, int nseg);
-int launch_proj_out(const uint16_t* y, int total_tokens, int d_model, const uint16_t* w_o, int Hr, int Kr, int gd,
-                    int nseg, const int32_t* seg_offsets, const int32_t* row_src, float* o, int accumulate,
-                    void* workspace, size_t workspace_bytes, uint32_t* dev_status, int sm_count, cudaStream_t stream);
-}  // namespace namoh
 
 namespace {
 // The row-tile list: at most ceil(R / 128) + nseg tiles, plus its length.
@@ -447,12 +506,16 @@ int proj_prologue(const int32_t* seg_offsets, int nseg, int Hr, long long R, voi
 }
 }  // namespace
 
-extern "C" size_t namoh_proj_workspace_size(int B, int total_tokens, int H, int K, int d_head, int group) {
-  if (B < 1 || total_tokens < 1 || group < 1 || H < 1 || K < 1 || H % group || K % group || d_head < 1) return 0;
+// namoh_proj_out's workspace: the tile list, then P [total_tokens * Kr, d_model] bf16.
+size_t out_workspace(long long total_tokens, int Kr, int nseg, int d_model) {
+  return align_up(tile_list_bytes(total_tokens * Kr, nseg), 256) +
+         align_up((size_t)total_tokens * Kr * d_model * sizeof(uint16_t), 256);
+}
+
+extern "C" size_t namoh_proj_workspace_size(int B, int total_tokens, int d_model, int H, int K, int group) {
+  if (B < 1 || total_tokens < 1 || d_model < 1 || group < 1 || H < 1 || K < 1 || H % group || K % group) return 0;
   const int Hr = H / group, Kr = K / group;
-  const size_t qkv = align_up(tile_list_bytes((long long)total_tokens * Kr, B * Hr), 256);
-  const size_t out = proj_out_workspace(total_tokens, Kr, group * d_head, B * Hr);
-  return qkv > out ? qkv : out;
+  return out_workspace(total_tokens, Kr, B * Hr, d_model);  // the larger of the two calls' needs
 }
 
 extern "C" int namoh_proj_qkv(const uint16_t* x, int total_tokens, int d_model, const uint16_t* w_qkv, int B, int H,
@@ -491,7 +554,7 @@ extern "C" int namoh_proj_qkv(const uint16_t* x, int total_tokens, int d_model, 
   p.out_aligned32 = ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k) |
                       reinterpret_cast<uintptr_t>(v)) & 31u) == 0;
   p.status = dev_status;
-  const cudaError_t e = proj::launch(bn, p, w_qkv, (long long)Hr * ncols, info.sm_count, stream);
+  const cudaError_t e = proj::launch<proj::kQKV>(bn, p, w_qkv, (long long)Hr * ncols, info.sm_count, stream);
   return e == cudaSuccess ? NAMOH_OK : cuda_fail(e, "proj_kernel (qkv) launch");
 }
 
@@ -501,12 +564,38 @@ extern "C" int namoh_proj_out(const uint16_t* y, int total_tokens, int d_model, 
                               void* stream_v) {
   if (!y || !w_o || !seg_offsets || !row_src || !o || !dev_status) return NAMOH_ERR_INVALID_ARG;
   int Hr, Kr;
-  const int st = proj::check_common(B, total_tokens, d_model, H, K, d_head, group, &Hr, &Kr);
+  int st = proj::check_common(B, total_tokens, d_model, H, K, d_head, group, &Hr, &Kr);
   if (st != NAMOH_OK) return st;
   if (!aligned16(y) || !aligned16(w_o) || !aligned16(o)) return NAMOH_ERR_INVALID_ARG;
+  const int bn = proj::pick_bn(d_model);
   DeviceInfo info;
   if (!current_device_info(&info) || info.major != 10) return NAMOH_ERR_UNSUPPORTED;
-  return launch_proj_out(y, total_tokens, d_model, w_o, Hr, Kr, group * d_head, B * Hr, seg_offsets, row_src, o,
-                         accumulate ? 1 : 0, workspace, workspace_bytes, dev_status, info.sm_count,
-                         reinterpret_cast<cudaStream_t>(stream_v));
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
+  const int nseg = B * Hr;
+  const long long R = (long long)total_tokens * Kr;
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) ||
+      workspace_bytes < out_workspace(total_tokens, Kr, nseg, d_model))
+    return NAMOH_ERR_WORKSPACE;
+  uint16_t* P = reinterpret_cast<uint16_t*>(static_cast<char*>(workspace) + align_up(tile_list_bytes(R, nseg), 256));
+  proj::Params p{};
+  st = proj_prologue(seg_offsets, nseg, Hr, R, workspace, workspace_bytes, &p, stream);
+  if (st != NAMOH_OK) return st;
+  p.seg_offsets = seg_offsets;
+  p.row_src = row_src;
+  p.nseg = nseg;
+  p.Hr = Hr;
+  p.Kr = Kr;
+  p.a = y;
+  p.a_rows = (int)R;
+  p.kdim = group * d_head;
+  p.ncols = d_model;
+  p.g = group;
+  p.d = d_head;
+  p.q = P;
+  p.out_aligned32 = 1;  // P starts 256-byte aligned and its rows are multiples of 128 bytes
+  p.status = dev_status;
+  cudaError_t e = proj::launch<proj::kOutP>(bn, p, w_o, (long long)Hr * d_model, info.sm_count, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "proj_kernel (out) launch");
+  proj::combine_kernel<<<info.sm_count * 8, 256, 0, stream>>>(P, total_tokens, Kr, d_model, o, accumulate ? 1 : 0);
+  return cuda_check_launch("combine_kernel launch");
 }
