@@ -478,7 +478,7 @@ def run_layer(args, dev, pk, pk_kind):
         "qkv_projection": {"ms": ms_qkv, "tflops": tf(f_qkv, ms_qkv), "frac_bf16": tf(f_qkv, ms_qkv) / peak,
                            "flops": f_qkv, "kernel": "proj_kernel (tcgen05, rows gathered by cp.async)"},
         "out_projection": {"ms": ms_out, "tflops": tf(f_out, ms_out), "frac_bf16": tf(f_out, ms_out) / peak,
-                           "flops": f_out, "kernel": "proj_out_kernel (token windows, fp32 o written once)"},
+                           "flops": f_out, "kernel": "proj_kernel, per-slot products (bf16), then combine_kernel (fp32 sums)"},
         "layer_step": {"ms": ms_step, "tflops": tf(f_qkv + f_attn + f_out, ms_step),
                        "frac_bf16": tf(f_qkv + f_attn + f_out, ms_step) / peak,
                        "flops": f_qkv + f_attn + f_out,
@@ -486,9 +486,9 @@ def run_layer(args, dev, pk, pk_kind):
         "peak_source": f"{pk_kind} bf16 dense (burst)",
         "l2": "flushed before every timed launch sequence (2 GB write)",
         "device_status": int(status.item()),
-        # timed launches: QKV (tile list + GEMM), OUT (pack, table, bounds, GEMM), and the step
-        # (route 2 + QKV 2 + prefill 2 + OUT 4)
-        "launches": args.steps * (2 + 4 + 10),
+        # timed launches: QKV (tile list + GEMM), OUT (tile list, GEMM, combine), and the step
+        # (route 2 + QKV 2 + prefill 2 + OUT 3)
+        "launches": args.steps * (2 + 3 + 9),
     }
 
 
