@@ -74,13 +74,15 @@ def _load():
         lib.oracle_prefill.argtypes = [P, P, P, i32, i32, i32, f64, P, P, P, P, P, i32, i32, P]
         lib.oracle_prefill_rows.argtypes = [P, P, P, i32, i32, i32, f64, P, P, P, P, P, i64, P, i32, P]
         lib.oracle_decode_step.argtypes = [P, P, P, P, P, i32, i32, i32, i32, i32, f64,
-                                           P, P, P, P, P, P, i32, P]
+                                           P, P, P, P, P, P, i32, P, i32]
+        lib.oracle_shared_prefill.argtypes = [P, P, P, i32, i32, i32, i32, i32, f64, i32, P, i32]
         lib.oracle_proj_qkv.argtypes = [P, i32, P, i32, i32, i32, i32, P, i32, P, P, P, P, i32]
         lib.oracle_proj_out.argtypes = [P, P, i64, i32, i32, i32, P, i32, i32, P, i32]
         lib.oracle_default_threads.argtypes = []
         for fn in ("oracle_route_topk", "oracle_route_biased", "oracle_dispatch", "oracle_dispatch_varlen",
                    "oracle_rope", "oracle_prefill",
                    "oracle_prefill_rows", "oracle_decode_step", "oracle_proj_qkv", "oracle_proj_out",
+                   "oracle_shared_prefill",
                    "oracle_default_threads"):
             getattr(lib, fn).restype = ctypes.c_int
         _lib = lib
@@ -294,11 +296,13 @@ def prefill_rows(q, k, v, seg_offsets, row_src, gate, d: int, g: int, base: floa
 
 def decode_step(topk_head, gate, q, k, v, Hr: int, d: int, g: int, base: float,
                 k_cache: np.ndarray, v_cache: np.ndarray, seg_base: np.ndarray, seg_len: np.ndarray,
-                seg_cap: np.ndarray, interleaved: bool = False, token_pos: np.ndarray | None = None) -> np.ndarray:
+                seg_cap: np.ndarray, interleaved: bool = False, token_pos: np.ndarray | None = None,
+                window: int = 0) -> np.ndarray:
     """One decode step.  k_cache/v_cache [cap_total, d] fp64 and seg_len are updated in place.
 
     topk_head/gate [B, Kr]; q [B, Kr*g, d], k/v [B, Kr, d] as bf16 bits.  Returns y [B, Kr*g, d].
     RoPE positions are the ranks, or token_pos [B] (the new tokens' indices) when given.
+    window > 0 attends over the last `window` rows only (the new one included).
     """
     lib = _load()
     topk_head = np.ascontiguousarray(topk_head, dtype=np.int32)
@@ -317,7 +321,7 @@ def decode_step(topk_head, gate, q, k, v, Hr: int, d: int, g: int, base: float,
     rc = lib.oracle_decode_step(_ptr(topk_head), _ptr(gate), _ptr(q), _ptr(k), _ptr(v), B, Hr, Kr, d, g,
                                 float(base), _ptr(k_cache), _ptr(v_cache), _ptr(seg_base), _ptr(seg_len),
                                 _ptr(seg_cap), _ptr(y), int(bool(interleaved)),
-                                _ptr(token_pos) if token_pos is not None else None)
+                                _ptr(token_pos) if token_pos is not None else None, int(window))
     _check(rc, "decode_step")
     return y
 
@@ -357,3 +361,28 @@ def proj_out(y, topk_head, w_o, g: int, d: int, nthreads: int | None = None):
     _check(lib.oracle_proj_out(_ptr(y), _ptr(topk), N, Kr, g, d, _ptr(w), Hr, d_model, _ptr(o), nthreads),
            "proj_out")
     return o
+
+
+def shared_prefill(q, k, v, window: int, base: float, interleaved: bool = False, nthreads: int | None = None):
+    """Shared heads (Sec. 5): q, k, v [B, Hs, T, d] bf16 bits; full causal (window 0) or sliding
+    window attention at global positions, no gate.  Returns y [B, T, Hs, d] fp64."""
+    lib = _load()
+    q = np.ascontiguousarray(q, dtype=np.uint16)
+    k = np.ascontiguousarray(k, dtype=np.uint16)
+    v = np.ascontiguousarray(v, dtype=np.uint16)
+    B, Hs, T, d = q.shape
+    y = np.empty((B, T, Hs, d))
+    nthreads = default_threads() if nthreads is None else int(nthreads)
+    _check(lib.oracle_shared_prefill(_ptr(q), _ptr(k), _ptr(v), B, Hs, T, d, int(window), float(base),
+                                     int(bool(interleaved)), _ptr(y), nthreads), "shared_prefill")
+    return y
+
+
+def shared_decode_step(q, k, v, d: int, base: float, k_cache, v_cache, seg_base, seg_len, seg_cap, window: int):
+    """One decode step of the shared heads: q, k, v [B, Hs, d] bf16 bits, every head active with
+    gate 1 (decode_step with all heads selected).  Returns y [B, Hs, d] fp64."""
+    q = np.ascontiguousarray(q, dtype=np.uint16)
+    B, Hs = q.shape[0], q.shape[1]
+    top = np.tile(np.arange(Hs, dtype=np.int32), (B, 1))
+    return decode_step(top, np.ones((B, Hs)), q, k, v, Hs, d, 1, base, k_cache, v_cache, seg_base, seg_len,
+                       seg_cap, window=window)

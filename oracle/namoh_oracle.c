@@ -24,6 +24,8 @@
  *                within only its selected heads' histories; its rank is the current length.
  *   - GQA:       App. C, "Adopted KV-group routing": K/g of H/g groups are selected, the g
  *                query heads of a group share its gate, key/value history and rank.
+ *   - shared:    the shared-head variant (Sec. 5): always-active heads over the full causal
+ *                prefix or a sliding window of the last w tokens, at global RoPE positions.
  *
  * Readings where the paper is silent (each listed in the design notes):
  *   - TopK compares the raw fp32 router logits (softmax is monotone, so the selected
@@ -573,7 +575,7 @@ int oracle_prefill_rows(const uint16_t *q, const uint16_t *k, const uint16_t *v,
 int oracle_decode_step(const int32_t *topk_head, const double *gate, const uint16_t *q, const uint16_t *k,
                        const uint16_t *v, int B, int Hr, int Kr, int d, int g, double base,
                        double *k_cache, double *v_cache, const int64_t *seg_base, int32_t *seg_len,
-                       const int32_t *seg_cap, double *y, int interleaved, const int64_t *token_pos)
+                       const int32_t *seg_cap, double *y, int interleaved, const int64_t *token_pos, int window)
 {
     if (!topk_head || !gate || !q || !k || !v || !k_cache || !v_cache || !seg_base || !seg_len || !seg_cap || !y)
         return ORACLE_ERR_ARG;
@@ -597,11 +599,14 @@ int oracle_decode_step(const int32_t *topk_head, const double *gate, const uint1
                 v_cache[(base_row + rho) * d + cc] = bf16_to_double(v[((long)b * Kr + kk) * d + cc]);
             double *w = (double *)malloc(sizeof(double) * (size_t)(rho + 1));
             if (!w) { st = ORACLE_ERR_NOMEM; break; }
+            /* a sliding window keeps the last `window` rows, the new one included */
+            const long first = (window > 0 && rho + 1 > window) ? rho + 1 - window : 0;
             for (int j = 0; j < g; ++j) {
                 long qi = ((long)b * Kr + kk) * g + j;
                 for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(q[qi * d + cc]);
                 rope_rotate(tmp, d, p, base, interleaved, qr);
-                attend(qr, k_cache + base_row * d, v_cache + base_row * d, rho + 1, d, w, h);
+                attend(qr, k_cache + (base_row + first) * d, v_cache + (base_row + first) * d, rho + 1 - first, d, w,
+                       h);
                 for (int cc = 0; cc < d; ++cc) y[qi * d + cc] = gate[b * Kr + kk] * h[cc];
             }
             free(w);
@@ -712,6 +717,67 @@ int oracle_proj_out(const double *y, const int32_t *topk_head, long N, int Kr, i
         if (topk_head[i] < 0 || topk_head[i] >= Hr) return ORACLE_ERR_ARG;
     struct proj_out_ctx c = {y, w, topk_head, Kr, g, d, d_model, o};
     parallel_for(N, nthreads, proj_out_token, &c);
+    return ORACLE_OK;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Shared heads (the always-active heads of the paper's shared-head variant)  */
+/* ------------------------------------------------------------------------- */
+
+struct shared_ctx {
+    const uint16_t *q, *k, *v;
+    int Hs, T, d, window, interleaved;
+    double base;
+    double *y;
+};
+
+/* One (sequence, shared head): every token, keys at global positions. */
+static void shared_head(long bj, void *arg)
+{
+    const struct shared_ctx *c = (const struct shared_ctx *)arg;
+    const int T = c->T, d = c->d;
+    const long b = bj / c->Hs, j = bj % c->Hs;
+    const long row0 = bj * (long)T;  /* q, k, v are [B, Hs, T, d] */
+    double *keys = (double *)malloc(sizeof(double) * (size_t)T * d);
+    double *vals = (double *)malloc(sizeof(double) * (size_t)T * d);
+    double *tmp = (double *)malloc(sizeof(double) * (size_t)d);
+    double *qr = (double *)malloc(sizeof(double) * (size_t)d);
+    double *w = (double *)malloc(sizeof(double) * (size_t)T);
+    double *h = (double *)malloc(sizeof(double) * (size_t)d);
+    if (!keys || !vals || !tmp || !qr || !w || !h) goto done;
+    for (long t = 0; t < T; ++t) {
+        for (int cc = 0; cc < d; ++cc) {
+            tmp[cc] = bf16_to_double(c->k[(row0 + t) * d + cc]);
+            vals[t * d + cc] = bf16_to_double(c->v[(row0 + t) * d + cc]);
+        }
+        rope_rotate(tmp, d, (double)t, c->base, c->interleaved, keys + t * d);
+    }
+    for (long t = 0; t < T; ++t) {
+        /* the full causal prefix, or the most recent `window` tokens including t */
+        const long lo = (c->window > 0 && t + 1 > c->window) ? t + 1 - c->window : 0;
+        for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(c->q[(row0 + t) * d + cc]);
+        rope_rotate(tmp, d, (double)t, c->base, c->interleaved, qr);
+        attend(qr, keys + lo * d, vals + lo * d, t + 1 - lo, d, w, h);
+        for (int cc = 0; cc < d; ++cc) c->y[((b * T + t) * c->Hs + j) * d + cc] = h[cc];
+    }
+done:
+    free(keys); free(vals); free(tmp); free(qr); free(w); free(h);
+}
+
+/*
+ * oracle_shared_prefill: the always-active shared heads of the paper's shared-head variant
+ * (Sec. 5, "Shared heads for local context"): every token, causal attention over the full
+ * prefix (window = 0) or over the most recent `window` tokens including itself, RoPE at the
+ * global position t, no gate.
+ *   q, k, v  [B, Hs, T, d] bf16 bits (each head's sequence contiguous)
+ *   y        [B, T, Hs, d] fp64 out
+ */
+int oracle_shared_prefill(const uint16_t *q, const uint16_t *k, const uint16_t *v, int B, int Hs, int T, int d,
+                          int window, double base, int interleaved, double *y, int nthreads)
+{
+    if (!q || !k || !v || !y || B < 1 || Hs < 1 || T < 1 || d < 2 || d % 2 || window < 0) return ORACLE_ERR_ARG;
+    struct shared_ctx c = {q, k, v, Hs, T, d, window, interleaved, base, y};
+    parallel_for((long)B * Hs, nthreads, shared_head, &c);
     return ORACLE_OK;
 }
 

@@ -27,6 +27,10 @@ MUTATIONS = {
                                  "c->q[(r * c->g + (c->g - 1 - n / c->d)) * c->d + n % c->d] = acc;"),
     "proj_wrong_group": ("const int hr = lo % c->Hr;", "const int hr = (lo + 1) % c->Hr;"),
     "proj_out_drops_first_slot": ("for (int k = 0; k < c->Kr; ++k) {", "for (int k = 1; k < c->Kr; ++k) {"),
+    "shared_window_one_too_wide": ("(c->window > 0 && t + 1 > c->window) ? t + 1 - c->window : 0;",
+                                   "(c->window > 0 && t + 1 > c->window) ? t - c->window : 0;"),
+    "decode_window_one_too_wide": ("(window > 0 && rho + 1 > window) ? rho + 1 - window : 0;",
+                                   "(window > 0 && rho + 1 > window) ? rho - window : 0;"),
     "decode_ignores_token_pos": ("const double p = token_pos ? (double)token_pos[b] : (double)rho;",
                                  "const double p = token_pos ? (double)rho : (double)rho;"),
     "no_scale": ("double scale = 1.0 / sqrt((double)d);", "double scale = 1.0;"),
@@ -61,7 +65,7 @@ def test_pins_catch_mutation(tmp_path, name):
                     ignore=shutil.ignore_patterns("*.so", "__pycache__", "csrc", "_build"))
     os.makedirs(tmp_path / "tests")
     for f in ("conftest.py", "test_oracle_route.py", "test_oracle_attention.py", "test_oracle_layer.py",
-              "test_accounting.py"):
+              "test_oracle_shared.py", "test_accounting.py"):
         shutil.copy(os.path.join(ROOT, "tests", f), tmp_path / "tests")
     shutil.copytree(os.path.join(ROOT, "tests", "golden"), tmp_path / "tests" / "golden")
     r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider", "-m", "not gpu",
