@@ -335,6 +335,38 @@ NAMOH_API int namoh_decode_ex(const int32_t *topk_head, const float *gate, const
                               void *stream);
 
 /* ------------------------------------------------------------------------- *
+ * Shared heads: the paper's shared-head variant (Sec. 5, "Shared heads for local
+ * context"): Hs always-active heads, outside the routing, each attending to the full
+ * causal prefix (window = 0) or to the most recent `window` tokens including the current
+ * one, with RoPE at the token's global position and no gate.  Their outputs are summed
+ * into o by the caller's projection, like the routed heads'.
+ *
+ * namoh_shared_prefill
+ *   q, k, v     [B, Hs, T, d] bf16 (each head's sequence contiguous).
+ *   y           [B, T, Hs, d] bf16 out: h of every (token, shared head).
+ *   k_cache, v_cache, seg_base, seg_cap, cache_rows, seg_len: as namoh_prefill, segment
+ *               (b, j) = shared head j of sequence b (B*Hs segments of T rows).
+ *   rope_flags  NAMOH_ROPE_INTERLEAVED or 0 (positions are global already).
+ *   Workspace: namoh_shared_workspace_size.  Supports d_head in {64, 128}, T <= 2^20.
+ * namoh_shared_decode: one new token per sequence for every shared head: q, k, v and y
+ *   [B, Hs, d]; appends k~ (at position seg_len, which is t) and v, attends over the last
+ *   min(seg_len + 1, window) rows (all of them when window = 0), seg_len += 1.
+ *   Workspace: namoh_shared_decode_workspace_size.
+ * ------------------------------------------------------------------------- */
+NAMOH_API size_t namoh_shared_workspace_size(int B, int T, int Hs, int d_head);
+NAMOH_API int namoh_shared_prefill(const uint16_t *q, const uint16_t *k, const uint16_t *v, int B, int T, int Hs,
+                                   int d_head, int window, float rope_base, unsigned rope_flags, uint16_t *y,
+                                   uint16_t *k_cache, uint16_t *v_cache, const int64_t *seg_base,
+                                   const int32_t *seg_cap, int64_t cache_rows, int32_t *seg_len, void *workspace,
+                                   size_t workspace_bytes, uint32_t *dev_status, void *stream);
+NAMOH_API size_t namoh_shared_decode_workspace_size(int B, int Hs, int d_head);
+NAMOH_API int namoh_shared_decode(const uint16_t *q, const uint16_t *k, const uint16_t *v, int B, int Hs, int d_head,
+                                  int window, float rope_base, unsigned rope_flags, uint16_t *k_cache,
+                                  uint16_t *v_cache, const int64_t *seg_base, int32_t *seg_len,
+                                  const int32_t *seg_cap, int64_t cache_rows, uint16_t *y, void *workspace,
+                                  size_t workspace_bytes, uint32_t *dev_status, void *stream);
+
+/* ------------------------------------------------------------------------- *
  * The projections around the path (the full attention layer).
  * Sec. 3.1, Eq. (namoh-qkv): only an active token-head pair projects,
  *   q_{t,i} = x_t W_Q^(i), k_{t,i} = x_t W_K^(i), v_{t,i} = x_t W_V^(i), t in I_i.

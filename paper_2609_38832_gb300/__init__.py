@@ -18,7 +18,7 @@ from ._abi import (NAMOH_DEV_BAD_SEQLENS, NAMOH_DEV_CAPACITY, NAMOH_DEV_NONFINIT
                    NAMOH_ROPE_GLOBAL, NAMOH_ROPE_INTERLEAVED, NamohError)
 
 __all__ = ["namoh_route", "namoh_route_varlen", "namoh_prefill", "namoh_prefill_varlen", "namoh_decode",
-           "namoh_proj_qkv", "namoh_proj_out",
+           "namoh_proj_qkv", "namoh_proj_out", "namoh_shared_prefill", "namoh_shared_decode",
            "namoh_rope_pack", "namoh_attention_plan", "namoh_attention", "RouteOutputs", "Workspace", "NamohError",
            "NAMOH_DEV_BAD_SEQLENS", "NAMOH_DEV_CAPACITY", "NAMOH_DEV_NONFINITE_SCORE", "NAMOH_DEV_TIMEOUT",
            "NAMOH_ROPE_GLOBAL", "NAMOH_ROPE_INTERLEAVED", "library_path"]
@@ -292,6 +292,64 @@ def namoh_attention(q_rot: torch.Tensor, k_cache: torch.Tensor, v_cache: torch.T
                              _ptr(row_src), _ptr(gate), _ptr(seg_base), k_cache.shape[0], _ptr(plan), plan.numel(),
                              _ptr(y), _ptr(st), _stream(stream))
     _abi.check("namoh_attention", rc)
+    return y
+
+
+def namoh_shared_prefill(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, *, window: int = 0,
+                         rope_base: float = 10000.0, interleaved: bool = False, y: Optional[torch.Tensor] = None,
+                         k_cache: Optional[torch.Tensor] = None, v_cache: Optional[torch.Tensor] = None,
+                         seg_base: Optional[torch.Tensor] = None, seg_cap: Optional[torch.Tensor] = None,
+                         seg_len: Optional[torch.Tensor] = None, workspace: Optional[Workspace] = None,
+                         status: Optional[torch.Tensor] = None, stream=None):
+    """Shared heads (see namoh_shared_prefill in include/namoh.h): q, k, v [B, Hs, T, d] bf16;
+    window 0 = full causal prefix.  Returns (y [B, T, Hs, d], k_cache, v_cache)."""
+    lib = _abi.load()
+    for name, t in (("q", q), ("k", k), ("v", v)):
+        if t.dtype != torch.bfloat16 or t.dim() != 4:
+            raise ValueError(f"{name} must be a [B, Hs, T, d] bfloat16 tensor")
+    B, Hs, T, d = q.shape
+    dev = q.device
+    if y is None:
+        y = torch.empty((B, T, Hs, d), dtype=torch.bfloat16, device=dev)
+    if k_cache is None:
+        k_cache = torch.empty((B * Hs * T, d), dtype=torch.bfloat16, device=dev)
+    if v_cache is None:
+        v_cache = v if seg_base is None else torch.empty_like(k_cache)
+    nbytes = lib.namoh_shared_workspace_size(B, T, Hs, d)
+    if nbytes == 0:
+        raise NamohError("namoh_shared_workspace_size", _abi.NAMOH_ERR_UNSUPPORTED)
+    ws = _ws(workspace, nbytes, dev)
+    st = _status(status, dev)
+    cache_rows = k_cache.numel() // d
+    rc = lib.namoh_shared_prefill(_ptr(q), _ptr(k), _ptr(v), B, T, Hs, d, int(window), float(rope_base),
+                                  _rope_flags(interleaved, False), _ptr(y), _ptr(k_cache), _ptr(v_cache),
+                                  _ptr(seg_base), _ptr(seg_cap), cache_rows, _ptr(seg_len), _ptr(ws), ws.numel(),
+                                  _ptr(st), _stream(stream))
+    _abi.check("namoh_shared_prefill", rc)
+    return y, k_cache, v_cache
+
+
+def namoh_shared_decode(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, *, k_cache: torch.Tensor,
+                        v_cache: torch.Tensor, seg_base: torch.Tensor, seg_len: torch.Tensor, seg_cap: torch.Tensor,
+                        window: int = 0, rope_base: float = 10000.0, interleaved: bool = False,
+                        y: Optional[torch.Tensor] = None, workspace: Optional[Workspace] = None,
+                        status: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """One decode step of the shared heads: q, k, v [B, Hs, d] bf16.  Returns y [B, Hs, d]."""
+    lib = _abi.load()
+    B, Hs, d = q.shape
+    dev = q.device
+    if y is None:
+        y = torch.empty((B, Hs, d), dtype=torch.bfloat16, device=dev)
+    nbytes = lib.namoh_shared_decode_workspace_size(B, Hs, d)
+    if nbytes == 0:
+        raise NamohError("namoh_shared_decode_workspace_size", _abi.NAMOH_ERR_UNSUPPORTED)
+    ws = _ws(workspace, nbytes, dev)
+    st = _status(status, dev)
+    rc = lib.namoh_shared_decode(_ptr(q), _ptr(k), _ptr(v), B, Hs, d, int(window), float(rope_base),
+                                 _rope_flags(interleaved, False), _ptr(k_cache), _ptr(v_cache), _ptr(seg_base),
+                                 _ptr(seg_len), _ptr(seg_cap), k_cache.shape[0], _ptr(y), _ptr(ws), ws.numel(),
+                                 _ptr(st), _stream(stream))
+    _abi.check("namoh_shared_decode", rc)
     return y
 
 

@@ -61,6 +61,11 @@ SIGNATURES = {
     "namoh_proj_workspace_size": (_SZ, [_I, _I, _I, _I, _I, _I]),
     "namoh_proj_qkv": (_I, [_P, _I, _I, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _SZ, _P, _P]),
     "namoh_proj_out": (_I, [_P, _I, _I, _P, _I, _I, _I, _I, _I, _P, _P, _P, _I, _P, _SZ, _P, _P]),
+    "namoh_shared_workspace_size": (_SZ, [_I, _I, _I, _I]),
+    "namoh_shared_prefill": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _F, _U, _P, _P, _P, _P, _P, _I64, _P, _P, _SZ, _P,
+                                  _P]),
+    "namoh_shared_decode_workspace_size": (_SZ, [_I, _I, _I]),
+    "namoh_shared_decode": (_I, [_P, _P, _P, _I, _I, _I, _I, _F, _U, _P, _P, _P, _P, _P, _I64, _P, _P, _SZ, _P, _P]),
     "namoh_decode_workspace_size": (_SZ, [_I, _I, _I, _I, _I]),
     "namoh_decode": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P, _P, _I64, _P, _P, _SZ, _P,
                           _P]),

@@ -30,9 +30,10 @@ constexpr int kSplitThreads = 256;
 constexpr int kRowsInFlight = 4;
 
 struct PairInfo {
-  long long base;  // first cache row of the segment
-  int len;         // rows to attend over (rho + 1), 0 if the append was refused
+  long long base;  // first cache row attended over
+  int len;         // rows to attend over (rho + 1, or the last `window` of them), 0 if the append was refused
   int seg;
+  int new_len;     // the segment's length after the append (rho + 1)
 };
 
 template <int D>
@@ -43,7 +44,7 @@ __global__ void decode_append_kernel(const int32_t* __restrict__ topk_head, cons
                                      const int32_t* __restrict__ seg_cap, long long cache_rows, RopeTable tab,
                                      float* __restrict__ q_rot, PairInfo* __restrict__ info,
                                      uint32_t* __restrict__ status, const int64_t* __restrict__ token_pos,
-                                     int interleaved) {
+                                     int interleaved, int window) {
   constexpr int HALF = D / 2;
   const int pair = blockIdx.x;  // b * Kr + slot
   const int b = pair / Kr;
@@ -54,10 +55,13 @@ __global__ void decode_append_kernel(const int32_t* __restrict__ topk_head, cons
   const long long base = seg_base[s];
   const bool room = rho >= 0 && rho < seg_cap[s] && base + rho < cache_rows && base >= 0;
   if (lane == 0) {
+    // a sliding window attends over the last `window` rows, the new one included
+    const int first = (window > 0 && rho + 1 > window) ? rho + 1 - window : 0;
     PairInfo pi;
-    pi.base = base;
-    pi.len = room ? rho + 1 : 0;
+    pi.base = base + first;
+    pi.len = room ? rho + 1 - first : 0;
     pi.seg = s;
+    pi.new_len = rho + 1;
     info[pair] = pi;
     if (!room) report(status, NAMOH_DEV_CAPACITY);
   }
@@ -269,7 +273,7 @@ __global__ void decode_merge_kernel(const PairInfo* __restrict__ info, const flo
     const __nv_bfloat16 o = __float2bfloat16_rn(out);
     y[((size_t)pair * g + j) * D + d] = *reinterpret_cast<const uint16_t*>(&o);
   }
-  if (threadIdx.x == 0 && pi.len > 0) seg_len[pi.seg] = pi.len;
+  if (threadIdx.x == 0 && pi.len > 0) seg_len[pi.seg] = pi.new_len;
 }
 
 struct DecodeWs {
@@ -330,12 +334,14 @@ extern "C" size_t namoh_decode_workspace_size(int B, int H, int K, int d_head, i
   return align_up(ws.used, 256);
 }
 
-extern "C" int namoh_decode_ex(const int32_t* topk_head, const float* gate, const uint16_t* q, const uint16_t* k,
-                               const uint16_t* v, int B, int H, int K, int d_head, int group, float rope_base,
-                               unsigned rope_flags, const int64_t* token_pos, uint16_t* k_cache, uint16_t* v_cache,
-                               const int64_t* seg_base, int32_t* seg_len, const int32_t* seg_cap, int64_t cache_rows,
-                               uint16_t* y, void* workspace, size_t workspace_bytes, uint32_t* dev_status,
-                               void* stream_v) {
+namespace namoh {
+namespace {
+// The body of namoh_decode_ex and namoh_shared_decode; window 0 attends over every row.
+int decode_impl(const int32_t* topk_head, const float* gate, const uint16_t* q, const uint16_t* k, const uint16_t* v,
+                int B, int H, int K, int d_head, int group, float rope_base, unsigned rope_flags,
+                const int64_t* token_pos, int window, uint16_t* k_cache, uint16_t* v_cache, const int64_t* seg_base,
+                int32_t* seg_len, const int32_t* seg_cap, int64_t cache_rows, uint16_t* y, void* workspace,
+                size_t workspace_bytes, uint32_t* dev_status, void* stream_v) {
   if (!topk_head || !gate || !q || !k || !v || !k_cache || !v_cache || !seg_base || !seg_len || !seg_cap || !y ||
       !dev_status)
     return NAMOH_ERR_INVALID_ARG;
@@ -364,11 +370,11 @@ extern "C" int namoh_decode_ex(const int32_t* topk_head, const float* gate, cons
   if (D == 128)
     decode_append_kernel<128><<<pairs, 32, 0, stream>>>(topk_head, q, k, v, Hr, Kr, g, k_cache, v_cache, seg_base,
                                                         seg_len, seg_cap, cache_rows, tab, dw.q_rot, dw.info,
-                                                        dev_status, token_pos, interleaved);
+                                                        dev_status, token_pos, interleaved, window);
   else
     decode_append_kernel<64><<<pairs, 32, 0, stream>>>(topk_head, q, k, v, Hr, Kr, g, k_cache, v_cache, seg_base,
                                                        seg_len, seg_cap, cache_rows, tab, dw.q_rot, dw.info,
-                                                       dev_status, token_pos, interleaved);
+                                                       dev_status, token_pos, interleaved, window);
   if (const int st = cuda_check_launch("decode_append_kernel launch")) return st;
 
   const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)D));
@@ -385,6 +391,54 @@ extern "C" int namoh_decode_ex(const int32_t* topk_head, const float* gate, cons
     decode_merge_kernel<64><<<pairs, mthreads, 0, stream>>>(dw.info, gate, dw.part, splits, g, y, seg_len);
   if (const int st = cuda_check_launch("decode_merge_kernel launch")) return st;
   return NAMOH_OK;
+}
+
+__global__ void all_heads_kernel(int B, int Hs, int32_t* __restrict__ topk_head, float* __restrict__ gate) {
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < B * Hs; i += gridDim.x * blockDim.x) {
+    topk_head[i] = i % Hs;
+    gate[i] = 1.f;
+  }
+}
+}  // namespace
+}  // namespace namoh
+
+extern "C" int namoh_decode_ex(const int32_t* topk_head, const float* gate, const uint16_t* q, const uint16_t* k,
+                               const uint16_t* v, int B, int H, int K, int d_head, int group, float rope_base,
+                               unsigned rope_flags, const int64_t* token_pos, uint16_t* k_cache, uint16_t* v_cache,
+                               const int64_t* seg_base, int32_t* seg_len, const int32_t* seg_cap, int64_t cache_rows,
+                               uint16_t* y, void* workspace, size_t workspace_bytes, uint32_t* dev_status,
+                               void* stream_v) {
+  return decode_impl(topk_head, gate, q, k, v, B, H, K, d_head, group, rope_base, rope_flags, token_pos, 0, k_cache,
+                     v_cache, seg_base, seg_len, seg_cap, cache_rows, y, workspace, workspace_bytes, dev_status,
+                     stream_v);
+}
+
+extern "C" size_t namoh_shared_decode_workspace_size(int B, int Hs, int d_head) {
+  const size_t base = namoh_decode_workspace_size(B, Hs, Hs, d_head, 1);
+  if (base == 0) return 0;
+  return base + align_up((size_t)B * Hs * sizeof(int32_t), 256) + align_up((size_t)B * Hs * sizeof(float), 256);
+}
+
+extern "C" int namoh_shared_decode(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int Hs, int d_head,
+                                   int window, float rope_base, unsigned rope_flags, uint16_t* k_cache,
+                                   uint16_t* v_cache, const int64_t* seg_base, int32_t* seg_len,
+                                   const int32_t* seg_cap, int64_t cache_rows, uint16_t* y, void* workspace,
+                                   size_t workspace_bytes, uint32_t* dev_status, void* stream_v) {
+  if (window < 0 || (rope_flags & NAMOH_ROPE_GLOBAL)) return NAMOH_ERR_INVALID_ARG;
+  const size_t need = namoh_shared_decode_workspace_size(B, Hs, d_head);
+  if (need == 0) return NAMOH_ERR_INVALID_ARG;
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) || workspace_bytes < need)
+    return NAMOH_ERR_WORKSPACE;
+  const size_t base = namoh_decode_workspace_size(B, Hs, Hs, d_head, 1);
+  int32_t* topk = reinterpret_cast<int32_t*>(static_cast<char*>(workspace) + base);
+  float* gate = reinterpret_cast<float*>(static_cast<char*>(workspace) + base +
+                                         align_up((size_t)B * Hs * sizeof(int32_t), 256));
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
+  all_heads_kernel<<<(B * Hs + 255) / 256, 256, 0, stream>>>(B, Hs, topk, gate);
+  if (const int st = cuda_check_launch("all_heads_kernel launch")) return st;
+  // positions: the rank (every token of a shared head is in its segment, so the rank is t)
+  return decode_impl(topk, gate, q, k, v, B, Hs, Hs, d_head, 1, rope_base, rope_flags, nullptr, window, k_cache,
+                     v_cache, seg_base, seg_len, seg_cap, cache_rows, y, workspace, base, dev_status, stream_v);
 }
 
 extern "C" int namoh_decode(const int32_t* topk_head, const float* gate, const uint16_t* q, const uint16_t* k,

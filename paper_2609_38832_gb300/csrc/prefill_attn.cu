@@ -107,6 +107,7 @@ struct Params {
   int* sched;                  // [0] next item, [1] CTAs finished
   uint16_t* y;                 // [R * g, D] indexed by row_src * g + j
   int rows;                    // R: a row_src value at or above it is skipped (inconsistent layout)
+  int window;                  // 0: causal over the whole segment; w > 0: the last w keys only
   int g;
   int y_sector_aligned;        // y is 32-byte aligned: rows go out as whole 32-byte sectors
   float scale_log2;            // log2(e) / sqrt(D)
@@ -118,6 +119,12 @@ struct Params {
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, uint32_t* status) {
   const bool ok = mbar_wait(bar, parity, abort_flag, status);
   return __all_sync(0xffffffffu, ok);
+}
+
+// First key tile of query tile qt: 0, or under a sliding window of w keys the tile holding key
+// qt*BM - w + 1 (the earliest key the tile's first query sees).  Every role uses this.
+__device__ __forceinline__ int first_key_tile(int qt, int window) {
+  return window > 0 ? max(0, (qt * BM - window + 1) / BN) : 0;
 }
 
 // Consumer side of the item ring: every lane waits, reads the item, one lane releases the slot.
@@ -141,10 +148,11 @@ __device__ __forceinline__ bool take_item(Bars* bars, uint32_t idx, int4* item, 
 // as bf16 over the first half of the S columns, and O rescaled when the max moved (after
 // PV(tile - 1) completed, through wait_pv).  Returns false when a wait gave up.  Ends with the
 // TMEM stores complete and fenced for the arrive on p_full.
+// kv_rel is the tile's index within the item (0 = first), kv its index in the segment.
 template <int D, typename WaitPv>
-__device__ __forceinline__ bool softmax_tile(uint32_t s_addr, uint32_t o_addr, int kv, int qt, int row,
-                                             float scale_log2, float& m_use, float& l_sum, uint32_t tile,
-                                             WaitPv&& wait_pv) {
+__device__ __forceinline__ bool softmax_tile(uint32_t s_addr, uint32_t o_addr, int kv_rel, int kv, int qt, int row,
+                                             int window, float scale_log2, float& m_use, float& l_sum,
+                                             uint32_t tile, WaitPv&& wait_pv) {
   float sv[BN];
 #pragma unroll
   for (int c = 0; c < BN / 32; ++c) {
@@ -154,6 +162,13 @@ __device__ __forceinline__ bool softmax_tile(uint32_t s_addr, uint32_t o_addr, i
     for (int i = 0; i < 32; ++i) sv[c * 32 + i] = __uint_as_float(r[i]);
   }
   tmem_wait_ld();
+  // sliding window: keys older than query rank - window + 1 are out
+  if (window > 0) {
+    const int lo = qt * BM + row - window + 1 - kv * BN;  // first column in the window
+#pragma unroll
+    for (int c = 0; c < BN; ++c)
+      if (c < lo) sv[c] = -INFINITY;
+  }
   // causal mask on the diagonal tile: key rank kv*BN + c <= query rank
   if (kv == qt) {
 #pragma unroll
@@ -173,10 +188,12 @@ __device__ __forceinline__ bool softmax_tile(uint32_t s_addr, uint32_t o_addr, i
 #pragma unroll
   for (int i = 0; i < 8; ++i) m8[i] = fmaxf(m8[i], sv[120 + i]);
   const float mx = fmax3(fmax3(m8[0], m8[1], m8[2]), fmax3(m8[3], m8[4], m8[5]), fmaxf(m8[6], m8[7]));
-  const float m_tile = mx * scale_log2;
+  // a row with every key of the tile outside the window gets a finite floor, so that its
+  // P is exactly 0 and the next tile's rescale factor exp2(m_use - m_tile) is 0
+  const float m_tile = window > 0 ? fmaxf(mx * scale_log2, -1e30f) : mx * scale_log2;
   float alpha = 1.f;
   bool rescale = false;
-  if (kv == 0) {
+  if (kv_rel == 0) {
     m_use = m_tile;
   } else if (m_tile > m_use + kRescaleThreshold) {
     alpha = fast_exp2(m_use - m_tile);
@@ -210,7 +227,7 @@ __device__ __forceinline__ bool softmax_tile(uint32_t s_addr, uint32_t o_addr, i
   }
   // O may only be rescaled once the previous PV completed; without a rescale this
   // tile's softmax does not touch O and overlaps that PV
-  if (kv > 0 && __any_sync(0xffffffffu, rescale)) {
+  if (kv_rel > 0 && __any_sync(0xffffffffu, rescale)) {
     if (!wait_pv(tile - 1)) return false;
     tc_fence_after();
     {
@@ -318,7 +335,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (item.x < 0) break;
         const int j = item.x % p.g, qt = item.y;
         const int off = item.z;
-        const int nkv = qt + 1;
+        const int kv0 = first_key_tile(qt, p.window);
+        const int nkv = qt + 1 - kv0;
+        kvb += kv0 * BN;  // the item's first key tile
         if (item_iter > 0) ok = mbar_wait(&bars->q_empty, (item_iter - 1) & 1, abort_flag, p.status);
         if (!ok) break;
         mbar_arrive_expect_tx(&bars->q_full, L::kTileBytes);
@@ -381,8 +400,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       int4 item;
       ok = take_item(bars, item_iter, &item, abort_flag, p.status);
       if (!ok || item.x < 0) break;
-      const int qt = item.y, n = item.w;
-      const int nkv = qt + 1;
+      const int qt = item.y;
+      const int kv0 = first_key_tile(qt, p.window);
+      const int nkv = qt + 1 - kv0;
+      const int n = item.w - kv0 * BN;  // keys from the item's first key tile to the segment's end
       // ring entries of this item, in load order: K(0), K(1) if nkv > 1, then for each kv:
       // V(kv) followed by K(kv+2) while kv + 2 < nkv
       const uint32_t rk0 = ring_iter, rk1 = ring_iter + 1;
@@ -432,7 +453,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = ring_ready2(r_v, r_k2) &&
            (item_iter == 0 || warp_wait(&bars->o_free, (item_iter - 1) & 1, abort_flag, p.status)) && p_ready(p_iter);
       if (!ok) break;
-      if (n < BN) zero_v_tail(r_v, n);  // a one-tile item whose only tile is partial
+      if (n < BN) zero_v_tail(r_v, n);  // the item's first key tile is the segment's last, partial one
 
       // Everything a step needs besides its commits and P(kv+1) -- the next step's ring
       // entries, their waits, a partial last V tile -- is done in the middle of the burst,
@@ -522,17 +543,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (valid) src = ld_issue_s32(p.row_src + off + qrank);
       float gt = 0.f;
       float m_use = 0.f, l_sum = 0.f;
-      for (int kv = 0; kv <= qt && ok; ++kv) {
+      const int kv0 = first_key_tile(qt, p.window);
+      for (int kv = kv0; kv <= qt && ok; ++kv) {
         const uint32_t s_addr = tmem + lane_addr + tmem_s_col((int)(s_iter % kSBufs));
         ok = warp_wait(&bars->s_full[s_iter % kSBufs], (s_iter / kSBufs) & 1, abort_flag, p.status);
         const uint32_t tile = s_iter++;
         if (!ok) break;
         tc_fence_after();
-        ok = softmax_tile<D>(s_addr, o_addr, kv, qt, row, p.scale_log2, m_use, l_sum, tile, wait_pv);
+        ok = softmax_tile<D>(s_addr, o_addr, kv - kv0, kv, qt, row, p.window, p.scale_log2, m_use, l_sum, tile,
+                             wait_pv);
         if (!ok) break;
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars->p_full[tile & 1]);
-        if (kv == 0 && valid) {  // the gate, used in the epilogue only
+        if (kv == kv0 && valid) {  // the gate, used in the epilogue only
           if ((unsigned)src < (unsigned)p.rows) gt = ld_issue_f32(p.gate + src);
           else src = -1;
         }
@@ -708,7 +731,7 @@ int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v
 int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint16_t* v_cache, long long R, int D,
                      int g, const int32_t* seg_offsets, const int32_t* row_src, const float* gate,
                      const int64_t* seg_base, long long cache_rows, void* plan, uint16_t* y, uint32_t* dev_status,
-                     const DeviceInfo& info, cudaStream_t stream) {
+                     const DeviceInfo& info, cudaStream_t stream, int window = 0) {
   CUtensorMap tq, tk, tv;
   if (!attn::encode_rows_map(&tq, q_rot, R, g * D) || !attn::encode_rows_map(&tk, k_cache, cache_rows, D) ||
       !attn::encode_rows_map(&tv, v_cache, cache_rows, D))
@@ -723,6 +746,7 @@ int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint1
   p.items = reinterpret_cast<const int4*>(static_cast<char*>(plan) + 16);
   p.y = y;
   p.rows = (int)R;
+  p.window = window;
   p.g = g;
   p.y_sector_aligned = (reinterpret_cast<uintptr_t>(y) & 31u) == 0;
   p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)D));
@@ -939,4 +963,94 @@ extern "C" int namoh_prefill(const uint16_t* q, const uint16_t* k, const uint16_
   return namoh_prefill_ex(q, k, v, B, T, H, K, d_head, group, rope_base, 0u, seg_offsets, row_src, gate, y, k_cache,
                           v_cache, seg_base, seg_cap, cache_rows, seg_len, workspace, workspace_bytes, dev_status,
                           stream_v);
+}
+
+// ---------------------------------------------------------------------------
+// Shared heads (the paper's shared-head variant): every token of each always-active head,
+// full causal or sliding window, global RoPE (the rank in a segment holding every token is
+// t), no gate.  The layout is the identity one: segment (b, j) = rows (b Hs + j) T .. + T.
+// ---------------------------------------------------------------------------
+namespace namoh {
+namespace {
+__global__ void shared_layout_kernel(int B, int T, int Hs, int32_t* __restrict__ seg_offsets,
+                                     int32_t* __restrict__ row_src, float* __restrict__ gate) {
+  const long long R = (long long)B * Hs * T;
+  for (long long r = blockIdx.x * (long long)blockDim.x + threadIdx.x; r < R; r += (long long)gridDim.x * blockDim.x) {
+    const long long bj = r / T, t = r - bj * T;
+    const long long b = bj / Hs, j = bj - b * Hs;
+    row_src[r] = (int32_t)((b * T + t) * Hs + j);  // y is [B, T, Hs, d]
+    gate[r] = 1.f;
+    if (t == 0) seg_offsets[bj] = (int32_t)r;
+    if (r == R - 1) seg_offsets[B * Hs] = (int32_t)R;
+  }
+}
+
+struct SharedWs {
+  int32_t *seg_offsets, *row_src;
+  float* gate;
+  uint16_t* q_rot;
+  void* plan;
+};
+void carve_shared(WorkspaceCarver& ws, SharedWs* o, int B, int T, int Hs, int d_head) {
+  const long long R = (long long)B * Hs * T;
+  o->seg_offsets = ws.take<int32_t>((size_t)B * Hs + 1);
+  o->row_src = ws.take<int32_t>((size_t)R);
+  o->gate = ws.take<float>((size_t)R);
+  o->q_rot = ws.take<uint16_t>((size_t)R * d_head);
+  o->plan = ws.take<char>(plan_bytes_rows(R, B * Hs, 1));
+}
+}  // namespace
+}  // namespace namoh
+
+extern "C" size_t namoh_shared_workspace_size(int B, int T, int Hs, int d_head) {
+  int Hr, Kr;
+  long long R;
+  if (check_shape(B, T, Hs, Hs, d_head, 1, &Hr, &Kr, &R) != NAMOH_OK) return 0;
+  WorkspaceCarver ws{nullptr, 0, 0};
+  SharedWs o;
+  carve_shared(ws, &o, B, T, Hs, d_head);
+  return align_up(ws.used, 256);
+}
+
+extern "C" int namoh_shared_prefill(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int Hs,
+                                    int d_head, int window, float rope_base, unsigned rope_flags, uint16_t* y,
+                                    uint16_t* k_cache, uint16_t* v_cache, const int64_t* seg_base,
+                                    const int32_t* seg_cap, int64_t cache_rows, int32_t* seg_len, void* workspace,
+                                    size_t workspace_bytes, uint32_t* dev_status, void* stream_v) {
+  if (!q || !k || !v || !y || !k_cache || !v_cache || !dev_status) return NAMOH_ERR_INVALID_ARG;
+  int Hr, Kr;
+  long long R;
+  int st = check_shape(B, T, Hs, Hs, d_head, 1, &Hr, &Kr, &R);
+  if (st != NAMOH_OK) return st;
+  if (window < 0 || !(rope_base > 1.0f) || !isfinite(rope_base) || !rope_flags_ok(rope_flags))
+    return NAMOH_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(y) || !aligned16(k_cache) || !aligned16(v_cache))
+    return NAMOH_ERR_INVALID_ARG;
+  if (k_cache == k) return NAMOH_ERR_INVALID_ARG;
+  if (seg_base) {
+    if (!seg_cap || cache_rows < 1 || cache_rows >= (1ll << 31) || v_cache == v) return NAMOH_ERR_INVALID_ARG;
+  } else {
+    cache_rows = R;
+  }
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return NAMOH_ERR_WORKSPACE;
+  WorkspaceCarver ws{static_cast<char*>(workspace), workspace_bytes, 0};
+  SharedWs o;
+  carve_shared(ws, &o, B, T, Hs, d_head);
+  if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
+  DeviceInfo info;
+  if (!device_ok(&info)) return NAMOH_ERR_UNSUPPORTED;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
+  shared_layout_kernel<<<info.sm_count * 4, 256, 0, stream>>>(B, T, Hs, o.seg_offsets, o.row_src, o.gate);
+  if (const int e = cuda_check_launch("shared_layout_kernel launch")) return e;
+  // global positions: the rank in a segment holding every token is t (the global flag is redundant)
+  st = launch_rope_and_plan(q, k, v, B, T, Hs, Hs, (int)R, d_head, 1, rope_base, rope_flags & NAMOH_ROPE_INTERLEAVED,
+                            nullptr, o.seg_offsets, o.row_src, o.q_rot, k_cache, v_cache, seg_base, seg_cap,
+                            cache_rows, dev_status, o.plan, info, stream);
+  if (st != NAMOH_OK) return st;
+  if (seg_len) {
+    seg_len_kernel<<<(B * Hs + 255) / 256, 256, 0, stream>>>(o.seg_offsets, B * Hs, seg_len);
+    if (const int e = cuda_check_launch("seg_len_kernel launch")) return e;
+  }
+  return launch_attention(o.q_rot, k_cache, v_cache, R, d_head, 1, o.seg_offsets, o.row_src, o.gate, seg_base,
+                          cache_rows, o.plan, y, dev_status, info, stream, window);
 }
