@@ -398,6 +398,8 @@ def run_gpu(args, rank: int, world: int):
     if not args.no_layer:
         line["layer"] = run_layer(args, dev, pk, pk_kind)
         line["gpu_launches"] += line["layer"].pop("launches")
+        line["shared_heads"] = run_shared(args, dev, pk, pk_kind)
+        line["gpu_launches"] += line["shared_heads"].pop("launches")
     clocks.__exit__(None, None, None)
     line["clocks"] = clocks.summary()
     return line
@@ -466,6 +468,10 @@ def run_layer(args, dev, pk, pk_kind):
 
     step()
     torch.cuda.synchronize()
+    # the output projection runs one product-and-combine pair per token chunk of at most 1 GB of
+    # bf16 per-slot products (the library's chunking)
+    out_chunk = min(N, max(128, (1 << 30) // (Kr * d_model * 2)))
+    out_launches = 2 + 2 * (-(-N // out_chunk))
     n_seg = acc.segment_lengths(ro.seg_offsets.cpu().numpy())
     f_attn = acc.attention_flops(n_seg, d, g)
     f_qkv = 2.0 * R * d_model * (g + 2) * d
@@ -486,10 +492,51 @@ def run_layer(args, dev, pk, pk_kind):
         "peak_source": f"{pk_kind} bf16 dense (burst)",
         "l2": "flushed before every timed launch sequence (2 GB write)",
         "device_status": int(status.item()),
-        # timed launches: QKV (tile list + GEMM), OUT (tile list, GEMM, combine), and the step
-        # (route 2 + QKV 2 + prefill 2 + OUT 3)
-        "launches": args.steps * (2 + 3 + 9),
+        # timed launches: QKV (range table, tile list, GEMM), OUT (range table, tile list, then a
+        # GEMM and a combine per chunk), and the step (route 2 + QKV 3 + prefill 2 + OUT)
+        "launches": args.steps * (3 + out_launches + (2 + 3 + 2 + out_launches)),
     }
+
+
+def run_shared(args, dev, pk, pk_kind):
+    """Shared heads at the balanced workload's sizes (B4 T4096 d128), Hs = 4: the paper's
+    sliding window of 128 tokens and the full causal prefix (namoh_shared_prefill), L2 flushed
+    before every timed launch.  Flops: 4 d per causal (query, key) pair inside the window."""
+    import torch
+
+    import paper_2609_38832_gb300 as namoh
+
+    B, T, Hs, d = 4, 4096, 4, 128
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(7)
+    q, k, v = (torch.randn((B, Hs, T, d), generator=gen, device=dev).to(torch.bfloat16) for _ in range(3))
+    y = torch.empty((B, T, Hs, d), dtype=torch.bfloat16, device=dev)
+    k_cache = torch.empty((B * Hs * T, d), dtype=torch.bfloat16, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    ws = namoh.Workspace()
+    flush = torch.empty(2 << 30, dtype=torch.uint8, device=dev)
+    out = {"workload": f"B{B} T{T} Hs{Hs} d{d}, bf16 N(0,1) inputs", "peak_source": f"{pk_kind} bf16 dense (burst)"}
+    for name, window in (("window_128", 128), ("full_prefix", 0)):
+        def run():
+            namoh.namoh_shared_prefill(q, k, v, window=window, y=y, k_cache=k_cache, workspace=ws, status=status)
+
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+        for i in range(args.warmup + args.steps):
+            flush.fill_(i & 0xFF)
+            if i >= args.warmup:
+                evs[i - args.warmup][0].record()
+            run()
+            if i >= args.warmup:
+                evs[i - args.warmup][1].record()
+        torch.cuda.synchronize()
+        ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
+        pairs = B * Hs * sum(min(t + 1, window) if window else t + 1 for t in range(T))
+        flops = 4.0 * d * pairs
+        tf = flops / (ms * 1e-3) / 1e12
+        out[name] = {"ms": ms, "tflops": tf, "frac_bf16": tf / pk["bf16_tflops"], "flops": flops}
+    out["device_status"] = int(status.item())
+    out["launches"] = 2 * args.steps * 3  # layout, RoPE + plan, attention per call
+    return out
 
 
 def run_decode(args, dev, pk, pk_kind):

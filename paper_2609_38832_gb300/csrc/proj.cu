@@ -28,6 +28,8 @@
 // the loaders fetch the next item's row indices during the current one.
 // Two TMEM accumulators let the epilogue of one item overlap the main loop of the next.
 // Every wait is bounded (NAMOH_DEV_TIMEOUT).
+#include <algorithm>
+
 #include "common.cuh"
 
 namespace namoh {
@@ -54,9 +56,9 @@ struct Layout {
 };
 
 struct Params {
-  const int32_t* seg_offsets;  // [nseg + 1]
-  const int2* tiles;           // {segment, tile index in it}, in work order
-  const int32_t* ntiles;       // [1]: length of the list
+  const int4* tiles;           // {first row, rows, segment, 0}: the 128-row tiles, in work order
+  const int32_t* tile_off;     // the list's first entry for this launch
+  const int32_t* ntiles;       // the number of entries for this launch
   const int32_t* row_src;      // [R]
   int nseg, Hr, Kr;
   int a_rows;                  // tokens (rows of x)
@@ -66,6 +68,8 @@ struct Params {
   const void* a;               // x [a_rows, kdim] (QKV), y [a_rows = N*Kr, g d] (OUT_P)
   uint16_t *q, *k, *v;         // outputs (OUT_P: q = P [a_rows, ncols])
   int out_aligned32;           // q, k, v 32-byte aligned: whole-sector stores
+  long long p_row0;            // OUT_P: P row of token-slot row t Kr + k is t Kr + k - p_row0
+  long long p_rows;            // OUT_P: rows of P
   uint32_t* status;
 };
 
@@ -80,13 +84,12 @@ struct Tile {
   int seg, row0, rows, hr, nt;
 };
 
-// Row tile -> its segment, first row and rows.
-__device__ __forceinline__ Tile decode_tile(const Params& p, int2 st) {
+__device__ __forceinline__ Tile decode_tile(const Params& p, int4 e) {
   Tile t;
-  t.seg = st.x;
-  t.row0 = __ldg(p.seg_offsets + st.x) + st.y * BM;
-  t.rows = min(BM, __ldg(p.seg_offsets + st.x + 1) - t.row0);
-  t.hr = st.x % p.Hr;
+  t.row0 = e.x;
+  t.rows = e.y;
+  t.seg = e.z;
+  t.hr = e.z % p.Hr;
   t.nt = 0;
   return t;
 }
@@ -106,37 +109,75 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-// The row-tile list in work order (one block).  Sequence b's tiles come before b + 1's; inside
-// a sequence, tile p of every head before tile p + 1 of any, heads in order.  Tile (b, p, h)
-// lands at  (tiles of sequences before b) + sum_h' min(p, n_tiles(b, h')) + #{h' < h : n_tiles(b, h') > p}.
-__global__ void __launch_bounds__(1024) tile_list_kernel(const int32_t* __restrict__ seg_offsets, int nseg, int Hr,
-                                                         int2* __restrict__ tiles, int32_t* __restrict__ ntiles) {
+// Row ranges of the segments per token chunk: lo[c][s] = the first row of segment s whose token
+// is >= c * chunk (rows ascend in token inside a segment); lo[nchunk][s] = the segment's end.
+// With one chunk these are the segments' bounds.
+__global__ void range_table_kernel(const int32_t* __restrict__ seg_offsets, const int32_t* __restrict__ row_src,
+                                   int nseg, int nchunk, long long chunk, int Kr, int32_t* __restrict__ lo_tab) {
+  const long long n = (long long)(nchunk + 1) * nseg;
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+    const int c = (int)(i / nseg), s = (int)(i - (long long)c * nseg);
+    const int a = __ldg(seg_offsets + s), e = max(a, __ldg(seg_offsets + s + 1));
+    int lo = a, hi = e;
+    if (c == nchunk) {
+      lo = e;
+    } else if (c > 0) {
+      const long long target = (long long)c * chunk;
+      while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if ((long long)(__ldg(row_src + mid) / Kr) < target) lo = mid + 1; else hi = mid;
+      }
+    }
+    lo_tab[i] = lo;
+  }
+}
+
+// The row-tile list (one block), chunk by chunk.  Inside a chunk: sequence b's tiles before
+// b + 1's; tile p of every head before tile p + 1 of any, heads in order.  Tile (b, p, h) lands at
+//   (tiles of sequences before b) + sum_h' min(p, n_tiles(b, h')) + #{h' < h : n_tiles(b, h') > p}.
+// chunk_off[c] / chunk_cnt[c]: the chunk's first entry and its number of entries.
+__global__ void __launch_bounds__(1024) tile_list_kernel(const int32_t* __restrict__ lo_tab, int nseg, int Hr,
+                                                         int nchunk, int4* __restrict__ tiles,
+                                                         int32_t* __restrict__ chunk_off,
+                                                         int32_t* __restrict__ chunk_cnt) {
   extern __shared__ int s_nt[];  // [nseg] tiles per segment, then [nseg / Hr] per-sequence bases
   int* s_base = s_nt + nseg;
+  __shared__ int s_total;
   const int B = nseg / Hr;
   const int tid = threadIdx.x;
-  for (int s = tid; s < nseg; s += blockDim.x) {
-    const int n = __ldg(seg_offsets + s + 1) - __ldg(seg_offsets + s);
-    s_nt[s] = n > 0 ? (n + BM - 1) / BM : 0;
-  }
-  __syncthreads();
-  if (tid == 0) {
-    int run = 0;
-    for (int b = 0; b < B; ++b) {
-      s_base[b] = run;
-      for (int h = 0; h < Hr; ++h) run += s_nt[b * Hr + h];
+  int done = 0;
+  for (int c = 0; c < nchunk; ++c) {
+    const int32_t* lo = lo_tab + (long long)c * nseg;
+    const int32_t* hi = lo + nseg;
+    for (int s = tid; s < nseg; s += blockDim.x) {
+      const int n = __ldg(hi + s) - __ldg(lo + s);
+      s_nt[s] = n > 0 ? (n + BM - 1) / BM : 0;
     }
-    *ntiles = run;
-  }
-  __syncthreads();
-  for (int s = tid; s < nseg; s += blockDim.x) {
-    const int b = s / Hr, h = s - b * Hr;
-    const int* nt = s_nt + b * Hr;
-    for (int q = 0; q < nt[h]; ++q) {
-      int pos = s_base[b];
-      for (int h2 = 0; h2 < Hr; ++h2) pos += min(q, nt[h2]) + (h2 < h && nt[h2] > q ? 1 : 0);
-      tiles[pos] = make_int2(s, q);
+    __syncthreads();
+    if (tid == 0) {
+      int run = 0;
+      for (int b = 0; b < B; ++b) {
+        s_base[b] = run;
+        for (int h = 0; h < Hr; ++h) run += s_nt[b * Hr + h];
+      }
+      chunk_off[c] = done;
+      chunk_cnt[c] = run;
+      s_total = run;
     }
+    __syncthreads();
+    for (int s = tid; s < nseg; s += blockDim.x) {
+      const int b = s / Hr, h = s - b * Hr;
+      const int* nt = s_nt + b * Hr;
+      const int r0 = __ldg(lo + s), r1 = __ldg(hi + s);
+      for (int q = 0; q < nt[h]; ++q) {
+        int pos = s_base[b];
+        for (int h2 = 0; h2 < Hr; ++h2) pos += min(q, nt[h2]) + (h2 < h && nt[h2] > q ? 1 : 0);
+        const int row0 = r0 + q * BM;
+        tiles[done + pos] = make_int4(row0, min(BM, r1 - row0), s, 0);
+      }
+    }
+    done += s_total;
+    __syncthreads();
   }
 }
 
@@ -179,6 +220,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
   // before the next (the tile's rows are decoded once and re-gathered from L2).
   const int nt_count = p.ncols / BN;
   const int ntiles = __ldg(p.ntiles);
+  const int4* tiles = p.tiles + __ldg(p.tile_off);
   const int nk = p.kdim / BK;
 
   if (warp >= 4 && warp < 8) {
@@ -199,7 +241,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     Tile t{};
     int rows_a[8];
     if (mt < ntiles) {
-      t = decode_tile(p, __ldg(p.tiles + mt));
+      t = decode_tile(p, __ldg(tiles + mt));
 #pragma unroll
       for (int w = 0; w < 8; ++w) {
         const int r = rq + 16 * w;
@@ -211,7 +253,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     const bool prefetch = nt_count * nk >= 12;
     for (; mt < ntiles && ok; mt += gridDim.x) {
       const int next = mt + gridDim.x;
-      int nx_seg = 0, nx_q = 0, nx_lo = 0, nx_hi = 0;
+      int nx_row0 = 0, nx_rows = 0, nx_seg = 0;
       Tile nx{};
       int nx_src[8];
       const uint16_t* src[8];
@@ -223,17 +265,12 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
         for (int kb = 0; kb < nk; ++kb, ++it, ++kq) {
           if (prefetch && next < ntiles) {
             if (kq == 0) {
-              const int32_t* e = reinterpret_cast<const int32_t*>(p.tiles + next);
-              nx_seg = ld_issue_s32(e);
-              nx_q = ld_issue_s32(e + 1);
+              const int32_t* e = reinterpret_cast<const int32_t*>(tiles + next);
+              nx_row0 = ld_issue_s32(e);
+              nx_rows = ld_issue_s32(e + 1);
+              nx_seg = ld_issue_s32(e + 2);
             } else if (kq == 4) {
-              nx_lo = ld_issue_s32(p.seg_offsets + nx_seg);
-              nx_hi = ld_issue_s32(p.seg_offsets + nx_seg + 1);
-            } else if (kq == 8) {
-              nx.seg = nx_seg;
-              nx.row0 = nx_lo + nx_q * BM;
-              nx.rows = min(BM, nx_hi - nx.row0);
-              nx.hr = nx_seg % p.Hr;
+              nx = decode_tile(p, make_int4(nx_row0, nx_rows, nx_seg, 0));
 #pragma unroll
               for (int w = 0; w < 8; ++w) {
                 const int r = rq + 16 * w;
@@ -270,7 +307,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
 #pragma unroll
         for (int w = 0; w < 8; ++w) rows_a[w] = a_row_of(nx_src[w]);
       } else {
-        t = decode_tile(p, __ldg(p.tiles + next));
+        t = decode_tile(p, __ldg(tiles + next));
 #pragma unroll
         for (int w = 0; w < 8; ++w) {
           const int r = rq + 16 * w;
@@ -323,11 +360,11 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     int li = 0;
     bool ok = true;
     for (int mt = blockIdx.x; mt < ntiles && ok; mt += gridDim.x) {
-      const Tile t = decode_tile(p, __ldg(p.tiles + mt));
+      const Tile t = decode_tile(p, __ldg(tiles + mt));
       const bool valid = row < t.rows;
       const int r = t.row0 + row;
       // OUT_P writes row r's partial product at its token-slot row row_src[r]
-      const int dst_row = kMode == kOutP && valid ? ld_issue_s32(p.row_src + r) : r;
+      const long long dst_row = kMode == kOutP && valid ? ld_issue_s32(p.row_src + r) - p.p_row0 : r;
       for (int nt = 0; nt < nt_count; ++nt, ++li) {
         const int buf = li & 1;
         if (!warp_wait(&bars->acc_full[buf], (li >> 1) & 1, abort_flag, p.status)) {
@@ -349,7 +386,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
             else if (n < gd + p.d) dst = p.k + (long long)r * p.d + (n - gd);
             else dst = p.v + (long long)r * p.d + (n - gd - p.d);
           } else {
-            if (dst_row < 0 || dst_row >= p.a_rows) continue;  // an inconsistent layout
+            if (dst_row < 0 || dst_row >= p.p_rows) continue;  // an inconsistent layout
             dst = p.q + (long long)dst_row * p.ncols + n;
           }
           uint32_t w[16];
@@ -482,40 +519,70 @@ using namespace namoh;
 
 
 namespace {
-// The row-tile list: at most ceil(R / 128) + nseg tiles, plus its length.
-size_t tile_list_bytes(long long R, int nseg) {
-  return 16 + (size_t)((R + proj::BM - 1) / proj::BM + nseg) * sizeof(int2);
+// Workspace of the tile list for nchunk token chunks: the row-range table, the tiles (at most
+// ceil(R / 128) + nchunk * nseg of them) and each chunk's offset and count.
+struct TileList {
+  int32_t* lo_tab;
+  int4* tiles;
+  int32_t *off, *cnt;
+};
+void carve_tiles(WorkspaceCarver& ws, TileList* t, long long R, int nseg, int nchunk) {
+  t->lo_tab = ws.take<int32_t>((size_t)(nchunk + 1) * nseg);
+  t->tiles = ws.take<int4>((size_t)((R + proj::BM - 1) / proj::BM + (long long)nchunk * nseg));
+  t->off = ws.take<int32_t>((size_t)nchunk);
+  t->cnt = ws.take<int32_t>((size_t)nchunk);
 }
 
-int proj_prologue(const int32_t* seg_offsets, int nseg, int Hr, long long R, void* workspace, size_t workspace_bytes,
-                  proj::Params* p, cudaStream_t stream) {
-  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return NAMOH_ERR_WORKSPACE;
-  if (workspace_bytes < tile_list_bytes(R, nseg)) return NAMOH_ERR_WORKSPACE;
-  int32_t* ntiles = static_cast<int32_t*>(workspace);
-  int2* tiles = reinterpret_cast<int2*>(static_cast<char*>(workspace) + 16);
+int build_tiles(const int32_t* seg_offsets, const int32_t* row_src, int nseg, int Hr, int Kr, int nchunk,
+                long long chunk, const TileList& t, int sm_count, cudaStream_t stream) {
+  const long long n = (long long)(nchunk + 1) * nseg;
+  proj::range_table_kernel<<<(unsigned)std::min<long long>((n + 255) / 256, sm_count * 8LL), 256, 0, stream>>>(
+      seg_offsets, row_src, nseg, nchunk, chunk, Kr, t.lo_tab);
+  if (const int st = cuda_check_launch("range_table_kernel launch")) return st;
   const int smem = (nseg + nseg / Hr) * (int)sizeof(int);
   if (smem > 48 * 1024) {
     const cudaError_t e =
         cudaFuncSetAttribute(proj::tile_list_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return cuda_fail(e, "tile_list_kernel shared memory attribute");
   }
-  proj::tile_list_kernel<<<1, 1024, smem, stream>>>(seg_offsets, nseg, Hr, tiles, ntiles);
-  p->tiles = tiles;
-  p->ntiles = ntiles;
+  proj::tile_list_kernel<<<1, 1024, smem, stream>>>(t.lo_tab, nseg, Hr, nchunk, t.tiles, t.off, t.cnt);
   return cuda_check_launch("tile_list_kernel launch");
 }
-}  // namespace
 
-// namoh_proj_out's workspace: the tile list, then P [total_tokens * Kr, d_model] bf16.
-size_t out_workspace(long long total_tokens, int Kr, int nseg, int d_model) {
-  return align_up(tile_list_bytes(total_tokens * Kr, nseg), 256) +
-         align_up((size_t)total_tokens * Kr * d_model * sizeof(uint16_t), 256);
+// The output projection's token chunks bound the per-slot products kept at once (chunk Kr d_model
+// bf16) to kOutChunkBytes of workspace.  (Chunks small enough for the products to stay in L2,
+// 64 MB, measured slower: 184 against 147 us on the balanced layer, from the tail of each chunk's
+// smaller launch.)
+constexpr size_t kOutChunkBytes = 1ull << 30;
+long long out_chunk_tokens(long long total_tokens, int Kr, int d_model) {
+  long long c = (long long)(kOutChunkBytes / ((size_t)Kr * d_model * sizeof(uint16_t)));
+  c = c < 128 ? 128 : c;
+  return c < total_tokens ? c : total_tokens;
 }
+
+size_t qkv_workspace(long long total_tokens, int Kr, int nseg) {
+  WorkspaceCarver ws{nullptr, 0, 0};
+  TileList t;
+  carve_tiles(ws, &t, total_tokens * Kr, nseg, 1);
+  return align_up(ws.used, 256);
+}
+
+size_t out_workspace(long long total_tokens, int Kr, int nseg, int d_model) {
+  const long long chunk = out_chunk_tokens(total_tokens, Kr, d_model);
+  const int nchunk = (int)((total_tokens + chunk - 1) / chunk);
+  WorkspaceCarver ws{nullptr, 0, 0};
+  TileList t;
+  carve_tiles(ws, &t, total_tokens * Kr, nseg, nchunk);
+  ws.take<uint16_t>((size_t)chunk * Kr * d_model);
+  return align_up(ws.used, 256);
+}
+}  // namespace
 
 extern "C" size_t namoh_proj_workspace_size(int B, int total_tokens, int d_model, int H, int K, int group) {
   if (B < 1 || total_tokens < 1 || d_model < 1 || group < 1 || H < 1 || K < 1 || H % group || K % group) return 0;
   const int Hr = H / group, Kr = K / group;
-  return out_workspace(total_tokens, Kr, B * Hr, d_model);  // the larger of the two calls' needs
+  const size_t a = qkv_workspace(total_tokens, Kr, B * Hr), b = out_workspace(total_tokens, Kr, B * Hr, d_model);
+  return a > b ? a : b;  // one size serves both calls
 }
 
 extern "C" int namoh_proj_qkv(const uint16_t* x, int total_tokens, int d_model, const uint16_t* w_qkv, int B, int H,
@@ -534,10 +601,17 @@ extern "C" int namoh_proj_qkv(const uint16_t* x, int total_tokens, int d_model, 
   if (!current_device_info(&info) || info.major != 10) return NAMOH_ERR_UNSUPPORTED;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
   const int nseg = B * Hr;
-  proj::Params p{};
-  st = proj_prologue(seg_offsets, nseg, Hr, (long long)total_tokens * Kr, workspace, workspace_bytes, &p, stream);
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return NAMOH_ERR_WORKSPACE;
+  WorkspaceCarver ws{static_cast<char*>(workspace), workspace_bytes, 0};
+  TileList tl;
+  carve_tiles(ws, &tl, (long long)total_tokens * Kr, nseg, 1);
+  if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
+  st = build_tiles(seg_offsets, row_src, nseg, Hr, Kr, 1, total_tokens, tl, info.sm_count, stream);
   if (st != NAMOH_OK) return st;
-  p.seg_offsets = seg_offsets;
+  proj::Params p{};
+  p.tiles = tl.tiles;
+  p.tile_off = tl.off;
+  p.ntiles = tl.cnt;
   p.row_src = row_src;
   p.nseg = nseg;
   p.Hr = Hr;
@@ -573,14 +647,19 @@ extern "C" int namoh_proj_out(const uint16_t* y, int total_tokens, int d_model, 
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
   const int nseg = B * Hr;
   const long long R = (long long)total_tokens * Kr;
-  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) ||
-      workspace_bytes < out_workspace(total_tokens, Kr, nseg, d_model))
-    return NAMOH_ERR_WORKSPACE;
-  uint16_t* P = reinterpret_cast<uint16_t*>(static_cast<char*>(workspace) + align_up(tile_list_bytes(R, nseg), 256));
-  proj::Params p{};
-  st = proj_prologue(seg_offsets, nseg, Hr, R, workspace, workspace_bytes, &p, stream);
+  // token chunks whose per-slot products stay in L2 until the combine reads them
+  const long long chunk = out_chunk_tokens(total_tokens, Kr, d_model);
+  const int nchunk = (int)((total_tokens + chunk - 1) / chunk);
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return NAMOH_ERR_WORKSPACE;
+  WorkspaceCarver ws{static_cast<char*>(workspace), workspace_bytes, 0};
+  TileList tl;
+  carve_tiles(ws, &tl, R, nseg, nchunk);
+  uint16_t* P = ws.take<uint16_t>((size_t)chunk * Kr * d_model);
+  if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
+  st = build_tiles(seg_offsets, row_src, nseg, Hr, Kr, nchunk, chunk, tl, info.sm_count, stream);
   if (st != NAMOH_OK) return st;
-  p.seg_offsets = seg_offsets;
+  proj::Params p{};
+  p.tiles = tl.tiles;
   p.row_src = row_src;
   p.nseg = nseg;
   p.Hr = Hr;
@@ -594,8 +673,17 @@ extern "C" int namoh_proj_out(const uint16_t* y, int total_tokens, int d_model, 
   p.q = P;
   p.out_aligned32 = 1;  // P starts 256-byte aligned and its rows are multiples of 128 bytes
   p.status = dev_status;
-  cudaError_t e = proj::launch<proj::kOutP>(bn, p, w_o, (long long)Hr * d_model, info.sm_count, stream);
-  if (e != cudaSuccess) return cuda_fail(e, "proj_kernel (out) launch");
-  proj::combine_kernel<<<info.sm_count * 8, 256, 0, stream>>>(P, total_tokens, Kr, d_model, o, accumulate ? 1 : 0);
-  return cuda_check_launch("combine_kernel launch");
+  for (int c = 0; c < nchunk; ++c) {
+    const long long t0 = (long long)c * chunk, nt = std::min<long long>(chunk, total_tokens - t0);
+    p.tile_off = tl.off + c;
+    p.ntiles = tl.cnt + c;
+    p.p_row0 = t0 * Kr;
+    p.p_rows = nt * Kr;
+    const cudaError_t e = proj::launch<proj::kOutP>(bn, p, w_o, (long long)Hr * d_model, info.sm_count, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "proj_kernel (out) launch");
+    proj::combine_kernel<<<info.sm_count * 8, 256, 0, stream>>>(P, nt, Kr, d_model, o + t0 * d_model,
+                                                                 accumulate ? 1 : 0);
+    if (const int e2 = cuda_check_launch("combine_kernel launch")) return e2;
+  }
+  return NAMOH_OK;
 }
