@@ -19,6 +19,10 @@ it follows:
 * ``prefill_rows`` the same for a chosen subset of query rows.
 * ``decode_step``  Sec. 3.1 (last paragraph): append to and attend within only
                    the selected heads' histories.
+* ``sa_prefill``   App. B.4 "SA+NAMOH" with the block-selection model of App. B.3
+                   (Eqs. app-block-budget, app-selected-entries): blocks of the routed
+                   history in local order, the current block plus the highest-scoring
+                   completed blocks against their mean-pooled keys.
 """
 from __future__ import annotations
 
@@ -78,6 +82,9 @@ def _load():
         lib.oracle_shared_prefill.argtypes = [P, P, P, i32, i32, i32, i32, i32, f64, i32, P, i32]
         lib.oracle_proj_qkv.argtypes = [P, i32, P, i32, i32, i32, i32, P, i32, P, P, P, P, i32]
         lib.oracle_proj_out.argtypes = [P, P, i64, i32, i32, i32, P, i32, i32, P, i32]
+        lib.oracle_sa_prefill.argtypes = [P, P, P, i32, i32, i32, f64, P, P, P, i32, i64, i64, P, P, i32, P,
+                                          i32, i32, P]
+        lib.oracle_sa_scores_rows.argtypes = [P, P, i32, i32, i32, f64, P, i32, P, P, i64, i32, P, i32, P]
         lib.oracle_default_threads.argtypes = []
         for fn in ("oracle_route_topk", "oracle_route_biased", "oracle_dispatch", "oracle_dispatch_varlen",
                    "oracle_rope", "oracle_prefill",
@@ -386,3 +393,63 @@ def shared_decode_step(q, k, v, d: int, base: float, k_cache, v_cache, seg_base,
     top = np.tile(np.arange(Hs, dtype=np.int32), (B, 1))
     return decode_step(top, np.ones((B, Hs)), q, k, v, Hs, d, 1, base, k_cache, v_cache, seg_base, seg_len,
                        seg_cap, window=window)
+
+
+def sa_mask_words(n_max: int, block: int) -> int:
+    """32-bit words per query of a kept-block mask for histories of at most n_max entries."""
+    nblk = -(-int(n_max) // int(block))
+    return max(1, -(-nblk // 32))
+
+
+def sa_prefill(q, k, v, seg_offsets, row_src, gate, d: int, g: int, base: float, block: int,
+               alpha_num: int, alpha_den: int, mask_in: np.ndarray | None = None, want_mask: bool = False,
+               nthreads: int | None = None, interleaved: bool = False, pos: np.ndarray | None = None):
+    """SA + NAMOH prefill over packed rows (App. B.4, selection model of App. B.3).
+
+    alpha = alpha_num / alpha_den.  mask_in [R*g, W] uint32 (W = sa_mask_words) replaces the
+    selection; want_mask also returns the blocks kept.  Returns y [R*g, d] fp64 (and the mask).
+    """
+    lib = _load()
+    q = np.ascontiguousarray(q, dtype=np.uint16)
+    k = np.ascontiguousarray(k, dtype=np.uint16)
+    v = np.ascontiguousarray(v, dtype=np.uint16)
+    seg = np.ascontiguousarray(seg_offsets, dtype=np.int32)
+    rs = np.ascontiguousarray(row_src, dtype=np.int32)
+    gt = np.ascontiguousarray(gate, dtype=np.float64).reshape(-1)
+    R = int(seg[-1])
+    n_max = int(np.max(np.diff(seg))) if len(seg) > 1 else 0
+    W = sa_mask_words(n_max, block)
+    if mask_in is not None:
+        mask_in = np.ascontiguousarray(mask_in, dtype=np.uint32)
+        if mask_in.shape != (R * g, W):
+            raise OracleError(f"mask_in must be [{R * g}, {W}]")
+    mask_out = np.zeros((R * g, W), np.uint32) if want_mask else None
+    y = np.zeros((R * g, d), np.float64)
+    pos = None if pos is None else np.ascontiguousarray(pos, dtype=np.int64)
+    nthreads = default_threads() if nthreads is None else int(nthreads)
+    rc = lib.oracle_sa_prefill(_ptr(q), _ptr(k), _ptr(v), len(seg) - 1, d, g, float(base), _ptr(seg), _ptr(rs),
+                               _ptr(gt), int(block), int(alpha_num), int(alpha_den),
+                               _ptr(mask_in) if mask_in is not None else None,
+                               _ptr(mask_out) if mask_out is not None else None, W, _ptr(y), nthreads,
+                               int(bool(interleaved)), _ptr(pos) if pos is not None else None)
+    _check(rc, "sa_prefill")
+    return (y, mask_out) if want_mask else y
+
+
+def sa_scores_rows(q, k, seg_offsets, d: int, g: int, base: float, block: int, rows, heads, nblk: int,
+                   interleaved: bool = False, pos: np.ndarray | None = None) -> np.ndarray:
+    """fp64 scores of the completed blocks (before the current one) for chosen queries: [len(rows), nblk],
+    NaN where a block is not a completed block of that query's history."""
+    lib = _load()
+    q = np.ascontiguousarray(q, dtype=np.uint16)
+    k = np.ascontiguousarray(k, dtype=np.uint16)
+    seg = np.ascontiguousarray(seg_offsets, dtype=np.int32)
+    rows = np.ascontiguousarray(rows, dtype=np.int64)
+    heads = np.ascontiguousarray(heads, dtype=np.int32)
+    out = np.empty((len(rows), int(nblk)), np.float64)
+    pos = None if pos is None else np.ascontiguousarray(pos, dtype=np.int64)
+    rc = lib.oracle_sa_scores_rows(_ptr(q), _ptr(k), len(seg) - 1, d, g, float(base), _ptr(seg), int(block),
+                                   _ptr(rows), _ptr(heads), len(rows), int(nblk), _ptr(out),
+                                   int(bool(interleaved)), _ptr(pos) if pos is not None else None)
+    _check(rc, "sa_scores_rows")
+    return out

@@ -26,6 +26,10 @@
  *                query heads of a group share its gate, key/value history and rank.
  *   - shared:    the shared-head variant (Sec. 5): always-active heads over the full causal
  *                prefix or a sliding window of the last w tokens, at global RoPE positions.
+ *   - SA+NAMOH:  App. B.4 with the selection model of App. B.3, Eqs. (app-block-budget) and
+ *                (app-selected-entries): blocks of Bk entries in each routed history's local
+ *                order; the current block plus the ceil(alpha N_B(r)) - 1 completed blocks
+ *                scoring highest against their mean-pooled keys.
  *
  * Readings where the paper is silent (each listed in the design notes):
  *   - TopK compares the raw fp32 router logits (softmax is monotone, so the selected
@@ -779,6 +783,245 @@ int oracle_shared_prefill(const uint16_t *q, const uint16_t *k, const uint16_t *
     struct shared_ctx c = {q, k, v, Hs, T, d, window, interleaved, base, y};
     parallel_for((long)B * Hs, nthreads, shared_head, &c);
     return ORACLE_OK;
+}
+
+/* ------------------------------------------------------------------------- */
+/* SA + NAMOH: block selection inside each routed history (App. B.3 "Block-   */
+/* Selected Sparse Attention", App. B.4 "SA+NAMOH")                           */
+/* ------------------------------------------------------------------------- */
+
+/*
+ * Within one routed head history (local order, keys k~ after head-relative RoPE), a query at
+ * one-based local rank r sees N_B(r) = ceil(r / Bk) blocks of Bk entries (Eq. app-block-budget)
+ * and keeps R(r) = ceil(alpha N_B(r)) of them: its current block, causally, and the R(r) - 1
+ * completed historical blocks with the highest scores.  A block's score is the query's dot
+ * product with the block's mean-pooled key (the MoBA selector named in App. B.3).  The query
+ * then attends with scaled dot-product attention over the entries of those blocks, and the
+ * gate-weighted combine is that of the plain path.
+ * Readings: alpha = a_num / a_den exactly; ties between block scores go to the lower block
+ * index; the pooled keys are the rotated keys k~ the attention itself uses.
+ */
+static long sa_blocks_kept(long r1, int Bk, long a_num, long a_den)
+{
+    long nb = (r1 + Bk - 1) / Bk;               /* N_B(r) */
+    return (nb * a_num + a_den - 1) / a_den;    /* R(r) = ceil(alpha N_B(r)) */
+}
+
+struct sa_ctx {
+    const uint16_t *q, *v;
+    const double *krot, *kbar;   /* [R, d] rotated keys; [R, d] block means at off + b */
+    const int32_t *seg_offsets, *row_src;
+    const double *gate;
+    double *y;
+    const uint32_t *mask_in;
+    uint32_t *mask_out;
+    int mask_words;
+    int nseg, d, g, Bk;
+    long a_num, a_den;
+    double base;
+    int interleaved;
+    const int64_t *pos;
+    long *item_seg, *item_r0;
+    int chunk;
+    int status;
+};
+
+static void sa_item(long it, void *vctx)
+{
+    struct sa_ctx *c = (struct sa_ctx *)vctx;
+    int d = c->d, g = c->g, Bk = c->Bk;
+    long s = c->item_seg[it], r0 = c->item_r0[it];
+    long off = c->seg_offsets[s], n = c->seg_offsets[s + 1] - off;
+    long r1 = r0 + c->chunk < n ? r0 + c->chunk : n;
+    long nblk = (n + Bk - 1) / Bk;
+    double *keys = (double *)malloc(sizeof(double) * (size_t)(n > 0 ? n : 1) * d);
+    double *vals = (double *)malloc(sizeof(double) * (size_t)(n > 0 ? n : 1) * d);
+    double *vraw = (double *)malloc(sizeof(double) * (size_t)(r1 > 0 ? r1 : 1) * d);
+    double *w = (double *)malloc(sizeof(double) * (size_t)(n > 0 ? n : 1));
+    double *score = (double *)malloc(sizeof(double) * (size_t)(nblk > 0 ? nblk : 1));
+    char *take = (char *)malloc((size_t)(nblk > 0 ? nblk : 1));
+    double *qin = (double *)malloc(sizeof(double) * (size_t)d);
+    double *qr = (double *)malloc(sizeof(double) * (size_t)d);
+    double *h = (double *)malloc(sizeof(double) * (size_t)d);
+    if (!keys || !vals || !vraw || !w || !score || !take || !qin || !qr || !h) {
+        c->status = ORACLE_ERR_NOMEM;
+        goto done;
+    }
+    for (long t = 0; t < r1; ++t)
+        for (int cc = 0; cc < d; ++cc) vraw[t * d + cc] = bf16_to_double(c->v[(off + t) * d + cc]);
+    for (long r = r0; r < r1; ++r) {
+        long row = off + r;
+        long rank1 = r + 1;                       /* one-based local rank */
+        long cur = r / Bk;                        /* current block: N_B(r) - 1 */
+        long keep = sa_blocks_kept(rank1, Bk, c->a_num, c->a_den) - 1;  /* historical blocks kept */
+        long dst = c->row_src[row];
+        for (int j = 0; j < g; ++j) {
+            long qi = row * g + j;
+            for (int cc = 0; cc < d; ++cc) qin[cc] = bf16_to_double(c->q[qi * d + cc]);
+            rope_rotate(qin, d, c->pos ? (double)c->pos[row] : (double)r, c->base, c->interleaved, qr);
+            for (long b = 0; b < cur; ++b) take[b] = 0;
+            if (c->mask_in) {
+                for (long b = 0; b < cur; ++b)
+                    take[b] = (char)((c->mask_in[qi * c->mask_words + b / 32] >> (b % 32)) & 1u);
+            } else {
+                /* scores of the completed blocks against their mean-pooled keys */
+                for (long b = 0; b < cur; ++b) {
+                    double acc = 0.0;
+                    for (int cc = 0; cc < d; ++cc) acc += qr[cc] * c->kbar[(off + b) * d + cc];
+                    score[b] = acc;
+                }
+                /* the `keep` highest, ties to the lower block index */
+                for (long m = 0; m < keep; ++m) {
+                    long best = -1;
+                    for (long b = 0; b < cur; ++b)
+                        if (!take[b] && (best < 0 || score[b] > score[best])) best = b;
+                    if (best < 0) break;  /* keep <= cur always (alpha <= 1) */
+                    take[best] = 1;
+                }
+            }
+            if (c->mask_out) {
+                for (int wd = 0; wd < c->mask_words; ++wd) c->mask_out[qi * c->mask_words + wd] = 0u;
+                for (long b = 0; b < cur; ++b)
+                    if (take[b]) c->mask_out[qi * c->mask_words + b / 32] |= 1u << (b % 32);
+            }
+            /* the attended entries: kept historical blocks, then the current block up to r */
+            long len = 0;
+            for (long b = 0; b <= cur; ++b) {
+                if (b < cur && !take[b]) continue;
+                long e1 = b < cur ? (b + 1) * Bk : r + 1;
+                for (long t = b * Bk; t < e1; ++t, ++len) {
+                    memcpy(keys + len * d, c->krot + (off + t) * d, sizeof(double) * (size_t)d);
+                    memcpy(vals + len * d, vraw + t * d, sizeof(double) * (size_t)d);
+                }
+            }
+            attend(qr, keys, vals, len, d, w, h);
+            double gt = c->gate[dst];
+            for (int cc = 0; cc < d; ++cc) c->y[(dst * g + j) * d + cc] = gt * h[cc];
+        }
+    }
+done:
+    free(keys); free(vals); free(vraw); free(w); free(score); free(take); free(qin); free(qr); free(h);
+}
+
+/* mean-pooled rotated keys of the complete blocks of segment s, at rows off + b */
+struct sa_pool_ctx {
+    const double *krot;
+    const int32_t *seg_offsets;
+    double *kbar;
+    int d, Bk;
+};
+
+static void sa_pool_segment(long s, void *vctx)
+{
+    struct sa_pool_ctx *c = (struct sa_pool_ctx *)vctx;
+    int d = c->d, Bk = c->Bk;
+    long off = c->seg_offsets[s], n = c->seg_offsets[s + 1] - off;
+    for (long b = 0; b < n / Bk; ++b)
+        for (int cc = 0; cc < d; ++cc) {
+            double acc = 0.0;
+            for (long t = b * Bk; t < (b + 1) * Bk; ++t) acc += c->krot[(off + t) * d + cc];
+            c->kbar[(off + b) * d + cc] = acc / (double)Bk;
+        }
+}
+
+/*
+ * oracle_sa_prefill: SA + NAMOH prefill over packed rows (layout as oracle_prefill).
+ *   Bk          block size (>= 1); alpha = a_num / a_den in (0, 1]
+ *   mask_in     [R*g, mask_words] kept historical blocks per query (bit b of word b/32), or NULL
+ *               to select them here; only blocks before the query's current block are read
+ *   mask_out    [R*g, mask_words] the blocks kept, or NULL
+ *   y           [R*g, d] fp64 per-slot combine g*h at (row_src*g + j)
+ */
+int oracle_sa_prefill(const uint16_t *q, const uint16_t *k, const uint16_t *v, int nseg, int d, int g,
+                      double base, const int32_t *seg_offsets, const int32_t *row_src, const double *gate,
+                      int Bk, long a_num, long a_den, const uint32_t *mask_in, uint32_t *mask_out, int mask_words,
+                      double *y, int nthreads, int interleaved, const int64_t *pos)
+{
+    if (!q || !k || !v || !seg_offsets || !row_src || !gate || !y) return ORACLE_ERR_ARG;
+    if (nseg < 0 || d < 2 || (d & 1) || g < 1 || Bk < 1 || a_num < 1 || a_den < a_num) return ORACLE_ERR_ARG;
+    long R = seg_offsets[nseg];
+    long nmax = 0;
+    for (int s = 0; s < nseg; ++s)
+        if (seg_offsets[s + 1] - seg_offsets[s] > nmax) nmax = seg_offsets[s + 1] - seg_offsets[s];
+    if ((mask_in || mask_out) && (long)mask_words * 32 < (nmax + Bk - 1) / Bk) return ORACLE_ERR_ARG;
+    double *krot = (double *)malloc(sizeof(double) * (size_t)(R > 0 ? R : 1) * d);
+    double *kbar = (double *)malloc(sizeof(double) * (size_t)(R > 0 ? R : 1) * d);
+    if (!krot || !kbar) {
+        free(krot); free(kbar);
+        return ORACLE_ERR_NOMEM;
+    }
+    struct rotk_ctx rk = {k, seg_offsets, krot, d, base, interleaved, pos};
+    parallel_for(nseg, nthreads, rotate_k_segment, &rk);
+    struct sa_pool_ctx pc = {krot, seg_offsets, kbar, d, Bk};
+    parallel_for(nseg, nthreads, sa_pool_segment, &pc);
+
+    const int chunk = 64;
+    long nitems = 0;
+    for (int s = 0; s < nseg; ++s) nitems += (seg_offsets[s + 1] - seg_offsets[s] + chunk - 1) / chunk;
+    long *item_seg = (long *)malloc(sizeof(long) * (size_t)(nitems > 0 ? nitems : 1));
+    long *item_r0 = (long *)malloc(sizeof(long) * (size_t)(nitems > 0 ? nitems : 1));
+    if (!item_seg || !item_r0) {
+        free(item_seg); free(item_r0); free(krot); free(kbar);
+        return ORACLE_ERR_NOMEM;
+    }
+    long it = 0;
+    for (int s = 0; s < nseg; ++s)
+        for (long r0 = 0; r0 < seg_offsets[s + 1] - seg_offsets[s]; r0 += chunk) {
+            item_seg[it] = s;
+            item_r0[it] = r0;
+            ++it;
+        }
+    struct sa_ctx ctx = {q, v, krot, kbar, seg_offsets, row_src, gate, y, mask_in, mask_out, mask_words,
+                         nseg, d, g, Bk, a_num, a_den, base, interleaved, pos, item_seg, item_r0, chunk,
+                         ORACLE_OK};
+    parallel_for(nitems, nthreads, sa_item, &ctx);
+    free(item_seg); free(item_r0); free(krot); free(kbar);
+    return ctx.status;
+}
+
+/*
+ * oracle_sa_scores_rows: the fp64 block scores q~ . mean(k~ of block b), b < current block,
+ * for chosen queries (the checks of a selection made elsewhere).
+ *   rows [nrows] packed rows, heads [nrows] group heads; out [nrows, nblk_out], unused entries NaN
+ */
+int oracle_sa_scores_rows(const uint16_t *q, const uint16_t *k, int nseg, int d, int g, double base,
+                          const int32_t *seg_offsets, int Bk, const int64_t *rows, const int32_t *heads, long nrows,
+                          int nblk_out, double *out, int interleaved, const int64_t *pos)
+{
+    if (!q || !k || !seg_offsets || !rows || !heads || !out || Bk < 1 || nblk_out < 0) return ORACLE_ERR_ARG;
+    long R = seg_offsets[nseg];
+    double *tmp = (double *)malloc(sizeof(double) * (size_t)d);
+    double *qr = (double *)malloc(sizeof(double) * (size_t)d);
+    double *kr = (double *)malloc(sizeof(double) * (size_t)d);
+    double *mean = (double *)malloc(sizeof(double) * (size_t)d);
+    int st = (tmp && qr && kr && mean) ? ORACLE_OK : ORACLE_ERR_NOMEM;
+    for (long i = 0; i < nrows && st == ORACLE_OK; ++i) {
+        long row = rows[i];
+        int j = heads[i];
+        if (row < 0 || row >= R || j < 0 || j >= g) { st = ORACLE_ERR_ARG; break; }
+        int lo = 0, hi = nseg;
+        while (hi - lo > 1) {
+            int mid = (lo + hi) / 2;
+            if (seg_offsets[mid] <= row) lo = mid; else hi = mid;
+        }
+        long off = seg_offsets[lo], r = row - off, cur = r / Bk;
+        for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(q[(row * g + j) * d + cc]);
+        rope_rotate(tmp, d, pos ? (double)pos[row] : (double)r, base, interleaved, qr);
+        for (long b = 0; b < nblk_out; ++b) out[i * nblk_out + b] = NAN;
+        for (long b = 0; b < cur && b < nblk_out; ++b) {
+            for (int cc = 0; cc < d; ++cc) mean[cc] = 0.0;
+            for (long t = b * Bk; t < (b + 1) * Bk; ++t) {
+                for (int cc = 0; cc < d; ++cc) tmp[cc] = bf16_to_double(k[(off + t) * d + cc]);
+                rope_rotate(tmp, d, pos ? (double)pos[off + t] : (double)t, base, interleaved, kr);
+                for (int cc = 0; cc < d; ++cc) mean[cc] += kr[cc];
+            }
+            double acc = 0.0;
+            for (int cc = 0; cc < d; ++cc) acc += qr[cc] * (mean[cc] / (double)Bk);
+            out[i * nblk_out + b] = acc;
+        }
+    }
+    free(tmp); free(qr); free(kr); free(mean);
+    return st;
 }
 
 /* Number of worker threads the oracle would use by default. */

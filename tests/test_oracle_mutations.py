@@ -49,6 +49,14 @@ MUTATIONS = {
     "biased_key_drops_bias": ("kt[i] = a[i] + (double)bias[i];", "kt[i] = a[i];"),
     "biased_ties_to_upper_index": ("while (j > 0 && kt[i] > kt[order[j - 1]]) {",
                                    "while (j > 0 && kt[i] >= kt[order[j - 1]]) {"),
+    "sa_budget_floor": ("return (nb * a_num + a_den - 1) / a_den;", "return (nb * a_num) / a_den;"),
+    "sa_keeps_lowest_scores": ("if (!take[b] && (best < 0 || score[b] > score[best])) best = b;",
+                               "if (!take[b] && (best < 0 || score[b] < score[best])) best = b;"),
+    "sa_current_block_shift": ("long cur = r / Bk;                        /* current block: N_B(r) - 1 */",
+                               "long cur = (r + 1) / Bk;                  /* current block: N_B(r) - 1 */"),
+    "sa_drops_current_block": ("long e1 = b < cur ? (b + 1) * Bk : r + 1;", "long e1 = b < cur ? (b + 1) * Bk : r;"),
+    "sa_pools_shifted_rows": ("for (long t = b * Bk; t < (b + 1) * Bk; ++t) acc += c->krot[(off + t) * d + cc];",
+                              "for (long t = b * Bk; t < (b + 1) * Bk; ++t) acc += c->krot[(off + t + 1) * d + cc];"),
 }
 
 
@@ -65,7 +73,7 @@ def test_pins_catch_mutation(tmp_path, name):
                     ignore=shutil.ignore_patterns("*.so", "__pycache__", "csrc", "_build"))
     os.makedirs(tmp_path / "tests")
     for f in ("conftest.py", "test_oracle_route.py", "test_oracle_attention.py", "test_oracle_layer.py",
-              "test_oracle_shared.py", "test_accounting.py"):
+              "test_oracle_shared.py", "test_oracle_sa.py", "test_accounting.py"):
         shutil.copy(os.path.join(ROOT, "tests", f), tmp_path / "tests")
     shutil.copytree(os.path.join(ROOT, "tests", "golden"), tmp_path / "tests" / "golden")
     r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider", "-m", "not gpu",
