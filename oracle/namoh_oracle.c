@@ -857,8 +857,9 @@ static void sa_item(long it, void *vctx)
         long dst = c->row_src[row];
         for (int j = 0; j < g; ++j) {
             long qi = row * g + j;
+            const double qpos = c->pos ? (double)c->pos[row] : (double)r;
             for (int cc = 0; cc < d; ++cc) qin[cc] = bf16_to_double(c->q[qi * d + cc]);
-            rope_rotate(qin, d, c->pos ? (double)c->pos[row] : (double)r, c->base, c->interleaved, qr);
+            rope_rotate(qin, d, qpos, c->base, c->interleaved, qr);
             for (long b = 0; b < cur; ++b) take[b] = 0;
             if (c->mask_in) {
                 for (long b = 0; b < cur; ++b)
