@@ -400,6 +400,8 @@ def run_gpu(args, rank: int, world: int):
         line["gpu_launches"] += line["layer"].pop("launches")
         line["shared_heads"] = run_shared(args, dev, pk, pk_kind)
         line["gpu_launches"] += line["shared_heads"].pop("launches")
+        line["sa_namoh"] = run_sa(args, dev, pk, pk_kind)
+        line["gpu_launches"] += line["sa_namoh"].pop("launches")
     clocks.__exit__(None, None, None)
     line["clocks"] = clocks.summary()
     return line
@@ -537,6 +539,66 @@ def run_shared(args, dev, pk, pk_kind):
     out["device_status"] = int(status.item())
     out["launches"] = 2 * args.steps * 3  # layout, RoPE + plan, attention per call
     return out
+
+
+def run_sa(args, dev, pk, pk_kind):
+    """SA + NAMOH (namoh_sa_prefill) on the balanced workload: 32-key blocks, alpha = 1/5, L2 flushed
+    before every timed call, beside the dense routed prefill on the same routing.  Flops: 4 d per
+    attended (query, key) pair, sum over heads of Phi_{alpha,B}(n_i) (App. B.3 Eq.
+    app-fractional-causal-sum); the kernel still runs every causal key tile and masks the blocks a
+    query does not keep, so its time is the dense prefill's plus the selection."""
+    import torch
+
+    import paper_2609_38832_gb300 as namoh
+
+    wl = ni.BALANCED
+    block, num, den = 32, 1, 5
+    ro = namoh.namoh_route(torch.from_numpy(wl.scores()).to(dev), wl.Kr)
+    qh, kh, vh = wl.qkv()
+    up = lambda b: torch.from_numpy(b.view(np.int16)).to(dev).view(torch.bfloat16)
+    q, k, v = up(qh), up(kh), up(vh)
+    kw = dict(B=wl.B, T=wl.T, H=wl.H, K=wl.K, group=wl.g, rope_base=wl.base)
+    y = torch.empty((wl.B, wl.T, wl.K, wl.d), dtype=torch.bfloat16, device=dev)
+    k_cache = torch.empty_like(k)
+    mask = torch.empty((k.shape[0] * wl.g, namoh._abi.load().namoh_sa_mask_words(wl.T, block)), dtype=torch.int32,
+                       device=dev)
+    ws_sa, ws_dense = namoh.Workspace(), namoh.Workspace()
+    flush = torch.empty(2 << 30, dtype=torch.uint8, device=dev)
+    calls = {
+        "sa": lambda: namoh.namoh_sa_prefill(q, k, v, ro.seg_offsets, ro.row_src, ro.gate, block=block,
+                                             alpha_num=num, alpha_den=den, y=y, sa_mask=mask, k_cache=k_cache,
+                                             workspace=ws_sa, status=ro.status, **kw),
+        "dense": lambda: namoh.namoh_prefill(q, k, v, ro.seg_offsets, ro.row_src, ro.gate, y=y, k_cache=k_cache,
+                                             workspace=ws_dense, status=ro.status, **kw),
+    }
+    ms = {}
+    for name, run in calls.items():
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+        for i in range(args.warmup + args.steps):
+            flush.fill_(i & 0xFF)
+            if i >= args.warmup:
+                evs[i - args.warmup][0].record()
+            run()
+            if i >= args.warmup:
+                evs[i - args.warmup][1].record()
+        torch.cuda.synchronize()
+        ms[name] = float(np.mean([a.elapsed_time(b) for a, b in evs]))
+    n = np.diff(ro.seg_offsets.cpu().numpy()).astype(np.int64)
+    pairs_sa = 0
+    for ni_ in n:
+        r = np.arange(1, ni_ + 1, dtype=np.int64)
+        nb = (r + block - 1) // block
+        kept = (nb * num + den - 1) // den
+        pairs_sa += int(np.sum(r - block * (nb - kept)))  # a_{alpha,B}(r), Eq. app-selected-entries
+    pairs_dense = int(np.sum(n * (n + 1) // 2))
+    flops_sa = 4.0 * wl.d * wl.g * pairs_sa
+    tf = flops_sa / (ms["sa"] * 1e-3) / 1e12
+    return {"workload": f"{wl.name}, blocks of {block}, alpha {num}/{den}", "ms": ms["sa"],
+            "dense_prefill_ms": ms["dense"], "sa_pairs_over_dense": pairs_sa / pairs_dense,
+            "tflops_attended": tf, "frac_bf16": tf / pk["bf16_tflops"], "flops_attended": flops_sa,
+            "peak_source": f"{pk_kind} bf16 dense (burst)", "device_status": int(ro.status.item()),
+            "launches": 2 * args.steps * 4,  # per call: RoPE + plan, pooling, selection, attention
+            "note": "every causal key tile is computed; blocks not kept are masked in the softmax"}
 
 
 def run_decode(args, dev, pk, pk_kind):

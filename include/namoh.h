@@ -367,6 +367,43 @@ NAMOH_API int namoh_shared_decode(const uint16_t *q, const uint16_t *k, const ui
                                   size_t workspace_bytes, uint32_t *dev_status, void *stream);
 
 /* ------------------------------------------------------------------------- *
+ * SA + NAMOH: block-selected sparse attention inside each routed history (App. B.4
+ * "SA+NAMOH", with the selection model of App. B.3 "Block-Selected Sparse Attention",
+ * Eqs. app-block-budget and app-selected-entries).  The routed history of each (batch,
+ * head) is cut into blocks of `block` entries in its local order.  A query at one-based
+ * local rank r keeps R(r) = ceil(alpha * ceil(r / block)) blocks, alpha = alpha_num /
+ * alpha_den in (0, 1] (computed exactly): its current block, attended causally, and the
+ * R(r) - 1 completed earlier blocks whose mean-pooled rotated key k~ has the largest dot
+ * product with its rotated query q~ (fp32 scores; ties to the lower block index).  It then
+ * attends over the entries of the kept blocks; the gate-weighted combine is namoh_prefill's.
+ * alpha = 1 keeps every block (dense routed attention).
+ *
+ * namoh_sa_prefill
+ *   Arguments as namoh_prefill_ex (routing outputs, caches, seg_len, workspace), plus:
+ *   block       32, 64 or 128 keys per block; ceil(T / block) <= 1024.
+ *   alpha_num, alpha_den  1 <= alpha_num <= alpha_den.
+ *   sa_mask     [R*g, namoh_sa_mask_words(T, block)] uint32 out, 4-byte aligned: the kept
+ *               earlier blocks of query (packed row r, group head j) at row r*g + j, bit
+ *               b % 32 of word b / 32 for block b (the current block is implied).
+ *   Workspace: namoh_sa_prefill_workspace_size (namoh_prefill's plus the pooled keys,
+ *   (R / block + B*H/g) * d_head fp32).
+ *   The attention does every causal key tile and masks the blocks not kept: the cost is
+ *   that of namoh_prefill plus the selection.
+ * namoh_sa_mask_words: words per query of sa_mask (0 for an unsupported block).
+ * Errors: NAMOH_ERR_INVALID_ARG for an unsupported block or alpha, a null sa_mask, or the
+ * argument errors of namoh_prefill_ex.
+ * ------------------------------------------------------------------------- */
+NAMOH_API int namoh_sa_mask_words(int T, int block);
+NAMOH_API size_t namoh_sa_prefill_workspace_size(int B, int T, int H, int K, int d_head, int group, int block);
+NAMOH_API int namoh_sa_prefill(const uint16_t *q, const uint16_t *k, const uint16_t *v, int B, int T, int H, int K,
+                               int d_head, int group, float rope_base, unsigned rope_flags,
+                               const int32_t *seg_offsets, const int32_t *row_src, const float *gate, int block,
+                               int alpha_num, int alpha_den, uint32_t *sa_mask, uint16_t *y, uint16_t *k_cache,
+                               uint16_t *v_cache, const int64_t *seg_base, const int32_t *seg_cap,
+                               int64_t cache_rows, int32_t *seg_len, void *workspace, size_t workspace_bytes,
+                               uint32_t *dev_status, void *stream);
+
+/* ------------------------------------------------------------------------- *
  * The projections around the path (the full attention layer).
  * Sec. 3.1, Eq. (namoh-qkv): only an active token-head pair projects,
  *   q_{t,i} = x_t W_Q^(i), k_{t,i} = x_t W_K^(i), v_{t,i} = x_t W_V^(i), t in I_i.

@@ -406,8 +406,8 @@ def sa_prefill(q, k, v, seg_offsets, row_src, gate, d: int, g: int, base: float,
                nthreads: int | None = None, interleaved: bool = False, pos: np.ndarray | None = None):
     """SA + NAMOH prefill over packed rows (App. B.4, selection model of App. B.3).
 
-    alpha = alpha_num / alpha_den.  mask_in [R*g, W] uint32 (W = sa_mask_words) replaces the
-    selection; want_mask also returns the blocks kept.  Returns y [R*g, d] fp64 (and the mask).
+    alpha = alpha_num / alpha_den.  mask_in [R*g, W] uint32 (W >= sa_mask_words of the longest
+    history) replaces the selection; want_mask also returns the blocks kept.  Returns y [R*g, d] fp64 (and the mask).
     """
     lib = _load()
     q = np.ascontiguousarray(q, dtype=np.uint16)
@@ -419,10 +419,11 @@ def sa_prefill(q, k, v, seg_offsets, row_src, gate, d: int, g: int, base: float,
     R = int(seg[-1])
     n_max = int(np.max(np.diff(seg))) if len(seg) > 1 else 0
     W = sa_mask_words(n_max, block)
-    if mask_in is not None:
+    if mask_in is not None:  # any width that holds the longest history's blocks
         mask_in = np.ascontiguousarray(mask_in, dtype=np.uint32)
-        if mask_in.shape != (R * g, W):
-            raise OracleError(f"mask_in must be [{R * g}, {W}]")
+        if mask_in.ndim != 2 or mask_in.shape[0] != R * g or mask_in.shape[1] < W:
+            raise OracleError(f"mask_in must be [{R * g}, >= {W}]")
+        W = mask_in.shape[1]
     mask_out = np.zeros((R * g, W), np.uint32) if want_mask else None
     y = np.zeros((R * g, d), np.float64)
     pos = None if pos is None else np.ascontiguousarray(pos, dtype=np.int64)

@@ -18,7 +18,7 @@ from ._abi import (NAMOH_DEV_BAD_SEQLENS, NAMOH_DEV_CAPACITY, NAMOH_DEV_NONFINIT
                    NAMOH_ROPE_GLOBAL, NAMOH_ROPE_INTERLEAVED, NamohError)
 
 __all__ = ["namoh_route", "namoh_route_varlen", "namoh_prefill", "namoh_prefill_varlen", "namoh_decode",
-           "namoh_proj_qkv", "namoh_proj_out", "namoh_shared_prefill", "namoh_shared_decode",
+           "namoh_proj_qkv", "namoh_proj_out", "namoh_shared_prefill", "namoh_shared_decode", "namoh_sa_prefill",
            "namoh_rope_pack", "namoh_attention_plan", "namoh_attention", "RouteOutputs", "Workspace", "NamohError",
            "NAMOH_DEV_BAD_SEQLENS", "NAMOH_DEV_CAPACITY", "NAMOH_DEV_NONFINITE_SCORE", "NAMOH_DEV_TIMEOUT",
            "NAMOH_ROPE_GLOBAL", "NAMOH_ROPE_INTERLEAVED", "library_path"]
@@ -192,6 +192,49 @@ def namoh_prefill(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, seg_offsets
                               cache_rows, _ptr(seg_len), _ptr(ws), ws.numel(), _ptr(st), _stream(stream))
     _abi.check("namoh_prefill_ex", rc)
     return y, k_cache, v_cache
+
+
+def namoh_sa_prefill(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, seg_offsets: torch.Tensor,
+                     row_src: torch.Tensor, gate: torch.Tensor, *, B: int, T: int, H: int, K: int, block: int = 32,
+                     alpha_num: int = 1, alpha_den: int = 5, group: int = 1, rope_base: float = 10000.0,
+                     interleaved: bool = False, global_positions: bool = False, y: Optional[torch.Tensor] = None,
+                     sa_mask: Optional[torch.Tensor] = None, k_cache: Optional[torch.Tensor] = None,
+                     v_cache: Optional[torch.Tensor] = None, seg_base: Optional[torch.Tensor] = None,
+                     seg_cap: Optional[torch.Tensor] = None, seg_len: Optional[torch.Tensor] = None,
+                     workspace: Optional[Workspace] = None, status: Optional[torch.Tensor] = None, stream=None):
+    """SA + NAMOH prefill (see namoh_sa_prefill in include/namoh.h): block selection inside each routed
+    history (blocks of `block` keys, retained fraction alpha_num / alpha_den), then the routed attention
+    over the kept blocks.  Arguments as namoh_prefill; returns (y [B, T, K, d], sa_mask [R*g, W] int32
+    bit patterns of the kept earlier blocks, k_cache, v_cache)."""
+    lib = _abi.load()
+    d = q.shape[-1]
+    dev = q.device
+    for name, t in (("q", q), ("k", k), ("v", v)):
+        if t.dtype != torch.bfloat16:
+            raise ValueError(f"{name} must be bfloat16")
+    words = lib.namoh_sa_mask_words(T, block)
+    if words == 0:
+        raise NamohError("namoh_sa_mask_words", _abi.NAMOH_ERR_INVALID_ARG)
+    if y is None:
+        y = torch.empty((B, T, K, d), dtype=torch.bfloat16, device=dev)
+    if sa_mask is None:
+        sa_mask = torch.empty((k.shape[0] * group, words), dtype=torch.int32, device=dev)
+    if k_cache is None:
+        k_cache = torch.empty_like(k)
+    if v_cache is None:
+        v_cache = v if seg_base is None else torch.empty_like(v)
+    nbytes = lib.namoh_sa_prefill_workspace_size(B, T, H, K, d, group, block)
+    if nbytes == 0:
+        raise NamohError("namoh_sa_prefill_workspace_size", _abi.NAMOH_ERR_UNSUPPORTED)
+    ws = _ws(workspace, nbytes, dev)
+    st = _status(status, dev)
+    rc = lib.namoh_sa_prefill(_ptr(q), _ptr(k), _ptr(v), B, T, H, K, d, group, float(rope_base),
+                              _rope_flags(interleaved, global_positions), _ptr(seg_offsets), _ptr(row_src),
+                              _ptr(gate), int(block), int(alpha_num), int(alpha_den), _ptr(sa_mask), _ptr(y),
+                              _ptr(k_cache), _ptr(v_cache), _ptr(seg_base), _ptr(seg_cap), k_cache.shape[0],
+                              _ptr(seg_len), _ptr(ws), ws.numel(), _ptr(st), _stream(stream))
+    _abi.check("namoh_sa_prefill", rc)
+    return y, sa_mask, k_cache, v_cache
 
 
 def namoh_prefill_varlen(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, cu_seqlens: torch.Tensor,

@@ -61,6 +61,10 @@ SIGNATURES = {
     "namoh_proj_workspace_size": (_SZ, [_I, _I, _I, _I, _I, _I]),
     "namoh_proj_qkv": (_I, [_P, _I, _I, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _SZ, _P, _P]),
     "namoh_proj_out": (_I, [_P, _I, _I, _P, _I, _I, _I, _I, _I, _P, _P, _P, _I, _P, _SZ, _P, _P]),
+    "namoh_sa_mask_words": (_I, [_I, _I]),
+    "namoh_sa_prefill_workspace_size": (_SZ, [_I, _I, _I, _I, _I, _I, _I]),
+    "namoh_sa_prefill": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _F, _U, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P,
+                              _P, _P, _I64, _P, _P, _SZ, _P, _P]),
     "namoh_shared_workspace_size": (_SZ, [_I, _I, _I, _I]),
     "namoh_shared_prefill": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _F, _U, _P, _P, _P, _P, _P, _I64, _P, _P, _SZ, _P,
                                   _P]),

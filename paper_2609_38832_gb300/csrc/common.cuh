@@ -272,6 +272,11 @@ __device__ __forceinline__ float ld_issue_f32(const float* p) {
   asm volatile("ld.global.nc.f32 %0, [%1];" : "=f"(v) : "l"(p));
   return v;
 }
+__device__ __forceinline__ uint32_t ld_issue_u32(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.global.nc.b32 %0, [%1];" : "=r"(v) : "l"(p));
+  return v;
+}
 
 // 32-byte global store (one whole L2 sector); dst must be 32-byte aligned.
 __device__ __forceinline__ void st_global_v8(void* dst, const uint32_t* w) {

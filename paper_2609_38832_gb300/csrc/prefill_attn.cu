@@ -44,6 +44,10 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              void* plan, int plan_qtiles, const int32_t* plan_cap, const int32_t* pos_row_src,
                              int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved);
 
+int launch_sa_select(const uint16_t* q_rot, const uint16_t* k_cache, const int32_t* seg_offsets,
+                     const int64_t* seg_base, int nseg, int T, long long R, int d, int g, int lg, int alpha_num,
+                     int alpha_den, float* kbar, uint32_t* mask, int words, cudaStream_t stream);
+
 namespace attn {
 
 constexpr int BM = 128;              // query rows per tile (one tile per work item)
@@ -112,6 +116,11 @@ struct Params {
   int y_sector_aligned;        // y is 32-byte aligned: rows go out as whole 32-byte sectors
   float scale_log2;            // log2(e) / sqrt(D)
   uint32_t* status;
+  // SA + NAMOH: kept historical blocks of each query [(row * g + j), sa_words] (bit b % 32 of
+  // word b / 32), blocks of 2^sa_lg keys (32, 64 or 128); used by the kSA instantiation only
+  const uint32_t* sa_mask;
+  int sa_words;
+  int sa_lg;
 };
 
 // All lanes of a warp wait and agree on the outcome, so warp-collective tcgen05
@@ -149,10 +158,12 @@ __device__ __forceinline__ bool take_item(Bars* bars, uint32_t idx, int4* item, 
 // PV(tile - 1) completed, through wait_pv).  Returns false when a wait gave up.  Ends with the
 // TMEM stores complete and fenced for the arrive on p_full.
 // kv_rel is the tile's index within the item (0 = first), kv its index in the segment.
-template <int D, typename WaitPv>
+// kSA: allow4 bit w clear masks the tile's columns 32w..32w+31 (a block the query does not keep;
+// blocks are at least 32 keys, so each 32-column group lies in one block).
+template <int D, bool kSA, typename WaitPv>
 __device__ __forceinline__ bool softmax_tile(uint32_t s_addr, uint32_t o_addr, int kv_rel, int kv, int qt, int row,
                                              int window, float scale_log2, float& m_use, float& l_sum,
-                                             uint32_t tile, WaitPv&& wait_pv) {
+                                             uint32_t tile, WaitPv&& wait_pv, uint32_t allow4 = 0xFu) {
   float sv[BN];
 #pragma unroll
   for (int c = 0; c < BN / 32; ++c) {
@@ -168,6 +179,12 @@ __device__ __forceinline__ bool softmax_tile(uint32_t s_addr, uint32_t o_addr, i
 #pragma unroll
     for (int c = 0; c < BN; ++c)
       if (c < lo) sv[c] = -INFINITY;
+  }
+  // SA + NAMOH: keys of blocks the query does not keep are out
+  if (kSA && allow4 != 0xFu) {
+#pragma unroll
+    for (int c = 0; c < BN; ++c)
+      if (!((allow4 >> (c >> 5)) & 1u)) sv[c] = -INFINITY;
   }
   // causal mask on the diagonal tile: key rank kv*BN + c <= query rank
   if (kv == qt) {
@@ -188,17 +205,24 @@ __device__ __forceinline__ bool softmax_tile(uint32_t s_addr, uint32_t o_addr, i
 #pragma unroll
   for (int i = 0; i < 8; ++i) m8[i] = fmaxf(m8[i], sv[120 + i]);
   const float mx = fmax3(fmax3(m8[0], m8[1], m8[2]), fmax3(m8[3], m8[4], m8[5]), fmaxf(m8[6], m8[7]));
-  // a row with every key of the tile outside the window gets a finite floor, so that its
-  // P is exactly 0 and the next tile's rescale factor exp2(m_use - m_tile) is 0
-  const float m_tile = window > 0 ? fmaxf(mx * scale_log2, -1e30f) : mx * scale_log2;
+  // a row with every key of the tile outside the window (or in blocks it does not keep) gets a
+  // finite floor, so that its P is exactly 0 and the next tile's rescale factor
+  // exp2(m_use - m_tile) is 0
+  const float m_tile = (kSA || window > 0) ? fmaxf(mx * scale_log2, -1e30f) : mx * scale_log2;
   float alpha = 1.f;
   bool rescale = false;
   if (kv_rel == 0) {
     m_use = m_tile;
   } else if (m_tile > m_use + kRescaleThreshold) {
-    alpha = fast_exp2(m_use - m_tile);
+    if ((kSA || window > 0) && m_use <= -1e30f) {
+      // every earlier key of this row was masked: O and the row sum are exactly 0, so the
+      // first tile with a visible key just sets the max (no rescale, no wait for the PV)
+      alpha = 0.f;
+    } else {
+      alpha = fast_exp2(m_use - m_tile);
+      rescale = true;
+    }
     m_use = m_tile;
-    rescale = true;
   }
   // P = exp2(S * scale - m_use): scale-and-subtract and the row sum on fp32 pairs
   uint32_t pk[BN / 2];
@@ -247,7 +271,7 @@ __device__ __forceinline__ bool softmax_tile(uint32_t s_addr, uint32_t o_addr, i
   return true;
 }
 
-template <int D>
+template <int D, bool kSA>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                     const __grid_constant__ CUtensorMap tm_v, Params p) {
@@ -544,14 +568,34 @@ __global__ void __launch_bounds__(kThreads, 1)
       float gt = 0.f;
       float m_use = 0.f, l_sum = 0.f;
       const int kv0 = first_key_tile(qt, p.window);
+      // SA + NAMOH: this query's kept-block words, one tile ahead of their use
+      const uint32_t* mrow = nullptr;
+      int cur_blk = 0;
+      uint32_t w_next = ~0u;
+      if (kSA && valid) {
+        mrow = p.sa_mask + ((long long)(off + qrank) * p.g + j) * p.sa_words;
+        cur_blk = qrank >> p.sa_lg;
+        w_next = ld_issue_u32(mrow + (((kv0 * BN) >> p.sa_lg) >> 5));
+      }
       for (int kv = kv0; kv <= qt && ok; ++kv) {
         const uint32_t s_addr = tmem + lane_addr + tmem_s_col((int)(s_iter % kSBufs));
+        uint32_t allow4 = 0xFu;
+        if (kSA && mrow) {
+          const uint32_t w = w_next;
+          if (kv < qt) w_next = ld_issue_u32(mrow + ((((kv + 1) * BN) >> p.sa_lg) >> 5));
+          allow4 = 0u;
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            const int blk = (kv * BN + 32 * c) >> p.sa_lg;
+            if (blk == cur_blk || ((w >> (blk & 31)) & 1u)) allow4 |= 1u << c;
+          }
+        }
         ok = warp_wait(&bars->s_full[s_iter % kSBufs], (s_iter / kSBufs) & 1, abort_flag, p.status);
         const uint32_t tile = s_iter++;
         if (!ok) break;
         tc_fence_after();
-        ok = softmax_tile<D>(s_addr, o_addr, kv - kv0, kv, qt, row, p.window, p.scale_log2, m_use, l_sum, tile,
-                             wait_pv);
+        ok = softmax_tile<D, kSA>(s_addr, o_addr, kv - kv0, kv, qt, row, p.window, p.scale_log2, m_use, l_sum,
+                                  tile, wait_pv, allow4);
         if (!ok) break;
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars->p_full[tile & 1]);
@@ -629,13 +673,13 @@ bool encode_rows_map(CUtensorMap* map, const void* base, long long rows, int row
   return r == CUDA_SUCCESS;
 }
 
-template <int D>
+template <int D, bool kSA>
 cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv, const Params& p,
                         int grid, cudaStream_t stream) {
   const int smem = Smem<D>::kAlloc;
-  cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D, kSA>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  e = launch_pdl(attn_fwd_kernel<D>, dim3(grid), dim3(kThreads), (size_t)smem, stream, tq, tk, tv, p);
+  e = launch_pdl(attn_fwd_kernel<D, kSA>, dim3(grid), dim3(kThreads), (size_t)smem, stream, tq, tk, tv, p);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
@@ -731,7 +775,8 @@ int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v
 int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint16_t* v_cache, long long R, int D,
                      int g, const int32_t* seg_offsets, const int32_t* row_src, const float* gate,
                      const int64_t* seg_base, long long cache_rows, void* plan, uint16_t* y, uint32_t* dev_status,
-                     const DeviceInfo& info, cudaStream_t stream, int window = 0) {
+                     const DeviceInfo& info, cudaStream_t stream, int window = 0,
+                     const uint32_t* sa_mask = nullptr, int sa_words = 0, int sa_lg = 0) {
   CUtensorMap tq, tk, tv;
   if (!attn::encode_rows_map(&tq, q_rot, R, g * D) || !attn::encode_rows_map(&tk, k_cache, cache_rows, D) ||
       !attn::encode_rows_map(&tv, v_cache, cache_rows, D))
@@ -751,8 +796,16 @@ int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint1
   p.y_sector_aligned = (reinterpret_cast<uintptr_t>(y) & 31u) == 0;
   p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)D));
   p.status = dev_status;
-  const cudaError_t e = (D == 128) ? attn::launch_attn<128>(tq, tk, tv, p, info.sm_count, stream)
-                                   : attn::launch_attn<64>(tq, tk, tv, p, info.sm_count, stream);
+  p.sa_mask = sa_mask;
+  p.sa_words = sa_words;
+  p.sa_lg = sa_lg;
+  cudaError_t e;
+  if (sa_mask)
+    e = (D == 128) ? attn::launch_attn<128, true>(tq, tk, tv, p, info.sm_count, stream)
+                   : attn::launch_attn<64, true>(tq, tk, tv, p, info.sm_count, stream);
+  else
+    e = (D == 128) ? attn::launch_attn<128, false>(tq, tk, tv, p, info.sm_count, stream)
+                   : attn::launch_attn<64, false>(tq, tk, tv, p, info.sm_count, stream);
   return e == cudaSuccess ? NAMOH_OK : cuda_fail(e, "attn_fwd_kernel launch");
 }
 
@@ -963,6 +1016,94 @@ extern "C" int namoh_prefill(const uint16_t* q, const uint16_t* k, const uint16_
   return namoh_prefill_ex(q, k, v, B, T, H, K, d_head, group, rope_base, 0u, seg_offsets, row_src, gate, y, k_cache,
                           v_cache, seg_base, seg_cap, cache_rows, seg_len, workspace, workspace_bytes, dev_status,
                           stream_v);
+}
+
+// ---------------------------------------------------------------------------
+// SA + NAMOH (App. B.4, selection model of App. B.3): block selection inside each routed history,
+// then the routed attention over the kept blocks and the query's current block.
+// ---------------------------------------------------------------------------
+namespace namoh {
+namespace {
+constexpr int kSaMaxBlocks = 1024;  // blocks per history the selector holds
+
+int sa_block_lg(int block) {
+  return block == 32 ? 5 : block == 64 ? 6 : block == 128 ? 7 : -1;
+}
+
+int sa_words_for(int T, int block) { return ((T + block - 1) / block + 31) / 32; }
+
+size_t sa_workspace_rows(long long R, int nseg, int d_head, int group, int block) {
+  WorkspaceCarver ws{nullptr, 0, 0};
+  ws.take<uint16_t>((size_t)R * group * d_head);
+  ws.take<char>(plan_bytes_rows(R, nseg, group));
+  ws.take<float>((size_t)(R / block + nseg) * d_head);
+  return align_up(ws.used, 256);
+}
+}  // namespace
+}  // namespace namoh
+
+extern "C" int namoh_sa_mask_words(int T, int block) {
+  if (T < 1 || sa_block_lg(block) < 0) return 0;
+  return sa_words_for(T, block);
+}
+
+extern "C" size_t namoh_sa_prefill_workspace_size(int B, int T, int H, int K, int d_head, int group, int block) {
+  int Hr, Kr;
+  long long R;
+  if (sa_block_lg(block) < 0 || check_shape(B, T, H, K, d_head, group, &Hr, &Kr, &R) != NAMOH_OK) return 0;
+  return sa_workspace_rows(R, B * Hr, d_head, group, block);
+}
+
+extern "C" int namoh_sa_prefill(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int H, int K,
+                                int d_head, int group, float rope_base, unsigned rope_flags,
+                                const int32_t* seg_offsets, const int32_t* row_src, const float* gate, int block,
+                                int alpha_num, int alpha_den, uint32_t* sa_mask, uint16_t* y, uint16_t* k_cache,
+                                uint16_t* v_cache, const int64_t* seg_base, const int32_t* seg_cap,
+                                int64_t cache_rows, int32_t* seg_len, void* workspace, size_t workspace_bytes,
+                                uint32_t* dev_status, void* stream_v) {
+  int Hr, Kr;
+  long long R;
+  const int st = check_shape(B, T, H, K, d_head, group, &Hr, &Kr, &R);
+  if (st != NAMOH_OK) return st;
+  const int lg = sa_block_lg(block);
+  if (lg < 0 || alpha_num < 1 || alpha_den < alpha_num || !sa_mask) return NAMOH_ERR_INVALID_ARG;
+  if ((T + block - 1) / block > kSaMaxBlocks) return NAMOH_ERR_INVALID_ARG;
+  if (!q || !k || !v || !seg_offsets || !row_src || !gate || !y || !k_cache || !v_cache || !dev_status)
+    return NAMOH_ERR_INVALID_ARG;
+  if (!(rope_base > 1.0f) || !isfinite(rope_base) || !rope_flags_ok(rope_flags)) return NAMOH_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(y) || !aligned16(k_cache) || !aligned16(v_cache) ||
+      (reinterpret_cast<uintptr_t>(sa_mask) & 3u))
+    return NAMOH_ERR_INVALID_ARG;
+  if (k_cache == k) return NAMOH_ERR_INVALID_ARG;
+  if (seg_base) {
+    if (!seg_cap || cache_rows < 1 || cache_rows >= (1ll << 31) || v_cache == v) return NAMOH_ERR_INVALID_ARG;
+  } else {
+    cache_rows = R;
+  }
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u)) return NAMOH_ERR_WORKSPACE;
+  const int nseg = B * Hr;
+  WorkspaceCarver ws{static_cast<char*>(workspace), workspace_bytes, 0};
+  uint16_t* q_rot = ws.take<uint16_t>((size_t)R * group * d_head);
+  void* plan = ws.take<char>(plan_bytes_rows(R, nseg, group));
+  float* kbar = ws.take<float>((size_t)(R / block + nseg) * d_head);
+  if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
+  DeviceInfo info;
+  if (!device_ok(&info)) return NAMOH_ERR_UNSUPPORTED;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
+  int rc = launch_rope_and_plan(q, k, v, B, T, Hr, Kr, (int)R, d_head, group, rope_base, rope_flags, nullptr,
+                                seg_offsets, row_src, q_rot, k_cache, v_cache, seg_base, seg_cap, cache_rows,
+                                dev_status, plan, info, stream);
+  if (rc != NAMOH_OK) return rc;
+  if (seg_len) {
+    seg_len_kernel<<<(nseg + 255) / 256, 256, 0, stream>>>(seg_offsets, nseg, seg_len);
+    if (const int st2 = cuda_check_launch("seg_len_kernel launch")) return st2;
+  }
+  const int words = sa_words_for(T, block);
+  rc = launch_sa_select(q_rot, k_cache, seg_offsets, seg_base, nseg, T, R, d_head, group, lg, alpha_num, alpha_den,
+                        kbar, sa_mask, words, stream);
+  if (rc != NAMOH_OK) return rc;
+  return launch_attention(q_rot, k_cache, v_cache, R, d_head, group, seg_offsets, row_src, gate, seg_base, cache_rows,
+                          plan, y, dev_status, info, stream, 0, sa_mask, words, lg);
 }
 
 // ---------------------------------------------------------------------------
