@@ -11,9 +11,11 @@
 //                     the cache) summed in fp32 in row order and scaled by 1 / block (exact: block
 //                     is a power of two) -> kbar[blk_base(s) + b], blk_base(s) = seg_offsets[s] /
 //                     block + s (disjoint per segment, at most R / block + nseg rows).
-//   sa_select_kernel  one warp per query (packed row, group head j): lane l scores blocks
-//                     l, l + 32, ... before the current one (fp32 dot products, four partial sums),
-//                     then R(r) - 1 rounds of a warp arg-max pick the kept blocks; the mask row
+//   sa_select_kernel  one warp per query (packed row, group head j): for each group of 32 blocks
+//                     before the current one, lane l multiplies its d / 32 columns of q~ with those
+//                     columns of every block's pooled key (one coalesced row read per block), and a
+//                     warp reduce-scatter (31 shuffles) leaves block 32 i + l's fp32 score in lane l.
+//                     R(r) - 1 rounds of a warp arg-max then pick the kept blocks; the mask row
 //                     [row * g + j] gets one bit per kept block (bit b % 32 of word b / 32).
 #include "common.cuh"
 
@@ -58,7 +60,6 @@ __global__ void __launch_bounds__(256) sa_select_kernel(const uint16_t* __restri
                                                         const float* __restrict__ kbar, int d, int g, int lg,
                                                         int alpha_num, int alpha_den, long long nq,
                                                         uint32_t* __restrict__ mask, int words) {
-  __shared__ float qs[8][128];
   const int wib = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const long long qi = (long long)blockIdx.x * 8 + wib;  // query number: packed row * g + j
   if (qi >= nq) return;
@@ -74,32 +75,45 @@ __global__ void __launch_bounds__(256) sa_select_kernel(const uint16_t* __restri
   const int cur = r >> lg;                      // current block = N_B(r + 1) - 1
   // kept historical blocks: ceil(alpha (cur + 1)) - 1, computed exactly
   const int keep = (int)(((long long)(cur + 1) * alpha_num + alpha_den - 1) / alpha_den) - 1;
-  for (int c = lane; c < d; c += 32) qs[wib][c] = __uint_as_float((uint32_t)q_rot[qi * d + c] << 16);
-  __syncwarp();
-  const float* kb = kbar + (long long)blk_base(seg_offsets, lo, lg) * d;
+  const int per = d / 32;  // columns of q~ and of the pooled keys per lane (2 or 4)
+  float ql[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e)
+    ql[e] = e < per ? __uint_as_float((uint32_t)q_rot[qi * d + lane * per + e] << 16) : 0.f;
+  const float* kb = kbar + (long long)blk_base(seg_offsets, lo, lg) * d + lane * per;
   // score slots in use: blocks i * 32 + lane < cur (warp-uniform count; the loops below stop there)
   const int nslot = keep > 0 ? (cur + 31) >> 5 : 0;
   float sc[kPerLane];
 #pragma unroll
   for (int i = 0; i < kPerLane; ++i) {
     if (i >= nslot) break;
-    const int b = i * 32 + lane;
-    float acc = -INFINITY;
-    if (b < cur) {
-      // four partial sums (columns c = 4 c4 + e), eight 16-byte loads in flight
-      float a4[4] = {0.f, 0.f, 0.f, 0.f};
-      const float4* kr = reinterpret_cast<const float4*>(kb + (long long)b * d);
-#pragma unroll 8
-      for (int c4 = 0; c4 < d / 4; ++c4) {
-        const float4 x = __ldg(kr + c4);
-        a4[0] = fmaf(qs[wib][4 * c4], x.x, a4[0]);
-        a4[1] = fmaf(qs[wib][4 * c4 + 1], x.y, a4[1]);
-        a4[2] = fmaf(qs[wib][4 * c4 + 2], x.z, a4[2]);
-        a4[3] = fmaf(qs[wib][4 * c4 + 3], x.w, a4[3]);
+    float v[32];  // this lane's partial dot products for blocks 32 i + t
+#pragma unroll
+    for (int t = 0; t < 32; ++t) {
+      const int b = i * 32 + t;
+      float a = 0.f;
+      if (b < cur) {
+        const float* kr = kb + (long long)b * d;
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          if (e < per) a = fmaf(ql[e], __ldg(kr + e), a);
       }
-      acc = (a4[0] + a4[1]) + (a4[2] + a4[3]);
+      v[t] = a;
     }
-    sc[i] = acc;
+    // reduce-scatter: at the step of offset o a lane keeps the half of its live values whose
+    // block index has bit o equal to its own lane bit, adding the partner's copy of that half;
+    // afterwards v[0] of lane l is the whole sum for block 32 i + l
+#pragma unroll
+    for (int o = 16, n = 32; o > 0; o >>= 1, n >>= 1) {
+      const bool up = (lane & o) != 0;
+#pragma unroll
+      for (int jj = 0; jj < n / 2; ++jj) {
+        const float send = up ? v[jj] : v[jj + n / 2];
+        const float mine = up ? v[jj + n / 2] : v[jj];
+        v[jj] = mine + __shfl_xor_sync(0xffffffffu, send, o);
+      }
+    }
+    sc[i] = i * 32 + lane < cur ? v[0] : -INFINITY;
   }
   uint32_t taken = 0;  // bit i: block i * 32 + lane kept
   for (int m = 0; m < keep; ++m) {
