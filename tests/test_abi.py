@@ -100,3 +100,29 @@ def test_rope_flag_errors_return_before_any_launch(lib):
     assert lib.namoh_decode_ex(*a) == -1
     a = list(dargs); a[11] = 0x8; a[12] = None
     assert lib.namoh_decode_ex(*a) == -1
+
+
+def test_sa_sizes_and_argument_errors(lib):
+    """SA + NAMOH: mask words and workspace for the supported block sizes, and every argument error
+    (block size, alpha, null mask, too many blocks) returned before any launch."""
+    assert lib.namoh_sa_mask_words(4096, 32) == 4
+    assert lib.namoh_sa_mask_words(4097, 32) == 5
+    assert lib.namoh_sa_mask_words(4096, 128) == 1
+    assert lib.namoh_sa_mask_words(4096, 48) == 0 and lib.namoh_sa_mask_words(4096, 16) == 0
+    plain = lib.namoh_prefill_workspace_size(4, 4096, 16, 4, 128, 1)
+    # the dense prefill's workspace plus the pooled keys, (R / block + B H) d fp32
+    assert lib.namoh_sa_prefill_workspace_size(4, 4096, 16, 4, 128, 1, 32) >= plain + (65536 // 32 + 64) * 128 * 4
+    assert lib.namoh_sa_prefill_workspace_size(4, 4096, 16, 4, 128, 1, 48) == 0
+    P = ctypes.c_void_p
+    fake = P(256)
+    st = P(512)
+    # q k v B T H K d g base flags seg row_src gate block num den mask y kc vc seg_base seg_cap rows seg_len ws wsb st s
+    args = [fake, fake, fake, 1, 1024, 8, 2, 128, 1, 10000.0, 0, fake, fake, fake, 32, 1, 5, fake, fake, fake, fake,
+            None, None, 0, None, fake, 1 << 24, st, None]
+    for idx, bad in ((14, 48), (14, 16), (15, 0), (15, 6), (16, 0), (17, None), (0, None)):
+        a = list(args)
+        a[idx] = bad
+        assert lib.namoh_sa_prefill(*a) == -1, (idx, bad)
+    a = list(args)
+    a[4] = 32 * 1024 + 1  # 1025 blocks of 32 keys: more than the selector holds
+    assert lib.namoh_sa_prefill(*a) == -1
