@@ -609,7 +609,9 @@ def run_decode(args, dev, pk, pk_kind):
     wl = ni.DECODE
     B, Hr, Kr, d, g = wl.B, wl.Hr, wl.Kr, wl.d, wl.g
     steps = args.decode_steps
-    s = torch.from_numpy(ni.router_scores(wl.seed, B, wl.prefix, Hr)).to(dev)
+    # a shorter prefix only for small profiler captures; the timed workload is the full one
+    prefix = args.decode_prefix or wl.prefix
+    s = torch.from_numpy(ni.router_scores(wl.seed, B, prefix, Hr)).to(dev)
     ws = namoh.Workspace()
     ro = namoh.namoh_route(s, Kr, workspace=ws)
     torch.cuda.synchronize()
@@ -630,7 +632,7 @@ def run_decode(args, dev, pk, pk_kind):
     ev[5].record()
     torch.cuda.synchronize()
     route_biased_ms = ev[0].elapsed_time(ev[5]) / 5
-    route_bytes = acc.route_bytes(B, wl.prefix, Hr, Kr)
+    route_bytes = acc.route_bytes(B, prefix, Hr, Kr)
     seg = ro.seg_offsets.cpu().numpy().astype(np.int64)
     del s, ro
     torch.cuda.empty_cache()
@@ -694,7 +696,8 @@ def run_decode(args, dev, pk, pk_kind):
     bytes_per_step = total_bytes / steps
     gbs = bytes_per_step / (decode_ms * 1e-3) / 1e9
     out = {
-        "workload": wl.name, "steps": steps, "tokens_per_s": B / (step_ms * 1e-3), "ms_per_step": step_ms,
+        "workload": wl.name if prefix == wl.prefix else f"{wl.name} at prefix {prefix} (profiling size)",
+        "steps": steps, "tokens_per_s": B / (step_ms * 1e-3), "ms_per_step": step_ms,
         "route_ms": float(times[:, 0].mean()), "decode_ms": decode_ms, "bytes_per_step": bytes_per_step,
         "hbm_gbs": gbs, "frac_measured_hbm": gbs / pk["hbm_gbs"], "frac_nominal_8tbs": gbs / NOMINAL_HBM_GBS,
         "hbm_peak_source": f"{pk_kind} copy bandwidth {pk['hbm_gbs']} GB/s",
@@ -734,6 +737,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["namoh", "reference"], default="namoh")
     ap.add_argument("--decode-steps", type=int, default=64)
+    ap.add_argument("--decode-prefix", type=int, default=0,
+                    help="routed prefix length of the decode section (0: the workload's 131072); smaller only "
+                         "for profiler captures")
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-layer", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
