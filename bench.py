@@ -597,7 +597,8 @@ def run_sa(args, dev, pk, pk_kind):
             "dense_prefill_ms": ms["dense"], "sa_pairs_over_dense": pairs_sa / pairs_dense,
             "tflops_attended": tf, "frac_bf16": tf / pk["bf16_tflops"], "flops_attended": flops_sa,
             "peak_source": f"{pk_kind} bf16 dense (burst)", "device_status": int(ro.status.item()),
-            "launches": 2 * args.steps * 4,  # per call: RoPE + plan, pooling, selection, attention
+            # per timed pair: SA (RoPE + plan, pooling, selection, attention) and dense (RoPE + plan, attention)
+            "launches": args.steps * (4 + 2),
             "note": "every causal key tile is computed; blocks not kept are masked in the softmax"}
 
 
