@@ -27,7 +27,7 @@
  *
  * Notation (the paper's): B sequences of T tokens; H routed query heads, K
  * active per token; d_head the head width; g query heads per KV group
- * (App. C "Adopted KV-group routing"; g = 1 without grouping).  With grouping
+ * (App. B.7 "Adopted KV-group routing"; g = 1 without grouping).  With grouping
  * the router selects Kr = K/g of Hr = H/g groups, and everything keyed by
  * "head" below is keyed by group.  R = B*T*Kr packed key/value rows.
  */
@@ -197,7 +197,7 @@ NAMOH_API int namoh_route_noalloc(const float *scores, int B, int T, int H, int 
  * Sec. 3.1, Eq. (namoh-attention): h_{t,i} = softmax(q~ k~^T / sqrt(d)) v over
  *   s in I_i, s <= t; the combine writes the per-slot term g_{t,i} h_{t,i}
  *   (the W_O projection is outside this path).
- * App. C "Adopted KV-group routing": the g query heads of a group share its
+ * App. B.7 "Adopted KV-group routing": the g query heads of a group share its
  *   keys, values, gate and rank.
  * Sec. 3.2 "Efficient execution": length-aware scheduling of query tiles.
  *
@@ -335,7 +335,7 @@ NAMOH_API int namoh_decode_ex(const int32_t *topk_head, const float *gate, const
                               void *stream);
 
 /* ------------------------------------------------------------------------- *
- * Shared heads: the paper's shared-head variant (Sec. 5, "Shared heads for local
+ * Shared heads: the paper's shared-head variant (Sec. 4.4, "Shared heads for local
  * context"): Hs always-active heads, outside the routing, each attending to the full
  * causal prefix (window = 0) or to the most recent `window` tokens including the current
  * one, with RoPE at the token's global position and no gate.  Their outputs are summed
@@ -367,7 +367,7 @@ NAMOH_API int namoh_shared_decode(const uint16_t *q, const uint16_t *k, const ui
                                   size_t workspace_bytes, uint32_t *dev_status, void *stream);
 
 /* ------------------------------------------------------------------------- *
- * SA + NAMOH: block-selected sparse attention inside each routed history (App. B.4
+ * SA + NAMOH: block-selected sparse attention inside each routed history (App. B.8
  * "SA+NAMOH", with the selection model of App. B.3 "Block-Selected Sparse Attention",
  * Eqs. app-block-budget and app-selected-entries).  The routed history of each (batch,
  * head) is cut into blocks of `block` entries in its local order.  A query at one-based
@@ -408,9 +408,10 @@ NAMOH_API int namoh_sa_prefill(const uint16_t *q, const uint16_t *k, const uint1
  * Sec. 3.1, Eq. (namoh-qkv): only an active token-head pair projects,
  *   q_{t,i} = x_t W_Q^(i), k_{t,i} = x_t W_K^(i), v_{t,i} = x_t W_V^(i), t in I_i.
  * Sec. 3.1, Eq. (namoh-attention): o_t = sum_{i in S_K(t)} g_{t,i} h_{t,i} W_O^(i).
- * App. C: a KV group projects one key, one value and g queries (one per query head).
+ * App. B.7: a KV group projects one key, one value and g queries (one per query head).
  * Both run as one grouped GEMM over the packed rows of the routing (tcgen05 tiles of 128
- * rows, the rows gathered from the token axis by TMA), so they follow namoh_route or
+ * rows, the A rows gathered from the token axis by 16-byte cp.async copies, the weight
+ * tiles loaded by TMA), so they follow namoh_route or
  * namoh_route_varlen directly: seg_offsets [B*Hr + 1] and row_src [R] are its outputs,
  * R = total_tokens * Kr (total_tokens = B*T for a fixed-length batch).
  *

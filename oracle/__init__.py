@@ -14,12 +14,12 @@ it follows:
                    Sec. 3.2 Eq. (namoh-head-rope) for the rank rho.
 * ``rope``         Sec. 3.2 Eq. (namoh-head-rope), half-split RoPE.
 * ``prefill``      Sec. 3.1 Eq. (namoh-attention) over packed (batch, head)
-                   subsequences (Sec. 3.2 "Efficient execution"); App. C
+                   subsequences (Sec. 3.2 "Efficient execution"); App. B.7
                    "Adopted KV-group routing" for g > 1.
 * ``prefill_rows`` the same for a chosen subset of query rows.
 * ``decode_step``  Sec. 3.1 (last paragraph): append to and attend within only
                    the selected heads' histories.
-* ``sa_prefill``   App. B.4 "SA+NAMOH" with the block-selection model of App. B.3
+* ``sa_prefill``   App. B.8 "SA+NAMOH" with the block-selection model of App. B.3
                    (Eqs. app-block-budget, app-selected-entries): blocks of the routed
                    history in local order, the current block plus the highest-scoring
                    completed blocks against their mean-pooled keys.
@@ -371,7 +371,7 @@ def proj_out(y, topk_head, w_o, g: int, d: int, nthreads: int | None = None):
 
 
 def shared_prefill(q, k, v, window: int, base: float, interleaved: bool = False, nthreads: int | None = None):
-    """Shared heads (Sec. 5): q, k, v [B, Hs, T, d] bf16 bits; full causal (window 0) or sliding
+    """Shared heads (Sec. 4.4): q, k, v [B, Hs, T, d] bf16 bits; full causal (window 0) or sliding
     window attention at global positions, no gate.  Returns y [B, T, Hs, d] fp64."""
     lib = _load()
     q = np.ascontiguousarray(q, dtype=np.uint16)
@@ -404,7 +404,7 @@ def sa_mask_words(n_max: int, block: int) -> int:
 def sa_prefill(q, k, v, seg_offsets, row_src, gate, d: int, g: int, base: float, block: int,
                alpha_num: int, alpha_den: int, mask_in: np.ndarray | None = None, want_mask: bool = False,
                nthreads: int | None = None, interleaved: bool = False, pos: np.ndarray | None = None):
-    """SA + NAMOH prefill over packed rows (App. B.4, selection model of App. B.3).
+    """SA + NAMOH prefill over packed rows (App. B.8, selection model of App. B.3).
 
     alpha = alpha_num / alpha_den.  mask_in [R*g, W] uint32 (W >= sa_mask_words of the longest
     history) replaces the selection; want_mask also returns the blocks kept.  Returns y [R*g, d] fp64 (and the mask).

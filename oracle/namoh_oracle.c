@@ -9,7 +9,7 @@
  * Everything here follows the paper's definitions literally, in fp64:
  *   - routing:   Sec. 3.1, Eq. (namoh-gates)  a_t = softmax(x_t W_r), S_K(t) = TopK(a_t),
  *                m_{t,i} = 1{i in S_K(t)}, g_{t,i} = m_{t,i} a_{t,i}  (no renormalisation,
- *                App. A, Eq. (namoh-biased-routing) and the sentence after it).
+ *                App. A.3, Eq. (namoh-biased-routing) and the sentence after it).
  *   - dispatch:  Sec. 3.1, ordered index sets I_i = {t : m_{t,i} = 1}, n_i = |I_i|;
  *                Sec. 3.2 "Efficient execution": each (batch, head) subsequence is packed
  *                as an independent sequence.
@@ -22,11 +22,11 @@
  *                packed layout; Eq. (namoh-attention)  o_t = sum_i g_{t,i} h_{t,i} W_O^(i).
  *   - decode:    Sec. 3.1 (last paragraph) and Sec. 3.2: a new token appends to and attends
  *                within only its selected heads' histories; its rank is the current length.
- *   - GQA:       App. C, "Adopted KV-group routing": K/g of H/g groups are selected, the g
+ *   - GQA:       App. B.7, "Adopted KV-group routing": K/g of H/g groups are selected, the g
  *                query heads of a group share its gate, key/value history and rank.
- *   - shared:    the shared-head variant (Sec. 5): always-active heads over the full causal
+ *   - shared:    the shared-head variant (Sec. 4.4): always-active heads over the full causal
  *                prefix or a sliding window of the last w tokens, at global RoPE positions.
- *   - SA+NAMOH:  App. B.4 with the selection model of App. B.3, Eqs. (app-block-budget) and
+ *   - SA+NAMOH:  App. B.8 with the selection model of App. B.3, Eqs. (app-block-budget) and
  *                (app-selected-entries): blocks of Bk entries in each routed history's local
  *                order; the current block plus the ceil(alpha N_B(r)) - 1 completed blocks
  *                scoring highest against their mean-pooled keys.
@@ -156,7 +156,7 @@ int oracle_route_topk(const float *scores, long N, int H, int K, int32_t *topk_h
 }
 
 /*
- * oracle_route_biased: App. A, Eq. (namoh-biased-routing).  In fp64, per token:
+ * oracle_route_biased: App. A.3, Eq. (namoh-biased-routing).  In fp64, per token:
  *   a_t = softmax(x_t W_r) over all H heads,
  *   S_K(t) = TopK_i(a_{t,i} + b_i)  (larger first, ties to the lower index),
  *   g_{t,i} = a_{t,i} at the selected heads (the bias stays out of the gates).
@@ -658,7 +658,7 @@ static void proj_qkv_row(long r, void *arg)
 /*
  * oracle_proj_qkv: Sec. 3.1, Eq. (namoh-qkv): only active token-head pairs project,
  *   q_{t,i} = x_t W_Q^(i), k_{t,i} = x_t W_K^(i), v_{t,i} = x_t W_V^(i), t in I_i,
- * in the packed-row layout of the routing (App. C: a KV group projects one key and one
+ * in the packed-row layout of the routing (App. B.7: a KV group projects one key and one
  * value and g queries, one per query head of the group).
  *   x           [N, d_model] bf16 token representations (N tokens on the flat axis)
  *   w           [Hr, (g+2) d, d_model] bf16: for group i, rows j d .. j d + d - 1 hold
@@ -770,7 +770,7 @@ done:
 
 /*
  * oracle_shared_prefill: the always-active shared heads of the paper's shared-head variant
- * (Sec. 5, "Shared heads for local context"): every token, causal attention over the full
+ * (Sec. 4.4, "Shared heads for local context"): every token, causal attention over the full
  * prefix (window = 0) or over the most recent `window` tokens including itself, RoPE at the
  * global position t, no gate.
  *   q, k, v  [B, Hs, T, d] bf16 bits (each head's sequence contiguous)
@@ -787,7 +787,7 @@ int oracle_shared_prefill(const uint16_t *q, const uint16_t *k, const uint16_t *
 
 /* ------------------------------------------------------------------------- */
 /* SA + NAMOH: block selection inside each routed history (App. B.3 "Block-   */
-/* Selected Sparse Attention", App. B.4 "SA+NAMOH")                           */
+/* Selected Sparse Attention", App. B.8 "SA+NAMOH")                           */
 /* ------------------------------------------------------------------------- */
 
 /*

@@ -3,14 +3,14 @@
 These are the counts the benchmark divides by time; none of them runs on the
 GPU path and none depends on the oracle.
 
-* App. C, Eq. (app-routed-interactions): the causal interaction count of one
+* App. B.5, Eq. (app-routed-interactions): the causal interaction count of one
   sequence is C_attn = sum_i n_i (n_i + 1) / 2.
-* App. C, Eq. (app-group-prefill): under KV-group routing each local rank
+* App. B.7, Eq. (app-group-prefill): under KV-group routing each local rank
   produces g queries, so C_attn = g * sum_j n_j (n_j + 1) / 2.
-* App. C, Eq. (app-routed-kv): M_KV = sum_i n_i = T K (storage) and
+* App. B.5, Eq. (app-routed-kv): M_KV = sum_i n_i = T K (storage) and
   A_KV(T) = sum_{i in S_K(T)} n_i (activation of the next token).
-* App. C, Eq. (app-load-cv): CV(n)^2 with the population variance.
-* App. C, Eq. (app-interaction-bounds):
+* App. B.5, Eq. (app-load-cv): CV(n)^2 with the population variance.
+* App. B.5, Eq. (app-interaction-bounds):
   T^2 K^2 / (2H) + T K / 2 <= C_attn <= K T (T + 1) / 2.
 
 Each interaction costs one d-length dot product for Q K^T and one d-length

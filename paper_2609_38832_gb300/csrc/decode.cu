@@ -1,6 +1,6 @@
 // decode.cu -- one decode step over routed KV histories (Sec. 3.1 last paragraph; Sec. 3.2
 // "Efficient execution": only the active heads' queries run and only their caches are read
-// or updated; App. C "Adopted KV-group routing" for g > 1).
+// or updated; App. B.7 "Adopted KV-group routing" for g > 1).
 //
 // Three launches:
 //   1. decode_append_kernel  one warp per (sequence, slot): rho = seg_len[s]; k~ = k R(p)

@@ -1,7 +1,7 @@
 // prefill_attn.cu -- routed causal attention over packed (batch, head) segments with the
 // gate-weighted combine fused into the epilogue (Sec. 3.1, Eq. namoh-attention; Sec. 3.2
 // "Efficient execution": packed variable-length subsequences and length-aware scheduling;
-// App. C "Adopted KV-group routing" for g > 1).
+// App. B.7 "Adopted KV-group routing" for g > 1).
 //
 // Work unit ("item"): one 128-row query tile t of one segment for one group head j.  Within
 // a segment, queries and keys share local ranks, so tile t needs key tiles 0..t and only
@@ -1019,7 +1019,7 @@ extern "C" int namoh_prefill(const uint16_t* q, const uint16_t* k, const uint16_
 }
 
 // ---------------------------------------------------------------------------
-// SA + NAMOH (App. B.4, selection model of App. B.3): block selection inside each routed history,
+// SA + NAMOH (App. B.8, selection model of App. B.3): block selection inside each routed history,
 // then the routed attention over the kept blocks and the query's current block.
 // ---------------------------------------------------------------------------
 namespace namoh {

@@ -1,6 +1,6 @@
 // proj.cu -- the projections around the routed-attention path (Sec. 3.1).
 //
-// One grouped GEMM over the packed rows of the routing (one group per KV-group head i, App. C),
+// One grouped GEMM over the packed rows of the routing (one group per KV-group head i, App. B.7),
 // the A rows gathered from the token axis, in two modes:
 //   QKV   (Eq. namoh-qkv): row r of segment (b, i) computes x_t [W_Q^(ig..ig+g-1) | W_K^(i) |
 //         W_V^(i)] for t = row_src[r] / Kr, written as g query rows, one key row and one value

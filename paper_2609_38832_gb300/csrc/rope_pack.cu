@@ -8,7 +8,7 @@
 // g >= 4, half of its query heads or less): the row's segment s comes from a binary search
 // over seg_offsets (staged in shared memory), rho = r - seg_offsets[s], and each thread
 // rotates 8 pairs (j, j + D/2) with angles it computes once for the row; KV-group routing
-// shares the rank between the key and the row's g query heads (App. C).
+// shares the rank between the key and the row's g query heads (App. B.7).
 // Variants: the interleaved pairing (2j, 2j+1) keeps the same 16-byte accesses (elements
 // [8l, 8l+8) and [D/2 + 8l, D/2 + 8l + 8) for lane l of a group) and pairs adjacent elements
 // inside them, so the lane's angles are j = 4l..4l+3 and D/4 + 4l..D/4 + 4l+3; global

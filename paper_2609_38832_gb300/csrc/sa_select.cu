@@ -1,4 +1,4 @@
-// sa_select.cu -- block selection of SA + NAMOH (App. B.4 "SA+NAMOH", with the selection model of
+// sa_select.cu -- block selection of SA + NAMOH (App. B.8 "SA+NAMOH", with the selection model of
 // App. B.3 "Block-Selected Sparse Attention", Eqs. app-block-budget and app-selected-entries).
 //
 // Within each routed history (a segment of packed rows in local order), the keys form blocks of

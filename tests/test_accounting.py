@@ -1,4 +1,4 @@
-"""Host-side accounting (App. C) against brute-force counts and the paper's closed forms."""
+"""Host-side accounting (App. B.7) against brute-force counts and the paper's closed forms."""
 import numpy as np
 import pytest
 

@@ -97,7 +97,7 @@ def _decode_check(namoh, oracle_mod, B, T, Hr, Kr, d, g, steps, variant):
         assert_close_attention(bf16_to_f64(y), y_ref, gate, what=f"step {t}")
         np.testing.assert_array_equal(st["seg_len"].cpu().numpy(), olen)
     assert int(status.item()) == 0
-    # M_KV = T K after the prefix and + K per step (App. C Eq. app-routed-kv)
+    # M_KV = T K after the prefix and + K per step (App. B.5 Eq. app-routed-kv)
     assert int(st["seg_len"].sum().item()) == B * (T + steps) * Kr
     # the appended keys: the oracle's k~ rounded to bf16
     kc_got = bf16_to_f64(st["kc"])

@@ -1,7 +1,7 @@
 """GPU parity of the projections around the path (the full attention layer).
 
 Sec. 3.1 Eq. (namoh-qkv): q, k, v = x W^(i) for active token-head pairs only, in the packed
-layout.  Eq. (namoh-attention): o_t = sum_i g h W_O^(i).  App. C: g queries per KV group.
+layout.  Eq. (namoh-attention): o_t = sum_i g h W_O^(i).  App. B.7: g queries per KV group.
 Each stage is compared with the oracle on the same bf16 inputs: the projections' bf16 outputs
 within half a bf16 ulp of the fp64 value (|err| <= 2^-8 |ref| + 1e-3); the fp32 o sums per-slot
 products that were rounded to bf16, so |err| <= 2^-8 (sum of |y| |W_O| over its terms) + 1e-5.

@@ -1,6 +1,6 @@
 """GPU parity of prefill (RoPE at rank, routed causal attention, gate-weighted combine).
 
-Sec. 3.2 Eq. (namoh-head-rope); Sec. 3.1 Eq. (namoh-attention); App. C KV-group routing.
+Sec. 3.2 Eq. (namoh-head-rope); Sec. 3.1 Eq. (namoh-attention); App. B.7 KV-group routing.
 Small cases compare every output with the full oracle; the full-size workloads compare
 sampled query rows (each segment's first and last rows, both sides of the longest
 segment's tile boundaries, random rows) with the oracle's row-subset entry point.

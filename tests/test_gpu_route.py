@@ -125,7 +125,7 @@ def test_route_repeated_calls_reuse_workspace(namoh, oracle_mod):
 
 
 # --------------------------------------------------------------------------- biased selection
-# App. A, Eq. (namoh-biased-routing).  The GPU ranks fp32 affinities (exp2 of pre-scaled logit
+# App. A.3, Eq. (namoh-biased-routing).  The GPU ranks fp32 affinities (exp2 of pre-scaled logit
 # differences) plus the bias; the oracle ranks the same sums in fp64.  Where two sums lie
 # within the fp32 error bound of each other either order is correct, so the selection is
 # checked for validity within that bound, and for equality with the oracle wherever the

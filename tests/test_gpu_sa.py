@@ -1,4 +1,4 @@
-"""GPU parity of SA + NAMOH (App. B.4 with the selection model of App. B.3).
+"""GPU parity of SA + NAMOH (App. B.8 with the selection model of App. B.3).
 
 The kept blocks decide which keys each query sees, and they are decided by fp32 scores of
 bf16-rounded rotated queries and pooled keys.  So the test checks what is unique and that the rest

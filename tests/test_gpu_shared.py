@@ -1,4 +1,4 @@
-"""GPU parity of the shared heads (the paper's shared-head variant, Sec. 5): always-active heads
+"""GPU parity of the shared heads (the paper's shared-head variant, Sec. 4.4): always-active heads
 over the full causal prefix or a sliding window of the last w tokens, global RoPE, no gate.
 The attention kernel runs them as segments holding every token (rank = t) with its key tiles
 starting at the window; decode attends over the last min(n + 1, w) cached rows.

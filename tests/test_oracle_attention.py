@@ -9,8 +9,8 @@ What the paper fixes, each checked by a formulation unlike the oracle's:
     over the full T x T grid, zero outside routed causal pairs -> brute-force masks.
   * Sec. 3.1: each query attends only to earlier tokens (and itself) of the same head.
   * Sec. 3.1 (end): prefill and incremental decoding are the same causal computation.
-  * App. C Eq. (app-routed-kv): M_KV = T K after the prefix, + K per decode step.
-  * App. C "Adopted KV-group routing": g query heads share a group's keys, values,
+  * App. B.5 Eq. (app-routed-kv): M_KV = T K after the prefix, + K per decode step.
+  * App. B.7 "Adopted KV-group routing": g query heads share a group's keys, values,
     gate and rank.
   * Sec. 3.2 (end of "Head-relative positional encoding"): global RoPE replaces rho_i(t) by t
     -> the brute-force masks with t as the position, and prefill == decode at token index t.

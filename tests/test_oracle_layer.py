@@ -2,7 +2,7 @@
 
 Sec. 3.1 Eq. (namoh-qkv): only active token-head pairs project, q = x W_Q^(i), k = x W_K^(i),
 v = x W_V^(i), W in R^{d_model x d_head}.  Eq. (namoh-attention): o_t = sum_{i in S_K(t)}
-g_{t,i} h_{t,i} W_O^(i), W_O^(i) in R^{d_head x d_model}.  App. C: a KV group projects one key
+g_{t,i} h_{t,i} W_O^(i), W_O^(i) in R^{d_head x d_model}.  App. B.7: a KV group projects one key
 and one value, and one query per query head.
 Each check uses the paper's dense matrices and a formulation unlike the oracle's (dense
 products over every head, then the active pairs; torch scaled_dot_product_attention for K = H).

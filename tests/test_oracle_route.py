@@ -1,7 +1,7 @@
 """Pins of the oracle's routing and dispatch against what the paper fixes.
 
 Sec. 3.1 Eq. (namoh-gates): TopK over affinities, mask, gates (not renormalised).
-Sec. 3.1: ordered index sets I_i; App. C Eq. (app-assignment-count): sum_i n_i = T K.
+Sec. 3.1: ordered index sets I_i; App. B.5 Eq. (app-assignment-count): sum_i n_i = T K.
 Sec. 3.2 Eq. (namoh-head-rope): rho_i(t) = sum_{s<=t} m_{s,i} - 1.
 Each test uses a formulation that differs from the oracle's (counting ranks instead of
 sorting, cumulative sums of the mask instead of appending, library softmax / topk).
@@ -86,7 +86,7 @@ def test_dispatch_matches_mask_cumsum(oracle_mod, B, T, H, K):
     np.testing.assert_array_equal(out["rank"], np.take_along_axis(rho, top, axis=-1))
     n = mask.sum(axis=1)
     np.testing.assert_array_equal(out["n"], n)
-    # App. C Eq. (app-assignment-count): sum_i n_i = T K for every sequence
+    # App. B.5 Eq. (app-assignment-count): sum_i n_i = T K for every sequence
     np.testing.assert_array_equal(n.sum(-1), T * K)
     seg = np.concatenate([[0], np.cumsum(n.reshape(-1))])
     np.testing.assert_array_equal(out["seg_offsets"], seg)
@@ -103,7 +103,7 @@ def test_dispatch_matches_mask_cumsum(oracle_mod, B, T, H, K):
 
 
 def test_all_tokens_same_heads(oracle_mod):
-    # App. C after Eq. (app-interaction-bounds): every token selecting the same K heads
+    # App. B.5 after Eq. (app-interaction-bounds): every token selecting the same K heads
     B, T, H, K = 2, 50, 8, 3
     s = np.tile(np.linspace(1.0, -1.0, H, dtype=np.float32), (B, T, 1))
     out = oracle_mod.route(s, K)
@@ -165,7 +165,7 @@ def test_nonfinite_scores_rejected(oracle_mod):
 
 
 # --------------------------------------------------------------------------- biased selection
-# App. A, Eq. (namoh-biased-routing): S_K(t) = TopK_i(a_{t,i} + b_i), g_{t,i} = m_{t,i} a_{t,i}.
+# App. A.3, Eq. (namoh-biased-routing): S_K(t) = TopK_i(a_{t,i} + b_i), g_{t,i} = m_{t,i} a_{t,i}.
 
 def _affinity(scores: np.ndarray) -> np.ndarray:
     return scipy.special.softmax(scores.astype(np.float64), axis=-1)

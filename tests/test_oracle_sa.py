@@ -1,4 +1,4 @@
-"""Pins of the oracle's SA + NAMOH block selection (App. B.4 with the selection model of App. B.3).
+"""Pins of the oracle's SA + NAMOH block selection (App. B.8 with the selection model of App. B.3).
 
 What the paper fixes, each checked by a formulation unlike the oracle's:
   * Eq. (app-block-budget): N_B(r) = ceil(r / B) blocks, R(r) = ceil(alpha N_B(r)) kept, the current
@@ -11,7 +11,7 @@ What the paper fixes, each checked by a formulation unlike the oracle's:
     independent per-query scoring routine; planted block orders whose selection and output have
     closed forms.
   * Future blocks are excluded: outputs never depend on later keys or values.
-  * App. C "Adopted KV-group routing": the g query heads of a group select independently over
+  * App. B.7 "Adopted KV-group routing": the g query heads of a group select independently over
     shared keys -> equal to g separate single-head runs.
 """
 from fractions import Fraction

@@ -1,4 +1,4 @@
-"""Pins of the oracle's shared heads (the paper's shared-head variant, Sec. 5 "Shared heads for
+"""Pins of the oracle's shared heads (the paper's shared-head variant, Sec. 4.4 "Shared heads for
 local context"): always-active heads attending to the full causal prefix or to the most recent
 w tokens including the current one, with global RoPE and no gate.
 
