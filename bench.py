@@ -15,8 +15,11 @@ The end-to-end figure ("e2e") goes through namoh_route + namoh_prefill from pinn
 buffers: every step copies its own inputs in and its own y out, with consecutive steps
 overlapped on three streams, as a server would run them.
 
-The decode workload (64 sequences with 131072-token routed prefixes, H = 32, K = 4,
-d = 128, 17.4 GB KV cache) is measured in the same run and reported under "decode".
+The other prefill workloads (PR1, the skewed 32k-token workload, the H sweep at 16k tokens and
+its GQA variant) are measured in the same run under "configs", each with its attention kernel's
+roofline fraction and the oracle timed on the host cores beside it.  The decode workload (64
+sequences with 131072-token routed prefixes, H = 32, K = 4, d = 128, 17.4 GB KV cache, 256 steps)
+is reported under "decode", with the oracle timed on two of its sequences for every step.
 
 --impl reference runs the fp64 CPU oracle (the reference arm for this path) on a
 bounded sample of the same workload.  Under torchrun each rank runs its own replica
@@ -139,6 +142,13 @@ def cpu_model():
     return platform.processor() or platform.machine()
 
 
+def stats(ms):
+    """Summary of per-launch (or per-step) times in ms: mean, median, p10, p90."""
+    a = np.asarray(ms, dtype=np.float64)
+    return {"mean": float(a.mean()), "median": float(np.median(a)), "p10": float(np.percentile(a, 10)),
+            "p90": float(np.percentile(a, 90)), "n": int(a.size)}
+
+
 # --------------------------------------------------------------------------- oracle (CPU baseline)
 def oracle_prefill_sample(wl: ni.PrefillWorkload, min_seconds: float = 10.0, max_reps: int = 64):
     """The oracle, as it stands, on the full workload (route + prefill), repeated until min_seconds."""
@@ -239,8 +249,8 @@ def run_gpu(args, rank: int, world: int):
     flush_ms = [a.elapsed_time(b) for a, b in fl_ev]
     # the host finished enqueueing each step before the flush ahead of it ended
     gapless = all(e * 1e3 < f for e, f in zip(enqueue_s, flush_ms))
-    step_ms = float(np.mean([a.elapsed_time(b) for a, b in step_ev]))
-    step_ms = max_over_ranks(step_ms, world)
+    step_times = [a.elapsed_time(b) for a, b in step_ev]
+    step_ms = max_over_ranks(float(np.median(step_times)), world)
 
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
     for i in range(args.steps):
@@ -248,7 +258,7 @@ def run_gpu(args, rank: int, world: int):
         step(evs[i])
     torch.cuda.synchronize()
     stage = np.array([[evs[i][j].elapsed_time(evs[i][j + 1]) for j in range(3)] for i in range(args.steps)])
-    attn_ms = float(stage[:, 2].mean())
+    attn_ms = float(stage[:, 2].mean())  # the roofline divides by the kernel's average launch duration
     st = int(status.item())
 
     # ---- the RoPE/plan launch alone in each RoPE variant (Sec. 3.2: rank or global position;
@@ -370,12 +380,14 @@ def run_gpu(args, rank: int, world: int):
                    "l2": "flushed before every timed step (2 GB write)", "seed": wl.seed,
                    "c_attn": acc.interaction_count(n_seg, g), "flops_per_step": flops,
                    "cv2_mean": float(np.mean([acc.cv2(n_seg[b * wl.Hr:(b + 1) * wl.Hr]) for b in range(B)]))},
-        "stages_ms": {"route": float(stage[:, 0].mean()), "rope_pack_plan": float(stage[:, 1].mean()),
-                      "attention": attn_ms, "note": "separate pass, an event between stages (no overlap)"},
+        "step_ms_stats": stats(step_times),
+        "stages_ms": {"route": stats(stage[:, 0]), "rope_pack_plan": stats(stage[:, 1]),
+                      "attention": stats(stage[:, 2]), "note": "separate pass, an event between stages (no overlap)"},
         "rope_variants": rope_variants,
         "roofline": {"kernel": "attn_fwd_kernel<128>", "bound": "tensor", "achieved": achieved, "peak": peak_tf,
                      "unit": "TFLOP/s", "frac": achieved / peak_tf, "traffic": traffic,
-                     "peak_source": f"{pk_kind} bf16 dense (burst)",
+                     "frac_sustained": achieved / pk.get("bf16_tflops_sustained", peak_tf),
+                     "peak_source": f"{pk_kind} bf16 dense (burst); frac_sustained against the sustained figure",
                      "algorithmic": "4 * d_head * C_attn flops per launch (exact causal pairs)"},
         "e2e": {"value": world * flops / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s", "ms_per_step": e2e_ms,
                 "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
@@ -392,6 +404,9 @@ def run_gpu(args, rank: int, world: int):
         "device_status": st,
     }
 
+    if not args.no_configs:
+        line["configs"] = run_configs(args, dev, pk, pk_kind)
+        line["gpu_launches"] += line["configs"].pop("launches")
     if not args.no_decode:
         line["decode"] = run_decode(args, dev, pk, pk_kind)
         line["gpu_launches"] += line["decode"].pop("launches")
@@ -405,6 +420,109 @@ def run_gpu(args, rank: int, world: int):
     clocks.__exit__(None, None, None)
     line["clocks"] = clocks.summary()
     return line
+
+
+# The other prefill workloads: each is a parity case of the tests and is measured here as its own
+# section (the headline stays on the balanced workload).
+CONFIG_WORKLOADS = (ni.PR1, ni.SKEWED, *ni.H_SWEEP, ni.GQA)
+
+
+def run_configs(args, dev, pk, pk_kind):
+    """Every other prefill workload: route, RoPE + plan and attention timed apart (an event between
+    stages) and as whole steps, the L2 flushed before each; the attention kernel against the bf16
+    peaks; routing and RoPE against HBM; the per-token KV accesses of App. B.5 (C_attn / T in
+    prefill, Eq. app-routed-interactions; A_KV(T) of the last token, Eq. app-routed-kv); and the
+    oracle timed on the host cores on the same workload."""
+    import torch
+
+    import paper_2609_38832_gb300 as namoh
+
+    flush = torch.empty(2 << 30, dtype=torch.uint8, device=dev)
+    up = lambda b: torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).to(dev).view(torch.bfloat16)  # noqa: E731
+    out = {"peak_source": f"{pk_kind} bf16 dense: burst {pk['bf16_tflops']}, sustained "
+                          f"{pk.get('bf16_tflops_sustained')} TFLOP/s; HBM {pk['hbm_gbs']} GB/s",
+           "l2": "flushed before every timed step (2 GB write)"}
+    launches = 0
+    for wl in CONFIG_WORKLOADS:
+        B, T, H, K, d, g = wl.B, wl.T, wl.H, wl.K, wl.d, wl.g
+        scores_h = wl.scores()
+        q_h, k_h, v_h = wl.qkv()
+        scores = torch.from_numpy(scores_h).to(dev)
+        q, k, v = up(q_h), up(k_h), up(v_h)
+        ws = namoh.Workspace()
+        status = torch.zeros(1, dtype=torch.int32, device=dev)
+        ro = namoh.namoh_route(scores, wl.Kr, workspace=ws, status=status)
+        q_rot, k_cache = torch.empty_like(q), torch.empty_like(k)
+        plan = namoh.namoh_attention_plan(ro.seg_offsets, B=B, T=T, H=H, K=K, group=g)
+        y = torch.empty((B, T, K, d), dtype=torch.bfloat16, device=dev)
+        stages = (
+            lambda: namoh.namoh_route(scores, wl.Kr, workspace=ws, status=status, out=ro),
+            lambda: namoh.namoh_rope_pack(q, k, v, ro.seg_offsets, B=B, T=T, H=H, K=K, group=g, rope_base=wl.base,
+                                          q_rot=q_rot, k_cache=k_cache, v_cache=v, status=status, plan=plan),
+            lambda: namoh.namoh_attention(q_rot, k_cache, v, ro.seg_offsets, ro.row_src, ro.gate, plan, B=B, T=T,
+                                          H=H, K=K, group=g, y=y, status=status),
+        )
+        whole = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+        parts = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+        for i in range(args.warmup + args.steps):  # whole steps (kernels overlap by programmatic launch)
+            flush.fill_(i & 0xFF)
+            if i >= args.warmup:
+                whole[i - args.warmup][0].record()
+            for f in stages:
+                f()
+            if i >= args.warmup:
+                whole[i - args.warmup][1].record()
+        for i in range(args.steps):  # the stage breakdown
+            flush.fill_(i & 0xFF)
+            for j, f in enumerate(stages):
+                parts[i][j].record()
+                f()
+            parts[i][3].record()
+        torch.cuda.synchronize()
+        launches += 2 * args.steps * 4  # route 2 + RoPE/plan 1 + attention 1, in both passes
+        step_t = [a.elapsed_time(b) for a, b in whole]
+        st_t = np.array([[parts[i][j].elapsed_time(parts[i][j + 1]) for j in range(3)] for i in range(args.steps)])
+        seg = ro.seg_offsets.cpu().numpy()
+        n_seg = acc.segment_lengths(seg)
+        flops = acc.attention_flops(n_seg, d, g)
+        c_attn = acc.interaction_count(n_seg, g)
+        top = ro.topk_head.cpu().numpy()
+        a_kv = [acc.kv_activation(n_seg[b * wl.Hr:(b + 1) * wl.Hr], top[b, T - 1]) for b in range(B)]
+        R = B * T * wl.Kr
+        rbytes = acc.route_bytes(B, T, wl.Hr, wl.Kr)
+        pbytes = acc.rope_pack_bytes(R, d, g, copy_v=False)
+        attn_mean = float(st_t[:, 2].mean())
+        achieved = flops / (attn_mean * 1e-3) / 1e12
+        gbs = lambda nbytes, ms: nbytes / (ms * 1e-3) / 1e9  # noqa: E731
+        entry = {
+            "shape": {"B": B, "T": T, "H": H, "K": K, "d_head": d, "group": g, "rope_base": wl.base,
+                      "zipf_bias": wl.zipf_bias, "seed": wl.seed},
+            "segments": {"n_max": int(n_seg.max()), "n_min": int(n_seg.min()),
+                         "cv2_mean": float(np.mean([acc.cv2(n_seg[b * wl.Hr:(b + 1) * wl.Hr]) for b in range(B)]))},
+            "c_attn": c_attn, "flops": flops,
+            "kv_accesses_per_token_prefill": c_attn / (B * T),
+            "a_kv_last_token": float(np.mean(a_kv)),
+            "kv_storage_per_sequence": int(acc.kv_storage(n_seg)) // B,
+            "step_ms": stats(step_t), "step_tflops": flops / (np.median(step_t) * 1e-3) / 1e12,
+            "route": {"ms": stats(st_t[:, 0]), "bytes": rbytes, "hbm_gbs": gbs(rbytes, st_t[:, 0].mean()),
+                      "frac_measured_hbm": gbs(rbytes, st_t[:, 0].mean()) / pk["hbm_gbs"]},
+            "rope_pack_plan": {"ms": stats(st_t[:, 1]), "bytes": pbytes, "hbm_gbs": gbs(pbytes, st_t[:, 1].mean()),
+                               "frac_measured_hbm": gbs(pbytes, st_t[:, 1].mean()) / pk["hbm_gbs"]},
+            "roofline": {"kernel": f"attn_fwd_kernel<{d}>", "bound": "tensor", "achieved": achieved,
+                         "peak": pk["bf16_tflops"], "unit": "TFLOP/s", "frac": achieved / pk["bf16_tflops"],
+                         "frac_sustained": achieved / pk.get("bf16_tflops_sustained", pk["bf16_tflops"]),
+                         "ms": stats(st_t[:, 2])},
+            "device_status": int(status.item()),
+        }
+        if not args.no_cpu_baseline:
+            cb = oracle_prefill_sample(wl, min_seconds=3.0)
+            entry["cpu_baseline"] = {k_: cb[k_] for k_ in ("value", "unit", "cores", "kind", "sample")}
+            entry["cpu_baseline"]["seconds_per_step"] = cb["seconds_per_step"]
+        out[wl.name] = entry
+        del scores, q, k, v, q_rot, k_cache, y, ro, plan, ws
+        torch.cuda.empty_cache()
+    out["launches"] = launches
+    return out
 
 
 LAYER_D_MODEL = 2048  # the paper's model width (its experiments fix 2048)
@@ -650,6 +768,21 @@ def run_decode(args, dev, pk, pk_kind):
     seg_len = torch.from_numpy(n.astype(np.int32)).to(dev)
     sb, cp = torch.from_numpy(seg_base).to(dev), torch.from_numpy(cap).to(dev)
     sc_h, q_h, k_h, v_h = ni.decode_step_inputs(wl.seed, head, B, Hr, Kr, d, g)
+    # the oracle's sample (sequences 0 .. DECODE_CPU_SEQS - 1, every step): their seeded prefix
+    # rows, copied before any decode step appends to the cache
+    cpu_seqs = 0 if args.no_cpu_baseline else min(DECODE_CPU_SEQS, B)
+    cpu_state = None
+    if cpu_seqs:
+        segs = np.arange(cpu_seqs * Hr)
+        o_cap = (n[segs] + steps).astype(np.int32)
+        o_base = np.concatenate([[0], np.cumsum(o_cap)[:-1]]).astype(np.int64)
+        o_kc = np.zeros((int(o_cap.sum()), d))
+        o_vc = np.zeros((int(o_cap.sum()), d))
+        for s_ in segs:
+            lo, m = int(seg_base[s_]), int(n[s_])
+            o_kc[o_base[s_]:o_base[s_] + m] = kc[lo:lo + m].float().cpu().numpy()
+            o_vc[o_base[s_]:o_base[s_] + m] = vc[lo:lo + m].float().cpu().numpy()
+        cpu_state = (o_kc, o_vc, o_base, n[segs].astype(np.int32), o_cap)
     sc = torch.from_numpy(sc_h[:, :, None, :].copy()).to(dev)
     qd = torch.from_numpy(q_h.view(np.int16)).to(dev).view(torch.bfloat16)
     kd = torch.from_numpy(k_h.view(np.int16)).to(dev).view(torch.bfloat16)
@@ -692,13 +825,14 @@ def run_decode(args, dev, pk, pk_kind):
         total_bytes += acc.decode_bytes(after, d, g)
         lens[segs] = after
     assert np.array_equal(lens, seg_len.cpu().numpy()), "decode lengths diverged from the bookkeeping"
-    step_ms = float(times.sum(1).mean())
-    decode_ms = float(times[:, 1].mean())
+    step_ms = float(np.median(times.sum(1)))
+    decode_ms = float(times[:, 1].mean())  # HBM GB/s divides by the kernel's average duration
     bytes_per_step = total_bytes / steps
     gbs = bytes_per_step / (decode_ms * 1e-3) / 1e9
     out = {
         "workload": wl.name if prefix == wl.prefix else f"{wl.name} at prefix {prefix} (profiling size)",
         "steps": steps, "tokens_per_s": B / (step_ms * 1e-3), "ms_per_step": step_ms,
+        "step_ms_stats": stats(times.sum(1)), "decode_ms_stats": stats(times[:, 1]),
         "route_ms": float(times[:, 0].mean()), "decode_ms": decode_ms, "bytes_per_step": bytes_per_step,
         "hbm_gbs": gbs, "frac_measured_hbm": gbs / pk["hbm_gbs"], "frac_nominal_8tbs": gbs / NOMINAL_HBM_GBS,
         "hbm_peak_source": f"{pk_kind} copy bandwidth {pk['hbm_gbs']} GB/s",
@@ -712,7 +846,32 @@ def run_decode(args, dev, pk, pk_kind):
     }
     del kc, vc
     torch.cuda.empty_cache()
+    if cpu_state is not None:
+        out["cpu_baseline"] = oracle_decode_sample(cpu_state, cpu_seqs, sc_h[args.warmup:], q_h[args.warmup:],
+                                                   k_h[args.warmup:], v_h[args.warmup:], wl, steps)
     return out
+
+
+DECODE_CPU_SEQS = 2  # sequences of the decode workload the oracle runs in the CPU baseline
+
+
+def oracle_decode_sample(state, nseq, sc, q, k, v, wl, steps):
+    """The oracle, as it stands, on sequences 0 .. nseq-1 of the decode workload for every step:
+    routing of the new token and the decode step (append at rank, attend, gate)."""
+    import oracle
+    oracle.build()
+    o_kc, o_vc, o_base, o_len, o_cap = state
+    threads = oracle.default_threads()
+    t0 = time.perf_counter()
+    for t in range(steps):
+        r = oracle.route(sc[t][:nseq, None, :], wl.Kr)
+        oracle.decode_step(r["topk_head"][:, 0], r["gate"][:, 0], q[t][:nseq], k[t][:nseq], v[t][:nseq], wl.Hr,
+                           wl.d, wl.g, wl.base, o_kc, o_vc, o_base, o_len, o_cap)
+    sec = time.perf_counter() - t0
+    return {"value": nseq * steps / sec, "unit": "tokens/s", "cores": threads, "kind": "oracle",
+            "sample": f"sequences 0-{nseq - 1} of {wl.B} (their seeded 131072-token prefixes), all {steps} steps, "
+                      f"route + decode step per token, {sec:.1f} s, fp64 C on {threads} host threads ({cpu_model()})",
+            "seconds_per_step": sec / steps}
 
 
 def barrier(world):
@@ -737,12 +896,13 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["namoh", "reference"], default="namoh")
-    ap.add_argument("--decode-steps", type=int, default=64)
+    ap.add_argument("--decode-steps", type=int, default=256)
     ap.add_argument("--decode-prefix", type=int, default=0,
                     help="routed prefix length of the decode section (0: the workload's 131072); smaller only "
                          "for profiler captures")
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-layer", action="store_true")
+    ap.add_argument("--no-configs", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:

@@ -184,7 +184,10 @@ NAMOH_API int namoh_route_varlen(const float *scores, const float *bias, const i
  * leaves its last contents there; every word of it is written before it is
  * read.  Calls that overlap on the GPU -- on
  * different streams, or from different host threads -- race on it and must be
- * serialised by the caller.
+ * serialised by the caller.  The resolved address is kept for the life of the
+ * process: after cudaDeviceReset (or anything else that destroys and recreates
+ * the device's primary context) it is stale, so do not call this entry point on
+ * a device that has been reset since its first call.
  * ------------------------------------------------------------------------- */
 NAMOH_API int namoh_route_noalloc(const float *scores, int B, int T, int H, int K, int32_t *topk_head, float *gate,
                                   int32_t *rank, int32_t *row, int32_t *seg_offsets, int32_t *row_src,

@@ -45,8 +45,9 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved);
 
 int launch_sa_select(const uint16_t* q_rot, const uint16_t* k_cache, const int32_t* seg_offsets,
-                     const int64_t* seg_base, int nseg, int T, long long R, int d, int g, int lg, int alpha_num,
-                     int alpha_den, float* kbar, uint32_t* mask, int words, cudaStream_t stream);
+                     const int64_t* seg_base, const int32_t* seg_cap, long long cache_rows, int nseg, int T,
+                     long long R, int d, int g, int lg, int alpha_num, int alpha_den, float* kbar, uint32_t* mask,
+                     int words, cudaStream_t stream);
 
 namespace attn {
 
@@ -1099,8 +1100,8 @@ extern "C" int namoh_sa_prefill(const uint16_t* q, const uint16_t* k, const uint
     if (const int st2 = cuda_check_launch("seg_len_kernel launch")) return st2;
   }
   const int words = sa_words_for(T, block);
-  rc = launch_sa_select(q_rot, k_cache, seg_offsets, seg_base, nseg, T, R, d_head, group, lg, alpha_num, alpha_den,
-                        kbar, sa_mask, words, stream);
+  rc = launch_sa_select(q_rot, k_cache, seg_offsets, seg_base, seg_base ? seg_cap : nullptr, cache_rows, nseg, T, R,
+                        d_head, group, lg, alpha_num, alpha_den, kbar, sa_mask, words, stream);
   if (rc != NAMOH_OK) return rc;
   return launch_attention(q_rot, k_cache, v_cache, R, d_head, group, seg_offsets, row_src, gate, seg_base, cache_rows,
                           plan, y, dev_status, info, stream, 0, sa_mask, words, lg);

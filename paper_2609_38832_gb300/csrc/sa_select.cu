@@ -29,16 +29,26 @@ __device__ __forceinline__ int blk_base(const int32_t* seg_offsets, int s, int l
   return (seg_offsets[s] >> lg) + s;
 }
 
+// A segment is live when its rows are in the cache: always for the packed layout; with seg_base only
+// when n <= seg_cap (the RoPE pass skips the others' rows and the plan leaves them out).
+__device__ __forceinline__ bool seg_live(const int32_t* seg_offsets, const int64_t* seg_base,
+                                         const int32_t* seg_cap, int s) {
+  return !seg_base || seg_offsets[s + 1] - seg_offsets[s] <= seg_cap[s];
+}
+
 __global__ void __launch_bounds__(256) sa_pool_kernel(const uint16_t* __restrict__ k_cache,
                                                       const int32_t* __restrict__ seg_offsets,
-                                                      const int64_t* __restrict__ seg_base, int d, int lg,
-                                                      float* __restrict__ kbar) {
+                                                      const int64_t* __restrict__ seg_base,
+                                                      const int32_t* __restrict__ seg_cap, long long cache_rows,
+                                                      int d, int lg, float* __restrict__ kbar) {
   const int s = blockIdx.y;
   const int b = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   const int n = seg_offsets[s + 1] - seg_offsets[s];
-  if (b >= (n >> lg)) return;
+  if (b >= (n >> lg) || !seg_live(seg_offsets, seg_base, seg_cap, s)) return;
   const long long row0 = (seg_base ? seg_base[s] : (long long)seg_offsets[s]) + ((long long)b << lg);
+  // rows outside the cache were never written (the RoPE pass reports them): nothing to pool
+  if (row0 < 0 || row0 + (1ll << lg) > cache_rows) return;
   const int per = d / 32;  // columns per lane (2 or 4)
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll 8
@@ -57,6 +67,8 @@ __global__ void __launch_bounds__(256) sa_pool_kernel(const uint16_t* __restrict
 
 __global__ void __launch_bounds__(256) sa_select_kernel(const uint16_t* __restrict__ q_rot,
                                                         const int32_t* __restrict__ seg_offsets, int nseg,
+                                                        const int64_t* __restrict__ seg_base,
+                                                        const int32_t* __restrict__ seg_cap,
                                                         const float* __restrict__ kbar, int d, int g, int lg,
                                                         int alpha_num, int alpha_den, long long nq,
                                                         uint32_t* __restrict__ mask, int words) {
@@ -73,8 +85,11 @@ __global__ void __launch_bounds__(256) sa_select_kernel(const uint16_t* __restri
   }
   const int r = (int)(row - seg_offsets[lo]);  // zero-based local rank
   const int cur = r >> lg;                      // current block = N_B(r + 1) - 1
-  // kept historical blocks: ceil(alpha (cur + 1)) - 1, computed exactly
-  const int keep = (int)(((long long)(cur + 1) * alpha_num + alpha_den - 1) / alpha_den) - 1;
+  // kept historical blocks: ceil(alpha (cur + 1)) - 1, computed exactly; none in a segment that
+  // is not in the cache (its pooled keys were never written and the attention skips it)
+  const int keep = seg_live(seg_offsets, seg_base, seg_cap, lo)
+                       ? (int)(((long long)(cur + 1) * alpha_num + alpha_den - 1) / alpha_den) - 1
+                       : 0;
   const int per = d / 32;  // columns of q~ and of the pooled keys per lane (2 or 4)
   float ql[4];
 #pragma unroll
@@ -154,18 +169,20 @@ __global__ void __launch_bounds__(256) sa_select_kernel(const uint16_t* __restri
 }  // namespace sa
 
 int launch_sa_select(const uint16_t* q_rot, const uint16_t* k_cache, const int32_t* seg_offsets,
-                     const int64_t* seg_base, int nseg, int T, long long R, int d, int g, int lg, int alpha_num,
-                     int alpha_den, float* kbar, uint32_t* mask, int words, cudaStream_t stream) {
+                     const int64_t* seg_base, const int32_t* seg_cap, long long cache_rows, int nseg, int T,
+                     long long R, int d, int g, int lg, int alpha_num, int alpha_den, float* kbar, uint32_t* mask,
+                     int words, cudaStream_t stream) {
   const int max_blocks = (T + (1 << lg) - 1) >> lg;
   if (nseg > 0 && max_blocks > 0) {
     dim3 grid((max_blocks + 7) / 8, nseg);
-    sa::sa_pool_kernel<<<grid, 256, 0, stream>>>(k_cache, seg_offsets, seg_base, d, lg, kbar);
+    sa::sa_pool_kernel<<<grid, 256, 0, stream>>>(k_cache, seg_offsets, seg_base, seg_cap, cache_rows, d, lg, kbar);
     if (const int st = cuda_check_launch("sa_pool_kernel launch")) return st;
   }
   const long long nq = R * g;
   if (nq > 0) {
-    sa::sa_select_kernel<<<(unsigned)((nq + 7) / 8), 256, 0, stream>>>(q_rot, seg_offsets, nseg, kbar, d, g, lg,
-                                                                       alpha_num, alpha_den, nq, mask, words);
+    sa::sa_select_kernel<<<(unsigned)((nq + 7) / 8), 256, 0, stream>>>(q_rot, seg_offsets, nseg, seg_base, seg_cap, kbar,
+                                                                       d, g, lg, alpha_num, alpha_den, nq, mask,
+                                                                       words);
     if (const int st = cuda_check_launch("sa_select_kernel launch")) return st;
   }
   return NAMOH_OK;

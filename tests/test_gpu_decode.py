@@ -44,16 +44,31 @@ def _prefix_state(namoh, B, T, Hr, Kr, d, g, base, headroom, seed, variant="rank
                         seg_len=seg_len, status=ro.status, **_variant(variant))
     torch.cuda.synchronize()
     assert int(ro.status.item()) == 0
-    return dict(kc=kc, vc=vc, seg_len=seg_len, seg_base=seg_base, cap=cap, n=n,
-                seg_base_d=torch.from_numpy(seg_base).cuda(), cap_d=torch.from_numpy(cap).cuda())
+    return dict(kc=kc, vc=vc, seg_len=seg_len, seg_base=seg_base, cap=cap, n=n, rows=rows,
+                seg_base_d=torch.from_numpy(seg_base).cuda(), cap_d=torch.from_numpy(cap).cuda(),
+                host=dict(scores=scores, q=q, k=k, v=v, T=T, Kr=Kr, d=d, g=g, base=base, variant=variant))
 
 
-def _oracle_caches(st, d):
-    """fp64 copies of the GPU caches (the oracle continues from the same stored prefix)."""
-    kc = bf16_to_f64(st["kc"]).copy()
-    vc = bf16_to_f64(st["vc"]).copy()
-    return kc, vc, st["seg_base"].astype(np.int64).copy(), st["seg_len"].cpu().numpy().astype(np.int32).copy(), \
-        st["cap"].astype(np.int32).copy()
+def _oracle_caches(oracle_mod, st):
+    """The oracle's own prefix state: its routing of the prefix, its fp64 rotated keys and the exact
+    values, laid out at the same segment bases (nothing is taken from the GPU's caches)."""
+    h = st["host"]
+    d = h["d"]
+    ref = oracle_mod.route(h["scores"], h["Kr"])
+    vkw = _variant(h["variant"])
+    pos = oracle_mod.global_positions(ref["row_src"], h["T"], h["Kr"]) if vkw["global_positions"] else None
+    _, krot = oracle_mod.prefill(h["q"], h["k"], h["v"], ref["seg_offsets"], ref["row_src"], ref["gate"], d, h["g"],
+                                 h["base"], return_krot=True, interleaved=vkw["interleaved"], pos=pos)
+    seg = ref["seg_offsets"].astype(np.int64)
+    vals = ni.bf16_to_f32(h["v"]).astype(np.float64)
+    kc = np.zeros((st["rows"], d))
+    vc = np.zeros((st["rows"], d))
+    base = st["seg_base"].astype(np.int64).copy()
+    for s_ in range(len(seg) - 1):
+        lo, hi = int(seg[s_]), int(seg[s_ + 1])
+        kc[base[s_]:base[s_] + hi - lo] = krot[lo:hi]
+        vc[base[s_]:base[s_] + hi - lo] = vals[lo:hi]
+    return kc, vc, base, (seg[1:] - seg[:-1]).astype(np.int32), st["cap"].astype(np.int32).copy()
 
 
 @pytest.mark.parametrize("B,T,Hr,Kr,d,g,steps", [
@@ -77,7 +92,7 @@ def _decode_check(namoh, oracle_mod, B, T, Hr, Kr, d, g, steps, variant):
     base = 10000.0
     vkw = _variant(variant)
     st = _prefix_state(namoh, B, T, Hr, Kr, d, g, base, steps, seed=21, variant=variant)
-    okc, ovc, obase, olen, ocap = _oracle_caches(st, d)
+    okc, ovc, obase, olen, ocap = _oracle_caches(oracle_mod, st)
     sc, q, k, v = ni.decode_step_inputs(22, steps, B, Hr, Kr, d, g)
     status = torch.zeros(1, dtype=torch.int32, device="cuda")
     for t in range(steps):
@@ -175,9 +190,11 @@ def test_decode_full_segment_sets_capacity(namoh):
     assert float(y.float().abs().max().item()) == 0.0
 
 
-def test_decode_full_size_sampled(namoh, oracle_mod):
+def test_decode_full_size(namoh, oracle_mod):
     """64 sequences with 131072-token routed prefixes (H = 32, K = 4, d = 128): the 17 GB cache
-    is seeded N(0, 1) bf16 on the device; two decode steps; 8 sequences checked against the oracle."""
+    is seeded N(0, 1) bf16 on the device (already-rotated keys and values); two decode steps.
+    Every sequence and slot of both steps is compared with the oracle, which continues from the
+    seeded prefix rows and from the rows it appended itself (never from rows the GPU wrote)."""
     wl = ni.DECODE
     B, Hr, Kr, d = wl.B, wl.Hr, wl.Kr, wl.d
     s = ni.router_scores(wl.seed, B, wl.prefix, Hr)
@@ -195,17 +212,12 @@ def test_decode_full_size_sampled(namoh, oracle_mod):
     gen.manual_seed(wl.seed)
     kc = torch.randn((rows, d), generator=gen, device="cuda", dtype=torch.bfloat16)
     vc = torch.randn((rows, d), generator=gen, device="cuda", dtype=torch.bfloat16)
+    # the seeded prefix of every segment, as the oracle reads it: rows base .. base + n - 1 are
+    # never rewritten by decode (it appends after them), so they can be copied when first needed
     seg_len = torch.from_numpy(n.astype(np.int32)).cuda()
     sb, cp = torch.from_numpy(seg_base).cuda(), torch.from_numpy(cap).cuda()
     sc, q, k, v = ni.decode_step_inputs(wl.seed, steps, B, Hr, Kr, d)
-    check = list(range(0, B, 8))
-    # oracle copies of the checked sequences' segments
-    o_kc = {}
-    for b in check:
-        for h in range(Hr):
-            sidx = b * Hr + h
-            lo, hi = int(seg_base[sidx]), int(seg_base[sidx] + cap[sidx])
-            o_kc[sidx] = (bf16_to_f64(kc[lo:hi]), bf16_to_f64(vc[lo:hi]))
+    appended = {}  # segment -> (k~ rows, v rows) the oracle appended, fp64
     o_len = n.astype(np.int32).copy()
     status = torch.zeros(1, dtype=torch.int32, device="cuda")
     for t in range(steps):
@@ -214,23 +226,40 @@ def test_decode_full_size_sampled(namoh, oracle_mod):
                                dev_bf16(v[t]), H=Hr, K=Kr, rope_base=wl.base, k_cache=kc, v_cache=vc, seg_base=sb,
                                seg_len=seg_len, seg_cap=cp, status=status)
         torch.cuda.synchronize()
+        ref = oracle_mod.route(sc[t][:, None, :], Kr)
+        np.testing.assert_array_equal(rt.topk_head.view(B, Kr).cpu().numpy(), ref["topk_head"][:, 0])
+        top, gate = ref["topk_head"][:, 0], ref["gate"][:, 0]
         yh = bf16_to_f64(y)
-        top = rt.topk_head.view(B, Kr).cpu().numpy()
-        gate = rt.gate.view(B, Kr).cpu().numpy().astype(np.float64)
-        for b in check:
+        for b in range(B):
+            # this sequence's selected histories as a small cache: segment i = slot i
+            lens, parts_k, parts_v = [], [], []
             for slot in range(Kr):
                 sidx = b * Hr + int(top[b, slot])
-                okc, ovc = o_kc[sidx]
-                one_base = np.zeros(1, np.int64)
-                one_len = o_len[sidx:sidx + 1].copy()
-                one_cap = cap[sidx:sidx + 1].copy()
-                y_ref = oracle_mod.decode_step(np.zeros((1, 1), np.int32), gate[b:b + 1, slot:slot + 1],
-                                               q[t][b:b + 1, slot:slot + 1], k[t][b:b + 1, slot:slot + 1],
-                                               v[t][b:b + 1, slot:slot + 1], 1, d, 1, wl.base, okc, ovc, one_base,
-                                               one_len, one_cap)
-                o_len[sidx] = one_len[0]
-                assert_close_attention(yh[b:b + 1, slot:slot + 1], y_ref, gate[b:b + 1, slot:slot + 1],
-                                       what=f"step {t} seq {b} slot {slot}")
-        np.testing.assert_array_equal(seg_len.cpu().numpy()[[b * Hr + h for b in check for h in range(Hr)]],
-                                      o_len[[b * Hr + h for b in check for h in range(Hr)]])
+                lo = int(seg_base[sidx])
+                pk = bf16_to_f64(kc[lo:lo + int(n[sidx])])
+                pv = bf16_to_f64(vc[lo:lo + int(n[sidx])])
+                ak, av = appended.get(sidx, ([], []))
+                parts_k.append(np.concatenate([pk] + [a[None] for a in ak] + [np.zeros((1, d))]))
+                parts_v.append(np.concatenate([pv] + [a[None] for a in av] + [np.zeros((1, d))]))
+                lens.append(int(n[sidx]) + len(ak))
+                assert lens[-1] == o_len[sidx]
+            okc, ovc = np.ascontiguousarray(np.concatenate(parts_k)), np.ascontiguousarray(np.concatenate(parts_v))
+            caps = np.array([len(p_) for p_ in parts_k], np.int32)
+            bases = np.concatenate([[0], np.cumsum(caps)[:-1]]).astype(np.int64)
+            olen_b = np.array(lens, np.int32)
+            y_ref = oracle_mod.decode_step(np.arange(Kr, dtype=np.int32)[None], gate[b:b + 1], q[t][b:b + 1],
+                                           k[t][b:b + 1], v[t][b:b + 1], Kr, d, 1, wl.base, okc, ovc, bases, olen_b,
+                                           caps)
+            assert_close_attention(yh[b:b + 1], y_ref, gate[b:b + 1], what=f"step {t} seq {b}")
+            for slot in range(Kr):
+                sidx = b * Hr + int(top[b, slot])
+                row = int(bases[slot] + lens[slot])
+                ak, av = appended.setdefault(sidx, ([], []))
+                ak.append(okc[row].copy())
+                av.append(ovc[row].copy())
+                o_len[sidx] += 1
+                # the GPU's appended k~ is the oracle's rounded to bf16
+                got_k = bf16_to_f64(kc[int(seg_base[sidx]) + row - int(bases[slot])])
+                assert np.all(np.abs(got_k - okc[row]) <= np.abs(okc[row]) * 2.0 ** -7 + 1e-6), (t, b, slot)
+        np.testing.assert_array_equal(seg_len.cpu().numpy(), o_len)
     assert int(status.item()) == 0

@@ -167,3 +167,51 @@ def test_sa_rejects_bad_arguments(namoh):
     for kw in (dict(block=48), dict(block=16), dict(alpha_num=0), dict(alpha_num=3, alpha_den=2)):
         with pytest.raises(namoh.NamohError):
             namoh.namoh_sa_prefill(*args, B=wl.B, T=wl.T, H=wl.H, K=wl.K, **kw)
+
+
+def test_sa_segment_over_capacity(namoh, oracle_mod):
+    """Caches at seg_base with one segment one row too small: the status reports it, that segment's
+    rows are neither pooled nor attended, and every other segment matches the oracle."""
+    wl = ni.PrefillWorkload("sa_capacity", B=2, T=600, H=4, K=2, d=128, seed=28)
+    block, num, den = 32, 1, 4
+    scores = wl.scores()
+    q, k, v = wl.qkv()
+    ref = oracle_mod.route(scores, wl.Kr)
+    seg = ref["seg_offsets"].astype(np.int64)
+    nseg = len(seg) - 1
+    n = seg[1:] - seg[:-1]
+    head = 40
+    seg_base = seg[:-1] + np.arange(nseg) * head
+    cap = (n + head).astype(np.int32)
+    over = int(np.argmax(n))
+    cap[over] = n[over] - 1
+    rows = int(seg[-1] + nseg * head)
+    ro = namoh.namoh_route(torch.from_numpy(scores).cuda(), wl.Kr)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    kc = torch.zeros((rows, wl.d), dtype=torch.bfloat16, device="cuda")
+    vc = torch.zeros_like(kc)
+    y, mask, _, _ = namoh.namoh_sa_prefill(dev_bf16(q), dev_bf16(k), dev_bf16(v), ro.seg_offsets, ro.row_src,
+                                           ro.gate, B=wl.B, T=wl.T, H=wl.H, K=wl.K, block=block, alpha_num=num,
+                                           alpha_den=den, rope_base=wl.base, k_cache=kc, v_cache=vc,
+                                           seg_base=torch.from_numpy(seg_base).cuda(),
+                                           seg_cap=torch.from_numpy(cap).cuda(), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & namoh.NAMOH_DEV_CAPACITY
+    mask = mask.cpu().numpy().view(np.uint32)
+    assert not mask[seg[over]:seg[over + 1]].any()  # nothing selected in the skipped history
+    gate = ref["gate"].astype(np.float64)
+    y_ref = oracle_mod.sa_prefill(q, k, v, seg, ref["row_src"], gate, wl.d, 1, wl.base, block, num, den,
+                                  mask_in=mask)
+    keep = np.concatenate([np.arange(seg[s_], seg[s_ + 1]) for s_ in range(nseg) if s_ != over])
+    dst = ref["row_src"][keep]
+    assert_close_attention(bf16_to_f64(y).reshape(-1, wl.d)[dst], y_ref[dst], gate.reshape(-1)[dst])
+    keep_mask = np.concatenate([np.arange(seg[s_], seg[s_ + 1]) for s_ in range(nseg) if s_ != over])
+    _check_counts_rows(mask, seg, keep_mask, block, num, den)
+
+
+def _check_counts_rows(mask, seg, rows, block, num, den):
+    for row in rows:
+        s = int(np.searchsorted(seg, row, side="right") - 1)
+        r = int(row - seg[s])
+        keep = math.ceil(Fraction(num, den) * math.ceil(Fraction(r + 1, block))) - 1
+        assert sum(bin(int(w)).count("1") for w in mask[row]) == keep, row

@@ -46,8 +46,8 @@ def test_shared_prefill_matches_oracle(namoh, oracle_mod, B, Hs, T, d, window):
 @pytest.mark.parametrize("window", [0, 128])
 def test_shared_decode_matches_oracle_and_longer_prefill(namoh, oracle_mod, window):
     """Prefill over T tokens into caches with headroom, then decode steps (every shared head,
-    the same window): each step matches the oracle continuing from the GPU cache, and the GPU
-    prefill over T + steps tokens."""
+    the same window): each step matches the oracle continuing from its own prefix state, and the
+    GPU prefill over T + steps tokens."""
     B, Hs, T, d, steps = 2, 3, 300, 128, 3
     q, k, v = _qkv(61, (B, Hs, T + steps, d))
     nseg = B * Hs
@@ -65,8 +65,17 @@ def test_shared_decode_matches_oracle_and_longer_prefill(namoh, oracle_mod, wind
     torch.cuda.synchronize()
     assert int(status.item()) == 0
     np.testing.assert_array_equal(seg_len.cpu().numpy(), T)
-    okc, ovc = bf16_to_f64(kc).copy(), bf16_to_f64(vc).copy()
-    obase, olen, ocap = seg_base.cpu().numpy().copy(), seg_len.cpu().numpy().copy(), seg_cap.cpu().numpy().copy()
+    # the oracle's own prefix state: keys rotated at t = 0 .. T-1 in fp64, exact values
+    okc, ovc = np.zeros((nseg * cap, d)), np.zeros((nseg * cap, d))
+    import namoh_inputs as ni
+    for b in range(B):
+        for j in range(Hs):
+            lo = (b * Hs + j) * cap
+            okc[lo:lo + T] = oracle_mod.rope(np.ascontiguousarray(k[b, j, :T]), np.arange(T), 1e4)
+            ovc[lo:lo + T] = ni.bf16_to_f32(v[b, j, :T]).astype(np.float64)
+    obase = (np.arange(nseg) * cap).astype(np.int64)
+    olen = np.full(nseg, T, np.int32)
+    ocap = np.full(nseg, cap, np.int32)
     yf = bf16_to_f64(y_full)
     for st in range(steps):
         t = T + st
