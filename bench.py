@@ -689,7 +689,7 @@ def run_sa(args, dev, pk, pk_kind):
         "dense": lambda: namoh.namoh_prefill(q, k, v, ro.seg_offsets, ro.row_src, ro.gate, y=y, k_cache=k_cache,
                                              workspace=ws_dense, status=ro.status, **kw),
     }
-    ms = {}
+    ms, ms_stats = {}, {}
     for name, run in calls.items():
         evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
         for i in range(args.warmup + args.steps):
@@ -701,6 +701,7 @@ def run_sa(args, dev, pk, pk_kind):
                 evs[i - args.warmup][1].record()
         torch.cuda.synchronize()
         ms[name] = float(np.mean([a.elapsed_time(b) for a, b in evs]))
+        ms_stats[name] = stats([a.elapsed_time(b) for a, b in evs])
     n = np.diff(ro.seg_offsets.cpu().numpy()).astype(np.int64)
     pairs_sa = 0
     for ni_ in n:
@@ -709,10 +710,26 @@ def run_sa(args, dev, pk, pk_kind):
         kept = (nb * num + den - 1) // den
         pairs_sa += int(np.sum(r - block * (nb - kept)))  # a_{alpha,B}(r), Eq. app-selected-entries
     pairs_dense = int(np.sum(n * (n + 1) // 2))
+    # key tiles of 128 that some query of a 128-row tile keeps (a kept block, or its own block): the
+    # fraction of the causal tiles a tile-skipping kernel could leave out is 1 minus this
+    m = mask.cpu().numpy().view(np.uint32)
+    seg = ro.seg_offsets.cpu().numpy().astype(np.int64)
+    need, total = 0, 0
+    for s_ in range(len(seg) - 1):
+        nn = int(seg[s_ + 1] - seg[s_])
+        for qt in range((nn + 127) // 128):
+            rows = np.arange(qt * 128, min(nn, qt * 128 + 128))
+            words = np.bitwise_or.reduce(m[seg[s_] + rows], axis=0)
+            bits = np.unpackbits(words.view(np.uint8), bitorder="little")
+            for kv in range(qt):  # the diagonal tile is always needed
+                total += 1
+                need += int(bits[kv * 128 // block:(kv + 1) * 128 // block].any())
+    tiles_needed = need / total if total else 1.0
     flops_sa = 4.0 * wl.d * wl.g * pairs_sa
     tf = flops_sa / (ms["sa"] * 1e-3) / 1e12
     return {"workload": f"{wl.name}, blocks of {block}, alpha {num}/{den}", "ms": ms["sa"],
             "dense_prefill_ms": ms["dense"], "sa_pairs_over_dense": pairs_sa / pairs_dense,
+            "off_diagonal_key_tiles_needed": tiles_needed, "ms_stats": ms_stats,
             "tflops_attended": tf, "frac_bf16": tf / pk["bf16_tflops"], "flops_attended": flops_sa,
             "peak_source": f"{pk_kind} bf16 dense (burst)", "device_status": int(ro.status.item()),
             # per timed pair: SA (RoPE + plan, pooling, selection, attention) and dense (RoPE + plan, attention)
@@ -903,6 +920,8 @@ def main():
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-layer", action="store_true")
     ap.add_argument("--no-configs", action="store_true")
+    ap.add_argument("--only", choices=["configs", "decode", "layer", "shared", "sa"], default=None,
+                    help="run one section alone and print it (small profiler captures); not a bench line")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
@@ -934,6 +953,16 @@ def main():
         }))
         return
 
+    if args.only:
+        import torch
+        dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+        torch.cuda.set_device(dev)
+        pk, pk_kind = peaks()
+        fn = {"configs": run_configs, "decode": run_decode, "layer": run_layer, "shared": run_shared,
+              "sa": run_sa}[args.only]
+        if rank == 0:
+            print(json.dumps({"section": args.only, args.only: fn(args, dev, pk, pk_kind)}))
+        return
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl")

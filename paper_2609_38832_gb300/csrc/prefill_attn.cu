@@ -44,10 +44,11 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              void* plan, int plan_qtiles, const int32_t* plan_cap, const int32_t* pos_row_src,
                              int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved);
 
-int launch_sa_select(const uint16_t* q_rot, const uint16_t* k_cache, const int32_t* seg_offsets,
-                     const int64_t* seg_base, const int32_t* seg_cap, long long cache_rows, int nseg, int T,
-                     long long R, int d, int g, int lg, int alpha_num, int alpha_den, float* kbar, uint32_t* mask,
-                     int words, cudaStream_t stream);
+int launch_sa_select(const CUtensorMap& q_rot_map, const uint16_t* q_rot, const uint16_t* k_cache,
+                     const int32_t* seg_offsets, const int64_t* seg_base, const int32_t* seg_cap,
+                     long long cache_rows, int nseg, int T, long long R, int d, int g, int lg, int alpha_num,
+                     int alpha_den, uint16_t* kbar, long long kbar_rows, uint32_t* mask, int words, const void* plan,
+                     int max_items, uint32_t* status, cudaStream_t stream);
 
 namespace attn {
 
@@ -1037,7 +1038,7 @@ size_t sa_workspace_rows(long long R, int nseg, int d_head, int group, int block
   WorkspaceCarver ws{nullptr, 0, 0};
   ws.take<uint16_t>((size_t)R * group * d_head);
   ws.take<char>(plan_bytes_rows(R, nseg, group));
-  ws.take<float>((size_t)(R / block + nseg) * d_head);
+  ws.take<uint16_t>((size_t)(R / block + nseg) * d_head);
   return align_up(ws.used, 256);
 }
 }  // namespace
@@ -1086,7 +1087,8 @@ extern "C" int namoh_sa_prefill(const uint16_t* q, const uint16_t* k, const uint
   WorkspaceCarver ws{static_cast<char*>(workspace), workspace_bytes, 0};
   uint16_t* q_rot = ws.take<uint16_t>((size_t)R * group * d_head);
   void* plan = ws.take<char>(plan_bytes_rows(R, nseg, group));
-  float* kbar = ws.take<float>((size_t)(R / block + nseg) * d_head);
+  const long long kbar_rows = R / block + nseg;
+  uint16_t* kbar = ws.take<uint16_t>((size_t)kbar_rows * d_head);
   if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
   DeviceInfo info;
   if (!device_ok(&info)) return NAMOH_ERR_UNSUPPORTED;
@@ -1100,8 +1102,12 @@ extern "C" int namoh_sa_prefill(const uint16_t* q, const uint16_t* k, const uint
     if (const int st2 = cuda_check_launch("seg_len_kernel launch")) return st2;
   }
   const int words = sa_words_for(T, block);
-  rc = launch_sa_select(q_rot, k_cache, seg_offsets, seg_base, seg_base ? seg_cap : nullptr, cache_rows, nseg, T, R,
-                        d_head, group, lg, alpha_num, alpha_den, kbar, sa_mask, words, stream);
+  CUtensorMap tq;
+  if (!attn::encode_rows_map(&tq, q_rot, R, group * d_head)) return cuda_fail(cudaErrorInvalidValue, "cuTensorMapEncodeTiled");
+  const long long max_items = ((R + attn::kItemRows - 1) / attn::kItemRows + nseg) * group;
+  rc = launch_sa_select(tq, q_rot, k_cache, seg_offsets, seg_base, seg_base ? seg_cap : nullptr, cache_rows, nseg, T,
+                        R, d_head, group, lg, alpha_num, alpha_den, kbar, kbar_rows, sa_mask, words, plan,
+                        (int)max_items, dev_status, stream);
   if (rc != NAMOH_OK) return rc;
   return launch_attention(q_rot, k_cache, v_cache, R, d_head, group, seg_offsets, row_src, gate, seg_base, cache_rows,
                           plan, y, dev_status, info, stream, 0, sa_mask, words, lg);

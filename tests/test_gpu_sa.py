@@ -215,3 +215,27 @@ def _check_counts_rows(mask, seg, rows, block, num, den):
         r = int(row - seg[s])
         keep = math.ceil(Fraction(num, den) * math.ceil(Fraction(r + 1, block))) - 1
         assert sum(bin(int(w)).count("1") for w in mask[row]) == keep, row
+
+
+@pytest.mark.parametrize("num,den", [(1, 2), (3, 4)], ids=["alpha_1_2", "alpha_3_4"])
+def test_sa_long_histories_many_kept(namoh, oracle_mod, num, den):
+    """Histories of about 2048 rows (64 blocks of 32): a query keeps up to 31 blocks (alpha 1/2), or
+    drops up to 16 (alpha 3/4), more than the selector's 8-entry register list, so the kept set is
+    found by bisection over the selection keys."""
+    wl = ni.PrefillWorkload("sa_long", B=1, T=4096, H=2, K=1, d=128, seed=29)
+    _, qkv, ro, y, mask, _ = _run(namoh, wl, 32, num, den)
+    seg = _check_y(oracle_mod, wl, qkv, ro, y, mask, 32, num, den)
+    _check_counts(mask, seg, wl.g, 32, num, den)
+    rows = sample_rows(seg, 200, seed=5)
+    assert _check_scores(oracle_mod, wl, qkv[0], qkv[1], seg, mask, 32, rows) > 100
+
+
+def test_sa_history_longer_than_the_tmem_scores(namoh, oracle_mod):
+    """One history of 17000 rows (532 blocks of 32): rows whose current block is past the 512 block
+    scores one selection CTA holds in TMEM take the per-query selector; both meet at block 512."""
+    wl = ni.PrefillWorkload("sa_very_long", B=1, T=17000, H=1, K=1, d=64, seed=30)
+    _, qkv, ro, y, mask, _ = _run(namoh, wl, 32, 1, 5)
+    seg = _check_y(oracle_mod, wl, qkv, ro, y, mask, 32, 1, 5)
+    _check_counts(mask, seg, wl.g, 32, 1, 5)
+    rows = np.concatenate([sample_rows(seg, 100, seed=6), np.arange(512 * 32 - 40, 513 * 32 + 40)])
+    assert _check_scores(oracle_mod, wl, qkv[0], qkv[1], seg, np.asarray(mask), 32, np.unique(rows)) > 100
