@@ -29,6 +29,12 @@
 //               accumulators overlap, so with three S/P buffers the issuer interleaves
 //               PV(kv) (A = P in TMEM, B = V as the MN-major operand) with S(kv+2) = Q K^T
 //               instruction by instruction while the softmax works on S(kv+1).
+//   warps 6-7   (kRopeQ instantiations only) query rotation: the producer loads the raw query
+//               tile, and thread i rotates rows i and i + 64 in shared memory at their ranks (Sec. 3.2, Eq.
+//               namoh-head-rope) from a cos / sin table the RoPE pass wrote, with the RoPE
+//               pass's own arithmetic, so the rotated tile is bit for bit the one that pass
+//               would have written to HBM.  The next item's tile lands and is rotated while
+//               the current item's last steps run, so the MMA issuer rarely waits for it.
 // TMEM: S/P buffers at cols [0,128), [128,256), [256,384); O at [384, 384 + D).
 // Shared memory (d = 128): Q 32 KB + 6 x 32 KB ring = 224 KB.
 // Every mbarrier wait is bounded (NAMOH_DEV_TIMEOUT, then all roles drain and exit).
@@ -42,7 +48,8 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache, bool copy_v,
                              const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream,
                              void* plan, int plan_qtiles, const int32_t* plan_cap, const int32_t* pos_row_src,
-                             int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved);
+                             int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved,
+                             float2* cs_tab, int cs_rows);
 
 int launch_sa_select(const CUtensorMap& q_rot_map, const uint16_t* q_rot, const uint16_t* k_cache,
                      const int32_t* seg_offsets, const int64_t* seg_base, const int32_t* seg_cap,
@@ -59,7 +66,11 @@ static_assert(kItemRows == kPlanTileRows, "the plan and the kernel must agree on
 constexpr int kSoftmaxWarps = 4;     // warps 0-3: thread i owns query row i (TMEM lane i)
 constexpr int kWarpLoad = 4;
 constexpr int kWarpMma = 5;
+constexpr int kWarpRope0 = 6;        // warps 6-7: query rotation (kRopeQ instantiations)
+constexpr int kRopeWarps = 2;        // (two rows per thread: the block stays within 256 registers a thread)
 constexpr int kThreads = 192;
+// kRopeQ: 0 = the queries come rotated; 1 = rotate them here, half-split pairs; 2 = interleaved pairs
+__host__ __device__ constexpr int threads_for(int rope_q) { return rope_q ? kThreads + 32 * kRopeWarps : kThreads; }
 constexpr int kTmemCols = 512;
 constexpr int kSBufs = 3;            // S/P buffers in TMEM
 // TMEM columns: S/P buffers at 0, 128, 256; O at 384.  P (bf16, two per 32-bit column)
@@ -96,6 +107,7 @@ struct Bars {
                         // do not need and still wait on an exact phase.
   uint64_t o_free;      // epilogue finished reading O
   uint64_t drain;
+  uint64_t q_ready;     // (kRopeQ) the query tile is rotated in shared memory
   int4 item_slot[2];    // {segment * g + j, query tile, seg_offsets[segment], n}
   uint32_t tmem_base;
   int abort_flag;
@@ -123,6 +135,9 @@ struct Params {
   const uint32_t* sa_mask;
   int sa_words;
   int sa_lg;
+  // kRopeQ: cos / sin of rank p and pair j at cs_tab[p * D / 2 + j] (cs_rows ranks)
+  const float2* cs_tab;
+  int cs_rows;
 };
 
 // All lanes of a warp wait and agree on the outcome, so warp-collective tcgen05
@@ -273,10 +288,74 @@ __device__ __forceinline__ bool softmax_tile(uint32_t s_addr, uint32_t o_addr, i
   return true;
 }
 
-template <int D, bool kSA>
-__global__ void __launch_bounds__(kThreads, 1)
+// Rotates query row `row` of the 128B-swizzled tile at q_smem in place (rank RoPE, Sec. 3.2 Eq.
+// namoh-head-rope) with cos / sin from the table row of its rank.  Element e of a row sits in
+// 64-column atom e / 64, 16-byte chunk (e % 64) / 8, stored at chunk position chunk ^ (row % 8).
+// x'_j = x_j cos - x_{j+D/2} sin, x'_{j+D/2} = x_{j+D/2} cos + x_j sin (interleaved: the pair
+// (2j, 2j+1) in one bf16x2 word), each product and rounding as the RoPE pass does them.
+template <int D, int kRopeQ>
+__device__ __forceinline__ void rotate_query_row(uint8_t* q_smem, int row, const float2* __restrict__ cs) {
+  constexpr int kAtomBytes = BM * 128;
+  const int sw = row & 7;
+  auto chunk_ptr = [&](int e) -> uint4* {  // the 16-byte chunk holding element e (a multiple of 8)
+    return reinterpret_cast<uint4*>(q_smem + (e >> 6) * kAtomBytes + row * 128 + ((((e & 63) >> 3) ^ sw) << 4));
+  };
+  const float4* tb = reinterpret_cast<const float4*>(cs);  // {cos_j, sin_j, cos_j+1, sin_j+1}
+  if constexpr (kRopeQ == 1) {
+    constexpr int HALF = D / 2;
+#pragma unroll
+    for (int c = 0; c < HALF / 8; ++c) {
+      float cs8[8], sn8[8];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float4 t = __ldg(tb + 4 * c + i);
+        cs8[2 * i] = t.x;
+        sn8[2 * i] = t.y;
+        cs8[2 * i + 1] = t.z;
+        sn8[2 * i + 1] = t.w;
+      }
+      uint4* pa = chunk_ptr(8 * c);
+      uint4* pb = chunk_ptr(HALF + 8 * c);
+      const uint4 a = *pa, b = *pb;
+      const uint32_t av[4] = {a.x, a.y, a.z, a.w};
+      const uint32_t bv[4] = {b.x, b.y, b.z, b.w};
+      uint32_t oa[4], ob[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float x0 = bf16_lo(av[q]), x1 = bf16_hi(av[q]);
+        const float y0 = bf16_lo(bv[q]), y1 = bf16_hi(bv[q]);
+        const int i0 = 2 * q, i1 = 2 * q + 1;
+        oa[q] = pack_bf16x2(fmaf(x0, cs8[i0], -y0 * sn8[i0]), fmaf(x1, cs8[i1], -y1 * sn8[i1]));
+        ob[q] = pack_bf16x2(fmaf(y0, cs8[i0], x0 * sn8[i0]), fmaf(y1, cs8[i1], x1 * sn8[i1]));
+      }
+      *pa = make_uint4(oa[0], oa[1], oa[2], oa[3]);
+      *pb = make_uint4(ob[0], ob[1], ob[2], ob[3]);
+    }
+  } else {
+#pragma unroll
+    for (int c = 0; c < D / 8; ++c) {  // chunk c holds pairs j = 4c .. 4c + 3
+      const float4 t0 = __ldg(tb + 2 * c), t1 = __ldg(tb + 2 * c + 1);
+      const float cs4[4] = {t0.x, t0.z, t1.x, t1.z};
+      const float sn4[4] = {t0.y, t0.w, t1.y, t1.w};
+      uint4* pa = chunk_ptr(8 * c);
+      const uint4 a = *pa;
+      const uint32_t w[4] = {a.x, a.y, a.z, a.w};
+      uint32_t o[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float x0 = bf16_lo(w[q]), x1 = bf16_hi(w[q]);
+        o[q] = pack_bf16x2(fmaf(x0, cs4[q], -x1 * sn4[q]), fmaf(x1, cs4[q], x0 * sn4[q]));
+      }
+      *pa = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+  }
+}
+
+template <int D, bool kSA, int kRopeQ>
+__global__ void __launch_bounds__(threads_for(kRopeQ), 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                     const __grid_constant__ CUtensorMap tm_v, Params p) {
+  static_assert(!(kSA && kRopeQ), "SA + NAMOH selects on rotated queries the RoPE pass wrote");
   using L = Smem<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -290,8 +369,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     for (int i = 0; i < 2; ++i) {
       mbar_init(&bars->item_full[i], 1);
-      mbar_init(&bars->item_empty[i], 1 + kSoftmaxWarps);
+      mbar_init(&bars->item_empty[i], 1 + kSoftmaxWarps + (kRopeQ ? kRopeWarps : 0));
     }
+    mbar_init(&bars->q_ready, kRopeWarps);
     for (int i = 0; i < kRing; ++i) {
       mbar_init(&bars->ring_full[i], 1);
       mbar_init(&bars->ring_empty[i], 1);
@@ -439,8 +519,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto rk = [&](int kv) -> uint32_t { return base + 2u * (kv - 2) + 1u; };  // K(kv), kv >= 2
 
       // prologue: S(0) and S(1) interleaved (independent buffers), then PV(0)'s operands
-      ok = warp_wait(&bars->q_full, item_iter & 1, abort_flag, p.status) && ring_ready(rk0) &&
-           (nkv == 1 || ring_ready(rk1));
+      ok = warp_wait(kRopeQ ? &bars->q_ready : &bars->q_full, item_iter & 1, abort_flag, p.status) &&
+           ring_ready(rk0) && (nkv == 1 || ring_ready(rk1));
       if (!ok) break;
       tc_fence_after();
       {
@@ -544,7 +624,27 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     __syncwarp();
-  } else {
+  } else if (kRopeQ && warp >= kWarpRope0) {
+    // ------------------------------------------------------------------ query rotation
+    const int row = (warp - kWarpRope0) * 32 + lane;  // rows `row` and `row` + 64 of the tile
+    uint32_t item_iter = 0;
+    bool ok = true;
+    while (ok) {
+      int4 item;
+      ok = take_item(bars, item_iter, &item, abort_flag, p.status);
+      if (!ok || item.x < 0) break;
+      // ranks of the two rows (past the segment's end: rotated but never used)
+      const int pos0 = min(item.y * BM + row, p.cs_rows - 1), pos1 = min(item.y * BM + row + 64, p.cs_rows - 1);
+      ok = warp_wait(&bars->q_full, item_iter & 1, abort_flag, p.status);
+      if (!ok) break;
+      rotate_query_row<D, kRopeQ>(smem + L::kQ, row, p.cs_tab + (size_t)pos0 * (D / 2));
+      rotate_query_row<D, kRopeQ>(smem + L::kQ, row + 64, p.cs_tab + (size_t)pos1 * (D / 2));
+      fence_proxy_async_smem();  // the MMA reads the tile through the async proxy
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars->q_ready);
+      ++item_iter;
+    }
+  } else if (warp < kSoftmaxWarps) {
     // ------------------------------------------------------------------ softmax / epilogue
     const int row = warp * 32 + lane;  // query row within the tile (warp w reads TMEM lanes 32w..32w+31)
     const uint32_t lane_addr = (uint32_t)(warp * 32) << 16;
@@ -675,13 +775,14 @@ bool encode_rows_map(CUtensorMap* map, const void* base, long long rows, int row
   return r == CUDA_SUCCESS;
 }
 
-template <int D, bool kSA>
+template <int D, bool kSA, int kRopeQ>
 cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv, const Params& p,
                         int grid, cudaStream_t stream) {
   const int smem = Smem<D>::kAlloc;
-  cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D, kSA>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  const auto kernel = attn_fwd_kernel<D, kSA, kRopeQ>;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  e = launch_pdl(attn_fwd_kernel<D, kSA>, dim3(grid), dim3(kThreads), (size_t)smem, stream, tq, tk, tv, p);
+  e = launch_pdl(kernel, dim3(grid), dim3(threads_for(kRopeQ)), (size_t)smem, stream, tq, tk, tv, p);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
@@ -729,6 +830,8 @@ size_t plan_bytes_rows(long long R, int nseg, int g) {
 size_t plan_bytes_for(int B, int T, int Hr, int Kr, int g) { return plan_bytes_rows((long long)B * T * Kr, B * Hr, g); }
 
 int plan_qtiles_for(int T) { return (T + kPlanTileRows - 1) / kPlanTileRows; }  // query tiles per segment, at most
+// ranks the query-rotation table covers: every row of every query tile of a history of at most T
+int cs_rows_for(int T) { return plan_qtiles_for(T) * kPlanTileRows; }
 
 // The RoPE launch builds the plan in one extra block when the plan's shared memory is small
 // enough not to cut the RoPE blocks' occupancy.
@@ -753,11 +856,14 @@ int launch_plan(const int32_t* seg_offsets, int nseg, int T, int g, const int32_
 // the plan's shared memory is small, else as a second kernel).
 // rope_flags: NAMOH_ROPE_GLOBAL takes the positions from row_src: t = (row_src[r] / Kr) % T,
 // or row_src[r] / Kr - cu_seqlens[b] in a ragged batch (T is then the longest sequence).
+// With cs_tab the queries are not rotated here: the pass writes the cos / sin table of ranks
+// 0 .. cs_rows - 1 instead, and the attention kernel rotates the queries (rank positions only).
 int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int Hr, int Kr, int R,
                          int d_head, int group, float rope_base, unsigned rope_flags, const int32_t* cu_seqlens,
                          const int32_t* seg_offsets, const int32_t* row_src, uint16_t* q_rot, uint16_t* k_cache,
                          uint16_t* v_cache, const int64_t* seg_base, const int32_t* seg_cap, long long cache_rows,
-                         uint32_t* dev_status, void* plan, const DeviceInfo& info, cudaStream_t stream) {
+                         uint32_t* dev_status, void* plan, const DeviceInfo& info, cudaStream_t stream,
+                         float2* cs_tab = nullptr, int cs_rows = 0) {
   RopeTable tab;
   fill_rope_table(&tab, d_head, (double)rope_base);
   const int nseg = B * Hr;
@@ -768,7 +874,7 @@ int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v
                                          q_rot, k_cache, v_cache, v_cache != v, tab, dev_status, info.sm_count, stream,
                                          fuse_plan ? plan : nullptr, qtiles, plan_cap,
                                          (rope_flags & NAMOH_ROPE_GLOBAL) ? row_src : nullptr, Kr, T, cu_seqlens,
-                                         Hr, (rope_flags & NAMOH_ROPE_INTERLEAVED) != 0);
+                                         Hr, (rope_flags & NAMOH_ROPE_INTERLEAVED) != 0, cs_tab, cs_rows);
   if (e != cudaSuccess) return cuda_fail(e, "rope_pack_kernel launch");
   if (plan && !fuse_plan) return launch_plan(seg_offsets, nseg, T, group, plan_cap, plan, stream);
   return NAMOH_OK;
@@ -778,7 +884,9 @@ int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint1
                      int g, const int32_t* seg_offsets, const int32_t* row_src, const float* gate,
                      const int64_t* seg_base, long long cache_rows, void* plan, uint16_t* y, uint32_t* dev_status,
                      const DeviceInfo& info, cudaStream_t stream, int window = 0,
-                     const uint32_t* sa_mask = nullptr, int sa_words = 0, int sa_lg = 0) {
+                     const uint32_t* sa_mask = nullptr, int sa_words = 0, int sa_lg = 0, int rope_q = 0,
+                     const float2* cs_tab = nullptr, int cs_rows = 0) {
+  // rope_q > 0: q_rot holds the raw queries, rotated in the kernel (1 half-split, 2 interleaved)
   CUtensorMap tq, tk, tv;
   if (!attn::encode_rows_map(&tq, q_rot, R, g * D) || !attn::encode_rows_map(&tk, k_cache, cache_rows, D) ||
       !attn::encode_rows_map(&tv, v_cache, cache_rows, D))
@@ -801,13 +909,22 @@ int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint1
   p.sa_mask = sa_mask;
   p.sa_words = sa_words;
   p.sa_lg = sa_lg;
+  p.cs_tab = cs_tab;
+  p.cs_rows = cs_rows;
   cudaError_t e;
+  const int G = info.sm_count;
   if (sa_mask)
-    e = (D == 128) ? attn::launch_attn<128, true>(tq, tk, tv, p, info.sm_count, stream)
-                   : attn::launch_attn<64, true>(tq, tk, tv, p, info.sm_count, stream);
+    e = (D == 128) ? attn::launch_attn<128, true, 0>(tq, tk, tv, p, G, stream)
+                   : attn::launch_attn<64, true, 0>(tq, tk, tv, p, G, stream);
+  else if (rope_q == 1)
+    e = (D == 128) ? attn::launch_attn<128, false, 1>(tq, tk, tv, p, G, stream)
+                   : attn::launch_attn<64, false, 1>(tq, tk, tv, p, G, stream);
+  else if (rope_q == 2)
+    e = (D == 128) ? attn::launch_attn<128, false, 2>(tq, tk, tv, p, G, stream)
+                   : attn::launch_attn<64, false, 2>(tq, tk, tv, p, G, stream);
   else
-    e = (D == 128) ? attn::launch_attn<128, false>(tq, tk, tv, p, info.sm_count, stream)
-                   : attn::launch_attn<64, false>(tq, tk, tv, p, info.sm_count, stream);
+    e = (D == 128) ? attn::launch_attn<128, false, 0>(tq, tk, tv, p, G, stream)
+                   : attn::launch_attn<64, false, 0>(tq, tk, tv, p, G, stream);
   return e == cudaSuccess ? NAMOH_OK : cuda_fail(e, "attn_fwd_kernel launch");
 }
 
@@ -929,27 +1046,32 @@ int prefill_impl(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B,
   WorkspaceCarver ws{static_cast<char*>(workspace), workspace_bytes, 0};
   uint16_t* q_rot = ws.take<uint16_t>((size_t)R * group * d_head);
   void* plan = ws.take<char>(plan_bytes_rows(R, B * Hr, group));
+  const int cs_rows = cs_rows_for(T);
+  float2* cs_tab = ws.take<float2>((size_t)cs_rows * (d_head / 2));
   if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
   DeviceInfo info;
   if (!device_ok(&info)) return NAMOH_ERR_UNSUPPORTED;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
-
+  // rank positions: the attention kernel rotates the queries itself (no Q~ round trip through HBM)
+  const bool fuse_q = !(rope_flags & NAMOH_ROPE_GLOBAL);
   int st = launch_rope_and_plan(q, k, v, B, T, Hr, Kr, (int)R, d_head, group, rope_base, rope_flags, cu_seqlens,
                                 seg_offsets, row_src, q_rot, k_cache, v_cache, seg_base, seg_cap, cache_rows,
-                                dev_status, plan, info, stream);
+                                dev_status, plan, info, stream, fuse_q ? cs_tab : nullptr, cs_rows);
   if (st != NAMOH_OK) return st;
   if (seg_len) {
     seg_len_kernel<<<(B * Hr + 255) / 256, 256, 0, stream>>>(seg_offsets, B * Hr, seg_len);
     if (const int st2 = cuda_check_launch("seg_len_kernel launch")) return st2;
   }
-  return launch_attention(q_rot, k_cache, v_cache, R, d_head, group, seg_offsets, row_src, gate, seg_base, cache_rows,
-                          plan, y, dev_status, info, stream);
+  const int rope_q = fuse_q ? ((rope_flags & NAMOH_ROPE_INTERLEAVED) ? 2 : 1) : 0;
+  return launch_attention(fuse_q ? q : q_rot, k_cache, v_cache, R, d_head, group, seg_offsets, row_src, gate, seg_base,
+                          cache_rows, plan, y, dev_status, info, stream, 0, nullptr, 0, 0, rope_q, cs_tab, cs_rows);
 }
 
-size_t prefill_workspace_rows(long long R, int nseg, int d_head, int group) {
+size_t prefill_workspace_rows(long long R, int nseg, int T, int d_head, int group) {
   WorkspaceCarver ws{nullptr, 0, 0};
   ws.take<uint16_t>((size_t)R * group * d_head);
   ws.take<char>(plan_bytes_rows(R, nseg, group));
+  ws.take<float2>((size_t)cs_rows_for(T) * (d_head / 2));
   return align_up(ws.used, 256);
 }
 
@@ -966,7 +1088,7 @@ extern "C" size_t namoh_prefill_workspace_size(int B, int T, int H, int K, int d
   int Hr, Kr;
   long long R;
   if (check_shape(B, T, H, K, d_head, group, &Hr, &Kr, &R) != NAMOH_OK) return 0;
-  return prefill_workspace_rows(R, B * Hr, d_head, group);
+  return prefill_workspace_rows(R, B * Hr, T, d_head, group);
 }
 
 extern "C" int namoh_prefill_ex(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int H, int K,
@@ -989,7 +1111,7 @@ extern "C" size_t namoh_prefill_varlen_workspace_size(int B, int total_tokens, i
   int Hr, Kr;
   long long R;
   if (check_varlen(B, total_tokens, max_seqlen, H, K, d_head, group, &Hr, &Kr, &R) != NAMOH_OK) return 0;
-  return prefill_workspace_rows(R, B * Hr, d_head, group);
+  return prefill_workspace_rows(R, B * Hr, max_seqlen, d_head, group);
 }
 
 extern "C" int namoh_prefill_varlen(const uint16_t* q, const uint16_t* k, const uint16_t* v,
@@ -1136,16 +1258,16 @@ __global__ void shared_layout_kernel(int B, int T, int Hs, int32_t* __restrict__
 struct SharedWs {
   int32_t *seg_offsets, *row_src;
   float* gate;
-  uint16_t* q_rot;
   void* plan;
+  float2* cs_tab;  // the attention kernel rotates the queries (the rank in these segments is t)
 };
 void carve_shared(WorkspaceCarver& ws, SharedWs* o, int B, int T, int Hs, int d_head) {
   const long long R = (long long)B * Hs * T;
   o->seg_offsets = ws.take<int32_t>((size_t)B * Hs + 1);
   o->row_src = ws.take<int32_t>((size_t)R);
   o->gate = ws.take<float>((size_t)R);
-  o->q_rot = ws.take<uint16_t>((size_t)R * d_head);
   o->plan = ws.take<char>(plan_bytes_rows(R, B * Hs, 1));
+  o->cs_tab = ws.take<float2>((size_t)cs_rows_for(T) * (d_head / 2));
 }
 }  // namespace
 }  // namespace namoh
@@ -1191,14 +1313,16 @@ extern "C" int namoh_shared_prefill(const uint16_t* q, const uint16_t* k, const 
   shared_layout_kernel<<<info.sm_count * 4, 256, 0, stream>>>(B, T, Hs, o.seg_offsets, o.row_src, o.gate);
   if (const int e = cuda_check_launch("shared_layout_kernel launch")) return e;
   // global positions: the rank in a segment holding every token is t (the global flag is redundant)
-  st = launch_rope_and_plan(q, k, v, B, T, Hs, Hs, (int)R, d_head, 1, rope_base, rope_flags & NAMOH_ROPE_INTERLEAVED,
-                            nullptr, o.seg_offsets, o.row_src, o.q_rot, k_cache, v_cache, seg_base, seg_cap,
-                            cache_rows, dev_status, o.plan, info, stream);
+  const bool il = (rope_flags & NAMOH_ROPE_INTERLEAVED) != 0;
+  st = launch_rope_and_plan(q, k, v, B, T, Hs, Hs, (int)R, d_head, 1, rope_base, il ? NAMOH_ROPE_INTERLEAVED : 0u,
+                            nullptr, o.seg_offsets, o.row_src, nullptr, k_cache, v_cache, seg_base, seg_cap,
+                            cache_rows, dev_status, o.plan, info, stream, o.cs_tab, cs_rows_for(T));
   if (st != NAMOH_OK) return st;
   if (seg_len) {
     seg_len_kernel<<<(B * Hs + 255) / 256, 256, 0, stream>>>(o.seg_offsets, B * Hs, seg_len);
     if (const int e = cuda_check_launch("seg_len_kernel launch")) return e;
   }
-  return launch_attention(o.q_rot, k_cache, v_cache, R, d_head, 1, o.seg_offsets, o.row_src, o.gate, seg_base,
-                          cache_rows, o.plan, y, dev_status, info, stream, window);
+  return launch_attention(q, k_cache, v_cache, R, d_head, 1, o.seg_offsets, o.row_src, o.gate, seg_base,
+                          cache_rows, o.plan, y, dev_status, info, stream, window, nullptr, 0, 0, il ? 2 : 1, o.cs_tab,
+                          cs_rows_for(T));
 }

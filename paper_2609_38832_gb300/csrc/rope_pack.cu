@@ -34,14 +34,15 @@ constexpr size_t kSmemPerSm = 233472;  // shared memory per SM (228 KB); each re
 // the least dynamic shared memory with which three blocks no longer fit on one SM
 constexpr size_t kSmemThirdPlus = kSmemPerSm / 3 - 1024 + 16;
 
-template <int D, int G>
+// kNoQ: only K (and V) pass through; the queries are rotated by the attention kernel itself.
+template <int D, int G, bool kNoQ = false>
 struct RopeChunk {
   static constexpr int kLpr = D / 16;                    // threads per group (8 pairs each)
   static constexpr int kGroups = kRopeThreads / kLpr;    // 32 (D = 128) or 64 (D = 64)
   static constexpr int kGpr = G >= 4 ? G / 2 : 1;        // groups per packed row
   static constexpr int kHeads = G / kGpr;                // query heads per group
   static constexpr int kRows = kGroups / kGpr;           // packed rows per chunk
-  static constexpr int kQBytes = kRows * G * D * 2;
+  static constexpr int kQBytes = kNoQ ? 0 : kRows * G * D * 2;
   static constexpr int kKBytes = kRows * D * 2;
   static constexpr int kStageBytes = kQBytes + 2 * kKBytes;  // Q, K, V
   static_assert(kStageBytes % 128 == 0, "stage alignment");
@@ -51,14 +52,17 @@ __host__ __device__ constexpr size_t rope_offs_bytes(int nseg) {
   return nseg + 1 <= kRopeStageMax ? ((size_t)(nseg + 1) * 4 + 15) / 16 * 16 : 0;
 }
 
-template <int D, int G>
+template <int D, int G, bool kNoQ = false>
 __host__ __device__ constexpr size_t rope_smem_bytes(int nseg) {
-  return (size_t)kRopeStages * RopeChunk<D, G>::kStageBytes + rope_offs_bytes(nseg) + kRopeStages * sizeof(uint64_t);
+  return (size_t)kRopeStages * RopeChunk<D, G, kNoQ>::kStageBytes + rope_offs_bytes(nseg) +
+         kRopeStages * sizeof(uint64_t);
 }
 
-// kFlags: NAMOH_ROPE_INTERLEAVED, NAMOH_ROPE_GLOBAL and kRopeRagged (global positions in a
-// ragged batch), compile-time so that no variant carries another's branches
+// kFlags: NAMOH_ROPE_INTERLEAVED, NAMOH_ROPE_GLOBAL, kRopeRagged (global positions in a ragged
+// batch) and kRopeNoQ (keys only, plus the cos / sin table the attention kernel rotates the
+// queries with), compile-time so that no variant carries another's branches
 constexpr unsigned kRopeRagged = 0x4u;
+constexpr unsigned kRopeNoQ = 0x8u;
 
 template <int D, int G, unsigned kFlags>
 __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
@@ -68,19 +72,23 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     uint16_t* __restrict__ k_cache, uint16_t* __restrict__ v_cache, int copy_v, RopeTable tab,
     uint32_t* __restrict__ status, int* __restrict__ plan_header, int4* __restrict__ plan_items,
     const int32_t* __restrict__ plan_cap, int plan_qtiles, const int32_t* __restrict__ pos_row_src,
-    FastDiv pos_k, FastDiv pos_t, const int32_t* __restrict__ pos_cu, FastDiv pos_hr) {
-  using C = RopeChunk<D, G>;
+    FastDiv pos_k, FastDiv pos_t, const int32_t* __restrict__ pos_cu, FastDiv pos_hr, float2* __restrict__ cs_tab,
+    int cs_rows, int plan_g) {
+  constexpr bool kNoQ = (kFlags & kRopeNoQ) != 0;
+  using C = RopeChunk<D, G, kNoQ>;
   constexpr int HALF = D / 2;
   constexpr bool kInterleaved = (kFlags & NAMOH_ROPE_INTERLEAVED) != 0;
   constexpr bool kGlobal = (kFlags & NAMOH_ROPE_GLOBAL) != 0;
   constexpr bool kRagged = (kFlags & kRopeRagged) != 0;
+  static_assert(!kNoQ || (G == 1 && !kGlobal), "keys-only passes use the rank and the one-row layout");
   extern __shared__ __align__(128) uint8_t smem_raw[];
   __shared__ int s_abort;
   pdl_launch_dependents();  // the attention kernel may start launching; it waits for this grid
   const int first = plan_header ? 1 : 0;
   if ((int)blockIdx.x < first) {
     pdl_wait();
-    build_plan(seg_offsets, nseg, plan_cap, G, plan_qtiles, plan_header, plan_items, reinterpret_cast<int*>(smem_raw));
+    build_plan(seg_offsets, nseg, plan_cap, plan_g, plan_qtiles, plan_header, plan_items,
+               reinterpret_cast<int*>(smem_raw));
     return;
   }
   const int nblk = gridDim.x - first, blk = blockIdx.x - first;
@@ -95,9 +103,9 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     const int r0 = c * C::kRows;
     const int rows = min(C::kRows, R - r0);
     uint8_t* base = stages + st * C::kStageBytes;
-    const uint32_t qb = (uint32_t)rows * G * D * 2, kb = (uint32_t)rows * D * 2;
+    const uint32_t qb = kNoQ ? 0u : (uint32_t)rows * G * D * 2, kb = (uint32_t)rows * D * 2;
     mbar_arrive_expect_tx(&full[st], qb + kb + (copy_v ? kb : 0u));
-    bulk_load(base, q + (size_t)r0 * G * D, qb, &full[st]);
+    if (!kNoQ) bulk_load(base, q + (size_t)r0 * G * D, qb, &full[st]);
     bulk_load(base + C::kQBytes, k + (size_t)r0 * D, kb, &full[st]);
     if (copy_v) bulk_load(base + C::kQBytes + C::kKBytes, v + (size_t)r0 * D, kb, &full[st]);
   };
@@ -114,6 +122,18 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     for (int i = threadIdx.x; i <= nseg; i += blockDim.x) s_offs[i] = __ldg(seg_offsets + i);
   __syncthreads();
   const int32_t* offs = staged ? s_offs : seg_offsets;
+  if (kNoQ && cs_tab) {
+    // cos / sin of every (rank p, pair j) the queries need, computed exactly as the rotation below
+    // computes them, while the first chunks' copies are in flight
+    const long long total = (long long)cs_rows * HALF;
+    for (long long idx = (long long)blk * kRopeThreads + threadIdx.x; idx < total;
+         idx += (long long)nblk * kRopeThreads) {
+      const int pp = (int)(idx / HALF), jj = (int)(idx - (long long)pp * HALF);
+      float sn, cs;
+      rope_sincos((float)pp, tab.theta_hi[jj], tab.theta_lo[jj], tab, &sn, &cs);
+      cs_tab[idx] = make_float2(cs, sn);
+    }
+  }
 
   const int grp = threadIdx.x / C::kLpr, lig = threadIdx.x % C::kLpr;
   const int prow = grp / C::kGpr;  // packed row within the chunk
@@ -203,10 +223,12 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
           *reinterpret_cast<uint4*>(dst_row + HALF + j0) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
         }
       };
+      if (!kNoQ) {
 #pragma unroll
-      for (int h = 0; h < C::kHeads; ++h) {
-        const int head = hsub * C::kHeads + h;
-        rotate(base + ((size_t)prow * G + head) * D * 2, q_rot + ((size_t)r * G + head) * D);
+        for (int h = 0; h < C::kHeads; ++h) {
+          const int head = hsub * C::kHeads + h;
+          rotate(base + ((size_t)prow * G + head) * D * 2, q_rot + ((size_t)r * G + head) * D);
+        }
       }
       if (hsub == 0) {
         long long dst = r;
@@ -248,13 +270,17 @@ cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, 
                                int copy_v, const RopeTable& tab, uint32_t* status, int* plan_header,
                                int4* plan_items, const int32_t* plan_cap, int plan_qtiles,
                                const int32_t* pos_row_src, FastDiv pos_k, FastDiv pos_t, const int32_t* pos_cu,
-                               FastDiv pos_hr) {
+                               FastDiv pos_hr, float2* cs_tab, int cs_rows) {
+  constexpr bool kNoQ = (F & kRopeNoQ) != 0;
+  const int plan_g = g;
+  if (kNoQ) g = 1;  // keys only: one key row per packed row whatever the group size
   switch (g) {
 #define NAMOH_ROPE_CASE(GG)                                                                                       \
   case GG: {                                                                                                      \
-    using C = RopeChunk<D, GG>;                                                                                  \
-    const auto kernel = rope_pack_kernel<D, GG, F>;                                                              \
-    const size_t rope_smem = rope_smem_bytes<D, GG>(nseg);                                                       \
+    constexpr int GE = kNoQ ? 1 : GG;                                                                            \
+    using C = RopeChunk<D, GE, kNoQ>;                                                                            \
+    const auto kernel = rope_pack_kernel<D, GE, F>;                                                              \
+    const size_t rope_smem = rope_smem_bytes<D, GE, kNoQ>(nseg);                                                 \
     const size_t smem0 = rope_smem > plan_smem ? rope_smem : plan_smem;                                          \
     /* two blocks per SM when their shared memory fits (228 KB per SM, 1 KB reserved per block); the */          \
     /* block scheduler packs blocks as deep as resources allow, so each block also asks for more than */          \
@@ -274,7 +300,8 @@ cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, 
     }                                                                                                            \
     return launch_pdl(kernel, dim3((unsigned)grid), dim3(kRopeThreads), smem, stream, q, k, v, R, seg_offsets,     \
                       nseg, seg_base, seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v, tab, status,         \
-                      plan_header, plan_items, plan_cap, plan_qtiles, pos_row_src, pos_k, pos_t, pos_cu, pos_hr); \
+                      plan_header, plan_items, plan_cap, plan_qtiles, pos_row_src, pos_k, pos_t, pos_cu, pos_hr,  \
+                      cs_tab, cs_rows, plan_g);                                                                  \
   }
     NAMOH_ROPE_CASE(1)
     NAMOH_ROPE_CASE(2)
@@ -292,19 +319,22 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache, bool copy_v,
                              const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream,
                              void* plan, int plan_qtiles, const int32_t* plan_cap, const int32_t* pos_row_src,
-                             int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved) {
+                             int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved,
+                             float2* cs_tab, int cs_rows) {
   int* plan_header = static_cast<int*>(plan);
   int4* plan_items = plan ? reinterpret_cast<int4*>(static_cast<char*>(plan) + 16) : nullptr;
   const size_t plan_smem = plan ? (size_t)plan_smem_ints(plan_qtiles, nseg) * sizeof(int) : 0;
   if (R == 0 && !plan) return cudaSuccess;
+  // with a cos / sin table to fill, the queries are left to the attention kernel (rank positions only)
+  if (cs_tab && pos_row_src) return cudaErrorInvalidValue;
   const unsigned flags = (interleaved ? NAMOH_ROPE_INTERLEAVED : 0u) | (pos_row_src ? NAMOH_ROPE_GLOBAL : 0u) |
-                         (pos_row_src && pos_cu ? kRopeRagged : 0u);
+                         (pos_row_src && pos_cu ? kRopeRagged : 0u) | (cs_tab ? kRopeNoQ : 0u);
   auto go = [&](auto d_tag, auto f_tag) {
     return launch_rope_pack_d<decltype(d_tag)::value, decltype(f_tag)::value>(
         g, sm_count, nseg, plan_smem, plan != nullptr, stream, q, k, v, R, seg_offsets, seg_base, seg_cap, cache_rows,
         q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status, plan_header, plan_items, plan_cap, plan_qtiles,
         pos_row_src, make_fastdiv((uint32_t)pos_k), make_fastdiv((uint32_t)pos_t), pos_cu,
-        make_fastdiv((uint32_t)pos_hr));
+        make_fastdiv((uint32_t)pos_hr), cs_tab, cs_rows);
   };
   using D64 = std::integral_constant<int, 64>;
   using D128 = std::integral_constant<int, 128>;
@@ -314,7 +344,11 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
   using F3 = std::integral_constant<unsigned, 3u>;
   using F6 = std::integral_constant<unsigned, 6u>;
   using F7 = std::integral_constant<unsigned, 7u>;
+  using F8 = std::integral_constant<unsigned, 8u>;
+  using F9 = std::integral_constant<unsigned, 9u>;
   switch (flags) {
+    case 8u: return D == 128 ? go(D128{}, F8{}) : go(D64{}, F8{});
+    case 9u: return D == 128 ? go(D128{}, F9{}) : go(D64{}, F9{});
     case 0u: return D == 128 ? go(D128{}, F0{}) : go(D64{}, F0{});
     case 1u: return D == 128 ? go(D128{}, F1{}) : go(D64{}, F1{});
     case 2u: return D == 128 ? go(D128{}, F2{}) : go(D64{}, F2{});
