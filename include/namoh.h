@@ -219,7 +219,14 @@ NAMOH_API int namoh_route_noalloc(const float *scores, int B, int T, int H, int 
  *             rows and outputs are skipped.
  * seg_len     NULL or [B*Hr] int32 out: n of each segment (decode state).
  * Supports d_head in {64, 128}, g in {1, 2, 4, 8}, rope_base > 1, T <= 2^20.
- * k_cache must not alias k.  Runs the three stages below in order.
+ * k_cache must not alias k.  Computes what the three stages below compute in order.
+ * At rank positions (no NAMOH_ROPE_GLOBAL) the rotated queries never go to HBM: the
+ * RoPE pass writes k~ (and v) and a cos / sin table of the ranks 0 .. T-1 into the
+ * workspace, and the attention kernel rotates each query tile in shared memory with
+ * the same arithmetic (bit for bit the q~ namoh_rope_pack writes).  Under
+ * NAMOH_ROPE_GLOBAL the queries are rotated into the workspace first.
+ * Workspace: namoh_prefill_workspace_size covers either (q~ [R*g, d] bf16, the plan,
+ * the table ceil(T / 128) * 128 * d/2 fp32 pairs).
  * ------------------------------------------------------------------------- */
 NAMOH_API size_t namoh_prefill_workspace_size(int B, int T, int H, int K, int d_head, int group);
 NAMOH_API int namoh_prefill(const uint16_t *q, const uint16_t *k, const uint16_t *v, int B, int T, int H, int K,
@@ -388,10 +395,13 @@ NAMOH_API int namoh_shared_decode(const uint16_t *q, const uint16_t *k, const ui
  *   sa_mask     [R*g, namoh_sa_mask_words(T, block)] uint32 out, 4-byte aligned: the kept
  *               earlier blocks of query (packed row r, group head j) at row r*g + j, bit
  *               b % 32 of word b / 32 for block b (the current block is implied).
- *   Workspace: namoh_sa_prefill_workspace_size (namoh_prefill's plus the pooled keys,
- *   (R / block + B*H/g) * d_head fp32).
- *   The attention does every causal key tile and masks the blocks not kept: the cost is
- *   that of namoh_prefill plus the selection.
+ *   Workspace: namoh_sa_prefill_workspace_size (the rotated queries q~ [R*g, d] bf16, which the
+ *   selection reads, the plan, and the pooled keys, (R / block + B*H/g) * d_head bf16).
+ *   The block scores of each 128-query tile run on the tensor cores (bf16 q~ and pooled keys,
+ *   fp32 sums); scores within 2^-13 of each other (relative) count as tied, ties to the lower
+ *   block.  The attention does every causal key tile and masks the blocks not kept: the cost
+ *   is that of namoh_prefill plus the selection.  Rows of a segment longer than its seg_cap
+ *   are neither pooled nor attended; their sa_mask rows are zero.
  * namoh_sa_mask_words: words per query of sa_mask (0 for an unsupported block).
  * Errors: NAMOH_ERR_INVALID_ARG for an unsupported block or alpha, a null sa_mask, or the
  * argument errors of namoh_prefill_ex.
