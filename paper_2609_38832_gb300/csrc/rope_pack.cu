@@ -29,6 +29,8 @@ namespace namoh {
 
 constexpr int kRopeThreads = 256;
 constexpr int kRopeStages = 3;
+// keys-only passes move half the bytes per chunk, so they keep twice the chunks in flight
+__host__ __device__ constexpr int rope_stages(bool no_q) { return no_q ? 2 * kRopeStages : kRopeStages; }
 constexpr int kRopeStageMax = 8192;  // seg_offsets entries staged in shared memory (32 KB)
 constexpr size_t kSmemPerSm = 233472;  // shared memory per SM (228 KB); each resident block also takes 1 KB
 // the least dynamic shared memory with which three blocks no longer fit on one SM
@@ -54,8 +56,8 @@ __host__ __device__ constexpr size_t rope_offs_bytes(int nseg) {
 
 template <int D, int G, bool kNoQ = false>
 __host__ __device__ constexpr size_t rope_smem_bytes(int nseg) {
-  return (size_t)kRopeStages * RopeChunk<D, G, kNoQ>::kStageBytes + rope_offs_bytes(nseg) +
-         kRopeStages * sizeof(uint64_t);
+  return (size_t)rope_stages(kNoQ) * RopeChunk<D, G, kNoQ>::kStageBytes + rope_offs_bytes(nseg) +
+         rope_stages(kNoQ) * sizeof(uint64_t);
 }
 
 // kFlags: NAMOH_ROPE_INTERLEAVED, NAMOH_ROPE_GLOBAL, kRopeRagged (global positions in a ragged
@@ -75,6 +77,7 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     FastDiv pos_k, FastDiv pos_t, const int32_t* __restrict__ pos_cu, FastDiv pos_hr, float2* __restrict__ cs_tab,
     int cs_rows, int plan_g) {
   constexpr bool kNoQ = (kFlags & kRopeNoQ) != 0;
+  constexpr int kStages = rope_stages(kNoQ);
   using C = RopeChunk<D, G, kNoQ>;
   constexpr int HALF = D / 2;
   constexpr bool kInterleaved = (kFlags & NAMOH_ROPE_INTERLEAVED) != 0;
@@ -94,8 +97,8 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
   const int nblk = gridDim.x - first, blk = blockIdx.x - first;
   const int nchunks = (R + C::kRows - 1) / C::kRows;
   uint8_t* stages = smem_raw;
-  int32_t* s_offs = reinterpret_cast<int32_t*>(smem_raw + kRopeStages * C::kStageBytes);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + kRopeStages * C::kStageBytes + rope_offs_bytes(nseg));
+  int32_t* s_offs = reinterpret_cast<int32_t*>(smem_raw + kStages * C::kStageBytes);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + kStages * C::kStageBytes + rope_offs_bytes(nseg));
   const bool staged = nseg + 1 <= kRopeStageMax;
 
   // chunk c into stage st: its rows' Q (g rows each), K and V, one bulk copy per array
@@ -110,13 +113,13 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     if (copy_v) bulk_load(base + C::kQBytes + C::kKBytes, v + (size_t)r0 * D, kb, &full[st]);
   };
   if (threadIdx.x == 0) {
-    for (int i = 0; i < kRopeStages; ++i) mbar_init(&full[i], 1);
+    for (int i = 0; i < kStages; ++i) mbar_init(&full[i], 1);
     s_abort = 0;
     mbar_fence_init();
   }
   pdl_wait();  // routing outputs (and q, k, v) are visible from here
   if (threadIdx.x == 0)
-    for (int i = 0; i < kRopeStages; ++i)
+    for (int i = 0; i < kStages; ++i)
       if (blk + i * nblk < nchunks) issue(blk + i * nblk, i);
   if (staged)
     for (int i = threadIdx.x; i <= nseg; i += blockDim.x) s_offs[i] = __ldg(seg_offsets + i);
@@ -155,14 +158,14 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     if (blk < nchunks && r_first < R) token_next = __ldg(pos_row_src + r_first);
   }
   for (int c = blk; c < nchunks; c += nblk, ++it) {
-    const int st = it % kRopeStages;
+    const int st = it % kStages;
     int token_src = 0;  // row_src of this thread's row: (b*T + t)*Kr + slot
     if (kGlobal) {
       token_src = token_next;
       const long long r_next = (long long)(c + nblk) * C::kRows + prow;
       if (c + nblk < nchunks && r_next < R) token_next = __ldg(pos_row_src + r_next);
     }
-    ok = mbar_wait(&full[st], (it / kRopeStages) & 1, &s_abort, status);
+    ok = mbar_wait(&full[st], (it / kStages) & 1, &s_abort, status);
     if (!__syncthreads_and(ok)) {
       ok = false;
       break;
@@ -252,7 +255,7 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
       }
     }
     __syncthreads();  // stage st fully read: refill it
-    if (threadIdx.x == 0 && c + kRopeStages * nblk < nchunks) issue(c + kRopeStages * nblk, st);
+    if (threadIdx.x == 0 && c + kStages * nblk < nchunks) issue(c + kStages * nblk, st);
   }
   if (!ok && threadIdx.x == 0) {
     // a wait gave up: let bulk copies still in flight land before the block exits

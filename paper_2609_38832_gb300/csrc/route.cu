@@ -73,10 +73,13 @@ __device__ __forceinline__ void load_logits(const float* __restrict__ scores, si
   }
   // one sum decides whether any logit needs looking at (it is non-finite when one is, or on
   // overflow, where the per-logit check then finds nothing to replace)
-  float total = 0.f;
+  uint64_t total2 = 0ull;
 #pragma unroll
-  for (int h = 0; h < HMAX; ++h)
-    if (h < H) total += sc[h];
+  for (int h = 0; h < HMAX; h += 2)
+    total2 = f2_add(total2, f2_pack(h < H ? sc[h] : 0.f, h + 1 < H ? sc[h + 1] : 0.f));
+  float ta, tb;
+  f2_unpack(total2, ta, tb);
+  const float total = ta + tb;
   bad = false;
   if (!isfinite(total)) {
 #pragma unroll
@@ -91,18 +94,26 @@ __device__ __forceinline__ void load_logits(const float* __restrict__ scores, si
 
 // Softmax normaliser over all H logits (Sec. 3.1 Eq. namoh-gates), fp32: the max and
 // 1 / sum_h exp(sc_h - max), each exponential as exp2((sc_h - max) * log2 e).
+// The subtract and scale run on fp32 pairs (f32x2), each lane rounded as the scalar form
+// would be; even heads sum into one partial and odd heads into the other.
 template <int HMAX>
 __device__ __forceinline__ void softmax_norm(const float (&sc)[HMAX], int H, float& mx, float& inv_z) {
   mx = -FLT_MAX;
 #pragma unroll
-  for (int h = 0; h < HMAX; ++h)
-    if (h < H) mx = fmaxf(mx, sc[h]);
-  float z0 = 0.f, z1 = 0.f;
+  for (int h = 0; h < HMAX; h += 2)
+    mx = fmax3(mx, h < H ? sc[h] : -FLT_MAX, h + 1 < H ? sc[h + 1] : -FLT_MAX);
+  const uint64_t nmx2 = f2_pack(-mx, -mx), l2e2 = f2_pack(kLog2e, kLog2e);
+  uint64_t z2 = 0ull;
 #pragma unroll
   for (int h = 0; h < HMAX; h += 2) {
-    if (h < H) z0 += fast_exp2((sc[h] - mx) * kLog2e);
-    if (h + 1 < H) z1 += fast_exp2((sc[h + 1] - mx) * kLog2e);
+    if (h < H) {
+      float x0, x1;
+      f2_unpack(f2_mul(f2_add(f2_pack(sc[h], h + 1 < H ? sc[h + 1] : mx), nmx2), l2e2), x0, x1);
+      z2 = f2_add(z2, f2_pack(fast_exp2(x0), h + 1 < H ? fast_exp2(x1) : 0.f));
+    }
   }
+  float z0, z1;
+  f2_unpack(z2, z0, z1);
   inv_z = 1.0f / (z0 + z1);
 }
 
@@ -133,6 +144,69 @@ __device__ __forceinline__ void topk_sorted(const float (&sc)[HMAX], int H, int 
       hk[0] = beats[0] ? h : hk[0];
     }
   }
+}
+
+// Top-4 (score desc, index asc) with few instructions per head, for K <= 4:
+//   1. the four largest values as a multiset, by a min / max insertion chain (no indices);
+//   2. the heads at or above the fourth value t3, in ascending index order: every head above t3
+//      (exactly as many as there are values above t3 in the multiset), then heads equal to t3 in
+//      index order until four -- ties go to the lower index;
+//   3. a stable sort of the four picks by value, descending (equal values keep index order).
+// Entries past H (H < 4) hold head 0 and -inf, as the insertion list does.
+template <int HMAX>
+__device__ __forceinline__ void topk4_sorted(const float (&sc)[HMAX], int H, int (&hk)[4], float (&vk)[4]) {
+  float t0 = -INFINITY, t1 = -INFINITY, t2 = -INFINITY, t3 = -INFINITY;
+#pragma unroll
+  for (int h = 0; h < HMAX; ++h) {
+    if (h < H) {
+      float x = sc[h], m;
+      m = fmaxf(t0, x); x = fminf(t0, x); t0 = m;
+      m = fmaxf(t1, x); x = fminf(t1, x); t1 = m;
+      m = fmaxf(t2, x); x = fminf(t2, x); t2 = m;
+      t3 = fmaxf(t3, x);
+    }
+  }
+  uint64_t ge = 0ull;  // heads at or above t3
+  float loc[HMAX];     // a copy the picks are read back from by index
+#pragma unroll
+  for (int h = 0; h < HMAX; ++h) {
+    loc[h] = sc[h];
+    if (h < H && sc[h] >= t3) ge |= 1ull << h;
+  }
+  int eq_left = 4 - ((t0 > t3) + (t1 > t3) + (t2 > t3));  // picks equal to t3
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    hk[k] = 0;
+    vk[k] = -INFINITY;
+  }
+  int n = 0;
+  while (ge && n < 4) {
+    const int h = __ffsll((long long)ge) - 1;
+    ge &= ge - 1ull;
+    const float x = loc[h];
+    const bool take = x > t3 || eq_left > 0;
+    if (!take) continue;
+    if (!(x > t3)) --eq_left;
+    if (n == 0) { hk[0] = h; vk[0] = x; }
+    else if (n == 1) { hk[1] = h; vk[1] = x; }
+    else if (n == 2) { hk[2] = h; vk[2] = x; }
+    else { hk[3] = h; vk[3] = x; }
+    ++n;
+  }
+  // odd-even transposition sort, swapping only on a strictly larger right value (stable)
+  auto cas = [&](int a, int b) {
+    const bool sw = vk[b] > vk[a];
+    const float va = vk[a], vb = vk[b];
+    const int ia = hk[a], ib = hk[b];
+    vk[a] = sw ? vb : va;
+    vk[b] = sw ? va : vb;
+    hk[a] = sw ? ib : ia;
+    hk[b] = sw ? ia : ib;
+  };
+  cas(0, 1); cas(2, 3);
+  cas(1, 2);
+  cas(0, 1); cas(2, 3);
+  cas(1, 2);
 }
 
 // Top-K for any K <= H: pass k picks the best head strictly after the previous pick in the
@@ -196,7 +270,8 @@ __device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores,
     return topk_passes<HMAX, kBiased>(sc, a, H, K, mx, inv_z, tok, topk_head, gate);
   } else {
     float vk[KMAX];
-    topk_sorted<HMAX, KMAX>(sc, H, hk, vk);
+    if constexpr (KMAX == 4) topk4_sorted<HMAX>(sc, H, hk, vk);
+    else topk_sorted<HMAX, KMAX>(sc, H, hk, vk);
     float g[KMAX];
     uint64_t mask = 0;
 #pragma unroll
@@ -320,9 +395,19 @@ __global__ void __launch_bounds__(kChunk) route_local_kernel(const float* __rest
   uint64_t mask = 0;
   int hk[KMAX > 0 ? KMAX : 1];
   if (valid) mask = topk_token<HMAX, KMAX, kBiased>(scores, bias, tok, H, K, topk_head, gate, &s_bad, hk);
-  for (int h = 0; h < H; ++h) {
-    const uint32_t bal = __ballot_sync(0xffffffffu, (mask >> h) & 1ull);
-    if (lane == 0) s_bal[warp][h] = bal;
+  // s_bal[warp][h] = the warp's ballot of "selects head h": the 32 x 32 bit matrix of the lanes'
+  // head masks transposed in five shuffle stages (each swaps the off-diagonal blocks of size j)
+#pragma unroll
+  for (int half = 0; half < (HMAX > 32 ? 2 : 1); ++half) {
+    uint32_t m = (uint32_t)(mask >> (32 * half));
+#pragma unroll
+    for (int j = 16; j > 0; j >>= 1) {
+      const uint32_t lowj = j == 16 ? 0x0000FFFFu : j == 8 ? 0x00FF00FFu : j == 4 ? 0x0F0F0F0Fu
+                            : j == 2 ? 0x33333333u : 0x55555555u;
+      const uint32_t y = __shfl_xor_sync(0xffffffffu, m, j);
+      m = (lane & j) ? ((m & ~lowj) | ((y >> j) & lowj)) : ((m & lowj) | ((y << j) & ~lowj));
+    }
+    if (32 * half + lane < H) s_bal[warp][32 * half + lane] = m;
   }
   __syncthreads();
   if (tid < H) {
