@@ -221,12 +221,11 @@ NAMOH_API int namoh_route_noalloc(const float *scores, int B, int T, int H, int 
  * Supports d_head in {64, 128}, g in {1, 2, 4, 8}, rope_base > 1, T <= 2^20.
  * k_cache must not alias k.  Computes what the three stages below compute in order.
  * At rank positions (no NAMOH_ROPE_GLOBAL) the rotated queries never go to HBM: the
- * RoPE pass writes k~ (and v) and a cos / sin table of the ranks 0 .. T-1 into the
- * workspace, and the attention kernel rotates each query tile in shared memory with
- * the same arithmetic (bit for bit the q~ namoh_rope_pack writes).  Under
- * NAMOH_ROPE_GLOBAL the queries are rotated into the workspace first.
- * Workspace: namoh_prefill_workspace_size covers either (q~ [R*g, d] bf16, the plan,
- * the table ceil(T / 128) * 128 * d/2 fp32 pairs).
+ * RoPE pass writes only k~ (and v), and the attention kernel rotates each query tile
+ * in shared memory with the same angle and rotation arithmetic (bit for bit the q~
+ * namoh_rope_pack writes).  Under NAMOH_ROPE_GLOBAL the queries are rotated into the
+ * workspace first.  Workspace: namoh_prefill_workspace_size covers either (q~
+ * [R*g, d] bf16 and the plan).
  * ------------------------------------------------------------------------- */
 NAMOH_API size_t namoh_prefill_workspace_size(int B, int T, int H, int K, int d_head, int group);
 NAMOH_API int namoh_prefill(const uint16_t *q, const uint16_t *k, const uint16_t *v, int B, int T, int H, int K,

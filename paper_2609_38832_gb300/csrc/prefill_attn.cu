@@ -31,9 +31,8 @@
 //               instruction by instruction while the softmax works on S(kv+1).
 //   warps 6-7   (kRopeQ instantiations only) query rotation: the producer loads the raw query
 //               tile, and thread i rotates rows i and i + 64 in shared memory at their ranks (Sec. 3.2, Eq.
-//               namoh-head-rope) from a cos / sin table the RoPE pass wrote, with the RoPE
-//               pass's own arithmetic, so the rotated tile is bit for bit the one that pass
-//               would have written to HBM.  The next item's tile lands and is rotated while
+//               namoh-head-rope) with the RoPE pass's own angle and rotation arithmetic, so the
+//               rotated tile is bit for bit the one that pass would have written to HBM.  The next item's tile lands and is rotated while
 //               the current item's last steps run, so the MMA issuer rarely waits for it.
 // TMEM: S/P buffers at cols [0,128), [128,256), [256,384); O at [384, 384 + D).
 // Shared memory (d = 128): Q 32 KB + 6 x 32 KB ring = 224 KB.
@@ -49,7 +48,7 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream,
                              void* plan, int plan_qtiles, const int32_t* plan_cap, const int32_t* pos_row_src,
                              int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved,
-                             float2* cs_tab, int cs_rows);
+                             bool keys_only);
 
 int launch_sa_select(const CUtensorMap& q_rot_map, const uint16_t* q_rot, const uint16_t* k_cache,
                      const int32_t* seg_offsets, const int64_t* seg_base, const int32_t* seg_cap,
@@ -67,7 +66,7 @@ constexpr int kSoftmaxWarps = 4;     // warps 0-3: thread i owns query row i (TM
 constexpr int kWarpLoad = 4;
 constexpr int kWarpMma = 5;
 constexpr int kWarpRope0 = 6;        // warps 6-7: query rotation (kRopeQ instantiations)
-constexpr int kRopeWarps = 2;        // (two rows per thread: the block stays within 256 registers a thread)
+constexpr int kRopeWarps = 2;        // two rows a thread: 256 threads keep the 190-register budget
 constexpr int kThreads = 192;
 // kRopeQ: 0 = the queries come rotated; 1 = rotate them here, half-split pairs; 2 = interleaved pairs
 __host__ __device__ constexpr int threads_for(int rope_q) { return rope_q ? kThreads + 32 * kRopeWarps : kThreads; }
@@ -135,9 +134,7 @@ struct Params {
   const uint32_t* sa_mask;
   int sa_words;
   int sa_lg;
-  // kRopeQ: cos / sin of rank p and pair j at cs_tab[p * D / 2 + j] (cs_rows ranks)
-  const float2* cs_tab;
-  int cs_rows;
+  RopeTable tab;  // kRopeQ: the RoPE frequencies (the angles are computed as the RoPE pass does)
 };
 
 // All lanes of a warp wait and agree on the outcome, so warp-collective tcgen05
@@ -289,31 +286,25 @@ __device__ __forceinline__ bool softmax_tile(uint32_t s_addr, uint32_t o_addr, i
 }
 
 // Rotates query row `row` of the 128B-swizzled tile at q_smem in place (rank RoPE, Sec. 3.2 Eq.
-// namoh-head-rope) with cos / sin from the table row of its rank.  Element e of a row sits in
-// 64-column atom e / 64, 16-byte chunk (e % 64) / 8, stored at chunk position chunk ^ (row % 8).
-// x'_j = x_j cos - x_{j+D/2} sin, x'_{j+D/2} = x_{j+D/2} cos + x_j sin (interleaved: the pair
-// (2j, 2j+1) in one bf16x2 word), each product and rounding as the RoPE pass does them.
+// namoh-head-rope) to position `pos`.  Element e of a row sits in 64-column atom e / 64, 16-byte
+// chunk (e % 64) / 8, stored at chunk position chunk ^ (row % 8).  x'_j = x_j cos - x_{j+D/2} sin,
+// x'_{j+D/2} = x_{j+D/2} cos + x_j sin (interleaved: the pair (2j, 2j+1) in one bf16x2 word); the
+// angles, products and roundings are the RoPE pass's, so the tile is bit for bit the q~ that pass
+// would write.
 template <int D, int kRopeQ>
-__device__ __forceinline__ void rotate_query_row(uint8_t* q_smem, int row, const float2* __restrict__ cs) {
+__device__ __forceinline__ void rotate_query_row(uint8_t* q_smem, int row, float pos, const RopeTable& tab) {
   constexpr int kAtomBytes = BM * 128;
   const int sw = row & 7;
   auto chunk_ptr = [&](int e) -> uint4* {  // the 16-byte chunk holding element e (a multiple of 8)
     return reinterpret_cast<uint4*>(q_smem + (e >> 6) * kAtomBytes + row * 128 + ((((e & 63) >> 3) ^ sw) << 4));
   };
-  const float4* tb = reinterpret_cast<const float4*>(cs);  // {cos_j, sin_j, cos_j+1, sin_j+1}
   if constexpr (kRopeQ == 1) {
     constexpr int HALF = D / 2;
 #pragma unroll
     for (int c = 0; c < HALF / 8; ++c) {
       float cs8[8], sn8[8];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const float4 t = __ldg(tb + 4 * c + i);
-        cs8[2 * i] = t.x;
-        sn8[2 * i] = t.y;
-        cs8[2 * i + 1] = t.z;
-        sn8[2 * i + 1] = t.w;
-      }
+      for (int i = 0; i < 8; ++i) rope_sincos(pos, tab.theta_hi[8 * c + i], tab.theta_lo[8 * c + i], tab, &sn8[i], &cs8[i]);
       uint4* pa = chunk_ptr(8 * c);
       uint4* pb = chunk_ptr(HALF + 8 * c);
       const uint4 a = *pa, b = *pb;
@@ -334,9 +325,9 @@ __device__ __forceinline__ void rotate_query_row(uint8_t* q_smem, int row, const
   } else {
 #pragma unroll
     for (int c = 0; c < D / 8; ++c) {  // chunk c holds pairs j = 4c .. 4c + 3
-      const float4 t0 = __ldg(tb + 2 * c), t1 = __ldg(tb + 2 * c + 1);
-      const float cs4[4] = {t0.x, t0.z, t1.x, t1.z};
-      const float sn4[4] = {t0.y, t0.w, t1.y, t1.w};
+      float cs4[4], sn4[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) rope_sincos(pos, tab.theta_hi[4 * c + i], tab.theta_lo[4 * c + i], tab, &sn4[i], &cs4[i]);
       uint4* pa = chunk_ptr(8 * c);
       const uint4 a = *pa;
       const uint32_t w[4] = {a.x, a.y, a.z, a.w};
@@ -626,19 +617,18 @@ __global__ void __launch_bounds__(threads_for(kRopeQ), 1)
     __syncwarp();
   } else if (kRopeQ && warp >= kWarpRope0) {
     // ------------------------------------------------------------------ query rotation
-    const int row = (warp - kWarpRope0) * 32 + lane;  // rows `row` and `row` + 64 of the tile
+    const int row = (warp - kWarpRope0) * 32 + lane;  // query rows `row` and `row` + 64 of the tile
     uint32_t item_iter = 0;
     bool ok = true;
     while (ok) {
       int4 item;
       ok = take_item(bars, item_iter, &item, abort_flag, p.status);
       if (!ok || item.x < 0) break;
-      // ranks of the two rows (past the segment's end: rotated but never used)
-      const int pos0 = min(item.y * BM + row, p.cs_rows - 1), pos1 = min(item.y * BM + row + 64, p.cs_rows - 1);
       ok = warp_wait(&bars->q_full, item_iter & 1, abort_flag, p.status);
       if (!ok) break;
-      rotate_query_row<D, kRopeQ>(smem + L::kQ, row, p.cs_tab + (size_t)pos0 * (D / 2));
-      rotate_query_row<D, kRopeQ>(smem + L::kQ, row + 64, p.cs_tab + (size_t)pos1 * (D / 2));
+      // ranks of the rows (past the segment's end: rotated but never used)
+      rotate_query_row<D, kRopeQ>(smem + L::kQ, row, (float)(item.y * BM + row), p.tab);
+      rotate_query_row<D, kRopeQ>(smem + L::kQ, row + 64, (float)(item.y * BM + row + 64), p.tab);
       fence_proxy_async_smem();  // the MMA reads the tile through the async proxy
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars->q_ready);
@@ -830,8 +820,6 @@ size_t plan_bytes_rows(long long R, int nseg, int g) {
 size_t plan_bytes_for(int B, int T, int Hr, int Kr, int g) { return plan_bytes_rows((long long)B * T * Kr, B * Hr, g); }
 
 int plan_qtiles_for(int T) { return (T + kPlanTileRows - 1) / kPlanTileRows; }  // query tiles per segment, at most
-// ranks the query-rotation table covers: every row of every query tile of a history of at most T
-int cs_rows_for(int T) { return plan_qtiles_for(T) * kPlanTileRows; }
 
 // The RoPE launch builds the plan in one extra block when the plan's shared memory is small
 // enough not to cut the RoPE blocks' occupancy.
@@ -856,14 +844,13 @@ int launch_plan(const int32_t* seg_offsets, int nseg, int T, int g, const int32_
 // the plan's shared memory is small, else as a second kernel).
 // rope_flags: NAMOH_ROPE_GLOBAL takes the positions from row_src: t = (row_src[r] / Kr) % T,
 // or row_src[r] / Kr - cu_seqlens[b] in a ragged batch (T is then the longest sequence).
-// With cs_tab the queries are not rotated here: the pass writes the cos / sin table of ranks
-// 0 .. cs_rows - 1 instead, and the attention kernel rotates the queries (rank positions only).
+// keys_only: the queries are not rotated here; the attention kernel rotates them (rank positions only).
 int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int Hr, int Kr, int R,
                          int d_head, int group, float rope_base, unsigned rope_flags, const int32_t* cu_seqlens,
                          const int32_t* seg_offsets, const int32_t* row_src, uint16_t* q_rot, uint16_t* k_cache,
                          uint16_t* v_cache, const int64_t* seg_base, const int32_t* seg_cap, long long cache_rows,
                          uint32_t* dev_status, void* plan, const DeviceInfo& info, cudaStream_t stream,
-                         float2* cs_tab = nullptr, int cs_rows = 0) {
+                         bool keys_only = false) {
   RopeTable tab;
   fill_rope_table(&tab, d_head, (double)rope_base);
   const int nseg = B * Hr;
@@ -874,7 +861,7 @@ int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v
                                          q_rot, k_cache, v_cache, v_cache != v, tab, dev_status, info.sm_count, stream,
                                          fuse_plan ? plan : nullptr, qtiles, plan_cap,
                                          (rope_flags & NAMOH_ROPE_GLOBAL) ? row_src : nullptr, Kr, T, cu_seqlens,
-                                         Hr, (rope_flags & NAMOH_ROPE_INTERLEAVED) != 0, cs_tab, cs_rows);
+                                         Hr, (rope_flags & NAMOH_ROPE_INTERLEAVED) != 0, keys_only);
   if (e != cudaSuccess) return cuda_fail(e, "rope_pack_kernel launch");
   if (plan && !fuse_plan) return launch_plan(seg_offsets, nseg, T, group, plan_cap, plan, stream);
   return NAMOH_OK;
@@ -885,8 +872,9 @@ int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint1
                      const int64_t* seg_base, long long cache_rows, void* plan, uint16_t* y, uint32_t* dev_status,
                      const DeviceInfo& info, cudaStream_t stream, int window = 0,
                      const uint32_t* sa_mask = nullptr, int sa_words = 0, int sa_lg = 0, int rope_q = 0,
-                     const float2* cs_tab = nullptr, int cs_rows = 0) {
-  // rope_q > 0: q_rot holds the raw queries, rotated in the kernel (1 half-split, 2 interleaved)
+                     float rope_base = 0.f) {
+  // rope_q > 0: q_rot holds the raw queries, rotated in the kernel at their ranks with rope_base
+  // (1 half-split, 2 interleaved)
   CUtensorMap tq, tk, tv;
   if (!attn::encode_rows_map(&tq, q_rot, R, g * D) || !attn::encode_rows_map(&tk, k_cache, cache_rows, D) ||
       !attn::encode_rows_map(&tv, v_cache, cache_rows, D))
@@ -909,8 +897,7 @@ int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint1
   p.sa_mask = sa_mask;
   p.sa_words = sa_words;
   p.sa_lg = sa_lg;
-  p.cs_tab = cs_tab;
-  p.cs_rows = cs_rows;
+  if (rope_q) fill_rope_table(&p.tab, D, (double)rope_base);
   cudaError_t e;
   const int G = info.sm_count;
   if (sa_mask)
@@ -1046,8 +1033,6 @@ int prefill_impl(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B,
   WorkspaceCarver ws{static_cast<char*>(workspace), workspace_bytes, 0};
   uint16_t* q_rot = ws.take<uint16_t>((size_t)R * group * d_head);
   void* plan = ws.take<char>(plan_bytes_rows(R, B * Hr, group));
-  const int cs_rows = cs_rows_for(T);
-  float2* cs_tab = ws.take<float2>((size_t)cs_rows * (d_head / 2));
   if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
   DeviceInfo info;
   if (!device_ok(&info)) return NAMOH_ERR_UNSUPPORTED;
@@ -1056,7 +1041,7 @@ int prefill_impl(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B,
   const bool fuse_q = !(rope_flags & NAMOH_ROPE_GLOBAL);
   int st = launch_rope_and_plan(q, k, v, B, T, Hr, Kr, (int)R, d_head, group, rope_base, rope_flags, cu_seqlens,
                                 seg_offsets, row_src, q_rot, k_cache, v_cache, seg_base, seg_cap, cache_rows,
-                                dev_status, plan, info, stream, fuse_q ? cs_tab : nullptr, cs_rows);
+                                dev_status, plan, info, stream, fuse_q);
   if (st != NAMOH_OK) return st;
   if (seg_len) {
     seg_len_kernel<<<(B * Hr + 255) / 256, 256, 0, stream>>>(seg_offsets, B * Hr, seg_len);
@@ -1064,14 +1049,13 @@ int prefill_impl(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B,
   }
   const int rope_q = fuse_q ? ((rope_flags & NAMOH_ROPE_INTERLEAVED) ? 2 : 1) : 0;
   return launch_attention(fuse_q ? q : q_rot, k_cache, v_cache, R, d_head, group, seg_offsets, row_src, gate, seg_base,
-                          cache_rows, plan, y, dev_status, info, stream, 0, nullptr, 0, 0, rope_q, cs_tab, cs_rows);
+                          cache_rows, plan, y, dev_status, info, stream, 0, nullptr, 0, 0, rope_q, rope_base);
 }
 
 size_t prefill_workspace_rows(long long R, int nseg, int T, int d_head, int group) {
   WorkspaceCarver ws{nullptr, 0, 0};
   ws.take<uint16_t>((size_t)R * group * d_head);
   ws.take<char>(plan_bytes_rows(R, nseg, group));
-  ws.take<float2>((size_t)cs_rows_for(T) * (d_head / 2));
   return align_up(ws.used, 256);
 }
 
@@ -1258,8 +1242,7 @@ __global__ void shared_layout_kernel(int B, int T, int Hs, int32_t* __restrict__
 struct SharedWs {
   int32_t *seg_offsets, *row_src;
   float* gate;
-  void* plan;
-  float2* cs_tab;  // the attention kernel rotates the queries (the rank in these segments is t)
+  void* plan;  // (the attention kernel rotates the queries: the rank in these segments is t)
 };
 void carve_shared(WorkspaceCarver& ws, SharedWs* o, int B, int T, int Hs, int d_head) {
   const long long R = (long long)B * Hs * T;
@@ -1267,7 +1250,6 @@ void carve_shared(WorkspaceCarver& ws, SharedWs* o, int B, int T, int Hs, int d_
   o->row_src = ws.take<int32_t>((size_t)R);
   o->gate = ws.take<float>((size_t)R);
   o->plan = ws.take<char>(plan_bytes_rows(R, B * Hs, 1));
-  o->cs_tab = ws.take<float2>((size_t)cs_rows_for(T) * (d_head / 2));
 }
 }  // namespace
 }  // namespace namoh
@@ -1316,13 +1298,12 @@ extern "C" int namoh_shared_prefill(const uint16_t* q, const uint16_t* k, const 
   const bool il = (rope_flags & NAMOH_ROPE_INTERLEAVED) != 0;
   st = launch_rope_and_plan(q, k, v, B, T, Hs, Hs, (int)R, d_head, 1, rope_base, il ? NAMOH_ROPE_INTERLEAVED : 0u,
                             nullptr, o.seg_offsets, o.row_src, nullptr, k_cache, v_cache, seg_base, seg_cap,
-                            cache_rows, dev_status, o.plan, info, stream, o.cs_tab, cs_rows_for(T));
+                            cache_rows, dev_status, o.plan, info, stream, true);
   if (st != NAMOH_OK) return st;
   if (seg_len) {
     seg_len_kernel<<<(B * Hs + 255) / 256, 256, 0, stream>>>(o.seg_offsets, B * Hs, seg_len);
     if (const int e = cuda_check_launch("seg_len_kernel launch")) return e;
   }
   return launch_attention(q, k_cache, v_cache, R, d_head, 1, o.seg_offsets, o.row_src, o.gate, seg_base,
-                          cache_rows, o.plan, y, dev_status, info, stream, window, nullptr, 0, 0, il ? 2 : 1, o.cs_tab,
-                          cs_rows_for(T));
+                          cache_rows, o.plan, y, dev_status, info, stream, window, nullptr, 0, 0, il ? 2 : 1, rope_base);
 }

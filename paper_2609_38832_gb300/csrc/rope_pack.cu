@@ -61,8 +61,8 @@ __host__ __device__ constexpr size_t rope_smem_bytes(int nseg) {
 }
 
 // kFlags: NAMOH_ROPE_INTERLEAVED, NAMOH_ROPE_GLOBAL, kRopeRagged (global positions in a ragged
-// batch) and kRopeNoQ (keys only, plus the cos / sin table the attention kernel rotates the
-// queries with), compile-time so that no variant carries another's branches
+// batch) and kRopeNoQ (keys and values only: the attention kernel rotates the queries itself),
+// compile-time so that no variant carries another's branches
 constexpr unsigned kRopeRagged = 0x4u;
 constexpr unsigned kRopeNoQ = 0x8u;
 
@@ -74,8 +74,7 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     uint16_t* __restrict__ k_cache, uint16_t* __restrict__ v_cache, int copy_v, RopeTable tab,
     uint32_t* __restrict__ status, int* __restrict__ plan_header, int4* __restrict__ plan_items,
     const int32_t* __restrict__ plan_cap, int plan_qtiles, const int32_t* __restrict__ pos_row_src,
-    FastDiv pos_k, FastDiv pos_t, const int32_t* __restrict__ pos_cu, FastDiv pos_hr, float2* __restrict__ cs_tab,
-    int cs_rows, int plan_g) {
+    FastDiv pos_k, FastDiv pos_t, const int32_t* __restrict__ pos_cu, FastDiv pos_hr, int plan_g) {
   constexpr bool kNoQ = (kFlags & kRopeNoQ) != 0;
   constexpr int kStages = rope_stages(kNoQ);
   using C = RopeChunk<D, G, kNoQ>;
@@ -125,18 +124,6 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     for (int i = threadIdx.x; i <= nseg; i += blockDim.x) s_offs[i] = __ldg(seg_offsets + i);
   __syncthreads();
   const int32_t* offs = staged ? s_offs : seg_offsets;
-  if (kNoQ && cs_tab) {
-    // cos / sin of every (rank p, pair j) the queries need, computed exactly as the rotation below
-    // computes them, while the first chunks' copies are in flight
-    const long long total = (long long)cs_rows * HALF;
-    for (long long idx = (long long)blk * kRopeThreads + threadIdx.x; idx < total;
-         idx += (long long)nblk * kRopeThreads) {
-      const int pp = (int)(idx / HALF), jj = (int)(idx - (long long)pp * HALF);
-      float sn, cs;
-      rope_sincos((float)pp, tab.theta_hi[jj], tab.theta_lo[jj], tab, &sn, &cs);
-      cs_tab[idx] = make_float2(cs, sn);
-    }
-  }
 
   const int grp = threadIdx.x / C::kLpr, lig = threadIdx.x % C::kLpr;
   const int prow = grp / C::kGpr;  // packed row within the chunk
@@ -273,7 +260,7 @@ cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, 
                                int copy_v, const RopeTable& tab, uint32_t* status, int* plan_header,
                                int4* plan_items, const int32_t* plan_cap, int plan_qtiles,
                                const int32_t* pos_row_src, FastDiv pos_k, FastDiv pos_t, const int32_t* pos_cu,
-                               FastDiv pos_hr, float2* cs_tab, int cs_rows) {
+                               FastDiv pos_hr) {
   constexpr bool kNoQ = (F & kRopeNoQ) != 0;
   const int plan_g = g;
   if (kNoQ) g = 1;  // keys only: one key row per packed row whatever the group size
@@ -304,7 +291,7 @@ cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, 
     return launch_pdl(kernel, dim3((unsigned)grid), dim3(kRopeThreads), smem, stream, q, k, v, R, seg_offsets,     \
                       nseg, seg_base, seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v, tab, status,         \
                       plan_header, plan_items, plan_cap, plan_qtiles, pos_row_src, pos_k, pos_t, pos_cu, pos_hr,  \
-                      cs_tab, cs_rows, plan_g);                                                                  \
+                      plan_g);                                                                                   \
   }
     NAMOH_ROPE_CASE(1)
     NAMOH_ROPE_CASE(2)
@@ -323,21 +310,21 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream,
                              void* plan, int plan_qtiles, const int32_t* plan_cap, const int32_t* pos_row_src,
                              int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved,
-                             float2* cs_tab, int cs_rows) {
+                             bool keys_only) {
   int* plan_header = static_cast<int*>(plan);
   int4* plan_items = plan ? reinterpret_cast<int4*>(static_cast<char*>(plan) + 16) : nullptr;
   const size_t plan_smem = plan ? (size_t)plan_smem_ints(plan_qtiles, nseg) * sizeof(int) : 0;
   if (R == 0 && !plan) return cudaSuccess;
-  // with a cos / sin table to fill, the queries are left to the attention kernel (rank positions only)
-  if (cs_tab && pos_row_src) return cudaErrorInvalidValue;
+  // keys only: the queries are left to the attention kernel (rank positions only)
+  if (keys_only && pos_row_src) return cudaErrorInvalidValue;
   const unsigned flags = (interleaved ? NAMOH_ROPE_INTERLEAVED : 0u) | (pos_row_src ? NAMOH_ROPE_GLOBAL : 0u) |
-                         (pos_row_src && pos_cu ? kRopeRagged : 0u) | (cs_tab ? kRopeNoQ : 0u);
+                         (pos_row_src && pos_cu ? kRopeRagged : 0u) | (keys_only ? kRopeNoQ : 0u);
   auto go = [&](auto d_tag, auto f_tag) {
     return launch_rope_pack_d<decltype(d_tag)::value, decltype(f_tag)::value>(
         g, sm_count, nseg, plan_smem, plan != nullptr, stream, q, k, v, R, seg_offsets, seg_base, seg_cap, cache_rows,
         q_rot, k_cache, v_cache, copy_v ? 1 : 0, tab, status, plan_header, plan_items, plan_cap, plan_qtiles,
         pos_row_src, make_fastdiv((uint32_t)pos_k), make_fastdiv((uint32_t)pos_t), pos_cu,
-        make_fastdiv((uint32_t)pos_hr), cs_tab, cs_rows);
+        make_fastdiv((uint32_t)pos_hr));
   };
   using D64 = std::integral_constant<int, 64>;
   using D128 = std::integral_constant<int, 128>;

@@ -97,7 +97,8 @@ __global__ void __launch_bounds__(256) sa_pool_kernel(const uint16_t* __restrict
   const int piece = lane % P, sub = lane / P;
   float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
   const uint4* src = reinterpret_cast<const uint4*>(k_cache + row0 * d) + piece;
-  for (int t = sub; t < (1 << lg); t += rows_per) {
+#pragma unroll 8
+  for (int t = sub; t < (1 << lg); t += rows_per) {  // unrolled: eight 16-byte loads in flight per lane
     const uint4 w = __ldg(src + (long long)t * P);
     const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
@@ -244,6 +245,7 @@ __global__ void __launch_bounds__(kSelThreads) sa_select_tc_kernel(const __grid_
 #pragma unroll
       for (int i = 0; i < kListLen; ++i) best[i] = 0u;
       for (int c = 0; c < nchunks; ++c) {
+        if (__all_sync(0xffffffffu, !use_list || c * 32 >= cand)) continue;  // no lane has a candidate here
         uint32_t v[32];
         load_scores(lane_addr + (uint32_t)(c * 32), v);
 #pragma unroll
@@ -287,6 +289,10 @@ __global__ void __launch_bounds__(kSelThreads) sa_select_tc_kernel(const __grid_
     }
     // the mask: block b kept iff key >= tau (kept mode), ~key < tau (drop mode)
     for (int c = 0; c < nchunks; ++c) {
+      if (__all_sync(0xffffffffu, c * 32 >= cand)) {  // no candidate of any lane: an empty word
+        if (mine && c < p.words) mrow[c] = 0u;
+        continue;
+      }
       uint32_t v[32];
       load_scores(lane_addr + (uint32_t)(c * 32), v);
       uint32_t w = 0u;

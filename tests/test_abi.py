@@ -110,9 +110,8 @@ def test_sa_sizes_and_argument_errors(lib):
     assert lib.namoh_sa_mask_words(4096, 128) == 1
     assert lib.namoh_sa_mask_words(4096, 48) == 0 and lib.namoh_sa_mask_words(4096, 16) == 0
     plain = lib.namoh_prefill_workspace_size(4, 4096, 16, 4, 128, 1)
-    # the dense prefill's workspace: rotated queries (R g d bf16) or, at rank positions, the cos / sin
-    # table of the query rotation (ranks up to T rounded to 128, d / 2 pairs, fp32 pairs)
-    assert plain >= 65536 * 128 * 2 + 4096 * 64 * 8
+    # the dense prefill's workspace holds the rotated queries (R g d bf16) for the global-position path
+    assert plain >= 65536 * 128 * 2
     # SA: the rotated queries (the selection reads them) plus the pooled keys, (R / block + B H) d bf16
     assert lib.namoh_sa_prefill_workspace_size(4, 4096, 16, 4, 128, 1, 32) >= 65536 * 128 * 2 + (65536 // 32 + 64) * 128 * 2
     assert lib.namoh_sa_prefill_workspace_size(4, 4096, 16, 4, 128, 1, 48) == 0
