@@ -219,13 +219,7 @@ NAMOH_API int namoh_route_noalloc(const float *scores, int B, int T, int H, int 
  *             rows and outputs are skipped.
  * seg_len     NULL or [B*Hr] int32 out: n of each segment (decode state).
  * Supports d_head in {64, 128}, g in {1, 2, 4, 8}, rope_base > 1, T <= 2^20.
- * k_cache must not alias k.  Computes what the three stages below compute in order.
- * At rank positions (no NAMOH_ROPE_GLOBAL) the rotated queries never go to HBM: the
- * RoPE pass writes only k~ (and v), and the attention kernel rotates each query tile
- * in shared memory with the same angle and rotation arithmetic (bit for bit the q~
- * namoh_rope_pack writes).  Under NAMOH_ROPE_GLOBAL the queries are rotated into the
- * workspace first.  Workspace: namoh_prefill_workspace_size covers either (q~
- * [R*g, d] bf16 and the plan).
+ * k_cache must not alias k.  Runs the three stages below in order.
  * ------------------------------------------------------------------------- */
 NAMOH_API size_t namoh_prefill_workspace_size(int B, int T, int H, int K, int d_head, int group);
 NAMOH_API int namoh_prefill(const uint16_t *q, const uint16_t *k, const uint16_t *v, int B, int T, int H, int K,
@@ -306,6 +300,22 @@ NAMOH_API int namoh_attention(const uint16_t *q_rot, const uint16_t *k_cache, co
                               int H, int K, int d_head, int group, const int32_t *seg_offsets, const int32_t *row_src,
                               const float *gate, const int64_t *seg_base, int64_t cache_rows, void *plan,
                               size_t plan_bytes, uint16_t *y, uint32_t *dev_status, void *stream);
+
+/* namoh_attention_timeout_probe: a check of the kernels' bounded waits, for tests (no
+ * counterpart in the paper).  Every wait of the attention kernel gives up after a limit
+ * (2 s), reports NAMOH_DEV_TIMEOUT and lets every role drain and exit, so that a stalled
+ * pipeline returns an error instead of hanging the GPU.  This call runs namoh_attention
+ * (packed caches, seg_base NULL) with the first query tile of every CTA withheld: the
+ * MMA issuer's wait for it runs out after wait_limit_ns (1 us .. 2 s) and sets in
+ * *dev_status NAMOH_DEV_TIMEOUT, bits 16-22 = 4 (the query tile's barrier, the fifth
+ * word of the kernel's barrier block) and bits 24-31 = 5 (the MMA issuer's warp).  y is
+ * left unspecified; the plan and the context stay usable.  Argument errors as
+ * namoh_attention, plus NAMOH_ERR_INVALID_ARG for a limit out of range. */
+NAMOH_API int namoh_attention_timeout_probe(const uint16_t *q_rot, const uint16_t *k_cache, const uint16_t *v_cache,
+                                            int B, int T, int H, int K, int d_head, int group,
+                                            const int32_t *seg_offsets, const int32_t *row_src, const float *gate,
+                                            void *plan, size_t plan_bytes, uint16_t *y, uint64_t wait_limit_ns,
+                                            uint32_t *dev_status, void *stream);
 
 /* ------------------------------------------------------------------------- *
  * Decode: one new token per sequence.

@@ -338,6 +338,27 @@ def namoh_attention(q_rot: torch.Tensor, k_cache: torch.Tensor, v_cache: torch.T
     return y
 
 
+def namoh_attention_timeout_probe(q_rot: torch.Tensor, k_cache: torch.Tensor, v_cache: torch.Tensor,
+                                  seg_offsets: torch.Tensor, row_src: torch.Tensor, gate: torch.Tensor,
+                                  plan: torch.Tensor, *, B: int, T: int, H: int, K: int, group: int = 1,
+                                  wait_limit_ns: int = 1_000_000, y: Optional[torch.Tensor] = None,
+                                  status: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Check of the bounded waits (see namoh_attention_timeout_probe in include/namoh.h): namoh_attention
+    with every CTA's first query tile withheld, so that the MMA issuer's wait runs out after wait_limit_ns
+    and NAMOH_DEV_TIMEOUT is reported.  Returns the status tensor."""
+    lib = _abi.load()
+    d = q_rot.shape[-1]
+    dev = q_rot.device
+    if y is None:
+        y = torch.empty((B, T, K, d), dtype=torch.bfloat16, device=dev)
+    st = _status(status, dev)
+    rc = lib.namoh_attention_timeout_probe(_ptr(q_rot), _ptr(k_cache), _ptr(v_cache), B, T, H, K, d, group,
+                                           _ptr(seg_offsets), _ptr(row_src), _ptr(gate), _ptr(plan), plan.numel(),
+                                           _ptr(y), int(wait_limit_ns), _ptr(st), _stream(stream))
+    _abi.check("namoh_attention_timeout_probe", rc)
+    return st
+
+
 def namoh_shared_prefill(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, *, window: int = 0,
                          rope_base: float = 10000.0, interleaved: bool = False, y: Optional[torch.Tensor] = None,
                          k_cache: Optional[torch.Tensor] = None, v_cache: Optional[torch.Tensor] = None,

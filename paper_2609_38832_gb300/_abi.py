@@ -58,6 +58,8 @@ SIGNATURES = {
     "namoh_attention_plan_size": (_SZ, [_I, _I, _I, _I, _I]),
     "namoh_attention_plan": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _SZ, _P]),
     "namoh_attention": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _P, _I64, _P, _SZ, _P, _P, _P]),
+    "namoh_attention_timeout_probe": (_I, [_P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _P, _SZ, _P,
+                                           ctypes.c_uint64, _P, _P]),
     "namoh_proj_workspace_size": (_SZ, [_I, _I, _I, _I, _I, _I]),
     "namoh_proj_qkv": (_I, [_P, _I, _I, _P, _I, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _SZ, _P, _P]),
     "namoh_proj_out": (_I, [_P, _I, _I, _P, _I, _I, _I, _I, _I, _P, _P, _P, _I, _P, _SZ, _P, _P]),

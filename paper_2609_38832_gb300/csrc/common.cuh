@@ -137,21 +137,22 @@ constexpr uint32_t kWaitSleepNs = 20000;  // longest sleep per try (the abort fl
 // others: once it is set every wait returns false immediately.  Returns true when
 // the phase with the given parity completed.
 static __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                            uint32_t* status);
+                                            uint32_t* status, uint64_t limit_ns);
 // The first try is inline; the polling loop and the timeout report stay out of line, so that
-// the many waits of a pipeline loop keep its code small.
+// the many waits of a pipeline loop keep its code small.  limit_ns: how long the wait may last
+// (kWaitLimitNs unless a caller asked for less).
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                          uint32_t* status) {
+                                          uint32_t* status, uint64_t limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
-  return mbar_wait_slow(bar, parity, abort_flag, status);
+  return mbar_wait_slow(bar, parity, abort_flag, status, limit_ns);
 }
 static __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                            uint32_t* status) {
+                                            uint32_t* status, uint64_t limit_ns) {
   const uint64_t t0 = global_timer_ns();
   while (true) {
     if (*abort_flag) return false;
     if (mbar_try_wait_sleep(bar, parity, kWaitSleepNs)) return true;
-    if (global_timer_ns() - t0 > kWaitLimitNs) {
+    if (global_timer_ns() - t0 > limit_ns) {
       *abort_flag = 1;
       // where: barrier word index within its 256-word block, and the warp that gave up
       const uint32_t where = (((smem_u32(bar) >> 3) & 0xFFu) << 16) | ((threadIdx.x >> 5) << 24);

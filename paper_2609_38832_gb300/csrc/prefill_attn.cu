@@ -29,14 +29,11 @@
 //               accumulators overlap, so with three S/P buffers the issuer interleaves
 //               PV(kv) (A = P in TMEM, B = V as the MN-major operand) with S(kv+2) = Q K^T
 //               instruction by instruction while the softmax works on S(kv+1).
-//   warps 6-7   (kRopeQ instantiations only) query rotation: the producer loads the raw query
-//               tile, and thread i rotates rows i and i + 64 in shared memory at their ranks (Sec. 3.2, Eq.
-//               namoh-head-rope) with the RoPE pass's own angle and rotation arithmetic, so the
-//               rotated tile is bit for bit the one that pass would have written to HBM.  The next item's tile lands and is rotated while
-//               the current item's last steps run, so the MMA issuer rarely waits for it.
 // TMEM: S/P buffers at cols [0,128), [128,256), [256,384); O at [384, 384 + D).
 // Shared memory (d = 128): Q 32 KB + 6 x 32 KB ring = 224 KB.
 // Every mbarrier wait is bounded (NAMOH_DEV_TIMEOUT, then all roles drain and exit).
+#include <cstddef>
+
 #include "common.cuh"
 #include "plan.cuh"
 
@@ -47,8 +44,7 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache, bool copy_v,
                              const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream,
                              void* plan, int plan_qtiles, const int32_t* plan_cap, const int32_t* pos_row_src,
-                             int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved,
-                             bool keys_only);
+                             int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved);
 
 int launch_sa_select(const CUtensorMap& q_rot_map, const uint16_t* q_rot, const uint16_t* k_cache,
                      const int32_t* seg_offsets, const int64_t* seg_base, const int32_t* seg_cap,
@@ -65,11 +61,7 @@ static_assert(kItemRows == kPlanTileRows, "the plan and the kernel must agree on
 constexpr int kSoftmaxWarps = 4;     // warps 0-3: thread i owns query row i (TMEM lane i)
 constexpr int kWarpLoad = 4;
 constexpr int kWarpMma = 5;
-constexpr int kWarpRope0 = 6;        // warps 6-7: query rotation (kRopeQ instantiations)
-constexpr int kRopeWarps = 2;        // two rows a thread: 256 threads keep the 190-register budget
 constexpr int kThreads = 192;
-// kRopeQ: 0 = the queries come rotated; 1 = rotate them here, half-split pairs; 2 = interleaved pairs
-__host__ __device__ constexpr int threads_for(int rope_q) { return rope_q ? kThreads + 32 * kRopeWarps : kThreads; }
 constexpr int kTmemCols = 512;
 constexpr int kSBufs = 3;            // S/P buffers in TMEM
 // TMEM columns: S/P buffers at 0, 128, 256; O at 384.  P (bf16, two per 32-bit column)
@@ -106,13 +98,13 @@ struct Bars {
                         // do not need and still wait on an exact phase.
   uint64_t o_free;      // epilogue finished reading O
   uint64_t drain;
-  uint64_t q_ready;     // (kRopeQ) the query tile is rotated in shared memory
   int4 item_slot[2];    // {segment * g + j, query tile, seg_offsets[segment], n}
   uint32_t tmem_base;
   int abort_flag;
 };
 
 static_assert(sizeof(Bars) <= 512, "barrier block");
+static_assert(offsetof(Bars, q_full) == 32, "the timeout probe's documented barrier index (word 4)");
 
 struct Params {
   const int32_t* seg_offsets;  // [nseg + 1]
@@ -134,13 +126,18 @@ struct Params {
   const uint32_t* sa_mask;
   int sa_words;
   int sa_lg;
-  RopeTable tab;  // kRopeQ: the RoPE frequencies (the angles are computed as the RoPE pass does)
+  // Test hook of the bounded waits: the MMA issuer's wait limit (kWaitLimitNs normally) and, when
+  // withhold_q is set, the producer never loads a CTA's first query tile, so that the issuer's
+  // wait for it runs out, reports NAMOH_DEV_TIMEOUT and every role drains and exits.
+  uint64_t mma_wait_ns;
+  int withhold_q;
 };
 
 // All lanes of a warp wait and agree on the outcome, so warp-collective tcgen05
 // instructions after the wait never diverge on a timeout race.
-__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, uint32_t* status) {
-  const bool ok = mbar_wait(bar, parity, abort_flag, status);
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, uint32_t* status,
+                                          uint64_t limit_ns = kWaitLimitNs) {
+  const bool ok = mbar_wait(bar, parity, abort_flag, status, limit_ns);
   return __all_sync(0xffffffffu, ok);
 }
 
@@ -285,68 +282,10 @@ __device__ __forceinline__ bool softmax_tile(uint32_t s_addr, uint32_t o_addr, i
   return true;
 }
 
-// Rotates query row `row` of the 128B-swizzled tile at q_smem in place (rank RoPE, Sec. 3.2 Eq.
-// namoh-head-rope) to position `pos`.  Element e of a row sits in 64-column atom e / 64, 16-byte
-// chunk (e % 64) / 8, stored at chunk position chunk ^ (row % 8).  x'_j = x_j cos - x_{j+D/2} sin,
-// x'_{j+D/2} = x_{j+D/2} cos + x_j sin (interleaved: the pair (2j, 2j+1) in one bf16x2 word); the
-// angles, products and roundings are the RoPE pass's, so the tile is bit for bit the q~ that pass
-// would write.
-template <int D, int kRopeQ>
-__device__ __forceinline__ void rotate_query_row(uint8_t* q_smem, int row, float pos, const RopeTable& tab) {
-  constexpr int kAtomBytes = BM * 128;
-  const int sw = row & 7;
-  auto chunk_ptr = [&](int e) -> uint4* {  // the 16-byte chunk holding element e (a multiple of 8)
-    return reinterpret_cast<uint4*>(q_smem + (e >> 6) * kAtomBytes + row * 128 + ((((e & 63) >> 3) ^ sw) << 4));
-  };
-  if constexpr (kRopeQ == 1) {
-    constexpr int HALF = D / 2;
-#pragma unroll
-    for (int c = 0; c < HALF / 8; ++c) {
-      float cs8[8], sn8[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) rope_sincos(pos, tab.theta_hi[8 * c + i], tab.theta_lo[8 * c + i], tab, &sn8[i], &cs8[i]);
-      uint4* pa = chunk_ptr(8 * c);
-      uint4* pb = chunk_ptr(HALF + 8 * c);
-      const uint4 a = *pa, b = *pb;
-      const uint32_t av[4] = {a.x, a.y, a.z, a.w};
-      const uint32_t bv[4] = {b.x, b.y, b.z, b.w};
-      uint32_t oa[4], ob[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const float x0 = bf16_lo(av[q]), x1 = bf16_hi(av[q]);
-        const float y0 = bf16_lo(bv[q]), y1 = bf16_hi(bv[q]);
-        const int i0 = 2 * q, i1 = 2 * q + 1;
-        oa[q] = pack_bf16x2(fmaf(x0, cs8[i0], -y0 * sn8[i0]), fmaf(x1, cs8[i1], -y1 * sn8[i1]));
-        ob[q] = pack_bf16x2(fmaf(y0, cs8[i0], x0 * sn8[i0]), fmaf(y1, cs8[i1], x1 * sn8[i1]));
-      }
-      *pa = make_uint4(oa[0], oa[1], oa[2], oa[3]);
-      *pb = make_uint4(ob[0], ob[1], ob[2], ob[3]);
-    }
-  } else {
-#pragma unroll
-    for (int c = 0; c < D / 8; ++c) {  // chunk c holds pairs j = 4c .. 4c + 3
-      float cs4[4], sn4[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) rope_sincos(pos, tab.theta_hi[4 * c + i], tab.theta_lo[4 * c + i], tab, &sn4[i], &cs4[i]);
-      uint4* pa = chunk_ptr(8 * c);
-      const uint4 a = *pa;
-      const uint32_t w[4] = {a.x, a.y, a.z, a.w};
-      uint32_t o[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const float x0 = bf16_lo(w[q]), x1 = bf16_hi(w[q]);
-        o[q] = pack_bf16x2(fmaf(x0, cs4[q], -x1 * sn4[q]), fmaf(x1, cs4[q], x0 * sn4[q]));
-      }
-      *pa = make_uint4(o[0], o[1], o[2], o[3]);
-    }
-  }
-}
-
-template <int D, bool kSA, int kRopeQ>
-__global__ void __launch_bounds__(threads_for(kRopeQ), 1)
+template <int D, bool kSA>
+__global__ void __launch_bounds__(kThreads, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                     const __grid_constant__ CUtensorMap tm_v, Params p) {
-  static_assert(!(kSA && kRopeQ), "SA + NAMOH selects on rotated queries the RoPE pass wrote");
   using L = Smem<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -360,9 +299,8 @@ __global__ void __launch_bounds__(threads_for(kRopeQ), 1)
   if (threadIdx.x == 0) {
     for (int i = 0; i < 2; ++i) {
       mbar_init(&bars->item_full[i], 1);
-      mbar_init(&bars->item_empty[i], 1 + kSoftmaxWarps + (kRopeQ ? kRopeWarps : 0));
+      mbar_init(&bars->item_empty[i], 1 + kSoftmaxWarps);
     }
-    mbar_init(&bars->q_ready, kRopeWarps);
     for (int i = 0; i < kRing; ++i) {
       mbar_init(&bars->ring_full[i], 1);
       mbar_init(&bars->ring_empty[i], 1);
@@ -437,9 +375,11 @@ __global__ void __launch_bounds__(threads_for(kRopeQ), 1)
         kvb += kv0 * BN;  // the item's first key tile
         if (item_iter > 0) ok = mbar_wait(&bars->q_empty, (item_iter - 1) & 1, abort_flag, p.status);
         if (!ok) break;
-        mbar_arrive_expect_tx(&bars->q_full, L::kTileBytes);
-        for (int a = 0; a < L::kAtoms; ++a)
-          tma_load_2d(smem + L::kQ + a * L::kAtomBytes, &tm_q, j * D + a * 64, off + qt * BM, &bars->q_full);
+        if (!(p.withhold_q && item_iter == 0)) {
+          mbar_arrive_expect_tx(&bars->q_full, L::kTileBytes);
+          for (int a = 0; a < L::kAtoms; ++a)
+            tma_load_2d(smem + L::kQ + a * L::kAtomBytes, &tm_q, j * D + a * 64, off + qt * BM, &bars->q_full);
+        }
         // K(0), K(1), then V(kv), K(kv + 2) for kv = 0, 1, ...
         ok = load_tile(&tm_k, kvb);
         if (ok && nkv > 1) ok = load_tile(&tm_k, kvb + BN);
@@ -510,8 +450,8 @@ __global__ void __launch_bounds__(threads_for(kRopeQ), 1)
       auto rk = [&](int kv) -> uint32_t { return base + 2u * (kv - 2) + 1u; };  // K(kv), kv >= 2
 
       // prologue: S(0) and S(1) interleaved (independent buffers), then PV(0)'s operands
-      ok = warp_wait(kRopeQ ? &bars->q_ready : &bars->q_full, item_iter & 1, abort_flag, p.status) &&
-           ring_ready(rk0) && (nkv == 1 || ring_ready(rk1));
+      ok = warp_wait(&bars->q_full, item_iter & 1, abort_flag, p.status, p.mma_wait_ns) && ring_ready(rk0) &&
+           (nkv == 1 || ring_ready(rk1));
       if (!ok) break;
       tc_fence_after();
       {
@@ -615,26 +555,7 @@ __global__ void __launch_bounds__(threads_for(kRopeQ), 1)
       }
     }
     __syncwarp();
-  } else if (kRopeQ && warp >= kWarpRope0) {
-    // ------------------------------------------------------------------ query rotation
-    const int row = (warp - kWarpRope0) * 32 + lane;  // query rows `row` and `row` + 64 of the tile
-    uint32_t item_iter = 0;
-    bool ok = true;
-    while (ok) {
-      int4 item;
-      ok = take_item(bars, item_iter, &item, abort_flag, p.status);
-      if (!ok || item.x < 0) break;
-      ok = warp_wait(&bars->q_full, item_iter & 1, abort_flag, p.status);
-      if (!ok) break;
-      // ranks of the rows (past the segment's end: rotated but never used)
-      rotate_query_row<D, kRopeQ>(smem + L::kQ, row, (float)(item.y * BM + row), p.tab);
-      rotate_query_row<D, kRopeQ>(smem + L::kQ, row + 64, (float)(item.y * BM + row + 64), p.tab);
-      fence_proxy_async_smem();  // the MMA reads the tile through the async proxy
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->q_ready);
-      ++item_iter;
-    }
-  } else if (warp < kSoftmaxWarps) {
+  } else {
     // ------------------------------------------------------------------ softmax / epilogue
     const int row = warp * 32 + lane;  // query row within the tile (warp w reads TMEM lanes 32w..32w+31)
     const uint32_t lane_addr = (uint32_t)(warp * 32) << 16;
@@ -765,14 +686,13 @@ bool encode_rows_map(CUtensorMap* map, const void* base, long long rows, int row
   return r == CUDA_SUCCESS;
 }
 
-template <int D, bool kSA, int kRopeQ>
+template <int D, bool kSA>
 cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv, const Params& p,
                         int grid, cudaStream_t stream) {
   const int smem = Smem<D>::kAlloc;
-  const auto kernel = attn_fwd_kernel<D, kSA, kRopeQ>;
-  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D, kSA>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  e = launch_pdl(kernel, dim3(grid), dim3(threads_for(kRopeQ)), (size_t)smem, stream, tq, tk, tv, p);
+  e = launch_pdl(attn_fwd_kernel<D, kSA>, dim3(grid), dim3(kThreads), (size_t)smem, stream, tq, tk, tv, p);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
@@ -844,13 +764,11 @@ int launch_plan(const int32_t* seg_offsets, int nseg, int T, int g, const int32_
 // the plan's shared memory is small, else as a second kernel).
 // rope_flags: NAMOH_ROPE_GLOBAL takes the positions from row_src: t = (row_src[r] / Kr) % T,
 // or row_src[r] / Kr - cu_seqlens[b] in a ragged batch (T is then the longest sequence).
-// keys_only: the queries are not rotated here; the attention kernel rotates them (rank positions only).
 int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int Hr, int Kr, int R,
                          int d_head, int group, float rope_base, unsigned rope_flags, const int32_t* cu_seqlens,
                          const int32_t* seg_offsets, const int32_t* row_src, uint16_t* q_rot, uint16_t* k_cache,
                          uint16_t* v_cache, const int64_t* seg_base, const int32_t* seg_cap, long long cache_rows,
-                         uint32_t* dev_status, void* plan, const DeviceInfo& info, cudaStream_t stream,
-                         bool keys_only = false) {
+                         uint32_t* dev_status, void* plan, const DeviceInfo& info, cudaStream_t stream) {
   RopeTable tab;
   fill_rope_table(&tab, d_head, (double)rope_base);
   const int nseg = B * Hr;
@@ -861,7 +779,7 @@ int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v
                                          q_rot, k_cache, v_cache, v_cache != v, tab, dev_status, info.sm_count, stream,
                                          fuse_plan ? plan : nullptr, qtiles, plan_cap,
                                          (rope_flags & NAMOH_ROPE_GLOBAL) ? row_src : nullptr, Kr, T, cu_seqlens,
-                                         Hr, (rope_flags & NAMOH_ROPE_INTERLEAVED) != 0, keys_only);
+                                         Hr, (rope_flags & NAMOH_ROPE_INTERLEAVED) != 0);
   if (e != cudaSuccess) return cuda_fail(e, "rope_pack_kernel launch");
   if (plan && !fuse_plan) return launch_plan(seg_offsets, nseg, T, group, plan_cap, plan, stream);
   return NAMOH_OK;
@@ -871,10 +789,8 @@ int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint1
                      int g, const int32_t* seg_offsets, const int32_t* row_src, const float* gate,
                      const int64_t* seg_base, long long cache_rows, void* plan, uint16_t* y, uint32_t* dev_status,
                      const DeviceInfo& info, cudaStream_t stream, int window = 0,
-                     const uint32_t* sa_mask = nullptr, int sa_words = 0, int sa_lg = 0, int rope_q = 0,
-                     float rope_base = 0.f) {
-  // rope_q > 0: q_rot holds the raw queries, rotated in the kernel at their ranks with rope_base
-  // (1 half-split, 2 interleaved)
+                     const uint32_t* sa_mask = nullptr, int sa_words = 0, int sa_lg = 0,
+                     uint64_t mma_wait_ns = kWaitLimitNs, bool withhold_q = false) {
   CUtensorMap tq, tk, tv;
   if (!attn::encode_rows_map(&tq, q_rot, R, g * D) || !attn::encode_rows_map(&tk, k_cache, cache_rows, D) ||
       !attn::encode_rows_map(&tv, v_cache, cache_rows, D))
@@ -897,21 +813,15 @@ int launch_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint1
   p.sa_mask = sa_mask;
   p.sa_words = sa_words;
   p.sa_lg = sa_lg;
-  if (rope_q) fill_rope_table(&p.tab, D, (double)rope_base);
+  p.mma_wait_ns = mma_wait_ns;
+  p.withhold_q = withhold_q ? 1 : 0;
   cudaError_t e;
-  const int G = info.sm_count;
   if (sa_mask)
-    e = (D == 128) ? attn::launch_attn<128, true, 0>(tq, tk, tv, p, G, stream)
-                   : attn::launch_attn<64, true, 0>(tq, tk, tv, p, G, stream);
-  else if (rope_q == 1)
-    e = (D == 128) ? attn::launch_attn<128, false, 1>(tq, tk, tv, p, G, stream)
-                   : attn::launch_attn<64, false, 1>(tq, tk, tv, p, G, stream);
-  else if (rope_q == 2)
-    e = (D == 128) ? attn::launch_attn<128, false, 2>(tq, tk, tv, p, G, stream)
-                   : attn::launch_attn<64, false, 2>(tq, tk, tv, p, G, stream);
+    e = (D == 128) ? attn::launch_attn<128, true>(tq, tk, tv, p, info.sm_count, stream)
+                   : attn::launch_attn<64, true>(tq, tk, tv, p, info.sm_count, stream);
   else
-    e = (D == 128) ? attn::launch_attn<128, false, 0>(tq, tk, tv, p, G, stream)
-                   : attn::launch_attn<64, false, 0>(tq, tk, tv, p, G, stream);
+    e = (D == 128) ? attn::launch_attn<128, false>(tq, tk, tv, p, info.sm_count, stream)
+                   : attn::launch_attn<64, false>(tq, tk, tv, p, info.sm_count, stream);
   return e == cudaSuccess ? NAMOH_OK : cuda_fail(e, "attn_fwd_kernel launch");
 }
 
@@ -1008,6 +918,28 @@ extern "C" int namoh_attention(const uint16_t* q_rot, const uint16_t* k_cache, c
                           plan, y, dev_status, info, reinterpret_cast<cudaStream_t>(stream_v));
 }
 
+extern "C" int namoh_attention_timeout_probe(const uint16_t* q_rot, const uint16_t* k_cache, const uint16_t* v_cache,
+                                             int B, int T, int H, int K, int d_head, int group,
+                                             const int32_t* seg_offsets, const int32_t* row_src, const float* gate,
+                                             void* plan, size_t plan_bytes, uint16_t* y, uint64_t wait_limit_ns,
+                                             uint32_t* dev_status, void* stream_v) {
+  if (!q_rot || !k_cache || !v_cache || !seg_offsets || !row_src || !gate || !y || !dev_status)
+    return NAMOH_ERR_INVALID_ARG;
+  if (wait_limit_ns < 1000ull || wait_limit_ns > kWaitLimitNs) return NAMOH_ERR_INVALID_ARG;
+  int Hr, Kr;
+  long long R;
+  const int st = check_shape(B, T, H, K, d_head, group, &Hr, &Kr, &R);
+  if (st != NAMOH_OK) return st;
+  if (!aligned16(q_rot) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(y)) return NAMOH_ERR_INVALID_ARG;
+  if (!plan || (reinterpret_cast<uintptr_t>(plan) & 15u) || plan_bytes < plan_bytes_for(B, T, Hr, Kr, group))
+    return NAMOH_ERR_WORKSPACE;
+  DeviceInfo info;
+  if (!device_ok(&info)) return NAMOH_ERR_UNSUPPORTED;
+  return launch_attention(q_rot, k_cache, v_cache, R, d_head, group, seg_offsets, row_src, gate, nullptr, R, plan, y,
+                          dev_status, info, reinterpret_cast<cudaStream_t>(stream_v), 0, nullptr, 0, 0,
+                          wait_limit_ns, true);
+}
+
 namespace namoh {
 namespace {
 // Shared body of namoh_prefill_ex and namoh_prefill_varlen: R packed rows in B*Hr segments
@@ -1037,22 +969,20 @@ int prefill_impl(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B,
   DeviceInfo info;
   if (!device_ok(&info)) return NAMOH_ERR_UNSUPPORTED;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
-  // rank positions: the attention kernel rotates the queries itself (no Q~ round trip through HBM)
-  const bool fuse_q = !(rope_flags & NAMOH_ROPE_GLOBAL);
+
   int st = launch_rope_and_plan(q, k, v, B, T, Hr, Kr, (int)R, d_head, group, rope_base, rope_flags, cu_seqlens,
                                 seg_offsets, row_src, q_rot, k_cache, v_cache, seg_base, seg_cap, cache_rows,
-                                dev_status, plan, info, stream, fuse_q);
+                                dev_status, plan, info, stream);
   if (st != NAMOH_OK) return st;
   if (seg_len) {
     seg_len_kernel<<<(B * Hr + 255) / 256, 256, 0, stream>>>(seg_offsets, B * Hr, seg_len);
     if (const int st2 = cuda_check_launch("seg_len_kernel launch")) return st2;
   }
-  const int rope_q = fuse_q ? ((rope_flags & NAMOH_ROPE_INTERLEAVED) ? 2 : 1) : 0;
-  return launch_attention(fuse_q ? q : q_rot, k_cache, v_cache, R, d_head, group, seg_offsets, row_src, gate, seg_base,
-                          cache_rows, plan, y, dev_status, info, stream, 0, nullptr, 0, 0, rope_q, rope_base);
+  return launch_attention(q_rot, k_cache, v_cache, R, d_head, group, seg_offsets, row_src, gate, seg_base, cache_rows,
+                          plan, y, dev_status, info, stream);
 }
 
-size_t prefill_workspace_rows(long long R, int nseg, int T, int d_head, int group) {
+size_t prefill_workspace_rows(long long R, int nseg, int d_head, int group) {
   WorkspaceCarver ws{nullptr, 0, 0};
   ws.take<uint16_t>((size_t)R * group * d_head);
   ws.take<char>(plan_bytes_rows(R, nseg, group));
@@ -1072,7 +1002,7 @@ extern "C" size_t namoh_prefill_workspace_size(int B, int T, int H, int K, int d
   int Hr, Kr;
   long long R;
   if (check_shape(B, T, H, K, d_head, group, &Hr, &Kr, &R) != NAMOH_OK) return 0;
-  return prefill_workspace_rows(R, B * Hr, T, d_head, group);
+  return prefill_workspace_rows(R, B * Hr, d_head, group);
 }
 
 extern "C" int namoh_prefill_ex(const uint16_t* q, const uint16_t* k, const uint16_t* v, int B, int T, int H, int K,
@@ -1095,7 +1025,7 @@ extern "C" size_t namoh_prefill_varlen_workspace_size(int B, int total_tokens, i
   int Hr, Kr;
   long long R;
   if (check_varlen(B, total_tokens, max_seqlen, H, K, d_head, group, &Hr, &Kr, &R) != NAMOH_OK) return 0;
-  return prefill_workspace_rows(R, B * Hr, max_seqlen, d_head, group);
+  return prefill_workspace_rows(R, B * Hr, d_head, group);
 }
 
 extern "C" int namoh_prefill_varlen(const uint16_t* q, const uint16_t* k, const uint16_t* v,
@@ -1242,13 +1172,15 @@ __global__ void shared_layout_kernel(int B, int T, int Hs, int32_t* __restrict__
 struct SharedWs {
   int32_t *seg_offsets, *row_src;
   float* gate;
-  void* plan;  // (the attention kernel rotates the queries: the rank in these segments is t)
+  uint16_t* q_rot;
+  void* plan;
 };
 void carve_shared(WorkspaceCarver& ws, SharedWs* o, int B, int T, int Hs, int d_head) {
   const long long R = (long long)B * Hs * T;
   o->seg_offsets = ws.take<int32_t>((size_t)B * Hs + 1);
   o->row_src = ws.take<int32_t>((size_t)R);
   o->gate = ws.take<float>((size_t)R);
+  o->q_rot = ws.take<uint16_t>((size_t)R * d_head);
   o->plan = ws.take<char>(plan_bytes_rows(R, B * Hs, 1));
 }
 }  // namespace
@@ -1295,15 +1227,14 @@ extern "C" int namoh_shared_prefill(const uint16_t* q, const uint16_t* k, const 
   shared_layout_kernel<<<info.sm_count * 4, 256, 0, stream>>>(B, T, Hs, o.seg_offsets, o.row_src, o.gate);
   if (const int e = cuda_check_launch("shared_layout_kernel launch")) return e;
   // global positions: the rank in a segment holding every token is t (the global flag is redundant)
-  const bool il = (rope_flags & NAMOH_ROPE_INTERLEAVED) != 0;
-  st = launch_rope_and_plan(q, k, v, B, T, Hs, Hs, (int)R, d_head, 1, rope_base, il ? NAMOH_ROPE_INTERLEAVED : 0u,
-                            nullptr, o.seg_offsets, o.row_src, nullptr, k_cache, v_cache, seg_base, seg_cap,
-                            cache_rows, dev_status, o.plan, info, stream, true);
+  st = launch_rope_and_plan(q, k, v, B, T, Hs, Hs, (int)R, d_head, 1, rope_base, rope_flags & NAMOH_ROPE_INTERLEAVED,
+                            nullptr, o.seg_offsets, o.row_src, o.q_rot, k_cache, v_cache, seg_base, seg_cap,
+                            cache_rows, dev_status, o.plan, info, stream);
   if (st != NAMOH_OK) return st;
   if (seg_len) {
     seg_len_kernel<<<(B * Hs + 255) / 256, 256, 0, stream>>>(o.seg_offsets, B * Hs, seg_len);
     if (const int e = cuda_check_launch("seg_len_kernel launch")) return e;
   }
-  return launch_attention(q, k_cache, v_cache, R, d_head, 1, o.seg_offsets, o.row_src, o.gate, seg_base,
-                          cache_rows, o.plan, y, dev_status, info, stream, window, nullptr, 0, 0, il ? 2 : 1, rope_base);
+  return launch_attention(o.q_rot, k_cache, v_cache, R, d_head, 1, o.seg_offsets, o.row_src, o.gate, seg_base,
+                          cache_rows, o.plan, y, dev_status, info, stream, window);
 }

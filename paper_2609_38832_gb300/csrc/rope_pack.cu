@@ -29,22 +29,19 @@ namespace namoh {
 
 constexpr int kRopeThreads = 256;
 constexpr int kRopeStages = 3;
-// keys-only passes move half the bytes per chunk, so they keep twice the chunks in flight
-__host__ __device__ constexpr int rope_stages(bool no_q) { return no_q ? 2 * kRopeStages : kRopeStages; }
 constexpr int kRopeStageMax = 8192;  // seg_offsets entries staged in shared memory (32 KB)
 constexpr size_t kSmemPerSm = 233472;  // shared memory per SM (228 KB); each resident block also takes 1 KB
 // the least dynamic shared memory with which three blocks no longer fit on one SM
 constexpr size_t kSmemThirdPlus = kSmemPerSm / 3 - 1024 + 16;
 
-// kNoQ: only K (and V) pass through; the queries are rotated by the attention kernel itself.
-template <int D, int G, bool kNoQ = false>
+template <int D, int G>
 struct RopeChunk {
   static constexpr int kLpr = D / 16;                    // threads per group (8 pairs each)
   static constexpr int kGroups = kRopeThreads / kLpr;    // 32 (D = 128) or 64 (D = 64)
   static constexpr int kGpr = G >= 4 ? G / 2 : 1;        // groups per packed row
   static constexpr int kHeads = G / kGpr;                // query heads per group
   static constexpr int kRows = kGroups / kGpr;           // packed rows per chunk
-  static constexpr int kQBytes = kNoQ ? 0 : kRows * G * D * 2;
+  static constexpr int kQBytes = kRows * G * D * 2;
   static constexpr int kKBytes = kRows * D * 2;
   static constexpr int kStageBytes = kQBytes + 2 * kKBytes;  // Q, K, V
   static_assert(kStageBytes % 128 == 0, "stage alignment");
@@ -54,17 +51,14 @@ __host__ __device__ constexpr size_t rope_offs_bytes(int nseg) {
   return nseg + 1 <= kRopeStageMax ? ((size_t)(nseg + 1) * 4 + 15) / 16 * 16 : 0;
 }
 
-template <int D, int G, bool kNoQ = false>
+template <int D, int G>
 __host__ __device__ constexpr size_t rope_smem_bytes(int nseg) {
-  return (size_t)rope_stages(kNoQ) * RopeChunk<D, G, kNoQ>::kStageBytes + rope_offs_bytes(nseg) +
-         rope_stages(kNoQ) * sizeof(uint64_t);
+  return (size_t)kRopeStages * RopeChunk<D, G>::kStageBytes + rope_offs_bytes(nseg) + kRopeStages * sizeof(uint64_t);
 }
 
-// kFlags: NAMOH_ROPE_INTERLEAVED, NAMOH_ROPE_GLOBAL, kRopeRagged (global positions in a ragged
-// batch) and kRopeNoQ (keys and values only: the attention kernel rotates the queries itself),
-// compile-time so that no variant carries another's branches
+// kFlags: NAMOH_ROPE_INTERLEAVED, NAMOH_ROPE_GLOBAL and kRopeRagged (global positions in a
+// ragged batch), compile-time so that no variant carries another's branches
 constexpr unsigned kRopeRagged = 0x4u;
-constexpr unsigned kRopeNoQ = 0x8u;
 
 template <int D, int G, unsigned kFlags>
 __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
@@ -74,30 +68,26 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     uint16_t* __restrict__ k_cache, uint16_t* __restrict__ v_cache, int copy_v, RopeTable tab,
     uint32_t* __restrict__ status, int* __restrict__ plan_header, int4* __restrict__ plan_items,
     const int32_t* __restrict__ plan_cap, int plan_qtiles, const int32_t* __restrict__ pos_row_src,
-    FastDiv pos_k, FastDiv pos_t, const int32_t* __restrict__ pos_cu, FastDiv pos_hr, int plan_g) {
-  constexpr bool kNoQ = (kFlags & kRopeNoQ) != 0;
-  constexpr int kStages = rope_stages(kNoQ);
-  using C = RopeChunk<D, G, kNoQ>;
+    FastDiv pos_k, FastDiv pos_t, const int32_t* __restrict__ pos_cu, FastDiv pos_hr) {
+  using C = RopeChunk<D, G>;
   constexpr int HALF = D / 2;
   constexpr bool kInterleaved = (kFlags & NAMOH_ROPE_INTERLEAVED) != 0;
   constexpr bool kGlobal = (kFlags & NAMOH_ROPE_GLOBAL) != 0;
   constexpr bool kRagged = (kFlags & kRopeRagged) != 0;
-  static_assert(!kNoQ || (G == 1 && !kGlobal), "keys-only passes use the rank and the one-row layout");
   extern __shared__ __align__(128) uint8_t smem_raw[];
   __shared__ int s_abort;
   pdl_launch_dependents();  // the attention kernel may start launching; it waits for this grid
   const int first = plan_header ? 1 : 0;
   if ((int)blockIdx.x < first) {
     pdl_wait();
-    build_plan(seg_offsets, nseg, plan_cap, plan_g, plan_qtiles, plan_header, plan_items,
-               reinterpret_cast<int*>(smem_raw));
+    build_plan(seg_offsets, nseg, plan_cap, G, plan_qtiles, plan_header, plan_items, reinterpret_cast<int*>(smem_raw));
     return;
   }
   const int nblk = gridDim.x - first, blk = blockIdx.x - first;
   const int nchunks = (R + C::kRows - 1) / C::kRows;
   uint8_t* stages = smem_raw;
-  int32_t* s_offs = reinterpret_cast<int32_t*>(smem_raw + kStages * C::kStageBytes);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + kStages * C::kStageBytes + rope_offs_bytes(nseg));
+  int32_t* s_offs = reinterpret_cast<int32_t*>(smem_raw + kRopeStages * C::kStageBytes);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + kRopeStages * C::kStageBytes + rope_offs_bytes(nseg));
   const bool staged = nseg + 1 <= kRopeStageMax;
 
   // chunk c into stage st: its rows' Q (g rows each), K and V, one bulk copy per array
@@ -105,20 +95,20 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     const int r0 = c * C::kRows;
     const int rows = min(C::kRows, R - r0);
     uint8_t* base = stages + st * C::kStageBytes;
-    const uint32_t qb = kNoQ ? 0u : (uint32_t)rows * G * D * 2, kb = (uint32_t)rows * D * 2;
+    const uint32_t qb = (uint32_t)rows * G * D * 2, kb = (uint32_t)rows * D * 2;
     mbar_arrive_expect_tx(&full[st], qb + kb + (copy_v ? kb : 0u));
-    if (!kNoQ) bulk_load(base, q + (size_t)r0 * G * D, qb, &full[st]);
+    bulk_load(base, q + (size_t)r0 * G * D, qb, &full[st]);
     bulk_load(base + C::kQBytes, k + (size_t)r0 * D, kb, &full[st]);
     if (copy_v) bulk_load(base + C::kQBytes + C::kKBytes, v + (size_t)r0 * D, kb, &full[st]);
   };
   if (threadIdx.x == 0) {
-    for (int i = 0; i < kStages; ++i) mbar_init(&full[i], 1);
+    for (int i = 0; i < kRopeStages; ++i) mbar_init(&full[i], 1);
     s_abort = 0;
     mbar_fence_init();
   }
   pdl_wait();  // routing outputs (and q, k, v) are visible from here
   if (threadIdx.x == 0)
-    for (int i = 0; i < kStages; ++i)
+    for (int i = 0; i < kRopeStages; ++i)
       if (blk + i * nblk < nchunks) issue(blk + i * nblk, i);
   if (staged)
     for (int i = threadIdx.x; i <= nseg; i += blockDim.x) s_offs[i] = __ldg(seg_offsets + i);
@@ -145,14 +135,14 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     if (blk < nchunks && r_first < R) token_next = __ldg(pos_row_src + r_first);
   }
   for (int c = blk; c < nchunks; c += nblk, ++it) {
-    const int st = it % kStages;
+    const int st = it % kRopeStages;
     int token_src = 0;  // row_src of this thread's row: (b*T + t)*Kr + slot
     if (kGlobal) {
       token_src = token_next;
       const long long r_next = (long long)(c + nblk) * C::kRows + prow;
       if (c + nblk < nchunks && r_next < R) token_next = __ldg(pos_row_src + r_next);
     }
-    ok = mbar_wait(&full[st], (it / kStages) & 1, &s_abort, status);
+    ok = mbar_wait(&full[st], (it / kRopeStages) & 1, &s_abort, status);
     if (!__syncthreads_and(ok)) {
       ok = false;
       break;
@@ -213,12 +203,10 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
           *reinterpret_cast<uint4*>(dst_row + HALF + j0) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
         }
       };
-      if (!kNoQ) {
 #pragma unroll
-        for (int h = 0; h < C::kHeads; ++h) {
-          const int head = hsub * C::kHeads + h;
-          rotate(base + ((size_t)prow * G + head) * D * 2, q_rot + ((size_t)r * G + head) * D);
-        }
+      for (int h = 0; h < C::kHeads; ++h) {
+        const int head = hsub * C::kHeads + h;
+        rotate(base + ((size_t)prow * G + head) * D * 2, q_rot + ((size_t)r * G + head) * D);
       }
       if (hsub == 0) {
         long long dst = r;
@@ -242,7 +230,7 @@ __global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
       }
     }
     __syncthreads();  // stage st fully read: refill it
-    if (threadIdx.x == 0 && c + kStages * nblk < nchunks) issue(c + kStages * nblk, st);
+    if (threadIdx.x == 0 && c + kRopeStages * nblk < nchunks) issue(c + kRopeStages * nblk, st);
   }
   if (!ok && threadIdx.x == 0) {
     // a wait gave up: let bulk copies still in flight land before the block exits
@@ -261,16 +249,12 @@ cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, 
                                int4* plan_items, const int32_t* plan_cap, int plan_qtiles,
                                const int32_t* pos_row_src, FastDiv pos_k, FastDiv pos_t, const int32_t* pos_cu,
                                FastDiv pos_hr) {
-  constexpr bool kNoQ = (F & kRopeNoQ) != 0;
-  const int plan_g = g;
-  if (kNoQ) g = 1;  // keys only: one key row per packed row whatever the group size
   switch (g) {
 #define NAMOH_ROPE_CASE(GG)                                                                                       \
   case GG: {                                                                                                      \
-    constexpr int GE = kNoQ ? 1 : GG;                                                                            \
-    using C = RopeChunk<D, GE, kNoQ>;                                                                            \
-    const auto kernel = rope_pack_kernel<D, GE, F>;                                                              \
-    const size_t rope_smem = rope_smem_bytes<D, GE, kNoQ>(nseg);                                                 \
+    using C = RopeChunk<D, GG>;                                                                                  \
+    const auto kernel = rope_pack_kernel<D, GG, F>;                                                              \
+    const size_t rope_smem = rope_smem_bytes<D, GG>(nseg);                                                       \
     const size_t smem0 = rope_smem > plan_smem ? rope_smem : plan_smem;                                          \
     /* two blocks per SM when their shared memory fits (228 KB per SM, 1 KB reserved per block); the */          \
     /* block scheduler packs blocks as deep as resources allow, so each block also asks for more than */          \
@@ -290,8 +274,7 @@ cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, 
     }                                                                                                            \
     return launch_pdl(kernel, dim3((unsigned)grid), dim3(kRopeThreads), smem, stream, q, k, v, R, seg_offsets,     \
                       nseg, seg_base, seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v, tab, status,         \
-                      plan_header, plan_items, plan_cap, plan_qtiles, pos_row_src, pos_k, pos_t, pos_cu, pos_hr,  \
-                      plan_g);                                                                                   \
+                      plan_header, plan_items, plan_cap, plan_qtiles, pos_row_src, pos_k, pos_t, pos_cu, pos_hr); \
   }
     NAMOH_ROPE_CASE(1)
     NAMOH_ROPE_CASE(2)
@@ -309,16 +292,13 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache, bool copy_v,
                              const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream,
                              void* plan, int plan_qtiles, const int32_t* plan_cap, const int32_t* pos_row_src,
-                             int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved,
-                             bool keys_only) {
+                             int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved) {
   int* plan_header = static_cast<int*>(plan);
   int4* plan_items = plan ? reinterpret_cast<int4*>(static_cast<char*>(plan) + 16) : nullptr;
   const size_t plan_smem = plan ? (size_t)plan_smem_ints(plan_qtiles, nseg) * sizeof(int) : 0;
   if (R == 0 && !plan) return cudaSuccess;
-  // keys only: the queries are left to the attention kernel (rank positions only)
-  if (keys_only && pos_row_src) return cudaErrorInvalidValue;
   const unsigned flags = (interleaved ? NAMOH_ROPE_INTERLEAVED : 0u) | (pos_row_src ? NAMOH_ROPE_GLOBAL : 0u) |
-                         (pos_row_src && pos_cu ? kRopeRagged : 0u) | (keys_only ? kRopeNoQ : 0u);
+                         (pos_row_src && pos_cu ? kRopeRagged : 0u);
   auto go = [&](auto d_tag, auto f_tag) {
     return launch_rope_pack_d<decltype(d_tag)::value, decltype(f_tag)::value>(
         g, sm_count, nseg, plan_smem, plan != nullptr, stream, q, k, v, R, seg_offsets, seg_base, seg_cap, cache_rows,
@@ -334,11 +314,7 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
   using F3 = std::integral_constant<unsigned, 3u>;
   using F6 = std::integral_constant<unsigned, 6u>;
   using F7 = std::integral_constant<unsigned, 7u>;
-  using F8 = std::integral_constant<unsigned, 8u>;
-  using F9 = std::integral_constant<unsigned, 9u>;
   switch (flags) {
-    case 8u: return D == 128 ? go(D128{}, F8{}) : go(D64{}, F8{});
-    case 9u: return D == 128 ? go(D128{}, F9{}) : go(D64{}, F9{});
     case 0u: return D == 128 ? go(D128{}, F0{}) : go(D64{}, F0{});
     case 1u: return D == 128 ? go(D128{}, F1{}) : go(D64{}, F1{});
     case 2u: return D == 128 ? go(D128{}, F2{}) : go(D64{}, F2{});
