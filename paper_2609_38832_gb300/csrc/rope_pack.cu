@@ -27,9 +27,8 @@
 
 namespace namoh {
 
-constexpr int kRopeThreads = 256;                    // rotation threads (8 warps)
-constexpr int kRopeBlock = kRopeThreads + 32;        // plus one producer warp
-constexpr int kRopeStages = 4;
+constexpr int kRopeThreads = 256;
+constexpr int kRopeStages = 3;
 constexpr int kRopeStageMax = 8192;  // seg_offsets entries staged in shared memory (32 KB)
 constexpr size_t kSmemPerSm = 233472;  // shared memory per SM (228 KB); each resident block also takes 1 KB
 // the least dynamic shared memory with which three blocks no longer fit on one SM
@@ -54,8 +53,7 @@ __host__ __device__ constexpr size_t rope_offs_bytes(int nseg) {
 
 template <int D, int G>
 __host__ __device__ constexpr size_t rope_smem_bytes(int nseg) {
-  return (size_t)kRopeStages * RopeChunk<D, G>::kStageBytes + rope_offs_bytes(nseg) +
-         2 * kRopeStages * sizeof(uint64_t);
+  return (size_t)kRopeStages * RopeChunk<D, G>::kStageBytes + rope_offs_bytes(nseg) + kRopeStages * sizeof(uint64_t);
 }
 
 // kFlags: NAMOH_ROPE_INTERLEAVED, NAMOH_ROPE_GLOBAL and kRopeRagged (global positions in a
@@ -63,7 +61,7 @@ __host__ __device__ constexpr size_t rope_smem_bytes(int nseg) {
 constexpr unsigned kRopeRagged = 0x4u;
 
 template <int D, int G, unsigned kFlags>
-__global__ void __launch_bounds__(kRopeBlock) rope_pack_kernel(
+__global__ void __launch_bounds__(kRopeThreads) rope_pack_kernel(
     const uint16_t* __restrict__ q, const uint16_t* __restrict__ k, const uint16_t* __restrict__ v, int R,
     const int32_t* __restrict__ seg_offsets, int nseg, const int64_t* __restrict__ seg_base,
     const int32_t* __restrict__ seg_cap, long long cache_rows, uint16_t* __restrict__ q_rot,
@@ -90,7 +88,6 @@ __global__ void __launch_bounds__(kRopeBlock) rope_pack_kernel(
   uint8_t* stages = smem_raw;
   int32_t* s_offs = reinterpret_cast<int32_t*>(smem_raw + kRopeStages * C::kStageBytes);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + kRopeStages * C::kStageBytes + rope_offs_bytes(nseg));
-  uint64_t* empty = full + kRopeStages;  // the rotation warps are done reading a stage
   const bool staged = nseg + 1 <= kRopeStageMax;
 
   // chunk c into stage st: its rows' Q (g rows each), K and V, one bulk copy per array
@@ -105,38 +102,18 @@ __global__ void __launch_bounds__(kRopeBlock) rope_pack_kernel(
     if (copy_v) bulk_load(base + C::kQBytes + C::kKBytes, v + (size_t)r0 * D, kb, &full[st]);
   };
   if (threadIdx.x == 0) {
-    for (int i = 0; i < kRopeStages; ++i) {
-      mbar_init(&full[i], 1);
-      mbar_init(&empty[i], kRopeThreads / 32);
-    }
+    for (int i = 0; i < kRopeStages; ++i) mbar_init(&full[i], 1);
     s_abort = 0;
     mbar_fence_init();
   }
   pdl_wait();  // routing outputs (and q, k, v) are visible from here
-  const bool producer = threadIdx.x >= kRopeThreads;
+  if (threadIdx.x == 0)
+    for (int i = 0; i < kRopeStages; ++i)
+      if (blk + i * nblk < nchunks) issue(blk + i * nblk, i);
   if (staged)
     for (int i = threadIdx.x; i <= nseg; i += blockDim.x) s_offs[i] = __ldg(seg_offsets + i);
-  __syncthreads();  // the last block-wide barrier: from here the warps run decoupled
+  __syncthreads();
   const int32_t* offs = staged ? s_offs : seg_offsets;
-  if (producer) {
-    // refill each stage once all eight rotation warps have read it
-    bool pok = true;
-    if (threadIdx.x == kRopeThreads) {
-      int i = 0;
-      for (int c = blk; c < nchunks && pok; c += nblk, ++i) {
-        const int st = i % kRopeStages;
-        if (i >= kRopeStages) pok = mbar_wait(&empty[st], ((i / kRopeStages) - 1) & 1, &s_abort, status);
-        if (pok) issue(c, st);
-      }
-      if (!pok) {
-        // a wait gave up: let bulk copies still in flight land before the block exits
-        const uint64_t t0 = global_timer_ns();
-        while (global_timer_ns() - t0 < 1000000ull) {
-        }
-      }
-    }
-    return;
-  }
 
   const int grp = threadIdx.x / C::kLpr, lig = threadIdx.x % C::kLpr;
   const int prow = grp / C::kGpr;  // packed row within the chunk
@@ -165,8 +142,11 @@ __global__ void __launch_bounds__(kRopeBlock) rope_pack_kernel(
       const long long r_next = (long long)(c + nblk) * C::kRows + prow;
       if (c + nblk < nchunks && r_next < R) token_next = __ldg(pos_row_src + r_next);
     }
-    ok = __all_sync(0xffffffffu, mbar_wait(&full[st], (it / kRopeStages) & 1, &s_abort, status));
-    if (!ok) break;
+    ok = mbar_wait(&full[st], (it / kRopeStages) & 1, &s_abort, status);
+    if (!__syncthreads_and(ok)) {
+      ok = false;
+      break;
+    }
     const uint8_t* base = stages + st * C::kStageBytes;
     const long long r = (long long)c * C::kRows + prow;
     if (r < R) {
@@ -249,8 +229,8 @@ __global__ void __launch_bounds__(kRopeBlock) rope_pack_kernel(
         }
       }
     }
-    __syncwarp();  // this warp's reads of stage st are done
-    if ((threadIdx.x & 31) == 0) mbar_arrive(&empty[st]);
+    __syncthreads();  // stage st fully read: refill it
+    if (threadIdx.x == 0 && c + kRopeStages * nblk < nchunks) issue(c + kRopeStages * nblk, st);
   }
   if (!ok && threadIdx.x == 0) {
     // a wait gave up: let bulk copies still in flight land before the block exits
@@ -292,7 +272,7 @@ cudaError_t launch_rope_pack_d(int g, int sm_count, int nseg, size_t plan_smem, 
                                            (int)smem);                                                           \
       if (e != cudaSuccess) return e;                                                                            \
     }                                                                                                            \
-    return launch_pdl(kernel, dim3((unsigned)grid), dim3(kRopeBlock), smem, stream, q, k, v, R, seg_offsets,       \
+    return launch_pdl(kernel, dim3((unsigned)grid), dim3(kRopeThreads), smem, stream, q, k, v, R, seg_offsets,     \
                       nseg, seg_base, seg_cap, cache_rows, q_rot, k_cache, v_cache, copy_v, tab, status,         \
                       plan_header, plan_items, plan_cap, plan_qtiles, pos_row_src, pos_k, pos_t, pos_cu, pos_hr); \
   }
