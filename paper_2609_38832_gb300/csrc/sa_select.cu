@@ -128,7 +128,7 @@ struct SelParams {
   uint32_t* mask;      // [(row * g + j), words]
   uint32_t* status;
   int g, lg, alpha_num, alpha_den, words;
-  int kb_rows;         // pooled-key rows staged per CTA (multiple of kKbBox, <= kSelMaxCols)
+  int kb_rows;         // pooled-key rows of the streaming buffer (kKbBox)
 };
 
 // Row of block scores of this thread, 32 columns (blocks 32 c .. 32 c + 31) at a time.
@@ -192,39 +192,39 @@ __global__ void __launch_bounds__(kSelThreads) sa_select_tc_kernel(const __grid_
   const uint32_t tmem = tmem_base;
   bool ok = true;
   if (warp == 0) {
-    const int kb_boxes = (ncols + kKbBox - 1) / kKbBox;
-    if (lane == 0) {
-      const int kbase = (off >> p.lg) + s;  // first pooled-key row of the segment
-      mbar_arrive_expect_tx(&bar_load, (uint32_t)(kAtoms * (kQAtomBytes + kb_boxes * kKbBox * 128)));
-      for (int a = 0; a < kAtoms; ++a) {
-        tma_load_2d(sq + a * kQAtomBytes, &tm_q, j * D + a * 64, off + row0, &bar_load);
-        for (int bx = 0; bx < kb_boxes; ++bx)
-          tma_load_2d(skb + a * kb_atom_bytes + bx * kKbBox * 128, &tm_kb, a * 64, kbase + bx * kKbBox, &bar_load);
-      }
-    }
-    __syncwarp();
-    ok = __all_sync(0xffffffffu, mbar_wait(&bar_load, 0, &abort_flag, p.status));
-    if (ok) {
-      tc_fence_after();
-      const uint64_t q_desc = make_smem_desc_sw128(smem_u32(sq), 16, 1024);
-      // K steps of 16 elements: 32 bytes within the 128-byte atom, then the next atom
-      for (int n0 = 0; n0 < ncols; n0 += 256) {
-        const int N = min(256, ncols - n0);
-        const uint32_t idesc = make_idesc_bf16(kSelTileRows, N, false, false);
-        const uint64_t kb_desc = make_smem_desc_sw128(smem_u32(skb + n0 * 128), 16, 1024);
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint64_t qo = (uint64_t)(((kk >> 2) * kQAtomBytes + (kk & 3) * 32) >> 4);
-          const uint64_t ko = (uint64_t)(((kk >> 2) * kb_atom_bytes + (kk & 3) * 32) >> 4);
-          mma_bf16_ss(tmem + (uint32_t)n0, q_desc + qo, kb_desc + ko, idesc, kk > 0 ? 1u : 0u);
+    // The pooled keys stream through one buffer of kKbBox rows: load a box of blocks, issue its
+    // MMAs into the next kKbBox score columns, wait for them, then reuse the buffer.
+    const int kbase = (off >> p.lg) + s;  // first pooled-key row of the segment
+    const uint64_t q_desc = make_smem_desc_sw128(smem_u32(sq), 16, 1024);
+    const uint64_t kb_desc = make_smem_desc_sw128(smem_u32(skb), 16, 1024);
+    uint32_t phase = 0;
+    for (int n0 = 0; n0 < ncols && ok; n0 += kKbBox, ++phase) {
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&bar_load, (uint32_t)(kAtoms * ((n0 == 0 ? kQAtomBytes : 0) + kKbBox * 128)));
+        for (int a = 0; a < kAtoms; ++a) {
+          if (n0 == 0) tma_load_2d(sq + a * kQAtomBytes, &tm_q, j * D + a * 64, off + row0, &bar_load);
+          tma_load_2d(skb + a * kb_atom_bytes, &tm_kb, a * 64, kbase + n0, &bar_load);
         }
       }
+      __syncwarp();
+      ok = __all_sync(0xffffffffu, mbar_wait(&bar_load, phase & 1, &abort_flag, p.status));
+      if (!ok) break;
+      tc_fence_after();
+      const int N = min(kKbBox, ncols - n0);  // a multiple of 16
+      const uint32_t idesc = make_idesc_bf16(kSelTileRows, N, false, false);
+      // K steps of 16 elements: 32 bytes within the 128-byte atom, then the next atom
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const uint64_t qo = (uint64_t)(((kk >> 2) * kQAtomBytes + (kk & 3) * 32) >> 4);
+        const uint64_t ko = (uint64_t)(((kk >> 2) * kb_atom_bytes + (kk & 3) * 32) >> 4);
+        mma_bf16_ss(tmem + (uint32_t)n0, q_desc + qo, kb_desc + ko, idesc, kk > 0 ? 1u : 0u);
+      }
       mma_commit(&bar_mma);
+      ok = __all_sync(0xffffffffu, mbar_wait(&bar_mma, phase & 1, &abort_flag, p.status));  // buffer free again
     }
   }
-  ok = __syncthreads_and(ok);
-  if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bar_mma, 0, &abort_flag, p.status));
-  ok = __syncthreads_and(ok);
+  tc_fence_before();
+  ok = __syncthreads_and(ok);  // the scores are complete (the MMA warp saw its last commit)
   tc_fence_after();
   if (ok) {
     const uint32_t lane_addr = tmem + ((uint32_t)(warp * 32) << 16);
@@ -463,9 +463,7 @@ int launch_sa_select(const CUtensorMap& q_rot_map, const uint16_t* q_rot, const 
   p.alpha_num = alpha_num;
   p.alpha_den = alpha_den;
   p.words = words;
-  // candidate blocks of one tile: at most the current block of its last row, capped by TMEM
-  const int nb_max = std::min(max_blocks - 1, sa::kSelMaxCols);
-  p.kb_rows = std::max(sa::kKbBox, (((nb_max + 15) & ~15) + sa::kKbBox - 1) / sa::kKbBox * sa::kKbBox);
+  p.kb_rows = sa::kKbBox;  // the pooled keys stream through a buffer of one TMA box
   int rc = d == 128 ? sa::launch_select_tc<128>(q_rot_map, tkb, p, max_items, stream)
                     : sa::launch_select_tc<64>(q_rot_map, tkb, p, max_items, stream);
   if (rc != NAMOH_OK) return rc;
