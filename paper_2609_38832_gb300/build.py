@@ -42,7 +42,7 @@ def _stale(out: str, deps: list[str]) -> bool:
 def build(force: bool = False, verbose: bool = False) -> str:
     nvcc = _nvcc()
     os.makedirs(BUILD_DIR, exist_ok=True)
-    headers = [os.path.join(CSRC, "common.cuh"), os.path.join(CSRC, "plan.cuh"), os.path.join(INCLUDE, "namoh.h")]
+    headers = [os.path.join(CSRC, h) for h in ("common.cuh", "plan.cuh", "sa_select.cuh")] + [os.path.join(INCLUDE, "namoh.h")]
     objs = []
     jobs = []
     for src in SOURCES:

@@ -22,16 +22,11 @@
 //                         in TMEM: one warp per query, scores on the CUDA cores (lane l: d / 32 columns,
 //                         warp reduce-scatter per 32 blocks), R(r) - 1 rounds of a warp arg-max.
 //
-// Selection order.  Each block's score is keyed by its fp32 value mapped to an order-preserving
-// integer, with the low 10 bits replaced by 1023 - b: a larger key is a higher score, and scores
-// equal to within the 10 dropped bits (2^-13 relative, far inside the bf16 rounding the inputs
-// already carry) go to the lower block index.  Keys are unique, so "kept" is "key >= the k-th
-// largest key".  With k = R(r) - 1 kept of the c = N_B(r) - 1 completed blocks, a thread finds
-// min(k, c - k) extreme keys (the kept set, or the dropped one) with a sorted 8-entry register list
-// fed by a branch-free insertion network, or, past 8, by bisection over the 32-bit key range.
+// The per-query selection itself (keys, register list, bisection) is in sa_select.cuh.
 #include <algorithm>
 
 #include "common.cuh"
+#include "sa_select.cuh"
 
 namespace namoh {
 namespace sa {
@@ -42,7 +37,6 @@ constexpr int kSelMaxCols = 512;            // block scores one select CTA keeps
 constexpr int kSelThreads = 128;            // one thread per query row of a 128-row tile
 constexpr int kSelTileRows = 128;
 constexpr int kKbBox = 64;                  // pooled-key rows per TMA box
-constexpr int kListLen = 8;                 // register list of the streaming selection
 
 __device__ __forceinline__ int blk_base(const int32_t* seg_offsets, int s, int lg) {
   return (seg_offsets[s] >> lg) + s;
@@ -53,18 +47,6 @@ __device__ __forceinline__ int blk_base(const int32_t* seg_offsets, int s, int l
 __device__ __forceinline__ bool seg_live(const int32_t* seg_offsets, const int64_t* seg_base,
                                          const int32_t* seg_cap, int s) {
   return !seg_base || seg_offsets[s + 1] - seg_offsets[s] <= seg_cap[s];
-}
-
-// Kept historical blocks of a query whose current block is `cur`: ceil(alpha (cur + 1)) - 1, exact.
-__device__ __forceinline__ int kept_blocks(int cur, int alpha_num, int alpha_den) {
-  return (int)(((long long)(cur + 1) * alpha_num + alpha_den - 1) / alpha_den) - 1;
-}
-
-// Selection key of block b with fp32 score s (see the file header).  -0 and +0 map alike.
-__device__ __forceinline__ uint32_t score_key(float s, int b) {
-  uint32_t u = __float_as_uint(s + 0.0f);
-  u = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-  return (u & ~0x3FFu) | (uint32_t)(0x3FF - b);
 }
 
 __global__ void __launch_bounds__(256) sa_pool_kernel(const uint16_t* __restrict__ k_cache,
@@ -130,12 +112,6 @@ struct SelParams {
   int g, lg, alpha_num, alpha_den, words;
   int kb_rows;         // pooled-key rows of the streaming buffer (kKbBox)
 };
-
-// Row of block scores of this thread, 32 columns (blocks 32 c .. 32 c + 31) at a time.
-__device__ __forceinline__ void load_scores(uint32_t taddr, uint32_t (&r)[32]) {
-  tmem_ld32(taddr, r);
-  tmem_wait_ld();
-}
 
 template <int D>
 __global__ void __launch_bounds__(kSelThreads) sa_select_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
@@ -233,78 +209,9 @@ __global__ void __launch_bounds__(kSelThreads) sa_select_tc_kernel(const __grid_
     const bool mine = valid && cur <= kSelMaxCols;
     const int keep = mine ? keep_all : 0;
     const int cand = mine ? cur : 0;                 // candidate blocks 0 .. cur - 1
-    const bool drop_mode = 2 * keep > cand;          // find the dropped blocks instead
-    const int kx = drop_mode ? cand - keep : keep;   // extreme keys to find
-    const uint32_t flip = drop_mode ? 0xFFFFFFFFu : 0u;
-    uint32_t tau = 0xFFFFFFFFu;                      // the kx-th largest key (x = key ^ flip)
-    // Every loop below runs over the CTA-uniform chunk count: tcgen05.ld is warp-collective, so
-    // every lane takes part in every load and the lanes' own work is predicated.
-    const bool use_list = kx > 0 && kx <= kListLen;
-    {
-      uint32_t best[kListLen];
-#pragma unroll
-      for (int i = 0; i < kListLen; ++i) best[i] = 0u;
-      for (int c = 0; c < nchunks; ++c) {
-        if (__all_sync(0xffffffffu, !use_list || c * 32 >= cand)) continue;  // no lane has a candidate here
-        uint32_t v[32];
-        load_scores(lane_addr + (uint32_t)(c * 32), v);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const int b = c * 32 + i;
-          uint32_t x = (use_list && b < cand) ? score_key(__uint_as_float(v[i]), b) ^ flip : 0u;
-#pragma unroll
-          for (int e = 0; e < kListLen; ++e) {  // insertion into the sorted list, branch-free
-            const uint32_t hi = max(best[e], x);
-            x = min(best[e], x);
-            best[e] = hi;
-          }
-        }
-      }
-#pragma unroll
-      for (int e = 0; e < kListLen; ++e)
-        if (use_list && e == kx - 1) tau = best[e];
-    }
-    if (__any_sync(0xffffffffu, kx > kListLen)) {
-      // bisection for the lanes that need more than kListLen keys: the largest t with
-      // #{x >= t} >= kx, which (keys unique) is the kx-th largest key
-      uint32_t lo = 0u, hi = 0xFFFFFFFFu;
-      for (int it = 0; it < 32; ++it) {
-        const uint32_t mid = lo + ((hi - lo) >> 1) + ((hi - lo) & 1u);
-        int cnt = 0;
-        for (int c = 0; c < nchunks; ++c) {
-          uint32_t v[32];
-          load_scores(lane_addr + (uint32_t)(c * 32), v);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int b = c * 32 + i;
-            cnt += (b < cand && (score_key(__uint_as_float(v[i]), b) ^ flip) >= mid) ? 1 : 0;
-          }
-        }
-        if (lo < hi) {
-          if (cnt >= kx) lo = mid;
-          else hi = mid - 1u;
-        }
-      }
-      if (kx > kListLen) tau = lo;
-    }
-    // the mask: block b kept iff key >= tau (kept mode), ~key < tau (drop mode)
-    for (int c = 0; c < nchunks; ++c) {
-      if (__all_sync(0xffffffffu, c * 32 >= cand)) {  // no candidate of any lane: an empty word
-        if (mine && c < p.words) mrow[c] = 0u;
-        continue;
-      }
-      uint32_t v[32];
-      load_scores(lane_addr + (uint32_t)(c * 32), v);
-      uint32_t w = 0u;
-#pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const int b = c * 32 + i;
-        const uint32_t x = score_key(__uint_as_float(v[i]), b) ^ flip;
-        const bool kept = b < cand && keep > 0 && (drop_mode ? x < tau : x >= tau);
-        w |= (kept ? 1u : 0u) << i;
-      }
+    select_from_tmem(lane_addr, nchunks, cand, keep, [&](int c, uint32_t w) {
       if (mine && c < p.words) mrow[c] = w;
-    }
+    });
     if (mine)
       for (int w = nchunks; w < p.words; ++w) mrow[w] = 0u;
   } else if (warp == 0) {
