@@ -306,13 +306,15 @@ __device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores,
   }
 }
 
-// TopK and gates only (no packed layout), one thread per token.
-template <int HMAX, int KMAX, bool kBiased>
+// TopK and gates only (no packed layout), one thread per token.  kFullH: H == HMAX, so every
+// per-head guard folds away at compile time.
+template <int HMAX, int KMAX, bool kBiased, bool kFullH>
 __global__ void __launch_bounds__(kChunk) route_topk_kernel(const float* __restrict__ scores,
-                                                            const float* __restrict__ bias, int T, int H, int K,
+                                                            const float* __restrict__ bias, int T, int H_, int K,
                                                             int32_t* __restrict__ topk_head, float* __restrict__ gate,
                                                             uint32_t* __restrict__ status) {
   __shared__ int s_bad;
+  const int H = kFullH ? HMAX : H_;
   const int t = blockIdx.x * kChunk + threadIdx.x;
   if (threadIdx.x == 0) s_bad = 0;
   __syncthreads();
@@ -368,9 +370,9 @@ __global__ void __launch_bounds__(1024) route_scan_kernel(const int32_t* __restr
 // the chunk's head counts, and rank_local = the (token, slot)'s rank among this chunk's
 // earlier tokens for its head (Sec. 3.2 Eq. namoh-head-rope restricted to the chunk).
 // rank_local goes to `rank`, which the final pass turns into the full rank.
-template <int HMAX, int KMAX, bool kBiased>
+template <int HMAX, int KMAX, bool kBiased, bool kFullH>
 __global__ void __launch_bounds__(kChunk) route_local_kernel(const float* __restrict__ scores,
-                                                             const float* __restrict__ bias, int T, int H, int K,
+                                                             const float* __restrict__ bias, int T, int H_, int K,
                                                              int nchunks, int32_t* __restrict__ topk_head,
                                                              float* __restrict__ gate, int32_t* __restrict__ rank,
                                                              int32_t* __restrict__ chunk_count,
@@ -379,6 +381,7 @@ __global__ void __launch_bounds__(kChunk) route_local_kernel(const float* __rest
                                                              int total) {
   __shared__ uint32_t s_bal[kChunk / 32][NAMOH_MAX_HEADS];
   __shared__ int s_bad;
+  const int H = kFullH ? HMAX : H_;  // (kFullH: a compile-time head count)
   pdl_launch_dependents();
   const int c = blockIdx.x, b = blockIdx.y;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -558,15 +561,16 @@ struct RouteArgs {
 // pass; larger ones are scanned once by route_scan_kernel.
 constexpr int kFinalMaxTable = 1 << 12;
 
-template <int HMAX, int KMAX, bool kBiased>
+template <int HMAX, int KMAX, bool kBiased, bool kFullH = false>
 int launch_route(const RouteArgs& a, cudaStream_t stream) {
   const dim3 chunks((unsigned)a.nchunks, (unsigned)a.B);
   if (a.seg_offsets == nullptr) {
-    route_topk_kernel<HMAX, KMAX, kBiased><<<chunks, kChunk, 0, stream>>>(a.scores, a.bias, a.T, a.H, a.K, a.topk_head,
-                                                                          a.gate, a.status);
+    route_topk_kernel<HMAX, KMAX, kBiased, kFullH><<<chunks, kChunk, 0, stream>>>(a.scores, a.bias, a.T, a.H, a.K,
+                                                                                  a.topk_head, a.gate, a.status);
     return cuda_check_launch("route_topk_kernel launch");
   }
-  cudaError_t e = launch_pdl(route_local_kernel<HMAX, KMAX, kBiased>, chunks, dim3(kChunk), 0, stream, a.scores, a.bias,
+  cudaError_t e = launch_pdl(route_local_kernel<HMAX, KMAX, kBiased, kFullH>, chunks, dim3(kChunk), 0, stream, a.scores,
+                             a.bias,
                              a.T, a.H, a.K, a.nchunks, a.topk_head, a.gate, a.rank, a.chunk_count, a.status,
                              a.cu_seqlens, a.B, a.total);
   if (e != cudaSuccess) return cuda_fail(e, "route_local_kernel launch");
@@ -585,18 +589,23 @@ int launch_route(const RouteArgs& a, cudaStream_t stream) {
   return NAMOH_OK;
 }
 
-// picks held in registers for K <= 8; larger K takes K passes over the logits
+// picks held in registers for K <= 8; larger K takes K passes over the logits.  K <= 4 with H a
+// power of two takes the kernels with a compile-time head count.
+template <int HMAX, bool kBiased>
+int launch_route_k4(const RouteArgs& a, cudaStream_t stream) {
+  return a.H == HMAX ? launch_route<HMAX, 4, kBiased, true>(a, stream) : launch_route<HMAX, 4, kBiased>(a, stream);
+}
 template <bool kBiased>
 int launch_route_h(const RouteArgs& a, cudaStream_t stream) {
   const int H = a.H, K = a.K;
-  if (H <= 8) return K <= 4 ? launch_route<8, 4, kBiased>(a, stream) : launch_route<8, 8, kBiased>(a, stream);
+  if (H <= 8) return K <= 4 ? launch_route_k4<8, kBiased>(a, stream) : launch_route<8, 8, kBiased>(a, stream);
   if (H <= 16)
-    return K <= 4 ? launch_route<16, 4, kBiased>(a, stream)
+    return K <= 4 ? launch_route_k4<16, kBiased>(a, stream)
                   : K <= 8 ? launch_route<16, 8, kBiased>(a, stream) : launch_route<16, 0, kBiased>(a, stream);
   if (H <= 32)
-    return K <= 4 ? launch_route<32, 4, kBiased>(a, stream)
+    return K <= 4 ? launch_route_k4<32, kBiased>(a, stream)
                   : K <= 8 ? launch_route<32, 8, kBiased>(a, stream) : launch_route<32, 0, kBiased>(a, stream);
-  return K <= 4 ? launch_route<64, 4, kBiased>(a, stream)
+  return K <= 4 ? launch_route_k4<64, kBiased>(a, stream)
                 : K <= 8 ? launch_route<64, 8, kBiased>(a, stream) : launch_route<64, 0, kBiased>(a, stream);
 }
 
