@@ -22,6 +22,7 @@
 #include <float.h>
 
 #include <mutex>
+#include <type_traits>
 
 #include "common.cuh"
 
@@ -166,12 +167,13 @@ __device__ __forceinline__ void topk4_sorted(const float (&sc)[HMAX], int H, int
       t3 = fmaxf(t3, x);
     }
   }
-  uint64_t ge = 0ull;  // heads at or above t3
-  float loc[HMAX];     // a copy the picks are read back from by index
+  using Mask = typename std::conditional<(HMAX <= 32), uint32_t, uint64_t>::type;
+  Mask ge = 0;     // heads at or above t3
+  float loc[HMAX];  // a copy the picks are read back from by index
 #pragma unroll
   for (int h = 0; h < HMAX; ++h) {
     loc[h] = sc[h];
-    if (h < H && sc[h] >= t3) ge |= 1ull << h;
+    if (h < H && sc[h] >= t3) ge |= (Mask)1 << h;
   }
   int eq_left = 4 - ((t0 > t3) + (t1 > t3) + (t2 > t3));  // picks equal to t3
 #pragma unroll
@@ -181,8 +183,8 @@ __device__ __forceinline__ void topk4_sorted(const float (&sc)[HMAX], int H, int
   }
   int n = 0;
   while (ge && n < 4) {
-    const int h = __ffsll((long long)ge) - 1;
-    ge &= ge - 1ull;
+    const int h = (sizeof(Mask) == 4 ? __ffs((int)ge) : __ffsll((long long)ge)) - 1;
+    ge &= ge - 1;
     const float x = loc[h];
     const bool take = x > t3 || eq_left > 0;
     if (!take) continue;
