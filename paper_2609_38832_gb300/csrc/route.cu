@@ -461,6 +461,9 @@ __global__ void __launch_bounds__(kChunk) route_final_kernel(const int32_t* __re
   __shared__ int s_bef[kChunk];
   __shared__ int s_cbase[NAMOH_MAX_HEADS];
   __shared__ int s_soff[NAMOH_MAX_HEADS];
+  __shared__ int s_pos[NAMOH_MAX_HEADS];  // (K = 4) first staging slot of each head's rows
+  __shared__ int32_t s_src[kChunk * 4];   // (K = 4) row_src values, grouped by head in rank order
+  __shared__ int32_t s_dst[kChunk * 4];   // (K = 4) and the rows they go to
   pdl_launch_dependents();
   const int c = blockIdx.x, b = blockIdx.y;
   const int tid = threadIdx.x;
@@ -521,21 +524,40 @@ __global__ void __launch_bounds__(kChunk) route_final_kernel(const int32_t* __re
     if (c == 0 && b == B - 1 && tid == 0) seg_offsets[(size_t)B * H] = (sr.start + sr.len) * K;
   }
   __syncthreads();
-  if (!valid) return;
-  if (vec4) {
-    const int hs[4] = {h4.x, h4.y, h4.z, h4.w}, ls[4] = {r4.x, r4.y, r4.z, r4.w};
-    int rho[4], rw[4];
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      rho[k] = s_cbase[hs[k]] + ls[k];
-      rw[k] = s_soff[hs[k]] + rho[k];
+  if (K == 4 && __syncthreads_and(!valid || vec4)) {
+    // row_src through shared memory: this chunk's rows of head h are the contiguous run
+    // seg_offsets + chunk base .. + count of segment h, so staging the values by head (at their
+    // local rank) and writing the staged array in order turns 4 scattered stores per token into
+    // runs of consecutive rows
+    if (tid == 0) {
+      const int32_t* cc = chunk_count + ((size_t)b * nchunks + c) * H;
+      int pos = 0;
+      for (int hh = 0; hh < H; ++hh) {
+        s_pos[hh] = pos;
+        pos += __ldcg(cc + hh);
+      }
     }
-    *reinterpret_cast<int4*>(rank + base) = make_int4(rho[0], rho[1], rho[2], rho[3]);
-    *reinterpret_cast<int4*>(row + base) = make_int4(rw[0], rw[1], rw[2], rw[3]);
+    __syncthreads();
+    if (valid) {
+      const int hs[4] = {h4.x, h4.y, h4.z, h4.w}, ls[4] = {r4.x, r4.y, r4.z, r4.w};
+      int rho[4], rw[4];
 #pragma unroll
-    for (int k = 0; k < 4; ++k) row_src[rw[k]] = (int32_t)(base + k);
+      for (int k = 0; k < 4; ++k) {
+        rho[k] = s_cbase[hs[k]] + ls[k];
+        rw[k] = s_soff[hs[k]] + rho[k];
+        const int e = s_pos[hs[k]] + ls[k];
+        s_src[e] = (int32_t)(base + k);
+        s_dst[e] = rw[k];
+      }
+      *reinterpret_cast<int4*>(rank + base) = make_int4(rho[0], rho[1], rho[2], rho[3]);
+      *reinterpret_cast<int4*>(row + base) = make_int4(rw[0], rw[1], rw[2], rw[3]);
+    }
+    __syncthreads();
+    const int nent = 4 * max(0, min(kChunk, sr.len - c * kChunk));  // this chunk's (token, slot) rows
+    for (int e = tid; e < nent; e += kChunk) row_src[s_dst[e]] = s_src[e];
     return;
   }
+  if (!valid) return;
   for (int k = 0; k < K; ++k) {
     const size_t i = base + k;
     const int h = topk_head[i];
