@@ -359,6 +359,28 @@ def run_gpu(args, rank: int, world: int):
     h2d = scores_h.nbytes + q_h.nbytes + k_h.nbytes + v_h.nbytes
     d2h = y.numel() * 2
 
+    def copy_ms(pairs, n):
+        """Mean time of one round of the given copies alone, on a stream of their own."""
+        s = torch.cuda.Stream(dev)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(s):
+            for i in range(n + 2):
+                if i == 2:
+                    a.record(s)
+                for dst, src in pairs:
+                    dst.copy_(src, non_blocking=True)
+            b.record(s)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / n
+
+    # the host link alone, with the same buffers and bytes as a step's copies: the floor under e2e
+    h2d_ms = copy_ms(list(zip(sets[0][:4], (scores_p, q_p, k_p, v_p))), args.steps)
+    d2h_ms = copy_ms([(y_p[0], sets[0][4].view(torch.int16))], args.steps)
+    host_link = {"h2d_ms_per_step": h2d_ms, "d2h_ms_per_step": d2h_ms, "h2d_gbs": h2d / (h2d_ms * 1e-3) / 1e9,
+                 "d2h_gbs": d2h / (d2h_ms * 1e-3) / 1e9,
+                 "note": "the step's pinned copies timed alone (CUDA events on their own stream); the pipelined e2e "
+                         "step cannot be shorter than the longer direction"}
+
     peak_tf = pk["bf16_tflops"]
     achieved = flops / (attn_ms * 1e-3) / 1e12
     traffic = ncu_traffic()
@@ -394,7 +416,7 @@ def run_gpu(args, rank: int, world: int):
                 "api": "namoh_route + namoh_prefill from pinned host buffers, y copied back",
                 "pipeline": f"host->device copies, compute and device->host copies on three streams, consecutive "
                             f"steps overlapped; {NSET} rotating device input/output sets ({NSET} x 51 MB > L2), "
-                            f"no flush", "y_readback_matches_device": e2e_y_ok},
+                            f"no flush", "y_readback_matches_device": e2e_y_ok, "host_link": host_link},
         # per step: route (2 kernels) + RoPE/plan (1) + attention (1), in each of the three timed
         # passes (headline, stage breakdown, end to end), and one RoPE/plan launch per timed
         # step in each of the four RoPE variants

@@ -49,12 +49,14 @@ __device__ __forceinline__ bool seg_live(const int32_t* seg_offsets, const int64
   return !seg_base || seg_offsets[s + 1] - seg_offsets[s] <= seg_cap[s];
 }
 
+template <int D, int LG>
 __global__ void __launch_bounds__(256) sa_pool_kernel(const uint16_t* __restrict__ k_cache,
                                                       const int32_t* __restrict__ seg_offsets,
                                                       const int64_t* __restrict__ seg_base,
                                                       const int32_t* __restrict__ seg_cap, long long cache_rows,
-                                                      int d, int lg, int g, uint16_t* __restrict__ kbar,
-                                                      uint32_t* __restrict__ mask, int words) {
+                                                      int g, uint16_t* __restrict__ kbar, uint32_t* __restrict__ mask,
+                                                      int words) {
+  constexpr int d = D, lg = LG;
   pdl_launch_dependents();
   pdl_wait();  // the rotated keys come from the RoPE pass before it
   const int s = blockIdx.y;
@@ -73,23 +75,32 @@ __global__ void __launch_bounds__(256) sa_pool_kernel(const uint16_t* __restrict
   const long long row0 = (seg_base ? seg_base[s] : (long long)seg_offsets[s]) + ((long long)b << lg);
   // rows outside the cache were never written (the RoPE pass reports them): nothing to pool
   if (row0 < 0 || row0 + (1ll << lg) > cache_rows) return;
-  // lane l reads the 16-byte piece l % P of row t + l / P, P = d / 8 pieces per row
-  const int P = d >> 3;              // 8 or 16
-  const int rows_per = 32 / P;       // rows per warp instruction: 4 or 2
+  // lane l reads the 16-byte piece l % P of row t + l / P, P = d / 8 pieces per row; every load of
+  // the block is issued before the first is used (the block's rows a lane reads: 2^lg / (32 / P))
+  constexpr int P = D / 8;            // 8 or 16
+  constexpr int rows_per = 32 / P;    // rows per warp instruction: 4 or 2
+  constexpr int nld = (1 << LG) / rows_per;
   const int piece = lane % P, sub = lane / P;
   float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-  const uint4* src = reinterpret_cast<const uint4*>(k_cache + row0 * d) + piece;
-#pragma unroll 8
-  for (int t = sub; t < (1 << lg); t += rows_per) {  // unrolled: eight 16-byte loads in flight per lane
-    const uint4 w = __ldg(src + (long long)t * P);
-    const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
+  const uint4* src = reinterpret_cast<const uint4*>(k_cache + row0 * d) + piece + (long long)sub * P;
+  constexpr int kBatch = nld < 16 ? nld : 16;
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      acc[2 * e] += bf16_lo(wv[e]);
-      acc[2 * e + 1] += bf16_hi(wv[e]);
+  for (int i0 = 0; i0 < nld; i0 += kBatch) {
+    uint4 w[kBatch];
+#pragma unroll
+    for (int i = 0; i < kBatch; ++i) w[i] = __ldg(src + (long long)(i0 + i) * rows_per * P);
+#pragma unroll
+    for (int i = 0; i < kBatch; ++i) {
+      const uint32_t wv[4] = {w[i].x, w[i].y, w[i].z, w[i].w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        acc[2 * e] += bf16_lo(wv[e]);
+        acc[2 * e + 1] += bf16_hi(wv[e]);
+      }
     }
   }
   // lanes holding the same piece of different rows add up (fixed order: a butterfly over `sub`)
+#pragma unroll
   for (int o = P; o < 32; o <<= 1)
 #pragma unroll
     for (int e = 0; e < 8; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], o);
@@ -353,8 +364,12 @@ int launch_sa_select(const CUtensorMap& q_rot_map, const uint16_t* q_rot, const 
   const int max_blocks = (T + (1 << lg) - 1) >> lg;
   if (nseg > 0 && max_blocks > 0) {
     dim3 grid((max_blocks + 7) / 8, nseg);
-    const cudaError_t e = launch_pdl(sa::sa_pool_kernel, grid, dim3(256), 0, stream, k_cache, seg_offsets, seg_base,
-                                     seg_cap, cache_rows, d, lg, g, kbar, mask, words);
+    auto pool = d == 128 ? (lg == 5 ? sa::sa_pool_kernel<128, 5> : lg == 6 ? sa::sa_pool_kernel<128, 6>
+                                                                            : sa::sa_pool_kernel<128, 7>)
+                         : (lg == 5 ? sa::sa_pool_kernel<64, 5> : lg == 6 ? sa::sa_pool_kernel<64, 6>
+                                                                           : sa::sa_pool_kernel<64, 7>);
+    const cudaError_t e = launch_pdl(pool, grid, dim3(256), 0, stream, k_cache, seg_offsets, seg_base, seg_cap,
+                                     cache_rows, g, kbar, mask, words);
     if (e != cudaSuccess) return cuda_fail(e, "sa_pool_kernel launch");
   }
   if (R <= 0 || max_items <= 0) return NAMOH_OK;
