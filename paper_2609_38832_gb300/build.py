@@ -19,7 +19,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(PKG, "_build")
 LIB_PATH = os.path.join(PKG, "libnamoh.so")
 
-SOURCES = ["api.cu", "route.cu", "rope_pack.cu", "prefill_attn.cu", "decode.cu", "proj.cu", "sa_select.cu"]
+SOURCES = ["api.cu", "route.cu", "rope_pack.cu", "prefill_attn.cu", "window_attn.cu", "decode.cu", "proj.cu",
+           "sa_select.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
           "-diag-suppress", "177"]

@@ -46,6 +46,11 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              void* plan, int plan_qtiles, const int32_t* plan_cap, const int32_t* pos_row_src,
                              int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved);
 
+int launch_window_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint16_t* v_cache, int B, int T,
+                            int Hs, int D, int window, const int64_t* seg_base, long long cache_rows, uint16_t* y,
+                            uint32_t* dev_status, int sm_count, cudaStream_t stream);
+constexpr int kMaxBandWindow = 128;  // windows up to one key tile run as one 256-key band per query tile
+
 int launch_sa_select(const CUtensorMap& q_rot_map, const uint16_t* q_rot, const uint16_t* k_cache,
                      const int32_t* seg_offsets, const int64_t* seg_base, const int32_t* seg_cap,
                      long long cache_rows, int nseg, int T, long long R, int d, int g, int lg, int alpha_num,
@@ -1156,9 +1161,15 @@ extern "C" int namoh_sa_prefill(const uint16_t* q, const uint16_t* k, const uint
 // ---------------------------------------------------------------------------
 namespace namoh {
 namespace {
+// rows = false: seg_offsets only (the band kernel computes y's rows itself)
 __global__ void shared_layout_kernel(int B, int T, int Hs, int32_t* __restrict__ seg_offsets,
-                                     int32_t* __restrict__ row_src, float* __restrict__ gate) {
+                                     int32_t* __restrict__ row_src, float* __restrict__ gate, bool rows) {
   const long long R = (long long)B * Hs * T;
+  if (!rows) {
+    for (int s = blockIdx.x * blockDim.x + threadIdx.x; s <= B * Hs; s += gridDim.x * blockDim.x)
+      seg_offsets[s] = (int32_t)((long long)s * T);
+    return;
+  }
   for (long long r = blockIdx.x * (long long)blockDim.x + threadIdx.x; r < R; r += (long long)gridDim.x * blockDim.x) {
     const long long bj = r / T, t = r - bj * T;
     const long long b = bj / Hs, j = bj - b * Hs;
@@ -1224,17 +1235,25 @@ extern "C" int namoh_shared_prefill(const uint16_t* q, const uint16_t* k, const 
   DeviceInfo info;
   if (!device_ok(&info)) return NAMOH_ERR_UNSUPPORTED;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
-  shared_layout_kernel<<<info.sm_count * 4, 256, 0, stream>>>(B, T, Hs, o.seg_offsets, o.row_src, o.gate);
+  // a window of at most one key tile: the band kernel (no plan, no per-row layout)
+  const bool band = window > 0 && window <= kMaxBandWindow;
+  if (band)
+    shared_layout_kernel<<<(B * Hs + 256) / 256, 256, 0, stream>>>(B, T, Hs, o.seg_offsets, nullptr, nullptr, false);
+  else
+    shared_layout_kernel<<<info.sm_count * 4, 256, 0, stream>>>(B, T, Hs, o.seg_offsets, o.row_src, o.gate, true);
   if (const int e = cuda_check_launch("shared_layout_kernel launch")) return e;
   // global positions: the rank in a segment holding every token is t (the global flag is redundant)
   st = launch_rope_and_plan(q, k, v, B, T, Hs, Hs, (int)R, d_head, 1, rope_base, rope_flags & NAMOH_ROPE_INTERLEAVED,
                             nullptr, o.seg_offsets, o.row_src, o.q_rot, k_cache, v_cache, seg_base, seg_cap,
-                            cache_rows, dev_status, o.plan, info, stream);
+                            cache_rows, dev_status, band ? nullptr : o.plan, info, stream);
   if (st != NAMOH_OK) return st;
   if (seg_len) {
     seg_len_kernel<<<(B * Hs + 255) / 256, 256, 0, stream>>>(o.seg_offsets, B * Hs, seg_len);
     if (const int e = cuda_check_launch("seg_len_kernel launch")) return e;
   }
+  if (band)
+    return launch_window_attention(o.q_rot, k_cache, v_cache, B, T, Hs, d_head, window, seg_base, cache_rows, y,
+                                   dev_status, info.sm_count, stream);
   return launch_attention(o.q_rot, k_cache, v_cache, R, d_head, 1, o.seg_offsets, o.row_src, o.gate, seg_base,
                           cache_rows, o.plan, y, dev_status, info, stream, window);
 }
