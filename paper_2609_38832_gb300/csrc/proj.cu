@@ -21,6 +21,10 @@
 //              arrives on the stage's barrier.  (TMA gather4 moves only 512 bytes per
 //              instruction and measured 7x slower here.)
 //   warp 8     TMEM owner and MMA issue: tcgen05.mma kind::f16, M = 128, N = BN, K = 16
+// QKV with exactly two column tiles (e.g. g = 1, d = 128: 384 columns as 2 x 192) computes both in
+// one pass over the contraction: a stage holds the A slice once and both weight slices, and the
+// two accumulators' MMAs alternate instruction by instruction (two chains in the tensor pipe
+// instead of one; one TMEM buffer of 384 columns, so the epilogue does not overlap the next tile).
 // Work items are (128-row tile of a segment, BN-column tile) from a list ordered by sequence,
 // then position in the segment, then head: CTAs running at the same time work on the same
 // stretch of tokens across heads, so x rows are reused from L2, and
@@ -42,11 +46,23 @@ constexpr int kSmemBudget = 208 * 1024;
 constexpr int kMaxTileListBytes = 200 * 1024;  // shared memory of the tile-list builder
 
 
-template <int BN>
+// pipeline stages that fit the shared-memory budget (at most 6)
+constexpr int stages_for(int BN, int NT) {
+  return kSmemBudget / (BM * 128 + NT * BN * 128) > 6 ? 6 : kSmemBudget / (BM * 128 + NT * BN * 128);
+}
+
+// NT column tiles of BN columns are computed together (NT accumulators, their MMAs interleaved
+// per k-block, the stage holding the A slice once and NT weight slices).
+template <int BN, int NT>
 struct Layout {
   static_assert(BN % 32 == 0 && BN >= 64 && BN <= 256, "UMMA N and the 32-column epilogue chunks");
+  static_assert(NT >= 1 && NT * BN <= 512, "the accumulators fit in TMEM");
   static constexpr int kA = BM * 128;
-  static constexpr int kB = BN * 128;
+  static constexpr int kB = NT * BN * 128;
+  static constexpr int kBSlice = BN * 128;  // one column tile's weight slice (1024-byte multiple)
+  // TMEM accumulator buffers: two (the epilogue of one group overlaps the next) when a group
+  // takes at most 256 columns, else one
+  static constexpr int kBufs = NT * BN <= 256 ? 2 : 1;
   static constexpr int kStage = kA + kB;
   static constexpr int kStages = kSmemBudget / kStage > 6 ? 6 : kSmemBudget / kStage;
   static constexpr int kLag = kStages - 2;  // stages of copies a loader keeps in flight before retiring one
@@ -183,9 +199,10 @@ __global__ void __launch_bounds__(1024) tile_list_kernel(const int32_t* __restri
 
 enum Mode { kQKV = 0, kOutP = 1 };
 
-template <int BN, int kMode>
+template <int BN, int kMode, int NT>
 __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant__ CUtensorMap tm_b, Params p) {
-  using L = Layout<BN>;
+  using L = Layout<BN, NT>;
+  constexpr int NB = L::kBufs;
   constexpr int S = L::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -217,8 +234,9 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
   pdl_wait();  // the routing layout, the tile list and the inputs are visible from here
 
   // A CTA takes row tiles mt = blockIdx.x, + gridDim.x, ... and runs every column tile of each
-  // before the next (the tile's rows are decoded once and re-gathered from L2).
+  // before the next (the tile's rows are decoded once and re-gathered from L2), NT at a time.
   const int nt_count = p.ncols / BN;
+  const int ngroups = nt_count / NT;
   const int ntiles = __ldg(p.ntiles);
   const int4* tiles = p.tiles + __ldg(p.tile_off);
   const int nk = p.kdim / BK;
@@ -250,7 +268,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     }
     // the next row tile's entry, offsets and row indices are fetched during this one's k-blocks
     // (kq counts them across its column tiles), each load issued four k-blocks before its use
-    const bool prefetch = nt_count * nk >= 12;
+    const bool prefetch = ngroups * nk >= 12;
     for (; mt < ntiles && ok; mt += gridDim.x) {
       const int next = mt + gridDim.x;
       int nx_row0 = 0, nx_rows = 0, nx_seg = 0;
@@ -260,8 +278,8 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
 #pragma unroll
       for (int w = 0; w < 8; ++w) src[w] = a_base + (size_t)rows_a[w] * p.kdim + ch * 8;
       int kq = 0;
-      for (int nt = 0; nt < nt_count && ok; ++nt) {
-        const int b_row = t.hr * p.ncols + nt * BN;
+      for (int gi = 0; gi < ngroups && ok; ++gi) {
+        const int b_row = t.hr * p.ncols + gi * NT * BN;
         for (int kb = 0; kb < nk; ++kb, ++it, ++kq) {
           if (prefetch && next < ntiles) {
             if (kq == 0) {
@@ -286,7 +304,9 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
           uint8_t* a = smem + slot * L::kStage;
           if (lt == 0) {
             mbar_arrive_expect_tx(&bars->full[slot], L::kB);
-            tma_load_2d(a + L::kA, &tm_b, kb * BK, b_row, &bars->full[slot]);
+#pragma unroll
+            for (int j = 0; j < NT; ++j)
+              tma_load_2d(a + L::kA + j * L::kBSlice, &tm_b, kb * BK, b_row + j * BN, &bars->full[slot]);
           }
 #pragma unroll
           for (int w = 0; w < 8; ++w) {
@@ -327,9 +347,9 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     bool ok = true;
     int li = 0;
     for (int mt = blockIdx.x; mt < ntiles && ok; mt += gridDim.x) {
-      for (int nt = 0; nt < nt_count && ok; ++nt, ++li) {
-        const int buf = li & 1;
-        if (li >= 2 && !warp_wait(&bars->acc_empty[buf], ((li >> 1) - 1) & 1, abort_flag, p.status)) {
+      for (int gi = 0; gi < ngroups && ok; ++gi, ++li) {
+        const int buf = li % NB;
+        if (li >= NB && !warp_wait(&bars->acc_empty[buf], ((li / NB) - 1) & 1, abort_flag, p.status)) {
           ok = false;
           break;
         }
@@ -344,10 +364,13 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
           tc_fence_after();
           const uint64_t a_desc = make_smem_desc_sw128(smem_u32(smem + slot * L::kStage), 16, 1024);
           const uint64_t b_desc = make_smem_desc_sw128(smem_u32(smem + slot * L::kStage + L::kA), 16, 1024);
+          // the NT accumulators' MMAs interleaved: independent chains overlap in the tensor pipe
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk)
-            mma_bf16_ss(d_tmem, a_desc + (uint64_t)(kk * 2), b_desc + (uint64_t)(kk * 2), idesc,
-                        (kb | kk) ? 1u : 0u);
+#pragma unroll
+            for (int j = 0; j < NT; ++j)
+              mma_bf16_ss(d_tmem + j * BN, a_desc + (uint64_t)(kk * 2),
+                          b_desc + (uint64_t)((j * L::kBSlice) >> 4) + (uint64_t)(kk * 2), idesc, (kb | kk) ? 1u : 0u);
           mma_commit(&bars->empty[slot]);
         }
         if (ok) mma_commit(&bars->acc_full[buf]);
@@ -365,20 +388,20 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
       const int r = t.row0 + row;
       // OUT_P writes row r's partial product at its token-slot row row_src[r]
       const long long dst_row = kMode == kOutP && valid ? ld_issue_s32(p.row_src + r) - p.p_row0 : r;
-      for (int nt = 0; nt < nt_count; ++nt, ++li) {
-        const int buf = li & 1;
-        if (!warp_wait(&bars->acc_full[buf], (li >> 1) & 1, abort_flag, p.status)) {
+      for (int gi = 0; gi < ngroups; ++gi, ++li) {
+        const int buf = li % NB;
+        if (!warp_wait(&bars->acc_full[buf], (li / NB) & 1, abort_flag, p.status)) {
           ok = false;
           break;
         }
         tc_fence_after();
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
+        for (int c = 0; c < NT * BN / 32; ++c) {
           uint32_t v[32];
           tmem_ld32(tmem + lane_addr + buf * 256 + c * 32, v);
           tmem_wait_ld();
           if (!valid) continue;
-          const int n = nt * BN + c * 32;  // first output column of the chunk
+          const int n = gi * NT * BN + c * 32;  // first output column of the chunk
           uint16_t* dst;
           if constexpr (kMode == kQKV) {
             const int gd = p.g * p.d;
@@ -467,14 +490,24 @@ bool encode_map(CUtensorMap* map, const void* base, long long rows, int cols, in
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, int kMode>
-cudaError_t launch_bn(const Params& p, const void* b, long long b_rows, int grid, cudaStream_t stream) {
+template <int BN, int kMode, int NT>
+cudaError_t launch_bn_nt(const Params& p, const void* b, long long b_rows, int grid, cudaStream_t stream) {
   CUtensorMap tb;
   if (!encode_map(&tb, b, b_rows, p.kdim, BN)) return cudaErrorInvalidValue;
-  const int smem = Layout<BN>::kAlloc;
-  cudaError_t e = cudaFuncSetAttribute(proj_kernel<BN, kMode>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  const int smem = Layout<BN, NT>::kAlloc;
+  cudaError_t e = cudaFuncSetAttribute(proj_kernel<BN, kMode, NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  return launch_pdl(proj_kernel<BN, kMode>, dim3(grid), dim3(kThreads), (size_t)smem, stream, tb, p);
+  return launch_pdl(proj_kernel<BN, kMode, NT>, dim3(grid), dim3(kThreads), (size_t)smem, stream, tb, p);
+}
+
+// Two column tiles per group when the QKV projection has exactly two and the group's stages
+// still leave a 3-deep pipeline (A gathered once for both, two interleaved accumulators).
+template <int BN, int kMode>
+cudaError_t launch_bn(const Params& p, const void* b, long long b_rows, int grid, cudaStream_t stream) {
+  if constexpr (kMode == kQKV && 2 * BN <= 512 && stages_for(BN, 2) >= 3) {
+    if (p.ncols == 2 * BN) return launch_bn_nt<BN, kMode, 2>(p, b, b_rows, grid, stream);
+  }
+  return launch_bn_nt<BN, kMode, 1>(p, b, b_rows, grid, stream);
 }
 
 // The widest column tile (multiple of 32, at most 256) that divides the output columns.
