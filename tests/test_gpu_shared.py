@@ -31,6 +31,11 @@ def _qkv(seed, shape):
     (2, 1, 333, 128, 37),     # a window inside one key tile
     (1, 2, 257, 128, 1),      # each token attends to itself only
     (1, 2, 4096, 128, 128),   # a long sequence
+    # more query tiles than SMs: CTAs run several consecutive tiles, the diagonal key tile of one
+    # serving as the previous tile of the next, and runs cross segment boundaries
+    (4, 4, 4096, 128, 128),   # the bench's shape
+    (1, 8, 5000, 64, 100),    # d = 64, a window inside one key tile, a ragged last tile
+    (2, 3, 7000, 128, 2),     # the smallest window that reads the previous key tile
 ])
 def test_shared_prefill_matches_oracle(namoh, oracle_mod, B, Hs, T, d, window):
     q, k, v = _qkv(60, (B, Hs, T, d))
