@@ -611,9 +611,15 @@ def run_layer(args, dev, pk, pk_kind):
     step()
     torch.cuda.synchronize()
     # the output projection runs one product-and-combine pair per token chunk of at most 1 GB of
-    # bf16 per-slot products (the library's chunking)
+    # bf16 per-slot products (the library's chunking); a projection over one chunk of a small
+    # layout builds its tile list inside the GEMM, otherwise two list kernels run first
     out_chunk = min(N, max(128, (1 << 30) // (Kr * d_model * 2)))
-    out_launches = 2 + 2 * (-(-N // out_chunk))
+    nchunk = -(-N // out_chunk)
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    nseg = B * Hr
+    list_in_kernel = nseg <= 1024 and -(-(-(-R // 128) + nseg) // sms) <= 288
+    qkv_launches = 1 if list_in_kernel else 3
+    out_launches = 2 * nchunk + (0 if (list_in_kernel and nchunk == 1) else 2)
     n_seg = acc.segment_lengths(ro.seg_offsets.cpu().numpy())
     f_attn = acc.attention_flops(n_seg, d, g)
     f_qkv = 2.0 * R * d_model * (g + 2) * d
@@ -634,9 +640,9 @@ def run_layer(args, dev, pk, pk_kind):
         "peak_source": f"{pk_kind} bf16 dense (burst)",
         "l2": "flushed before every timed launch sequence (2 GB write)",
         "device_status": int(status.item()),
-        # timed launches: QKV (range table, tile list, GEMM), OUT (range table, tile list, then a
-        # GEMM and a combine per chunk), and the step (route 2 + QKV 3 + prefill 2 + OUT)
-        "launches": args.steps * (3 + out_launches + (2 + 3 + 2 + out_launches)),
+        # timed launches: QKV, OUT (a GEMM and a combine per chunk, after the list kernels when
+        # they run), and the step (route 2 + QKV + prefill 2 + OUT)
+        "launches": args.steps * (qkv_launches + out_launches + (2 + qkv_launches + 2 + out_launches)),
     }
 
 

@@ -25,6 +25,9 @@
 // one pass over the contraction: a stage holds the A slice once and both weight slices, and the
 // two accumulators' MMAs alternate instruction by instruction (two chains in the tensor pipe
 // instead of one; one TMEM buffer of 384 columns, so the epilogue does not overlap the next tile).
+// The row-tile list comes from range_table_kernel + tile_list_kernel, or, for one token chunk of
+// at most kListSeg segments, from each CTA itself: it reads the segment offsets and derives the
+// entries it will run (no list kernels between the routing and the GEMM).
 // Work items are (128-row tile of a segment, BN-column tile) from a list ordered by sequence,
 // then position in the segment, then head: CTAs running at the same time work on the same
 // stretch of tokens across heads, so x rows are reused from L2, and
@@ -44,6 +47,11 @@ constexpr int BK = 64;   // contraction elements per stage: one 128-byte swizzle
 constexpr int kThreads = 288;
 constexpr int kSmemBudget = 208 * 1024;
 constexpr int kMaxTileListBytes = 200 * 1024;  // shared memory of the tile-list builder
+// A layout of at most kListSeg segments in one token chunk, with at most kListTiles row tiles per
+// CTA, has its tile list computed by each CTA itself (no list kernels before the GEMM).
+constexpr int kListSeg = 1024;
+constexpr int kListTiles = 288;
+constexpr int kListBytes = kListTiles * 16 + (2 * kListSeg + 1) * 4;
 
 
 // pipeline stages that fit the shared-memory budget (at most 6)
@@ -68,11 +76,14 @@ struct Layout {
   static constexpr int kLag = kStages - 2;  // stages of copies a loader keeps in flight before retiring one
   static_assert(kLag >= 1, "pipeline depth");
   static constexpr int kBar = kStages * kStage;
-  static constexpr int kAlloc = kBar + 256 + 1024;  // barriers, plus slack for 1024-byte alignment
+  static constexpr int kList = kBar + 256;          // the CTA's own tile list (when built in-kernel)
+  static constexpr int kAlloc = kList + kListBytes + 1024;  // plus slack for 1024-byte alignment
 };
 
 struct Params {
-  const int4* tiles;           // {first row, rows, segment, 0}: the 128-row tiles, in work order
+  const int4* tiles;           // {first row, rows, segment, 0}: the 128-row tiles, in work order;
+                               // null: each CTA derives its own tiles from seg_offsets
+  const int32_t* seg_offsets;  // [nseg + 1] (the in-kernel list)
   const int32_t* tile_off;     // the list's first entry for this launch
   const int32_t* ntiles;       // the number of entries for this launch
   const int32_t* row_src;      // [R]
@@ -237,9 +248,78 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
   // before the next (the tile's rows are decoded once and re-gathered from L2), NT at a time.
   const int nt_count = p.ncols / BN;
   const int ngroups = nt_count / NT;
-  const int ntiles = __ldg(p.ntiles);
-  const int4* tiles = p.tiles + __ldg(p.tile_off);
   const int nk = p.kdim / BK;
+  const int G = gridDim.x;
+  const bool local_list = p.tiles == nullptr;
+  int4* s_tiles = reinterpret_cast<int4*>(smem + L::kList);
+  __shared__ int s_ntiles;
+  int ntiles = 0;
+  const int4* tiles = nullptr;
+  if (!local_list) {
+    ntiles = __ldg(p.ntiles);
+    tiles = p.tiles + __ldg(p.tile_off);
+  } else {
+    // The list in the order tile_list_kernel writes: sequence b's tiles before b + 1's, tile q of
+    // every head before tile q + 1 of any, heads in order.  Tile (b, q, h) is entry
+    //   base(b) + cnt_b(q) + #{h' < h : nt(b, h') > q},  cnt_b(q) = sum_h' min(q, nt(b, h')),
+    // so entry mt is found by the last b with base(b) <= mt, then the last q with
+    // cnt_b(q) <= mt - base(b) (cnt_b grows with q), then the head.
+    int* s_nt = reinterpret_cast<int*>(s_tiles + kListTiles);  // [nseg] row tiles per segment
+    int* s_base = s_nt + kListSeg;                             // [B + 1] first entry per sequence
+    const int B = p.nseg / p.Hr, Hr = p.Hr;
+    for (int i = threadIdx.x; i < p.nseg; i += blockDim.x) {
+      const int n = __ldg(p.seg_offsets + i + 1) - __ldg(p.seg_offsets + i);
+      s_nt[i] = n > 0 ? (n + BM - 1) / BM : 0;
+    }
+    __syncthreads();
+    for (int b = threadIdx.x; b < B; b += blockDim.x) {
+      int tot = 0;
+      for (int h = 0; h < Hr; ++h) tot += s_nt[b * Hr + h];
+      s_base[b + 1] = tot;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      s_base[0] = 0;
+      for (int b = 0; b < B; ++b) s_base[b + 1] += s_base[b];
+      s_ntiles = s_base[B];
+    }
+    __syncthreads();
+    ntiles = s_ntiles;
+    for (int k = threadIdx.x; (int)blockIdx.x + k * G < ntiles && k < kListTiles; k += blockDim.x) {
+      const int mt = (int)blockIdx.x + k * G;
+      int lo = 0, hi = B;
+      while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (s_base[mid] <= mt) lo = mid; else hi = mid;
+      }
+      const int b = lo, local = mt - s_base[b];
+      const int* nt = s_nt + b * Hr;
+      int qmax = 0;
+      for (int h = 0; h < Hr; ++h) qmax = max(qmax, nt[h]);
+      auto cnt = [&](int q) {
+        int c = 0;
+        for (int h = 0; h < Hr; ++h) c += min(q, nt[h]);
+        return c;
+      };
+      int qlo = 0, qhi = qmax;  // cnt(qlo) <= local < cnt(qhi)
+      while (qhi - qlo > 1) {
+        const int mid = (qlo + qhi) >> 1;
+        if (cnt(mid) <= local) qlo = mid; else qhi = mid;
+      }
+      int idx = local - cnt(qlo), h = 0;
+      for (; h < Hr; ++h)
+        if (nt[h] > qlo) {
+          if (idx == 0) break;
+          --idx;
+        }
+      const int sg = b * Hr + h;
+      const int o0 = __ldg(p.seg_offsets + sg), n = __ldg(p.seg_offsets + sg + 1) - o0;
+      s_tiles[k] = make_int4(o0 + qlo * BM, min(BM, n - qlo * BM), sg, 0);
+    }
+    __syncthreads();
+  }
+  // entry mt of the list (mt one of this CTA's: blockIdx.x + k G)
+  auto tile_at = [&](int mt) -> int4 { return local_list ? s_tiles[(mt - (int)blockIdx.x) / G] : __ldg(tiles + mt); };
 
   if (warp >= 4 && warp < 8) {
     // ---- loads: thread lt moves 16-byte chunk (lt & 7) of rows (lt >> 3) + 16 w, w = 0..7
@@ -259,7 +339,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     Tile t{};
     int rows_a[8];
     if (mt < ntiles) {
-      t = decode_tile(p, __ldg(tiles + mt));
+      t = decode_tile(p, tile_at(mt));
 #pragma unroll
       for (int w = 0; w < 8; ++w) {
         const int r = rq + 16 * w;
@@ -283,10 +363,17 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
         for (int kb = 0; kb < nk; ++kb, ++it, ++kq) {
           if (prefetch && next < ntiles) {
             if (kq == 0) {
-              const int32_t* e = reinterpret_cast<const int32_t*>(tiles + next);
-              nx_row0 = ld_issue_s32(e);
-              nx_rows = ld_issue_s32(e + 1);
-              nx_seg = ld_issue_s32(e + 2);
+              if (local_list) {
+                const int4 e = tile_at(next);
+                nx_row0 = e.x;
+                nx_rows = e.y;
+                nx_seg = e.z;
+              } else {
+                const int32_t* e = reinterpret_cast<const int32_t*>(tiles + next);
+                nx_row0 = ld_issue_s32(e);
+                nx_rows = ld_issue_s32(e + 1);
+                nx_seg = ld_issue_s32(e + 2);
+              }
             } else if (kq == 4) {
               nx = decode_tile(p, make_int4(nx_row0, nx_rows, nx_seg, 0));
 #pragma unroll
@@ -327,7 +414,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
 #pragma unroll
         for (int w = 0; w < 8; ++w) rows_a[w] = a_row_of(nx_src[w]);
       } else {
-        t = decode_tile(p, __ldg(tiles + next));
+        t = decode_tile(p, tile_at(next));
 #pragma unroll
         for (int w = 0; w < 8; ++w) {
           const int r = rq + 16 * w;
@@ -383,7 +470,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     int li = 0;
     bool ok = true;
     for (int mt = blockIdx.x; mt < ntiles && ok; mt += gridDim.x) {
-      const Tile t = decode_tile(p, __ldg(tiles + mt));
+      const Tile t = decode_tile(p, tile_at(mt));
       const bool valid = row < t.rows;
       const int r = t.row0 + row;
       // OUT_P writes row r's partial product at its token-slot row row_src[r]
@@ -582,6 +669,13 @@ int build_tiles(const int32_t* seg_offsets, const int32_t* row_src, int nseg, in
   return cuda_check_launch("tile_list_kernel launch");
 }
 
+// Whether each CTA can derive its own row tiles (one token chunk): the segment counts fit its
+// shared-memory table and the CTA's share of the at most ceil(R / 128) + nseg tiles fits its list.
+bool list_in_kernel(long long R, int nseg, int grid) {
+  const long long max_tiles = (R + proj::BM - 1) / proj::BM + nseg;
+  return nseg <= proj::kListSeg && (max_tiles + grid - 1) / grid <= proj::kListTiles;
+}
+
 // The output projection's token chunks bound the per-slot products kept at once (chunk Kr d_model
 // bf16) to kOutChunkBytes of workspace.  (Chunks small enough for the products to stay in L2,
 // 64 MB, measured slower: 184 against 147 us on the balanced layer, from the tail of each chunk's
@@ -639,10 +733,14 @@ extern "C" int namoh_proj_qkv(const uint16_t* x, int total_tokens, int d_model, 
   TileList tl;
   carve_tiles(ws, &tl, (long long)total_tokens * Kr, nseg, 1);
   if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
-  st = build_tiles(seg_offsets, row_src, nseg, Hr, Kr, 1, total_tokens, tl, info.sm_count, stream);
-  if (st != NAMOH_OK) return st;
+  const bool local_list = list_in_kernel((long long)total_tokens * Kr, nseg, info.sm_count);
+  if (!local_list) {
+    st = build_tiles(seg_offsets, row_src, nseg, Hr, Kr, 1, total_tokens, tl, info.sm_count, stream);
+    if (st != NAMOH_OK) return st;
+  }
   proj::Params p{};
-  p.tiles = tl.tiles;
+  p.tiles = local_list ? nullptr : tl.tiles;
+  p.seg_offsets = seg_offsets;
   p.tile_off = tl.off;
   p.ntiles = tl.cnt;
   p.row_src = row_src;
@@ -689,10 +787,14 @@ extern "C" int namoh_proj_out(const uint16_t* y, int total_tokens, int d_model, 
   carve_tiles(ws, &tl, R, nseg, nchunk);
   uint16_t* P = ws.take<uint16_t>((size_t)chunk * Kr * d_model);
   if (!ws.fits()) return NAMOH_ERR_WORKSPACE;
-  st = build_tiles(seg_offsets, row_src, nseg, Hr, Kr, nchunk, chunk, tl, info.sm_count, stream);
-  if (st != NAMOH_OK) return st;
+  const bool local_list = nchunk == 1 && list_in_kernel(R, nseg, info.sm_count);
+  if (!local_list) {
+    st = build_tiles(seg_offsets, row_src, nseg, Hr, Kr, nchunk, chunk, tl, info.sm_count, stream);
+    if (st != NAMOH_OK) return st;
+  }
   proj::Params p{};
-  p.tiles = tl.tiles;
+  p.tiles = local_list ? nullptr : tl.tiles;
+  p.seg_offsets = seg_offsets;
   p.row_src = row_src;
   p.nseg = nseg;
   p.Hr = Hr;

@@ -71,6 +71,7 @@ def _run_qkv(namoh, oracle_mod, ro, ref, x, w_qkv, B, H, K, g, d, rows=None):
     (2, 130, 16, 8, 64, 4, 128),    # 384 columns, two k-blocks
     (1, 200, 64, 32, 128, 8, 64),   # 1280 columns in five 256-wide tiles, one k-block
     (3, 1, 8, 2, 128, 1, 192),      # one token per sequence: tiles of one row
+    (72, 24, 16, 2, 128, 1, 128),   # 1152 segments: the tile list comes from the list kernels
 ])
 def test_proj_qkv_matches_oracle(namoh, oracle_mod, B, T, H, K, d, g, d_model):
     Hr, Kr = H // g, K // g
@@ -136,6 +137,21 @@ def test_proj_out_matches_oracle(namoh, oracle_mod, g):
     top = ref["topk_head"].reshape(B * T, Kr)
     _check_out(oracle_mod, o, y_bits, top, w_o, g, d)
     _check_out(oracle_mod, o2, y_bits, top, w_o, g, d, base=base.cpu().numpy().astype(np.float64))
+
+
+def test_proj_out_many_segments(namoh, oracle_mod):
+    """1152 segments (more than a CTA's own tile table holds): the list kernels' tile list."""
+    B, T, H, K, d, d_model = 72, 24, 16, 2, 128, 256
+    s = ni.router_scores(44, B, T, H)
+    ro = namoh.namoh_route(torch.from_numpy(s).cuda(), K)
+    ref = oracle_mod.route(s, K)
+    y_bits = _y(44, B * T, K, 1, d)
+    _, w_o = _weights(44, H, 1, d, d_model)
+    o = namoh.namoh_proj_out(dev_bf16(y_bits).view(B, T, K, d), dev_bf16(w_o), ro.seg_offsets, ro.row_src, B=B, H=H,
+                             K=K, status=ro.status)
+    torch.cuda.synchronize()
+    assert int(ro.status.item()) == 0
+    _check_out(oracle_mod, o, y_bits, ref["topk_head"].reshape(B * T, K), w_o, 1, d)
 
 
 def test_layer_full_size(namoh, oracle_mod):
