@@ -162,12 +162,23 @@ __global__ void __launch_bounds__(kSelThreads) sa_select_tc_kernel(const __grid_
   const int ncols = (nb + 15) & ~15;                 // N of the MMA (multiple of 16)
   uint32_t alloc = 32;
   while ((int)alloc < ncols) alloc <<= 1;
+  const int kbase = (off >> p.lg) + s;  // first pooled-key row of the segment
+  // the first loads (the query tile and the first box of pooled keys) go out before the TMEM
+  // allocation and the barrier, which they then overlap
+  auto issue_loads = [&](int n0) {
+    mbar_arrive_expect_tx(&bar_load, (uint32_t)(kAtoms * ((n0 == 0 ? kQAtomBytes : 0) + kKbBox * 128)));
+    for (int a = 0; a < kAtoms; ++a) {
+      if (n0 == 0) tma_load_2d(sq + a * kQAtomBytes, &tm_q, j * D + a * 64, off + row0, &bar_load);
+      tma_load_2d(skb + a * kb_atom_bytes, &tm_kb, a * 64, kbase + n0, &bar_load);
+    }
+  };
   if (threadIdx.x == 0) {
     mbar_init(&bar_load, 1);
     mbar_init(&bar_mma, 1);
     mbar_init(&bar_drain, 1);
     abort_flag = 0;
     mbar_fence_init();
+    issue_loads(0);
   }
   if (warp == 0) {
     tmem_alloc(&tmem_base, alloc);
@@ -181,18 +192,11 @@ __global__ void __launch_bounds__(kSelThreads) sa_select_tc_kernel(const __grid_
   if (warp == 0) {
     // The pooled keys stream through one buffer of kKbBox rows: load a box of blocks, issue its
     // MMAs into the next kKbBox score columns, wait for them, then reuse the buffer.
-    const int kbase = (off >> p.lg) + s;  // first pooled-key row of the segment
     const uint64_t q_desc = make_smem_desc_sw128(smem_u32(sq), 16, 1024);
     const uint64_t kb_desc = make_smem_desc_sw128(smem_u32(skb), 16, 1024);
     uint32_t phase = 0;
     for (int n0 = 0; n0 < ncols && ok; n0 += kKbBox, ++phase) {
-      if (lane == 0) {
-        mbar_arrive_expect_tx(&bar_load, (uint32_t)(kAtoms * ((n0 == 0 ? kQAtomBytes : 0) + kKbBox * 128)));
-        for (int a = 0; a < kAtoms; ++a) {
-          if (n0 == 0) tma_load_2d(sq + a * kQAtomBytes, &tm_q, j * D + a * 64, off + row0, &bar_load);
-          tma_load_2d(skb + a * kb_atom_bytes, &tm_kb, a * 64, kbase + n0, &bar_load);
-        }
-      }
+      if (lane == 0 && n0 > 0) issue_loads(n0);
       __syncwarp();
       ok = __all_sync(0xffffffffu, mbar_wait(&bar_load, phase & 1, &abort_flag, p.status));
       if (!ok) break;

@@ -9,8 +9,9 @@
 // and scores equal to within the 10 dropped bits (2^-13 relative, far inside the bf16 rounding the
 // inputs already carry) go to the lower block index.  Keys are unique, so "kept" is "key >= the k-th
 // largest key".  With k = R(r) - 1 kept of the c = N_B(r) - 1 completed blocks, a thread finds the
-// min(k, c - k)-th extreme key (of the kept set, or of the dropped one) with a sorted 8-entry register
-// list fed by a branch-free insertion network, or, past 8, by bisection over the 32-bit key range.
+// min(k, c - k)-th extreme key (of the kept set, or of the dropped one) with a sorted register list of
+// 2, 4 or 8 entries (the shortest the warp's largest count allows) fed by a branch-free insertion
+// network, or, past 8, by bisection over the 32-bit key range.
 #pragma once
 
 #include "common.cuh"
@@ -38,42 +39,54 @@ __device__ __forceinline__ void load_scores(uint32_t taddr, uint32_t (&r)[32]) {
   tmem_wait_ld();
 }
 
+// The kx-th largest key (x = key ^ flip) among blocks 0 .. cand - 1 of this thread's row, kept in a
+// sorted LL-entry register list fed by a branch-free insertion network; lanes with use = false
+// take part in the warp-collective loads only.  LL >= every participating lane's kx.
+template <int LL>
+__device__ __forceinline__ uint32_t list_pass(uint32_t taddr, int nchunks, int cand, int kx, uint32_t flip, bool use) {
+  uint32_t best[LL];
+#pragma unroll
+  for (int i = 0; i < LL; ++i) best[i] = 0u;
+  for (int c = 0; c < nchunks; ++c) {
+    if (__all_sync(0xffffffffu, !use || c * 32 >= cand)) continue;  // no lane has a candidate here
+    uint32_t v[32];
+    load_scores(taddr + (uint32_t)(c * 32), v);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const int b = c * 32 + i;
+      uint32_t x = (use && b < cand) ? score_key(__uint_as_float(v[i]), b) ^ flip : 0u;
+#pragma unroll
+      for (int e = 0; e < LL; ++e) {  // insertion into the sorted list, branch-free
+        const uint32_t hi = max(best[e], x);
+        x = min(best[e], x);
+        best[e] = hi;
+      }
+    }
+  }
+  uint32_t tau = 0xFFFFFFFFu;
+#pragma unroll
+  for (int e = 0; e < LL; ++e)
+    if (use && e == kx - 1) tau = best[e];
+  return tau;
+}
+
 // The kept blocks of one query from its row of block scores in TMEM (lane = this thread, columns
 // taddr .. taddr + 32 nchunks - 1): candidates are blocks 0 .. cand - 1, `keep` of them are kept.
 // emit(c, w) receives mask word c (bit i: block 32 c + i kept) for c = 0 .. nchunks - 1.
 // Warp-collective: tcgen05.ld needs every lane of the warp, so every lane calls this with the same
 // nchunks (a lane without a query passes cand = keep = 0) and the lanes' own work is predicated.
+// The list is as short as the warp's largest kx allows (2, 4 or kListLen entries).
 template <typename Emit>
 __device__ __forceinline__ void select_from_tmem(uint32_t taddr, int nchunks, int cand, int keep, Emit&& emit) {
   const bool drop_mode = 2 * keep > cand;          // find the dropped blocks instead
   const int kx = drop_mode ? cand - keep : keep;   // extreme keys to find
   const uint32_t flip = drop_mode ? 0xFFFFFFFFu : 0u;
-  uint32_t tau = 0xFFFFFFFFu;                      // the kx-th largest key (x = key ^ flip)
   const bool use_list = kx > 0 && kx <= kListLen;
-  {
-    uint32_t best[kListLen];
-#pragma unroll
-    for (int i = 0; i < kListLen; ++i) best[i] = 0u;
-    for (int c = 0; c < nchunks; ++c) {
-      if (__all_sync(0xffffffffu, !use_list || c * 32 >= cand)) continue;  // no lane has a candidate here
-      uint32_t v[32];
-      load_scores(taddr + (uint32_t)(c * 32), v);
-#pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const int b = c * 32 + i;
-        uint32_t x = (use_list && b < cand) ? score_key(__uint_as_float(v[i]), b) ^ flip : 0u;
-#pragma unroll
-        for (int e = 0; e < kListLen; ++e) {  // insertion into the sorted list, branch-free
-          const uint32_t hi = max(best[e], x);
-          x = min(best[e], x);
-          best[e] = hi;
-        }
-      }
-    }
-#pragma unroll
-    for (int e = 0; e < kListLen; ++e)
-      if (use_list && e == kx - 1) tau = best[e];
-  }
+  const int need = (int)__reduce_max_sync(0xffffffffu, use_list ? (unsigned)kx : 0u);
+  uint32_t tau = 0xFFFFFFFFu;                      // the kx-th largest key (x = key ^ flip)
+  if (need > 4) tau = list_pass<kListLen>(taddr, nchunks, cand, kx, flip, use_list);
+  else if (need > 2) tau = list_pass<4>(taddr, nchunks, cand, kx, flip, use_list);
+  else if (need > 0) tau = list_pass<2>(taddr, nchunks, cand, kx, flip, use_list);
   if (__any_sync(0xffffffffu, kx > kListLen)) {
     // bisection for the lanes that need more than kListLen keys: the largest t with #{x >= t} >= kx,
     // which (keys unique) is the kx-th largest key
