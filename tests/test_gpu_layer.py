@@ -117,10 +117,14 @@ def _check_out(oracle_mod, o, y_bits, top, w_o, g, d, base=None):
         assert np.all(err <= 2.0 ** -8 * scale + 1e-6 * np.abs(base) + 1e-5)
 
 
-@pytest.mark.parametrize("g", [1, 2])
-def test_proj_out_matches_oracle(namoh, oracle_mod, g):
+@pytest.mark.parametrize("g,d_model", [
+    (1, 512),   # two 256-column tiles
+    (2, 512),
+    (1, 192),   # one 192-column tile
+])
+def test_proj_out_matches_oracle(namoh, oracle_mod, g, d_model):
     """o = sum over slots of y W_O on a seeded y, and accumulate adds onto o."""
-    B, T, H, K, d, d_model = 2, 400, 8 * g, 2 * g, 128, 512
+    B, T, H, K, d = 2, 400, 8 * g, 2 * g, 128
     Hr, Kr = H // g, K // g
     s = ni.router_scores(42, B, T, Hr)
     ro = namoh.namoh_route(torch.from_numpy(s).cuda(), Kr)
