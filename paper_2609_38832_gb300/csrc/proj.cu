@@ -87,6 +87,7 @@ struct Params {
   const int32_t* tile_off;     // the list's first entry for this launch
   const int32_t* ntiles;       // the number of entries for this launch
   const int32_t* row_src;      // [R]
+  int R;                       // packed rows: a tile row at or past R (an inconsistent layout) is skipped
   int nseg, Hr, Kr;
   int a_rows;                  // tokens (rows of x)
   int kdim;                    // contraction length: d_model
@@ -329,6 +330,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     const uint16_t* a_base = static_cast<const uint16_t*>(p.a);
     // routing row_src value -> the gathered A row, clamped into the tensor (rows past the
     // segment's end load row 0 and are not stored)
+    auto in_rows = [&](const Tile& tt, int r) { return r < tt.rows && tt.row0 + r >= 0 && tt.row0 + r < p.R; };
     auto a_row_of = [&](int src) -> int {
       const int row = kMode == kQKV ? src / p.Kr : src;
       return min(max(row, 0), p.a_rows - 1);
@@ -343,7 +345,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
 #pragma unroll
       for (int w = 0; w < 8; ++w) {
         const int r = rq + 16 * w;
-        rows_a[w] = a_row_of(r < t.rows ? ld_issue_s32(p.row_src + t.row0 + r) : 0);
+        rows_a[w] = a_row_of(in_rows(t, r) ? ld_issue_s32(p.row_src + t.row0 + r) : 0);
       }
     }
     // the next row tile's entry, offsets and row indices are fetched during this one's k-blocks
@@ -379,7 +381,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
 #pragma unroll
               for (int w = 0; w < 8; ++w) {
                 const int r = rq + 16 * w;
-                nx_src[w] = r < nx.rows ? ld_issue_s32(p.row_src + nx.row0 + r) : 0;
+                nx_src[w] = in_rows(nx, r) ? ld_issue_s32(p.row_src + nx.row0 + r) : 0;
               }
             }
           }
@@ -418,7 +420,7 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
 #pragma unroll
         for (int w = 0; w < 8; ++w) {
           const int r = rq + 16 * w;
-          rows_a[w] = a_row_of(r < t.rows ? ld_issue_s32(p.row_src + t.row0 + r) : 0);
+          rows_a[w] = a_row_of(in_rows(t, r) ? ld_issue_s32(p.row_src + t.row0 + r) : 0);
         }
       }
     }
@@ -471,8 +473,8 @@ __global__ void __launch_bounds__(kThreads, 1) proj_kernel(const __grid_constant
     bool ok = true;
     for (int mt = blockIdx.x; mt < ntiles && ok; mt += gridDim.x) {
       const Tile t = decode_tile(p, tile_at(mt));
-      const bool valid = row < t.rows;
       const int r = t.row0 + row;
+      const bool valid = row < t.rows && r >= 0 && r < p.R;
       // OUT_P writes row r's partial product at its token-slot row row_src[r]
       const long long dst_row = kMode == kOutP && valid ? ld_issue_s32(p.row_src + r) - p.p_row0 : r;
       for (int gi = 0; gi < ngroups; ++gi, ++li) {
@@ -744,6 +746,7 @@ extern "C" int namoh_proj_qkv(const uint16_t* x, int total_tokens, int d_model, 
   p.tile_off = tl.off;
   p.ntiles = tl.cnt;
   p.row_src = row_src;
+  p.R = (int)((long long)total_tokens * Kr);
   p.nseg = nseg;
   p.Hr = Hr;
   p.Kr = Kr;
@@ -796,6 +799,7 @@ extern "C" int namoh_proj_out(const uint16_t* y, int total_tokens, int d_model, 
   p.tiles = local_list ? nullptr : tl.tiles;
   p.seg_offsets = seg_offsets;
   p.row_src = row_src;
+  p.R = (int)R;
   p.nseg = nseg;
   p.Hr = Hr;
   p.Kr = Kr;
