@@ -260,11 +260,13 @@ __device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores,
   softmax_norm<HMAX>(sc, H, mx, inv_z);
   // biased selection ranks the affinities a_h plus the head biases b_h; without a bias the
   // logits themselves are ranked (softmax is monotone)
+  // the affinity of head h: exp2((logit - max) log2 e) / z, the logit as loaded (non-finite -> -FLT_MAX)
+  auto affinity = [&](float l) { return fast_exp2((l - mx) * kLog2e) * inv_z; };
   float a[HMAX];
   if constexpr (kBiased) {
 #pragma unroll
     for (int h = 0; h < HMAX; ++h) {
-      a[h] = h < H ? fast_exp2((sc[h] - mx) * kLog2e) * inv_z : 0.f;
+      a[h] = h < H ? affinity(sc[h]) : 0.f;
       sc[h] = h < H ? a[h] + __ldg(bias + h) : 0.f;
     }
   }
@@ -279,10 +281,11 @@ __device__ __forceinline__ uint64_t topk_token(const float* __restrict__ scores,
 #pragma unroll
     for (int k = 0; k < KMAX; ++k) {
       if constexpr (kBiased) {
-        float ge = 0.f;
-#pragma unroll
-        for (int h = 0; h < HMAX; ++h) ge = (h == hk[k]) ? a[h] : ge;
-        g[k] = ge;
+        // the picked head's affinity again from its logit (the row is in L1), rather than a
+        // select over all H registers
+        float l = __ldg(scores + tok * H + hk[k]);
+        if (!isfinite(l)) l = -FLT_MAX;
+        g[k] = affinity(l);
       } else {
         g[k] = fast_exp2((vk[k] - mx) * kLog2e) * inv_z;
       }
@@ -382,6 +385,7 @@ __global__ void __launch_bounds__(kChunk) route_local_kernel(const float* __rest
                                                              const int32_t* __restrict__ cu_seqlens, int B,
                                                              int total) {
   __shared__ uint32_t s_bal[kChunk / 32][NAMOH_MAX_HEADS];
+  __shared__ int s_pre[kChunk / 32][NAMOH_MAX_HEADS];
   __shared__ int s_bad;
   const int H = kFullH ? HMAX : H_;  // (kFullH: a compile-time head count)
   pdl_launch_dependents();
@@ -416,19 +420,20 @@ __global__ void __launch_bounds__(kChunk) route_local_kernel(const float* __rest
   }
   __syncthreads();
   if (tid < H) {
+    // s_pre[w][h]: tokens of warps before w that picked head h; the chunk's count
     int n = 0;
 #pragma unroll
-    for (int w = 0; w < kChunk / 32; ++w) n += __popc(s_bal[w][tid]);
+    for (int w = 0; w < kChunk / 32; ++w) {
+      s_pre[w][tid] = n;
+      n += __popc(s_bal[w][tid]);
+    }
     chunk_count[((size_t)b * nchunks + c) * H + tid] = n;
   }
+  __syncthreads();
   if (tid == 0 && s_bad) report(status, NAMOH_DEV_NONFINITE_SCORE);
   if (!valid) return;
   const uint32_t lt = (1u << lane) - 1u;
-  auto local_rank = [&](int h) {
-    int before = 0;
-    for (int w = 0; w < warp; ++w) before += __popc(s_bal[w][h]);
-    return before + __popc(s_bal[warp][h] & lt);
-  };
+  auto local_rank = [&](int h) { return s_pre[warp][h] + __popc(s_bal[warp][h] & lt); };
   const size_t base = tok * K;
   if constexpr (KMAX > 0) {
     int rk[KMAX];
