@@ -534,12 +534,15 @@ __global__ void __launch_bounds__(kChunk) route_final_kernel(const int32_t* __re
     // seg_offsets + chunk base .. + count of segment h, so staging the values by head (at their
     // local rank) and writing the staged array in order turns 4 scattered stores per token into
     // runs of consecutive rows
+    // the chunk's head counts (loaded in parallel), then their exclusive prefix
+    if (tid < H) s_pos[tid] = __ldcg(chunk_count + ((size_t)b * nchunks + c) * H + tid);
+    __syncthreads();
     if (tid == 0) {
-      const int32_t* cc = chunk_count + ((size_t)b * nchunks + c) * H;
       int pos = 0;
       for (int hh = 0; hh < H; ++hh) {
+        const int n = s_pos[hh];
         s_pos[hh] = pos;
-        pos += __ldcg(cc + hh);
+        pos += n;
       }
     }
     __syncthreads();
