@@ -487,6 +487,8 @@ __global__ void __launch_bounds__(kChunk) route_final_kernel(const int32_t* __re
     h4 = __ldcg(reinterpret_cast<const int4*>(topk_head + base));
     r4 = __ldcg(reinterpret_cast<const int4*>(rank + base));
   }
+  // (K = 4) the chunk's head counts, for the staging slots below
+  if (K == 4 && tid < H) s_pos[tid] = __ldcg(chunk_count + ((size_t)b * nchunks + c) * H + tid);
   if (chunk_base) {
     if (tid < H) {
       s_cbase[tid] = chunk_base[((size_t)b * nchunks + c) * H + tid];
@@ -528,21 +530,29 @@ __global__ void __launch_bounds__(kChunk) route_final_kernel(const int32_t* __re
     if (c == 0 && tid < H) seg_offsets[(size_t)b * H + tid] = s_soff[tid];
     if (c == 0 && b == B - 1 && tid == 0) seg_offsets[(size_t)B * H] = (sr.start + sr.len) * K;
   }
-  __syncthreads();
-  if (K == 4 && __syncthreads_and(!valid || vec4)) {
+  // every thread: the count-table results above are visible after this barrier
+  const bool staged = __syncthreads_and(!valid || vec4);
+  if (K == 4 && staged) {
     // row_src through shared memory: this chunk's rows of head h are the contiguous run
     // seg_offsets + chunk base .. + count of segment h, so staging the values by head (at their
     // local rank) and writing the staged array in order turns 4 scattered stores per token into
     // runs of consecutive rows
-    // the chunk's head counts (loaded in parallel), then their exclusive prefix
-    if (tid < H) s_pos[tid] = __ldcg(chunk_count + ((size_t)b * nchunks + c) * H + tid);
-    __syncthreads();
-    if (tid == 0) {
-      int pos = 0;
-      for (int hh = 0; hh < H; ++hh) {
-        const int n = s_pos[hh];
-        s_pos[hh] = pos;
-        pos += n;
+    // the exclusive prefix of the chunk's head counts (warp 0, two scans of up to 32 heads)
+    if (tid < 32) {
+      const int lane = tid;
+      int carry = 0;
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        const int h = 32 * half + lane;
+        const int v = h < H ? s_pos[h] : 0;
+        int inc = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int y = __shfl_up_sync(0xffffffffu, inc, o);
+          if (lane >= o) inc += y;
+        }
+        if (h < H) s_pos[h] = carry + inc - v;
+        carry += __shfl_sync(0xffffffffu, inc, 31);
       }
     }
     __syncthreads();
