@@ -36,6 +36,7 @@ def _qkv(seed, shape):
     (4, 4, 4096, 128, 128),   # the bench's shape
     (1, 8, 5000, 64, 100),    # d = 64, a window inside one key tile, a ragged last tile
     (2, 3, 7000, 128, 2),     # the smallest window that reads the previous key tile
+    (3, 2, 100, 128, 50),     # sequences shorter than one query tile
 ])
 def test_shared_prefill_matches_oracle(namoh, oracle_mod, B, Hs, T, d, window):
     q, k, v = _qkv(60, (B, Hs, T, d))
