@@ -433,6 +433,15 @@ struct RopeTable {
 };
 void fill_rope_table(RopeTable* t, int d, double base);  // host, api.cu
 
+// SA + NAMOH block pooling done by the RoPE pass (App. B.8, the mean-pooled keys of App. B.3): the
+// pass walks each segment in chunks that start at multiples of its chunk height, so every block of
+// 2^lg keys lies in one chunk and is summed there.
+struct RopePool {
+  uint16_t* kbar;   // pooled keys: row (seg_offsets[s] >> lg) + s + b holds block b of segment s (bf16)
+  uint32_t* mask;   // SA mask rows [(r g + j), words]: zeroed for the segments not in the cache
+  int lg, words;
+};
+
 // Angle rho * theta_j reduced to about [-pi, pi] with ~1 ulp absolute error, then
 // hardware sin/cos (accurate on that interval).  The product is carried as an unevaluated sum (Dekker-style exact product
 // via FMA) and reduced modulo 2*pi by Cody and Waite's three-part subtraction.

@@ -44,7 +44,9 @@ cudaError_t launch_rope_pack(int D, const uint16_t* q, const uint16_t* k, const 
                              long long cache_rows, uint16_t* q_rot, uint16_t* k_cache, uint16_t* v_cache, bool copy_v,
                              const RopeTable& tab, uint32_t* status, int sm_count, cudaStream_t stream,
                              void* plan, int plan_qtiles, const int32_t* plan_cap, const int32_t* pos_row_src,
-                             int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved);
+                             int pos_k, int pos_t, const int32_t* pos_cu, int pos_hr, bool interleaved,
+                             const RopePool* pool);
+int rope_chunk_rows(int D, int g);
 
 int launch_window_attention(const uint16_t* q_rot, const uint16_t* k_cache, const uint16_t* v_cache, int B, int T,
                             int Hs, int D, int window, const int64_t* seg_base, long long cache_rows, uint16_t* y,
@@ -55,7 +57,7 @@ int launch_sa_select(const CUtensorMap& q_rot_map, const uint16_t* q_rot, const 
                      const int32_t* seg_offsets, const int64_t* seg_base, const int32_t* seg_cap,
                      long long cache_rows, int nseg, int T, long long R, int d, int g, int lg, int alpha_num,
                      int alpha_den, uint16_t* kbar, long long kbar_rows, uint32_t* mask, int words, const void* plan,
-                     int max_items, uint32_t* status, cudaStream_t stream);
+                     int max_items, uint32_t* status, cudaStream_t stream, bool pooled);
 
 namespace attn {
 
@@ -773,7 +775,8 @@ int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v
                          int d_head, int group, float rope_base, unsigned rope_flags, const int32_t* cu_seqlens,
                          const int32_t* seg_offsets, const int32_t* row_src, uint16_t* q_rot, uint16_t* k_cache,
                          uint16_t* v_cache, const int64_t* seg_base, const int32_t* seg_cap, long long cache_rows,
-                         uint32_t* dev_status, void* plan, const DeviceInfo& info, cudaStream_t stream) {
+                         uint32_t* dev_status, void* plan, const DeviceInfo& info, cudaStream_t stream,
+                         const RopePool* pool = nullptr) {
   RopeTable tab;
   fill_rope_table(&tab, d_head, (double)rope_base);
   const int nseg = B * Hr;
@@ -784,7 +787,7 @@ int launch_rope_and_plan(const uint16_t* q, const uint16_t* k, const uint16_t* v
                                          q_rot, k_cache, v_cache, v_cache != v, tab, dev_status, info.sm_count, stream,
                                          fuse_plan ? plan : nullptr, qtiles, plan_cap,
                                          (rope_flags & NAMOH_ROPE_GLOBAL) ? row_src : nullptr, Kr, T, cu_seqlens,
-                                         Hr, (rope_flags & NAMOH_ROPE_INTERLEAVED) != 0);
+                                         Hr, (rope_flags & NAMOH_ROPE_INTERLEAVED) != 0, pool);
   if (e != cudaSuccess) return cuda_fail(e, "rope_pack_kernel launch");
   if (plan && !fuse_plan) return launch_plan(seg_offsets, nseg, T, group, plan_cap, plan, stream);
   return NAMOH_OK;
@@ -1134,21 +1137,24 @@ extern "C" int namoh_sa_prefill(const uint16_t* q, const uint16_t* k, const uint
   DeviceInfo info;
   if (!device_ok(&info)) return NAMOH_ERR_UNSUPPORTED;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_v);
+  const int words = sa_words_for(T, block);
+  // blocks no taller than the RoPE pass's chunks are pooled by that pass, the others by their own kernel
+  const bool pool_in_rope = block <= rope_chunk_rows(d_head, group);
+  const RopePool pool{kbar, sa_mask, lg, words};
   int rc = launch_rope_and_plan(q, k, v, B, T, Hr, Kr, (int)R, d_head, group, rope_base, rope_flags, nullptr,
                                 seg_offsets, row_src, q_rot, k_cache, v_cache, seg_base, seg_cap, cache_rows,
-                                dev_status, plan, info, stream);
+                                dev_status, plan, info, stream, pool_in_rope ? &pool : nullptr);
   if (rc != NAMOH_OK) return rc;
   if (seg_len) {
     seg_len_kernel<<<(nseg + 255) / 256, 256, 0, stream>>>(seg_offsets, nseg, seg_len);
     if (const int st2 = cuda_check_launch("seg_len_kernel launch")) return st2;
   }
-  const int words = sa_words_for(T, block);
   CUtensorMap tq;
   if (!attn::encode_rows_map(&tq, q_rot, R, group * d_head)) return cuda_fail(cudaErrorInvalidValue, "cuTensorMapEncodeTiled");
   const long long max_items = ((R + attn::kItemRows - 1) / attn::kItemRows + nseg) * group;
   rc = launch_sa_select(tq, q_rot, k_cache, seg_offsets, seg_base, seg_base ? seg_cap : nullptr, cache_rows, nseg, T,
                         R, d_head, group, lg, alpha_num, alpha_den, kbar, kbar_rows, sa_mask, words, plan,
-                        (int)max_items, dev_status, stream);
+                        (int)max_items, dev_status, stream, pool_in_rope);
   if (rc != NAMOH_OK) return rc;
   return launch_attention(q_rot, k_cache, v_cache, R, d_head, group, seg_offsets, row_src, gate, seg_base, cache_rows,
                           plan, y, dev_status, info, stream, 0, sa_mask, words, lg);

@@ -356,17 +356,18 @@ int launch_select_tc(const CUtensorMap& tq, const CUtensorMap& tkb, const SelPar
 
 }  // namespace sa
 
-// Pooled keys, then the selection: the tensor-core selector over the attention plan's items, and
-// for histories longer than kSelMaxCols blocks the per-query selector for the rows past that.
+// Pooled keys (unless the RoPE pass pooled them: pooled = true), then the selection: the tensor-core
+// selector over the attention plan's items, and for histories longer than kSelMaxCols blocks the
+// per-query selector for the rows past that.
 // q_rot_map is the attention's tensor map of Q~ ([R, g d] rows, 64 x 128 boxes).  kbar holds
 // kbar_rows bf16 rows of d.
 int launch_sa_select(const CUtensorMap& q_rot_map, const uint16_t* q_rot, const uint16_t* k_cache,
                      const int32_t* seg_offsets, const int64_t* seg_base, const int32_t* seg_cap,
                      long long cache_rows, int nseg, int T, long long R, int d, int g, int lg, int alpha_num,
                      int alpha_den, uint16_t* kbar, long long kbar_rows, uint32_t* mask, int words, const void* plan,
-                     int max_items, uint32_t* status, cudaStream_t stream) {
+                     int max_items, uint32_t* status, cudaStream_t stream, bool pooled) {
   const int max_blocks = (T + (1 << lg) - 1) >> lg;
-  if (nseg > 0 && max_blocks > 0) {
+  if (nseg > 0 && max_blocks > 0 && !pooled) {
     dim3 grid((max_blocks + 7) / 8, nseg);
     auto pool = d == 128 ? (lg == 5 ? sa::sa_pool_kernel<128, 5> : lg == 6 ? sa::sa_pool_kernel<128, 6>
                                                                             : sa::sa_pool_kernel<128, 7>)

@@ -29,13 +29,14 @@ def namoh():
     return pkg
 
 
-def _run(namoh, wl, block, num, den, scores=None):
+def _run(namoh, wl, block, num, den, scores=None, **rope):
     scores = wl.scores() if scores is None else scores
     q, k, v = wl.qkv()
     ro = namoh.namoh_route(torch.from_numpy(scores).cuda(), wl.Kr)
     y, mask, kc, _ = namoh.namoh_sa_prefill(dev_bf16(q), dev_bf16(k), dev_bf16(v), ro.seg_offsets, ro.row_src,
                                             ro.gate, B=wl.B, T=wl.T, H=wl.H, K=wl.K, group=wl.g, block=block,
-                                            alpha_num=num, alpha_den=den, rope_base=wl.base, status=ro.status)
+                                            alpha_num=num, alpha_den=den, rope_base=wl.base, status=ro.status,
+                                            **rope)
     torch.cuda.synchronize()
     assert int(ro.status.item()) == 0
     return scores, (q, k, v), ro, y, mask.cpu().numpy().view(np.uint32), kc
@@ -60,17 +61,20 @@ def _check_counts(mask, seg, g, block, num, den):
                     assert not (int(m[b // 32]) >> (b % 32)) & 1, (row, j, b)
 
 
-def _check_scores(oracle_mod, wl, q, k, seg, mask, block, rows):
+def _check_scores(oracle_mod, wl, q, k, seg, mask, block, rows, interleaved=False, pos=None):
+    """pos: the RoPE position of every packed row (global positions), else the local ranks."""
     g, d = wl.g, wl.d
     rows = np.repeat(np.asarray(rows, np.int64), g)
     heads = np.tile(np.arange(g, dtype=np.int32), len(rows) // g)
     nblk = -(-int(np.diff(seg).max()) // block)
-    sc = oracle_mod.sa_scores_rows(q, k, seg, d, g, wl.base, block, rows, heads, nblk)
+    sc = oracle_mod.sa_scores_rows(q, k, seg, d, g, wl.base, block, rows, heads, nblk, interleaved=interleaved,
+                                   pos=pos)
     # |q~ . mean k~ - bf16(q~) . mean bf16(k~)| <= u sum_c |q~_c| (|mean k~_c| + mean |k~_c|), u = 2^-8 for the
     # bf16 rounding; u = 2^-7 covers the fp32 rotation before it as well (+ a floor for the fp32 sums)
     seg_of = np.searchsorted(seg, rows, side="right") - 1
     local = rows - seg[seg_of]
-    qrot = oracle_mod.rope(q.reshape(-1, d)[rows * g + heads], local, wl.base)
+    qrot = oracle_mod.rope(q.reshape(-1, d)[rows * g + heads], local if pos is None else pos[rows], wl.base,
+                           interleaved)
     compared = 0
     for i in range(len(rows)):
         valid = ~np.isnan(sc[i])
@@ -82,7 +86,8 @@ def _check_scores(oracle_mod, wl, q, k, seg, mask, block, rows):
             continue
         s0 = int(seg[seg_of[i]])
         nb = int(valid.sum())
-        krot = oracle_mod.rope(k[s0:s0 + nb * block], np.arange(nb * block), wl.base).reshape(nb, block, d)
+        kpos = np.arange(nb * block) if pos is None else pos[s0:s0 + nb * block]
+        krot = oracle_mod.rope(k[s0:s0 + nb * block], kpos, wl.base, interleaved).reshape(nb, block, d)
         bound = 2.0 ** -7 * (np.abs(qrot[i]) * (np.abs(krot.mean(1)) + np.abs(krot).mean(1))).sum(1) + 1e-4
         kept_v, drop_v = kept[:nb], ~kept[:nb]
         worst_kept = np.min(sc[i][:nb][kept_v] + bound[kept_v])
@@ -92,12 +97,13 @@ def _check_scores(oracle_mod, wl, q, k, seg, mask, block, rows):
     return compared
 
 
-def _check_y(oracle_mod, wl, qkv, ro, y, mask, block, num, den):
+def _check_y(oracle_mod, wl, qkv, ro, y, mask, block, num, den, interleaved=False, pos=None):
     q, k, v = qkv
     seg = ro.seg_offsets.cpu().numpy()
     row_src = ro.row_src.cpu().numpy()
     gate = ro.gate.cpu().numpy().astype(np.float64)
-    y_ref = oracle_mod.sa_prefill(q, k, v, seg, row_src, gate, wl.d, wl.g, wl.base, block, num, den, mask_in=mask)
+    y_ref = oracle_mod.sa_prefill(q, k, v, seg, row_src, gate, wl.d, wl.g, wl.base, block, num, den, mask_in=mask,
+                                  interleaved=interleaved, pos=pos)
     got = bf16_to_f64(y).reshape(-1, wl.d)
     assert_close_attention(got, y_ref, np.repeat(gate.reshape(-1), wl.g))
     return seg
@@ -114,6 +120,24 @@ def test_sa_prefill_matches_oracle(namoh, oracle_mod, wl, block, num, den):
     seg = _check_y(oracle_mod, wl, qkv, ro, y, mask, block, num, den)
     _check_counts(mask, seg, wl.g, block, num, den)
     assert _check_scores(oracle_mod, wl, qkv[0], qkv[1], seg, mask, block, np.arange(int(seg[-1]))) > 50
+
+
+@pytest.mark.parametrize("wl,block,il,gp", [
+    (ni.PrefillWorkload("sa_interleaved", B=2, T=700, H=8, K=2, d=128, seed=31), 32, True, False),
+    (ni.PrefillWorkload("sa_global", B=2, T=700, H=8, K=2, d=128, seed=32), 32, False, True),
+    (ni.PrefillWorkload("sa_d64_block64_both", B=1, T=1500, H=4, K=2, d=64, seed=33), 64, True, True),
+    (ni.PrefillWorkload("sa_d64_g4", B=1, T=900, H=8, K=4, d=64, g=4, seed=34), 32, False, False),
+    (ni.PrefillWorkload("sa_g2_global", B=2, T=500, H=8, K=2, d=128, g=2, seed=35), 32, False, True),
+], ids=lambda x: getattr(x, "name", str(x)))
+def test_sa_rope_variants(namoh, oracle_mod, wl, block, il, gp):
+    """The RoPE variants (interleaved pairs, global positions) and the head sizes and groups whose
+    blocks the RoPE pass pools itself (blocks no taller than its chunks of packed rows)."""
+    _, qkv, ro, y, mask, _ = _run(namoh, wl, block, 1, 4, interleaved=il, global_positions=gp)
+    pos = oracle_mod.global_positions(ro.row_src.cpu().numpy(), wl.T, wl.Kr) if gp else None
+    seg = _check_y(oracle_mod, wl, qkv, ro, y, mask, block, 1, 4, interleaved=il, pos=pos)
+    _check_counts(mask, seg, wl.g, block, 1, 4)
+    assert _check_scores(oracle_mod, wl, qkv[0], qkv[1], seg, mask, block, np.arange(int(seg[-1])),
+                         interleaved=il, pos=pos) > 50
 
 
 def test_sa_alpha_one_is_prefill(namoh):
