@@ -142,8 +142,10 @@ __global__ void __launch_bounds__(kSelThreads) sa_select_tc_kernel(const __grid_
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   pdl_launch_dependents();
   pdl_wait();  // plan, Q~ and the pooled keys come from the kernels before it
-  if ((int)blockIdx.x >= *p.nitems) return;
+  // the item count and this CTA's item load together (the plan holds one item per CTA of the grid)
+  const int nitems = *p.nitems;
   const int4 item = p.items[blockIdx.x];
+  if ((int)blockIdx.x >= nitems) return;
   const int s = item.x / p.g, j = item.x - s * p.g, qt = item.y, off = item.z, n = item.w;
   const int row0 = qt * kSelTileRows;
   const int r = row0 + (int)threadIdx.x;            // this thread's query rank

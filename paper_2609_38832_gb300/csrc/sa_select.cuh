@@ -33,27 +33,32 @@ __device__ __forceinline__ uint32_t score_key(float s, int b) {
   return (u & ~0x3FFu) | (uint32_t)(0x3FF - b);
 }
 
-// 32 block scores of this thread's row (TMEM lane), columns taddr .. taddr + 31.
-__device__ __forceinline__ void load_scores(uint32_t taddr, uint32_t (&r)[32]) {
-  tmem_ld32(taddr, r);
+// 16 block scores of this thread's row (TMEM lane), columns taddr .. taddr + 15.  The passes below
+// walk the scores 16 columns at a time in a loop that is not unrolled, which keeps the code small
+// (every CTA runs it once, from a cold instruction cache).
+constexpr int kSelGroup = 16;
+__device__ __forceinline__ void load_scores(uint32_t taddr, uint32_t (&r)[kSelGroup]) {
+  tmem_ld16(taddr, r);
   tmem_wait_ld();
 }
 
 // The kx-th largest key (x = key ^ flip) among blocks 0 .. cand - 1 of this thread's row, kept in a
 // sorted LL-entry register list fed by a branch-free insertion network; lanes with use = false
-// take part in the warp-collective loads only.  LL >= every participating lane's kx.
+// take part in the warp-collective loads only.  LL >= every participating lane's kx.  The columns
+// stop at the warp's largest candidate count.
 template <int LL>
-__device__ __forceinline__ uint32_t list_pass(uint32_t taddr, int nchunks, int cand, int kx, uint32_t flip, bool use) {
+__device__ __forceinline__ uint32_t list_pass(uint32_t taddr, int cand, int kx, uint32_t flip, bool use) {
   uint32_t best[LL];
 #pragma unroll
   for (int i = 0; i < LL; ++i) best[i] = 0u;
-  for (int c = 0; c < nchunks; ++c) {
-    if (__all_sync(0xffffffffu, !use || c * 32 >= cand)) continue;  // no lane has a candidate here
-    uint32_t v[32];
-    load_scores(taddr + (uint32_t)(c * 32), v);
+  const int wmax = (int)__reduce_max_sync(0xffffffffu, use ? (unsigned)cand : 0u);
+#pragma unroll 1
+  for (int g0 = 0; g0 < wmax; g0 += kSelGroup) {
+    uint32_t v[kSelGroup];
+    load_scores(taddr + (uint32_t)g0, v);
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      const int b = c * 32 + i;
+    for (int i = 0; i < kSelGroup; ++i) {
+      const int b = g0 + i;
       uint32_t x = (use && b < cand) ? score_key(__uint_as_float(v[i]), b) ^ flip : 0u;
 #pragma unroll
       for (int e = 0; e < LL; ++e) {  // insertion into the sorted list, branch-free
@@ -75,7 +80,9 @@ __device__ __forceinline__ uint32_t list_pass(uint32_t taddr, int nchunks, int c
 // emit(c, w) receives mask word c (bit i: block 32 c + i kept) for c = 0 .. nchunks - 1.
 // Warp-collective: tcgen05.ld needs every lane of the warp, so every lane calls this with the same
 // nchunks (a lane without a query passes cand = keep = 0) and the lanes' own work is predicated.
-// The list is as short as the warp's largest kx allows (2, 4 or kListLen entries).
+// Scores are read only below the warp's largest candidate count, which the caller's TMEM
+// allocation covers.  The list is as short as the warp's largest kx allows (2, 4 or kListLen
+// entries).
 template <typename Emit>
 __device__ __forceinline__ void select_from_tmem(uint32_t taddr, int nchunks, int cand, int keep, Emit&& emit) {
   const bool drop_mode = 2 * keep > cand;          // find the dropped blocks instead
@@ -84,22 +91,25 @@ __device__ __forceinline__ void select_from_tmem(uint32_t taddr, int nchunks, in
   const bool use_list = kx > 0 && kx <= kListLen;
   const int need = (int)__reduce_max_sync(0xffffffffu, use_list ? (unsigned)kx : 0u);
   uint32_t tau = 0xFFFFFFFFu;                      // the kx-th largest key (x = key ^ flip)
-  if (need > 4) tau = list_pass<kListLen>(taddr, nchunks, cand, kx, flip, use_list);
-  else if (need > 2) tau = list_pass<4>(taddr, nchunks, cand, kx, flip, use_list);
-  else if (need > 0) tau = list_pass<2>(taddr, nchunks, cand, kx, flip, use_list);
+  if (need > 4) tau = list_pass<kListLen>(taddr, cand, kx, flip, use_list);
+  else if (need > 2) tau = list_pass<4>(taddr, cand, kx, flip, use_list);
+  else if (need > 0) tau = list_pass<2>(taddr, cand, kx, flip, use_list);
   if (__any_sync(0xffffffffu, kx > kListLen)) {
     // bisection for the lanes that need more than kListLen keys: the largest t with #{x >= t} >= kx,
     // which (keys unique) is the kx-th largest key
+    const bool bis = kx > kListLen;
+    const int wmax = (int)__reduce_max_sync(0xffffffffu, bis ? (unsigned)cand : 0u);
     uint32_t lo = 0u, hi = 0xFFFFFFFFu;
     for (int it = 0; it < 32; ++it) {
       const uint32_t mid = lo + ((hi - lo) >> 1) + ((hi - lo) & 1u);
       int cnt = 0;
-      for (int c = 0; c < nchunks; ++c) {
-        uint32_t v[32];
-        load_scores(taddr + (uint32_t)(c * 32), v);
+#pragma unroll 1
+      for (int g0 = 0; g0 < wmax; g0 += kSelGroup) {
+        uint32_t v[kSelGroup];
+        load_scores(taddr + (uint32_t)g0, v);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const int b = c * 32 + i;
+        for (int i = 0; i < kSelGroup; ++i) {
+          const int b = g0 + i;
           cnt += (b < cand && (score_key(__uint_as_float(v[i]), b) ^ flip) >= mid) ? 1 : 0;
         }
       }
@@ -108,23 +118,27 @@ __device__ __forceinline__ void select_from_tmem(uint32_t taddr, int nchunks, in
         else hi = mid - 1u;
       }
     }
-    if (kx > kListLen) tau = lo;
+    if (bis) tau = lo;
   }
-  // the mask: block b kept iff key >= tau (kept mode), ~key < tau (drop mode)
+  // the mask: block b kept iff key >= tau (kept mode), ~key < tau (drop mode); the columns stop at
+  // the warp's largest candidate count
+  const int wmax = (int)__reduce_max_sync(0xffffffffu, keep > 0 ? (unsigned)cand : 0u);
+#pragma unroll 1
   for (int c = 0; c < nchunks; ++c) {
-    if (__all_sync(0xffffffffu, c * 32 >= cand)) {  // no candidate of any lane: an empty word
-      emit(c, 0u);
-      continue;
-    }
-    uint32_t v[32];
-    load_scores(taddr + (uint32_t)(c * 32), v);
     uint32_t w = 0u;
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      const int b = c * 32 + i;
-      const uint32_t x = score_key(__uint_as_float(v[i]), b) ^ flip;
-      const bool kept = b < cand && keep > 0 && (drop_mode ? x < tau : x >= tau);
-      w |= (kept ? 1u : 0u) << i;
+    for (int h = 0; h < 32 / kSelGroup; ++h) {
+      const int g0 = c * 32 + h * kSelGroup;
+      if (g0 >= wmax) break;
+      uint32_t v[kSelGroup];
+      load_scores(taddr + (uint32_t)g0, v);
+#pragma unroll
+      for (int i = 0; i < kSelGroup; ++i) {
+        const int b = g0 + i;
+        const uint32_t x = score_key(__uint_as_float(v[i]), b) ^ flip;
+        const bool kept = b < cand && keep > 0 && (drop_mode ? x < tau : x >= tau);
+        w |= (kept ? 1u : 0u) << (h * kSelGroup + i);
+      }
     }
     emit(c, w);
   }
