@@ -20,6 +20,10 @@
 // builds the attention work list in the same launch.  Launched with programmatic dependent
 // launch: set-up overlaps the routing kernel's tail, and every read of routing outputs or
 // inputs comes after pdl_wait().
+// Pooling variants (SA + NAMOH, App. B.8 with the mean-pooled keys of App. B.3): the chunks start at
+// multiples of the chunk height within each segment, so each block of 2^lg <= kRows keys lies in
+// one chunk; the pass sums the rotated keys it wrote (as bf16) per block and column and stores the
+// block means, the pooled keys the selection kernel reads.
 #include <type_traits>
 
 #include "common.cuh"
